@@ -1,0 +1,172 @@
+/*
+ * libsoap -- the SOAP optimizer step (arXiv 2607.20548, Alg. 1 "KL-SOAP used in
+ * experiments", with the standard Shampoo factor EMAs of section 2) batched over
+ * every weight matrix of a model, on one NVIDIA GB300 (sm_103a).
+ *
+ * Conventions shared by every entry point
+ *   - Matrices are fp32, row-major, contiguous: element (i, j) of a rows x cols
+ *     matrix sits at i * cols + j. Orientation follows Alg. 1's state list:
+ *     W, G, m, v are rows x cols ("in x out"); L, Q_L are rows x rows; R, Q_R are
+ *     cols x cols.
+ *   - Device pointers must be 16-byte aligned and must not alias each other.
+ *   - Every call that takes a stream only enqueues work on it (no host
+ *     synchronisation) unless its comment says otherwise. Streams are
+ *     cudaStream_t values passed as soap_stream_t; 0 is the legacy default stream.
+ *   - The library owns all optimizer state and workspace; the caller owns params,
+ *     grads, the stream, and any buffer it passes in.
+ *   - Host-side validation failures return immediately with an error code and
+ *     leave the state untouched. Conditions found on the device (non-finite
+ *     values, a QR breakdown, a bounded wait that ran out) set a sticky status
+ *     word that soap_status() reads and that the next soap_step() returns. No
+ *     kernel traps.
+ */
+#ifndef SOAP_H_
+#define SOAP_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* soap_stream_t; /* identical to cudaStream_t */
+typedef struct soap_s* soap_handle;        /* opaque, owned by the library */
+
+typedef enum {
+  SOAP_OK = 0,
+  SOAP_ERR_INVALID_ARG = 1, /* bad shape, index, pointer alignment or null pointer */
+  SOAP_ERR_CUDA = 2,        /* a CUDA runtime call failed; see soap_last_error */
+  SOAP_ERR_OOM = 3,         /* device memory for state or workspace not available */
+  SOAP_ERR_NONFINITE = 4,   /* NaN or Inf seen in a gradient or in the state */
+  SOAP_ERR_QR_BREAKDOWN = 5,/* a QR pivot norm was not finite */
+  SOAP_ERR_TIMEOUT = 6      /* a bounded device-side wait gave up */
+} soap_status_t;
+
+/* One weight matrix. precond_left = 0 keeps Q_L = I fixed and stores no L (an
+ * "identity side"); likewise precond_right for Q_R and R. */
+typedef struct {
+  int64_t rows, cols;
+  int32_t precond_left, precond_right;
+} soap_shape;
+
+/* Hyper-parameters of Alg. 1 and its table.
+ *   lr, weight_decay: eta_t and lambda_t of the update W <- (1 - eta lambda) W - eta dW
+ *   beta1, beta2:     first/second-moment EMA coefficients in the rotated basis
+ *   factor_beta:      Kronecker-factor EMA coefficient b in L <- b L + (1-b) G G^T
+ *                     (every EMA weights the OLD state by its coefficient)
+ *   eps:              added outside the square root, N = m / (sqrt(v) + eps)
+ *   eig_every:        F; the basis is refreshed when t mod F == 0 (the paper uses 1)
+ *   bias_correction:  0 = literal Alg. 1 (none); 1 = divide m, v by (1 - beta^t)
+ *   qr_tol:           a Householder column whose remaining norm is <= qr_tol*||P||_F
+ *                     is treated as exactly zero (no reflector, R_kk = 0, sign +1)
+ *   guard:            1 = rows/cols of N that belong to such zero columns are 0 */
+typedef struct {
+  float lr, beta1, beta2, factor_beta, eps, weight_decay;
+  int32_t eig_every;
+  int32_t bias_correction;
+  float qr_tol;
+  int32_t guard;
+} soap_hparams;
+
+/* Fills *hp with the defaults used for the paper's workloads: lr 3e-3,
+ * beta1 = beta2 = factor_beta = 0.95, eps 1e-8, weight_decay 0.1, F = 1, no bias
+ * correction, qr_tol 1e-4, guard on. */
+void soap_default_hparams(soap_hparams* hp);
+
+/* Creates the optimizer for n matrices on CUDA device `device` and allocates all
+ * state (Alg. 1 "Optimizer States") and workspace up front: L = R = 0, Q = I,
+ * m = v = 0, t = 0. shapes[] is copied. Returns SOAP_ERR_OOM if the state does
+ * not fit; *out is then NULL. The device becomes current for the calling thread. */
+soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparams* hp,
+                          int32_t device, soap_handle* out);
+
+/* One SOAP step (Alg. 1) over all n matrices, enqueued on `stream`:
+ * factor EMAs with the current gradient, power step P = L Q and QR refresh with
+ * diag(R) >= 0, first-moment re-projection, rotation G' = Q_L^T G Q_R, Adam in the
+ * rotated basis, back-rotation dW = Q_L N Q_R^T and W <- (1 - eta lambda) W - eta dW.
+ * params[i] / grads[i]: device pointers to matrix i (rows_i x cols_i, fp32); params
+ * are updated in place, grads are only read. Both pointer arrays are host arrays
+ * and are copied before the call returns. Returns a pending sticky device status
+ * from an earlier step, if any, before enqueuing anything. */
+soap_status_t soap_step(soap_handle h, float* const* params, const float* const* grads,
+                        soap_stream_t stream);
+
+/* Sets eta_t and lambda_t for the following steps (Alg. 1 takes them per step). */
+soap_status_t soap_set_lr(soap_handle h, float lr, float weight_decay);
+
+/* Which piece of a matrix's state soap_state_get/set move. */
+typedef enum {
+  SOAP_STATE_M = 0,     /* first moment m in the current eigenbasis (rows x cols) */
+  SOAP_STATE_V = 1,     /* second moment v in the current eigenbasis (rows x cols) */
+  SOAP_STATE_L = 2,     /* left factor L (rows x rows) */
+  SOAP_STATE_QL = 3,    /* left eigenbasis Q_L (rows x rows) */
+  SOAP_STATE_R = 4,     /* right factor R (cols x cols) */
+  SOAP_STATE_QR = 5,    /* right eigenbasis Q_R (cols x cols) */
+  SOAP_STATE_MHAT = 6,  /* first moment in the original basis, Q_L m Q_R^T (rows x cols);
+                           the library's own storage, bit-exact for checkpoints */
+  SOAP_STATE_SKIP_L = 7,/* uint8 per row: 1 where Q_L's column came from a zero QR column */
+  SOAP_STATE_SKIP_R = 8 /* uint8 per col: same for Q_R */
+} soap_state_which;
+
+/* Number of bytes soap_state_get/set move for (idx, which); 0 if that piece does not
+ * exist (an identity side) or the arguments are invalid. */
+size_t soap_state_bytes(soap_handle h, int32_t idx, int32_t which);
+
+/* Copies one piece of matrix idx's state to dst (host or device memory; the copy is
+ * ordered on `stream`; a host dst is complete when the stream is). SOAP_STATE_M is
+ * computed on the fly as Q_L^T M_hat Q_R (fp32 GEMMs), so it is not bit-exact with
+ * what a later soap_state_set(SOAP_STATE_M) stores; use SOAP_STATE_MHAT to
+ * checkpoint. Returns SOAP_ERR_INVALID_ARG for an identity side's L/Q/R. */
+soap_status_t soap_state_get(soap_handle h, int32_t idx, int32_t which, void* dst,
+                             soap_stream_t stream);
+
+/* Copies src (host or device) into one piece of matrix idx's state, ordered on
+ * `stream`. Setting SOAP_STATE_M stores Q_L m Q_R^T with the Q_L, Q_R held at that
+ * moment, so set Q_L and Q_R first. */
+soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const void* src,
+                             soap_stream_t stream);
+
+/* Step counter t (number of completed soap_step calls, or the value last set). */
+int64_t soap_get_step(soap_handle h);
+soap_status_t soap_set_step(soap_handle h, int64_t t);
+
+/* Synchronises `stream`, then returns the sticky device status (SOAP_OK if clean). */
+soap_status_t soap_status(soap_handle h, soap_stream_t stream);
+
+/* Clears the sticky device status (ordered on `stream`). */
+soap_status_t soap_clear_status(soap_handle h, soap_stream_t stream);
+
+/* Human-readable text of the last error on this handle (never NULL). */
+const char* soap_last_error(soap_handle h);
+
+/* Frees all state and workspace. Safe on NULL. Synchronises the device first. */
+void soap_destroy(soap_handle h);
+
+/* ---- stand-alone sub-steps (the same kernels soap_step runs) ------------------- */
+
+/* S3, Alg. 1 "QR(L_t Q_L).Q": for `batch` square n x n matrices P (device,
+ * contiguous, batch stride n*n), writes Q with P = Q R and diag(R) >= 0 (blocked
+ * Householder QR, explicit Q) and skip[b*n + k] = 1 where column k was treated as
+ * exactly zero (remaining norm <= tol * ||P_b||_F). P is read only. `workspace`
+ * must hold soap_qr_workspace_bytes(n, batch) bytes of device memory. */
+size_t soap_qr_workspace_bytes(int32_t n, int32_t batch);
+soap_status_t soap_qr(int32_t n, int32_t batch, const float* P, float* Q, uint8_t* skip,
+                      float tol, void* workspace, size_t workspace_bytes,
+                      soap_stream_t stream);
+
+/* The fp32-accurate batched product used by every contraction of the step (S1, S2,
+ * S4, S5, S7 and the QR updates): for b < batch,
+ *   C_b = alpha * op(A_b) * op(B_b) + beta * C_b,
+ * op(X) = X or X^T (trans_x != 0), op(A_b) is M x K, op(B_b) is K x N, all
+ * row-major with leading dimensions lda/ldb/ldc and batch strides in elements.
+ * beta == 0 does not read C. */
+soap_status_t soap_gemm(int32_t trans_a, int32_t trans_b, int32_t M, int32_t N, int32_t K,
+                        float alpha, const float* A, int64_t lda, int64_t stride_a,
+                        const float* B, int64_t ldb, int64_t stride_b, float beta, float* C,
+                        int64_t ldc, int64_t stride_c, int32_t batch, soap_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SOAP_H_ */

@@ -1,0 +1,247 @@
+"""Pins of the fp64 oracle against facts fixed by the paper or by mathematics.
+
+Each test compares the oracle with something other than itself: a closed form, an
+invariant, a library routine solving the same textbook problem, or brute force.
+"""
+import numpy as np
+import pytest
+
+from oracle.soap_ref import (HParams, MatrixState, factor_ema, householder_q, rotate_in,
+                             rotate_out, soap_step)
+
+RNG = np.random.default_rng(1234)
+
+
+# ---- S3: the QR refresh ------------------------------------------------------------
+
+@pytest.mark.parametrize("n", [1, 2, 5, 33, 128])
+def test_qr_matches_library_qr_with_positive_diagonal(n):
+    """Full-rank P: Q with diag(R) > 0 is unique, so it equals LAPACK's after its sign fix."""
+    P = RNG.standard_normal((n, n))
+    Q, skipped, rdiag = householder_q(P, 0.0)
+    Ql, Rl = np.linalg.qr(P)
+    s = np.sign(np.diag(Rl))
+    s[s == 0] = 1
+    assert not skipped.any()
+    np.testing.assert_allclose(Q, Ql * s, atol=1e-12)
+    np.testing.assert_allclose(rdiag, np.abs(np.diag(Rl)), rtol=1e-12)
+
+
+@pytest.mark.parametrize("n", [3, 64, 200])
+def test_qr_orthogonal_and_triangular(n):
+    """Q^T Q = I and Q^T P is upper triangular with a non-negative diagonal."""
+    P = RNG.standard_normal((n, n))
+    Q, _, rdiag = householder_q(P, 0.0)
+    assert np.abs(Q.T @ Q - np.eye(n)).max() < 1e-13
+    R = Q.T @ P
+    assert np.abs(np.tril(R, -1)).max() < 1e-12 * np.abs(P).max() * n
+    np.testing.assert_allclose(np.diag(R), rdiag, atol=1e-12 * np.linalg.norm(P))
+    assert (np.diag(R) > 0).all()
+
+
+def test_qr_exactly_rank_deficient_columns_are_skipped():
+    """Dependent columns (exact integer combinations) get no reflector, Q stays orthogonal,
+    P = Q R still holds with R upper triangular and R_kk = 0 at the skipped columns."""
+    a = np.array([1.0, 2.0, 0.0, -1.0, 3.0])
+    b = np.array([0.0, 1.0, 1.0, 2.0, -2.0])
+    c = np.array([4.0, 0.0, 1.0, 1.0, 1.0])
+    P = np.stack([a, 2 * a, b, a - b, c], axis=1)
+    Q, skipped, rdiag = householder_q(P, 1e-10)
+    assert skipped.tolist() == [False, True, False, True, False]
+    assert np.abs(Q.T @ Q - np.eye(5)).max() < 1e-14
+    R = Q.T @ P
+    assert np.abs(np.tril(R, -1)).max() < 1e-12
+    assert np.abs(np.diag(R)[[1, 3]]).max() < 1e-12
+    assert (rdiag[[0, 2, 4]] > 0).all()
+
+
+def test_qr_zero_matrix_gives_identity():
+    Q, skipped, _ = householder_q(np.zeros((7, 7)), 0.0)
+    assert skipped.all()
+    np.testing.assert_array_equal(Q, np.eye(7))
+
+
+def test_qr_float32_twin_is_orthogonal():
+    P = RNG.standard_normal((96, 96)).astype(np.float32)
+    Q, _, _ = householder_q(P, 0.0)
+    assert Q.dtype == np.float32
+    assert np.abs(Q.T.astype(np.float64) @ Q - np.eye(96)).max() < 2e-6
+
+
+def test_subspace_iteration_converges_to_planted_eigenvectors():
+    """Repeated refreshes Q <- QR(L Q).Q are subspace iteration (Golub & Van Loan 8.2.4): with a
+    planted spectrum the k-th column converges to the k-th eigenvector at rate lambda_k+1/lambda_k."""
+    n = 24
+    U, _ = np.linalg.qr(RNG.standard_normal((n, n)))
+    lam = 2.0 ** -np.arange(n)          # ratio 1/2 between neighbours
+    L = (U * lam) @ U.T
+    Q = np.eye(n)
+    for _ in range(80):
+        Q, _, _ = householder_q(L @ Q, 0.0)
+    cos = np.abs(np.sum(Q[:, :12] * U[:, :12], axis=0))
+    assert cos.min() > 1 - 1e-10
+    # every leading prefix spans the planted invariant subspace (principal angles ~ 0)
+    for k in (1, 4, 8, 12):
+        s = np.linalg.svd(U[:, :k].T @ Q[:, :k], compute_uv=False)
+        assert s.min() > 1 - 1e-10
+
+
+# ---- S1: factor EMAs --------------------------------------------------------------
+
+def test_factor_ema_closed_form():
+    """L_t = sum_s (1-b) b^(t-s) G_s G_s^T and R_t likewise (section 2 Shampoo EMAs, unrolled)."""
+    b = 0.95
+    Gs = [RNG.standard_normal((6, 9)) for _ in range(7)]
+    L = np.zeros((6, 6))
+    R = np.zeros((9, 9))
+    for G in Gs:
+        L = factor_ema(L, G, b, "L")
+        R = factor_ema(R, G, b, "R")
+    T = len(Gs)
+    Lc = sum((1 - b) * b ** (T - 1 - s) * np.einsum("ik,jk->ij", Gs[s], Gs[s]) for s in range(T))
+    Rc = sum((1 - b) * b ** (T - 1 - s) * np.einsum("ki,kj->ij", Gs[s], Gs[s]) for s in range(T))
+    np.testing.assert_allclose(L, Lc, rtol=1e-13)
+    np.testing.assert_allclose(R, Rc, rtol=1e-13)
+
+
+# ---- S6/S8: reduction to AdamW when Q = I -----------------------------------------
+
+@pytest.mark.parametrize("sides", [(False, False), (True, True), (True, False)])
+@pytest.mark.parametrize("bias_correction", [False, True])
+def test_constant_gradient_reduces_to_adam_closed_form(sides, bias_correction):
+    """With Q = I (section 2: identity eigenvectors recover AdamW) and a constant gradient g,
+    the EMAs sum to m_t = (1-b1^t) g and v_t = (1-b2^t) g^2, so
+    N_t = (1-b1^t) g / (sqrt(1-b2^t) |g| + eps), or g / (|g| + eps) with bias correction.
+    One entry has |g| = 2e-8 ~ eps, where eps inside the root would change N by 1e3x.
+    A diagonal gradient keeps L, R diagonal, so preconditioned sides stay at Q = I."""
+    n = 5
+    gd = np.array([0.3, -0.2, 0.5, -0.7, 2e-8])
+    g = np.diag(gd)
+    hp = HParams(lr=1e-2, weight_decay=0.0, bias_correction=bias_correction, qr_tol=0.0)
+    st = MatrixState(n, n, sides[0], sides[1])
+    W0 = np.full((n, n), 0.25)
+    W = W0.copy()
+    expected = W0.copy()
+    for t in range(1, 9):
+        W, _ = soap_step(st, W, g, hp)
+        if bias_correction:
+            N = gd / (np.abs(gd) + 1e-8)
+        else:
+            N = (1 - 0.95 ** t) * gd / (np.sqrt(1 - 0.95 ** t) * np.abs(gd) + 1e-8)
+        expected = expected - hp.lr * np.diag(N)
+        np.testing.assert_allclose(W, expected, rtol=0, atol=1e-15)
+    if sides[0]:
+        np.testing.assert_allclose(st.QL, np.eye(n), atol=1e-15)
+
+
+def test_zero_gradient_is_pure_weight_decay():
+    """G = 0: every EMA stays 0, N = 0/(0+eps) = 0, so W_t = (1 - lr*wd)^t W_0 (Alg. 1 last line)."""
+    hp = HParams(lr=3e-3, weight_decay=0.1)
+    st = MatrixState(4, 6, True, True)
+    W0 = RNG.standard_normal((4, 6))
+    W = W0.copy()
+    for _ in range(5):
+        W, dW = soap_step(st, W, np.zeros((4, 6)), hp)
+        assert np.all(dW == 0)
+    np.testing.assert_allclose(W, (1 - 3e-4) ** 5 * W0, rtol=1e-14)
+    assert st.skipL.all() and st.skipR.all()
+
+
+# ---- S7: update-RMS invariance ------------------------------------------------------
+
+def test_update_norm_equals_adam_norm():
+    """||dW||_F = ||N||_F because Q_L, Q_R are orthogonal (section 5, update RMS matching)."""
+    hp = HParams()
+    st = MatrixState(12, 20, True, True)
+    W = RNG.standard_normal((12, 20))
+    for t in range(4):
+        G = RNG.standard_normal((12, 20))
+        W, dW = soap_step(st, W, G, hp)
+        N = st.m / (np.sqrt(st.v) + hp.eps)
+        N[st.skipL, :] = 0
+        N[:, st.skipR] = 0
+        assert abs(np.linalg.norm(dW) - np.linalg.norm(N)) < 1e-12 * np.linalg.norm(N)
+
+
+# ---- S4: first-moment re-projection -------------------------------------------------
+
+def test_reprojection_preserves_momentum_in_original_space():
+    """With beta1 = 1 the Adam block leaves m unchanged, so across a basis change
+    Q_L,new m_new Q_R,new^T must equal Q_L,old m_old Q_R,old^T (Alg. 1 re-projection)."""
+    hp = HParams(beta1=0.95)
+    st = MatrixState(8, 10, True, True)
+    W = np.zeros((8, 10))
+    for _ in range(3):
+        W, _ = soap_step(st, W, RNG.standard_normal((8, 10)), hp)
+    before = st.QL @ st.m @ st.QR.T
+    QL_old = st.QL.copy()
+    hp1 = HParams(beta1=1.0)
+    soap_step(st, W, RNG.standard_normal((8, 10)), hp1)
+    assert np.abs(st.QL - QL_old).max() > 1e-3  # the basis really changed
+    after = st.QL @ st.m @ st.QR.T
+    np.testing.assert_allclose(after, before, atol=1e-13)
+
+
+def test_rotations_are_the_two_sided_products():
+    QL, _ = np.linalg.qr(RNG.standard_normal((4, 4)))
+    QR, _ = np.linalg.qr(RNG.standard_normal((6, 6)))
+    G = RNG.standard_normal((4, 6))
+    Gp = rotate_in(QL, G, QR)
+    np.testing.assert_allclose(np.einsum("ki,kl,lj->ij", QL, G, QR), Gp, atol=1e-14)
+    np.testing.assert_allclose(rotate_out(QL, Gp, QR), G, atol=1e-14)
+
+
+# ---- S1-S3 against a brute-force eigendecomposition ---------------------------------
+
+@pytest.mark.parametrize("shape", [(4, 6), (6, 3), (5, 5)])
+def test_constant_gradient_basis_converges_to_eigh(shape):
+    """Constant G: L_t -> G G^T and R_t -> G^T G, and the refreshed bases converge to their
+    eigenvectors, ordered by decreasing eigenvalue (Q_0 = I is generic), up to sign --
+    checked against the library's symmetric eigensolver."""
+    m, n = shape
+    G = RNG.standard_normal(shape)
+    st = MatrixState(m, n, True, True)
+    hp = HParams(factor_beta=0.5, qr_tol=1e-10)
+    W = np.zeros(shape)
+    for _ in range(300):
+        W, _ = soap_step(st, W, G, hp)
+    for Q, F, skip in ((st.QL, G @ G.T, st.skipL), (st.QR, G.T @ G, st.skipR)):
+        w, U = np.linalg.eigh(F)
+        order = np.argsort(-w)
+        w, U = w[order], U[:, order]
+        r = int(np.sum(w > 1e-10 * w[0]))
+        cos = np.abs(np.sum(Q[:, :r] * U[:, :r], axis=0))
+        assert cos.min() > 1 - 1e-8, cos
+
+
+# ---- S1-S7: the SVD view with the EMAs switched off ---------------------------------
+
+def test_emas_off_gives_polar_factor():
+    """Appendix (SVD view of SOAP): with b = beta1 = beta2 = 0 and a constant full-rank G, the
+    bases converge to U, V of G = U S V^T, G' -> S (diagonal), N -> sign(S) = I and the update
+    direction dW -> U V^T, the polar factor; compared with the library SVD."""
+    n = 6
+    G = RNG.standard_normal((n, n))
+    hp = HParams(beta1=0.0, beta2=0.0, factor_beta=0.0, lr=0.0, weight_decay=0.0, qr_tol=1e-12)
+    st = MatrixState(n, n, True, True)
+    W = np.zeros((n, n))
+    for _ in range(400):
+        W, dW = soap_step(st, W, G, hp)
+    U, s, Vt = np.linalg.svd(G)
+    np.testing.assert_allclose(dW, U @ Vt, atol=1e-6)
+    Gp = rotate_in(st.QL, G, st.QR)
+    np.testing.assert_allclose(np.abs(np.diag(Gp)), s, rtol=1e-8)
+    assert np.abs(Gp - np.diag(np.diag(Gp))).max() < 1e-8 * s[0]
+
+
+# ---- guard and rank deficiency -----------------------------------------------------
+
+def test_first_step_of_rectangular_matrix_is_null_space_free():
+    """At t = 1 R = (1-b) G^T G has rank = rows < cols; the zero QR columns span G's null
+    space, so G Q_R is exactly 0 there and the guarded N is 0 there (exact arithmetic)."""
+    G = RNG.standard_normal((5, 9))
+    st = MatrixState(5, 9, True, True)
+    soap_step(st, np.zeros((5, 9)), G, HParams(qr_tol=1e-9))
+    assert st.skipR.sum() == 4
+    assert np.abs(G @ st.QR[:, st.skipR]).max() < 1e-12
+    assert np.abs(G @ st.QR[:, ~st.skipR]).min(axis=0).max() > 1e-3
