@@ -1,0 +1,315 @@
+#!/usr/bin/env python
+"""Throughput of the batched SOAP step (Alg. 1) on one dense transformer block.
+
+Workload: hidden 2048, 16 heads, SwiGLU FFN 8192 -- Wq, Wk, Wv, Wo 2048x2048, W_gate and
+W_up 2048x8192, W_down 8192x2048, fp32 master weights, every side preconditioned, seeded
+synthetic gradients (rank-structured power law + noise). One "step" = one soap_step over
+all 7 matrices. Metric: SOAP steps/s for the whole block, plus effective TFLOP/s from the
+fixed FLOP model of Alg. 1 (S1 as a SYRK, S2 power step, S3 Householder QR with explicit
+Q, S4 re-projection with four two-sided products, S5/S7 rotations).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {soap,reference}]
+
+N > 1 (torchrun, one rank per GPU) runs N independent replicas of the block: the step
+has no exchange, so value = N * K / max-over-ranks time. --impl reference times the
+fp64 CPU oracle on the host cores instead (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "dense_block_h2048_ffn8192"
+METRIC = "SOAP steps/sec per model + effective TFLOP/s (fraction of dense peak)"
+# fp32 FMA peak of the CUDA cores: 152 SMs x 128 lanes x 2 flop x 2.07 GHz
+FP32_SIMT_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def model_flops(rows, cols, left, right) -> float:
+    """FLOPs of one literal Alg. 1 step for one matrix (2 per multiply-add)."""
+    m, n = float(rows), float(cols)
+    f = 0.0
+    if left:
+        f += m * m * n + 2 * m ** 3 + (8.0 / 3.0) * m ** 3      # S1 (SYRK), S2, S3
+    if right:
+        f += n * n * m + 2 * n ** 3 + (8.0 / 3.0) * n ** 3
+    rot = (m * m * n if left else 0.0) + (m * n * n if right else 0.0)
+    f += (4 + 2 + 2) * rot                                      # S4, S5, S7
+    return f
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples every 200 ms while the timed region runs."""
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index),
+                 "--query-gpu=index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons, power = [], [], set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+                power.append(float(parts[3]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "samples": len(sm),
+                "power_w_max": max(power), "reasons": sorted(reasons)}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        try:
+            return json.load(open(p)), "measured"
+        except ValueError:
+            pass
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+def oracle_sample(steps: int, warmup: int):
+    """Times the fp64 oracle's SOAP step on Wq (2048x2048) of the block, on the host cores.
+    Returns (seconds per sampled step, block steps/s extrapolated by the FLOP model, threads)."""
+    from oracle.soap_ref import HParams, MatrixState, soap_step
+    from paper_2607_20548_gb300.workloads import WORKLOADS, make_stream
+
+    specs, _ = WORKLOADS[WORKLOAD]
+    stream = make_stream(WORKLOAD, seed=0, device="cpu", specs=[0])
+    W = stream.weights()[0][0].numpy().astype(np.float64)
+    st = MatrixState(2048, 2048, True, True, np.float64)
+    hp = HParams()
+    times = []
+    for t in range(1, steps + warmup + 1):
+        G = stream.grads(t)[0][0].numpy()
+        t0 = time.perf_counter()
+        W, _ = soap_step(st, W, G, hp)
+        if t > warmup:
+            times.append(time.perf_counter() - t0)
+    per = float(np.mean(times))
+    block = sum(model_flops(s.rows, s.cols, s.left, s.right) for s in specs)
+    scale = block / model_flops(2048, 2048, True, True)
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return per, 1.0 / (per * scale), threads, scale
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    per, sps, threads, scale = oracle_sample(args.steps, args.warmup)
+    sample = (f"oracle fp64 step of Wq (2048x2048) timed over {args.steps} steps after {args.warmup} warm-up; "
+              f"whole-block time = {scale:.1f}x by the FLOP model")
+    line = {"impl": "reference", "metric": METRIC, "value": sps, "unit": "steps/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / sps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "matrices": 7, "parallelism": "replicas"},
+            "cpu_baseline": {"value": sps, "unit": "steps/s", "cores": threads, "kind": "oracle", "sample": sample},
+            "e2e": {"value": sps, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_soap(args):
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("gloo")
+    from paper_2607_20548_gb300 import SoapOptimizer, build, default_hparams
+    from paper_2607_20548_gb300 import soap as S
+    from paper_2607_20548_gb300.workloads import WORKLOADS, make_stream
+
+    if not os.path.exists(S.LIB_PATH):
+        build.build()
+    specs, _ = WORKLOADS[WORKLOAD]
+    gen = make_stream(WORKLOAD, seed=rank, device=dev)
+    opt = SoapOptimizer([(s.rows, s.cols, s.left, s.right) for s in specs], default_hparams(), device=local)
+
+    def flat(tensors):
+        out = [None] * len(specs)
+        for (spec, idx), t in zip(gen.groups, tensors):
+            for b, j in enumerate(idx):
+                out[j] = t[b]
+        return out
+
+    W = flat([w.contiguous() for w in gen.weights()])
+    npool = min(args.steps + args.warmup, 4)
+    pool = [flat(gen.grads(t + 1)) for t in range(npool)]
+    stream = torch.cuda.current_stream()
+    for t in range(args.warmup):
+        opt.step(W, pool[t % npool])
+    torch.cuda.synchronize()
+    if opt.status() != 0:
+        raise RuntimeError("device status after warm-up: " + opt.last_error())
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    # timed region: K steps, inputs resident in HBM (state 3 GB >> 129 MB L2)
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    opt.profile_begin(1 << 18)
+    barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for t in range(args.steps):
+            opt.step(W, pool[(args.warmup + t) % npool])
+        stop.record(stream)
+        torch.cuda.synchronize()
+    prof = opt.profile_end()
+    barrier()
+    elapsed = start.elapsed_time(stop) / 1e3
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([elapsed], dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        elapsed = float(tt.item())
+    value = world * args.steps / elapsed
+
+    # end to end through the public API: pinned host gradients in, updated weights out
+    host_g = [[g.cpu().pin_memory() for g in pool[i]] for i in range(npool)]
+    host_w = [w.cpu().pin_memory() for w in W]
+    dev_g = [torch.empty_like(g) for g in pool[0]]
+    h2d = sum(g.numel() * 4 for g in dev_g)
+    d2h = sum(w.numel() * 4 for w in W)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for t in range(args.steps):
+        for d, h in zip(dev_g, host_g[t % npool]):
+            d.copy_(h, non_blocking=True)
+        opt.step(W, dev_g)
+        for h, w in zip(host_w, W):
+            h.copy_(w, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_s = e0.elapsed_time(e1) / 1e3
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([e2e_s], dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_s = float(tt.item())
+    if opt.status() != 0:
+        raise RuntimeError("device status after timed steps: " + opt.last_error())
+
+    if rank != 0:
+        opt.destroy()
+        return
+    block_flops = sum(model_flops(s.rows, s.cols, s.left, s.right) for s in specs)
+    peaks, peak_src = measured_peaks()
+    fams = {k: v for k, v in prof.items() if k != "overflow"}
+    top = max(fams, key=lambda k: fams[k]["ms"])
+    st = fams[top]
+    launches = sum(v["launches"] for v in fams.values())
+    if top in ("gemm_simt",):
+        achieved = st["flops"] / (st["ms"] / 1e3) / 1e12
+        roof = {"kernel": top, "bound": "alu", "achieved": achieved, "peak": FP32_SIMT_PEAK_TFLOPS,
+                "unit": "TFLOP/s", "frac": achieved / FP32_SIMT_PEAK_TFLOPS,
+                "peak_source": "fp32 FMA peak of the CUDA cores, 152 SMs x 128 lanes x 2 x 2.07 GHz",
+                "traffic": None, "launches": st["launches"], "avg_launch_us": 1e3 * st["ms"] / max(1, st["launches"])}
+    else:
+        achieved = st["bytes"] / (st["ms"] / 1e3) / 1e9
+        roof = {"kernel": top, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"], "peak_source": peak_src, "traffic": None,
+                "launches": st["launches"], "avg_launch_us": 1e3 * st["ms"] / max(1, st["launches"])}
+    per, sps, threads, scale = oracle_sample(1, 0)
+    line = {
+        "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "matrices": 7,
+                   "shapes": "4x 2048x2048, 2x 2048x8192, 1x 8192x2048, all sides preconditioned",
+                   "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (3 GB of optimizer state per step)"},
+        "effective_tflops": block_flops * value / world / 1e12,
+        "effective_frac_of_fp32_simt_peak": block_flops * value / world / 1e12 / FP32_SIMT_PEAK_TFLOPS,
+        "model_flop_per_step": block_flops,
+        "roofline": roof,
+        "kernel_time_share": {k: round(v["ms"] / max(1e-9, sum(x["ms"] for x in fams.values())), 4)
+                              for k, v in fams.items()},
+        "cpu_baseline": {"value": sps, "unit": "steps/s", "cores": threads, "kind": "oracle",
+                         "sample": f"one fp64 oracle step of Wq (2048x2048) took {per:.1f} s; whole block "
+                                   f"= {scale:.1f}x that by the FLOP model"},
+        "e2e": {"value": world * args.steps / e2e_s, "unit": "steps/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    opt.destroy()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["soap", "reference"], default="soap")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_soap(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -143,6 +143,35 @@ const char* soap_last_error(soap_handle h);
 /* Frees all state and workspace. Safe on NULL. Synchronises the device first. */
 void soap_destroy(soap_handle h);
 
+/* ---- kernel timing (diagnostics; the paper has no counterpart) ---------------------- */
+
+/* Kernel families the library launches. */
+typedef enum {
+  SOAP_KERNEL_GEMM_SIMT = 0,   /* CUDA-core fp32 batched GEMM */
+  SOAP_KERNEL_GEMM_TC = 1,     /* tcgen05 3xTF32 batched GEMM */
+  SOAP_KERNEL_QR_PANEL = 2,    /* cluster panel factorisation of the QR */
+  SOAP_KERNEL_ELEMENTWISE = 3, /* momentum, Adam, weight update */
+  SOAP_KERNEL_OTHER = 4        /* norms, identity fills */
+} soap_kernel_family;
+
+typedef struct {
+  int32_t family;    /* soap_kernel_family */
+  int64_t launches;  /* kernel launches timed */
+  double ms;         /* sum of per-launch CUDA-event durations */
+  double flops;      /* sum of algorithmic FLOPs of those launches */
+  double bytes;      /* sum of algorithmic bytes moved by those launches */
+} soap_kernel_stats;
+
+/* Starts timing every kernel launch the calling thread makes through the library
+ * (up to max_launches; later launches are counted as overflow and not timed). Each
+ * launch is bracketed by two CUDA events on its own stream. */
+soap_status_t soap_profile_begin(soap_handle h, int64_t max_launches);
+
+/* Synchronises `stream`, stops timing and writes one soap_kernel_stats per family
+ * (5 entries) to out[]. *overflow is set to 1 if max_launches was exceeded. */
+soap_status_t soap_profile_end(soap_handle h, soap_stream_t stream, soap_kernel_stats* out,
+                               int32_t* overflow);
+
 /* ---- stand-alone sub-steps (the same kernels soap_step runs) ------------------- */
 
 /* S3, Alg. 1 "QR(L_t Q_L).Q": for `batch` square n x n matrices P (device,

@@ -1,0 +1,150 @@
+// Elementwise parts of the SOAP step (HBM-bound; grid-stride, float4 where aligned).
+//
+//  * momentum_and_copy: the first moment kept in the ORIGINAL basis,
+//      M_hat <- beta1 M_hat + (1 - beta1) G,
+//    which is Alg. 1's re-projection m <- Q_new^T (Q_old m Q_old^T) Q_new followed
+//    by m <- beta1 m + (1 - beta1) Q_new^T G Q_new, written as M_hat = Q m Q^T
+//    (exact for the square orthogonal Q of both sides). It also copies G into the
+//    library's contiguous gradient arena and flags non-finite gradients.
+//  * adam_in_basis: v <- beta2 v + (1 - beta2) G'^2 and N = m / (sqrt(v) + eps)
+//    (Alg. 1 "Calculate Adam update"; v is never re-projected), with the zero-column
+//    guard.
+//  * weight_update: W <- (1 - lr wd) W - lr N for a matrix with no preconditioned
+//    side (Alg. 1 "Weight decay and update" with Q_L = Q_R = I).
+#include "profile.h"
+#include "soap_internal.h"
+
+namespace soap {
+namespace {
+
+constexpr int kThreads = 256;
+
+inline int blocks_for(int64_t elems, int batch) {
+  int64_t want = (elems / 4 + kThreads - 1) / kThreads;
+  if (want < 1) want = 1;
+  const int64_t cap = batch >= 64 ? 4 : (batch >= 8 ? 32 : 256);
+  return (int)(want < cap ? want : cap);
+}
+
+__global__ void momentum_copy_kernel(const float* const* grads, float* Gc, float* Mh,
+                                     int64_t elems, float beta1, int* status) {
+  const int b = blockIdx.y;
+  const float* g = grads[b];
+  float* gc = Gc + (int64_t)b * elems;
+  float* mh = Mh + (int64_t)b * elems;
+  const float c1 = 1.f - beta1;
+  int bad = 0;
+  const bool vec = ((reinterpret_cast<uintptr_t>(g) | reinterpret_cast<uintptr_t>(gc) |
+                     reinterpret_cast<uintptr_t>(mh)) & 15) == 0;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  int64_t start = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  int64_t tail = 0;
+  if (vec) {
+    const int64_t n4 = elems / 4;
+    for (int64_t i = start; i < n4; i += stride) {
+      float4 x = reinterpret_cast<const float4*>(g)[i];
+      float4 m = reinterpret_cast<float4*>(mh)[i];
+      bad |= !isfinite(x.x) | !isfinite(x.y) | !isfinite(x.z) | !isfinite(x.w);
+      m.x = fmaf(beta1, m.x, c1 * x.x);
+      m.y = fmaf(beta1, m.y, c1 * x.y);
+      m.z = fmaf(beta1, m.z, c1 * x.z);
+      m.w = fmaf(beta1, m.w, c1 * x.w);
+      reinterpret_cast<float4*>(gc)[i] = x;
+      reinterpret_cast<float4*>(mh)[i] = m;
+    }
+    tail = n4 * 4;
+  }
+  for (int64_t i = tail + start; i < elems; i += stride) {
+    const float x = g[i];
+    bad |= !isfinite(x);
+    mh[i] = fmaf(beta1, mh[i], c1 * x);
+    gc[i] = x;
+  }
+  if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(status, kStatusNonFinite);
+}
+
+__global__ void adam_kernel(float* Gp, const float* Mp, float* V, int rows, int cols, float beta2,
+                            float eps, float inv_bc1, float inv_sqrt_bc2, const uint8_t* skipL,
+                            const uint8_t* skipR, int* status) {
+  const int b = blockIdx.y;
+  const int64_t elems = (int64_t)rows * cols;
+  float* gp = Gp + (int64_t)b * elems;
+  const float* mp = Mp + (int64_t)b * elems;
+  float* v = V + (int64_t)b * elems;
+  const uint8_t* sl = skipL ? skipL + (int64_t)b * rows : nullptr;
+  const uint8_t* sr = skipR ? skipR + (int64_t)b * cols : nullptr;
+  const float c2 = 1.f - beta2;
+  int bad = 0;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < elems; i += stride) {
+    const float g = gp[i];
+    const float m = mp[i];
+    const float vn = fmaf(beta2, v[i], c2 * g * g);
+    v[i] = vn;
+    float nv = (m * inv_bc1) / (sqrtf(vn) * inv_sqrt_bc2 + eps);
+    if ((sl && sl[i / cols]) || (sr && sr[i % cols])) nv = 0.f;
+    bad |= !isfinite(nv);
+    gp[i] = nv;
+  }
+  if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(status, kStatusNonFinite);
+}
+
+__global__ void weight_update_kernel(float* const* params, const float* D, int64_t elems, float lr,
+                                     float wd) {
+  const int b = blockIdx.y;
+  float* w = params[b];
+  const float* d = D + (int64_t)b * elems;
+  const float keep = 1.f - lr * wd;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < elems; i += stride)
+    w[i] = fmaf(keep, w[i], -lr * d[i]);
+}
+
+__global__ void identity_kernel(float* Q, int n) {
+  const int b = blockIdx.y;
+  float* q = Q + (int64_t)b * n * n;
+  const int64_t nn = (int64_t)n * n;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nn; i += stride)
+    q[i] = (i / n == i % n) ? 1.f : 0.f;
+}
+
+}  // namespace
+
+cudaError_t momentum_and_copy(const float* const* grads, float* Gc, float* Mhat, int64_t elems,
+                              int batch, float beta1, int* status, cudaStream_t s) {
+  if (elems <= 0 || batch <= 0) return cudaSuccess;
+  ProfScope prof(kFamElementwise, 3.0 * elems * batch, 16.0 * elems * batch, s);
+  momentum_copy_kernel<<<dim3(blocks_for(elems, batch), batch), kThreads, 0, s>>>(grads, Gc, Mhat, elems,
+                                                                                   beta1, status);
+  return cudaGetLastError();
+}
+
+cudaError_t adam_in_basis(float* Gp, const float* Mp, float* V, int rows, int cols, int batch,
+                          float beta1, float beta2, float eps, float bc1, float bc2,
+                          const uint8_t* skipL, const uint8_t* skipR, int* status, cudaStream_t s) {
+  (void)beta1;
+  const int64_t elems = (int64_t)rows * cols;
+  if (elems <= 0 || batch <= 0) return cudaSuccess;
+  ProfScope prof(kFamElementwise, 8.0 * elems * batch, 16.0 * elems * batch, s);
+  adam_kernel<<<dim3(blocks_for(elems, batch), batch), kThreads, 0, s>>>(
+      Gp, Mp, V, rows, cols, beta2, eps, 1.f / bc1, 1.f / sqrtf(bc2), skipL, skipR, status);
+  return cudaGetLastError();
+}
+
+cudaError_t weight_update(float* const* params, const float* D, int64_t elems, int batch, float lr,
+                          float wd, cudaStream_t s) {
+  if (elems <= 0 || batch <= 0) return cudaSuccess;
+  ProfScope prof(kFamElementwise, 3.0 * elems * batch, 12.0 * elems * batch, s);
+  weight_update_kernel<<<dim3(blocks_for(elems, batch), batch), kThreads, 0, s>>>(params, D, elems, lr, wd);
+  return cudaGetLastError();
+}
+
+cudaError_t set_identity(float* Q, int n, int batch, cudaStream_t s) {
+  if (n <= 0 || batch <= 0) return cudaSuccess;
+  ProfScope prof(kFamOther, 0, 4.0 * n * n * batch, s);
+  identity_kernel<<<dim3(blocks_for((int64_t)n * n, batch), batch), kThreads, 0, s>>>(Q, n);
+  return cudaGetLastError();
+}
+
+}  // namespace soap

@@ -1,0 +1,640 @@
+// libsoap: the C ABI of include/soap.h.
+//
+// Plan: matrices with the same (rows, cols, sides) form a class; each class keeps
+// its state in contiguous arenas ([count][rows][cols], [count][rows][rows], ...)
+// so every contraction of the step is one batched GEMM per class. Classes run one
+// after another on the caller's stream and share one workspace sized for the
+// largest class.
+//
+// Per class, the step (Alg. 1 with the standard factor EMAs of section 2) is:
+//   M_hat <- b1 M_hat + (1-b1) G, Gc <- G                 momentum in the original basis
+//   L <- b L + (1-b) Gc Gc^T, R <- b R + (1-b) Gc^T Gc     S1
+//   P = L Q_L -> Q_L = QR(P).Q; same for R                 S2, S3 (when t mod F == 0)
+//   X1 = Q_L^T Gc, X2 = Q_L^T M_hat                        S5, S4 (re-projected m)
+//   G' = X1 Q_R, m = X2 Q_R
+//   v <- b2 v + (1-b2) G'^2, N = m / (sqrt(v) + eps)        S6
+//   X1 = Q_L N; W <- (1 - lr wd) W - lr X1 Q_R^T           S7, S8 (fused in the GEMM epilogue)
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "profile.h"
+#include "soap_internal.h"
+
+namespace {
+
+struct ClassState {
+  int64_t rows = 0, cols = 0;
+  bool left = false, right = false;
+  int count = 0;
+  std::vector<int> members;
+  float* Gc = nullptr;
+  float* Mhat = nullptr;
+  float* V = nullptr;
+  float* L = nullptr;
+  float* QL = nullptr;
+  float* R = nullptr;
+  float* QR = nullptr;
+  uint8_t* skipL = nullptr;
+  uint8_t* skipR = nullptr;
+  size_t ptr_offset = 0;  // index of this class's params pointers in the pointer table
+};
+
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+    if (prev != dev) cudaSetDevice(dev);
+  }
+  ~DeviceGuard() {
+    int cur = -1;
+    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+  }
+};
+
+}  // namespace
+
+struct soap_s {
+  int device = 0;
+  soap_hparams hp{};
+  float lr = 0.f, wd = 0.f;
+  int64_t t = 0;
+  std::vector<soap_shape> shapes;
+  std::vector<std::pair<int, int>> loc;  // matrix index -> (class, slot)
+  std::vector<ClassState> classes;
+  float* X1 = nullptr;
+  float* X2 = nullptr;
+  float* Gp = nullptr;
+  float* Mp = nullptr;
+  void* qr_ws = nullptr;
+  size_t qr_ws_bytes = 0;
+  int* d_status = nullptr;
+  int* h_status = nullptr;          // pinned mirror, refreshed after every step
+  cudaEvent_t status_ev = nullptr;
+  bool status_pending = false;
+  void** h_ptrs = nullptr;          // pinned staging for the params/grads pointer table
+  void** d_ptrs = nullptr;
+  size_t nptrs = 0;
+  cudaEvent_t stage_ev = nullptr;
+  bool stage_pending = false;
+  std::vector<void*> last_ptrs;
+  std::vector<void*> allocs;
+  soap::Profiler prof;
+  std::string err;
+};
+
+namespace {
+
+soap_status_t fail(soap_handle h, soap_status_t code, const std::string& msg) {
+  if (h) h->err = msg;
+  return code;
+}
+
+soap_status_t cuda_fail(soap_handle h, cudaError_t e, const char* what) {
+  std::string m = std::string(what) + ": " + cudaGetErrorString(e);
+  if (e == cudaErrorMemoryAllocation) return fail(h, SOAP_ERR_OOM, m);
+  return fail(h, SOAP_ERR_CUDA, m);
+}
+
+#define SOAP_CUDA(h, expr)                              \
+  do {                                                  \
+    cudaError_t e_ = (expr);                            \
+    if (e_ != cudaSuccess) return cuda_fail(h, e_, #expr); \
+  } while (0)
+
+soap_status_t status_code(int bits) {
+  if (bits & soap::kStatusTimeout) return SOAP_ERR_TIMEOUT;
+  if (bits & soap::kStatusQrBreakdown) return SOAP_ERR_QR_BREAKDOWN;
+  if (bits & soap::kStatusNonFinite) return SOAP_ERR_NONFINITE;
+  return SOAP_OK;
+}
+
+cudaError_t dalloc(soap_handle h, void** p, size_t bytes) {
+  *p = nullptr;
+  if (bytes == 0) return cudaSuccess;
+  cudaError_t e = cudaMalloc(p, bytes);
+  if (e == cudaSuccess) h->allocs.push_back(*p);
+  return e;
+}
+
+void free_all(soap_handle h) {
+  if (soap::t_profiler == &h->prof) soap::t_profiler = nullptr;
+  for (cudaEvent_t ev : h->prof.events) cudaEventDestroy(ev);
+  h->prof.events.clear();
+  for (void* p : h->allocs) cudaFree(p);
+  h->allocs.clear();
+  if (h->h_status) cudaFreeHost(h->h_status);
+  if (h->h_ptrs) cudaFreeHost(h->h_ptrs);
+  if (h->status_ev) cudaEventDestroy(h->status_ev);
+  if (h->stage_ev) cudaEventDestroy(h->stage_ev);
+  h->h_status = nullptr;
+  h->h_ptrs = nullptr;
+  h->status_ev = h->stage_ev = nullptr;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+}  // namespace
+
+extern "C" {
+
+void soap_default_hparams(soap_hparams* hp) {
+  if (!hp) return;
+  hp->lr = 3e-3f;
+  hp->beta1 = 0.95f;
+  hp->beta2 = 0.95f;
+  hp->factor_beta = 0.95f;
+  hp->eps = 1e-8f;
+  hp->weight_decay = 0.1f;
+  hp->eig_every = 1;
+  hp->bias_correction = 0;
+  hp->qr_tol = 1e-4f;
+  hp->guard = 1;
+}
+
+soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparams* hp,
+                          int32_t device, soap_handle* out) {
+  if (!out) return SOAP_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!shapes || n <= 0 || !hp) return SOAP_ERR_INVALID_ARG;
+  if (hp->eig_every < 1 || !(hp->eps >= 0.f) || !(hp->qr_tol >= 0.f)) return SOAP_ERR_INVALID_ARG;
+  for (int i = 0; i < n; ++i) {
+    const soap_shape& s = shapes[i];
+    if (s.rows < 1 || s.cols < 1 || s.rows > (1 << 20) || s.cols > (1 << 20)) return SOAP_ERR_INVALID_ARG;
+    if (s.rows * s.cols > (int64_t(1) << 31) - 1) return SOAP_ERR_INVALID_ARG;
+    if ((s.precond_left && s.rows > 8192) || (s.precond_right && s.cols > 8192)) return SOAP_ERR_INVALID_ARG;
+  }
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) return SOAP_ERR_CUDA;
+  DeviceGuard g(device);
+  soap_handle h = new soap_s();
+  h->device = device;
+  h->hp = *hp;
+  h->lr = hp->lr;
+  h->wd = hp->weight_decay;
+  h->shapes.assign(shapes, shapes + n);
+  h->loc.resize(n);
+
+  std::map<std::tuple<int64_t, int64_t, bool, bool>, int> index;
+  for (int i = 0; i < n; ++i) {
+    const soap_shape& s = shapes[i];
+    auto key = std::make_tuple(s.rows, s.cols, s.precond_left != 0, s.precond_right != 0);
+    auto it = index.find(key);
+    int ci;
+    if (it == index.end()) {
+      ci = (int)h->classes.size();
+      index[key] = ci;
+      ClassState c;
+      c.rows = s.rows;
+      c.cols = s.cols;
+      c.left = s.precond_left != 0;
+      c.right = s.precond_right != 0;
+      h->classes.push_back(c);
+    } else {
+      ci = it->second;
+    }
+    h->loc[i] = {ci, h->classes[ci].count};
+    h->classes[ci].members.push_back(i);
+    h->classes[ci].count++;
+  }
+  for (auto& c : h->classes) {
+    if (c.count > 65535) {
+      delete h;
+      return SOAP_ERR_INVALID_ARG;
+    }
+  }
+
+  size_t ws_mat = 0, ws_qr = 0;
+  size_t off = 0;
+  cudaError_t e = cudaSuccess;
+  for (auto& c : h->classes) {
+    const size_t mn = (size_t)c.count * c.rows * c.cols;
+    c.ptr_offset = off;
+    off += 2 * (size_t)c.count;
+    if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gc, mn * 4);
+    if (e == cudaSuccess) e = dalloc(h, (void**)&c.Mhat, mn * 4);
+    if (e == cudaSuccess) e = dalloc(h, (void**)&c.V, mn * 4);
+    if (c.left) {
+      const size_t mm = (size_t)c.count * c.rows * c.rows;
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.L, mm * 4);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.QL, mm * 4);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.skipL, (size_t)c.count * c.rows);
+      ws_qr = std::max(ws_qr, soap::qr_workspace_bytes((int)c.rows, c.count));
+    }
+    if (c.right) {
+      const size_t nn = (size_t)c.count * c.cols * c.cols;
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.R, nn * 4);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.QR, nn * 4);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.skipR, (size_t)c.count * c.cols);
+      ws_qr = std::max(ws_qr, soap::qr_workspace_bytes((int)c.cols, c.count));
+    }
+    ws_mat = std::max(ws_mat, mn);
+  }
+  h->nptrs = off;
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->X1, ws_mat * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->X2, ws_mat * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Gp, ws_mat * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Mp, ws_mat * 4);
+  if (e == cudaSuccess) e = dalloc(h, &h->qr_ws, ws_qr);
+  h->qr_ws_bytes = ws_qr;
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_status, sizeof(int));
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_ptrs, h->nptrs * sizeof(void*));
+  if (e == cudaSuccess) e = cudaMallocHost((void**)&h->h_status, sizeof(int));
+  if (e == cudaSuccess) e = cudaMallocHost((void**)&h->h_ptrs, h->nptrs * sizeof(void*));
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->status_ev, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->stage_ev, cudaEventDisableTiming);
+  if (e != cudaSuccess) {
+    soap_status_t code = e == cudaErrorMemoryAllocation ? SOAP_ERR_OOM : SOAP_ERR_CUDA;
+    free_all(h);
+    delete h;
+    cudaGetLastError();
+    return code;
+  }
+  *h->h_status = 0;
+  // initial state: L = R = 0, Q = I, M_hat = v = 0
+  for (auto& c : h->classes) {
+    const size_t mn = (size_t)c.count * c.rows * c.cols;
+    if (e == cudaSuccess) e = cudaMemset(c.Mhat, 0, mn * 4);
+    if (e == cudaSuccess) e = cudaMemset(c.V, 0, mn * 4);
+    if (c.left) {
+      if (e == cudaSuccess) e = cudaMemset(c.L, 0, (size_t)c.count * c.rows * c.rows * 4);
+      if (e == cudaSuccess) e = soap::set_identity(c.QL, (int)c.rows, c.count, 0);
+      if (e == cudaSuccess) e = cudaMemset(c.skipL, 0, (size_t)c.count * c.rows);
+    }
+    if (c.right) {
+      if (e == cudaSuccess) e = cudaMemset(c.R, 0, (size_t)c.count * c.cols * c.cols * 4);
+      if (e == cudaSuccess) e = soap::set_identity(c.QR, (int)c.cols, c.count, 0);
+      if (e == cudaSuccess) e = cudaMemset(c.skipR, 0, (size_t)c.count * c.cols);
+    }
+  }
+  if (e == cudaSuccess) e = cudaMemset(h->d_status, 0, sizeof(int));
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    free_all(h);
+    delete h;
+    cudaGetLastError();
+    return SOAP_ERR_CUDA;
+  }
+  h->last_ptrs.assign(h->nptrs, nullptr);
+  *out = h;
+  return SOAP_OK;
+}
+
+soap_status_t soap_set_lr(soap_handle h, float lr, float weight_decay) {
+  if (!h || !(lr >= 0.f) || !(weight_decay >= 0.f)) return SOAP_ERR_INVALID_ARG;
+  h->lr = lr;
+  h->wd = weight_decay;
+  return SOAP_OK;
+}
+
+soap_status_t soap_step(soap_handle h, float* const* params, const float* const* grads,
+                        soap_stream_t stream_) {
+  if (!h) return SOAP_ERR_INVALID_ARG;
+  if (!params || !grads) return fail(h, SOAP_ERR_INVALID_ARG, "soap_step: null pointer array");
+  const int n = (int)h->shapes.size();
+  for (int i = 0; i < n; ++i) {
+    if (!params[i] || !grads[i] || !aligned16(params[i]) || !aligned16(grads[i]))
+      return fail(h, SOAP_ERR_INVALID_ARG, "soap_step: matrix " + std::to_string(i) +
+                                               " has a null or non-16-byte-aligned pointer");
+  }
+  DeviceGuard g(h->device);
+  cudaStream_t s = (cudaStream_t)stream_;
+  // sticky status from a finished earlier step
+  if (h->status_pending && cudaEventQuery(h->status_ev) == cudaSuccess) {
+    h->status_pending = false;
+    soap_status_t st = status_code(*h->h_status);
+    if (st != SOAP_OK) return fail(h, st, "soap_step: sticky device status from an earlier step");
+  }
+  // pointer table: [class][params..., grads...], uploaded only when it changed
+  bool changed = false;
+  for (auto& c : h->classes) {
+    for (int j = 0; j < c.count; ++j) {
+      const int m = c.members[j];
+      void* pp = params[m];
+      void* gp = const_cast<float*>(grads[m]);
+      if (h->last_ptrs[c.ptr_offset + j] != pp || h->last_ptrs[c.ptr_offset + c.count + j] != gp) changed = true;
+      h->last_ptrs[c.ptr_offset + j] = pp;
+      h->last_ptrs[c.ptr_offset + c.count + j] = gp;
+    }
+  }
+  if (changed) {
+    if (h->stage_pending) SOAP_CUDA(h, cudaEventSynchronize(h->stage_ev));
+    std::memcpy(h->h_ptrs, h->last_ptrs.data(), h->nptrs * sizeof(void*));
+    SOAP_CUDA(h, cudaMemcpyAsync(h->d_ptrs, h->h_ptrs, h->nptrs * sizeof(void*), cudaMemcpyHostToDevice, s));
+    SOAP_CUDA(h, cudaEventRecord(h->stage_ev, s));
+    h->stage_pending = true;
+  }
+
+  h->t += 1;
+  const int64_t t = h->t;
+  const soap_hparams& hp = h->hp;
+  const bool refresh = (t % hp.eig_every) == 0;
+  const float bc1 = hp.bias_correction ? 1.f - powf(hp.beta1, (float)t) : 1.f;
+  const float bc2 = hp.bias_correction ? 1.f - powf(hp.beta2, (float)t) : 1.f;
+  using soap::strided;
+  using soap::strided_mut;
+
+  for (auto& c : h->classes) {
+    const int B = c.count;
+    const int m = (int)c.rows, nc = (int)c.cols;
+    const int64_t mn = (int64_t)m * nc;
+    float* const* d_params = reinterpret_cast<float* const*>(h->d_ptrs + c.ptr_offset);
+    const float* const* d_grads = reinterpret_cast<const float* const*>(h->d_ptrs + c.ptr_offset + B);
+
+    SOAP_CUDA(h, soap::momentum_and_copy(d_grads, c.Gc, c.Mhat, mn, B, hp.beta1, h->d_status, s));
+    const float fb = hp.factor_beta;
+    if (c.left) {  // S1: L <- b L + (1-b) G G^T
+      SOAP_CUDA(h, soap::gemm(false, true, m, m, nc, 1.f - fb, strided(c.Gc, nc, mn), strided(c.Gc, nc, mn), fb,
+                              strided_mut(c.L, m, (int64_t)m * m), B, s));
+    }
+    if (c.right) {  // S1: R <- b R + (1-b) G^T G
+      SOAP_CUDA(h, soap::gemm(true, false, nc, nc, m, 1.f - fb, strided(c.Gc, nc, mn), strided(c.Gc, nc, mn), fb,
+                              strided_mut(c.R, nc, (int64_t)nc * nc), B, s));
+    }
+    if (refresh) {
+      float* P = (float*)h->qr_ws;  // the QR factors its workspace's first matrix block in place
+      if (c.left) {  // S2 + S3 on the left side
+        SOAP_CUDA(h, soap::gemm(false, false, m, m, m, 1.f, strided(c.L, m, (int64_t)m * m),
+                                strided(c.QL, m, (int64_t)m * m), 0.f, strided_mut(P, m, (int64_t)m * m), B, s));
+        SOAP_CUDA(h, soap::qr_q(m, B, P, c.QL, c.skipL, hp.qr_tol, h->qr_ws, h->qr_ws_bytes, h->d_status, s));
+      }
+      if (c.right) {
+        SOAP_CUDA(h, soap::gemm(false, false, nc, nc, nc, 1.f, strided(c.R, nc, (int64_t)nc * nc),
+                                strided(c.QR, nc, (int64_t)nc * nc), 0.f, strided_mut(P, nc, (int64_t)nc * nc), B, s));
+        SOAP_CUDA(h, soap::qr_q(nc, B, P, c.QR, c.skipR, hp.qr_tol, h->qr_ws, h->qr_ws_bytes, h->d_status, s));
+      }
+    }
+    // S5 and the re-projected first moment: G' = Q_L^T G Q_R, m = Q_L^T M_hat Q_R
+    const float* xg = c.Gc;
+    const float* xm = c.Mhat;
+    if (c.left) {
+      SOAP_CUDA(h, soap::gemm(true, false, m, nc, m, 1.f, strided(c.QL, m, (int64_t)m * m), strided(c.Gc, nc, mn), 0.f,
+                              strided_mut(h->X1, nc, mn), B, s));
+      SOAP_CUDA(h, soap::gemm(true, false, m, nc, m, 1.f, strided(c.QL, m, (int64_t)m * m), strided(c.Mhat, nc, mn), 0.f,
+                              strided_mut(h->X2, nc, mn), B, s));
+      xg = h->X1;
+      xm = h->X2;
+    }
+    float* gp;
+    const float* mp;
+    if (c.right) {
+      SOAP_CUDA(h, soap::gemm(false, false, m, nc, nc, 1.f, strided(xg, nc, mn), strided(c.QR, nc, (int64_t)nc * nc), 0.f,
+                              strided_mut(h->Gp, nc, mn), B, s));
+      SOAP_CUDA(h, soap::gemm(false, false, m, nc, nc, 1.f, strided(xm, nc, mn), strided(c.QR, nc, (int64_t)nc * nc), 0.f,
+                              strided_mut(h->Mp, nc, mn), B, s));
+      gp = h->Gp;
+      mp = h->Mp;
+    } else {
+      gp = const_cast<float*>(xg);  // X1, or the gradient arena copy when no side rotates
+      mp = xm;
+    }
+    // S6
+    SOAP_CUDA(h, soap::adam_in_basis(gp, mp, c.V, m, nc, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
+                                     (hp.guard && c.left) ? c.skipL : nullptr,
+                                     (hp.guard && c.right) ? c.skipR : nullptr, h->d_status, s));
+    // S7 + S8: W <- (1 - lr wd) W - lr Q_L N Q_R^T
+    const float keep = 1.f - h->lr * h->wd;
+    soap::MutOperand W{nullptr, d_params, 0, 0, nc};
+    if (c.left && c.right) {
+      SOAP_CUDA(h, soap::gemm(false, false, m, nc, m, 1.f, strided(c.QL, m, (int64_t)m * m), strided(gp, nc, mn), 0.f,
+                              strided_mut(h->X1, nc, mn), B, s));
+      SOAP_CUDA(h, soap::gemm(false, true, m, nc, nc, -h->lr, strided(h->X1, nc, mn), strided(c.QR, nc, (int64_t)nc * nc),
+                              keep, W, B, s));
+    } else if (c.left) {
+      SOAP_CUDA(h, soap::gemm(false, false, m, nc, m, -h->lr, strided(c.QL, m, (int64_t)m * m), strided(gp, nc, mn), keep,
+                              W, B, s));
+    } else if (c.right) {
+      SOAP_CUDA(h, soap::gemm(false, true, m, nc, nc, -h->lr, strided(gp, nc, mn), strided(c.QR, nc, (int64_t)nc * nc),
+                              keep, W, B, s));
+    } else {
+      SOAP_CUDA(h, soap::weight_update(d_params, gp, mn, B, h->lr, h->wd, s));
+    }
+  }
+  SOAP_CUDA(h, cudaMemcpyAsync(h->h_status, h->d_status, sizeof(int), cudaMemcpyDeviceToHost, s));
+  SOAP_CUDA(h, cudaEventRecord(h->status_ev, s));
+  h->status_pending = true;
+  return SOAP_OK;
+}
+
+size_t soap_state_bytes(soap_handle h, int32_t idx, int32_t which) {
+  if (!h || idx < 0 || idx >= (int)h->shapes.size()) return 0;
+  const soap_shape& s = h->shapes[idx];
+  switch (which) {
+    case SOAP_STATE_M:
+    case SOAP_STATE_V:
+    case SOAP_STATE_MHAT: return (size_t)s.rows * s.cols * 4;
+    case SOAP_STATE_L:
+    case SOAP_STATE_QL: return s.precond_left ? (size_t)s.rows * s.rows * 4 : 0;
+    case SOAP_STATE_R:
+    case SOAP_STATE_QR: return s.precond_right ? (size_t)s.cols * s.cols * 4 : 0;
+    case SOAP_STATE_SKIP_L: return s.precond_left ? (size_t)s.rows : 0;
+    case SOAP_STATE_SKIP_R: return s.precond_right ? (size_t)s.cols : 0;
+    default: return 0;
+  }
+}
+
+namespace {
+// Address of a stored state piece (not SOAP_STATE_M, which is derived).
+void* state_ptr(soap_handle h, int idx, int which) {
+  const auto [ci, slot] = h->loc[idx];
+  ClassState& c = h->classes[ci];
+  const size_t mn = (size_t)c.rows * c.cols, mm = (size_t)c.rows * c.rows, nn = (size_t)c.cols * c.cols;
+  switch (which) {
+    case SOAP_STATE_V: return c.V + slot * mn;
+    case SOAP_STATE_MHAT: return c.Mhat + slot * mn;
+    case SOAP_STATE_L: return c.L ? c.L + slot * mm : nullptr;
+    case SOAP_STATE_QL: return c.QL ? c.QL + slot * mm : nullptr;
+    case SOAP_STATE_R: return c.R ? c.R + slot * nn : nullptr;
+    case SOAP_STATE_QR: return c.QR ? c.QR + slot * nn : nullptr;
+    case SOAP_STATE_SKIP_L: return c.skipL ? c.skipL + slot * c.rows : nullptr;
+    case SOAP_STATE_SKIP_R: return c.skipR ? c.skipR + slot * c.cols : nullptr;
+    default: return nullptr;
+  }
+}
+}  // namespace
+
+soap_status_t soap_state_get(soap_handle h, int32_t idx, int32_t which, void* dst, soap_stream_t stream_) {
+  if (!h) return SOAP_ERR_INVALID_ARG;
+  const size_t bytes = soap_state_bytes(h, idx, which);
+  if (bytes == 0 || !dst) return fail(h, SOAP_ERR_INVALID_ARG, "soap_state_get: no such state piece");
+  DeviceGuard g(h->device);
+  cudaStream_t s = (cudaStream_t)stream_;
+  if (which != SOAP_STATE_M) {
+    SOAP_CUDA(h, cudaMemcpyAsync(dst, state_ptr(h, idx, which), bytes, cudaMemcpyDefault, s));
+    return SOAP_OK;
+  }
+  // m = Q_L^T M_hat Q_R, computed into the workspace
+  const auto [ci, slot] = h->loc[idx];
+  ClassState& c = h->classes[ci];
+  const int m = (int)c.rows, nc = (int)c.cols;
+  const int64_t mn = (int64_t)m * nc;
+  const float* x = c.Mhat + slot * mn;
+  using soap::strided;
+  using soap::strided_mut;
+  if (c.left) {
+    SOAP_CUDA(h, soap::gemm(true, false, m, nc, m, 1.f, strided(c.QL + (int64_t)slot * m * m, m, 0), strided(x, nc, 0),
+                            0.f, strided_mut(h->X1, nc, 0), 1, s));
+    x = h->X1;
+  }
+  if (c.right) {
+    SOAP_CUDA(h, soap::gemm(false, false, m, nc, nc, 1.f, strided(x, nc, 0), strided(c.QR + (int64_t)slot * nc * nc, nc, 0),
+                            0.f, strided_mut(h->Gp, nc, 0), 1, s));
+    x = h->Gp;
+  }
+  SOAP_CUDA(h, cudaMemcpyAsync(dst, x, bytes, cudaMemcpyDefault, s));
+  return SOAP_OK;
+}
+
+soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const void* src, soap_stream_t stream_) {
+  if (!h) return SOAP_ERR_INVALID_ARG;
+  const size_t bytes = soap_state_bytes(h, idx, which);
+  if (bytes == 0 || !src) return fail(h, SOAP_ERR_INVALID_ARG, "soap_state_set: no such state piece");
+  DeviceGuard g(h->device);
+  cudaStream_t s = (cudaStream_t)stream_;
+  if (which != SOAP_STATE_M) {
+    SOAP_CUDA(h, cudaMemcpyAsync(state_ptr(h, idx, which), src, bytes, cudaMemcpyDefault, s));
+    return SOAP_OK;
+  }
+  // M_hat = Q_L m Q_R^T
+  const auto [ci, slot] = h->loc[idx];
+  ClassState& c = h->classes[ci];
+  const int m = (int)c.rows, nc = (int)c.cols;
+  const int64_t mn = (int64_t)m * nc;
+  float* dstm = c.Mhat + slot * mn;
+  using soap::strided;
+  using soap::strided_mut;
+  SOAP_CUDA(h, cudaMemcpyAsync(h->Gp, src, bytes, cudaMemcpyDefault, s));
+  const float* x = h->Gp;
+  if (c.left) {
+    float* out = c.right ? h->X1 : dstm;
+    SOAP_CUDA(h, soap::gemm(false, false, m, nc, m, 1.f, strided(c.QL + (int64_t)slot * m * m, m, 0), strided(x, nc, 0),
+                            0.f, strided_mut(out, nc, 0), 1, s));
+    x = out;
+  }
+  if (c.right) {
+    SOAP_CUDA(h, soap::gemm(false, true, m, nc, nc, 1.f, strided(x, nc, 0), strided(c.QR + (int64_t)slot * nc * nc, nc, 0),
+                            0.f, strided_mut(dstm, nc, 0), 1, s));
+  } else if (!c.left) {
+    SOAP_CUDA(h, cudaMemcpyAsync(dstm, x, bytes, cudaMemcpyDeviceToDevice, s));
+  }
+  return SOAP_OK;
+}
+
+int64_t soap_get_step(soap_handle h) { return h ? h->t : -1; }
+
+soap_status_t soap_set_step(soap_handle h, int64_t t) {
+  if (!h || t < 0) return SOAP_ERR_INVALID_ARG;
+  h->t = t;
+  return SOAP_OK;
+}
+
+soap_status_t soap_status(soap_handle h, soap_stream_t stream_) {
+  if (!h) return SOAP_ERR_INVALID_ARG;
+  DeviceGuard g(h->device);
+  SOAP_CUDA(h, cudaStreamSynchronize((cudaStream_t)stream_));
+  int bits = 0;
+  SOAP_CUDA(h, cudaMemcpy(&bits, h->d_status, sizeof(int), cudaMemcpyDeviceToHost));
+  soap_status_t st = status_code(bits);
+  if (st != SOAP_OK) h->err = "device status word " + std::to_string(bits);
+  return st;
+}
+
+soap_status_t soap_clear_status(soap_handle h, soap_stream_t stream_) {
+  if (!h) return SOAP_ERR_INVALID_ARG;
+  DeviceGuard g(h->device);
+  SOAP_CUDA(h, cudaMemsetAsync(h->d_status, 0, sizeof(int), (cudaStream_t)stream_));
+  h->status_pending = false;
+  *h->h_status = 0;
+  return SOAP_OK;
+}
+
+const char* soap_last_error(soap_handle h) { return h ? h->err.c_str() : "null handle"; }
+
+void soap_destroy(soap_handle h) {
+  if (!h) return;
+  DeviceGuard g(h->device);
+  cudaDeviceSynchronize();
+  free_all(h);
+  delete h;
+}
+
+soap_status_t soap_profile_begin(soap_handle h, int64_t max_launches) {
+  if (!h || max_launches < 1 || max_launches > (int64_t(1) << 22)) return SOAP_ERR_INVALID_ARG;
+  DeviceGuard g(h->device);
+  soap::Profiler& p = h->prof;
+  while ((int64_t)p.events.size() < 2 * max_launches) {
+    cudaEvent_t ev;
+    SOAP_CUDA(h, cudaEventCreate(&ev));
+    p.events.push_back(ev);
+  }
+  p.capacity = (size_t)max_launches;
+  p.recs.clear();
+  p.overflow = false;
+  soap::t_profiler = &p;
+  return SOAP_OK;
+}
+
+soap_status_t soap_profile_end(soap_handle h, soap_stream_t stream, soap_kernel_stats* out, int32_t* overflow) {
+  if (!h || !out) return SOAP_ERR_INVALID_ARG;
+  DeviceGuard g(h->device);
+  if (soap::t_profiler == &h->prof) soap::t_profiler = nullptr;
+  SOAP_CUDA(h, cudaStreamSynchronize((cudaStream_t)stream));
+  SOAP_CUDA(h, cudaDeviceSynchronize());
+  for (int f = 0; f < soap::kNumFamilies; ++f) out[f] = soap_kernel_stats{f, 0, 0.0, 0.0, 0.0};
+  const soap::Profiler& p = h->prof;
+  for (size_t i = 0; i < p.recs.size(); ++i) {
+    float ms = 0.f;
+    SOAP_CUDA(h, cudaEventElapsedTime(&ms, p.events[2 * i], p.events[2 * i + 1]));
+    soap_kernel_stats& o = out[p.recs[i].family];
+    o.launches += 1;
+    o.ms += ms;
+    o.flops += p.recs[i].flops;
+    o.bytes += p.recs[i].bytes;
+  }
+  if (overflow) *overflow = p.overflow ? 1 : 0;
+  h->prof.recs.clear();
+  return SOAP_OK;
+}
+
+size_t soap_qr_workspace_bytes(int32_t n, int32_t batch) {
+  if (n <= 0 || batch <= 0) return 0;
+  return soap::qr_workspace_bytes(n, batch) + 256;
+}
+
+soap_status_t soap_qr(int32_t n, int32_t batch, const float* P, float* Q, uint8_t* skip, float tol, void* workspace,
+                      size_t workspace_bytes, soap_stream_t stream) {
+  if (n <= 0 || n > 8192 || batch <= 0 || batch > 65535 || !P || !Q || !skip || !workspace || !(tol >= 0.f))
+    return SOAP_ERR_INVALID_ARG;
+  if (!aligned16(P) || !aligned16(Q) || (reinterpret_cast<uintptr_t>(workspace) & 255))
+    return SOAP_ERR_INVALID_ARG;
+  if (workspace_bytes < soap_qr_workspace_bytes(n, batch)) return SOAP_ERR_INVALID_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  // the status word lives in the last 256 bytes of the caller's workspace
+  const size_t qb = soap::qr_workspace_bytes(n, batch);
+  int* status = reinterpret_cast<int*>(static_cast<char*>(workspace) + qb);
+  if (cudaMemsetAsync(status, 0, sizeof(int), s) != cudaSuccess) return SOAP_ERR_CUDA;
+  cudaError_t e = soap::qr_q(n, batch, P, Q, skip, tol, workspace, qb, status, s);
+  return e == cudaSuccess ? SOAP_OK : SOAP_ERR_CUDA;
+}
+
+soap_status_t soap_gemm(int32_t trans_a, int32_t trans_b, int32_t M, int32_t N, int32_t K, float alpha,
+                        const float* A, int64_t lda, int64_t stride_a, const float* B, int64_t ldb, int64_t stride_b,
+                        float beta, float* C, int64_t ldc, int64_t stride_c, int32_t batch, soap_stream_t stream) {
+  if (M < 0 || N < 0 || K < 0 || batch < 0 || batch > 65535) return SOAP_ERR_INVALID_ARG;
+  if (M == 0 || N == 0 || batch == 0) return SOAP_OK;
+  if (!C || (K > 0 && (!A || !B))) return SOAP_ERR_INVALID_ARG;
+  const int64_t a_rows = trans_a ? K : M, a_cols = trans_a ? M : K;
+  const int64_t b_rows = trans_b ? N : K, b_cols = trans_b ? K : N;
+  if ((K > 0 && (lda < a_cols || ldb < b_cols)) || ldc < N) return SOAP_ERR_INVALID_ARG;
+  (void)a_rows;
+  (void)b_rows;
+  cudaError_t e = soap::gemm(trans_a != 0, trans_b != 0, M, N, K, alpha, soap::strided(A, lda, stride_a),
+                             soap::strided(B, ldb, stride_b), beta, soap::strided_mut(C, ldc, stride_c), batch,
+                             (cudaStream_t)stream);
+  return e == cudaSuccess ? SOAP_OK : SOAP_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,72 @@
+// Internal declarations shared by the libsoap translation units (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/soap.h"
+
+namespace soap {
+
+// Sticky device status bits (combined with atomicOr by the kernels).
+enum : int {
+  kStatusNonFinite = 1,
+  kStatusQrBreakdown = 2,
+  kStatusTimeout = 4,
+};
+
+// A batched matrix operand: matrix b starts at (ptrs ? ptrs[b] : base + b * stride) + offset.
+struct Operand {
+  const float* base;
+  const float* const* ptrs;  // device array of per-matrix pointers, or nullptr
+  int64_t stride;
+  int64_t offset;
+  int64_t ld;
+};
+
+struct MutOperand {
+  float* base;
+  float* const* ptrs;
+  int64_t stride;
+  int64_t offset;
+  int64_t ld;
+};
+
+inline Operand strided(const float* base, int64_t ld, int64_t stride, int64_t offset = 0) {
+  return Operand{base, nullptr, stride, offset, ld};
+}
+inline MutOperand strided_mut(float* base, int64_t ld, int64_t stride, int64_t offset = 0) {
+  return MutOperand{base, nullptr, stride, offset, ld};
+}
+
+// C_b = alpha * op(A_b) op(B_b) + beta * C_b for b < batch (fp32-accurate).
+// Returns a cudaError_t from the launch.
+cudaError_t gemm(bool trans_a, bool trans_b, int M, int N, int K, float alpha, Operand A,
+                 Operand B, float beta, MutOperand C, int batch, cudaStream_t stream);
+
+// CUDA-core fp32 engine (exact fp32 FMAs); any shape.
+cudaError_t gemm_simt(bool trans_a, bool trans_b, int M, int N, int K, float alpha, Operand A,
+                      Operand B, float beta, MutOperand C, int batch, cudaStream_t stream);
+
+// Householder QR (explicit Q) of `batch` contiguous n x n matrices.
+size_t qr_workspace_bytes(int n, int batch);
+cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, float tol,
+                 void* workspace, size_t workspace_bytes, int* status, cudaStream_t stream);
+
+// Elementwise kernels of the step.
+// M_hat <- b1 M_hat + (1-b1) G and Gc <- G for each matrix of a class.
+cudaError_t momentum_and_copy(const float* const* grads, float* Gc, float* Mhat, int64_t elems,
+                              int batch, float beta1, int* status, cudaStream_t stream);
+// v <- b2 v + (1-b2) G'^2; N = m' / (sqrt(v) + eps) (bias-corrected if t > 0 given),
+// written over Gp; guard rows/cols zeroed.
+cudaError_t adam_in_basis(float* Gp, const float* Mp, float* V, int rows, int cols, int batch,
+                          float beta1, float beta2, float eps, float bc1, float bc2,
+                          const uint8_t* skipL, const uint8_t* skipR, int* status,
+                          cudaStream_t stream);
+// W <- (1 - lr*wd) W - lr * D (both sides identity).
+cudaError_t weight_update(float* const* params, const float* D, int64_t elems, int batch,
+                          float lr, float wd, cudaStream_t stream);
+// Sets `batch` n x n matrices to the identity.
+cudaError_t set_identity(float* Q, int n, int batch, cudaStream_t stream);
+
+}  // namespace soap

@@ -1,0 +1,288 @@
+"""ctypes binding of libsoap (include/soap.h): argument marshalling only.
+
+Every step of the optimizer runs in the library's CUDA kernels; this module only
+turns torch tensors into pointers and streams. It never computes anything itself,
+and it raises at import if the compiled library is missing (there is no fallback).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import platform
+from dataclasses import dataclass
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", platform.machine(), "libsoap.so")
+
+SOAP_OK = 0
+STATUS_NAMES = {0: "SOAP_OK", 1: "SOAP_ERR_INVALID_ARG", 2: "SOAP_ERR_CUDA", 3: "SOAP_ERR_OOM",
+                4: "SOAP_ERR_NONFINITE", 5: "SOAP_ERR_QR_BREAKDOWN", 6: "SOAP_ERR_TIMEOUT"}
+STATE_M, STATE_V, STATE_L, STATE_QL, STATE_R, STATE_QR, STATE_MHAT, STATE_SKIP_L, STATE_SKIP_R = range(9)
+
+# every symbol include/soap.h declares
+EXPORTS = ("soap_default_hparams", "soap_create", "soap_step", "soap_set_lr", "soap_state_bytes",
+           "soap_state_get", "soap_state_set", "soap_get_step", "soap_set_step", "soap_status",
+           "soap_clear_status", "soap_last_error", "soap_destroy", "soap_qr_workspace_bytes",
+           "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end")
+KERNEL_FAMILIES = ("gemm_simt", "gemm_tc", "qr_panel", "elementwise", "other")
+
+
+class soap_shape(ctypes.Structure):
+    _fields_ = [("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
+                ("precond_left", ctypes.c_int32), ("precond_right", ctypes.c_int32)]
+
+
+class soap_hparams(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+                ("factor_beta", ctypes.c_float), ("eps", ctypes.c_float),
+                ("weight_decay", ctypes.c_float), ("eig_every", ctypes.c_int32),
+                ("bias_correction", ctypes.c_int32), ("qr_tol", ctypes.c_float),
+                ("guard", ctypes.c_int32)]
+
+
+class soap_kernel_stats(ctypes.Structure):
+    _fields_ = [("family", ctypes.c_int32), ("launches", ctypes.c_int64), ("ms", ctypes.c_double),
+                ("flops", ctypes.c_double), ("bytes", ctypes.c_double)]
+
+
+class SoapError(RuntimeError):
+    def __init__(self, code, msg=""):
+        super().__init__(f"{STATUS_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH):
+    """Loads libsoap.so; raises if it has not been built (no fallback path exists)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise ImportError(f"libsoap.so not built ({path}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(path)
+    P, I32, I64, F, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+    sig = {
+        "soap_default_hparams": (None, [ctypes.POINTER(soap_hparams)]),
+        "soap_create": (I32, [ctypes.POINTER(soap_shape), I32, ctypes.POINTER(soap_hparams), I32, ctypes.POINTER(P)]),
+        "soap_step": (I32, [P, P, P, P]),
+        "soap_set_lr": (I32, [P, F, F]),
+        "soap_state_bytes": (SZ, [P, I32, I32]),
+        "soap_state_get": (I32, [P, I32, I32, P, P]),
+        "soap_state_set": (I32, [P, I32, I32, P, P]),
+        "soap_get_step": (I64, [P]),
+        "soap_set_step": (I32, [P, I64]),
+        "soap_status": (I32, [P, P]),
+        "soap_clear_status": (I32, [P, P]),
+        "soap_last_error": (ctypes.c_char_p, [P]),
+        "soap_destroy": (None, [P]),
+        "soap_qr_workspace_bytes": (SZ, [I32, I32]),
+        "soap_qr": (I32, [I32, I32, P, P, P, F, P, SZ, P]),
+        "soap_profile_begin": (I32, [P, I64]),
+        "soap_profile_end": (I32, [P, P, ctypes.POINTER(soap_kernel_stats), ctypes.POINTER(I32)]),
+        "soap_gemm": (I32, [I32, I32, I32, I32, I32, F, P, I64, I64, P, I64, I64, F, P, I64, I64, I32, P]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _stream(stream=None):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(code, h=None):
+    if code != SOAP_OK:
+        msg = load_library().soap_last_error(h).decode() if h else ""
+        raise SoapError(code, msg)
+
+
+def default_hparams(**overrides) -> soap_hparams:
+    hp = soap_hparams()
+    load_library().soap_default_hparams(ctypes.byref(hp))
+    for k, v in overrides.items():
+        setattr(hp, k, v)
+    return hp
+
+
+@dataclass
+class Shape:
+    rows: int
+    cols: int
+    left: bool = True
+    right: bool = True
+
+
+class SoapOptimizer:
+    """One libsoap handle: soap_create / soap_step / soap_state_get / soap_state_set."""
+
+    def __init__(self, shapes, hparams: soap_hparams | None = None, device: int | None = None):
+        lib = load_library()
+        self.shapes = [Shape(*s) if not isinstance(s, Shape) else s for s in shapes]
+        arr = (soap_shape * len(self.shapes))(*[soap_shape(s.rows, s.cols, int(s.left), int(s.right))
+                                               for s in self.shapes])
+        self.hparams = hparams if hparams is not None else default_hparams()
+        self.device = torch.cuda.current_device() if device is None else device
+        h = ctypes.c_void_p()
+        _check(lib.soap_create(arr, len(self.shapes), ctypes.byref(self.hparams), self.device, ctypes.byref(h)))
+        self._h = h
+        n = len(self.shapes)
+        self._pp = (ctypes.c_void_p * n)()
+        self._gp = (ctypes.c_void_p * n)()
+
+    def _handle(self):
+        if self._h is None:
+            raise SoapError(1, "handle destroyed")
+        return self._h
+
+    def step(self, params, grads, stream=None):
+        """soap_step on device tensors (fp32, contiguous); params are updated in place."""
+        n = len(self.shapes)
+        if len(params) != n or len(grads) != n:
+            raise ValueError("need one param and one grad per matrix")
+        for i, (p, g, s) in enumerate(zip(params, grads, self.shapes)):
+            if p.dtype != torch.float32 or g.dtype != torch.float32 or not p.is_cuda or not g.is_cuda:
+                raise TypeError(f"matrix {i}: params/grads must be fp32 CUDA tensors")
+            if tuple(p.shape) != (s.rows, s.cols) or tuple(g.shape) != (s.rows, s.cols):
+                raise ValueError(f"matrix {i}: expected {(s.rows, s.cols)}")
+            if not p.is_contiguous() or not g.is_contiguous():
+                raise ValueError(f"matrix {i}: tensors must be contiguous")
+            self._pp[i] = p.data_ptr()
+            self._gp[i] = g.data_ptr()
+        _check(load_library().soap_step(self._handle(), self._pp, self._gp, _stream(stream)), self._h)
+
+    def set_lr(self, lr: float, weight_decay: float):
+        _check(load_library().soap_set_lr(self._handle(), lr, weight_decay), self._h)
+
+    def state_bytes(self, idx: int, which: int) -> int:
+        return load_library().soap_state_bytes(self._handle(), idx, which)
+
+    def state_get(self, idx: int, which: int, stream=None) -> torch.Tensor:
+        """Returns a new device tensor holding one piece of matrix idx's state."""
+        s = self.shapes[idx]
+        shape = {STATE_M: (s.rows, s.cols), STATE_V: (s.rows, s.cols), STATE_MHAT: (s.rows, s.cols),
+                 STATE_L: (s.rows, s.rows), STATE_QL: (s.rows, s.rows), STATE_R: (s.cols, s.cols),
+                 STATE_QR: (s.cols, s.cols), STATE_SKIP_L: (s.rows,), STATE_SKIP_R: (s.cols,)}[which]
+        dtype = torch.uint8 if which in (STATE_SKIP_L, STATE_SKIP_R) else torch.float32
+        out = torch.empty(shape, dtype=dtype, device=f"cuda:{self.device}")
+        _check(load_library().soap_state_get(self._handle(), idx, which, ctypes.c_void_p(out.data_ptr()),
+                                             _stream(stream)), self._h)
+        return out
+
+    def state_set(self, idx: int, which: int, src: torch.Tensor, stream=None):
+        if src.numel() * src.element_size() != self.state_bytes(idx, which) or not src.is_contiguous():
+            raise ValueError("state_set: wrong size or non-contiguous source")
+        _check(load_library().soap_state_set(self._handle(), idx, which, ctypes.c_void_p(src.data_ptr()),
+                                             _stream(stream)), self._h)
+
+    @property
+    def t(self) -> int:
+        return load_library().soap_get_step(self._handle())
+
+    @t.setter
+    def t(self, value: int):
+        _check(load_library().soap_set_step(self._handle(), value), self._h)
+
+    def status(self, stream=None) -> int:
+        """Synchronises the stream and returns the sticky device status code."""
+        return load_library().soap_status(self._handle(), _stream(stream))
+
+    def clear_status(self, stream=None):
+        _check(load_library().soap_clear_status(self._handle(), _stream(stream)), self._h)
+
+    def profile_begin(self, max_launches: int = 1 << 16):
+        """Time every kernel launch of the following calls with CUDA events."""
+        _check(load_library().soap_profile_begin(self._handle(), max_launches), self._h)
+
+    def profile_end(self, stream=None) -> dict:
+        """Synchronise and return {family: {launches, ms, flops, bytes}} plus an overflow flag."""
+        out = (soap_kernel_stats * len(KERNEL_FAMILIES))()
+        ov = ctypes.c_int32(0)
+        _check(load_library().soap_profile_end(self._handle(), _stream(stream), out, ctypes.byref(ov)), self._h)
+        res = {KERNEL_FAMILIES[o.family]: dict(launches=o.launches, ms=o.ms, flops=o.flops, bytes=o.bytes)
+               for o in out}
+        res["overflow"] = bool(ov.value)
+        return res
+
+    def last_error(self) -> str:
+        return load_library().soap_last_error(self._handle()).decode()
+
+    def destroy(self):
+        if self._h is not None:
+            load_library().soap_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+# ---- module-level names matching the C ABI ------------------------------------------
+
+def soap_create(shapes, hparams=None, device=None) -> SoapOptimizer:
+    return SoapOptimizer(shapes, hparams, device)
+
+
+def soap_step(opt: SoapOptimizer, params, grads, stream=None):
+    opt.step(params, grads, stream)
+
+
+def soap_state_get(opt: SoapOptimizer, idx, which, stream=None):
+    return opt.state_get(idx, which, stream)
+
+
+def soap_state_set(opt: SoapOptimizer, idx, which, src, stream=None):
+    opt.state_set(idx, which, src, stream)
+
+
+def soap_qr(P: torch.Tensor, tol: float = 0.0, stream=None):
+    """Batched QR refresh on device: P [batch, n, n] fp32 -> (Q, skip[batch, n] uint8)."""
+    lib = load_library()
+    if P.dim() == 2:
+        P = P.unsqueeze(0)
+    if P.dtype != torch.float32 or not P.is_cuda or P.shape[1] != P.shape[2]:
+        raise TypeError("soap_qr: P must be a [batch, n, n] fp32 CUDA tensor")
+    P = P.contiguous()
+    batch, n = P.shape[0], P.shape[1]
+    Q = torch.empty_like(P)
+    skip = torch.empty(batch, n, dtype=torch.uint8, device=P.device)
+    ws_bytes = lib.soap_qr_workspace_bytes(n, batch)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=P.device)
+    _check(lib.soap_qr(n, batch, ctypes.c_void_p(P.data_ptr()), ctypes.c_void_p(Q.data_ptr()),
+                       ctypes.c_void_p(skip.data_ptr()), float(tol), ctypes.c_void_p(ws.data_ptr()), ws_bytes,
+                       _stream(stream)))
+    return Q, skip
+
+
+def soap_gemm(A: torch.Tensor, B: torch.Tensor, trans_a=False, trans_b=False, alpha=1.0, beta=0.0,
+              C: torch.Tensor | None = None, stream=None):
+    """C = alpha op(A) op(B) + beta C on [batch, r, c] (or 2-D) fp32 CUDA tensors."""
+    lib = load_library()
+    squeeze = A.dim() == 2
+    A3 = (A.unsqueeze(0) if A.dim() == 2 else A).contiguous()
+    B3 = (B.unsqueeze(0) if B.dim() == 2 else B).contiguous()
+    batch = A3.shape[0]
+    M = A3.shape[2] if trans_a else A3.shape[1]
+    K = A3.shape[1] if trans_a else A3.shape[2]
+    N = B3.shape[1] if trans_b else B3.shape[2]
+    if C is None:
+        C3 = torch.zeros(batch, M, N, dtype=torch.float32, device=A.device)
+    else:
+        C3 = C.unsqueeze(0) if C.dim() == 2 else C
+        if not C3.is_contiguous():
+            raise ValueError("C must be contiguous")
+    _check(lib.soap_gemm(int(trans_a), int(trans_b), M, N, K, float(alpha),
+                         ctypes.c_void_p(A3.data_ptr()), A3.shape[2], A3.shape[1] * A3.shape[2],
+                         ctypes.c_void_p(B3.data_ptr()), B3.shape[2], B3.shape[1] * B3.shape[2], float(beta),
+                         ctypes.c_void_p(C3.data_ptr()), N, M * N, batch, _stream(stream)))
+    return C3[0] if squeeze else C3
