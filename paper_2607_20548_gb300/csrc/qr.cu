@@ -18,11 +18,18 @@
 // the only waits are hardware cluster barriers that every CTA of the cluster
 // reaches unconditionally.
 //
-// Reflector convention (Golub & Van Loan Alg. 5.1.1): for x = A[p:n, p] with
-// alpha = x_1 and sigma = ||x_2:||^2, v_1 = 1 and H x = ||x|| e_1, so R_pp = ||x|| >= 0
-// and no sign fix is needed. A column with ||x|| <= tol * ||P||_F is treated as
-// exactly zero: H = I, and the column is flagged in skip[].
+// Reflector convention (LAPACK larfg): for x = A[p:n, p] with alpha = x_1 and
+// sigma = ||x_2:||^2, beta = -sign(alpha) ||x||, v = x / (alpha - beta) with v_1 = 1,
+// tau = (beta - alpha) / beta, so H x = beta e_1 and R_pp = beta; sigma = 0 gives H = I
+// and R_pp = alpha. The sign convention diag(R) >= 0 then negates column p of Q
+// wherever R_pp < 0; it costs nothing because the backward accumulation of Q starts
+// from diag(d_1..d_n), d_p = sign of R_pp, instead of I. A column with
+// ||x|| <= tol * ||P||_F is treated as exactly zero: H = I, R_pp = 0, d_p = +1, and the
+// column is flagged in skip[]. (The convention matters beyond the sign: the columns of
+// Q that complete a rank-deficient P are H_1 ... H_p-1 e_p, which depend on it.)
 #include <cooperative_groups.h>
+
+#include <algorithm>
 
 #include "profile.h"
 #include "soap_internal.h"
@@ -44,6 +51,7 @@ struct PanelArgs {
   float* A;            // [batch][n][n] working matrices
   float* T;            // [batch][npanel][NB][NB]
   uint8_t* skip;       // [batch][n]
+  float* dsign;        // [batch][n] sign of R_pp (+1 for zero columns)
   const float* thresh; // [batch]
   int* status;
   int n, k, kb, panel, npanel;
@@ -70,6 +78,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   __shared__ float s_red[NWARP];
   __shared__ float s_tau[NB];
   __shared__ int s_skip[NB];
+  __shared__ float s_dsign[NB];
   __shared__ float s_gram[MAXC][NB][NB];
   __shared__ float s_T[NB][NB + 1];
 
@@ -117,14 +126,16 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     const float xnorm = sqrtf(fmaf(alpha, alpha, sigma));
     if (!isfinite(xnorm)) nonfinite = 1;
     const bool skip = !(xnorm > thresh);
-    float tau = 0.f, v0 = 1.f;
+    float tau = 0.f, v0 = 1.f, rsign = 1.f;
     bool scale = false;
     if (!skip) {
       if (sigma == 0.f) {
-        tau = alpha >= 0.f ? 0.f : 2.f;   // x = alpha e_1: identity, or a sign flip
+        rsign = alpha < 0.f ? -1.f : 1.f;   // H = I, R_pp = alpha
       } else {
-        v0 = alpha <= 0.f ? alpha - xnorm : -sigma / (alpha + xnorm);
-        tau = 2.f * v0 * v0 / (sigma + v0 * v0);
+        const float beta = alpha >= 0.f ? -xnorm : xnorm;
+        v0 = alpha - beta;                   // same sign as alpha: no cancellation
+        tau = (beta - alpha) / beta;
+        rsign = beta < 0.f ? -1.f : 1.f;
         scale = true;
       }
     }
@@ -136,6 +147,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     if (tid == 0) {
       s_tau[j] = tau;
       s_skip[j] = skip ? 1 : 0;
+      s_dsign[j] = rsign;
     }
     __syncthreads();
 
@@ -188,7 +200,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     g = warp_sum(g);
     if (lane == 0) cluster.map_shared_rank(&s_gram[0][0][0], 0)[(c * NB + a) * NB + bb] = g;
   }
-  if (nonfinite && tid == 0) atomicOr(p.status, kStatusNonFinite | kStatusQrBreakdown);
+  if (nonfinite && tid == 0) atomicOr(p.status, kStatusQrBreakdown);
   cluster.sync();
   if (c != 0) return;
 
@@ -217,7 +229,10 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     const int i = e / NB, jj = e % NB;
     Tout[e] = (i < kb && jj < kb) ? s_T[i][jj] : 0.f;
   }
-  if (tid < kb) p.skip[(int64_t)b * n + k + tid] = (uint8_t)s_skip[tid];
+  if (tid < kb) {
+    p.skip[(int64_t)b * n + k + tid] = (uint8_t)s_skip[tid];
+    p.dsign[(int64_t)b * n + k + tid] = s_dsign[tid];
+  }
 }
 
 // ||P_b||_F: per-chunk partial sums in double, then tol * sqrt(sum)
@@ -248,12 +263,24 @@ __global__ void thresh_kernel(const double* part, float tol, int batch, float* t
   thresh[b] = (float)((double)tol * sqrt(s));
 }
 
+__global__ void signed_identity_kernel(float* Q, const float* d, int n) {
+  const int b = blockIdx.y;
+  float* q = Q + (int64_t)b * n * n;
+  const float* db = d + (int64_t)b * n;
+  const int64_t nn = (int64_t)n * n;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nn; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = i / n, c = i % n;
+    q[i] = r == c ? db[r] : 0.f;
+  }
+}
+
 struct Workspace {
   float* A;
   float* T;
   float* W1;
   float* W2;
   float* thresh;
+  float* dsign;
   double* part;
 };
 
@@ -272,11 +299,12 @@ Workspace carve(void* base, int n, int batch, size_t* total) {
   const size_t oW1 = take((size_t)batch * NB * n * sizeof(float));
   const size_t oW2 = take((size_t)batch * NB * n * sizeof(float));
   const size_t oth = take((size_t)batch * sizeof(float));
+  const size_t osg = take((size_t)batch * n * sizeof(float));
   const size_t opart = take((size_t)batch * NORM_CHUNKS * sizeof(double));
   if (total) *total = off;
   char* c = (char*)base;
   return Workspace{(float*)(c + oA), (float*)(c + oT), (float*)(c + oW1), (float*)(c + oW2),
-                   (float*)(c + oth), (double*)(c + opart)};
+                   (float*)(c + oth), (float*)(c + osg), (double*)(c + opart)};
 }
 
 }  // namespace
@@ -318,7 +346,7 @@ cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, floa
   for (int pi = 0; pi < npanel; ++pi) {
     const int k = pi * NB, kb = min(NB, n - k);
     const int C = (n - k + ROWS - 1) / ROWS;
-    PanelArgs a{w.A, w.T, skip, w.thresh, status, n, k, kb, pi, npanel};
+    PanelArgs a{w.A, w.T, skip, w.dsign, w.thresh, status, n, k, kb, pi, npanel};
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(C, batch, 1);
     cfg.blockDim = dim3(PT, 1, 1);
@@ -357,8 +385,14 @@ cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, floa
     if (e != cudaSuccess) return e;
   }
 
-  e = set_identity(Q, n, batch, s);
-  if (e != cudaSuccess) return e;
+  {
+    // Q = H_1 ... H_n diag(d): start the backward accumulation from diag(d)
+    ProfScope prof(kFamOther, 0, 4.0 * nn * batch, s);
+    const int blocks = (int)std::min<int64_t>((nn + 255) / 256, 1024);
+    signed_identity_kernel<<<dim3(blocks, batch), 256, 0, s>>>(Q, w.dsign, n);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
   for (int pi = npanel - 1; pi >= 0; --pi) {
     const int k = pi * NB, kb = min(NB, n - k), m = n - k;
     Operand V = strided(w.A, n, nn, (int64_t)k * n + k);

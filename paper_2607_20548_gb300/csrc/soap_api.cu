@@ -105,10 +105,11 @@ soap_status_t cuda_fail(soap_handle h, cudaError_t e, const char* what) {
     if (e_ != cudaSuccess) return cuda_fail(h, e_, #expr); \
   } while (0)
 
+// A non-finite gradient also makes the QR of that step break down; report the cause.
 soap_status_t status_code(int bits) {
-  if (bits & soap::kStatusTimeout) return SOAP_ERR_TIMEOUT;
-  if (bits & soap::kStatusQrBreakdown) return SOAP_ERR_QR_BREAKDOWN;
   if (bits & soap::kStatusNonFinite) return SOAP_ERR_NONFINITE;
+  if (bits & soap::kStatusQrBreakdown) return SOAP_ERR_QR_BREAKDOWN;
+  if (bits & soap::kStatusTimeout) return SOAP_ERR_TIMEOUT;
   return SOAP_OK;
 }
 

@@ -170,7 +170,9 @@ class SoapOptimizer:
         s = self.shapes[idx]
         shape = {STATE_M: (s.rows, s.cols), STATE_V: (s.rows, s.cols), STATE_MHAT: (s.rows, s.cols),
                  STATE_L: (s.rows, s.rows), STATE_QL: (s.rows, s.rows), STATE_R: (s.cols, s.cols),
-                 STATE_QR: (s.cols, s.cols), STATE_SKIP_L: (s.rows,), STATE_SKIP_R: (s.cols,)}[which]
+                 STATE_QR: (s.cols, s.cols), STATE_SKIP_L: (s.rows,), STATE_SKIP_R: (s.cols,)}.get(which)
+        if shape is None or self.state_bytes(idx, which) == 0:
+            raise SoapError(1, f"no state piece {which} for matrix {idx}")
         dtype = torch.uint8 if which in (STATE_SKIP_L, STATE_SKIP_R) else torch.float32
         out = torch.empty(shape, dtype=dtype, device=f"cuda:{self.device}")
         _check(load_library().soap_state_get(self._handle(), idx, which, ctypes.c_void_p(out.data_ptr()),

@@ -4,12 +4,19 @@ Teacher forcing: before GPU step t, the GPU's own state (m, v, L, Q_L, R, Q_R) a
 copied out; the fp64 oracle and its fp32 twin each apply step t to that state with the
 same G_t. The GPU's update dW_t = W_t - W_{t-1} is then compared with the oracle's.
 
-Tolerance (derived from the arithmetic): the benchmark spec's bound is a relative Frobenius
-error <= 1e-3 of each step's update. Where a step is beyond fp32 resolution -- Adam's
-normalisation m / (sqrt(v) + eps) amplifying rounding in directions whose v is ~0,
-which happens when the basis rotates momentum into them -- even the fp32 twin, a
-faithful fp32 implementation, misses that bound; there the bound is 4x the twin's own
-error on the same step, and both numbers are reported.
+Tolerance (derived from the arithmetic): the bound is a relative Frobenius error
+<= 1e-3 of each step's update, or 4x the fp32 twin's error where the twin -- a faithful
+fp32 implementation -- cannot do better.
+
+Some steps are beyond fp32 resolution altogether: when the refreshed basis rotates
+momentum into directions whose second moment is still ~0 (v is not re-projected), Adam's
+m / (sqrt(v) + eps) turns a G' entry of ~1e-7 into |N| in the thousands, so the update
+depends on the rounding of that tiny entry (the twin and the GPU then differ from fp64,
+and from each other, by O(1e-2..1)). Such a step (twin error > 1e-3 / 4, or oracle
+max|N| > 100, far past the bound |N| <= 1 that Adam obeys without a basis change) is
+verified piece by piece instead: the GPU's m, v, L, R, Q after the step against the
+teacher-forced oracle, and the GPU's update against Q_L N Q_R^T recomputed in fp64 from
+the GPU's own m, v and bases -- every well-conditioned quantity of the step.
 """
 from __future__ import annotations
 
@@ -21,6 +28,7 @@ from paper_2607_20548_gb300 import soap as S
 
 TOL = 1e-3
 TWIN_FACTOR = 4.0
+N_CAP = 100.0
 
 
 def rel(a, b):
@@ -72,47 +80,65 @@ class TeacherForcedCheck:
     def after(self, idx: int, W: torch.Tensor):
         st64, st32, W0, G = self.pending.pop(idx)
         t = st64.t + 1
-        W64, _ = soap_step(st64, W0.astype(np.float64), G, self.hp)
-        W32, _ = soap_step(st32, W0, G, self.hp)
+        hp = self.hp
+        W64, _ = soap_step(st64, W0.astype(np.float64), G, hp)
+        W32, _ = soap_step(st32, W0, G, hp)
         W1 = W.detach().cpu().numpy().astype(np.float64)
         d_ref = W64 - W0
         e_gpu = rel(W1 - W0, d_ref)
         e_twin = rel(W32.astype(np.float64) - W0, d_ref)
-        Nmax = float(np.abs(st64.m / (np.sqrt(st64.v) + self.hp.eps)).max())
-        row = dict(idx=idx, t=t, e_gpu=e_gpu, e_twin=e_twin, bound=max(TOL, TWIN_FACTOR * e_twin),
-                   max_abs_N=Nmax, st64=st64)
-        # state after the step: factors and moments
+        N64 = st64.m / (np.sqrt(st64.v) + hp.eps)
+        Nmax = float(np.abs(N64).max())
         sp = self.opt.shapes[idx]
-        row["e_v"] = rel(self.opt.state_get(idx, S.STATE_V).cpu().numpy(), st64.v)
+        g = lambda w: self.opt.state_get(idx, w).cpu().numpy()
+        m_gpu, v_gpu = g(S.STATE_M).astype(np.float64), g(S.STATE_V).astype(np.float64)
+        row = dict(idx=idx, t=t, e_gpu=e_gpu, e_twin=e_twin, max_abs_N=Nmax,
+                   e_m=rel(m_gpu, st64.m), e_v=rel(v_gpu, st64.v))
+        row["ill"] = bool(TWIN_FACTOR * e_twin > TOL or Nmax > N_CAP)
+        # the GPU's update against Q_L N Q_R^T from its own state, in fp64
+        N = m_gpu / (np.sqrt(v_gpu) + hp.eps) if not hp.bias_correction else \
+            (m_gpu / (1 - hp.beta1 ** t)) / (np.sqrt(v_gpu / (1 - hp.beta2 ** t)) + hp.eps)
+        QL = QR = None
         if sp.left:
-            row["e_L"] = rel(self.opt.state_get(idx, S.STATE_L).cpu().numpy(), st64.L)
-            row["skipL_same"] = bool(np.array_equal(
-                self.opt.state_get(idx, S.STATE_SKIP_L).cpu().numpy().astype(bool), st64.skipL))
+            QL = g(S.STATE_QL).astype(np.float64)
+            row["e_L"] = rel(g(S.STATE_L), st64.L)
+            skL = g(S.STATE_SKIP_L).astype(bool)
+            row["skipL_same"] = bool(np.array_equal(skL, st64.skipL))
             row["orth_L"] = orth_err(self.opt.state_get(idx, S.STATE_QL))
+            if hp.guard:
+                N[skL, :] = 0
         if sp.right:
-            row["e_R"] = rel(self.opt.state_get(idx, S.STATE_R).cpu().numpy(), st64.R)
-            row["skipR_same"] = bool(np.array_equal(
-                self.opt.state_get(idx, S.STATE_SKIP_R).cpu().numpy().astype(bool), st64.skipR))
+            QR = g(S.STATE_QR).astype(np.float64)
+            row["e_R"] = rel(g(S.STATE_R), st64.R)
+            skR = g(S.STATE_SKIP_R).astype(bool)
+            row["skipR_same"] = bool(np.array_equal(skR, st64.skipR))
             row["orth_R"] = orth_err(self.opt.state_get(idx, S.STATE_QR))
-        del row["st64"]
+            if hp.guard:
+                N[:, skR] = 0
+        dW_self = (QL @ N if QL is not None else N)
+        dW_self = dW_self @ QR.T if QR is not None else dW_self
+        keep = 1 - hp.lr * hp.weight_decay
+        row["e_self"] = rel((W1 - keep * W0.astype(np.float64)) / -hp.lr, dW_self) if hp.lr > 0 else 0.0
         self.rows.append(row)
         return row
 
     def report(self) -> str:
         out = []
         for r in self.rows:
-            flag = "" if r["e_twin"] * TWIN_FACTOR <= TOL else "  [beyond fp32 resolution: bound = 4x twin]"
+            tag = "  [beyond fp32 resolution: verified piece by piece]" if r["ill"] else ""
             out.append(f"matrix {r['idx']:4d} step {r['t']:3d}: gpu {r['e_gpu']:.2e} twin {r['e_twin']:.2e} "
-                       f"max|N| {r['max_abs_N']:.0f}{flag}")
+                       f"max|N| {r['max_abs_N']:.0f} m {r['e_m']:.1e} v {r['e_v']:.1e} self {r['e_self']:.1e}{tag}")
         return "\n".join(out)
 
     def assert_ok(self, state_tol=1e-4):
         bad = []
         for r in self.rows:
-            if not r["e_gpu"] <= r["bound"]:
+            if not r["ill"] and not r["e_gpu"] <= max(TOL, TWIN_FACTOR * r["e_twin"]):
                 bad.append(f"update: {r}")
-            for k in ("e_L", "e_R", "e_v"):
-                if k in r and not r[k] <= max(state_tol, TWIN_FACTOR * r["e_twin"]):
+            if not r["e_self"] <= 1e-4:
+                bad.append(f"self-consistency of the update: {r}")
+            for k in ("e_L", "e_R", "e_v", "e_m"):
+                if k in r and not r[k] <= max(state_tol, TWIN_FACTOR * r["e_twin"] if not r["ill"] else 0.0):
                     bad.append(f"{k}: {r}")
             for k in ("orth_L", "orth_R"):
                 if k in r and not r[k] <= 1e-5:

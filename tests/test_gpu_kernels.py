@@ -75,26 +75,33 @@ def test_qr_matches_oracle(cuda, n, batch, kind):
         e_twin = _rel(Q32[:, keep].astype(np.float64), Q64[:, keep])
         assert e_gpu <= max(1e-5, 4 * e_twin), (e_gpu, e_twin)
         if s64.any():
-            # the completion columns are orthogonal to the range of P (exact arithmetic: P's columns)
-            Pn = P[b].astype(np.float64)
-            proj = np.abs(Q[b][:, s64].astype(np.float64).T @ Pn).max() / np.abs(Pn).max()
-            assert proj < 1e-3, proj
+            # the columns completing a rank-deficient P (H_1 ... H_k-1 e_k) follow the oracle too
+            c_gpu = _rel(Q[b][:, s64], Q64[:, s64])
+            c_twin = _rel(Q32[:, s64].astype(np.float64), Q64[:, s64])
+            assert c_gpu <= max(1e-5, 4 * c_twin), (c_gpu, c_twin)
 
 
 def test_qr_full_size_8192_properties(cuda):
-    """n = 8192 (the largest factor of the dense block and the 8192-wide layer): Q^T Q = I to 1e-5
-    and R = Q^T P upper triangular with diag(R) >= 0, checked in fp64 on the device."""
-    n = 8192
+    """n = 8192 (the largest factor of the dense block and the 8192-wide layer), on a PSD factor of
+    rank 2048 plus a tiny ridge, like L after a few steps: Q^T Q = I to 1e-5; R = Q^T P is upper
+    triangular with diag(R) >= 0 in every Householder column; a column treated as zero keeps its
+    unreflected sub-column, whose norm is at most tol * ||P||_F by the zero-column reading."""
+    n, tol = 8192, 1e-4
     g = torch.Generator(device=cuda).manual_seed(5)
     X = torch.randn(n, 2048, device=cuda, generator=g)
     P = (X @ X.T + 1e-3 * torch.eye(n, device=cuda)).unsqueeze(0)
-    Q, skip = S.soap_qr(P, 1e-4)
+    Q, skip = S.soap_qr(P, tol)
+    skip = skip[0].bool()
+    assert 0 < int(skip.sum()) < n
     Qd = Q[0].double()
     I = torch.eye(n, dtype=torch.float64, device=cuda)
     assert (Qd.T @ Qd - I).abs().max().item() <= 1e-5
+    del I
     R = Qd.T @ P[0].double()
-    scale = P[0].double().norm().item()
-    assert torch.tril(R, -1).abs().max().item() <= 1e-5 * scale
-    assert torch.diagonal(R).min().item() >= -1e-6 * scale
-    del P, Q, R, Qd, I, X
+    fro = P[0].double().norm().item()
+    low = torch.tril(R, -1)
+    assert low[:, ~skip].abs().max().item() <= 1e-5 * fro
+    assert low[:, skip].norm(dim=0).max().item() <= tol * fro * (1 + 1e-3)
+    assert torch.diagonal(R)[~skip].min().item() >= 0.0
+    del P, Q, R, Qd, X, low
     torch.cuda.empty_cache()
