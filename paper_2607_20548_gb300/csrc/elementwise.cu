@@ -65,7 +65,7 @@ __global__ void momentum_copy_kernel(const float* const* grads, float* Gc, float
 
 __global__ void adam_kernel(float* Gp, const float* Mp, float* V, int rows, int cols, float beta2,
                             float eps, float inv_bc1, float inv_sqrt_bc2, const uint8_t* skipL,
-                            const uint8_t* skipR, int* status) {
+                            const uint8_t* skipR, float* N_lo, int* status) {
   const int b = blockIdx.y;
   const int64_t elems = (int64_t)rows * cols;
   float* gp = Gp + (int64_t)b * elems;
@@ -85,6 +85,11 @@ __global__ void adam_kernel(float* Gp, const float* Mp, float* V, int rows, int 
     if ((sl && sl[i / cols]) || (sr && sr[i % cols])) nv = 0.f;
     bad |= !isfinite(nv);
     gp[i] = nv;
+    if (N_lo) {
+      uint32_t r;
+      asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(nv));
+      N_lo[(int64_t)b * elems + i] = nv - __uint_as_float(r);
+    }
   }
   if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(status, kStatusNonFinite);
 }
@@ -109,7 +114,121 @@ __global__ void identity_kernel(float* Q, int n) {
     q[i] = (i / n == i % n) ? 1.f : 0.f;
 }
 
+__device__ __forceinline__ float lo_part(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+  return x - __uint_as_float(r);
+}
+
+// One 32 x 32 tile of one matrix per block (32 x 8 threads). Reads G, updates M_hat and
+// writes the tensor-core operands: G (copy) and its lo part, G^T and its lo part, and
+// the lo part of the new M_hat.
+__global__ void momentum_split_kernel(const float* const* grads, float* Gc, float* Gc_lo, float* Gt, float* Gt_lo,
+                                      float* Mh, float* Mh_lo, int rows, int cols, float beta1, int* status) {
+  __shared__ float tile[32][33];
+  const int b = blockIdx.z;
+  const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
+  const int64_t mn = (int64_t)rows * cols;
+  const float* g = grads[b];
+  const float c1 = 1.f - beta1;
+  int bad = 0;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = r0 + i, c = c0 + threadIdx.x;
+    float x = 0.f;
+    if (r < rows && c < cols) {
+      const int64_t o = (int64_t)b * mn + (int64_t)r * cols + c;
+      x = g[(int64_t)r * cols + c];
+      bad |= !isfinite(x);
+      Gc[o] = x;
+      Gc_lo[o] = lo_part(x);
+      const float m = fmaf(beta1, Mh[o], c1 * x);
+      Mh[o] = m;
+      Mh_lo[o] = lo_part(m);
+    }
+    tile[i][threadIdx.x] = x;
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int c = c0 + i, r = r0 + threadIdx.x;  // G^T[c][r]
+    if (r < rows && c < cols) {
+      const float x = tile[threadIdx.x][i];
+      const int64_t o = (int64_t)b * mn + (int64_t)c * rows + r;
+      Gt[o] = x;
+      Gt_lo[o] = lo_part(x);
+    }
+  }
+  if (__syncthreads_or(bad) && threadIdx.x == 0 && threadIdx.y == 0) atomicOr(status, kStatusNonFinite);
+}
+
+// Q -> Q_lo, Q^T, Q^T_lo for `batch` n x n matrices (32 x 32 tiles, 32 x 8 threads).
+__global__ void basis_split_kernel(const float* Q, float* Q_lo, float* Qt, float* Qt_lo, int n) {
+  __shared__ float tile[32][33];
+  const int b = blockIdx.z;
+  const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
+  const int64_t nn = (int64_t)n * n;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = r0 + i, c = c0 + threadIdx.x;
+    float x = 0.f;
+    if (r < n && c < n) {
+      const int64_t o = (int64_t)b * nn + (int64_t)r * n + c;
+      x = Q[o];
+      Q_lo[o] = lo_part(x);
+    }
+    tile[i][threadIdx.x] = x;
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int c = c0 + i, r = r0 + threadIdx.x;
+    if (r < n && c < n) {
+      const float x = tile[threadIdx.x][i];
+      const int64_t o = (int64_t)b * nn + (int64_t)c * n + r;
+      Qt[o] = x;
+      Qt_lo[o] = lo_part(x);
+    }
+  }
+}
+
+__global__ void split_kernel(const float* x, float* hi, float* lo, int64_t n) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const float v = x[i];
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(v));
+    const float h = __uint_as_float(r);
+    if (hi) hi[i] = h;
+    lo[i] = v - h;
+  }
+}
+
 }  // namespace
+
+cudaError_t momentum_split(const float* const* grads, float* Gc, float* Gc_lo, float* Gt, float* Gt_lo, float* Mhat,
+                           float* Mhat_lo, int rows, int cols, int batch, float beta1, int* status, cudaStream_t s) {
+  if (rows <= 0 || cols <= 0 || batch <= 0) return cudaSuccess;
+  const double e = (double)rows * cols * batch;
+  ProfScope prof(kFamElementwise, 3.0 * e, 32.0 * e, s);
+  dim3 grid((cols + 31) / 32, (rows + 31) / 32, batch);
+  momentum_split_kernel<<<grid, dim3(32, 8), 0, s>>>(grads, Gc, Gc_lo, Gt, Gt_lo, Mhat, Mhat_lo, rows, cols, beta1,
+                                                     status);
+  return cudaGetLastError();
+}
+
+cudaError_t basis_split(const float* Q, float* Q_lo, float* Qt, float* Qt_lo, int n, int batch, cudaStream_t s) {
+  if (n <= 0 || batch <= 0) return cudaSuccess;
+  const double e = (double)n * n * batch;
+  ProfScope prof(kFamElementwise, 2.0 * e, 16.0 * e, s);
+  dim3 grid((n + 31) / 32, (n + 31) / 32, batch);
+  basis_split_kernel<<<grid, dim3(32, 8), 0, s>>>(Q, Q_lo, Qt, Qt_lo, n);
+  return cudaGetLastError();
+}
+
+cudaError_t split_tf32(const float* x, float* hi, float* lo, int64_t n, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  ProfScope prof(kFamElementwise, 2.0 * n, 12.0 * n, s);
+  const int64_t want = (n + kThreads - 1) / kThreads;
+  split_kernel<<<(int)(want < 4096 ? want : 4096), kThreads, 0, s>>>(x, hi, lo, n);
+  return cudaGetLastError();
+}
 
 cudaError_t momentum_and_copy(const float* const* grads, float* Gc, float* Mhat, int64_t elems,
                               int batch, float beta1, int* status, cudaStream_t s) {
@@ -122,13 +241,14 @@ cudaError_t momentum_and_copy(const float* const* grads, float* Gc, float* Mhat,
 
 cudaError_t adam_in_basis(float* Gp, const float* Mp, float* V, int rows, int cols, int batch,
                           float beta1, float beta2, float eps, float bc1, float bc2,
-                          const uint8_t* skipL, const uint8_t* skipR, int* status, cudaStream_t s) {
+                          const uint8_t* skipL, const uint8_t* skipR, float* N_lo, int* status,
+                          cudaStream_t s) {
   (void)beta1;
   const int64_t elems = (int64_t)rows * cols;
   if (elems <= 0 || batch <= 0) return cudaSuccess;
-  ProfScope prof(kFamElementwise, 8.0 * elems * batch, 16.0 * elems * batch, s);
+  ProfScope prof(kFamElementwise, 8.0 * elems * batch, (N_lo ? 24.0 : 20.0) * elems * batch, s);
   adam_kernel<<<dim3(blocks_for(elems, batch), batch), kThreads, 0, s>>>(
-      Gp, Mp, V, rows, cols, beta2, eps, 1.f / bc1, 1.f / sqrtf(bc2), skipL, skipR, status);
+      Gp, Mp, V, rows, cols, beta2, eps, 1.f / bc1, 1.f / sqrtf(bc2), skipL, skipR, N_lo, status);
   return cudaGetLastError();
 }
 

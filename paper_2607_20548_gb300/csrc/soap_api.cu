@@ -41,6 +41,20 @@ struct ClassState {
   uint8_t* skipL = nullptr;
   uint8_t* skipR = nullptr;
   size_t ptr_offset = 0;  // index of this class's params pointers in the pointer table
+  // tensor-core path (both sides preconditioned): operand copies and their lo parts
+  bool tc = false;
+  float* GM_lo = nullptr;  // lo parts of [G copy | M_hat]
+  float* Gt = nullptr;
+  float* Gt_lo = nullptr;
+  float* L_lo = nullptr;
+  float* R_lo = nullptr;
+  float* QL_lo = nullptr;
+  float* QLt = nullptr;
+  float* QLt_lo = nullptr;
+  float* QR_lo = nullptr;
+  float* QRt = nullptr;
+  float* QRt_lo = nullptr;
+  bool basis_dirty = true;  // Q^T and lo parts must be rebuilt from Q before use
 };
 
 struct DeviceGuard {
@@ -67,8 +81,13 @@ struct soap_s {
   std::vector<ClassState> classes;
   float* X1 = nullptr;
   float* X2 = nullptr;
-  float* Gp = nullptr;
-  float* Mp = nullptr;
+  float* Gp = nullptr;   // [G' | m'] for the tensor-core path: Gp .. Gp + 2 * ws_mat
+  float* Mp = nullptr;   // m' for the CUDA-core path (Gp + ws_mat)
+  float* YMt = nullptr;  // (G Q_R)^T and (M_hat Q_R)^T
+  float* YMt_lo = nullptr;
+  float* N_lo = nullptr;
+  float* Zt = nullptr;   // (N Q_R^T)^T
+  float* Zt_lo = nullptr;
   void* qr_ws = nullptr;
   size_t qr_ws_bytes = 0;
   int* d_status = nullptr;
@@ -137,6 +156,71 @@ void free_all(soap_handle h) {
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+soap::TcOperand opnd(const float* hi, const float* lo, int64_t ld, int64_t stride, int batch) {
+  return soap::TcOperand{hi, lo, ld, stride, batch};
+}
+
+soap::TcEpilogue epi(soap_handle h, float* C, int64_t ldc, int64_t c_stride, float* C_lo, int transpose, float alpha,
+                     float beta) {
+  return soap::TcEpilogue{C, nullptr, ldc, c_stride, C_lo, ldc, c_stride, transpose, alpha, beta, h->d_status};
+}
+
+// One step of a two-sided class with every contraction as a tcgen05 3xTF32 product
+// C = A B^T of K-major operands:
+//   S1  L <- b L + (1-b) G G^T       A = G,     B = G
+//       R <- b R + (1-b) G^T G       A = G^T,   B = G^T
+//   S2  P = L Q_L                    A = L,     B = Q_L^T    -> QR -> Q_L, Q_L^T
+//   S5  Y^T = ([G | M_hat] Q_R)^T    A = [G|M], B = Q_R^T    (transposed epilogue)
+//       [G' | m'] = Q_L^T Y          A = Q_L^T, B = Y^T
+//   S6  N = Adam(G', m', v)
+//   S7  Z^T = (N Q_R^T)^T            A = N,     B = Q_R      (transposed epilogue)
+//   S8  W <- (1 - lr wd) W - lr Q_L Z  A = Q_L, B = Z^T      (epilogue into W)
+soap_status_t step_tensor_core(soap_handle h, ClassState& c, float* const* d_params, const float* const* d_grads,
+                               bool refresh, float bc1, float bc2, cudaStream_t s) {
+  const soap_hparams& hp = h->hp;
+  const int B = c.count, m = (int)c.rows, n = (int)c.cols;
+  const int64_t mn = (int64_t)m * n, mm = (int64_t)m * m, nn = (int64_t)n * n;
+  const int64_t cls = (int64_t)B * mn;
+  float* GM = c.Gc;
+  SOAP_CUDA(h, soap::momentum_split(d_grads, GM, c.GM_lo, c.Gt, c.Gt_lo, c.Mhat, c.GM_lo + cls, m, n, B, hp.beta1,
+                                    h->d_status, s));
+  if (c.basis_dirty) {
+    SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, B, s));
+    SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, n, B, s));
+    c.basis_dirty = false;
+  }
+  const float fb = hp.factor_beta;
+  SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(GM, c.GM_lo, n, mn, B), opnd(GM, c.GM_lo, n, mn, B),
+                                epi(h, c.L, m, mm, c.L_lo, 0, 1.f - fb, fb), s));
+  SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(c.Gt, c.Gt_lo, m, mn, B), opnd(c.Gt, c.Gt_lo, m, mn, B),
+                                epi(h, c.R, n, nn, c.R_lo, 0, 1.f - fb, fb), s));
+  if (refresh) {
+    float* P = (float*)h->qr_ws;  // the QR factors its workspace's first matrix block in place
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, m, m, B, opnd(c.L, c.L_lo, m, mm, B), opnd(c.QLt, c.QLt_lo, m, mm, B),
+                                  epi(h, P, m, mm, nullptr, 0, 1.f, 0.f), s));
+    SOAP_CUDA(h, soap::qr_q(m, B, P, c.QL, c.skipL, hp.qr_tol, h->qr_ws, h->qr_ws_bytes, h->d_status, s));
+    SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, B, s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(n, n, n, B, opnd(c.R, c.R_lo, n, nn, B), opnd(c.QRt, c.QRt_lo, n, nn, B),
+                                  epi(h, P, n, nn, nullptr, 0, 1.f, 0.f), s));
+    SOAP_CUDA(h, soap::qr_q(n, B, P, c.QR, c.skipR, hp.qr_tol, h->qr_ws, h->qr_ws_bytes, h->d_status, s));
+    SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, n, B, s));
+  }
+  // rotations of the gradient and of the momentum in one launch each (batch 2B)
+  SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, 2 * B, opnd(GM, c.GM_lo, n, mn, 2 * B), opnd(c.QRt, c.QRt_lo, n, nn, B),
+                                epi(h, h->YMt, m, mn, h->YMt_lo, 1, 1.f, 0.f), s));
+  SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, 2 * B, opnd(c.QLt, c.QLt_lo, m, mm, B), opnd(h->YMt, h->YMt_lo, m, mn, 2 * B),
+                                epi(h, h->Gp, n, mn, nullptr, 0, 1.f, 0.f), s));
+  SOAP_CUDA(h, soap::adam_in_basis(h->Gp, h->Gp + cls, c.V, m, n, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
+                                   hp.guard ? c.skipL : nullptr, hp.guard ? c.skipR : nullptr, h->N_lo, h->d_status,
+                                   s));
+  SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, B, opnd(h->Gp, h->N_lo, n, mn, B), opnd(c.QR, c.QR_lo, n, nn, B),
+                                epi(h, h->Zt, m, mn, h->Zt_lo, 1, 1.f, 0.f), s));
+  soap::TcEpilogue ew = epi(h, nullptr, n, 0, nullptr, 0, -h->lr, 1.f - h->lr * h->wd);
+  ew.C_ptrs = d_params;
+  SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, B, opnd(c.QL, c.QL_lo, m, mm, B), opnd(h->Zt, h->Zt_lo, m, mn, B), ew, s));
+  return SOAP_OK;
+}
 
 }  // namespace
 
@@ -215,14 +299,26 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
     const size_t mn = (size_t)c.count * c.rows * c.cols;
     c.ptr_offset = off;
     off += 2 * (size_t)c.count;
-    if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gc, mn * 4);
-    if (e == cudaSuccess) e = dalloc(h, (void**)&c.Mhat, mn * 4);
+    c.tc = c.left && c.right && (c.rows % 4 == 0) && (c.cols % 4 == 0);
+    if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gc, 2 * mn * 4);  // [G copy | M_hat]
+    c.Mhat = c.Gc ? c.Gc + mn : nullptr;
     if (e == cudaSuccess) e = dalloc(h, (void**)&c.V, mn * 4);
+    if (c.tc) {
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.GM_lo, 2 * mn * 4);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gt, mn * 4);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gt_lo, mn * 4);
+    }
     if (c.left) {
       const size_t mm = (size_t)c.count * c.rows * c.rows;
       if (e == cudaSuccess) e = dalloc(h, (void**)&c.L, mm * 4);
       if (e == cudaSuccess) e = dalloc(h, (void**)&c.QL, mm * 4);
       if (e == cudaSuccess) e = dalloc(h, (void**)&c.skipL, (size_t)c.count * c.rows);
+      if (c.tc) {
+        if (e == cudaSuccess) e = dalloc(h, (void**)&c.L_lo, mm * 4);
+        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QL_lo, mm * 4);
+        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QLt, mm * 4);
+        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QLt_lo, mm * 4);
+      }
       ws_qr = std::max(ws_qr, soap::qr_workspace_bytes((int)c.rows, c.count));
     }
     if (c.right) {
@@ -230,15 +326,30 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
       if (e == cudaSuccess) e = dalloc(h, (void**)&c.R, nn * 4);
       if (e == cudaSuccess) e = dalloc(h, (void**)&c.QR, nn * 4);
       if (e == cudaSuccess) e = dalloc(h, (void**)&c.skipR, (size_t)c.count * c.cols);
+      if (c.tc) {
+        if (e == cudaSuccess) e = dalloc(h, (void**)&c.R_lo, nn * 4);
+        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QR_lo, nn * 4);
+        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QRt, nn * 4);
+        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QRt_lo, nn * 4);
+      }
       ws_qr = std::max(ws_qr, soap::qr_workspace_bytes((int)c.cols, c.count));
     }
     ws_mat = std::max(ws_mat, mn);
   }
   h->nptrs = off;
+  bool any_tc = false;
+  for (auto& c : h->classes) any_tc |= c.tc;
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->X1, ws_mat * 4);
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->X2, ws_mat * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Gp, ws_mat * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Mp, ws_mat * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Gp, 2 * ws_mat * 4);
+  h->Mp = h->Gp ? h->Gp + ws_mat : nullptr;
+  if (any_tc) {
+    if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt, 2 * ws_mat * 4);
+    if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt_lo, 2 * ws_mat * 4);
+    if (e == cudaSuccess) e = dalloc(h, (void**)&h->N_lo, ws_mat * 4);
+    if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt, ws_mat * 4);
+    if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt_lo, ws_mat * 4);
+  }
   if (e == cudaSuccess) e = dalloc(h, &h->qr_ws, ws_qr);
   h->qr_ws_bytes = ws_qr;
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_status, sizeof(int));
@@ -345,6 +456,11 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
     float* const* d_params = reinterpret_cast<float* const*>(h->d_ptrs + c.ptr_offset);
     const float* const* d_grads = reinterpret_cast<const float* const*>(h->d_ptrs + c.ptr_offset + B);
 
+    if (c.tc) {
+      soap_status_t st = step_tensor_core(h, c, d_params, d_grads, refresh, bc1, bc2, s);
+      if (st != SOAP_OK) return st;
+      continue;
+    }
     SOAP_CUDA(h, soap::momentum_and_copy(d_grads, c.Gc, c.Mhat, mn, B, hp.beta1, h->d_status, s));
     const float fb = hp.factor_beta;
     if (c.left) {  // S1: L <- b L + (1-b) G G^T
@@ -395,7 +511,7 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
     // S6
     SOAP_CUDA(h, soap::adam_in_basis(gp, mp, c.V, m, nc, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
                                      (hp.guard && c.left) ? c.skipL : nullptr,
-                                     (hp.guard && c.right) ? c.skipR : nullptr, h->d_status, s));
+                                     (hp.guard && c.right) ? c.skipR : nullptr, nullptr, h->d_status, s));
     // S7 + S8: W <- (1 - lr wd) W - lr Q_L N Q_R^T
     const float keep = 1.f - h->lr * h->wd;
     soap::MutOperand W{nullptr, d_params, 0, 0, nc};
@@ -497,6 +613,7 @@ soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const vo
   cudaStream_t s = (cudaStream_t)stream_;
   if (which != SOAP_STATE_M) {
     SOAP_CUDA(h, cudaMemcpyAsync(state_ptr(h, idx, which), src, bytes, cudaMemcpyDefault, s));
+    if (which == SOAP_STATE_QL || which == SOAP_STATE_QR) h->classes[h->loc[idx].first].basis_dirty = true;
     return SOAP_OK;
   }
   // M_hat = Q_L m Q_R^T
@@ -636,6 +753,32 @@ soap_status_t soap_gemm(int32_t trans_a, int32_t trans_b, int32_t M, int32_t N, 
                              soap::strided(B, ldb, stride_b), beta, soap::strided_mut(C, ldc, stride_c), batch,
                              (cudaStream_t)stream);
   return e == cudaSuccess ? SOAP_OK : SOAP_ERR_CUDA;
+}
+
+soap_status_t soap_gemm_tf32x3(int32_t M, int32_t N, int32_t K, int32_t batch, const float* A_hi, const float* A_lo,
+                               int64_t lda, int64_t stride_a, const float* B_hi, const float* B_lo, int64_t ldb,
+                               int64_t stride_b, int32_t b_batch, float alpha, float beta, float* C, int64_t ldc,
+                               int64_t stride_c, int32_t transpose_c, float* C_lo, int32_t* status,
+                               soap_stream_t stream) {
+  if (M < 0 || N < 0 || K < 0 || batch < 0 || batch > 65535 || b_batch < 0) return SOAP_ERR_INVALID_ARG;
+  if (M == 0 || N == 0 || batch == 0) return SOAP_OK;
+  if (!A_hi || !A_lo || !B_hi || !B_lo || !C) return SOAP_ERR_INVALID_ARG;
+  const void* ptrs[6] = {A_hi, A_lo, B_hi, B_lo, C, C_lo ? C_lo : C};
+  for (const void* p : ptrs)
+    if (!aligned16(p)) return SOAP_ERR_INVALID_ARG;
+  if ((lda | ldb | ldc | stride_a | stride_b | stride_c) & 3) return SOAP_ERR_INVALID_ARG;
+  if (lda < K || ldb < K || ldc < (transpose_c ? M : N)) return SOAP_ERR_INVALID_ARG;
+  soap::TcOperand A{A_hi, A_lo, lda, stride_a, batch};
+  soap::TcOperand B{B_hi, B_lo, ldb, stride_b, b_batch > 0 ? b_batch : batch};
+  soap::TcEpilogue ep{C, nullptr, ldc, stride_c, C_lo, ldc, stride_c, transpose_c, alpha, beta,
+                      reinterpret_cast<int*>(status)};
+  cudaError_t e = soap::gemm_tc_nt(M, N, K, batch, A, B, ep, (cudaStream_t)stream);
+  return e == cudaSuccess ? SOAP_OK : (e == cudaErrorInvalidValue ? SOAP_ERR_INVALID_ARG : SOAP_ERR_CUDA);
+}
+
+soap_status_t soap_split_tf32(const float* x, float* hi, float* lo, int64_t n, soap_stream_t stream) {
+  if (n < 0 || (n > 0 && (!x || !lo))) return SOAP_ERR_INVALID_ARG;
+  return soap::split_tf32(x, hi, lo, n, (cudaStream_t)stream) == cudaSuccess ? SOAP_OK : SOAP_ERR_CUDA;
 }
 
 }  // extern "C"

@@ -48,6 +48,32 @@ cudaError_t gemm(bool trans_a, bool trans_b, int M, int N, int K, float alpha, O
 cudaError_t gemm_simt(bool trans_a, bool trans_b, int M, int N, int K, float alpha, Operand A,
                       Operand B, float beta, MutOperand C, int batch, cudaStream_t stream);
 
+// ---- tcgen05 3xTF32 engine: C_b = alpha * A_b B_(b mod B.batch)^T + beta * C_b ----------
+// An operand is `batch` row-major (rows x K) matrices split as hi = tf32(x), lo = x - hi.
+struct TcOperand {
+  const float* hi;
+  const float* lo;
+  int64_t ld;      // elements between rows
+  int64_t stride;  // elements between matrices
+  int batch;       // distinct matrices (0: one per launch batch entry)
+};
+struct TcEpilogue {
+  float* C;              // output (or nullptr), offset b * c_stride ...
+  float* const* C_ptrs;  // ... or a device array of per-matrix output pointers
+  int64_t ldc;
+  int64_t c_stride;
+  float* C_lo;           // optional: also write out - tf32(out) here (same layout, ld_lo)
+  int64_t ld_lo;
+  int64_t lo_stride;
+  int transpose;         // write C^T (C_b is then N x M with leading dimension ldc)
+  float alpha, beta;     // beta != 0 reads C
+  int* status;           // device status word for a timed-out wait (may be nullptr)
+};
+cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const TcOperand& B,
+                       const TcEpilogue& ep, cudaStream_t stream);
+// hi = tf32(x) (round to nearest, ties away), lo = x - hi, elementwise over n values.
+cudaError_t split_tf32(const float* x, float* hi, float* lo, int64_t n, cudaStream_t stream);
+
 // Householder QR (explicit Q) of `batch` contiguous n x n matrices.
 size_t qr_workspace_bytes(int n, int batch);
 cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, float tol,
@@ -61,8 +87,16 @@ cudaError_t momentum_and_copy(const float* const* grads, float* Gc, float* Mhat,
 // written over Gp; guard rows/cols zeroed.
 cudaError_t adam_in_basis(float* Gp, const float* Mp, float* V, int rows, int cols, int batch,
                           float beta1, float beta2, float eps, float bc1, float bc2,
-                          const uint8_t* skipL, const uint8_t* skipR, int* status,
+                          const uint8_t* skipL, const uint8_t* skipR, float* N_lo, int* status,
                           cudaStream_t stream);
+// Tensor-core operand preparation for a two-sided class: G copy, G^T and their lo parts,
+// M_hat <- b1 M_hat + (1-b1) G and its lo part.
+cudaError_t momentum_split(const float* const* grads, float* Gc, float* Gc_lo, float* Gt, float* Gt_lo,
+                           float* Mhat, float* Mhat_lo, int rows, int cols, int batch, float beta1,
+                           int* status, cudaStream_t stream);
+// Q -> lo part, Q^T, lo part of Q^T for `batch` n x n bases.
+cudaError_t basis_split(const float* Q, float* Q_lo, float* Qt, float* Qt_lo, int n, int batch,
+                        cudaStream_t stream);
 // W <- (1 - lr*wd) W - lr * D (both sides identity).
 cudaError_t weight_update(float* const* params, const float* D, int64_t elems, int batch,
                           float lr, float wd, cudaStream_t stream);

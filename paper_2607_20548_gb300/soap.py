@@ -25,7 +25,8 @@ STATE_M, STATE_V, STATE_L, STATE_QL, STATE_R, STATE_QR, STATE_MHAT, STATE_SKIP_L
 EXPORTS = ("soap_default_hparams", "soap_create", "soap_step", "soap_set_lr", "soap_state_bytes",
            "soap_state_get", "soap_state_set", "soap_get_step", "soap_set_step", "soap_status",
            "soap_clear_status", "soap_last_error", "soap_destroy", "soap_qr_workspace_bytes",
-           "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end")
+           "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_gemm_tf32x3",
+           "soap_split_tf32")
 KERNEL_FAMILIES = ("gemm_simt", "gemm_tc", "qr_panel", "elementwise", "other")
 
 
@@ -84,6 +85,9 @@ def load_library(path: str = LIB_PATH):
         "soap_profile_begin": (I32, [P, I64]),
         "soap_profile_end": (I32, [P, P, ctypes.POINTER(soap_kernel_stats), ctypes.POINTER(I32)]),
         "soap_gemm": (I32, [I32, I32, I32, I32, I32, F, P, I64, I64, P, I64, I64, F, P, I64, I64, I32, P]),
+        "soap_gemm_tf32x3": (I32, [I32, I32, I32, I32, P, P, I64, I64, P, P, I64, I64, I32, F, F, P, I64, I64,
+                                   I32, P, P, P]),
+        "soap_split_tf32": (I32, [P, P, P, I64, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -288,3 +292,44 @@ def soap_gemm(A: torch.Tensor, B: torch.Tensor, trans_a=False, trans_b=False, al
                          ctypes.c_void_p(B3.data_ptr()), B3.shape[2], B3.shape[1] * B3.shape[2], float(beta),
                          ctypes.c_void_p(C3.data_ptr()), N, M * N, batch, _stream(stream)))
     return C3[0] if squeeze else C3
+
+
+def soap_split_tf32(x: torch.Tensor, stream=None):
+    """(hi, lo) with hi = tf32(x) and lo = x - hi, computed on the device."""
+    x = x.contiguous()
+    hi, lo = torch.empty_like(x), torch.empty_like(x)
+    _check(load_library().soap_split_tf32(ctypes.c_void_p(x.data_ptr()), ctypes.c_void_p(hi.data_ptr()),
+                                          ctypes.c_void_p(lo.data_ptr()), x.numel(), _stream(stream)))
+    return hi, lo
+
+
+def soap_gemm_tf32x3(A, B, alpha=1.0, beta=0.0, C=None, transpose_c=False, A_split=None, B_split=None,
+                     with_lo=False, status=None, stream=None):
+    """Tensor-core C = alpha A B^T + beta C for [batch, M, K] x [b_batch, N, K] fp32 CUDA tensors.
+
+    A_split / B_split give (hi, lo) explicitly; by default they come from soap_split_tf32.
+    Returns C (and C_lo if with_lo)."""
+    lib = load_library()
+    A3 = (A.unsqueeze(0) if A.dim() == 2 else A).contiguous()
+    B3 = (B.unsqueeze(0) if B.dim() == 2 else B).contiguous()
+    batch, M, K = A3.shape
+    bb, N, K2 = B3.shape
+    assert K == K2
+    ahi, alo = A_split if A_split is not None else soap_split_tf32(A3, stream)
+    bhi, blo = B_split if B_split is not None else soap_split_tf32(B3, stream)
+    shape = (batch, N, M) if transpose_c else (batch, M, N)
+    C3 = torch.zeros(shape, dtype=torch.float32, device=A3.device) if C is None else \
+        (C.unsqueeze(0) if C.dim() == 2 else C)
+    lo = torch.zeros_like(C3) if with_lo else None
+    ldc = shape[2]
+    _check(lib.soap_gemm_tf32x3(M, N, K, batch, ctypes.c_void_p(ahi.data_ptr()), ctypes.c_void_p(alo.data_ptr()),
+                                K, M * K, ctypes.c_void_p(bhi.data_ptr()), ctypes.c_void_p(blo.data_ptr()), K,
+                                N * K, bb, float(alpha), float(beta), ctypes.c_void_p(C3.data_ptr()), ldc,
+                                shape[1] * shape[2], int(transpose_c),
+                                ctypes.c_void_p(lo.data_ptr()) if with_lo else None,
+                                ctypes.c_void_p(status.data_ptr()) if status is not None else None,
+                                _stream(stream)))
+    out = C3[0] if A.dim() == 2 and (C is None or C.dim() == 2) else C3
+    if with_lo:
+        return out, (lo[0] if out.dim() == 2 else lo)
+    return out

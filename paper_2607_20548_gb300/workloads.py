@@ -15,8 +15,9 @@ cols), N_t i.i.d. N(0, 1/cols) drawn afresh every step, W_0 ~ N(0, 0.02^2), and 
 except for MoE experts, whose c is drawn once per expert, log-uniform in [1e-2, 1],
 to mimic uneven token routing.
 
-All tensors are float32 and generated with torch on the requested device; the oracle
-gets host copies of exactly the same values.
+All tensors are float32. U, V (and so A) are drawn on the host; W_0 and the per-step
+noise are drawn with torch on the requested device; the oracle gets host copies of
+exactly the same values.
 """
 from __future__ import annotations
 
@@ -111,16 +112,17 @@ class GradientStream:
         self._A = []
         self._c = []
         for gi, (s, idx) in enumerate(self.groups):
+            # U, V and A are drawn on the host (the same values whatever the device), then moved
             k = min(s.rows, s.cols)
-            g = torch.Generator(device=self.device).manual_seed(_seed(seed, gi, 1))
+            g = torch.Generator().manual_seed(_seed(seed, gi, 1))
             B = len(idx)
-            U = torch.linalg.qr(torch.randn(B, s.rows, k, generator=g, device=self.device))[0]
-            V = torch.linalg.qr(torch.randn(B, s.cols, k, generator=g, device=self.device))[0]
-            i = torch.arange(1, k + 1, dtype=torch.float64, device=self.device)
+            U = torch.linalg.qr(torch.randn(B, s.rows, k, generator=g))[0]
+            V = torch.linalg.qr(torch.randn(B, s.cols, k, generator=g))[0]
+            i = torch.arange(1, k + 1, dtype=torch.float64)
             sv = i.pow(-1.5)
             sv = (sv / sv.norm()).to(torch.float32)
             A = torch.matmul(U * sv, V.transpose(1, 2))
-            self._A.append(A.contiguous())
+            self._A.append(A.contiguous().to(self.device))
             self._c.append(torch.tensor([self.scales[j] for j in idx], dtype=torch.float32,
                                         device=self.device).view(B, 1, 1))
 
