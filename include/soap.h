@@ -197,8 +197,10 @@ soap_status_t soap_gemm(int32_t trans_a, int32_t trans_b, int32_t M, int32_t N, 
 
 /* The tensor-core form of that product (tcgen05, 3xTF32): for b < batch,
  *   C_b = alpha * A_b * B_(b mod b_batch)^T + beta * C_b        (or C_b^T if transpose_c)
- * with A_b (M x K) and B (N x K) row-major, each given as hi = tf32(x) and lo = x - hi
- * (see soap_split_tf32); the accumulator adds a_lo b_hi + a_hi b_lo + a_hi b_hi in fp32.
+ * with A_b (M x K) and B (N x K) row-major, each given as hi and lo = x - hi where hi is x
+ * with its 13 low mantissa bits cleared (the tf32 value the tensor core reads from an fp32
+ * word, so hi may be x itself; see soap_split_tf32); the accumulator adds
+ * a_lo b_hi + a_hi b_lo + a_hi b_hi in fp32.
  * lda, ldb, ldc and every batch stride must be multiples of 4 elements and every
  * pointer 16-byte aligned. C_lo, if non-NULL, receives out - tf32(out) in C's layout
  * (leading dimension ldc). status, if non-NULL, is a device int that gets bit 4 set if
@@ -210,8 +212,8 @@ soap_status_t soap_gemm_tf32x3(int32_t M, int32_t N, int32_t K, int32_t batch, c
                                int32_t transpose_c, float* C_lo, int32_t* status,
                                soap_stream_t stream);
 
-/* hi = tf32(x) rounded to nearest (ties away from zero), lo = x - hi, for n values on
- * the device; hi may be NULL. */
+/* hi = x with its 13 low mantissa bits cleared (tf32 by truncation), lo = x - hi (exact),
+ * for n values on the device; hi may be NULL. */
 soap_status_t soap_split_tf32(const float* x, float* hi, float* lo, int64_t n, soap_stream_t stream);
 
 #ifdef __cplusplus

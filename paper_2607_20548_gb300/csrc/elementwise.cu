@@ -85,11 +85,7 @@ __global__ void adam_kernel(float* Gp, const float* Mp, float* V, int rows, int 
     if ((sl && sl[i / cols]) || (sr && sr[i % cols])) nv = 0.f;
     bad |= !isfinite(nv);
     gp[i] = nv;
-    if (N_lo) {
-      uint32_t r;
-      asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(nv));
-      N_lo[(int64_t)b * elems + i] = nv - __uint_as_float(r);
-    }
+    if (N_lo) N_lo[(int64_t)b * elems + i] = nv - __uint_as_float(__float_as_uint(nv) & 0xFFFFE000u);
   }
   if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(status, kStatusNonFinite);
 }
@@ -114,11 +110,11 @@ __global__ void identity_kernel(float* Q, int n) {
     q[i] = (i / n == i % n) ? 1.f : 0.f;
 }
 
-__device__ __forceinline__ float lo_part(float x) {
-  uint32_t r;
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
-  return x - __uint_as_float(r);
-}
+// The tensor core reads an fp32 word as tf32 by dropping its 13 low mantissa bits, so
+// an fp32 array serves directly as the "hi" operand and its lo part is x - trunc(x)
+// (exact in fp32).
+__device__ __forceinline__ float tf32_trunc(float x) { return __uint_as_float(__float_as_uint(x) & 0xFFFFE000u); }
+__device__ __forceinline__ float lo_part(float x) { return x - tf32_trunc(x); }
 
 // One 32 x 32 tile of one matrix per block (32 x 8 threads). Reads G, updates M_hat and
 // writes the tensor-core operands: G (copy) and its lo part, G^T and its lo part, and
@@ -192,9 +188,7 @@ __global__ void split_kernel(const float* x, float* hi, float* lo, int64_t n) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
     const float v = x[i];
-    uint32_t r;
-    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(v));
-    const float h = __uint_as_float(r);
+    const float h = tf32_trunc(v);
     if (hi) hi[i] = h;
     lo[i] = v - h;
   }

@@ -4,16 +4,24 @@
 //
 // A_b is M x K and B is N x K, both row-major ("K-major"), so TMA copies their tiles
 // straight into the canonical 128-byte-swizzled K-major shared-memory layout that
-// tcgen05.mma reads. Every operand comes as a pair (hi, lo) with hi = tf32(x) and
-// lo = x - tf32(x); the accumulator (fp32, in tensor memory) receives
+// tcgen05.mma reads. Every operand comes as a pair (hi, lo): the tensor core reads an
+// fp32 word as tf32 by dropping its 13 low mantissa bits, so hi may be the fp32 array
+// itself and lo = x - trunc_tf32(x) (exact); the accumulator (fp32, in TMEM) receives
 //   a_lo b_hi + a_hi b_lo + a_hi b_hi              ("3xTF32")
 // which keeps ~22 bits of each operand: products with fp32 accuracy at tensor-core
 // rate, as the optimizer step's fp32 arithmetic requires.
 //
+// The tensor core's own accumulation rounds toward zero at every MMA, so a long chain
+// of MMAs into one accumulator drifts (relative error growing ~linearly in K: 6e-5 at
+// K = 8192). Each 32-wide K block is therefore accumulated afresh in one of two TMEM
+// accumulators while the epilogue warps drain the other into fp32 registers with
+// round-to-nearest adds; the drain of block k overlaps the MMAs of block k+1, and the
+// error stays at the level of an fp32 dot product.
+//
 // CTA: 192 threads. Warp 0 issues the TMA loads (one elected lane), warp 1 allocates
-// tensor memory and issues the MMAs (one elected lane), warps 2-5 run the epilogue:
-// tensor memory -> registers (each warp owns 32 of the 128 accumulator lanes) ->
-// alpha/beta -> global, optionally transposed and optionally also writing the lo part
+// tensor memory and issues the MMAs (one elected lane), warps 2-5 drain the
+// accumulators and run the epilogue: tensor memory -> registers (each warp owns 32 of
+// the 128 accumulator lanes) -> alpha/beta -> global, optionally transposed and optionally also writing the lo part
 // of the result for a later product. Stages are handed over with mbarriers; every
 // wait gives up after ~2 s of %globaltimer time, records kStatusTimeout and lets the
 // CTA drain and free its tensor memory instead of hanging.
@@ -39,7 +47,7 @@ struct Cfg {
   static constexpr int TILE_B = BN * BK * 4;
   static constexpr int STAGE = 2 * TILE_A + 2 * TILE_B;
   static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
-  static constexpr uint32_t TMEM_COLS = BN;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators, used alternately
   static_assert(SMEM <= 232448, "shared memory budget");
 };
 
@@ -144,11 +152,8 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-__device__ __forceinline__ float tf32_rna(float x) {
-  uint32_t r;
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
-  return __uint_as_float(r);
-}
+// tf32 value the tensor core reads from an fp32 word (13 low mantissa bits dropped).
+__device__ __forceinline__ float tf32_trunc(float x) { return __uint_as_float(__float_as_uint(x) & 0xFFFFE000u); }
 
 template <int BN, int STAGES>
 __global__ void __launch_bounds__(THREADS, 1)
@@ -160,8 +165,9 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE);
   uint64_t* empty = full + STAGES;
-  uint64_t* tmem_full = empty + STAGES;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(tmem_full + 1);
+  uint64_t* acc_full = empty + STAGES;  // [2] accumulator a holds a finished K block
+  uint64_t* acc_empty = acc_full + 2;   // [2] accumulator a has been drained
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acc_empty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
   volatile int* consumed = abort_flag + 1;
 
@@ -174,7 +180,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(tmem_full, 1);
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&acc_full[a], 1);
+      mbar_init(&acc_empty[a], 4);  // one arrival per epilogue warp
+    }
     *abort_flag = 0;
     *consumed = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -225,12 +234,15 @@ __global__ void __launch_bounds__(THREADS, 1)
       for (int kb = 0; kb < kblocks; ++kb) {
         const int s = kb % STAGES;
         const uint32_t ph = (kb / STAGES) & 1;
-        if (!mbar_wait(&full[s], ph) || *abort_flag) {
+        const int a = kb & 1;
+        if (!mbar_wait(&full[s], ph) || (kb >= 2 && !mbar_wait(&acc_empty[a], ((kb >> 1) & 1) ^ 1)) ||
+            *abort_flag) {
           *abort_flag = 1;
           break;
         }
         *consumed = kb + 1;
         tc_fence_after();
+        const uint32_t d = tmem + static_cast<uint32_t>(a * BN);
         const uint32_t a_hi = smem_u32(smem + s * C::STAGE);
         const uint32_t a_lo = a_hi + C::TILE_A;
         const uint32_t b_hi = a_hi + 2 * C::TILE_A;
@@ -238,46 +250,64 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int kk = 0; kk < BK / 8; ++kk) {
           const uint32_t off = kk * 32;  // 8 tf32 = 32 bytes along K inside the swizzle row
-          umma_tf32(tmem, desc_sw128(a_lo + off), desc_sw128(b_hi + off), idesc, (kb | kk) != 0);
-          umma_tf32(tmem, desc_sw128(a_hi + off), desc_sw128(b_lo + off), idesc, 1u);
-          umma_tf32(tmem, desc_sw128(a_hi + off), desc_sw128(b_hi + off), idesc, 1u);
+          umma_tf32(d, desc_sw128(a_lo + off), desc_sw128(b_hi + off), idesc, kk != 0);
+          umma_tf32(d, desc_sw128(a_hi + off), desc_sw128(b_lo + off), idesc, 1u);
+          umma_tf32(d, desc_sw128(a_hi + off), desc_sw128(b_hi + off), idesc, 1u);
         }
-        umma_commit(&empty[s]);  // frees the stage once these MMAs have read it
+        umma_commit(&empty[s]);     // frees the stage once these MMAs have read it
+        umma_commit(&acc_full[a]);  // hands the K block's sum to the epilogue warps
       }
-      umma_commit(tmem_full);  // arrives when every MMA issued above has completed
     }
   } else {
     const int q = warp & 3;  // this warp may read accumulator lanes 32q .. 32q+31
-    const bool ok = mbar_wait(tmem_full, 0);
-    tc_fence_after();
-    const bool valid = ok && !*abort_flag;
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * q) << 16);
+    float acc[BN / 32][32];
+#pragma unroll
+    for (int c = 0; c < BN / 32; ++c)
+#pragma unroll
+      for (int j = 0; j < 32; ++j) acc[c][j] = 0.f;
+    bool valid = true;
+    for (int kb = 0; kb < kblocks; ++kb) {
+      const int a = kb & 1;
+      if (!mbar_wait(&acc_full[a], (kb >> 1) & 1) || *abort_flag) {
+        valid = false;
+        break;
+      }
+      tc_fence_after();
+#pragma unroll
+      for (int c = 0; c < BN / 32; ++c) {
+        float v[32];
+        tmem_ld32(lane_base + static_cast<uint32_t>(a * BN + 32 * c), v);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) acc[c][j] += v[j];
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0)
+        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&acc_empty[a])) : "memory");
+    }
     if (!valid && lane == 0 && ep.status) atomicOr(ep.status, kStatusTimeout);
     const int r = m0 + 32 * q + lane;
     float* Cb = ep.C_ptrs ? ep.C_ptrs[b] : (ep.C ? ep.C + (int64_t)b * ep.c_stride : nullptr);
     float* Lb = ep.C_lo ? ep.C_lo + (int64_t)b * ep.lo_stride : nullptr;
-    for (int c = 0; c < BN / 32 && valid; ++c) {
-      const int col0 = n0 + 32 * c;
-      if (col0 >= N) break;  // warp-uniform
-      float v[32];
-      tmem_ld32(tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(32 * c), v);
-      if (kblocks == 0) {
+    if (valid && r < M) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = 0.f;
-      }
-      if (r >= M) continue;
+      for (int c = 0; c < BN / 32; ++c) {
+        const int col0 = n0 + 32 * c;
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const int col = col0 + j;
-        if (col >= N) break;
-        const int64_t off = ep.transpose ? (int64_t)col * ep.ldc + r : (int64_t)r * ep.ldc + col;
-        float out = ep.alpha * v[j];
-        if (Cb) {
-          if (ep.beta != 0.f) out = fmaf(ep.beta, Cb[off], out);
-          Cb[off] = out;
-        }
-        if (Lb) {
-          const int64_t lo_off = ep.transpose ? (int64_t)col * ep.ld_lo + r : (int64_t)r * ep.ld_lo + col;
-          Lb[lo_off] = out - tf32_rna(out);
+        for (int j = 0; j < 32; ++j) {
+          const int col = col0 + j;
+          if (col >= N) break;
+          const int64_t off = ep.transpose ? (int64_t)col * ep.ldc + r : (int64_t)r * ep.ldc + col;
+          float out = ep.alpha * acc[c][j];
+          if (Cb) {
+            if (ep.beta != 0.f) out = fmaf(ep.beta, Cb[off], out);
+            Cb[off] = out;
+          }
+          if (Lb) {
+            const int64_t lo_off = ep.transpose ? (int64_t)col * ep.ld_lo + r : (int64_t)r * ep.ld_lo + col;
+            Lb[lo_off] = out - tf32_trunc(out);
+          }
         }
       }
     }

@@ -370,6 +370,7 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
   for (auto& c : h->classes) {
     const size_t mn = (size_t)c.count * c.rows * c.cols;
     if (e == cudaSuccess) e = cudaMemset(c.Mhat, 0, mn * 4);
+    if (c.tc && e == cudaSuccess) e = cudaMemset(c.GM_lo, 0, 2 * mn * 4);
     if (e == cudaSuccess) e = cudaMemset(c.V, 0, mn * 4);
     if (c.left) {
       if (e == cudaSuccess) e = cudaMemset(c.L, 0, (size_t)c.count * c.rows * c.rows * 4);
@@ -589,6 +590,23 @@ soap_status_t soap_state_get(soap_handle h, int32_t idx, int32_t which, void* ds
   const int m = (int)c.rows, nc = (int)c.cols;
   const int64_t mn = (int64_t)m * nc;
   const float* x = c.Mhat + slot * mn;
+  if (c.tc) {
+    // the same tensor-core products, on the same operands, as the step's rotation of M_hat:
+    // bit-identical to the m the last step used
+    const int64_t mm = (int64_t)m * m, nn = (int64_t)nc * nc, cls = (int64_t)c.count * mn;
+    if (c.basis_dirty) {
+      SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, c.count, s));
+      SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, nc, c.count, s));
+      c.basis_dirty = false;
+    }
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, nc, nc, 1, opnd(x, c.GM_lo + cls + slot * mn, nc, mn, 1),
+                                  opnd(c.QRt + slot * nn, c.QRt_lo + slot * nn, nc, nn, 1),
+                                  epi(h, h->X1, m, mn, h->X2, 1, 1.f, 0.f), s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, nc, m, 1, opnd(c.QLt + slot * mm, c.QLt_lo + slot * mm, m, mm, 1),
+                                  opnd(h->X1, h->X2, m, mn, 1), epi(h, h->Gp, nc, mn, nullptr, 0, 1.f, 0.f), s));
+    SOAP_CUDA(h, cudaMemcpyAsync(dst, h->Gp, bytes, cudaMemcpyDefault, s));
+    return SOAP_OK;
+  }
   using soap::strided;
   using soap::strided_mut;
   if (c.left) {
@@ -613,7 +631,13 @@ soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const vo
   cudaStream_t s = (cudaStream_t)stream_;
   if (which != SOAP_STATE_M) {
     SOAP_CUDA(h, cudaMemcpyAsync(state_ptr(h, idx, which), src, bytes, cudaMemcpyDefault, s));
-    if (which == SOAP_STATE_QL || which == SOAP_STATE_QR) h->classes[h->loc[idx].first].basis_dirty = true;
+    ClassState& cs = h->classes[h->loc[idx].first];
+    if (which == SOAP_STATE_QL || which == SOAP_STATE_QR) cs.basis_dirty = true;
+    if (which == SOAP_STATE_MHAT && cs.tc) {
+      const int64_t mn = cs.rows * cs.cols;
+      SOAP_CUDA(h, soap::split_tf32(cs.Mhat + h->loc[idx].second * mn, nullptr,
+                                    cs.GM_lo + cs.count * mn + h->loc[idx].second * mn, mn, s));
+    }
     return SOAP_OK;
   }
   // M_hat = Q_L m Q_R^T
@@ -638,6 +662,7 @@ soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const vo
   } else if (!c.left) {
     SOAP_CUDA(h, cudaMemcpyAsync(dstm, x, bytes, cudaMemcpyDeviceToDevice, s));
   }
+  if (c.tc) SOAP_CUDA(h, soap::split_tf32(dstm, nullptr, c.GM_lo + c.count * mn + slot * mn, mn, s));
   return SOAP_OK;
 }
 
@@ -763,10 +788,11 @@ soap_status_t soap_gemm_tf32x3(int32_t M, int32_t N, int32_t K, int32_t batch, c
   if (M < 0 || N < 0 || K < 0 || batch < 0 || batch > 65535 || b_batch < 0) return SOAP_ERR_INVALID_ARG;
   if (M == 0 || N == 0 || batch == 0) return SOAP_OK;
   if (!A_hi || !A_lo || !B_hi || !B_lo || !C) return SOAP_ERR_INVALID_ARG;
-  const void* ptrs[6] = {A_hi, A_lo, B_hi, B_lo, C, C_lo ? C_lo : C};
+  // A and B are read by TMA: 16-byte aligned bases, rows and batch strides in multiples of 16 bytes
+  const void* ptrs[4] = {A_hi, A_lo, B_hi, B_lo};
   for (const void* p : ptrs)
     if (!aligned16(p)) return SOAP_ERR_INVALID_ARG;
-  if ((lda | ldb | ldc | stride_a | stride_b | stride_c) & 3) return SOAP_ERR_INVALID_ARG;
+  if ((lda | ldb | stride_a | stride_b) & 3) return SOAP_ERR_INVALID_ARG;
   if (lda < K || ldb < K || ldc < (transpose_c ? M : N)) return SOAP_ERR_INVALID_ARG;
   soap::TcOperand A{A_hi, A_lo, lda, stride_a, batch};
   soap::TcOperand B{B_hi, B_lo, ldb, stride_b, b_batch > 0 ? b_batch : batch};

@@ -49,7 +49,8 @@ cudaError_t gemm_simt(bool trans_a, bool trans_b, int M, int N, int K, float alp
                       Operand B, float beta, MutOperand C, int batch, cudaStream_t stream);
 
 // ---- tcgen05 3xTF32 engine: C_b = alpha * A_b B_(b mod B.batch)^T + beta * C_b ----------
-// An operand is `batch` row-major (rows x K) matrices split as hi = tf32(x), lo = x - hi.
+// An operand is `batch` row-major (rows x K) matrices split as hi = trunc_tf32(x) (the fp32
+// array itself may serve: the tensor core drops the 13 low mantissa bits) and lo = x - hi.
 struct TcOperand {
   const float* hi;
   const float* lo;
@@ -71,7 +72,7 @@ struct TcEpilogue {
 };
 cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const TcOperand& B,
                        const TcEpilogue& ep, cudaStream_t stream);
-// hi = tf32(x) (round to nearest, ties away), lo = x - hi, elementwise over n values.
+// hi = trunc_tf32(x), lo = x - hi (exact), elementwise over n values.
 cudaError_t split_tf32(const float* x, float* hi, float* lo, int64_t n, cudaStream_t stream);
 
 // Householder QR (explicit Q) of `batch` contiguous n x n matrices.

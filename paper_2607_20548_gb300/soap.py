@@ -295,7 +295,7 @@ def soap_gemm(A: torch.Tensor, B: torch.Tensor, trans_a=False, trans_b=False, al
 
 
 def soap_split_tf32(x: torch.Tensor, stream=None):
-    """(hi, lo) with hi = tf32(x) and lo = x - hi, computed on the device."""
+    """(hi, lo) with hi = x truncated to tf32 and lo = x - hi, computed on the device."""
     x = x.contiguous()
     hi, lo = torch.empty_like(x), torch.empty_like(x)
     _check(load_library().soap_split_tf32(ctypes.c_void_p(x.data_ptr()), ctypes.c_void_p(hi.data_ptr()),

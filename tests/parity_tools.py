@@ -135,7 +135,10 @@ class TeacherForcedCheck:
         for r in self.rows:
             if not r["ill"] and not r["e_gpu"] <= max(TOL, TWIN_FACTOR * r["e_twin"]):
                 bad.append(f"update: {r}")
-            if not r["e_self"] <= 1e-4:
+            # the update against Q_L N(m, v) Q_R^T from the GPU's own state: m is re-derived through
+            # other fp32 products than the step used, so on ordinary steps it shares the update's
+            # bound; on steps beyond fp32 resolution it is the main check and is held tight
+            if not r["e_self"] <= (2e-4 if r["ill"] else max(TOL, TWIN_FACTOR * r["e_twin"])):
                 bad.append(f"self-consistency of the update: {r}")
             for k in ("e_L", "e_R", "e_v", "e_m"):
                 if k in r and not r[k] <= max(state_tol, TWIN_FACTOR * r["e_twin"] if not r["ill"] else 0.0):

@@ -23,7 +23,8 @@ def _rel(a, b):
 
 
 @pytest.mark.parametrize("M,N,K,batch,bb", [(128, 128, 32, 1, 1), (128, 128, 1024, 2, 2), (200, 130, 100, 3, 3),
-                                            (1, 5, 4, 1, 1), (384, 256, 2048, 2, 1), (1000, 520, 260, 1, 1)])
+                                            (1, 5, 4, 1, 1), (384, 256, 2048, 2, 1), (1000, 520, 260, 1, 1),
+                                            (256, 256, 8192, 1, 1)])
 def test_tc_gemm_matches_fp64(cuda, M, N, K, batch, bb):
     g = torch.Generator(device=cuda).manual_seed(M + N + K)
     A = torch.randn(batch, M, K, device=cuda, generator=g)
@@ -35,8 +36,9 @@ def test_tc_gemm_matches_fp64(cuda, M, N, K, batch, bb):
     torch.cuda.synchronize()
     assert status.item() == 0
     e = _rel(C.double().cpu().numpy(), _ref(A, B, 0.5, -1.25, C0))
-    # fp32-accurate: ~sqrt(K) * 2^-22 at worst for the dropped lo*lo term and fp32 accumulation
-    assert e < 2e-6 * max(1.0, np.sqrt(K) / 16), e
+    # fp32 level at any K: each 32-wide K block is summed afresh and drained with fp32 adds
+    print(f"\nM={M} N={N} K={K}: relative error {e:.2e}")
+    assert e < 2e-6, e
 
 
 def test_tc_gemm_transposed_output_and_lo(cuda):
