@@ -184,6 +184,24 @@ soap_status_t soap_qr(int32_t n, int32_t batch, const float* P, float* Q, uint8_
                       float tol, void* workspace, size_t workspace_bytes,
                       soap_stream_t stream);
 
+/* soap_qr for callers that cannot give this library device memory. The paper has no
+ * counterpart; it exists for callers that cannot allocate when they need a QR: a
+ * cudaMalloc or cudaFree may wait until the whole device is idle, and some programs do
+ * not own their device memory at all (a framework's caching pool, or a fixed budget
+ * handed out at start-up, owns it). Same arguments and results as soap_qr, without the
+ * workspace: it uses a 32 MiB array compiled into libsoap.so, which every GPU that
+ * loads the library keeps until the process exits. That is room for one 2048 x 2048
+ * matrix or, e.g., seven of 1024 x 1024; a (n, batch) whose soap_qr_workspace_bytes()
+ * exceeds 32 MiB - 256 B is refused with SOAP_ERR_INVALID_ARG before anything is
+ * enqueued. It never calls cudaMalloc, cudaFree or any allocating routine.
+ * The first call on each device looks up the array's device address with that device
+ * current (cudaGetSymbolAddress); make that first call before any stream capture. All
+ * calls in the process share the one array per device and it keeps the last call's
+ * contents, so two calls that can overlap on the GPU (different streams without
+ * ordering between them) race: order them, e.g. on one stream. */
+soap_status_t soap_qr_static(int32_t n, int32_t batch, const float* P, float* Q, uint8_t* skip,
+                             float tol, soap_stream_t stream);
+
 /* The fp32-accurate batched product used by every contraction of the step (S1, S2,
  * S4, S5, S7 and the QR updates): for b < batch,
  *   C_b = alpha * op(A_b) * op(B_b) + beta * C_b,

@@ -26,7 +26,7 @@ EXPORTS = ("soap_default_hparams", "soap_create", "soap_step", "soap_set_lr", "s
            "soap_state_get", "soap_state_set", "soap_get_step", "soap_set_step", "soap_status",
            "soap_clear_status", "soap_last_error", "soap_destroy", "soap_qr_workspace_bytes",
            "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_gemm_tf32x3",
-           "soap_split_tf32")
+           "soap_split_tf32", "soap_qr_static")
 KERNEL_FAMILIES = ("gemm_simt", "gemm_tc", "qr_panel", "elementwise", "other")
 
 
@@ -88,6 +88,7 @@ def load_library(path: str = LIB_PATH):
         "soap_gemm_tf32x3": (I32, [I32, I32, I32, I32, P, P, I64, I64, P, P, I64, I64, I32, F, F, P, I64, I64,
                                    I32, P, P, P]),
         "soap_split_tf32": (I32, [P, P, P, I64, P]),
+        "soap_qr_static": (I32, [I32, I32, P, P, P, F, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -267,6 +268,30 @@ def soap_qr(P: torch.Tensor, tol: float = 0.0, stream=None):
     _check(lib.soap_qr(n, batch, ctypes.c_void_p(P.data_ptr()), ctypes.c_void_p(Q.data_ptr()),
                        ctypes.c_void_p(skip.data_ptr()), float(tol), ctypes.c_void_p(ws.data_ptr()), ws_bytes,
                        _stream(stream)))
+    return Q, skip
+
+
+def soap_qr_static(P: torch.Tensor, tol: float = 0.0, stream=None):
+    """soap_qr without a caller-supplied workspace, for code that cannot allocate device memory
+    when it needs the QR: libsoap.so uses a fixed 32 MiB array of its own (enough for one
+    2048 x 2048 matrix). The output tensors here are allocated by torch for convenience; a
+    caller without an allocator passes its own buffers to the C entry point. Raises
+    SoapError(SOAP_ERR_INVALID_ARG) for work larger than the array."""
+    lib = load_library()
+    if P.dim() == 2:
+        P = P.unsqueeze(0)
+    if P.dtype != torch.float32 or not P.is_cuda or P.shape[1] != P.shape[2]:
+        raise TypeError("soap_qr_static: P must be a [batch, n, n] fp32 CUDA tensor")
+    P = P.contiguous()
+    batch, n = P.shape[0], P.shape[1]
+    Q = torch.empty_like(P)
+    skip = torch.empty(batch, n, dtype=torch.uint8, device=P.device)
+    code = lib.soap_qr_static(n, batch, ctypes.c_void_p(P.data_ptr()), ctypes.c_void_p(Q.data_ptr()),
+                              ctypes.c_void_p(skip.data_ptr()), float(tol), _stream(stream))
+    if code != SOAP_OK:
+        raise SoapError(code, f"soap_qr_static(n={n}, batch={batch}): needs "
+                              f"{lib.soap_qr_workspace_bytes(n, batch)} bytes of workspace; the fixed array "
+                              "holds 32 MiB" if code == 1 else "soap_qr_static failed")
     return Q, skip
 
 
