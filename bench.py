@@ -123,6 +123,32 @@ def measured_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
+# tensor-core fp32 products take 4 tf32 MMAs (hi/lo split of both operands); TF32 runs at
+# half the bf16 rate on this part
+TC_PRODUCTS = 4
+
+
+def roofline(family, st, peaks, peak_src):
+    """Roofline of one kernel family from its CUDA-event time and algorithmic FLOPs/bytes."""
+    secs = st["ms"] / 1e3
+    base = {"kernel": family, "launches": st["launches"], "avg_launch_us": 1e3 * st["ms"] / max(1, st["launches"]),
+            "traffic": None}
+    if family == "gemm_simt":
+        ach = st["flops"] / secs / 1e12
+        return dict(base, bound="alu", achieved=ach, peak=FP32_SIMT_PEAK_TFLOPS, unit="TFLOP/s",
+                    frac=ach / FP32_SIMT_PEAK_TFLOPS,
+                    peak_source="fp32 FMA peak of the CUDA cores, 152 SMs x 128 lanes x 2 x 2.07 GHz")
+    tc_peak = peaks["bf16_tflops"] / 2.0 / TC_PRODUCTS
+    ridge = tc_peak * 1e12 / (peaks["hbm_gbs"] * 1e9)  # FLOP per byte where the two bounds meet
+    if family == "gemm_tc" and st["flops"] / max(1.0, st["bytes"]) >= ridge:
+        ach = st["flops"] / secs / 1e12
+        return dict(base, bound="tensor", achieved=ach, peak=tc_peak, unit="TFLOP/s", frac=ach / tc_peak,
+                    peak_source=f"{peak_src} bf16 dense / 2 (tf32) / {TC_PRODUCTS} (tf32 products per fp32 product)")
+    ach = st["bytes"] / secs / 1e9
+    return dict(base, bound="hbm", achieved=ach, peak=peaks["hbm_gbs"], unit="GB/s", frac=ach / peaks["hbm_gbs"],
+                peak_source=peak_src)
+
+
 def oracle_sample(steps: int, warmup: int):
     """Times the fp64 oracle's SOAP step on Wq (2048x2048) of the block, on the host cores.
     Returns (seconds per sampled step, block steps/s extrapolated by the FLOP model, threads)."""
@@ -260,17 +286,7 @@ def run_soap(args):
     top = max(fams, key=lambda k: fams[k]["ms"])
     st = fams[top]
     launches = sum(v["launches"] for v in fams.values())
-    if top in ("gemm_simt",):
-        achieved = st["flops"] / (st["ms"] / 1e3) / 1e12
-        roof = {"kernel": top, "bound": "alu", "achieved": achieved, "peak": FP32_SIMT_PEAK_TFLOPS,
-                "unit": "TFLOP/s", "frac": achieved / FP32_SIMT_PEAK_TFLOPS,
-                "peak_source": "fp32 FMA peak of the CUDA cores, 152 SMs x 128 lanes x 2 x 2.07 GHz",
-                "traffic": None, "launches": st["launches"], "avg_launch_us": 1e3 * st["ms"] / max(1, st["launches"])}
-    else:
-        achieved = st["bytes"] / (st["ms"] / 1e3) / 1e9
-        roof = {"kernel": top, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "frac": achieved / peaks["hbm_gbs"], "peak_source": peak_src, "traffic": None,
-                "launches": st["launches"], "avg_launch_us": 1e3 * st["ms"] / max(1, st["launches"])}
+    roof = roofline(top, st, peaks, peak_src)
     per, sps, threads, scale = oracle_sample(1, 0)
     line = {
         "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": args.steps,
@@ -281,7 +297,7 @@ def run_soap(args):
                    "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2 (3 GB of optimizer state per step)"},
         "effective_tflops": block_flops * value / world / 1e12,
-        "effective_frac_of_fp32_simt_peak": block_flops * value / world / 1e12 / FP32_SIMT_PEAK_TFLOPS,
+        "effective_frac_of_tensor_fp32_peak": block_flops * value / world / 1e12 / (peaks["bf16_tflops"] / 2.0 / TC_PRODUCTS),
         "model_flop_per_step": block_flops,
         "roofline": roof,
         "kernel_time_share": {k: round(v["ms"] / max(1e-9, sum(x["ms"] for x in fams.values())), 4)

@@ -9,6 +9,8 @@
  *     W, G, m, v are rows x cols ("in x out"); L, Q_L are rows x rows; R, Q_R are
  *     cols x cols.
  *   - Device pointers must be 16-byte aligned and must not alias each other.
+ *   - A preconditioned side must be a multiple of 4 long and at most 8192 (the tensor-core
+ *     products read rows with TMA); identity sides have no such limit.
  *   - Every call that takes a stream only enqueues work on it (no host
  *     synchronisation) unless its comment says otherwise. Streams are
  *     cudaStream_t values passed as soap_stream_t; 0 is the legacy default stream.
@@ -151,7 +153,8 @@ typedef enum {
   SOAP_KERNEL_GEMM_TC = 1,     /* tcgen05 3xTF32 batched GEMM */
   SOAP_KERNEL_QR_PANEL = 2,    /* cluster panel factorisation of the QR */
   SOAP_KERNEL_ELEMENTWISE = 3, /* momentum, Adam, weight update */
-  SOAP_KERNEL_OTHER = 4        /* norms, identity fills */
+  SOAP_KERNEL_OTHER = 4,       /* norms, identity fills */
+  SOAP_KERNEL_QR_UPDATE = 5    /* rank-32 updates of the QR */
 } soap_kernel_family;
 
 typedef struct {
@@ -168,7 +171,7 @@ typedef struct {
 soap_status_t soap_profile_begin(soap_handle h, int64_t max_launches);
 
 /* Synchronises `stream`, stops timing and writes one soap_kernel_stats per family
- * (5 entries) to out[]. *overflow is set to 1 if max_launches was exceeded. */
+ * (6 entries) to out[]. *overflow is set to 1 if max_launches was exceeded. */
 soap_status_t soap_profile_end(soap_handle h, soap_stream_t stream, soap_kernel_stats* out,
                                int32_t* overflow);
 
@@ -190,8 +193,8 @@ soap_status_t soap_qr(int32_t n, int32_t batch, const float* P, float* Q, uint8_
  * not own their device memory at all (a framework's caching pool, or a fixed budget
  * handed out at start-up, owns it). Same arguments and results as soap_qr, without the
  * workspace: it uses a 32 MiB array compiled into libsoap.so, which every GPU that
- * loads the library keeps until the process exits. That is room for one 2048 x 2048
- * matrix or, e.g., seven of 1024 x 1024; a (n, batch) whose soap_qr_workspace_bytes()
+ * loads the library keeps until the process exits. That is room for one 1024 x 1024
+ * matrix or, e.g., four of 512 x 512; a (n, batch) whose soap_qr_workspace_bytes()
  * exceeds 32 MiB - 256 B is refused with SOAP_ERR_INVALID_ARG before anything is
  * enqueued. It never calls cudaMalloc, cudaFree or any allocating routine.
  * The first call on each device looks up the array's device address with that device

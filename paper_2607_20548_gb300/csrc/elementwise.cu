@@ -19,6 +19,17 @@ namespace {
 
 constexpr int kThreads = 256;
 
+// The tensor core reads an fp32 word as tf32 by dropping its 13 low mantissa bits, so
+// an fp32 array serves directly as the "hi" operand. Its lo part is x - trunc(x) (exact
+// in fp32) rounded to the nearest tf32, so that the tensor core's own truncation of it
+// is exact and hi + lo is x to within half a tf32 unit of lo, without bias.
+__device__ __forceinline__ float tf32_trunc(float x) { return __uint_as_float(__float_as_uint(x) & 0xFFFFE000u); }
+__device__ __forceinline__ float lo_part(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x - tf32_trunc(x)));
+  return __uint_as_float(r);
+}
+
 inline int blocks_for(int64_t elems, int batch) {
   int64_t want = (elems / 4 + kThreads - 1) / kThreads;
   if (want < 1) want = 1;
@@ -85,7 +96,7 @@ __global__ void adam_kernel(float* Gp, const float* Mp, float* V, int rows, int 
     if ((sl && sl[i / cols]) || (sr && sr[i % cols])) nv = 0.f;
     bad |= !isfinite(nv);
     gp[i] = nv;
-    if (N_lo) N_lo[(int64_t)b * elems + i] = nv - __uint_as_float(__float_as_uint(nv) & 0xFFFFE000u);
+    if (N_lo) N_lo[(int64_t)b * elems + i] = lo_part(nv);
   }
   if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(status, kStatusNonFinite);
 }
@@ -110,11 +121,6 @@ __global__ void identity_kernel(float* Q, int n) {
     q[i] = (i / n == i % n) ? 1.f : 0.f;
 }
 
-// The tensor core reads an fp32 word as tf32 by dropping its 13 low mantissa bits, so
-// an fp32 array serves directly as the "hi" operand and its lo part is x - trunc(x)
-// (exact in fp32).
-__device__ __forceinline__ float tf32_trunc(float x) { return __uint_as_float(__float_as_uint(x) & 0xFFFFE000u); }
-__device__ __forceinline__ float lo_part(float x) { return x - tf32_trunc(x); }
 
 // One 32 x 32 tile of one matrix per block (32 x 8 threads). Reads G, updates M_hat and
 // writes the tensor-core operands: G (copy) and its lo part, G^T and its lo part, and
@@ -168,7 +174,7 @@ __global__ void basis_split_kernel(const float* Q, float* Q_lo, float* Qt, float
     if (r < n && c < n) {
       const int64_t o = (int64_t)b * nn + (int64_t)r * n + c;
       x = Q[o];
-      Q_lo[o] = lo_part(x);
+      if (Q_lo) Q_lo[o] = lo_part(x);
     }
     tile[i][threadIdx.x] = x;
   }
@@ -184,13 +190,44 @@ __global__ void basis_split_kernel(const float* Q, float* Q_lo, float* Qt, float
   }
 }
 
+// From Q^T and its lo part (one group slice of `batch` n x n bases): a copy of both, and Q
+// with its lo part, 32 x 32 tiles (32 x 8 threads). Any output may be null.
+__global__ void basis_from_qt_kernel(const float* Qt, const float* Qt_lo, float* Qt_out, float* Qt_lo_out, float* Q,
+                                     float* Q_lo, int n) {
+  __shared__ float tile[32][33];
+  const int b = blockIdx.z;
+  const int64_t nn = (int64_t)n * n;
+  const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = r0 + i, c = c0 + threadIdx.x;
+    float x = 0.f;
+    if (r < n && c < n) {
+      const int64_t o = (int64_t)b * nn + (int64_t)r * n + c;
+      x = Qt[o];
+      if (Qt_out) Qt_out[o] = x;
+      if (Qt_lo_out) Qt_lo_out[o] = Qt_lo[o];
+    }
+    tile[i][threadIdx.x] = x;
+  }
+  __syncthreads();
+  if (!Q) return;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int c = c0 + i, r = r0 + threadIdx.x;
+    if (r < n && c < n) {
+      const float x = tile[threadIdx.x][i];
+      const int64_t o = (int64_t)b * nn + (int64_t)c * n + r;
+      Q[o] = x;
+      if (Q_lo) Q_lo[o] = lo_part(x);
+    }
+  }
+}
+
 __global__ void split_kernel(const float* x, float* hi, float* lo, int64_t n) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
     const float v = x[i];
-    const float h = tf32_trunc(v);
-    if (hi) hi[i] = h;
-    lo[i] = v - h;
+    if (hi) hi[i] = tf32_trunc(v);
+    lo[i] = lo_part(v);
   }
 }
 
@@ -213,6 +250,16 @@ cudaError_t basis_split(const float* Q, float* Q_lo, float* Qt, float* Qt_lo, in
   ProfScope prof(kFamElementwise, 2.0 * e, 16.0 * e, s);
   dim3 grid((n + 31) / 32, (n + 31) / 32, batch);
   basis_split_kernel<<<grid, dim3(32, 8), 0, s>>>(Q, Q_lo, Qt, Qt_lo, n);
+  return cudaGetLastError();
+}
+
+cudaError_t basis_from_qt(const float* Qt, const float* Qt_lo, float* Qt_out, float* Qt_lo_out, float* Q, float* Q_lo,
+                          int n, int batch, cudaStream_t s) {
+  if (n <= 0 || batch <= 0) return cudaSuccess;
+  const double e = (double)n * n * batch;
+  ProfScope prof(kFamElementwise, 0.0, (4.0 + (Qt_out ? 4 : 0) + (Qt_lo_out ? 8 : 0) + (Q ? 4 : 0) + (Q_lo ? 4 : 0)) * e, s);
+  dim3 grid((n + 31) / 32, (n + 31) / 32, batch);
+  basis_from_qt_kernel<<<grid, dim3(32, 8), 0, s>>>(Qt, Qt_lo, Qt_out, Qt_lo_out, Q, Q_lo, n);
   return cudaGetLastError();
 }
 

@@ -6,10 +6,12 @@
 // straight into the canonical 128-byte-swizzled K-major shared-memory layout that
 // tcgen05.mma reads. Every operand comes as a pair (hi, lo): the tensor core reads an
 // fp32 word as tf32 by dropping its 13 low mantissa bits, so hi may be the fp32 array
-// itself and lo = x - trunc_tf32(x) (exact); the accumulator (fp32, in TMEM) receives
-//   a_lo b_hi + a_hi b_lo + a_hi b_hi              ("3xTF32")
-// which keeps ~22 bits of each operand: products with fp32 accuracy at tensor-core
-// rate, as the optimizer step's fp32 arithmetic requires.
+// itself, and lo = x - trunc_tf32(x) rounded to the nearest tf32 (read exactly). The
+// accumulator (fp32, in TMEM) receives
+//   a_lo b_lo + a_lo b_hi + a_hi b_lo + a_hi b_hi
+// = (hi + lo)(hi + lo), each operand within 2^-22 of x and without the bias that
+// truncation would leave: products with fp32 accuracy at tensor-core rate, as the
+// optimizer step's fp32 arithmetic requires.
 //
 // The tensor core's own accumulation rounds toward zero at every MMA, so a long chain
 // of MMAs into one accumulator drifts (relative error growing ~linearly in K: 6e-5 at
@@ -46,7 +48,8 @@ struct Cfg {
   static constexpr int TILE_A = BM * BK * 4;
   static constexpr int TILE_B = BN * BK * 4;
   static constexpr int STAGE = 2 * TILE_A + 2 * TILE_B;
-  static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
+  static constexpr int STAGING = 4 * 32 * 33 * 4;  // per epilogue warp: one 32 x 32 block (+pad)
+  static constexpr int SMEM = STAGES * STAGE + STAGING + 1024 + 256;
   static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators, used alternately
   static_assert(SMEM <= 232448, "shared memory budget");
 };
@@ -152,8 +155,14 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// tf32 value the tensor core reads from an fp32 word (13 low mantissa bits dropped).
+// tf32 value the tensor core reads from an fp32 word (13 low mantissa bits dropped), and
+// the lo part x - trunc(x) rounded to the nearest tf32 (so the tensor core reads it exactly).
 __device__ __forceinline__ float tf32_trunc(float x) { return __uint_as_float(__float_as_uint(x) & 0xFFFFE000u); }
+__device__ __forceinline__ float tf32_lo(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x - tf32_trunc(x)));
+  return __uint_as_float(r);
+}
 
 template <int BN, int STAGES>
 __global__ void __launch_bounds__(THREADS, 1)
@@ -163,7 +172,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   using C = Cfg<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE);
+  float* staging = reinterpret_cast<float*>(smem + STAGES * C::STAGE);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE + C::STAGING);
   uint64_t* empty = full + STAGES;
   uint64_t* acc_full = empty + STAGES;  // [2] accumulator a holds a finished K block
   uint64_t* acc_empty = acc_full + 2;   // [2] accumulator a has been drained
@@ -250,7 +260,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int kk = 0; kk < BK / 8; ++kk) {
           const uint32_t off = kk * 32;  // 8 tf32 = 32 bytes along K inside the swizzle row
-          umma_tf32(d, desc_sw128(a_lo + off), desc_sw128(b_hi + off), idesc, kk != 0);
+          umma_tf32(d, desc_sw128(a_lo + off), desc_sw128(b_lo + off), idesc, kk != 0);
+          umma_tf32(d, desc_sw128(a_lo + off), desc_sw128(b_hi + off), idesc, 1u);
           umma_tf32(d, desc_sw128(a_hi + off), desc_sw128(b_lo + off), idesc, 1u);
           umma_tf32(d, desc_sw128(a_hi + off), desc_sw128(b_hi + off), idesc, 1u);
         }
@@ -287,28 +298,54 @@ __global__ void __launch_bounds__(THREADS, 1)
         asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&acc_empty[a])) : "memory");
     }
     if (!valid && lane == 0 && ep.status) atomicOr(ep.status, kStatusTimeout);
-    const int r = m0 + 32 * q + lane;
     float* Cb = ep.C_ptrs ? ep.C_ptrs[b] : (ep.C ? ep.C + (int64_t)b * ep.c_stride : nullptr);
     float* Lb = ep.C_lo ? ep.C_lo + (int64_t)b * ep.lo_stride : nullptr;
-    if (valid && r < M) {
+    const int row0 = m0 + 32 * q;  // first of this warp's 32 rows
+    if (valid && ep.transpose) {
+      // C^T: for a fixed column the 32 lanes (32 consecutive rows) write 128 contiguous bytes
+      const int r = row0 + lane;
 #pragma unroll
       for (int c = 0; c < BN / 32; ++c) {
         const int col0 = n0 + 32 * c;
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
           const int col = col0 + j;
-          if (col >= N) break;
-          const int64_t off = ep.transpose ? (int64_t)col * ep.ldc + r : (int64_t)r * ep.ldc + col;
+          if (col >= N || r >= M) continue;
+          const int64_t off = (int64_t)col * ep.ldc + r;
           float out = ep.alpha * acc[c][j];
           if (Cb) {
             if (ep.beta != 0.f) out = fmaf(ep.beta, Cb[off], out);
             Cb[off] = out;
           }
-          if (Lb) {
-            const int64_t lo_off = ep.transpose ? (int64_t)col * ep.ld_lo + r : (int64_t)r * ep.ld_lo + col;
-            Lb[lo_off] = out - tf32_trunc(out);
+          if (Lb) Lb[(int64_t)col * ep.ld_lo + r] = tf32_lo(out);
+        }
+      }
+    } else if (valid) {
+      // C: each lane holds one row; stage the warp's 32 x 32 block in shared memory so that
+      // every global access instruction covers 32 consecutive columns of one row
+      float* st = staging + q * (32 * 33);
+#pragma unroll
+      for (int c = 0; c < BN / 32; ++c) {
+        const int col0 = n0 + 32 * c;
+        if (col0 >= N) break;  // warp-uniform
+#pragma unroll
+        for (int j = 0; j < 32; ++j) st[lane * 33 + j] = acc[c][j];
+        __syncwarp();
+        const int col = col0 + lane;
+        for (int rr = 0; rr < 32; ++rr) {
+          const int r = row0 + rr;
+          if (r >= M) break;  // warp-uniform
+          if (col < N) {
+            float out = ep.alpha * st[rr * 33 + lane];
+            if (Cb) {
+              const int64_t off = (int64_t)r * ep.ldc + col;
+              if (ep.beta != 0.f) out = fmaf(ep.beta, Cb[off], out);
+              Cb[off] = out;
+            }
+            if (Lb) Lb[(int64_t)r * ep.ld_lo + col] = tf32_lo(out);
           }
         }
+        __syncwarp();
       }
     }
   }
@@ -381,11 +418,12 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
                        cudaStream_t s) {
   if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
   if (batch > 65535 || (M + tc::BM - 1) / tc::BM > 65535) return cudaErrorInvalidValue;
-  const double flops = 3.0 * 2.0 * M * N * (double)K * batch;
+  const double flops = 2.0 * M * N * (double)K * batch;  // algorithmic (4 tf32 products each on the pipe)
   const double bytes = 4.0 * (2.0 * (double)M * K * (A.batch > 0 ? A.batch : batch) +
                               2.0 * (double)N * K * (B.batch > 0 ? B.batch : batch) +
                               (double)M * N * batch * ((ep.beta != 0.f ? 2 : 1) + (ep.C_lo ? 1 : 0)));
-  ProfScope prof(kFamGemmTc, flops / 3.0, bytes, s);
+  ProfScope prof(kFamGemmTc, flops, bytes, s);
+  if (N <= 32) return tc::launch<32, 5>(A, B, M, N, K, batch, ep, s);
   return tc::launch<128, 3>(A, B, M, N, K, batch, ep, s);
 }
 

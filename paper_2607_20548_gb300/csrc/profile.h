@@ -18,7 +18,8 @@ enum KernelFamily : int {
   kFamQrPanel = 2,    // cluster panel factorisation of the QR
   kFamElementwise = 3,// momentum / Adam / weight update
   kFamOther = 4,      // norms, identity fills
-  kNumFamilies = 5,
+  kFamQrUpdate = 5,   // rank-32 updates of the QR (HBM-bound)
+  kNumFamilies = 6,
 };
 
 struct Profiler {

@@ -1,29 +1,36 @@
 // Batched Householder QR with explicit Q for the eigenbasis refresh
 // (Alg. 1, "Eigenbasis Re-computation": Q <- QR(L_t Q).Q, every step as the
-// appendix on eigh vs QR settles), with diag(R) >= 0.
+// appendix on eigh vs QR settles), with diag(R) >= 0, on tensor cores.
 //
-// Blocked right-looking Householder QR (Golub & Van Loan, 4th ed., section 5.2.3):
-//   for each 32-column panel k:
-//     1. factor the panel A[k:n, k:k+32] in shared memory          (qr_panel_kernel)
-//        -> Householder vectors V (written over the panel) and the
-//           compact-WY factor T with H_1...H_32 = I - V T V^T
-//     2. trailing update A[k:, k+32:] <- (I - V T^T V^T) A[k:, k+32:] (three GEMMs)
-//   then Q = H_1 ... H_n I, accumulated backwards one block at a time (three GEMMs
-//   per block).
+// The QR works on At = P^T (row j of At is column j of P), so every product of the
+// blocked algorithm is a C = A B^T of K-major operands: the long reductions run on the
+// tcgen05 engine, the rank-32 updates (HBM-bound) on the CUDA cores:
 //
-// The panel of an n x n matrix has up to n rows; it is spread over a thread-block
-// cluster of ceil((n-k)/1024) CTAs (<= 8 for n <= 8192), 1024 rows each, and the
-// column reductions of each Householder step are combined through distributed
-// shared memory with one cluster barrier per reduction. No CTA waits on a flag:
-// the only waits are hardware cluster barriers that every CTA of the cluster
-// reaches unconditionally.
+//   for each 32-column panel at k (rows k..k+31 of At):
+//     1. qr_panel_kernel factors the panel rows in distributed shared memory and writes
+//        the Householder vectors as rows of Vt (row k+a = v_a over positions k..n-1,
+//        zeros before its pivot), T with H_1..H_32 = I - V T V^T, and V T^T and V T
+//        (positions x 32), each with its tf32 lo part.
+//     2. trailing rows r > k+31 (columns of P): a_r <- a_r - (a_r V) T V^T, i.e.
+//          W1  = At_trail Vt^T                (tensor cores: M = rows, N = 32, K = positions)
+//          At_trail -= W1 (V T^T)^T           (rank-32 update streaming At_trail once)
+//   then Q^T is accumulated backwards from diag(d) (d_j = sign of R_jj) one block at a
+//   time, Q^T <- Q^T (I - V T^T V^T):
+//          W   = Qt_sub Vt^T ;  Qt_sub -= W (V T)^T
+//   and Q = (Q^T)^T is written with its lo part.
+//
+// The panel of an n x n matrix spans up to n positions; it is spread over a thread-block
+// cluster of ceil((n-k)/1024) CTAs (<= 8 for n <= 8192), 1024 positions each, and the
+// reductions of each Householder step are combined through distributed shared memory
+// with one cluster barrier per reduction. No CTA waits on a flag: the only waits are
+// hardware cluster barriers that every CTA of the cluster reaches unconditionally.
 //
 // Reflector convention (LAPACK larfg): for x = A[p:n, p] with alpha = x_1 and
 // sigma = ||x_2:||^2, beta = -sign(alpha) ||x||, v = x / (alpha - beta) with v_1 = 1,
 // tau = (beta - alpha) / beta, so H x = beta e_1 and R_pp = beta; sigma = 0 gives H = I
 // and R_pp = alpha. The sign convention diag(R) >= 0 then negates column p of Q
-// wherever R_pp < 0; it costs nothing because the backward accumulation of Q starts
-// from diag(d_1..d_n), d_p = sign of R_pp, instead of I. A column with
+// wherever R_pp < 0; it costs nothing because the backward accumulation starts from
+// diag(d_1..d_n), d_p = sign of R_pp, instead of I. A column with
 // ||x|| <= tol * ||P||_F is treated as exactly zero: H = I, R_pp = 0, d_p = +1, and the
 // column is flagged in skip[]. (The convention matters beyond the sign: the columns of
 // Q that complete a rank-deficient P are H_1 ... H_p-1 e_p, which depend on it.)
@@ -41,14 +48,27 @@ namespace soap {
 namespace {
 
 constexpr int NB = 32;            // panel width
-constexpr int ROWS = 1024;        // panel rows held by one CTA
+constexpr int COLS = 1024;        // panel positions held by one CTA
 constexpr int PT = 512;           // threads per panel CTA
-constexpr int LDS = ROWS + 1;     // column stride of the shared panel (bank-conflict padding)
+constexpr int LDS = COLS + 1;     // row stride of the shared panel (bank-conflict padding)
 constexpr int MAXC = 8;           // largest cluster (portable limit) -> n <= 8192
 constexpr int NWARP = PT / 32;
 
+// lo part of x for the tensor-core products: x - trunc_tf32(x) rounded to the nearest tf32
+__device__ __forceinline__ float tf32_lo(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x - __uint_as_float(__float_as_uint(x) & 0xFFFFE000u)));
+  return __uint_as_float(r);
+}
+
 struct PanelArgs {
-  float* A;            // [batch][n][n] working matrices
+  float* At;           // [batch][n][n] working P^T
+  float* Vt;           // [batch][n][n] Householder vectors as rows
+  float* Vt_lo;
+  float* VTr;          // [batch][n][NB]   V T^T of this panel (row = position)
+  float* VTr_lo;
+  float* VTq;          // [batch][npanel][n][NB]  V T of every panel
+  float* VTq_lo;
   float* T;            // [batch][npanel][NB][NB]
   uint8_t* skip;       // [batch][n]
   float* dsign;        // [batch][n] sign of R_pp (+1 for zero columns)
@@ -70,7 +90,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   const int b = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
-  extern __shared__ float sA[];  // [NB][LDS], column-major panel slice
+  extern __shared__ float sA[];  // [NB][LDS]: panel row jj (a column of P), position offset i
   __shared__ float s_sig[2][MAXC];
   __shared__ float s_alpha[2];
   __shared__ float s_dot[2][MAXC][NB];
@@ -83,13 +103,14 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   __shared__ float s_T[NB][NB + 1];
 
   const int n = p.n, k = p.k, kb = p.kb;
-  float* A = p.A + (int64_t)b * n * n;
-  const int row0 = k + c * ROWS;
-  const int nrows = max(0, min(ROWS, n - row0));
+  const int64_t nn = (int64_t)n * n;
+  float* At = p.At + (int64_t)b * nn;
+  const int pos0 = k + c * COLS;  // first position held by this CTA
+  const int npos = max(0, min(COLS, n - pos0));
 
-  for (int e = tid; e < nrows * kb; e += PT) {
-    const int i = e / kb, jj = e % kb;
-    sA[jj * LDS + i] = A[(int64_t)(row0 + i) * n + k + jj];
+  for (int e = tid; e < npos * kb; e += PT) {
+    const int jj = e / npos, i = e % npos;
+    sA[jj * LDS + i] = At[(int64_t)(k + jj) * n + pos0 + i];
   }
   __syncthreads();
   const float thresh = p.thresh[b];
@@ -97,10 +118,10 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
 
   for (int j = 0; j < kb; ++j) {
     const int par = j & 1;
-    // rows strictly below the pivot (pivot = local row j of rank 0)
+    // positions strictly after the pivot (pivot = local position j of rank 0)
     const int ibeg = (c == 0) ? j + 1 : 0;
     float s = 0.f;
-    for (int i = ibeg + tid; i < nrows; i += PT) {
+    for (int i = ibeg + tid; i < npos; i += PT) {
       const float x = sA[j * LDS + i];
       s = fmaf(x, x, s);
     }
@@ -139,8 +160,8 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
         scale = true;
       }
     }
-    // v below the pivot: x / v0, or 0 where H = I or x_2: = 0
-    for (int i = ibeg + tid; i < nrows; i += PT) {
+    // v after the pivot: x / v0, or 0 where H = I or x_2: = 0
+    for (int i = ibeg + tid; i < npos; i += PT) {
       float& x = sA[j * LDS + i];
       x = scale ? x / v0 : 0.f;
     }
@@ -151,12 +172,12 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     }
     __syncthreads();
 
-    // apply H_j = I - tau v v^T to the panel columns right of j
+    // apply H_j = I - tau v v^T to the panel rows after j
     if (tau != 0.f && j + 1 < kb) {
-      const int pivot_rows = (c == 0) ? j : 0;  // local rows >= this take part
+      const int piv = (c == 0) ? j : 0;  // local positions >= this take part
       for (int jj = j + 1 + warp; jj < kb; jj += NWARP) {
         float d = 0.f;
-        for (int i = ibeg + lane; i < nrows; i += 32) d = fmaf(sA[j * LDS + i], sA[jj * LDS + i], d);
+        for (int i = ibeg + lane; i < npos; i += 32) d = fmaf(sA[j * LDS + i], sA[jj * LDS + i], d);
         d = warp_sum(d);
         if (c == 0) d += sA[jj * LDS + j];  // v_pivot = 1
         if (lane < C) cluster.map_shared_rank(&s_dot[par][0][0], lane)[c * NB + jj] = d;
@@ -168,7 +189,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
         s_dtot[tid] = d;
       }
       __syncthreads();
-      for (int i = pivot_rows + tid; i < nrows; i += PT) {
+      for (int i = piv + tid; i < npos; i += PT) {
         const float vi = (c == 0 && i == j) ? 1.f : sA[j * LDS + i];
         const float tv = tau * vi;
         for (int jj = j + 1; jj < kb; ++jj) sA[jj * LDS + i] = fmaf(-tv, s_dtot[jj], sA[jj * LDS + i]);
@@ -177,7 +198,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     }
   }
 
-  // V with its unit diagonal and zeros above it (rank 0 holds the top kb rows)
+  // V with its unit diagonal and zeros before it (rank 0 holds the first kb positions)
   if (c == 0) {
     for (int e = tid; e < kb * kb; e += PT) {
       const int jj = e / kb, i = e % kb;
@@ -186,53 +207,174 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     }
   }
   __syncthreads();
-  for (int e = tid; e < nrows * kb; e += PT) {
-    const int i = e / kb, jj = e % kb;
-    A[(int64_t)(row0 + i) * n + k + jj] = sA[jj * LDS + i];
+  float* Vt = p.Vt + (int64_t)b * nn;
+  float* Vt_lo = p.Vt_lo + (int64_t)b * nn;
+  for (int e = tid; e < npos * kb; e += PT) {
+    const int jj = e / npos, i = e % npos;
+    const float v = sA[jj * LDS + i];
+    const int64_t o = (int64_t)(k + jj) * n + pos0 + i;
+    Vt[o] = v;
+    Vt_lo[o] = tf32_lo(v);
   }
 
-  // partial Gram V^T V of this CTA's rows, gathered in rank 0
+  // partial Gram V^T V over this CTA's positions, gathered in rank 0
   for (int pr = warp; pr < kb * kb; pr += NWARP) {
     const int a = pr / kb, bb = pr % kb;
     if (bb < a) continue;
     float g = 0.f;
-    for (int i = lane; i < nrows; i += 32) g = fmaf(sA[a * LDS + i], sA[bb * LDS + i], g);
+    for (int i = lane; i < npos; i += 32) g = fmaf(sA[a * LDS + i], sA[bb * LDS + i], g);
     g = warp_sum(g);
     if (lane == 0) cluster.map_shared_rank(&s_gram[0][0][0], 0)[(c * NB + a) * NB + bb] = g;
   }
   if (nonfinite && tid == 0) atomicOr(p.status, kStatusQrBreakdown);
   cluster.sync();
-  if (c != 0) return;
 
-  // T: T_jj = tau_j, T(0:j, j) = -tau_j T(0:j, 0:j) (V(:,0:j)^T v_j)   (LAPACK larft, forward)
-  for (int j = 0; j < kb; ++j) {
-    if (tid < kb) {
-      const int i = tid;
-      float t = 0.f;
-      if (i < j) {
-        float acc = 0.f;
-        for (int l = i; l < j; ++l) {
-          float g = 0.f;
-          for (int q = 0; q < C; ++q) g += s_gram[q][l][j];
-          acc = fmaf(s_T[i][l], g, acc);
-        }
-        t = -s_tau[j] * acc;
-      } else if (i == j) {
-        t = s_tau[j];
-      }
-      s_T[i][j] = t;
+  if (c == 0) {
+    // sum the partial Grams once, then T: T_jj = tau_j, T(0:j, j) = -tau_j T(0:j, 0:j) g(0:j, j)
+    for (int e = tid; e < kb * kb; e += PT) {
+      const int l = e / kb, jj = e % kb;
+      float g = 0.f;
+      if (l < jj)
+        for (int q = 0; q < C; ++q) g += s_gram[q][l][jj];
+      s_gram[0][l][jj] = g;  // only (l < jj) entries are read below
     }
     __syncthreads();
+    for (int j = 0; j < kb; ++j) {
+      if (tid < kb) {
+        const int i = tid;
+        float t = 0.f;
+        if (i < j) {
+          float acc = 0.f;
+          for (int l = i; l < j; ++l) acc = fmaf(s_T[i][l], s_gram[0][l][j], acc);
+          t = -s_tau[j] * acc;
+        } else if (i == j) {
+          t = s_tau[j];
+        }
+        s_T[i][j] = t;
+      }
+      __syncthreads();
+    }
+    // hand T to every CTA of the cluster
+    for (int q = 1; q < C; ++q) {
+      float* dst = cluster.map_shared_rank(&s_T[0][0], q);
+      for (int e = tid; e < NB * (NB + 1); e += PT) dst[e] = (&s_T[0][0])[e];
+    }
+    float* Tout = p.T + ((int64_t)b * p.npanel + p.panel) * NB * NB;
+    for (int e = tid; e < NB * NB; e += PT) {
+      const int i = e / NB, jj = e % NB;
+      Tout[e] = (i < kb && jj < kb) ? s_T[i][jj] : 0.f;
+    }
+    if (tid < kb) {
+      p.skip[(int64_t)b * n + k + tid] = (uint8_t)s_skip[tid];
+      p.dsign[(int64_t)b * n + k + tid] = s_dsign[tid];
+    }
   }
-  float* Tout = p.T + ((int64_t)b * p.npanel + p.panel) * NB * NB;
-  for (int e = tid; e < NB * NB; e += PT) {
-    const int i = e / NB, jj = e % NB;
-    Tout[e] = (i < kb && jj < kb) ? s_T[i][jj] : 0.f;
+  cluster.sync();
+
+  // V T^T (for this panel's trailing update) and V T (for the Q accumulation), position-major:
+  // warp w takes 32 positions at a time, lane a computes output column a (coalesced rows of 32)
+  float* VTr = p.VTr + (int64_t)b * n * NB;
+  float* VTr_lo = p.VTr_lo + (int64_t)b * n * NB;
+  float* VTq = p.VTq + ((int64_t)b * p.npanel + p.panel) * n * NB;
+  float* VTq_lo = p.VTq_lo + ((int64_t)b * p.npanel + p.panel) * n * NB;
+  const int a = lane;
+  for (int i0 = warp * 32; i0 < npos; i0 += NWARP * 32) {
+    const int iend = min(i0 + 32, npos);
+    for (int i = i0; i < iend; ++i) {
+      float r = 0.f, q = 0.f;
+      for (int bb = 0; bb < kb; ++bb) {
+        const float v = sA[bb * LDS + i];
+        r = fmaf((a < kb) ? s_T[a][bb] : 0.f, v, r);
+        q = fmaf((a < kb) ? s_T[bb][a] : 0.f, v, q);
+      }
+      const int64_t o = (int64_t)(pos0 + i) * NB + a;
+      VTr[o] = r;
+      VTr_lo[o] = tf32_lo(r);
+      VTq[o] = q;
+      VTq_lo[o] = tf32_lo(q);
+    }
   }
-  if (tid < kb) {
-    p.skip[(int64_t)b * n + k + tid] = (uint8_t)s_skip[tid];
-    p.dsign[(int64_t)b * n + k + tid] = s_dsign[tid];
+}
+
+// Rank-32 update C_b <- C_b - A_b B_b^T (A: M x K, B: N x K, K <= 32, all row-major) with
+// the lo part of the result, in exact fp32 FMAs. It streams C once (read, write, lo write;
+// 32 FMAs per element), so it is bound by HBM, not by a matrix unit: each thread issues its
+// 32 loads of C before any arithmetic, and two 256-thread CTAs share an SM.
+// Tile 64 x 128: warp w owns rows 8w..8w+7, lane l columns l, l+32, l+64, l+96.
+constexpr int RU_BM = 64, RU_BN = 128;
+
+__global__ void __launch_bounds__(256, 2)
+    rank_update_kernel(int M, int N, int K, const float* __restrict__ A, int64_t lda, int64_t sa,
+                       const float* __restrict__ B, int64_t ldb, int64_t sb, float* C, float* C_lo, int64_t ldc,
+                       int64_t sc) {
+  __shared__ float As[NB][RU_BM + 1];  // [k][row]
+  __shared__ float Bs[NB][RU_BN + 1];  // [k][col]
+  const int b = blockIdx.z;
+  const int r0 = blockIdx.y * RU_BM, c0 = blockIdx.x * RU_BN;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  const float* Ab = A + (int64_t)b * sa;
+  const float* Bb = B + (int64_t)b * sb;
+  float* Cb = C + (int64_t)b * sc;
+  float* Lb = C_lo + (int64_t)b * sc;
+  // C first: 32 independent loads per thread in flight
+  float cv[8][4];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int r = r0 + 8 * w + i;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int col = c0 + lane + 32 * j;
+      cv[i][j] = (r < M && col < N) ? Cb[(int64_t)r * ldc + col] : 0.f;
+    }
   }
+  for (int e = tid; e < RU_BM * NB; e += 256) {
+    const int r = e / NB, kk = e % NB;
+    As[kk][r] = (r0 + r < M && kk < K) ? Ab[(int64_t)(r0 + r) * lda + kk] : 0.f;
+  }
+  for (int e = tid; e < RU_BN * NB; e += 256) {
+    const int cc = e / NB, kk = e % NB;
+    Bs[kk][cc] = (c0 + cc < N && kk < K) ? Bb[(int64_t)(c0 + cc) * ldb + kk] : 0.f;
+  }
+  __syncthreads();
+  float acc[8][4];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+#pragma unroll 8
+  for (int kk = 0; kk < NB; ++kk) {
+    float a[8], bv[4];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a[i] = As[kk][8 * w + i];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) bv[j] = Bs[kk][lane + 32 * j];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], bv[j], acc[i][j]);
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int r = r0 + 8 * w + i;
+    if (r >= M) break;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int col = c0 + lane + 32 * j;
+      if (col >= N) continue;
+      const float out = cv[i][j] - acc[i][j];
+      Cb[(int64_t)r * ldc + col] = out;
+      Lb[(int64_t)r * ldc + col] = tf32_lo(out);
+    }
+  }
+}
+
+cudaError_t rank_update(int M, int N, int K, int batch, const float* A, int64_t lda, int64_t sa, const float* B,
+                        int64_t ldb, int64_t sb, float* C, float* C_lo, int64_t ldc, int64_t sc, cudaStream_t s) {
+  if (M <= 0 || N <= 0) return cudaSuccess;
+  ProfScope prof(kFamQrUpdate, 2.0 * M * N * (double)K * batch, 12.0 * M * (double)N * batch, s);
+  dim3 grid((N + RU_BN - 1) / RU_BN, (M + RU_BM - 1) / RU_BM, batch);
+  rank_update_kernel<<<grid, 256, 0, s>>>(M, N, K, A, lda, sa, B, ldb, sb, C, C_lo, ldc, sc);
+  return cudaGetLastError();
 }
 
 // ||P_b||_F: per-chunk partial sums in double, then tol * sqrt(sum)
@@ -263,22 +405,54 @@ __global__ void thresh_kernel(const double* part, float tol, int batch, float* t
   thresh[b] = (float)((double)tol * sqrt(s));
 }
 
-__global__ void signed_identity_kernel(float* Q, const float* d, int n) {
+// Q^T <- diag(d) (its lo part is zero: +-1 are tf32 values)
+__global__ void signed_identity_kernel(float* Qt, float* Qt_lo, const float* d, int n) {
   const int b = blockIdx.y;
-  float* q = Q + (int64_t)b * n * n;
-  const float* db = d + (int64_t)b * n;
   const int64_t nn = (int64_t)n * n;
+  float* q = Qt + (int64_t)b * nn;
+  float* ql = Qt_lo + (int64_t)b * nn;
+  const float* db = d + (int64_t)b * n;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nn; i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = i / n, c = i % n;
-    q[i] = r == c ? db[r] : 0.f;
+    const int64_t r = i / n, cc = i % n;
+    q[i] = r == cc ? db[r] : 0.f;
+    ql[i] = 0.f;
+  }
+}
+
+// Q = (Q^T)^T and its lo part, 32 x 32 tiles through shared memory
+__global__ void transpose_out_kernel(const float* Qt, float* Q, float* Q_lo, int n) {
+  __shared__ float tile[32][33];
+  const int b = blockIdx.z;
+  const int64_t nn = (int64_t)n * n;
+  const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = r0 + i, cc = c0 + threadIdx.x;
+    tile[i][threadIdx.x] = (r < n && cc < n) ? Qt[(int64_t)b * nn + (int64_t)r * n + cc] : 0.f;
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = c0 + i, cc = r0 + threadIdx.x;
+    if (r < n && cc < n) {
+      const float x = tile[threadIdx.x][i];
+      const int64_t o = (int64_t)b * nn + (int64_t)r * n + cc;
+      Q[o] = x;
+      if (Q_lo) Q_lo[o] = tf32_lo(x);
+    }
   }
 }
 
 struct Workspace {
-  float* A;
+  float* At;
+  float* At_lo;
+  float* Vt;
+  float* Vt_lo;
+  float* VTq;
+  float* VTq_lo;
+  float* VTr;
+  float* VTr_lo;
+  float* W;
+  float* W_lo;
   float* T;
-  float* W1;
-  float* W2;
   float* thresh;
   float* dsign;
   double* part;
@@ -294,17 +468,29 @@ Workspace carve(void* base, int n, int batch, size_t* total) {
     off += align256(bytes);
     return o;
   };
-  const size_t oA = take((size_t)batch * n * n * sizeof(float));
+  const size_t mat = (size_t)batch * n * n * sizeof(float);
+  const size_t pan = (size_t)batch * npanel * n * NB * sizeof(float);
+  const size_t thin = (size_t)batch * n * NB * sizeof(float);
+  const size_t oAt = take(mat), oAtl = take(mat), oVt = take(mat), oVtl = take(mat);
+  const size_t oVq = take(pan), oVql = take(pan), oVr = take(thin), oVrl = take(thin);
+  const size_t oW = take(thin), oWl = take(thin);
   const size_t oT = take((size_t)batch * npanel * NB * NB * sizeof(float));
-  const size_t oW1 = take((size_t)batch * NB * n * sizeof(float));
-  const size_t oW2 = take((size_t)batch * NB * n * sizeof(float));
   const size_t oth = take((size_t)batch * sizeof(float));
   const size_t osg = take((size_t)batch * n * sizeof(float));
   const size_t opart = take((size_t)batch * NORM_CHUNKS * sizeof(double));
   if (total) *total = off;
   char* c = (char*)base;
-  return Workspace{(float*)(c + oA), (float*)(c + oT), (float*)(c + oW1), (float*)(c + oW2),
-                   (float*)(c + oth), (float*)(c + osg), (double*)(c + opart)};
+  auto f = [&](size_t o) { return (float*)(c + o); };
+  return Workspace{f(oAt), f(oAtl), f(oVt), f(oVtl), f(oVq), f(oVql), f(oVr), f(oVrl),
+                   f(oW),  f(oWl),  f(oT),  f(oth),  f(osg), (double*)(c + opart)};
+}
+
+TcOperand op(const float* hi, const float* lo, int64_t ld, int64_t stride, int batch) {
+  return TcOperand{hi, lo, ld, stride, batch};
+}
+
+TcEpilogue out(float* C, float* C_lo, int64_t ldc, int64_t stride, float alpha, float beta, int* status) {
+  return TcEpilogue{C, nullptr, ldc, stride, C_lo, ldc, stride, 0, alpha, beta, status};
 }
 
 }  // namespace
@@ -315,38 +501,45 @@ size_t qr_workspace_bytes(int n, int batch) {
   return total;
 }
 
-cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, float tol,
-                 void* workspace, size_t workspace_bytes, int* status, cudaStream_t s) {
+void qr_input_buffers(void* workspace, int n, int batch, float** At, float** At_lo) {
+  Workspace w = carve(workspace, n, batch, nullptr);
+  *At = w.At;
+  *At_lo = w.At_lo;
+}
+
+cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q_lo, uint8_t* skip, float tol,
+                   void* workspace, size_t workspace_bytes, int* status, cudaStream_t s) {
   if (n <= 0 || batch <= 0) return cudaSuccess;
-  if (n > MAXC * ROWS || batch > 65535) return cudaErrorInvalidValue;
+  if (n > MAXC * COLS || batch > 65535 || (n & 3)) return cudaErrorInvalidValue;
   size_t need = 0;
   Workspace w = carve(workspace, n, batch, &need);
   if (workspace_bytes < need) return cudaErrorInvalidValue;
+  if (!Qt) {  // the Q accumulation may reuse the factored matrix's buffers
+    Qt = w.At;
+    Qt_lo = w.At_lo;
+  }
   const int npanel = (n + NB - 1) / NB;
   const int64_t nn = (int64_t)n * n;
   cudaError_t e;
 
-  if (P != w.A) {
-    e = cudaMemcpyAsync(w.A, P, (size_t)batch * nn * sizeof(float), cudaMemcpyDeviceToDevice, s);
-    if (e != cudaSuccess) return e;
-  }
   {
     ProfScope prof(kFamOther, 2.0 * nn * batch, 4.0 * nn * batch, s);
-    frob_partial_kernel<<<dim3(NORM_CHUNKS, batch), 256, 0, s>>>(w.A, nn, w.part);
+    frob_partial_kernel<<<dim3(NORM_CHUNKS, batch), 256, 0, s>>>(w.At, nn, w.part);
   }
   {
     ProfScope prof(kFamOther, 0, 8.0 * NORM_CHUNKS * batch, s);
     thresh_kernel<<<(batch + 127) / 128, 128, 0, s>>>(w.part, tol, batch, w.thresh);
   }
-
   const size_t smem = (size_t)NB * LDS * sizeof(float);
   e = cudaFuncSetAttribute(qr_panel_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
 
+  const int64_t pan_stride = (int64_t)npanel * n * NB;
   for (int pi = 0; pi < npanel; ++pi) {
-    const int k = pi * NB, kb = min(NB, n - k);
-    const int C = (n - k + ROWS - 1) / ROWS;
-    PanelArgs a{w.A, w.T, skip, w.dsign, w.thresh, status, n, k, kb, pi, npanel};
+    const int k = pi * NB, kb = std::min(NB, n - k);
+    const int C = (n - k + COLS - 1) / COLS;
+    PanelArgs a{w.At, w.Vt, w.Vt_lo, w.VTr, w.VTr_lo, w.VTq, w.VTq_lo, w.T, skip, w.dsign, w.thresh, status,
+                n, k, kb, pi, npanel};
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(C, batch, 1);
     cfg.blockDim = dim3(PT, 1, 1);
@@ -360,55 +553,69 @@ cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, floa
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     {
-      // Householder work on the (n-k) x kb panel: ~4 (n-k) kb^2 flops, panel read + written
-      ProfScope prof(kFamQrPanel, 4.0 * (n - k) * kb * kb * batch, 8.0 * (n - k) * kb * batch, s);
+      // Householder work on the kb x (n-k) panel plus V T^T and V T: ~(4 kb^2 + 4 kb^2) (n-k)
+      ProfScope prof(kFamQrPanel, 8.0 * (n - k) * kb * kb * batch, 24.0 * (n - k) * kb * batch, s);
       e = cudaLaunchKernelEx(&cfg, qr_panel_kernel, a);
     }
     if (e != cudaSuccess) return e;
 
-    const int nc = n - k - kb;
+    const int nc = n - k - kb;  // trailing rows of At (columns of P)
     if (nc <= 0) continue;
-    const int m = n - k;
-    Operand V = strided(w.A, n, nn, (int64_t)k * n + k);
-    Operand Cin = strided(w.A, n, nn, (int64_t)k * n + k + kb);
-    MutOperand Cout = strided_mut(w.A, n, nn, (int64_t)k * n + k + kb);
-    Operand Tp = strided(w.T, NB, (int64_t)npanel * NB * NB, (int64_t)pi * NB * NB);
-    // W1 = V^T C  (kb x nc)
-    e = gemm(true, false, kb, nc, m, 1.f, V, Cin, 0.f, strided_mut(w.W1, n, (int64_t)NB * n), batch, s);
+    const int m = n - k;        // positions from the panel's first pivot on
+    const int64_t tr = (int64_t)(k + kb) * n + k;
+    // W1 = At_trail Vt^T   (nc x kb)
+    e = gemm_tc_nt(nc, kb, m, batch, op(w.At + tr, w.At_lo + tr, n, nn, batch),
+                   op(w.Vt + (int64_t)k * n + k, w.Vt_lo + (int64_t)k * n + k, n, nn, batch),
+                   out(w.W, w.W_lo, NB, (int64_t)n * NB, 1.f, 0.f, status), s);
     if (e != cudaSuccess) return e;
-    // W2 = T^T W1
-    e = gemm(true, false, kb, nc, kb, 1.f, Tp, strided(w.W1, n, (int64_t)NB * n), 0.f,
-             strided_mut(w.W2, n, (int64_t)NB * n), batch, s);
-    if (e != cudaSuccess) return e;
-    // C -= V W2
-    e = gemm(false, false, m, nc, kb, -1.f, V, strided(w.W2, n, (int64_t)NB * n), 1.f, Cout, batch, s);
+    // At_trail -= W1 (V T^T)^T
+    e = rank_update(nc, m, kb, batch, w.W, NB, (int64_t)n * NB, w.VTr + (int64_t)k * NB, NB, (int64_t)n * NB,
+                    w.At + tr, w.At_lo + tr, n, nn, s);
     if (e != cudaSuccess) return e;
   }
 
   {
-    // Q = H_1 ... H_n diag(d): start the backward accumulation from diag(d)
-    ProfScope prof(kFamOther, 0, 4.0 * nn * batch, s);
+    // Q^T = diag(d) H_n ... H_1 accumulated backwards: start from diag(d)
+    ProfScope prof(kFamOther, 0, 8.0 * nn * batch, s);
     const int blocks = (int)std::min<int64_t>((nn + 255) / 256, 1024);
-    signed_identity_kernel<<<dim3(blocks, batch), 256, 0, s>>>(Q, w.dsign, n);
+    signed_identity_kernel<<<dim3(blocks, batch), 256, 0, s>>>(Qt, Qt_lo, w.dsign, n);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
   for (int pi = npanel - 1; pi >= 0; --pi) {
-    const int k = pi * NB, kb = min(NB, n - k), m = n - k;
-    Operand V = strided(w.A, n, nn, (int64_t)k * n + k);
-    Operand Qs = strided(Q, n, nn, (int64_t)k * n + k);
-    MutOperand Qo = strided_mut(Q, n, nn, (int64_t)k * n + k);
-    Operand Tp = strided(w.T, NB, (int64_t)npanel * NB * NB, (int64_t)pi * NB * NB);
-    // W1 = V^T Q[k:, k:]; W2 = T W1; Q[k:, k:] -= V W2
-    e = gemm(true, false, kb, m, m, 1.f, V, Qs, 0.f, strided_mut(w.W1, n, (int64_t)NB * n), batch, s);
+    const int k = pi * NB, kb = std::min(NB, n - k), m = n - k;
+    const int64_t sub = (int64_t)k * n + k;
+    // W = Qt_sub Vt^T  (m x kb)
+    e = gemm_tc_nt(m, kb, m, batch, op(Qt + sub, Qt_lo + sub, n, nn, batch),
+                   op(w.Vt + sub, w.Vt_lo + sub, n, nn, batch), out(w.W, w.W_lo, NB, (int64_t)n * NB, 1.f, 0.f, status),
+                   s);
     if (e != cudaSuccess) return e;
-    e = gemm(false, false, kb, m, kb, 1.f, Tp, strided(w.W1, n, (int64_t)NB * n), 0.f,
-             strided_mut(w.W2, n, (int64_t)NB * n), batch, s);
+    // Qt_sub -= W (V T)^T
+    const int64_t vq = (int64_t)pi * n * NB + (int64_t)k * NB;
+    e = rank_update(m, m, kb, batch, w.W, NB, (int64_t)n * NB, w.VTq + vq, NB, pan_stride, Qt + sub, Qt_lo + sub, n,
+                    nn, s);
     if (e != cudaSuccess) return e;
-    e = gemm(false, false, m, m, kb, -1.f, V, strided(w.W2, n, (int64_t)NB * n), 1.f, Qo, batch, s);
+  }
+  if (Q) {
+    ProfScope prof(kFamOther, 0, 12.0 * nn * batch, s);
+    dim3 grid((n + 31) / 32, (n + 31) / 32, batch);
+    transpose_out_kernel<<<grid, dim3(32, 8), 0, s>>>(Qt, Q, Q_lo, n);
+    e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
+}
+
+cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, float tol, void* workspace,
+                 size_t workspace_bytes, int* status, cudaStream_t s) {
+  if (n <= 0 || batch <= 0) return cudaSuccess;
+  size_t need = 0;
+  Workspace w = carve(workspace, n, batch, &need);
+  if (workspace_bytes < need || (n & 3)) return cudaErrorInvalidValue;
+  // At = P^T and its lo part
+  cudaError_t e = basis_split(P, nullptr, w.At, w.At_lo, n, batch, s);
+  if (e != cudaSuccess) return e;
+  return qr_q_t(n, batch, nullptr, nullptr, Q, nullptr, skip, tol, workspace, workspace_bytes, status, s);
 }
 
 }  // namespace soap

@@ -14,9 +14,9 @@
 
 namespace {
 
-// 32 MiB: room for the workspace of one 2048 x 2048 matrix (about 17 MB) or of several
-// smaller ones (e.g. 7 of 1024 x 1024). Every GPU that loads the library keeps this
-// array until the process exits.
+// 32 MiB: room for the workspace of one 1024 x 1024 matrix (about 25 MB) or of several
+// smaller ones (e.g. 4 of 512 x 512). Every GPU that loads the library keeps this array
+// until the process exits.
 constexpr size_t kScratchBytes = size_t(32) << 20;
 __device__ __align__(256) unsigned char g_qr_scratch[kScratchBytes];
 
@@ -29,7 +29,7 @@ void* g_scratch_addr[kMaxDevices] = {};
 
 extern "C" soap_status_t soap_qr_static(int32_t n, int32_t batch, const float* P, float* Q, uint8_t* skip,
                                         float tol, soap_stream_t stream) {
-  if (n <= 0 || n > 8192 || batch <= 0 || batch > 65535 || !P || !Q || !skip || !(tol >= 0.f))
+  if (n <= 0 || n > 8192 || (n & 3) || batch <= 0 || batch > 65535 || !P || !Q || !skip || !(tol >= 0.f))
     return SOAP_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(P) | reinterpret_cast<uintptr_t>(Q)) & 15) return SOAP_ERR_INVALID_ARG;
   const size_t qb = soap::qr_workspace_bytes(n, batch);

@@ -57,6 +57,25 @@ struct ClassState {
   bool basis_dirty = true;  // Q^T and lo parts must be rebuilt from Q before use
 };
 
+// One preconditioned side of one class: `count` factors of size n in a QR group.
+struct QrJob {
+  int cls;
+  bool left;
+  int offset;  // first batch index of this job inside its group
+};
+
+// All factors of one size, refreshed by one batched QR on their own stream.
+struct QrGroup {
+  int n = 0;
+  int batch = 0;
+  std::vector<QrJob> jobs;
+  void* ws = nullptr;
+  size_t ws_bytes = 0;
+  uint8_t* skip = nullptr;  // [batch][n]
+  cudaStream_t stream = nullptr;
+  cudaEvent_t done = nullptr;
+};
+
 struct DeviceGuard {
   int prev = -1;
   explicit DeviceGuard(int dev) {
@@ -88,8 +107,8 @@ struct soap_s {
   float* N_lo = nullptr;
   float* Zt = nullptr;   // (N Q_R^T)^T
   float* Zt_lo = nullptr;
-  void* qr_ws = nullptr;
-  size_t qr_ws_bytes = 0;
+  std::vector<QrGroup> groups;  // largest n first
+  cudaEvent_t fork_ev = nullptr;
   int* d_status = nullptr;
   int* h_status = nullptr;          // pinned mirror, refreshed after every step
   cudaEvent_t status_ev = nullptr;
@@ -150,6 +169,14 @@ void free_all(soap_handle h) {
   if (h->h_ptrs) cudaFreeHost(h->h_ptrs);
   if (h->status_ev) cudaEventDestroy(h->status_ev);
   if (h->stage_ev) cudaEventDestroy(h->stage_ev);
+  if (h->fork_ev) cudaEventDestroy(h->fork_ev);
+  h->fork_ev = nullptr;
+  for (auto& g : h->groups) {
+    if (g.stream) cudaStreamDestroy(g.stream);
+    if (g.done) cudaEventDestroy(g.done);
+    g.stream = nullptr;
+    g.done = nullptr;
+  }
   h->h_status = nullptr;
   h->h_ptrs = nullptr;
   h->status_ev = h->stage_ev = nullptr;
@@ -166,59 +193,171 @@ soap::TcEpilogue epi(soap_handle h, float* C, int64_t ldc, int64_t c_stride, flo
   return soap::TcEpilogue{C, nullptr, ldc, c_stride, C_lo, ldc, c_stride, transpose, alpha, beta, h->d_status};
 }
 
-// One step of a two-sided class with every contraction as a tcgen05 3xTF32 product
-// C = A B^T of K-major operands:
+// A class's step in three phases, so that the QR refreshes of all classes can be batched by size:
+//   A  operand preparation and S1 (per class, caller's stream)
+//   B  S2 + S3 for every preconditioned side, one batched QR per size group (refresh_bases)
+//   C  S5-S8: rotations, Adam in the basis, back-rotation and update (per class)
+//
+// Two-sided classes run every contraction as a tcgen05 product C = A B^T of K-major operands:
 //   S1  L <- b L + (1-b) G G^T       A = G,     B = G
 //       R <- b R + (1-b) G^T G       A = G^T,   B = G^T
-//   S2  P = L Q_L                    A = L,     B = Q_L^T    -> QR -> Q_L, Q_L^T
+//   S2  P^T = Q_L^T L                A = Q_L^T, B = L (symmetric)  -> QR -> Q_L, Q_L^T
 //   S5  Y^T = ([G | M_hat] Q_R)^T    A = [G|M], B = Q_R^T    (transposed epilogue)
 //       [G' | m'] = Q_L^T Y          A = Q_L^T, B = Y^T
 //   S6  N = Adam(G', m', v)
 //   S7  Z^T = (N Q_R^T)^T            A = N,     B = Q_R      (transposed epilogue)
 //   S8  W <- (1 - lr wd) W - lr Q_L Z  A = Q_L, B = Z^T      (epilogue into W)
-soap_status_t step_tensor_core(soap_handle h, ClassState& c, float* const* d_params, const float* const* d_grads,
-                               bool refresh, float bc1, float bc2, cudaStream_t s) {
+soap_status_t prepare_class(soap_handle h, ClassState& c, const float* const* d_grads, cudaStream_t s) {
   const soap_hparams& hp = h->hp;
   const int B = c.count, m = (int)c.rows, n = (int)c.cols;
   const int64_t mn = (int64_t)m * n, mm = (int64_t)m * m, nn = (int64_t)n * n;
+  const float fb = hp.factor_beta;
+  using soap::strided;
+  using soap::strided_mut;
+  if (!c.tc) {
+    SOAP_CUDA(h, soap::momentum_and_copy(d_grads, c.Gc, c.Mhat, mn, B, hp.beta1, h->d_status, s));
+    if (c.left)  // S1: L <- b L + (1-b) G G^T
+      SOAP_CUDA(h, soap::gemm(false, true, m, m, n, 1.f - fb, strided(c.Gc, n, mn), strided(c.Gc, n, mn), fb,
+                              strided_mut(c.L, m, mm), B, s));
+    if (c.right)  // S1: R <- b R + (1-b) G^T G
+      SOAP_CUDA(h, soap::gemm(true, false, n, n, m, 1.f - fb, strided(c.Gc, n, mn), strided(c.Gc, n, mn), fb,
+                              strided_mut(c.R, n, nn), B, s));
+    return SOAP_OK;
+  }
   const int64_t cls = (int64_t)B * mn;
-  float* GM = c.Gc;
-  SOAP_CUDA(h, soap::momentum_split(d_grads, GM, c.GM_lo, c.Gt, c.Gt_lo, c.Mhat, c.GM_lo + cls, m, n, B, hp.beta1,
+  SOAP_CUDA(h, soap::momentum_split(d_grads, c.Gc, c.GM_lo, c.Gt, c.Gt_lo, c.Mhat, c.GM_lo + cls, m, n, B, hp.beta1,
                                     h->d_status, s));
   if (c.basis_dirty) {
     SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, B, s));
     SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, n, B, s));
     c.basis_dirty = false;
   }
-  const float fb = hp.factor_beta;
-  SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(GM, c.GM_lo, n, mn, B), opnd(GM, c.GM_lo, n, mn, B),
+  SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(c.Gc, c.GM_lo, n, mn, B), opnd(c.Gc, c.GM_lo, n, mn, B),
                                 epi(h, c.L, m, mm, c.L_lo, 0, 1.f - fb, fb), s));
   SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(c.Gt, c.Gt_lo, m, mn, B), opnd(c.Gt, c.Gt_lo, m, mn, B),
                                 epi(h, c.R, n, nn, c.R_lo, 0, 1.f - fb, fb), s));
-  if (refresh) {
-    float* P = (float*)h->qr_ws;  // the QR factors its workspace's first matrix block in place
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, m, m, B, opnd(c.L, c.L_lo, m, mm, B), opnd(c.QLt, c.QLt_lo, m, mm, B),
-                                  epi(h, P, m, mm, nullptr, 0, 1.f, 0.f), s));
-    SOAP_CUDA(h, soap::qr_q(m, B, P, c.QL, c.skipL, hp.qr_tol, h->qr_ws, h->qr_ws_bytes, h->d_status, s));
-    SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, B, s));
-    SOAP_CUDA(h, soap::gemm_tc_nt(n, n, n, B, opnd(c.R, c.R_lo, n, nn, B), opnd(c.QRt, c.QRt_lo, n, nn, B),
-                                  epi(h, P, n, nn, nullptr, 0, 1.f, 0.f), s));
-    SOAP_CUDA(h, soap::qr_q(n, B, P, c.QR, c.skipR, hp.qr_tol, h->qr_ws, h->qr_ws_bytes, h->d_status, s));
-    SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, n, B, s));
+  return SOAP_OK;
+}
+
+// S2 + S3 for every preconditioned side: per size group, P^T = Q^T F for each member (F the
+// factor, symmetric) into one batched input, one QR, then Q^T, Q (and lo parts) and the
+// zero-column flags back to the classes. Groups run concurrently on their own streams.
+soap_status_t refresh_bases(soap_handle h, cudaStream_t s) {
+  const soap_hparams& hp = h->hp;
+  using soap::strided;
+  using soap::strided_mut;
+  SOAP_CUDA(h, cudaEventRecord(h->fork_ev, s));
+  for (auto& g : h->groups) {
+    cudaStream_t gs = g.stream;
+    SOAP_CUDA(h, cudaStreamWaitEvent(gs, h->fork_ev, 0));
+    const int n = g.n;
+    const int64_t nn = (int64_t)n * n;
+    float *At, *At_lo;
+    soap::qr_input_buffers(g.ws, n, g.batch, &At, &At_lo);
+    for (const QrJob& j : g.jobs) {
+      ClassState& c = h->classes[j.cls];
+      float* F = j.left ? c.L : c.R;
+      float* at = At + (int64_t)j.offset * nn;
+      float* at_lo = At_lo + (int64_t)j.offset * nn;
+      if (c.tc) {
+        SOAP_CUDA(h, soap::gemm_tc_nt(n, n, n, c.count, opnd(j.left ? c.QLt : c.QRt, j.left ? c.QLt_lo : c.QRt_lo, n, nn,
+                                                             c.count),
+                                      opnd(F, j.left ? c.L_lo : c.R_lo, n, nn, c.count),
+                                      epi(h, at, n, nn, at_lo, 0, 1.f, 0.f), gs));
+      } else {
+        SOAP_CUDA(h, soap::gemm(true, false, n, n, n, 1.f, strided(j.left ? c.QL : c.QR, n, nn), strided(F, n, nn), 0.f,
+                                strided_mut(at, n, nn), c.count, gs));
+        SOAP_CUDA(h, soap::split_tf32(at, nullptr, at_lo, (int64_t)c.count * nn, gs));
+      }
+    }
+    // the Q accumulation ends with Q^T and its lo part in the input buffers
+    SOAP_CUDA(h, soap::qr_q_t(n, g.batch, nullptr, nullptr, nullptr, nullptr, g.skip, hp.qr_tol, g.ws, g.ws_bytes,
+                              h->d_status, gs));
+    for (const QrJob& j : g.jobs) {
+      ClassState& c = h->classes[j.cls];
+      const float* qt = At + (int64_t)j.offset * nn;
+      const float* qt_lo = At_lo + (int64_t)j.offset * nn;
+      float* Q = j.left ? c.QL : c.QR;
+      if (c.tc)
+        SOAP_CUDA(h, soap::basis_from_qt(qt, qt_lo, j.left ? c.QLt : c.QRt, j.left ? c.QLt_lo : c.QRt_lo, Q,
+                                         j.left ? c.QL_lo : c.QR_lo, n, c.count, gs));
+      else
+        SOAP_CUDA(h, soap::basis_from_qt(qt, qt_lo, nullptr, nullptr, Q, nullptr, n, c.count, gs));
+      SOAP_CUDA(h, cudaMemcpyAsync(j.left ? c.skipL : c.skipR, g.skip + (int64_t)j.offset * n, (size_t)c.count * n,
+                                   cudaMemcpyDeviceToDevice, gs));
+    }
+    SOAP_CUDA(h, cudaEventRecord(g.done, gs));
   }
-  // rotations of the gradient and of the momentum in one launch each (batch 2B)
-  SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, 2 * B, opnd(GM, c.GM_lo, n, mn, 2 * B), opnd(c.QRt, c.QRt_lo, n, nn, B),
-                                epi(h, h->YMt, m, mn, h->YMt_lo, 1, 1.f, 0.f), s));
-  SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, 2 * B, opnd(c.QLt, c.QLt_lo, m, mm, B), opnd(h->YMt, h->YMt_lo, m, mn, 2 * B),
-                                epi(h, h->Gp, n, mn, nullptr, 0, 1.f, 0.f), s));
-  SOAP_CUDA(h, soap::adam_in_basis(h->Gp, h->Gp + cls, c.V, m, n, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
-                                   hp.guard ? c.skipL : nullptr, hp.guard ? c.skipR : nullptr, h->N_lo, h->d_status,
-                                   s));
-  SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, B, opnd(h->Gp, h->N_lo, n, mn, B), opnd(c.QR, c.QR_lo, n, nn, B),
-                                epi(h, h->Zt, m, mn, h->Zt_lo, 1, 1.f, 0.f), s));
-  soap::TcEpilogue ew = epi(h, nullptr, n, 0, nullptr, 0, -h->lr, 1.f - h->lr * h->wd);
-  ew.C_ptrs = d_params;
-  SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, B, opnd(c.QL, c.QL_lo, m, mm, B), opnd(h->Zt, h->Zt_lo, m, mn, B), ew, s));
+  for (auto& g : h->groups) SOAP_CUDA(h, cudaStreamWaitEvent(s, g.done, 0));
+  return SOAP_OK;
+}
+
+soap_status_t rotate_update_class(soap_handle h, ClassState& c, float* const* d_params, float bc1, float bc2,
+                                  cudaStream_t s) {
+  const soap_hparams& hp = h->hp;
+  const int B = c.count, m = (int)c.rows, n = (int)c.cols;
+  const int64_t mn = (int64_t)m * n, mm = (int64_t)m * m, nn = (int64_t)n * n;
+  using soap::strided;
+  using soap::strided_mut;
+  if (c.tc) {
+    const int64_t cls = (int64_t)B * mn;
+    // rotations of the gradient and of the momentum in one launch each (batch 2B)
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, 2 * B, opnd(c.Gc, c.GM_lo, n, mn, 2 * B), opnd(c.QRt, c.QRt_lo, n, nn, B),
+                                  epi(h, h->YMt, m, mn, h->YMt_lo, 1, 1.f, 0.f), s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, 2 * B, opnd(c.QLt, c.QLt_lo, m, mm, B),
+                                  opnd(h->YMt, h->YMt_lo, m, mn, 2 * B), epi(h, h->Gp, n, mn, nullptr, 0, 1.f, 0.f), s));
+    SOAP_CUDA(h, soap::adam_in_basis(h->Gp, h->Gp + cls, c.V, m, n, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
+                                     hp.guard ? c.skipL : nullptr, hp.guard ? c.skipR : nullptr, h->N_lo, h->d_status,
+                                     s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, B, opnd(h->Gp, h->N_lo, n, mn, B), opnd(c.QR, c.QR_lo, n, nn, B),
+                                  epi(h, h->Zt, m, mn, h->Zt_lo, 1, 1.f, 0.f), s));
+    soap::TcEpilogue ew = epi(h, nullptr, n, 0, nullptr, 0, -h->lr, 1.f - h->lr * h->wd);
+    ew.C_ptrs = d_params;
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, B, opnd(c.QL, c.QL_lo, m, mm, B), opnd(h->Zt, h->Zt_lo, m, mn, B), ew, s));
+    return SOAP_OK;
+  }
+  // S5 and the re-projected first moment: G' = Q_L^T G Q_R, m = Q_L^T M_hat Q_R
+  const float* xg = c.Gc;
+  const float* xm = c.Mhat;
+  if (c.left) {
+    SOAP_CUDA(h, soap::gemm(true, false, m, n, m, 1.f, strided(c.QL, m, mm), strided(c.Gc, n, mn), 0.f,
+                            strided_mut(h->X1, n, mn), B, s));
+    SOAP_CUDA(h, soap::gemm(true, false, m, n, m, 1.f, strided(c.QL, m, mm), strided(c.Mhat, n, mn), 0.f,
+                            strided_mut(h->X2, n, mn), B, s));
+    xg = h->X1;
+    xm = h->X2;
+  }
+  float* gp;
+  const float* mp;
+  if (c.right) {
+    SOAP_CUDA(h, soap::gemm(false, false, m, n, n, 1.f, strided(xg, n, mn), strided(c.QR, n, nn), 0.f,
+                            strided_mut(h->Gp, n, mn), B, s));
+    SOAP_CUDA(h, soap::gemm(false, false, m, n, n, 1.f, strided(xm, n, mn), strided(c.QR, n, nn), 0.f,
+                            strided_mut(h->Mp, n, mn), B, s));
+    gp = h->Gp;
+    mp = h->Mp;
+  } else {
+    gp = const_cast<float*>(xg);  // X1, or the gradient arena copy when no side rotates
+    mp = xm;
+  }
+  // S6
+  SOAP_CUDA(h, soap::adam_in_basis(gp, mp, c.V, m, n, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
+                                   (hp.guard && c.left) ? c.skipL : nullptr, (hp.guard && c.right) ? c.skipR : nullptr,
+                                   nullptr, h->d_status, s));
+  // S7 + S8: W <- (1 - lr wd) W - lr Q_L N Q_R^T
+  const float keep = 1.f - h->lr * h->wd;
+  soap::MutOperand W{nullptr, d_params, 0, 0, n};
+  if (c.left && c.right) {
+    SOAP_CUDA(h, soap::gemm(false, false, m, n, m, 1.f, strided(c.QL, m, mm), strided(gp, n, mn), 0.f,
+                            strided_mut(h->X1, n, mn), B, s));
+    SOAP_CUDA(h, soap::gemm(false, true, m, n, n, -h->lr, strided(h->X1, n, mn), strided(c.QR, n, nn), keep, W, B, s));
+  } else if (c.left) {
+    SOAP_CUDA(h, soap::gemm(false, false, m, n, m, -h->lr, strided(c.QL, m, mm), strided(gp, n, mn), keep, W, B, s));
+  } else if (c.right) {
+    SOAP_CUDA(h, soap::gemm(false, true, m, n, n, -h->lr, strided(gp, n, mn), strided(c.QR, n, nn), keep, W, B, s));
+  } else {
+    SOAP_CUDA(h, soap::weight_update(d_params, gp, mn, B, h->lr, h->wd, s));
+  }
   return SOAP_OK;
 }
 
@@ -251,6 +390,8 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
     if (s.rows < 1 || s.cols < 1 || s.rows > (1 << 20) || s.cols > (1 << 20)) return SOAP_ERR_INVALID_ARG;
     if (s.rows * s.cols > (int64_t(1) << 31) - 1) return SOAP_ERR_INVALID_ARG;
     if ((s.precond_left && s.rows > 8192) || (s.precond_right && s.cols > 8192)) return SOAP_ERR_INVALID_ARG;
+    // the QR's tensor-core products read the factors with TMA: 16-byte rows
+    if ((s.precond_left && (s.rows & 3)) || (s.precond_right && (s.cols & 3))) return SOAP_ERR_INVALID_ARG;
   }
   int ndev = 0;
   if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) return SOAP_ERR_CUDA;
@@ -292,7 +433,7 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
     }
   }
 
-  size_t ws_mat = 0, ws_qr = 0;
+  size_t ws_mat = 0;
   size_t off = 0;
   cudaError_t e = cudaSuccess;
   for (auto& c : h->classes) {
@@ -319,7 +460,6 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
         if (e == cudaSuccess) e = dalloc(h, (void**)&c.QLt, mm * 4);
         if (e == cudaSuccess) e = dalloc(h, (void**)&c.QLt_lo, mm * 4);
       }
-      ws_qr = std::max(ws_qr, soap::qr_workspace_bytes((int)c.rows, c.count));
     }
     if (c.right) {
       const size_t nn = (size_t)c.count * c.cols * c.cols;
@@ -332,9 +472,48 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
         if (e == cudaSuccess) e = dalloc(h, (void**)&c.QRt, nn * 4);
         if (e == cudaSuccess) e = dalloc(h, (void**)&c.QRt_lo, nn * 4);
       }
-      ws_qr = std::max(ws_qr, soap::qr_workspace_bytes((int)c.cols, c.count));
     }
     ws_mat = std::max(ws_mat, mn);
+  }
+  // QR groups: every preconditioned side, grouped by size
+  {
+    std::map<int, int, std::greater<int>> by_n;
+    for (int ci = 0; ci < (int)h->classes.size(); ++ci) {
+      const ClassState& c = h->classes[ci];
+      for (int side = 0; side < 2; ++side) {
+        if (side == 0 ? !c.left : !c.right) continue;
+        const int n = (int)(side == 0 ? c.rows : c.cols);
+        auto it = by_n.find(n);
+        if (it == by_n.end()) it = by_n.emplace(n, (int)by_n.size()).first;
+        (void)it;
+      }
+    }
+    for (auto& kv : by_n) {
+      QrGroup g;
+      g.n = kv.first;
+      h->groups.push_back(g);
+    }
+    for (int ci = 0; ci < (int)h->classes.size(); ++ci) {
+      const ClassState& c = h->classes[ci];
+      for (int side = 0; side < 2; ++side) {
+        if (side == 0 ? !c.left : !c.right) continue;
+        const int n = (int)(side == 0 ? c.rows : c.cols);
+        for (auto& g : h->groups)
+          if (g.n == n) {
+            g.jobs.push_back(QrJob{ci, side == 0, g.batch});
+            g.batch += c.count;
+          }
+      }
+    }
+    for (auto& g : h->groups) {
+      if (g.batch > 65535) e = cudaErrorInvalidValue;
+      g.ws_bytes = soap::qr_workspace_bytes(g.n, g.batch);
+      if (e == cudaSuccess) e = dalloc(h, &g.ws, g.ws_bytes);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&g.skip, (size_t)g.batch * g.n);
+      if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&g.stream, cudaStreamNonBlocking);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.done, cudaEventDisableTiming);
+    }
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->fork_ev, cudaEventDisableTiming);
   }
   h->nptrs = off;
   bool any_tc = false;
@@ -350,8 +529,6 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
     if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt, ws_mat * 4);
     if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt_lo, ws_mat * 4);
   }
-  if (e == cudaSuccess) e = dalloc(h, &h->qr_ws, ws_qr);
-  h->qr_ws_bytes = ws_qr;
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_status, sizeof(int));
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_ptrs, h->nptrs * sizeof(void*));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&h->h_status, sizeof(int));
@@ -447,89 +624,21 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
   const bool refresh = (t % hp.eig_every) == 0;
   const float bc1 = hp.bias_correction ? 1.f - powf(hp.beta1, (float)t) : 1.f;
   const float bc2 = hp.bias_correction ? 1.f - powf(hp.beta2, (float)t) : 1.f;
-  using soap::strided;
-  using soap::strided_mut;
-
+  auto params_of = [&](const ClassState& c) { return reinterpret_cast<float* const*>(h->d_ptrs + c.ptr_offset); };
+  auto grads_of = [&](const ClassState& c) {
+    return reinterpret_cast<const float* const*>(h->d_ptrs + c.ptr_offset + c.count);
+  };
   for (auto& c : h->classes) {
-    const int B = c.count;
-    const int m = (int)c.rows, nc = (int)c.cols;
-    const int64_t mn = (int64_t)m * nc;
-    float* const* d_params = reinterpret_cast<float* const*>(h->d_ptrs + c.ptr_offset);
-    const float* const* d_grads = reinterpret_cast<const float* const*>(h->d_ptrs + c.ptr_offset + B);
-
-    if (c.tc) {
-      soap_status_t st = step_tensor_core(h, c, d_params, d_grads, refresh, bc1, bc2, s);
-      if (st != SOAP_OK) return st;
-      continue;
-    }
-    SOAP_CUDA(h, soap::momentum_and_copy(d_grads, c.Gc, c.Mhat, mn, B, hp.beta1, h->d_status, s));
-    const float fb = hp.factor_beta;
-    if (c.left) {  // S1: L <- b L + (1-b) G G^T
-      SOAP_CUDA(h, soap::gemm(false, true, m, m, nc, 1.f - fb, strided(c.Gc, nc, mn), strided(c.Gc, nc, mn), fb,
-                              strided_mut(c.L, m, (int64_t)m * m), B, s));
-    }
-    if (c.right) {  // S1: R <- b R + (1-b) G^T G
-      SOAP_CUDA(h, soap::gemm(true, false, nc, nc, m, 1.f - fb, strided(c.Gc, nc, mn), strided(c.Gc, nc, mn), fb,
-                              strided_mut(c.R, nc, (int64_t)nc * nc), B, s));
-    }
-    if (refresh) {
-      float* P = (float*)h->qr_ws;  // the QR factors its workspace's first matrix block in place
-      if (c.left) {  // S2 + S3 on the left side
-        SOAP_CUDA(h, soap::gemm(false, false, m, m, m, 1.f, strided(c.L, m, (int64_t)m * m),
-                                strided(c.QL, m, (int64_t)m * m), 0.f, strided_mut(P, m, (int64_t)m * m), B, s));
-        SOAP_CUDA(h, soap::qr_q(m, B, P, c.QL, c.skipL, hp.qr_tol, h->qr_ws, h->qr_ws_bytes, h->d_status, s));
-      }
-      if (c.right) {
-        SOAP_CUDA(h, soap::gemm(false, false, nc, nc, nc, 1.f, strided(c.R, nc, (int64_t)nc * nc),
-                                strided(c.QR, nc, (int64_t)nc * nc), 0.f, strided_mut(P, nc, (int64_t)nc * nc), B, s));
-        SOAP_CUDA(h, soap::qr_q(nc, B, P, c.QR, c.skipR, hp.qr_tol, h->qr_ws, h->qr_ws_bytes, h->d_status, s));
-      }
-    }
-    // S5 and the re-projected first moment: G' = Q_L^T G Q_R, m = Q_L^T M_hat Q_R
-    const float* xg = c.Gc;
-    const float* xm = c.Mhat;
-    if (c.left) {
-      SOAP_CUDA(h, soap::gemm(true, false, m, nc, m, 1.f, strided(c.QL, m, (int64_t)m * m), strided(c.Gc, nc, mn), 0.f,
-                              strided_mut(h->X1, nc, mn), B, s));
-      SOAP_CUDA(h, soap::gemm(true, false, m, nc, m, 1.f, strided(c.QL, m, (int64_t)m * m), strided(c.Mhat, nc, mn), 0.f,
-                              strided_mut(h->X2, nc, mn), B, s));
-      xg = h->X1;
-      xm = h->X2;
-    }
-    float* gp;
-    const float* mp;
-    if (c.right) {
-      SOAP_CUDA(h, soap::gemm(false, false, m, nc, nc, 1.f, strided(xg, nc, mn), strided(c.QR, nc, (int64_t)nc * nc), 0.f,
-                              strided_mut(h->Gp, nc, mn), B, s));
-      SOAP_CUDA(h, soap::gemm(false, false, m, nc, nc, 1.f, strided(xm, nc, mn), strided(c.QR, nc, (int64_t)nc * nc), 0.f,
-                              strided_mut(h->Mp, nc, mn), B, s));
-      gp = h->Gp;
-      mp = h->Mp;
-    } else {
-      gp = const_cast<float*>(xg);  // X1, or the gradient arena copy when no side rotates
-      mp = xm;
-    }
-    // S6
-    SOAP_CUDA(h, soap::adam_in_basis(gp, mp, c.V, m, nc, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
-                                     (hp.guard && c.left) ? c.skipL : nullptr,
-                                     (hp.guard && c.right) ? c.skipR : nullptr, nullptr, h->d_status, s));
-    // S7 + S8: W <- (1 - lr wd) W - lr Q_L N Q_R^T
-    const float keep = 1.f - h->lr * h->wd;
-    soap::MutOperand W{nullptr, d_params, 0, 0, nc};
-    if (c.left && c.right) {
-      SOAP_CUDA(h, soap::gemm(false, false, m, nc, m, 1.f, strided(c.QL, m, (int64_t)m * m), strided(gp, nc, mn), 0.f,
-                              strided_mut(h->X1, nc, mn), B, s));
-      SOAP_CUDA(h, soap::gemm(false, true, m, nc, nc, -h->lr, strided(h->X1, nc, mn), strided(c.QR, nc, (int64_t)nc * nc),
-                              keep, W, B, s));
-    } else if (c.left) {
-      SOAP_CUDA(h, soap::gemm(false, false, m, nc, m, -h->lr, strided(c.QL, m, (int64_t)m * m), strided(gp, nc, mn), keep,
-                              W, B, s));
-    } else if (c.right) {
-      SOAP_CUDA(h, soap::gemm(false, true, m, nc, nc, -h->lr, strided(gp, nc, mn), strided(c.QR, nc, (int64_t)nc * nc),
-                              keep, W, B, s));
-    } else {
-      SOAP_CUDA(h, soap::weight_update(d_params, gp, mn, B, h->lr, h->wd, s));
-    }
+    soap_status_t st = prepare_class(h, c, grads_of(c), s);
+    if (st != SOAP_OK) return st;
+  }
+  if (refresh) {
+    soap_status_t st = refresh_bases(h, s);
+    if (st != SOAP_OK) return st;
+  }
+  for (auto& c : h->classes) {
+    soap_status_t st = rotate_update_class(h, c, params_of(c), bc1, bc2, s);
+    if (st != SOAP_OK) return st;
   }
   SOAP_CUDA(h, cudaMemcpyAsync(h->h_status, h->d_status, sizeof(int), cudaMemcpyDeviceToHost, s));
   SOAP_CUDA(h, cudaEventRecord(h->status_ev, s));
@@ -749,7 +858,8 @@ size_t soap_qr_workspace_bytes(int32_t n, int32_t batch) {
 
 soap_status_t soap_qr(int32_t n, int32_t batch, const float* P, float* Q, uint8_t* skip, float tol, void* workspace,
                       size_t workspace_bytes, soap_stream_t stream) {
-  if (n <= 0 || n > 8192 || batch <= 0 || batch > 65535 || !P || !Q || !skip || !workspace || !(tol >= 0.f))
+  if (n <= 0 || n > 8192 || (n & 3) || batch <= 0 || batch > 65535 || !P || !Q || !skip || !workspace ||
+      !(tol >= 0.f))
     return SOAP_ERR_INVALID_ARG;
   if (!aligned16(P) || !aligned16(Q) || (reinterpret_cast<uintptr_t>(workspace) & 255))
     return SOAP_ERR_INVALID_ARG;

@@ -75,10 +75,19 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
 // hi = trunc_tf32(x), lo = x - hi (exact), elementwise over n values.
 cudaError_t split_tf32(const float* x, float* hi, float* lo, int64_t n, cudaStream_t stream);
 
-// Householder QR (explicit Q) of `batch` contiguous n x n matrices.
+// Householder QR (explicit Q) of `batch` contiguous n x n matrices (n a multiple of 4).
 size_t qr_workspace_bytes(int n, int batch);
+// P read only; Q written. Uses the tensor-core QR on P^T (staged in the workspace).
 cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, float tol,
                  void* workspace, size_t workspace_bytes, int* status, cudaStream_t stream);
+// Where the factored matrix P^T and its tf32 lo part must be placed before qr_q_t.
+void qr_input_buffers(void* workspace, int n, int batch, float** At, float** At_lo);
+// QR of P whose transpose (and lo part) is already in qr_input_buffers(). Writes Q^T and its
+// lo part into Qt/Qt_lo (or, if Qt is nullptr, into the workspace) and, if Q is given, Q and
+// (if Q_lo is given) its lo part.
+cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q_lo, uint8_t* skip,
+                   float tol, void* workspace, size_t workspace_bytes, int* status,
+                   cudaStream_t stream);
 
 // Elementwise kernels of the step.
 // M_hat <- b1 M_hat + (1-b1) G and Gc <- G for each matrix of a class.
@@ -95,6 +104,9 @@ cudaError_t adam_in_basis(float* Gp, const float* Mp, float* V, int rows, int co
 cudaError_t momentum_split(const float* const* grads, float* Gc, float* Gc_lo, float* Gt, float* Gt_lo,
                            float* Mhat, float* Mhat_lo, int rows, int cols, int batch, float beta1,
                            int* status, cudaStream_t stream);
+// From Q^T and its lo part: copies of both and Q with its lo part (any output may be null).
+cudaError_t basis_from_qt(const float* Qt, const float* Qt_lo, float* Qt_out, float* Qt_lo_out, float* Q,
+                          float* Q_lo, int n, int batch, cudaStream_t stream);
 // Q -> lo part, Q^T, lo part of Q^T for `batch` n x n bases.
 cudaError_t basis_split(const float* Q, float* Q_lo, float* Qt, float* Qt_lo, int n, int batch,
                         cudaStream_t stream);

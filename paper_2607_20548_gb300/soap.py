@@ -27,7 +27,7 @@ EXPORTS = ("soap_default_hparams", "soap_create", "soap_step", "soap_set_lr", "s
            "soap_clear_status", "soap_last_error", "soap_destroy", "soap_qr_workspace_bytes",
            "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_gemm_tf32x3",
            "soap_split_tf32", "soap_qr_static")
-KERNEL_FAMILIES = ("gemm_simt", "gemm_tc", "qr_panel", "elementwise", "other")
+KERNEL_FAMILIES = ("gemm_simt", "gemm_tc", "qr_panel", "elementwise", "other", "qr_update")
 
 
 class soap_shape(ctypes.Structure):
@@ -274,7 +274,7 @@ def soap_qr(P: torch.Tensor, tol: float = 0.0, stream=None):
 def soap_qr_static(P: torch.Tensor, tol: float = 0.0, stream=None):
     """soap_qr without a caller-supplied workspace, for code that cannot allocate device memory
     when it needs the QR: libsoap.so uses a fixed 32 MiB array of its own (enough for one
-    2048 x 2048 matrix). The output tensors here are allocated by torch for convenience; a
+    1024 x 1024 matrix). The output tensors here are allocated by torch for convenience; a
     caller without an allocator passes its own buffers to the C entry point. Raises
     SoapError(SOAP_ERR_INVALID_ARG) for work larger than the array."""
     lib = load_library()

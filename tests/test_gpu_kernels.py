@@ -53,8 +53,8 @@ def _qr_case(n, batch, kind, seed):
     raise ValueError(kind)
 
 
-@pytest.mark.parametrize("n,batch,kind", [(1, 1, "well"), (31, 2, "well"), (32, 1, "gauss"), (33, 3, "gauss"),
-                                          (100, 2, "lowrank"), (513, 2, "well"), (1025, 1, "well"),
+@pytest.mark.parametrize("n,batch,kind", [(4, 1, "well"), (36, 2, "well"), (32, 1, "gauss"), (36, 3, "gauss"),
+                                          (100, 2, "lowrank"), (516, 2, "well"), (1028, 1, "well"),
                                           (768, 2, "lowrank"), (2048, 1, "well"), (2048, 1, "lowrank")])
 def test_qr_matches_oracle(cuda, n, batch, kind):
     """S3 on identical fp32 inputs: skip flags equal the oracle's, Q^T Q = I to 1e-5, and Q agrees
@@ -79,6 +79,13 @@ def test_qr_matches_oracle(cuda, n, batch, kind):
             c_gpu = _rel(Q[b][:, s64], Q64[:, s64])
             c_twin = _rel(Q32[:, s64].astype(np.float64), Q64[:, s64])
             assert c_gpu <= max(1e-5, 4 * c_twin), (c_gpu, c_twin)
+
+
+def test_qr_rejects_sizes_not_multiple_of_4(cuda):
+    """The QR's tensor-core products read rows with TMA (16-byte rows): n must be a multiple of 4."""
+    with pytest.raises(S.SoapError) as err:
+        S.soap_qr(torch.eye(33, device=cuda).unsqueeze(0), 1e-4)
+    assert err.value.code == 1
 
 
 def test_qr_full_size_8192_properties(cuda):
