@@ -204,7 +204,10 @@ def run_soap(args):
     if not os.path.exists(S.LIB_PATH):
         build.build()
     specs, _ = WORKLOADS[WORKLOAD]
-    gen = make_stream(WORKLOAD, seed=rank, device=dev)
+    subset = [int(x) for x in args.matrices.split(",") if x.strip()] if args.matrices else None
+    if subset:
+        specs = [specs[j] for j in subset]
+    gen = make_stream(WORKLOAD, seed=rank, device=dev, specs=subset)
     opt = SoapOptimizer([(s.rows, s.cols, s.left, s.right) for s in specs], default_hparams(), device=local)
 
     def flat(tensors):
@@ -292,7 +295,8 @@ def run_soap(args):
         "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "matrices": 7,
+        "config": {"workload": WORKLOAD if not subset else f"{WORKLOAD}[matrices {args.matrices}]",
+                   "matrices": len(specs),
                    "shapes": "4x 2048x2048, 2x 2048x8192, 1x 8192x2048, all sides preconditioned",
                    "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2 (3 GB of optimizer state per step)"},
@@ -302,6 +306,10 @@ def run_soap(args):
         "roofline": roof,
         "kernel_time_share": {k: round(v["ms"] / max(1e-9, sum(x["ms"] for x in fams.values())), 4)
                               for k, v in fams.items()},
+        "kernel_families": {k: {"ms_per_step": v["ms"] / args.steps, "launches_per_step": v["launches"] / args.steps,
+                                "tflops": v["flops"] / max(1e-12, v["ms"] / 1e3) / 1e12,
+                                "gbs": v["bytes"] / max(1e-12, v["ms"] / 1e3) / 1e9}
+                            for k, v in fams.items() if v["launches"]},
         "cpu_baseline": {"value": sps, "unit": "steps/s", "cores": threads, "kind": "oracle",
                          "sample": f"one fp64 oracle step of Wq (2048x2048) took {per:.1f} s; whole block "
                                    f"= {scale:.1f}x that by the FLOP model"},
@@ -320,6 +328,9 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["soap", "reference"], default="soap")
+    ap.add_argument("--matrices", default="",
+                    help="comma-separated matrix indices of the block to run (a smaller case for profiling); "
+                         "default: all 7")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)

@@ -296,84 +296,129 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   }
 }
 
-// Rank-32 update C_b <- C_b - A_b B_b^T (A: M x K, B: N x K, K <= 32, all row-major) with
-// the lo part of the result, in exact fp32 FMAs. It streams C once (read, write, lo write;
-// 32 FMAs per element), so it is bound by HBM, not by a matrix unit: each thread issues its
-// 32 loads of C before any arithmetic, and two 256-thread CTAs share an SM.
-// Tile 64 x 128: warp w owns rows 8w..8w+7, lane l columns l, l+32, l+64, l+96.
-constexpr int RU_BM = 64, RU_BN = 128;
+// Rank-32 update C_b <- C_b - A_b B_b^T (A: M x K, B: N x K, K <= 32, all row-major, N a
+// multiple of 4) with the lo part of the result, in exact fp32 FMAs. It streams C once
+// (read, write, lo write; 32 FMAs per element), so it is bound by HBM, not by a matrix
+// unit. A CTA owns one 128-column strip: it loads that strip's B once (k-major in shared
+// memory), then walks down the rows in 64 x 128 tiles, with the C and A tiles of the next
+// tile copied in by cp.async while the current one is computed (two stages), so ~64 KB per
+// CTA is in flight. Warp w computes rows 8w..8w+7, lane l columns 4l..4l+3; every global
+// access to C is a 16-byte vector and a warp covers 512 contiguous bytes of a row.
+constexpr int RU_BM = 64, RU_BN = 128, RU_STAGES = 2;
+constexpr int RU_SMEM = (RU_STAGES * RU_BM * RU_BN + RU_STAGES * RU_BM * NB + NB * RU_BN) * 4;
+
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src, bool valid) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(gmem_src), "r"(valid ? 16 : 0)
+               : "memory");
+}
 
 __global__ void __launch_bounds__(256, 2)
     rank_update_kernel(int M, int N, int K, const float* __restrict__ A, int64_t lda, int64_t sa,
                        const float* __restrict__ B, int64_t ldb, int64_t sb, float* C, float* C_lo, int64_t ldc,
                        int64_t sc) {
-  __shared__ float As[NB][RU_BM + 1];  // [k][row]
-  __shared__ float Bs[NB][RU_BN + 1];  // [k][col]
+  extern __shared__ float4 ru_smem[];
+  float* Cs = reinterpret_cast<float*>(ru_smem);     // [stage][RU_BM][RU_BN]
+  float* As = Cs + RU_STAGES * RU_BM * RU_BN;        // [stage][RU_BM][NB]
+  float* Bs = As + RU_STAGES * RU_BM * NB;           // [NB][RU_BN]
   const int b = blockIdx.z;
-  const int r0 = blockIdx.y * RU_BM, c0 = blockIdx.x * RU_BN;
+  const int c0 = blockIdx.x * RU_BN;
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const float* Ab = A + (int64_t)b * sa;
   const float* Bb = B + (int64_t)b * sb;
   float* Cb = C + (int64_t)b * sc;
   float* Lb = C_lo + (int64_t)b * sc;
-  // C first: 32 independent loads per thread in flight
-  float cv[8][4];
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int r = r0 + 8 * w + i;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int col = c0 + lane + 32 * j;
-      cv[i][j] = (r < M && col < N) ? Cb[(int64_t)r * ldc + col] : 0.f;
+  const int ntiles = (M + RU_BM - 1) / RU_BM;
+  const int col = c0 + 4 * lane;
+
+  // one 64 x 128 tile of C and its 64 x 32 slice of A into stage st (zero-filled past the edges)
+  auto issue = [&](int tile, int st) {
+    const int r0 = tile * RU_BM;
+    float* cs = Cs + st * RU_BM * RU_BN;
+    float* as = As + st * RU_BM * NB;
+    for (int e = tid; e < RU_BM * (RU_BN / 4); e += 256) {
+      const int r = e / (RU_BN / 4), q = e % (RU_BN / 4);
+      const bool ok = (r0 + r < M) && (c0 + 4 * q < N);
+      cp_async16(cs + r * RU_BN + 4 * q, ok ? Cb + (int64_t)(r0 + r) * ldc + c0 + 4 * q : Cb, ok);
     }
-  }
-  for (int e = tid; e < RU_BM * NB; e += 256) {
-    const int r = e / NB, kk = e % NB;
-    As[kk][r] = (r0 + r < M && kk < K) ? Ab[(int64_t)(r0 + r) * lda + kk] : 0.f;
-  }
+    for (int e = tid; e < RU_BM * (NB / 4); e += 256) {
+      const int r = e / (NB / 4), q = e % (NB / 4);
+      const bool ok = (r0 + r < M) && (4 * q < K);
+      cp_async16(as + r * NB + 4 * q, ok ? Ab + (int64_t)(r0 + r) * lda + 4 * q : Ab, ok);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+
+  int tile = blockIdx.y;
+  if (tile < ntiles) issue(tile, 0);
   for (int e = tid; e < RU_BN * NB; e += 256) {
     const int cc = e / NB, kk = e % NB;
-    Bs[kk][cc] = (c0 + cc < N && kk < K) ? Bb[(int64_t)(c0 + cc) * ldb + kk] : 0.f;
+    Bs[kk * RU_BN + cc] = (c0 + cc < N && kk < K) ? Bb[(int64_t)(c0 + cc) * ldb + kk] : 0.f;
   }
-  __syncthreads();
-  float acc[8][4];
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
-#pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
-#pragma unroll 8
-  for (int kk = 0; kk < NB; ++kk) {
-    float a[8], bv[4];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) a[i] = As[kk][8 * w + i];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) bv[j] = Bs[kk][lane + 32 * j];
+  for (int it = 0; tile < ntiles; ++it, tile += gridDim.y) {
+    const int st = it & 1;
+    const int next = tile + gridDim.y;
+    if (next < ntiles) {
+      issue(next, st ^ 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    }
+    __syncthreads();
+    const float* cs = Cs + st * RU_BM * RU_BN;
+    const float* as = As + st * RU_BM * NB;
+    float acc[8][4];
 #pragma unroll
     for (int i = 0; i < 8; ++i)
 #pragma unroll
-      for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], bv[j], acc[i][j]);
-  }
+      for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+#pragma unroll 4
+    for (int kk = 0; kk < NB; ++kk) {
+      const float4 bv = *reinterpret_cast<const float4*>(&Bs[kk * RU_BN + 4 * lane]);
+      const float bb[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int r = r0 + 8 * w + i;
-    if (r >= M) break;
+      for (int i = 0; i < 8; ++i) {
+        const float a = as[(8 * w + i) * NB + kk];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int col = c0 + lane + 32 * j;
-      if (col >= N) continue;
-      const float out = cv[i][j] - acc[i][j];
-      Cb[(int64_t)r * ldc + col] = out;
-      Lb[(int64_t)r * ldc + col] = tf32_lo(out);
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a, bb[j], acc[i][j]);
+      }
     }
+    const int r0 = tile * RU_BM;
+    if (col < N) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int r = r0 + 8 * w + i;
+        if (r >= M) break;
+        const float4 c = *reinterpret_cast<const float4*>(&cs[(8 * w + i) * RU_BN + 4 * lane]);
+        float4 o;
+        o.x = c.x - acc[i][0];
+        o.y = c.y - acc[i][1];
+        o.z = c.z - acc[i][2];
+        o.w = c.w - acc[i][3];
+        *reinterpret_cast<float4*>(Cb + (int64_t)r * ldc + col) = o;
+        *reinterpret_cast<float4*>(Lb + (int64_t)r * ldc + col) =
+            make_float4(tf32_lo(o.x), tf32_lo(o.y), tf32_lo(o.z), tf32_lo(o.w));
+      }
+    }
+    __syncthreads();  // this stage is refilled by the next iteration's prefetch
   }
 }
 
 cudaError_t rank_update(int M, int N, int K, int batch, const float* A, int64_t lda, int64_t sa, const float* B,
                         int64_t ldb, int64_t sb, float* C, float* C_lo, int64_t ldc, int64_t sc, cudaStream_t s) {
   if (M <= 0 || N <= 0) return cudaSuccess;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(rank_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, RU_SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
   ProfScope prof(kFamQrUpdate, 2.0 * M * N * (double)K * batch, 12.0 * M * (double)N * batch, s);
-  dim3 grid((N + RU_BN - 1) / RU_BN, (M + RU_BM - 1) / RU_BM, batch);
-  rank_update_kernel<<<grid, 256, 0, s>>>(M, N, K, A, lda, sa, B, ldb, sb, C, C_lo, ldc, sc);
+  const int strips = (N + RU_BN - 1) / RU_BN, ntiles = (M + RU_BM - 1) / RU_BM;
+  // about two waves of 2 CTAs per SM; each CTA walks ntiles / gridDim.y row tiles
+  const int want = std::max(1, (2 * 2 * 152) / std::max(1, strips * batch));
+  dim3 grid(strips, std::min(ntiles, want), batch);
+  rank_update_kernel<<<grid, 256, RU_SMEM, s>>>(M, N, K, A, lda, sa, B, ldb, sb, C, C_lo, ldc, sc);
   return cudaGetLastError();
 }
 
