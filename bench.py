@@ -238,11 +238,15 @@ def run_soap(args):
     barrier()
     torch.cuda.synchronize()
     with ClockSampler(local) as clk:
+        # cudaProfilerStart/Stop bracket the timed steps, so that a profiler started with
+        # profiling off (ncu --profile-from-start off) records exactly these launches
+        torch.cuda.profiler.start()
         start.record(stream)
         for t in range(args.steps):
             opt.step(W, pool[(args.warmup + t) % npool])
         stop.record(stream)
         torch.cuda.synchronize()
+        torch.cuda.profiler.stop()
     prof = opt.profile_end()
     barrier()
     elapsed = start.elapsed_time(stop) / 1e3

@@ -154,7 +154,7 @@ typedef enum {
   SOAP_KERNEL_QR_PANEL = 2,    /* cluster panel factorisation of the QR */
   SOAP_KERNEL_ELEMENTWISE = 3, /* momentum, Adam, weight update */
   SOAP_KERNEL_OTHER = 4,       /* norms, identity fills */
-  SOAP_KERNEL_QR_UPDATE = 5    /* rank-32 updates of the QR */
+  SOAP_KERNEL_QR_UPDATE = 5    /* tensor-core products of the QR's block updates */
 } soap_kernel_family;
 
 typedef struct {

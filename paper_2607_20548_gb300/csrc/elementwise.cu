@@ -122,11 +122,14 @@ __global__ void identity_kernel(float* Q, int n) {
 }
 
 
-// One 32 x 32 tile of one matrix per block (32 x 8 threads). Reads G, updates M_hat and
-// writes the tensor-core operands: G (copy) and its lo part, G^T and its lo part, and
-// the lo part of the new M_hat.
-__global__ void momentum_split_kernel(const float* const* grads, float* Gc, float* Gc_lo, float* Gt, float* Gt_lo,
-                                      float* Mh, float* Mh_lo, int rows, int cols, float beta1, int* status) {
+// One 32 x 32 tile of one matrix per block (32 x 8 threads). Reads G and writes the
+// tensor-core operands: G and its lo part, G^T and its lo part, and the momentum EMA
+// M_hat <- b1 M_hat + (1-b1) G with its lo part. M_hat is kept in G's orientation or, with
+// mh_transposed, as M_hat^T (the working orientation of a matrix preconditioned on its
+// left side only).
+__global__ void momentum_split_kernel(const float* const* grads, float* Gn, float* Gn_lo, float* Gt, float* Gt_lo,
+                                      float* Mh, float* Mh_lo, int rows, int cols, float beta1, int mh_transposed,
+                                      int* status) {
   __shared__ float tile[32][33];
   const int b = blockIdx.z;
   const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
@@ -141,11 +144,13 @@ __global__ void momentum_split_kernel(const float* const* grads, float* Gc, floa
       const int64_t o = (int64_t)b * mn + (int64_t)r * cols + c;
       x = g[(int64_t)r * cols + c];
       bad |= !isfinite(x);
-      Gc[o] = x;
-      Gc_lo[o] = lo_part(x);
-      const float m = fmaf(beta1, Mh[o], c1 * x);
-      Mh[o] = m;
-      Mh_lo[o] = lo_part(m);
+      Gn[o] = x;
+      Gn_lo[o] = lo_part(x);
+      if (!mh_transposed) {
+        const float m = fmaf(beta1, Mh[o], c1 * x);
+        Mh[o] = m;
+        Mh_lo[o] = lo_part(m);
+      }
     }
     tile[i][threadIdx.x] = x;
   }
@@ -157,9 +162,31 @@ __global__ void momentum_split_kernel(const float* const* grads, float* Gc, floa
       const int64_t o = (int64_t)b * mn + (int64_t)c * rows + r;
       Gt[o] = x;
       Gt_lo[o] = lo_part(x);
+      if (mh_transposed) {
+        const float m = fmaf(beta1, Mh[o], c1 * x);
+        Mh[o] = m;
+        Mh_lo[o] = lo_part(m);
+      }
     }
   }
   if (__syncthreads_or(bad) && threadIdx.x == 0 && threadIdx.y == 0) atomicOr(status, kStatusNonFinite);
+}
+
+// dst_b = src_b^T for `batch` contiguous rows x cols matrices (32 x 32 tiles, 32 x 8 threads).
+__global__ void transpose_kernel(const float* src, float* dst, int rows, int cols) {
+  __shared__ float tile[32][33];
+  const int b = blockIdx.z;
+  const int64_t mn = (int64_t)rows * cols;
+  const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = r0 + i, c = c0 + threadIdx.x;
+    tile[i][threadIdx.x] = (r < rows && c < cols) ? src[(int64_t)b * mn + (int64_t)r * cols + c] : 0.f;
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int c = c0 + i, r = r0 + threadIdx.x;
+    if (r < rows && c < cols) dst[(int64_t)b * mn + (int64_t)c * rows + r] = tile[threadIdx.x][i];
+  }
 }
 
 // Q -> Q_lo, Q^T, Q^T_lo for `batch` n x n matrices (32 x 32 tiles, 32 x 8 threads).
@@ -233,14 +260,24 @@ __global__ void split_kernel(const float* x, float* hi, float* lo, int64_t n) {
 
 }  // namespace
 
-cudaError_t momentum_split(const float* const* grads, float* Gc, float* Gc_lo, float* Gt, float* Gt_lo, float* Mhat,
-                           float* Mhat_lo, int rows, int cols, int batch, float beta1, int* status, cudaStream_t s) {
+cudaError_t momentum_split(const float* const* grads, float* Gn, float* Gn_lo, float* Gt, float* Gt_lo, float* Mhat,
+                           float* Mhat_lo, int rows, int cols, int batch, float beta1, bool mhat_transposed, int* status,
+                           cudaStream_t s) {
   if (rows <= 0 || cols <= 0 || batch <= 0) return cudaSuccess;
   const double e = (double)rows * cols * batch;
   ProfScope prof(kFamElementwise, 3.0 * e, 32.0 * e, s);
   dim3 grid((cols + 31) / 32, (rows + 31) / 32, batch);
-  momentum_split_kernel<<<grid, dim3(32, 8), 0, s>>>(grads, Gc, Gc_lo, Gt, Gt_lo, Mhat, Mhat_lo, rows, cols, beta1,
-                                                     status);
+  momentum_split_kernel<<<grid, dim3(32, 8), 0, s>>>(grads, Gn, Gn_lo, Gt, Gt_lo, Mhat, Mhat_lo, rows, cols, beta1,
+                                                     mhat_transposed ? 1 : 0, status);
+  return cudaGetLastError();
+}
+
+cudaError_t transpose(const float* src, float* dst, int rows, int cols, int batch, cudaStream_t s) {
+  if (rows <= 0 || cols <= 0 || batch <= 0) return cudaSuccess;
+  if (batch > 65535 || (rows + 31) / 32 > 65535) return cudaErrorInvalidValue;
+  ProfScope prof(kFamOther, 0.0, 8.0 * rows * (double)cols * batch, s);
+  dim3 grid((cols + 31) / 32, (rows + 31) / 32, batch);
+  transpose_kernel<<<grid, dim3(32, 8), 0, s>>>(src, dst, rows, cols);
   return cudaGetLastError();
 }
 

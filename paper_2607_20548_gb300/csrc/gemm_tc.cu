@@ -24,7 +24,10 @@
 // tensor memory and issues the MMAs (one elected lane), warps 2-5 drain the
 // accumulators and run the epilogue: tensor memory -> registers (each warp owns 32 of
 // the 128 accumulator lanes) -> alpha/beta -> global, optionally transposed and optionally also writing the lo part
-// of the result for a later product. Stages are handed over with mbarriers; every
+// of the result for a later product. When the epilogue reads C (beta != 0), the
+// epilogue warps copy their part of the C tile into shared memory with cp.async while
+// the MMAs run, so the epilogue does not wait on one global load per output row.
+// Stages are handed over with mbarriers; every
 // wait gives up after ~2 s of %globaltimer time, records kStatusTimeout and lets the
 // CTA drain and free its tensor memory instead of hanging.
 #include <cuda.h>
@@ -43,13 +46,14 @@ constexpr int BK = 32;  // fp32 elements per K block = one 128-byte swizzle row
 constexpr int THREADS = 192;
 constexpr uint64_t kWaitNs = 2000000000ull;
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, bool PRE>
 struct Cfg {
   static constexpr int TILE_A = BM * BK * 4;
   static constexpr int TILE_B = BN * BK * 4;
   static constexpr int STAGE = 2 * TILE_A + 2 * TILE_B;
   static constexpr int STAGING = 4 * 32 * 33 * 4;  // per epilogue warp: one 32 x 32 block (+pad)
-  static constexpr int SMEM = STAGES * STAGE + STAGING + 1024 + 256;
+  static constexpr int CPRE = PRE ? 4 * 32 * BN * 4 : 0;  // prefetched C tile (32 rows per warp)
+  static constexpr int SMEM = STAGES * STAGE + STAGING + CPRE + 1024 + 256;
   static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators, used alternately
   static_assert(SMEM <= 232448, "shared memory budget");
 };
@@ -164,16 +168,23 @@ __device__ __forceinline__ float tf32_lo(float x) {
   return __uint_as_float(r);
 }
 
-template <int BN, int STAGES>
+__device__ __forceinline__ void cp_async16(float* smem_dst, const float* gmem_src, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(smem_dst)), "l"(gmem_src),
+               "r"(valid ? 16 : 0)
+               : "memory");
+}
+
+template <int BN, int STAGES, bool PRE>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap ta_hi, const __grid_constant__ CUtensorMap ta_lo,
                    const __grid_constant__ CUtensorMap tb_hi, const __grid_constant__ CUtensorMap tb_lo, int M,
                    int N, int K, int a_mod, int b_mod, TcEpilogue ep) {
-  using C = Cfg<BN, STAGES>;
+  using C = Cfg<BN, STAGES, PRE>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   float* staging = reinterpret_cast<float*>(smem + STAGES * C::STAGE);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE + C::STAGING);
+  float* cpre_all = reinterpret_cast<float*>(smem + STAGES * C::STAGE + C::STAGING);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE + C::STAGING + C::CPRE);
   uint64_t* empty = full + STAGES;
   uint64_t* acc_full = empty + STAGES;  // [2] accumulator a holds a finished K block
   uint64_t* acc_empty = acc_full + 2;   // [2] accumulator a has been drained
@@ -272,6 +283,32 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else {
     const int q = warp & 3;  // this warp may read accumulator lanes 32q .. 32q+31
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * q) << 16);
+    float* Cb = ep.C_ptrs ? ep.C_ptrs[b] : (ep.C ? ep.C + (int64_t)b * ep.c_stride : nullptr);
+    const int row0 = m0 + 32 * q;  // first of this warp's 32 rows
+    // this warp's part of the C tile, copied in while the MMAs run: rows row0.. x BN columns
+    // ([row][col]), or for a transposed C the BN columns' 32 entries each ([col][row]);
+    // only 16-byte chunks wholly inside C are copied, so partial chunks disable it
+    float* cpre = cpre_all + q * 32 * BN;
+    const bool pre = PRE && Cb && ep.beta != 0.f && (ep.ldc & 3) == 0 &&
+                     (reinterpret_cast<uintptr_t>(Cb) & 15) == 0 && ((ep.transpose ? M : N) & 3) == 0;
+    if (pre) {
+      if (!ep.transpose) {
+        for (int i = lane; i < 32 * (BN / 4); i += 32) {
+          const int rr = i / (BN / 4), ch = i % (BN / 4);
+          const int r = row0 + rr, col = n0 + 4 * ch;
+          const bool ok = r < M && col < N;
+          cp_async16(cpre + rr * BN + 4 * ch, ok ? Cb + (int64_t)r * ep.ldc + col : Cb, ok);
+        }
+      } else {
+        for (int i = lane; i < BN * 8; i += 32) {
+          const int cc = i / 8, ch = i % 8;
+          const int col = n0 + cc, r = row0 + 4 * ch;
+          const bool ok = r < M && col < N;
+          cp_async16(cpre + cc * 32 + 4 * ch, ok ? Cb + (int64_t)col * ep.ldc + r : Cb, ok);
+        }
+      }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    }
     float acc[BN / 32][32];
 #pragma unroll
     for (int c = 0; c < BN / 32; ++c)
@@ -298,9 +335,12 @@ __global__ void __launch_bounds__(THREADS, 1)
         asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&acc_empty[a])) : "memory");
     }
     if (!valid && lane == 0 && ep.status) atomicOr(ep.status, kStatusTimeout);
-    float* Cb = ep.C_ptrs ? ep.C_ptrs[b] : (ep.C ? ep.C + (int64_t)b * ep.c_stride : nullptr);
+    if (pre) {
+      // the copies complete even when a wait gave up, before the CTA's shared memory goes away
+      asm volatile("cp.async.wait_all;" ::: "memory");
+      __syncwarp();
+    }
     float* Lb = ep.C_lo ? ep.C_lo + (int64_t)b * ep.lo_stride : nullptr;
-    const int row0 = m0 + 32 * q;  // first of this warp's 32 rows
     if (valid && ep.transpose) {
       // C^T: for a fixed column the 32 lanes (32 consecutive rows) write 128 contiguous bytes
       const int r = row0 + lane;
@@ -314,7 +354,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const int64_t off = (int64_t)col * ep.ldc + r;
           float out = ep.alpha * acc[c][j];
           if (Cb) {
-            if (ep.beta != 0.f) out = fmaf(ep.beta, Cb[off], out);
+            if (ep.beta != 0.f) out = fmaf(ep.beta, pre ? cpre[(32 * c + j) * 32 + lane] : Cb[off], out);
             Cb[off] = out;
           }
           if (Lb) Lb[(int64_t)col * ep.ld_lo + r] = tf32_lo(out);
@@ -339,7 +379,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             float out = ep.alpha * st[rr * 33 + lane];
             if (Cb) {
               const int64_t off = (int64_t)r * ep.ldc + col;
-              if (ep.beta != 0.f) out = fmaf(ep.beta, Cb[off], out);
+              if (ep.beta != 0.f) out = fmaf(ep.beta, pre ? cpre[rr * BN + 32 * c + lane] : Cb[off], out);
               Cb[off] = out;
             }
             if (Lb) Lb[(int64_t)r * ep.ld_lo + col] = tf32_lo(out);
@@ -391,10 +431,10 @@ bool make_map(CUtensorMap* map, const float* base, int rows, int K, int64_t ld, 
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, bool PRE>
 cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, int batch, const TcEpilogue& ep,
                    cudaStream_t s) {
-  using C = Cfg<BN, STAGES>;
+  using C = Cfg<BN, STAGES, PRE>;
   CUtensorMap m[4];
   const int amod = A.batch > 0 ? A.batch : batch;
   const int bmod = B.batch > 0 ? B.batch : batch;
@@ -403,28 +443,33 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
     return cudaErrorInvalidValue;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    cudaError_t e =
+        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
   dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM, batch);
-  gemm_tc_kernel<BN, STAGES><<<grid, THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, amod, bmod, ep);
+  gemm_tc_kernel<BN, STAGES, PRE><<<grid, THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, amod, bmod, ep);
   return cudaGetLastError();
 }
 
 }  // namespace tc
 
 cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const TcOperand& B, const TcEpilogue& ep,
-                       cudaStream_t s) {
+                       cudaStream_t s, int family) {
   if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
   if (batch > 65535 || (M + tc::BM - 1) / tc::BM > 65535) return cudaErrorInvalidValue;
   const double flops = 2.0 * M * N * (double)K * batch;  // algorithmic (4 tf32 products each on the pipe)
   const double bytes = 4.0 * (2.0 * (double)M * K * (A.batch > 0 ? A.batch : batch) +
                               2.0 * (double)N * K * (B.batch > 0 ? B.batch : batch) +
                               (double)M * N * batch * ((ep.beta != 0.f ? 2 : 1) + (ep.C_lo ? 1 : 0)));
-  ProfScope prof(kFamGemmTc, flops, bytes, s);
-  if (N <= 32) return tc::launch<32, 5>(A, B, M, N, K, batch, ep, s);
-  return tc::launch<128, 3>(A, B, M, N, K, batch, ep, s);
+  ProfScope prof(family, flops, bytes, s);
+  // an epilogue that reads C gives one pipeline stage's shared memory to the C tile
+  const bool pre = ep.beta != 0.f && (ep.C || ep.C_ptrs);
+  if (N <= 32) return pre ? tc::launch<32, 4, true>(A, B, M, N, K, batch, ep, s)
+                          : tc::launch<32, 5, false>(A, B, M, N, K, batch, ep, s);
+  return pre ? tc::launch<128, 2, true>(A, B, M, N, K, batch, ep, s)
+             : tc::launch<128, 3, false>(A, B, M, N, K, batch, ep, s);
 }
 
 }  // namespace soap

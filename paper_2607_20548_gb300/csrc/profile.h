@@ -18,7 +18,7 @@ enum KernelFamily : int {
   kFamQrPanel = 2,    // cluster panel factorisation of the QR
   kFamElementwise = 3,// momentum / Adam / weight update
   kFamOther = 4,      // norms, identity fills
-  kFamQrUpdate = 5,   // rank-32 updates of the QR (HBM-bound)
+  kFamQrUpdate = 5,   // tensor-core products of the QR's block updates (HBM-bound)
   kNumFamilies = 6,
 };
 

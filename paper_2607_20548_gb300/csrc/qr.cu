@@ -3,27 +3,35 @@
 // appendix on eigh vs QR settles), with diag(R) >= 0, on tensor cores.
 //
 // The QR works on At = P^T (row j of At is column j of P), so every product of the
-// blocked algorithm is a C = A B^T of K-major operands: the long reductions run on the
-// tcgen05 engine, the rank-32 updates (HBM-bound) on the CUDA cores:
+// blocked algorithm is a C = A B^T of K-major operands for the tcgen05 engine. It is
+// blocked on two levels: 32-column panels are factored in distributed shared memory,
+// and the trailing matrix -- the HBM-bound part -- is updated once per 128-column block
+// of four panels:
 //
-//   for each 32-column panel at k (rows k..k+31 of At):
-//     1. qr_panel_kernel factors the panel rows in distributed shared memory and writes
-//        the Householder vectors as rows of Vt (row k+a = v_a over positions k..n-1,
-//        zeros before its pivot), T with H_1..H_32 = I - V T V^T, and V T^T and V T
-//        (positions x 32), each with its tf32 lo part.
-//     2. trailing rows r > k+31 (columns of P): a_r <- a_r - (a_r V) T V^T, i.e.
-//          W1  = At_trail Vt^T                (tensor cores: M = rows, N = 32, K = positions)
-//          At_trail -= W1 (V T^T)^T           (rank-32 update streaming At_trail once)
+//   for each block of 128 rows of At at k0 (columns k0..k0+127 of P):
+//     for each 32-row panel at k in the block:
+//       qr_panel_kernel factors the panel rows, writes the Householder vectors as rows of
+//       Vt (row k+a = v_a over positions k0..n-1, zeros before its pivot) and as columns
+//       of Vpos (position-major), extends the block's T (H_k0 ... H_k+31 = I - V T V^T)
+//       by this panel's columns, and applies the panel's reflectors to the block's rows
+//       after the panel;
+//     VTr = V T^T and VTq = V T                     (tensor cores, K = 128)
+//     trailing rows r >= k0+128: a_r <- a_r - (a_r V) T V^T, i.e.
+//       W  = At_trail Vt^T                          (tensor cores: N = 128, K = positions)
+//       At_trail -= W VTr^T                         (tensor cores: K = 128, C read in place)
 //   then Q^T is accumulated backwards from diag(d) (d_j = sign of R_jj) one block at a
 //   time, Q^T <- Q^T (I - V T^T V^T):
-//          W   = Qt_sub Vt^T ;  Qt_sub -= W (V T)^T
+//       W = Qt_sub Vt^T ;  Qt_sub -= W VTq^T
 //   and Q = (Q^T)^T is written with its lo part.
 //
 // The panel of an n x n matrix spans up to n positions; it is spread over a thread-block
-// cluster of ceil((n-k)/1024) CTAs (<= 8 for n <= 8192), 1024 positions each, and the
-// reductions of each Householder step are combined through distributed shared memory
-// with one cluster barrier per reduction. No CTA waits on a flag: the only waits are
-// hardware cluster barriers that every CTA of the cluster reaches unconditionally.
+// cluster of ceil((n-k)/1024) CTAs (<= 8 for n <= 8192), 1024 positions each. Each
+// Householder step needs one cluster-wide reduction: the squared norm of the column
+// below the pivot and its dot products with the later panel columns are reduced
+// together (the dot products with v follow from them once the reflector is known), and
+// the partial sums are combined through distributed shared memory at one cluster
+// barrier. No CTA waits on a flag: the only waits are hardware cluster barriers that
+// every CTA of the cluster reaches unconditionally.
 //
 // Reflector convention (LAPACK larfg): for x = A[p:n, p] with alpha = x_1 and
 // sigma = ||x_2:||^2, beta = -sign(alpha) ||x||, v = x / (alpha - beta) with v_1 = 1,
@@ -48,6 +56,7 @@ namespace soap {
 namespace {
 
 constexpr int NB = 32;            // panel width
+constexpr int NBO = 128;          // block width: the trailing matrix is updated once per block
 constexpr int COLS = 1024;        // panel positions held by one CTA
 constexpr int PT = 512;           // threads per panel CTA
 constexpr int LDS = COLS + 1;     // row stride of the shared panel (bank-conflict padding)
@@ -65,16 +74,18 @@ struct PanelArgs {
   float* At;           // [batch][n][n] working P^T
   float* Vt;           // [batch][n][n] Householder vectors as rows
   float* Vt_lo;
-  float* VTr;          // [batch][n][NB]   V T^T of this panel (row = position)
-  float* VTr_lo;
-  float* VTq;          // [batch][npanel][n][NB]  V T of every panel
-  float* VTq_lo;
-  float* T;            // [batch][npanel][NB][NB]
+  float* Vpos;         // [batch][n][NBO] the block's Householder vectors, position-major
+  float* Vpos_lo;
+  float* T;            // [batch][NBO][NBO] the block's T (upper triangular)
+  float* T_lo;
+  float* Tt;           // [batch][NBO][NBO] T^T
+  float* Tt_lo;
+  float* Ypart;        // [batch][MAXC][NBO][NB] per-CTA partial products S V_panel
   uint8_t* skip;       // [batch][n]
   float* dsign;        // [batch][n] sign of R_pp (+1 for zero columns)
   const float* thresh; // [batch]
   int* status;
-  int n, k, kb, panel, npanel;
+  int n, k0, kbo, k, kb;  // block start and width, panel start and width
 };
 
 __device__ __forceinline__ float warp_sum(float v) {
@@ -91,26 +102,28 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
   extern __shared__ float sA[];  // [NB][LDS]: panel row jj (a column of P), position offset i
-  __shared__ float s_sig[2][MAXC];
-  __shared__ float s_alpha[2];
-  __shared__ float s_dot[2][MAXC][NB];
-  __shared__ float s_dtot[NB];
-  __shared__ float s_red[NWARP];
+  __shared__ float s_part[2][MAXC][NB];  // per-CTA partial [sigma | x . a_c], by source CTA
+  __shared__ float s_piv[2][NB];         // pivot-row values held by rank 0: [alpha | a_c,pivot]
+  __shared__ float s_sum[NB];
+  __shared__ float s_w[NB];              // v^T a_c
   __shared__ float s_tau[NB];
   __shared__ int s_skip[NB];
   __shared__ float s_dsign[NB];
-  __shared__ float s_gram[MAXC][NB][NB];
   __shared__ float s_T[NB][NB + 1];
+  __shared__ float s_Y[NBO][NB + 1];     // rank 0: S V_panel summed over the cluster
+  __shared__ float s_Z[NBO - NB][NB];    // (S_rest V_panel) T_panel for the in-block update
 
-  const int n = p.n, k = p.k, kb = p.kb;
+  const int n = p.n, k = p.k, kb = p.kb, k0 = p.k0, kbo = p.kbo;
+  const int jb = k - k0;                // panel offset inside its block
+  const int nrest = kbo - jb - kb;      // block rows after the panel
   const int64_t nn = (int64_t)n * n;
   float* At = p.At + (int64_t)b * nn;
   const int pos0 = k + c * COLS;  // first position held by this CTA
   const int npos = max(0, min(COLS, n - pos0));
 
-  for (int e = tid; e < npos * kb; e += PT) {
+  for (int e = tid; e < npos * NB; e += PT) {
     const int jj = e / npos, i = e % npos;
-    sA[jj * LDS + i] = At[(int64_t)(k + jj) * n + pos0 + i];
+    sA[jj * LDS + i] = jj < kb ? At[(int64_t)(k + jj) * n + pos0 + i] : 0.f;
   }
   __syncthreads();
   const float thresh = p.thresh[b];
@@ -120,35 +133,32 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     const int par = j & 1;
     // positions strictly after the pivot (pivot = local position j of rank 0)
     const int ibeg = (c == 0) ? j + 1 : 0;
-    float s = 0.f;
-    for (int i = ibeg + tid; i < npos; i += PT) {
-      const float x = sA[j * LDS + i];
-      s = fmaf(x, x, s);
+    // partial sums over this CTA: sigma (cc = j) and x . a_cc (cc > j)
+    for (int cc = j + warp; cc < kb; cc += NWARP) {
+      float d = 0.f;
+      for (int i = ibeg + lane; i < npos; i += 32) d = fmaf(sA[j * LDS + i], sA[cc * LDS + i], d);
+      d = warp_sum(d);
+      if (lane < C) cluster.map_shared_rank(&s_part[par][0][0], lane)[c * NB + cc] = d;
     }
-    s = warp_sum(s);
-    if (lane == 0) s_red[warp] = s;
-    __syncthreads();
-    if (tid == 0) {
-      float tot = 0.f;
-      for (int w = 0; w < NWARP; ++w) tot += s_red[w];
-      const float alpha = (c == 0) ? sA[j * LDS + j] : 0.f;
-      for (int q = 0; q < C; ++q) {
-        float* rs = cluster.map_shared_rank(&s_sig[par][0], q);
-        rs[c] = tot;
-        if (c == 0) *cluster.map_shared_rank(&s_alpha[par], q) = alpha;
-      }
+    if (c == 0 && tid >= j && tid < kb) {
+      const float v = sA[tid * LDS + j];  // alpha (tid == j) or a_tid at the pivot
+      for (int q = 0; q < C; ++q) cluster.map_shared_rank(&s_piv[par][0], q)[tid] = v;
     }
     cluster.sync();
+    if (tid >= j && tid < kb) {
+      float d = 0.f;
+      for (int q = 0; q < C; ++q) d += s_part[par][q][tid];
+      s_sum[tid] = d;
+    }
+    __syncthreads();
 
-    // every CTA derives the same reflector from the same reduced values
-    float sigma = 0.f;
-    for (int q = 0; q < C; ++q) sigma += s_sig[par][q];
-    const float alpha = s_alpha[par];
+    // every thread derives the same reflector from the same reduced values
+    const float sigma = s_sum[j];
+    const float alpha = s_piv[par][j];
     const float xnorm = sqrtf(fmaf(alpha, alpha, sigma));
     if (!isfinite(xnorm)) nonfinite = 1;
     const bool skip = !(xnorm > thresh);
     float tau = 0.f, v0 = 1.f, rsign = 1.f;
-    bool scale = false;
     if (!skip) {
       if (sigma == 0.f) {
         rsign = alpha < 0.f ? -1.f : 1.f;   // H = I, R_pp = alpha
@@ -157,14 +167,10 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
         v0 = alpha - beta;                   // same sign as alpha: no cancellation
         tau = (beta - alpha) / beta;
         rsign = beta < 0.f ? -1.f : 1.f;
-        scale = true;
       }
     }
-    // v after the pivot: x / v0, or 0 where H = I or x_2: = 0
-    for (int i = ibeg + tid; i < npos; i += PT) {
-      float& x = sA[j * LDS + i];
-      x = scale ? x / v0 : 0.f;
-    }
+    // v^T a_cc = a_cc,pivot + (x . a_cc) / v0, with v = x / v0 after the pivot
+    if (tau != 0.f && tid > j && tid < kb) s_w[tid] = s_piv[par][tid] + s_sum[tid] / v0;
     if (tid == 0) {
       s_tau[j] = tau;
       s_skip[j] = skip ? 1 : 0;
@@ -172,31 +178,21 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     }
     __syncthreads();
 
-    // apply H_j = I - tau v v^T to the panel rows after j
-    if (tau != 0.f && j + 1 < kb) {
-      const int piv = (c == 0) ? j : 0;  // local positions >= this take part
-      for (int jj = j + 1 + warp; jj < kb; jj += NWARP) {
-        float d = 0.f;
-        for (int i = ibeg + lane; i < npos; i += 32) d = fmaf(sA[j * LDS + i], sA[jj * LDS + i], d);
-        d = warp_sum(d);
-        if (c == 0) d += sA[jj * LDS + j];  // v_pivot = 1
-        if (lane < C) cluster.map_shared_rank(&s_dot[par][0][0], lane)[c * NB + jj] = d;
-      }
-      cluster.sync();
-      if (tid < kb && tid > j) {
-        float d = 0.f;
-        for (int q = 0; q < C; ++q) d += s_dot[par][q][tid];
-        s_dtot[tid] = d;
-      }
-      __syncthreads();
-      for (int i = piv + tid; i < npos; i += PT) {
-        const float vi = (c == 0 && i == j) ? 1.f : sA[j * LDS + i];
+    // v after the pivot (x / v0, or 0 where H = I), and H_j = I - tau v v^T on the later
+    // panel rows; every thread owns its positions
+    const int piv = (c == 0) ? j : 0;  // local positions >= this take part
+    for (int i = piv + tid; i < npos; i += PT) {
+      const bool at_pivot = (c == 0 && i == j);
+      const float vi = at_pivot ? 1.f : (tau != 0.f ? sA[j * LDS + i] / v0 : 0.f);
+      if (!at_pivot) sA[j * LDS + i] = vi;
+      if (tau != 0.f) {
         const float tv = tau * vi;
-        for (int jj = j + 1; jj < kb; ++jj) sA[jj * LDS + i] = fmaf(-tv, s_dtot[jj], sA[jj * LDS + i]);
+        for (int cc = j + 1; cc < kb; ++cc) sA[cc * LDS + i] = fmaf(-tv, s_w[cc], sA[cc * LDS + i]);
       }
-      __syncthreads();
     }
+    __syncthreads();
   }
+  if (nonfinite && tid == 0) atomicOr(p.status, kStatusQrBreakdown);
 
   // V with its unit diagonal and zeros before it (rank 0 holds the first kb positions)
   if (c == 0) {
@@ -207,8 +203,13 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     }
   }
   __syncthreads();
+
+  // V as rows of Vt (zeros at the block's positions before the panel) and as columns jb..
+  // of the block's position-major Vpos
   float* Vt = p.Vt + (int64_t)b * nn;
   float* Vt_lo = p.Vt_lo + (int64_t)b * nn;
+  float* Vpos = p.Vpos + (int64_t)b * n * NBO;
+  float* Vpos_lo = p.Vpos_lo + (int64_t)b * n * NBO;
   for (int e = tid; e < npos * kb; e += PT) {
     const int jj = e / npos, i = e % npos;
     const float v = sA[jj * LDS + i];
@@ -216,36 +217,77 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     Vt[o] = v;
     Vt_lo[o] = tf32_lo(v);
   }
-
-  // partial Gram V^T V over this CTA's positions, gathered in rank 0
-  for (int pr = warp; pr < kb * kb; pr += NWARP) {
-    const int a = pr / kb, bb = pr % kb;
-    if (bb < a) continue;
-    float g = 0.f;
-    for (int i = lane; i < npos; i += 32) g = fmaf(sA[a * LDS + i], sA[bb * LDS + i], g);
-    g = warp_sum(g);
-    if (lane == 0) cluster.map_shared_rank(&s_gram[0][0][0], 0)[(c * NB + a) * NB + bb] = g;
+  for (int i = warp; i < npos; i += NWARP) {
+    const float v = sA[lane * LDS + i];  // rows kb.. of sA are zero
+    const int64_t o = (int64_t)(pos0 + i) * NBO + jb + lane;
+    Vpos[o] = v;
+    Vpos_lo[o] = tf32_lo(v);
   }
-  if (nonfinite && tid == 0) atomicOr(p.status, kStatusQrBreakdown);
-  cluster.sync();
+  if (c == 0) {
+    for (int e = tid; e < kb * jb; e += PT) {
+      const int jj = e / jb, i = e % jb;
+      const int64_t o = (int64_t)(k + jj) * n + k0 + i;
+      Vt[o] = 0.f;
+      Vt_lo[o] = 0.f;
+    }
+    for (int e = tid; e < jb * NB; e += PT) {
+      const int64_t o = (int64_t)(k0 + e / NB) * NBO + jb + e % NB;
+      Vpos[o] = 0.f;
+      Vpos_lo[o] = 0.f;
+    }
+  }
+  __syncthreads();  // this CTA's Vt rows are read back below
+
+  // Y = S V_panel over this CTA's positions, S = the block's rows k0 .. k0+kbo-1: the block's
+  // Householder vectors so far (rows before the panel's end, from Vt) and the block rows
+  // still to be factored (from At). Warp w takes rows w, w+16, ...; lane jj column jj.
+  {
+    float y[NBO / NWARP];
+    const float* srow[NBO / NWARP];
+#pragma unroll
+    for (int u = 0; u < NBO / NWARP; ++u) {
+      const int r = warp + NWARP * u;
+      const int row = k0 + r;
+      y[u] = 0.f;
+      srow[u] = r < kbo ? ((row < k + kb) ? Vt : At) + (int64_t)row * n + pos0 : nullptr;
+    }
+    for (int i = 0; i < npos; i += 4) {  // npos is a multiple of 4
+      const float v0 = sA[lane * LDS + i], v1 = sA[lane * LDS + i + 1];
+      const float v2 = sA[lane * LDS + i + 2], v3 = sA[lane * LDS + i + 3];
+#pragma unroll
+      for (int u = 0; u < NBO / NWARP; ++u) {
+        if (!srow[u]) continue;
+        const float4 x = *reinterpret_cast<const float4*>(srow[u] + i);
+        y[u] = fmaf(x.w, v3, fmaf(x.z, v2, fmaf(x.y, v1, fmaf(x.x, v0, y[u]))));
+      }
+    }
+    float* yp = p.Ypart + ((int64_t)b * MAXC + c) * NBO * NB;
+#pragma unroll
+    for (int u = 0; u < NBO / NWARP; ++u) {
+      const int r = warp + NWARP * u;
+      if (r < kbo) yp[r * NB + lane] = y[u];
+    }
+  }
+  cluster.sync();  // orders the partials in global memory before rank 0 reads them
 
   if (c == 0) {
-    // sum the partial Grams once, then T: T_jj = tau_j, T(0:j, j) = -tau_j T(0:j, 0:j) g(0:j, j)
-    for (int e = tid; e < kb * kb; e += PT) {
-      const int l = e / kb, jj = e % kb;
-      float g = 0.f;
-      if (l < jj)
-        for (int q = 0; q < C; ++q) g += s_gram[q][l][jj];
-      s_gram[0][l][jj] = g;  // only (l < jj) entries are read below
+    // sum the partials in a fixed order
+    const float* yp = p.Ypart + (int64_t)b * MAXC * NBO * NB;
+    for (int e = tid; e < kbo * NB; e += PT) {
+      float sum = 0.f;
+      for (int q = 0; q < C; ++q) sum += yp[(int64_t)q * NBO * NB + e];
+      s_Y[e / NB][e % NB] = sum;
     }
     __syncthreads();
+    // T of the panel from its Gram matrix (rows jb.. of Y): T_jj = tau_j,
+    // T(0:j, j) = -tau_j T(0:j, 0:j) g(0:j, j)
     for (int j = 0; j < kb; ++j) {
       if (tid < kb) {
         const int i = tid;
         float t = 0.f;
         if (i < j) {
           float acc = 0.f;
-          for (int l = i; l < j; ++l) acc = fmaf(s_T[i][l], s_gram[0][l][j], acc);
+          for (int l = i; l < j; ++l) acc = fmaf(s_T[i][l], s_Y[jb + l][j], acc);
           t = -s_tau[j] * acc;
         } else if (i == j) {
           t = s_tau[j];
@@ -254,15 +296,54 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       }
       __syncthreads();
     }
-    // hand T to every CTA of the cluster
-    for (int q = 1; q < C; ++q) {
-      float* dst = cluster.map_shared_rank(&s_T[0][0], q);
-      for (int e = tid; e < NB * (NB + 1); e += PT) dst[e] = (&s_T[0][0])[e];
+    // U = X T_panel with X = V_before^T V_panel (rows 0..jb-1 of Y), in place, and
+    // Z = (S_rest V_panel) T_panel for the block rows after the panel, sent to every CTA
+    for (int r = tid; r < kbo; r += PT) {
+      if (r >= jb && r < jb + kb) continue;
+      float x[NB];
+#pragma unroll
+      for (int l = 0; l < NB; ++l) x[l] = l < kb ? s_Y[r][l] : 0.f;
+      for (int cc = 0; cc < NB; ++cc) {
+        float acc = 0.f;
+        for (int l = 0; l <= cc && l < kb; ++l) acc = fmaf(x[l], s_T[l][cc], acc);
+        if (cc >= kb) acc = 0.f;
+        if (r < jb) {
+          s_Y[r][cc] = acc;
+        } else {
+          for (int q = 0; q < C; ++q) cluster.map_shared_rank(&s_Z[0][0], q)[(r - jb - kb) * NB + cc] = acc;
+        }
+      }
     }
-    float* Tout = p.T + ((int64_t)b * p.npanel + p.panel) * NB * NB;
-    for (int e = tid; e < NB * NB; e += PT) {
-      const int i = e / NB, jj = e % NB;
-      Tout[e] = (i < kb && jj < kb) ? s_T[i][jj] : 0.f;
+    __syncthreads();
+    // the block's T: column block jb = [-T_before U ; T_panel ; 0], row block jb left of it = 0
+    float* T = p.T + (int64_t)b * NBO * NBO;
+    float* T_lo = p.T_lo + (int64_t)b * NBO * NBO;
+    float* Tt = p.Tt + (int64_t)b * NBO * NBO;
+    float* Tt_lo = p.Tt_lo + (int64_t)b * NBO * NBO;
+    for (int e = tid; e < NBO * NB; e += PT) {
+      const int r = e / NB, cc = e % NB;
+      float t = 0.f;
+      if (cc < kb) {
+        if (r < jb) {
+          float acc = 0.f;
+          for (int l = r; l < jb; ++l) acc = fmaf(T[r * NBO + l], s_Y[l][cc], acc);
+          t = -acc;
+        } else if (r < jb + kb && r - jb <= cc) {
+          t = s_T[r - jb][cc];
+        }
+      }
+      const int col = jb + cc;
+      T[r * NBO + col] = t;
+      T_lo[r * NBO + col] = tf32_lo(t);
+      Tt[col * NBO + r] = t;
+      Tt_lo[col * NBO + r] = tf32_lo(t);
+    }
+    for (int e = tid; e < NB * jb; e += PT) {
+      const int r = jb + e / jb, col = e % jb;
+      T[r * NBO + col] = 0.f;
+      T_lo[r * NBO + col] = 0.f;
+      Tt[col * NBO + r] = 0.f;
+      Tt_lo[col * NBO + r] = 0.f;
     }
     if (tid < kb) {
       p.skip[(int64_t)b * n + k + tid] = (uint8_t)s_skip[tid];
@@ -271,155 +352,18 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   }
   cluster.sync();
 
-  // V T^T (for this panel's trailing update) and V T (for the Q accumulation), position-major:
-  // warp w takes 32 positions at a time, lane a computes output column a (coalesced rows of 32)
-  float* VTr = p.VTr + (int64_t)b * n * NB;
-  float* VTr_lo = p.VTr_lo + (int64_t)b * n * NB;
-  float* VTq = p.VTq + ((int64_t)b * p.npanel + p.panel) * n * NB;
-  float* VTq_lo = p.VTq_lo + ((int64_t)b * p.npanel + p.panel) * n * NB;
-  const int a = lane;
-  for (int i0 = warp * 32; i0 < npos; i0 += NWARP * 32) {
-    const int iend = min(i0 + 32, npos);
-    for (int i = i0; i < iend; ++i) {
-      float r = 0.f, q = 0.f;
-      for (int bb = 0; bb < kb; ++bb) {
-        const float v = sA[bb * LDS + i];
-        r = fmaf((a < kb) ? s_T[a][bb] : 0.f, v, r);
-        q = fmaf((a < kb) ? s_T[bb][a] : 0.f, v, q);
-      }
-      const int64_t o = (int64_t)(pos0 + i) * NB + a;
-      VTr[o] = r;
-      VTr_lo[o] = tf32_lo(r);
-      VTq[o] = q;
-      VTq_lo[o] = tf32_lo(q);
+  // the panel's reflectors on the block rows after it: a_r -= Z_r V^T at this CTA's positions
+  for (int i = tid; i < npos; i += PT) {
+    float v[NB];
+#pragma unroll
+    for (int jj = 0; jj < NB; ++jj) v[jj] = sA[jj * LDS + i];
+    for (int r = 0; r < nrest; ++r) {
+      float acc = 0.f;
+#pragma unroll
+      for (int jj = 0; jj < NB; ++jj) acc = fmaf(s_Z[r][jj], v[jj], acc);
+      At[(int64_t)(k + kb + r) * n + pos0 + i] -= acc;
     }
   }
-}
-
-// Rank-32 update C_b <- C_b - A_b B_b^T (A: M x K, B: N x K, K <= 32, all row-major, N a
-// multiple of 4) with the lo part of the result, in exact fp32 FMAs. It streams C once
-// (read, write, lo write; 32 FMAs per element), so it is bound by HBM, not by a matrix
-// unit. A CTA owns one 128-column strip: it loads that strip's B once (k-major in shared
-// memory), then walks down the rows in 64 x 128 tiles, with the C and A tiles of the next
-// tile copied in by cp.async while the current one is computed (two stages), so ~64 KB per
-// CTA is in flight. Warp w computes rows 8w..8w+7, lane l columns 4l..4l+3; every global
-// access to C is a 16-byte vector and a warp covers 512 contiguous bytes of a row.
-constexpr int RU_BM = 64, RU_BN = 128, RU_STAGES = 2;
-constexpr int RU_SMEM = (RU_STAGES * RU_BM * RU_BN + RU_STAGES * RU_BM * NB + NB * RU_BN) * 4;
-
-__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src, bool valid) {
-  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(gmem_src), "r"(valid ? 16 : 0)
-               : "memory");
-}
-
-__global__ void __launch_bounds__(256, 2)
-    rank_update_kernel(int M, int N, int K, const float* __restrict__ A, int64_t lda, int64_t sa,
-                       const float* __restrict__ B, int64_t ldb, int64_t sb, float* C, float* C_lo, int64_t ldc,
-                       int64_t sc) {
-  extern __shared__ float4 ru_smem[];
-  float* Cs = reinterpret_cast<float*>(ru_smem);     // [stage][RU_BM][RU_BN]
-  float* As = Cs + RU_STAGES * RU_BM * RU_BN;        // [stage][RU_BM][NB]
-  float* Bs = As + RU_STAGES * RU_BM * NB;           // [NB][RU_BN]
-  const int b = blockIdx.z;
-  const int c0 = blockIdx.x * RU_BN;
-  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-  const float* Ab = A + (int64_t)b * sa;
-  const float* Bb = B + (int64_t)b * sb;
-  float* Cb = C + (int64_t)b * sc;
-  float* Lb = C_lo + (int64_t)b * sc;
-  const int ntiles = (M + RU_BM - 1) / RU_BM;
-  const int col = c0 + 4 * lane;
-
-  // one 64 x 128 tile of C and its 64 x 32 slice of A into stage st (zero-filled past the edges)
-  auto issue = [&](int tile, int st) {
-    const int r0 = tile * RU_BM;
-    float* cs = Cs + st * RU_BM * RU_BN;
-    float* as = As + st * RU_BM * NB;
-    for (int e = tid; e < RU_BM * (RU_BN / 4); e += 256) {
-      const int r = e / (RU_BN / 4), q = e % (RU_BN / 4);
-      const bool ok = (r0 + r < M) && (c0 + 4 * q < N);
-      cp_async16(cs + r * RU_BN + 4 * q, ok ? Cb + (int64_t)(r0 + r) * ldc + c0 + 4 * q : Cb, ok);
-    }
-    for (int e = tid; e < RU_BM * (NB / 4); e += 256) {
-      const int r = e / (NB / 4), q = e % (NB / 4);
-      const bool ok = (r0 + r < M) && (4 * q < K);
-      cp_async16(as + r * NB + 4 * q, ok ? Ab + (int64_t)(r0 + r) * lda + 4 * q : Ab, ok);
-    }
-    asm volatile("cp.async.commit_group;" ::: "memory");
-  };
-
-  int tile = blockIdx.y;
-  if (tile < ntiles) issue(tile, 0);
-  for (int e = tid; e < RU_BN * NB; e += 256) {
-    const int cc = e / NB, kk = e % NB;
-    Bs[kk * RU_BN + cc] = (c0 + cc < N && kk < K) ? Bb[(int64_t)(c0 + cc) * ldb + kk] : 0.f;
-  }
-  for (int it = 0; tile < ntiles; ++it, tile += gridDim.y) {
-    const int st = it & 1;
-    const int next = tile + gridDim.y;
-    if (next < ntiles) {
-      issue(next, st ^ 1);
-      asm volatile("cp.async.wait_group 1;" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-    }
-    __syncthreads();
-    const float* cs = Cs + st * RU_BM * RU_BN;
-    const float* as = As + st * RU_BM * NB;
-    float acc[8][4];
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
-#pragma unroll 4
-    for (int kk = 0; kk < NB; ++kk) {
-      const float4 bv = *reinterpret_cast<const float4*>(&Bs[kk * RU_BN + 4 * lane]);
-      const float bb[4] = {bv.x, bv.y, bv.z, bv.w};
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const float a = as[(8 * w + i) * NB + kk];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a, bb[j], acc[i][j]);
-      }
-    }
-    const int r0 = tile * RU_BM;
-    if (col < N) {
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int r = r0 + 8 * w + i;
-        if (r >= M) break;
-        const float4 c = *reinterpret_cast<const float4*>(&cs[(8 * w + i) * RU_BN + 4 * lane]);
-        float4 o;
-        o.x = c.x - acc[i][0];
-        o.y = c.y - acc[i][1];
-        o.z = c.z - acc[i][2];
-        o.w = c.w - acc[i][3];
-        *reinterpret_cast<float4*>(Cb + (int64_t)r * ldc + col) = o;
-        *reinterpret_cast<float4*>(Lb + (int64_t)r * ldc + col) =
-            make_float4(tf32_lo(o.x), tf32_lo(o.y), tf32_lo(o.z), tf32_lo(o.w));
-      }
-    }
-    __syncthreads();  // this stage is refilled by the next iteration's prefetch
-  }
-}
-
-cudaError_t rank_update(int M, int N, int K, int batch, const float* A, int64_t lda, int64_t sa, const float* B,
-                        int64_t ldb, int64_t sb, float* C, float* C_lo, int64_t ldc, int64_t sc, cudaStream_t s) {
-  if (M <= 0 || N <= 0) return cudaSuccess;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(rank_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, RU_SMEM);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
-  ProfScope prof(kFamQrUpdate, 2.0 * M * N * (double)K * batch, 12.0 * M * (double)N * batch, s);
-  const int strips = (N + RU_BN - 1) / RU_BN, ntiles = (M + RU_BM - 1) / RU_BM;
-  // about two waves of 2 CTAs per SM; each CTA walks ntiles / gridDim.y row tiles
-  const int want = std::max(1, (2 * 2 * 152) / std::max(1, strips * batch));
-  dim3 grid(strips, std::min(ntiles, want), batch);
-  rank_update_kernel<<<grid, 256, RU_SMEM, s>>>(M, N, K, A, lda, sa, B, ldb, sb, C, C_lo, ldc, sc);
-  return cudaGetLastError();
 }
 
 // ||P_b||_F: per-chunk partial sums in double, then tol * sqrt(sum)
@@ -491,13 +435,19 @@ struct Workspace {
   float* At_lo;
   float* Vt;
   float* Vt_lo;
-  float* VTq;
+  float* VTq;     // [batch][nblock][n][NBO] V T of every block (kept for the Q accumulation)
   float* VTq_lo;
-  float* VTr;
+  float* VTr;     // [batch][n][NBO] V T^T of the current block
   float* VTr_lo;
-  float* W;
+  float* Vpos;    // [batch][n][NBO]
+  float* Vpos_lo;
+  float* W;       // [batch][n][NBO]
   float* W_lo;
-  float* T;
+  float* T;       // [batch][NBO][NBO], and T^T, each with its lo part
+  float* T_lo;
+  float* Tt;
+  float* Tt_lo;
+  float* Ypart;   // [batch][MAXC][NBO][NB]
   float* thresh;
   float* dsign;
   double* part;
@@ -506,7 +456,7 @@ struct Workspace {
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 Workspace carve(void* base, int n, int batch, size_t* total) {
-  const int npanel = (n + NB - 1) / NB;
+  const int nblock = (n + NBO - 1) / NBO;
   size_t off = 0;
   auto take = [&](size_t bytes) {
     size_t o = off;
@@ -514,20 +464,22 @@ Workspace carve(void* base, int n, int batch, size_t* total) {
     return o;
   };
   const size_t mat = (size_t)batch * n * n * sizeof(float);
-  const size_t pan = (size_t)batch * npanel * n * NB * sizeof(float);
-  const size_t thin = (size_t)batch * n * NB * sizeof(float);
+  const size_t blocks = (size_t)batch * nblock * n * NBO * sizeof(float);
+  const size_t thin = (size_t)batch * n * NBO * sizeof(float);
+  const size_t tsq = (size_t)batch * NBO * NBO * sizeof(float);
   const size_t oAt = take(mat), oAtl = take(mat), oVt = take(mat), oVtl = take(mat);
-  const size_t oVq = take(pan), oVql = take(pan), oVr = take(thin), oVrl = take(thin);
-  const size_t oW = take(thin), oWl = take(thin);
-  const size_t oT = take((size_t)batch * npanel * NB * NB * sizeof(float));
+  const size_t oVq = take(blocks), oVql = take(blocks), oVr = take(thin), oVrl = take(thin);
+  const size_t oVp = take(thin), oVpl = take(thin), oW = take(thin), oWl = take(thin);
+  const size_t oT = take(tsq), oTl = take(tsq), oTt = take(tsq), oTtl = take(tsq);
+  const size_t oY = take((size_t)batch * MAXC * NBO * NB * sizeof(float));
   const size_t oth = take((size_t)batch * sizeof(float));
   const size_t osg = take((size_t)batch * n * sizeof(float));
   const size_t opart = take((size_t)batch * NORM_CHUNKS * sizeof(double));
   if (total) *total = off;
   char* c = (char*)base;
   auto f = [&](size_t o) { return (float*)(c + o); };
-  return Workspace{f(oAt), f(oAtl), f(oVt), f(oVtl), f(oVq), f(oVql), f(oVr), f(oVrl),
-                   f(oW),  f(oWl),  f(oT),  f(oth),  f(osg), (double*)(c + opart)};
+  return Workspace{f(oAt), f(oAtl), f(oVt), f(oVtl), f(oVq), f(oVql), f(oVr), f(oVrl), f(oVp), f(oVpl),
+                   f(oW),  f(oWl),  f(oT),  f(oTl),  f(oTt), f(oTtl), f(oY),  f(oth),  f(osg), (double*)(c + opart)};
 }
 
 TcOperand op(const float* hi, const float* lo, int64_t ld, int64_t stride, int batch) {
@@ -563,8 +515,8 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     Qt = w.At;
     Qt_lo = w.At_lo;
   }
-  const int npanel = (n + NB - 1) / NB;
-  const int64_t nn = (int64_t)n * n;
+  const int nblock = (n + NBO - 1) / NBO;
+  const int64_t nn = (int64_t)n * n, thin = (int64_t)n * NBO, vq_stride = (int64_t)nblock * thin;
   cudaError_t e;
 
   {
@@ -579,43 +531,57 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
   e = cudaFuncSetAttribute(qr_panel_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
 
-  const int64_t pan_stride = (int64_t)npanel * n * NB;
-  for (int pi = 0; pi < npanel; ++pi) {
-    const int k = pi * NB, kb = std::min(NB, n - k);
-    const int C = (n - k + COLS - 1) / COLS;
-    PanelArgs a{w.At, w.Vt, w.Vt_lo, w.VTr, w.VTr_lo, w.VTq, w.VTq_lo, w.T, skip, w.dsign, w.thresh, status,
-                n, k, kb, pi, npanel};
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(C, batch, 1);
-    cfg.blockDim = dim3(PT, 1, 1);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = C;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    {
-      // Householder work on the kb x (n-k) panel plus V T^T and V T: ~(4 kb^2 + 4 kb^2) (n-k)
-      ProfScope prof(kFamQrPanel, 8.0 * (n - k) * kb * kb * batch, 24.0 * (n - k) * kb * batch, s);
-      e = cudaLaunchKernelEx(&cfg, qr_panel_kernel, a);
+  for (int blk = 0; blk < nblock; ++blk) {
+    const int k0 = blk * NBO, kbo = std::min(NBO, n - k0), m = n - k0;
+    for (int k = k0; k < k0 + kbo; k += NB) {
+      const int kb = std::min(NB, n - k);
+      const int C = (n - k + COLS - 1) / COLS;
+      PanelArgs a{w.At, w.Vt, w.Vt_lo, w.Vpos, w.Vpos_lo, w.T, w.T_lo, w.Tt, w.Tt_lo, w.Ypart, skip, w.dsign,
+                  w.thresh, status, n, k0, kbo, k, kb};
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(C, batch, 1);
+      cfg.blockDim = dim3(PT, 1, 1);
+      cfg.dynamicSmemBytes = smem;
+      cfg.stream = s;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = C;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      {
+        // Householder steps on the kb x (n-k) panel (~4 kb^2 (n-k)), S V over kbo rows
+        // (2 kbo kb (n-k)) and the in-block update (2 kb (kbo-kb) (n-k))
+        const double mk = (double)(n - k) * batch;
+        ProfScope prof(kFamQrPanel, (4.0 * kb * kb + 4.0 * kbo * kb) * mk, 4.0 * (3.0 * kb + 2.0 * kbo) * mk, s);
+        e = cudaLaunchKernelEx(&cfg, qr_panel_kernel, a);
+      }
+      if (e != cudaSuccess) return e;
     }
+    // VTq = V T (the Q accumulation) and VTr = V T^T (this block's trailing update)
+    float* vq = w.VTq + (int64_t)blk * thin + (int64_t)k0 * NBO;
+    float* vq_lo = w.VTq_lo + (int64_t)blk * thin + (int64_t)k0 * NBO;
+    const TcOperand vpos = op(w.Vpos + (int64_t)k0 * NBO, w.Vpos_lo + (int64_t)k0 * NBO, NBO, thin, batch);
+    e = gemm_tc_nt(m, kbo, kbo, batch, vpos, op(w.Tt, w.Tt_lo, NBO, NBO * NBO, batch),
+                   out(vq, vq_lo, NBO, vq_stride, 1.f, 0.f, status), s, kFamQrUpdate);
     if (e != cudaSuccess) return e;
-
-    const int nc = n - k - kb;  // trailing rows of At (columns of P)
+    const int nc = n - k0 - kbo;  // trailing rows of At (columns of P)
     if (nc <= 0) continue;
-    const int m = n - k;        // positions from the panel's first pivot on
-    const int64_t tr = (int64_t)(k + kb) * n + k;
-    // W1 = At_trail Vt^T   (nc x kb)
-    e = gemm_tc_nt(nc, kb, m, batch, op(w.At + tr, w.At_lo + tr, n, nn, batch),
-                   op(w.Vt + (int64_t)k * n + k, w.Vt_lo + (int64_t)k * n + k, n, nn, batch),
-                   out(w.W, w.W_lo, NB, (int64_t)n * NB, 1.f, 0.f, status), s);
+    e = gemm_tc_nt(m, kbo, kbo, batch, vpos, op(w.T, w.T_lo, NBO, NBO * NBO, batch),
+                   out(w.VTr + (int64_t)k0 * NBO, w.VTr_lo + (int64_t)k0 * NBO, NBO, thin, 1.f, 0.f, status), s,
+                   kFamQrUpdate);
     if (e != cudaSuccess) return e;
-    // At_trail -= W1 (V T^T)^T
-    e = rank_update(nc, m, kb, batch, w.W, NB, (int64_t)n * NB, w.VTr + (int64_t)k * NB, NB, (int64_t)n * NB,
-                    w.At + tr, w.At_lo + tr, n, nn, s);
+    // W = At_trail Vt^T over positions k0.. (nc x kbo)
+    const int64_t tr = (int64_t)(k0 + kbo) * n;
+    e = gemm_tc_nt(nc, kbo, m, batch, op(w.At + tr + k0, w.At_lo + tr + k0, n, nn, batch),
+                   op(w.Vt + (int64_t)k0 * n + k0, w.Vt_lo + (int64_t)k0 * n + k0, n, nn, batch),
+                   out(w.W, w.W_lo, NBO, thin, 1.f, 0.f, status), s, kFamQrUpdate);
+    if (e != cudaSuccess) return e;
+    // At_trail -= W VTr^T at positions k0+kbo.. (the earlier positions of these rows are R's)
+    e = gemm_tc_nt(nc, nc, kbo, batch, op(w.W, w.W_lo, NBO, thin, batch),
+                   op(w.VTr + (int64_t)(k0 + kbo) * NBO, w.VTr_lo + (int64_t)(k0 + kbo) * NBO, NBO, thin, batch),
+                   out(w.At + tr + k0 + kbo, w.At_lo + tr + k0 + kbo, n, nn, -1.f, 1.f, status), s, kFamQrUpdate);
     if (e != cudaSuccess) return e;
   }
 
@@ -627,18 +593,19 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  for (int pi = npanel - 1; pi >= 0; --pi) {
-    const int k = pi * NB, kb = std::min(NB, n - k), m = n - k;
-    const int64_t sub = (int64_t)k * n + k;
-    // W = Qt_sub Vt^T  (m x kb)
-    e = gemm_tc_nt(m, kb, m, batch, op(Qt + sub, Qt_lo + sub, n, nn, batch),
-                   op(w.Vt + sub, w.Vt_lo + sub, n, nn, batch), out(w.W, w.W_lo, NB, (int64_t)n * NB, 1.f, 0.f, status),
-                   s);
+  for (int blk = nblock - 1; blk >= 0; --blk) {
+    const int k0 = blk * NBO, kbo = std::min(NBO, n - k0), m = n - k0;
+    const int64_t sub = (int64_t)k0 * n + k0;
+    // W = Qt_sub Vt^T  (m x kbo)
+    e = gemm_tc_nt(m, kbo, m, batch, op(Qt + sub, Qt_lo + sub, n, nn, batch),
+                   op(w.Vt + sub, w.Vt_lo + sub, n, nn, batch), out(w.W, w.W_lo, NBO, thin, 1.f, 0.f, status), s,
+                   kFamQrUpdate);
     if (e != cudaSuccess) return e;
-    // Qt_sub -= W (V T)^T
-    const int64_t vq = (int64_t)pi * n * NB + (int64_t)k * NB;
-    e = rank_update(m, m, kb, batch, w.W, NB, (int64_t)n * NB, w.VTq + vq, NB, pan_stride, Qt + sub, Qt_lo + sub, n,
-                    nn, s);
+    // Qt_sub -= W VTq^T
+    const int64_t vq = (int64_t)blk * thin + (int64_t)k0 * NBO;
+    e = gemm_tc_nt(m, m, kbo, batch, op(w.W, w.W_lo, NBO, thin, batch),
+                   op(w.VTq + vq, w.VTq_lo + vq, NBO, vq_stride, batch),
+                   out(Qt + sub, Qt_lo + sub, n, nn, -1.f, 1.f, status), s, kFamQrUpdate);
     if (e != cudaSuccess) return e;
   }
   if (Q) {

@@ -31,8 +31,8 @@ struct ClassState {
   bool left = false, right = false;
   int count = 0;
   std::vector<int> members;
-  float* Gc = nullptr;
-  float* Mhat = nullptr;
+  float* Gc = nullptr;    // G (copy of the caller's gradient); [G | M_hat] unless `tr`
+  float* Mhat = nullptr;  // first moment in the original basis, in the working orientation
   float* V = nullptr;
   float* L = nullptr;
   float* QL = nullptr;
@@ -41,11 +41,15 @@ struct ClassState {
   uint8_t* skipL = nullptr;
   uint8_t* skipR = nullptr;
   size_t ptr_offset = 0;  // index of this class's params pointers in the pointer table
-  // tensor-core path (both sides preconditioned): operand copies and their lo parts
+  // tensor-core path: operand copies and their lo parts
   bool tc = false;
-  float* GM_lo = nullptr;  // lo parts of [G copy | M_hat]
-  float* Gt = nullptr;
+  // working orientation transposed: a class preconditioned on its left only runs as the
+  // right-only problem of G^T, and keeps M_hat and v as M_hat^T and v^T
+  bool tr = false;
+  float* Gc_lo = nullptr;  // lo parts of the Gc arena
+  float* Gt = nullptr;     // G^T; [G^T | M_hat^T] if `tr`
   float* Gt_lo = nullptr;
+  float* Mhat_lo = nullptr;
   float* L_lo = nullptr;
   float* R_lo = nullptr;
   float* QL_lo = nullptr;
@@ -207,6 +211,9 @@ soap::TcEpilogue epi(soap_handle h, float* C, int64_t ldc, int64_t c_stride, flo
 //   S6  N = Adam(G', m', v)
 //   S7  Z^T = (N Q_R^T)^T            A = N,     B = Q_R      (transposed epilogue)
 //   S8  W <- (1 - lr wd) W - lr Q_L Z  A = Q_L, B = Z^T      (epilogue into W)
+// One-sided classes take the same route with one rotation on each side of Adam (a left-only
+// class as the right-only problem of G^T). Classes whose rows or columns are not a multiple
+// of 4 (rows of an operand must be 16-byte multiples for TMA) run on CUDA cores.
 soap_status_t prepare_class(soap_handle h, ClassState& c, const float* const* d_grads, cudaStream_t s) {
   const soap_hparams& hp = h->hp;
   const int B = c.count, m = (int)c.rows, n = (int)c.cols;
@@ -224,18 +231,19 @@ soap_status_t prepare_class(soap_handle h, ClassState& c, const float* const* d_
                               strided_mut(c.R, n, nn), B, s));
     return SOAP_OK;
   }
-  const int64_t cls = (int64_t)B * mn;
-  SOAP_CUDA(h, soap::momentum_split(d_grads, c.Gc, c.GM_lo, c.Gt, c.Gt_lo, c.Mhat, c.GM_lo + cls, m, n, B, hp.beta1,
+  SOAP_CUDA(h, soap::momentum_split(d_grads, c.Gc, c.Gc_lo, c.Gt, c.Gt_lo, c.Mhat, c.Mhat_lo, m, n, B, hp.beta1, c.tr,
                                     h->d_status, s));
   if (c.basis_dirty) {
-    SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, B, s));
-    SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, n, B, s));
+    if (c.left) SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, B, s));
+    if (c.right) SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, n, B, s));
     c.basis_dirty = false;
   }
-  SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(c.Gc, c.GM_lo, n, mn, B), opnd(c.Gc, c.GM_lo, n, mn, B),
-                                epi(h, c.L, m, mm, c.L_lo, 0, 1.f - fb, fb), s));
-  SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(c.Gt, c.Gt_lo, m, mn, B), opnd(c.Gt, c.Gt_lo, m, mn, B),
-                                epi(h, c.R, n, nn, c.R_lo, 0, 1.f - fb, fb), s));
+  if (c.left)
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(c.Gc, c.Gc_lo, n, mn, B), opnd(c.Gc, c.Gc_lo, n, mn, B),
+                                  epi(h, c.L, m, mm, c.L_lo, 0, 1.f - fb, fb), s));
+  if (c.right)
+    SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(c.Gt, c.Gt_lo, m, mn, B), opnd(c.Gt, c.Gt_lo, m, mn, B),
+                                  epi(h, c.R, n, nn, c.R_lo, 0, 1.f - fb, fb), s));
   return SOAP_OK;
 }
 
@@ -299,10 +307,34 @@ soap_status_t rotate_update_class(soap_handle h, ClassState& c, float* const* d_
   const int64_t mn = (int64_t)m * n, mm = (int64_t)m * m, nn = (int64_t)n * n;
   using soap::strided;
   using soap::strided_mut;
+  if (c.tc && !(c.left && c.right)) {
+    // one preconditioned side, as a right-sided problem in the working orientation: the
+    // rr x cc matrices X = G (or G^T) with basis Q = Q_R (or Q_L)
+    //   [G' | m'] = [X | M_hat] Q    A = [X | M_hat],  B = Q^T   (batch 2B)
+    //   N = Adam(G', m', v)
+    //   W <- (1 - lr wd) W - lr N Q^T  A = N,  B = Q   (epilogue into W, transposed if c.tr)
+    const int rr = c.tr ? n : m, cc = c.tr ? m : n;
+    const int64_t cls = (int64_t)B * mn, qq = (int64_t)cc * cc;
+    const float* X = c.tr ? c.Gt : c.Gc;
+    const float* X_lo = c.tr ? c.Gt_lo : c.Gc_lo;
+    const float* Q = c.tr ? c.QL : c.QR;
+    const float* Q_lo = c.tr ? c.QL_lo : c.QR_lo;
+    const float* Qt = c.tr ? c.QLt : c.QRt;
+    const float* Qt_lo = c.tr ? c.QLt_lo : c.QRt_lo;
+    SOAP_CUDA(h, soap::gemm_tc_nt(rr, cc, cc, 2 * B, opnd(X, X_lo, cc, mn, 2 * B), opnd(Qt, Qt_lo, cc, qq, B),
+                                  epi(h, h->Gp, cc, mn, nullptr, 0, 1.f, 0.f), s));
+    const uint8_t* skip = hp.guard ? (c.tr ? c.skipL : c.skipR) : nullptr;
+    SOAP_CUDA(h, soap::adam_in_basis(h->Gp, h->Gp + cls, c.V, rr, cc, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2, nullptr,
+                                     skip, h->N_lo, h->d_status, s));
+    soap::TcEpilogue ew = epi(h, nullptr, n, 0, nullptr, c.tr ? 1 : 0, -h->lr, 1.f - h->lr * h->wd);
+    ew.C_ptrs = d_params;
+    SOAP_CUDA(h, soap::gemm_tc_nt(rr, cc, cc, B, opnd(h->Gp, h->N_lo, cc, mn, B), opnd(Q, Q_lo, cc, qq, B), ew, s));
+    return SOAP_OK;
+  }
   if (c.tc) {
     const int64_t cls = (int64_t)B * mn;
     // rotations of the gradient and of the momentum in one launch each (batch 2B)
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, 2 * B, opnd(c.Gc, c.GM_lo, n, mn, 2 * B), opnd(c.QRt, c.QRt_lo, n, nn, B),
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, 2 * B, opnd(c.Gc, c.Gc_lo, n, mn, 2 * B), opnd(c.QRt, c.QRt_lo, n, nn, B),
                                   epi(h, h->YMt, m, mn, h->YMt_lo, 1, 1.f, 0.f), s));
     SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, 2 * B, opnd(c.QLt, c.QLt_lo, m, mm, B),
                                   opnd(h->YMt, h->YMt_lo, m, mn, 2 * B), epi(h, h->Gp, n, mn, nullptr, 0, 1.f, 0.f), s));
@@ -440,14 +472,21 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
     const size_t mn = (size_t)c.count * c.rows * c.cols;
     c.ptr_offset = off;
     off += 2 * (size_t)c.count;
-    c.tc = c.left && c.right && (c.rows % 4 == 0) && (c.cols % 4 == 0);
-    if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gc, 2 * mn * 4);  // [G copy | M_hat]
-    c.Mhat = c.Gc ? c.Gc + mn : nullptr;
+    // tensor-core operands are read with TMA: rows of both G and G^T must be 16-byte multiples
+    c.tc = (c.left || c.right) && (c.rows % 4 == 0) && (c.cols % 4 == 0);
+    c.tr = c.tc && c.left && !c.right;
+    // the arena holding M_hat directly after G (or G^T), so that one batch-2B product rotates both
+    const size_t ga = c.tr ? mn : 2 * mn, ta = c.tr ? 2 * mn : mn;
+    if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gc, (c.tc ? ga : 2 * mn) * 4);
     if (e == cudaSuccess) e = dalloc(h, (void**)&c.V, mn * 4);
     if (c.tc) {
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.GM_lo, 2 * mn * 4);
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gt, mn * 4);
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gt_lo, mn * 4);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gc_lo, ga * 4);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gt, ta * 4);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gt_lo, ta * 4);
+    }
+    if (e == cudaSuccess) {
+      c.Mhat = c.tr ? c.Gt + mn : c.Gc + mn;
+      c.Mhat_lo = !c.tc ? nullptr : c.tr ? c.Gt_lo + mn : c.Gc_lo + mn;
     }
     if (c.left) {
       const size_t mm = (size_t)c.count * c.rows * c.rows;
@@ -516,19 +555,25 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->fork_ev, cudaEventDisableTiming);
   }
   h->nptrs = off;
-  bool any_tc = false;
-  for (auto& c : h->classes) any_tc |= c.tc;
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->X1, ws_mat * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->X2, ws_mat * 4);
+  // workspaces: [G' | m'] for every class; N's lo part for tensor-core classes; the
+  // intermediate products of two-sided tensor-core classes; X1/X2 for CUDA-core classes and
+  // for single-matrix state reads and writes
+  size_t ws_tc = 0, ws_two = 0, ws_x = 0;
+  for (auto& c : h->classes) {
+    const size_t mn = (size_t)c.count * c.rows * c.cols;
+    if (c.tc) ws_tc = std::max(ws_tc, mn);
+    if (c.tc && c.left && c.right) ws_two = std::max(ws_two, mn);
+    ws_x = std::max(ws_x, c.tc ? (size_t)(c.rows * c.cols) : mn);
+  }
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->X1, ws_x * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->X2, ws_x * 4);
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->Gp, 2 * ws_mat * 4);
   h->Mp = h->Gp ? h->Gp + ws_mat : nullptr;
-  if (any_tc) {
-    if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt, 2 * ws_mat * 4);
-    if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt_lo, 2 * ws_mat * 4);
-    if (e == cudaSuccess) e = dalloc(h, (void**)&h->N_lo, ws_mat * 4);
-    if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt, ws_mat * 4);
-    if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt_lo, ws_mat * 4);
-  }
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->N_lo, ws_tc * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt, 2 * ws_two * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt_lo, 2 * ws_two * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt, ws_two * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt_lo, ws_two * 4);
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_status, sizeof(int));
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_ptrs, h->nptrs * sizeof(void*));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&h->h_status, sizeof(int));
@@ -547,7 +592,7 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
   for (auto& c : h->classes) {
     const size_t mn = (size_t)c.count * c.rows * c.cols;
     if (e == cudaSuccess) e = cudaMemset(c.Mhat, 0, mn * 4);
-    if (c.tc && e == cudaSuccess) e = cudaMemset(c.GM_lo, 0, 2 * mn * 4);
+    if (c.tc && e == cudaSuccess) e = cudaMemset(c.Mhat_lo, 0, mn * 4);
     if (e == cudaSuccess) e = cudaMemset(c.V, 0, mn * 4);
     if (c.left) {
       if (e == cudaSuccess) e = cudaMemset(c.L, 0, (size_t)c.count * c.rows * c.rows * 4);
@@ -689,26 +734,44 @@ soap_status_t soap_state_get(soap_handle h, int32_t idx, int32_t which, void* ds
   if (bytes == 0 || !dst) return fail(h, SOAP_ERR_INVALID_ARG, "soap_state_get: no such state piece");
   DeviceGuard g(h->device);
   cudaStream_t s = (cudaStream_t)stream_;
+  const auto [ci, slot] = h->loc[idx];
+  ClassState& c = h->classes[ci];
+  const int m = (int)c.rows, nc = (int)c.cols;
+  const int64_t mn = (int64_t)m * nc;
+  if (c.tr && (which == SOAP_STATE_V || which == SOAP_STATE_MHAT)) {
+    // stored transposed (n x m): hand out the m x n matrix
+    SOAP_CUDA(h, soap::transpose((const float*)state_ptr(h, idx, which), h->X1, nc, m, 1, s));
+    SOAP_CUDA(h, cudaMemcpyAsync(dst, h->X1, bytes, cudaMemcpyDefault, s));
+    return SOAP_OK;
+  }
   if (which != SOAP_STATE_M) {
     SOAP_CUDA(h, cudaMemcpyAsync(dst, state_ptr(h, idx, which), bytes, cudaMemcpyDefault, s));
     return SOAP_OK;
   }
   // m = Q_L^T M_hat Q_R, computed into the workspace
-  const auto [ci, slot] = h->loc[idx];
-  ClassState& c = h->classes[ci];
-  const int m = (int)c.rows, nc = (int)c.cols;
-  const int64_t mn = (int64_t)m * nc;
   const float* x = c.Mhat + slot * mn;
+  if (c.tc && c.basis_dirty) {
+    if (c.left) SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, c.count, s));
+    if (c.right) SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, nc, c.count, s));
+    c.basis_dirty = false;
+  }
+  if (c.tc && !(c.left && c.right)) {
+    // the step's product [X | M_hat] Q for this matrix alone (bit-identical), written in the
+    // original orientation
+    const int rr = c.tr ? nc : m, cc = c.tr ? m : nc;
+    const int64_t qq = (int64_t)cc * cc;
+    const float* Qt = (c.tr ? c.QLt : c.QRt) + slot * qq;
+    const float* Qt_lo = (c.tr ? c.QLt_lo : c.QRt_lo) + slot * qq;
+    SOAP_CUDA(h, soap::gemm_tc_nt(rr, cc, cc, 1, opnd(x, c.Mhat_lo + slot * mn, cc, mn, 1), opnd(Qt, Qt_lo, cc, qq, 1),
+                                  epi(h, h->Gp, c.tr ? rr : cc, mn, nullptr, c.tr ? 1 : 0, 1.f, 0.f), s));
+    SOAP_CUDA(h, cudaMemcpyAsync(dst, h->Gp, bytes, cudaMemcpyDefault, s));
+    return SOAP_OK;
+  }
   if (c.tc) {
     // the same tensor-core products, on the same operands, as the step's rotation of M_hat:
     // bit-identical to the m the last step used
-    const int64_t mm = (int64_t)m * m, nn = (int64_t)nc * nc, cls = (int64_t)c.count * mn;
-    if (c.basis_dirty) {
-      SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, c.count, s));
-      SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, nc, c.count, s));
-      c.basis_dirty = false;
-    }
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, nc, nc, 1, opnd(x, c.GM_lo + cls + slot * mn, nc, mn, 1),
+    const int64_t mm = (int64_t)m * m, nn = (int64_t)nc * nc;
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, nc, nc, 1, opnd(x, c.Mhat_lo + slot * mn, nc, mn, 1),
                                   opnd(c.QRt + slot * nn, c.QRt_lo + slot * nn, nc, nn, 1),
                                   epi(h, h->X1, m, mn, h->X2, 1, 1.f, 0.f), s));
     SOAP_CUDA(h, soap::gemm_tc_nt(m, nc, m, 1, opnd(c.QLt + slot * mm, c.QLt_lo + slot * mm, m, mm, 1),
@@ -738,29 +801,31 @@ soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const vo
   if (bytes == 0 || !src) return fail(h, SOAP_ERR_INVALID_ARG, "soap_state_set: no such state piece");
   DeviceGuard g(h->device);
   cudaStream_t s = (cudaStream_t)stream_;
-  if (which != SOAP_STATE_M) {
-    SOAP_CUDA(h, cudaMemcpyAsync(state_ptr(h, idx, which), src, bytes, cudaMemcpyDefault, s));
-    ClassState& cs = h->classes[h->loc[idx].first];
-    if (which == SOAP_STATE_QL || which == SOAP_STATE_QR) cs.basis_dirty = true;
-    if (which == SOAP_STATE_MHAT && cs.tc) {
-      const int64_t mn = cs.rows * cs.cols;
-      SOAP_CUDA(h, soap::split_tf32(cs.Mhat + h->loc[idx].second * mn, nullptr,
-                                    cs.GM_lo + cs.count * mn + h->loc[idx].second * mn, mn, s));
-    }
-    return SOAP_OK;
-  }
-  // M_hat = Q_L m Q_R^T
   const auto [ci, slot] = h->loc[idx];
   ClassState& c = h->classes[ci];
   const int m = (int)c.rows, nc = (int)c.cols;
   const int64_t mn = (int64_t)m * nc;
   float* dstm = c.Mhat + slot * mn;
+  if (which != SOAP_STATE_M) {
+    if (c.tr && (which == SOAP_STATE_V || which == SOAP_STATE_MHAT)) {
+      // stored transposed (n x m)
+      SOAP_CUDA(h, cudaMemcpyAsync(h->X1, src, bytes, cudaMemcpyDefault, s));
+      SOAP_CUDA(h, soap::transpose(h->X1, (float*)state_ptr(h, idx, which), m, nc, 1, s));
+    } else {
+      SOAP_CUDA(h, cudaMemcpyAsync(state_ptr(h, idx, which), src, bytes, cudaMemcpyDefault, s));
+    }
+    if (which == SOAP_STATE_QL || which == SOAP_STATE_QR) c.basis_dirty = true;
+    if (which == SOAP_STATE_MHAT && c.tc)
+      SOAP_CUDA(h, soap::split_tf32(dstm, nullptr, c.Mhat_lo + slot * mn, mn, s));
+    return SOAP_OK;
+  }
+  // M_hat = Q_L m Q_R^T
   using soap::strided;
   using soap::strided_mut;
   SOAP_CUDA(h, cudaMemcpyAsync(h->Gp, src, bytes, cudaMemcpyDefault, s));
   const float* x = h->Gp;
   if (c.left) {
-    float* out = c.right ? h->X1 : dstm;
+    float* out = (c.right || c.tr) ? h->X1 : dstm;
     SOAP_CUDA(h, soap::gemm(false, false, m, nc, m, 1.f, strided(c.QL + (int64_t)slot * m * m, m, 0), strided(x, nc, 0),
                             0.f, strided_mut(out, nc, 0), 1, s));
     x = out;
@@ -768,10 +833,12 @@ soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const vo
   if (c.right) {
     SOAP_CUDA(h, soap::gemm(false, true, m, nc, nc, 1.f, strided(x, nc, 0), strided(c.QR + (int64_t)slot * nc * nc, nc, 0),
                             0.f, strided_mut(dstm, nc, 0), 1, s));
+  } else if (c.tr) {
+    SOAP_CUDA(h, soap::transpose(x, dstm, m, nc, 1, s));
   } else if (!c.left) {
     SOAP_CUDA(h, cudaMemcpyAsync(dstm, x, bytes, cudaMemcpyDeviceToDevice, s));
   }
-  if (c.tc) SOAP_CUDA(h, soap::split_tf32(dstm, nullptr, c.GM_lo + c.count * mn + slot * mn, mn, s));
+  if (c.tc) SOAP_CUDA(h, soap::split_tf32(dstm, nullptr, c.Mhat_lo + slot * mn, mn, s));
   return SOAP_OK;
 }
 

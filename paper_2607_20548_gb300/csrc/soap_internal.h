@@ -5,6 +5,7 @@
 #include <stdint.h>
 
 #include "../../include/soap.h"
+#include "profile.h"
 
 namespace soap {
 
@@ -70,8 +71,9 @@ struct TcEpilogue {
   float alpha, beta;     // beta != 0 reads C
   int* status;           // device status word for a timed-out wait (may be nullptr)
 };
+// `family` tags the launch for the library's profiler.
 cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const TcOperand& B,
-                       const TcEpilogue& ep, cudaStream_t stream);
+                       const TcEpilogue& ep, cudaStream_t stream, int family = kFamGemmTc);
 // hi = trunc_tf32(x), lo = x - hi (exact), elementwise over n values.
 cudaError_t split_tf32(const float* x, float* hi, float* lo, int64_t n, cudaStream_t stream);
 
@@ -99,11 +101,14 @@ cudaError_t adam_in_basis(float* Gp, const float* Mp, float* V, int rows, int co
                           float beta1, float beta2, float eps, float bc1, float bc2,
                           const uint8_t* skipL, const uint8_t* skipR, float* N_lo, int* status,
                           cudaStream_t stream);
-// Tensor-core operand preparation for a two-sided class: G copy, G^T and their lo parts,
-// M_hat <- b1 M_hat + (1-b1) G and its lo part.
-cudaError_t momentum_split(const float* const* grads, float* Gc, float* Gc_lo, float* Gt, float* Gt_lo,
+// Tensor-core operand preparation: G and G^T with their lo parts, and the momentum EMA
+// M_hat <- b1 M_hat + (1-b1) G with its lo part, M_hat stored in G's orientation or (if
+// mhat_transposed) as M_hat^T.
+cudaError_t momentum_split(const float* const* grads, float* Gn, float* Gn_lo, float* Gt, float* Gt_lo,
                            float* Mhat, float* Mhat_lo, int rows, int cols, int batch, float beta1,
-                           int* status, cudaStream_t stream);
+                           bool mhat_transposed, int* status, cudaStream_t stream);
+// dst_b = src_b^T for `batch` contiguous rows x cols matrices.
+cudaError_t transpose(const float* src, float* dst, int rows, int cols, int batch, cudaStream_t stream);
 // From Q^T and its lo part: copies of both and Q with its lo part (any output may be null).
 cudaError_t basis_from_qt(const float* Qt, const float* Qt_lo, float* Qt_out, float* Qt_lo_out, float* Q,
                           float* Q_lo, int n, int batch, cudaStream_t stream);

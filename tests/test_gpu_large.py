@@ -1,0 +1,202 @@
+"""Full-size parity of the 8192-wide dense layer: 2 x 8192x8192 preconditioned on both sides,
+2 x 8192x28672 on the left only and 1 x 28672x8192 on the right only, stepped as one batch
+through the C ABI.
+
+The oracle cannot run these sizes whole, so each checked step is verified on outputs that it
+computes one at a time, teacher-forced from the GPU's state before the step:
+  * S1 on sampled rows: F[I, :] = b F_old[I, :] + (1 - b) X[I, :] X^T (X = G or G^T);
+  * the refresh (S2, S3) on sampled columns j: Q_new^T (F Q_old[:, j]) vanishes below row j and
+    is non-negative on it (a column under the zero-column rule keeps a sub-column of norm at
+    most qr_tol ||P||_F), and Q_new is orthogonal;
+  * one-sided matrices: once Q is fixed, the rest of the step (rotation, Adam, back-rotation,
+    update) maps each column (left side) or row (right side) of G on its own, so sampled
+    columns or rows of the update are compared with the oracle's in fp64 and with its fp32
+    twin, under the bound of the whole-step tests (rel. Frobenius <= max(1e-3, 4 x twin));
+  * two-sided matrices: sampled rows of G' = Q_L^T G Q_R and m against the oracle (through v),
+    and the update's rows against Q_L[I, :] N Q_R^T from the GPU's own m and v.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle.soap_ref import adam_in_basis, rotate_in, rotate_out, weight_update
+from paper_2607_20548_gb300 import soap as S
+from paper_2607_20548_gb300.workloads import make_stream
+
+from tests.parity_tools import N_CAP, TOL, TWIN_FACTOR, oracle_hparams, orth_err, rel
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+
+def _flat(stream, tensors):
+    out = [None] * sum(len(idx) for _, idx in stream.groups)
+    for (spec, idx), t in zip(stream.groups, tensors):
+        for b, j in enumerate(idx):
+            out[j] = t[b]
+    return out
+
+
+def _np(x, dtype=np.float64):
+    return x.detach().cpu().numpy().astype(dtype)
+
+
+def _pick(n, rng, k=12):
+    return np.unique(np.concatenate([[0, n - 1], rng.choice(n, k, replace=False)]))
+
+
+def _snapshot(opt, i, W, G):
+    sp = opt.shapes[i]
+    d = dict(W=W.clone(), G=G, Mh=opt.state_get(i, S.STATE_MHAT), V=opt.state_get(i, S.STATE_V))
+    if sp.left:
+        d["L"], d["QL"] = opt.state_get(i, S.STATE_L), opt.state_get(i, S.STATE_QL)
+    if sp.right:
+        d["R"], d["QR"] = opt.state_get(i, S.STATE_R), opt.state_get(i, S.STATE_QR)
+    return d
+
+
+def _check_factor_and_qr(opt, i, pre, rng, hp, report):
+    """S1 rows and the refresh's triangularity on sampled columns, for each side of matrix i."""
+    sp = opt.shapes[i]
+    G = _np(pre["G"])
+    for side, X in (("L", G), ("R", G.T)):
+        if not getattr(sp, "left" if side == "L" else "right"):
+            continue
+        n = X.shape[0]
+        F_old = _np(pre[side])
+        F = _np(opt.state_get(i, S.STATE_L if side == "L" else S.STATE_R))
+        I = _pick(n, rng)
+        expect = hp.factor_beta * F_old[I] + (1 - hp.factor_beta) * (X[I] @ X.T)
+        e_f = rel(F[I], expect)
+        assert e_f <= 1e-5, (i, side, e_f)
+        Q_old = _np(pre["Q" + side])
+        Q_new = opt.state_get(i, S.STATE_QL if side == "L" else S.STATE_QR)
+        e_o = orth_err(Q_new)
+        assert e_o <= 1e-5, (i, side, e_o)
+        Q_new = _np(Q_new)
+        skip = _np(opt.state_get(i, S.STATE_SKIP_L if side == "L" else S.STATE_SKIP_R), np.uint8).astype(bool)
+        fro = np.linalg.norm(F)  # ||P||_F = ||F Q_old||_F for an orthogonal Q_old
+        J = _pick(n, rng)
+        Rj = Q_new.T @ (F @ Q_old[:, J])
+        worst = 0.0
+        for jj, j in enumerate(J):
+            below = Rj[j + 1:, jj]
+            if skip[j]:
+                assert np.linalg.norm(below) <= (hp.qr_tol + 1e-5) * fro, (i, side, j)
+            else:
+                worst = max(worst, np.abs(below).max(initial=0.0) / fro)
+                assert Rj[j, jj] >= -1e-5 * fro, (i, side, j, Rj[j, jj])
+        assert worst <= 1e-5, (i, side, worst)
+        report.append(f"matrix {i} {side}: S1 rows {e_f:.1e}, orth {e_o:.1e}, "
+                      f"max |R below diag| / ||P||_F {worst:.1e}, {int(skip.sum())} zero columns")
+
+
+def _check_one_sided(opt, i, pre, W_new, rng, hp, t, report):
+    """Sampled columns (left side) or rows (right side) of the whole update, teacher-forced."""
+    sp = opt.shapes[i]
+    left = sp.left
+    n_samples = sp.cols if left else sp.rows
+    K = _pick(n_samples, rng)
+    take = (lambda A: A[:, K]) if left else (lambda A: A[K, :])
+    Q32 = _np(opt.state_get(i, S.STATE_QL if left else S.STATE_QR), np.float32)
+    skip = _np(opt.state_get(i, S.STATE_SKIP_L if left else S.STATE_SKIP_R), np.uint8).astype(bool)
+    W0 = _np(take(pre["W"]), np.float32)
+    W1 = _np(take(W_new))
+    ins = {k: _np(take(pre[k]), np.float32) for k in ("G", "Mh", "V")}
+    out = {}
+    for dt in (np.float64, np.float32):
+        Q = Q32.astype(dt)
+        QL, QR = (Q, None) if left else (None, Q)
+        m0 = rotate_in(QL, ins["Mh"].astype(dt), QR)  # Alg. 1: m re-projected into the new basis
+        Gp = rotate_in(QL, ins["G"].astype(dt), QR)
+        m, v, N = adam_in_basis(m0, ins["V"].astype(dt), Gp, hp, t, skip if left else None,
+                                None if left else skip)
+        Wn = weight_update(W0.astype(dt), rotate_out(QL, N, QR), hp.lr, hp.weight_decay)
+        out[dt] = (m, v, N, Wn.astype(np.float64))
+    m64, v64, N64, Wn64 = out[np.float64]
+    d_ref = Wn64 - W0
+    e_gpu = rel(W1 - W0, d_ref)
+    e_twin = rel(out[np.float32][3] - W0, d_ref)
+    ill = TWIN_FACTOR * e_twin > TOL or np.abs(N64).max() > N_CAP
+    m_gpu = _np(take(opt.state_get(i, S.STATE_M)))
+    v_gpu = _np(take(opt.state_get(i, S.STATE_V)))
+    e_m, e_v = rel(m_gpu, m64), rel(v_gpu, v64)
+    N_self = m_gpu / (np.sqrt(v_gpu) + hp.eps)
+    if hp.guard:
+        if left:
+            N_self[skip, :] = 0
+        else:
+            N_self[:, skip] = 0
+    Q64 = Q32.astype(np.float64)
+    dW_self = Q64 @ N_self if left else N_self @ Q64.T
+    keep = 1 - hp.lr * hp.weight_decay
+    e_self = rel((W1 - keep * W0) / -hp.lr, dW_self)
+    report.append(f"matrix {i} step {t} ({len(K)} {'columns' if left else 'rows'}): gpu {e_gpu:.2e} "
+                  f"twin {e_twin:.2e} m {e_m:.1e} v {e_v:.1e} self {e_self:.1e}"
+                  + ("  [beyond fp32 resolution]" if ill else ""))
+    bound = max(TOL, TWIN_FACTOR * e_twin)
+    if not ill:
+        assert e_gpu <= bound, report[-1]
+    assert e_self <= (2e-4 if ill else bound), report[-1]
+    assert e_m <= 1e-4 and e_v <= 1e-4, report[-1]
+
+
+def _check_two_sided(opt, i, pre, W_new, rng, hp, t, report):
+    """Sampled rows of m and v against the oracle; the update rows against Q_L N Q_R^T from the
+    GPU's own m and v (N needs all of G', which the oracle cannot form at this size)."""
+    I = _pick(opt.shapes[i].rows, rng)
+    QL = _np(opt.state_get(i, S.STATE_QL))
+    QR = _np(opt.state_get(i, S.STATE_QR))
+    skL = _np(opt.state_get(i, S.STATE_SKIP_L), np.uint8).astype(bool)
+    skR = _np(opt.state_get(i, S.STATE_SKIP_R), np.uint8).astype(bool)
+    m0 = rotate_in(QL[:, I], _np(pre["Mh"]), QR)
+    Gp = rotate_in(QL[:, I], _np(pre["G"]), QR)
+    m64, v64, N64 = adam_in_basis(m0, _np(pre["V"])[I], Gp, hp, t, skL[I], skR)
+    m_all = _np(opt.state_get(i, S.STATE_M))
+    v_all = _np(opt.state_get(i, S.STATE_V))
+    e_m, e_v = rel(m_all[I], m64), rel(v_all[I], v64)
+    N = m_all / (np.sqrt(v_all) + hp.eps)
+    if hp.guard:
+        N[skL, :] = 0
+        N[:, skR] = 0
+    dW_self = QL[I] @ N @ QR.T
+    W0, W1 = _np(pre["W"])[I], _np(W_new)[I]
+    keep = 1 - hp.lr * hp.weight_decay
+    e_self = rel((W1 - keep * W0) / -hp.lr, dW_self)
+    ill = np.abs(N64).max() > N_CAP
+    report.append(f"matrix {i} step {t} ({len(I)} rows): m {e_m:.1e} v {e_v:.1e} self {e_self:.1e}"
+                  + ("  [beyond fp32 resolution]" if ill else ""))
+    assert e_m <= 1e-4 and e_v <= 1e-4, report[-1]
+    assert e_self <= (2e-4 if ill else TOL), report[-1]
+
+
+def test_dense_8192_ffn28672_full_size(cuda):
+    hp = S.default_hparams()
+    ohp = oracle_hparams(hp)
+    stream = make_stream("dense_8192_ffn28672", seed=0, device=cuda)
+    shapes = [(s.rows, s.cols, s.left, s.right) for s in stream.specs]
+    opt = S.SoapOptimizer(shapes, hp)
+    W = _flat(stream, [w.contiguous() for w in stream.weights()])
+    rng = np.random.default_rng(8192)
+    report = []
+    for t in range(1, 4):
+        G = _flat(stream, stream.grads(t))
+        checked = t in (2, 3)
+        pre = {i: _snapshot(opt, i, W[i], G[i]) for i in (0, 2, 4)} if checked else {}
+        opt.step(W, G)
+        torch.cuda.synchronize()
+        assert opt.status() == 0, opt.last_error()
+        if not checked:
+            continue
+        for i in (1, 3):
+            for w in (S.STATE_QL, S.STATE_QR):
+                if opt.state_bytes(i, w):
+                    assert orth_err(opt.state_get(i, w)) <= 1e-5
+        for i, d in pre.items():
+            _check_factor_and_qr(opt, i, d, rng, ohp, report)
+        _check_two_sided(opt, 0, pre[0], W[0], rng, ohp, t, report)
+        _check_one_sided(opt, 2, pre[2], W[2], rng, ohp, t, report)
+        _check_one_sided(opt, 4, pre[4], W[4], rng, ohp, t, report)
+        del pre
+        torch.cuda.empty_cache()
+    print("\n" + "\n".join(report))
+    opt.destroy()

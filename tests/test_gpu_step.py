@@ -85,9 +85,13 @@ def test_single_256x512_free_running_against_fp64(cuda):
 
 
 @pytest.mark.parametrize("shape", [(64, 300, True, False), (300, 64, False, True), (16, 24, False, False),
-                                   (48, 40, True, True)])
+                                   (48, 40, True, True), (64, 304, True, False), (304, 64, False, True),
+                                   (1028, 96, True, False), (96, 1028, False, True), (260, 1028, True, False)])
 def test_one_sided_and_identity_matrices(cuda, shape):
-    """Identity sides (Q fixed at I, no factor stored) in one batched step, 8 steps."""
+    """Identity sides (Q fixed at I, no factor stored), 8 steps against the oracle. Sides
+    that are multiples of 4 run on the tensor-core path (a left-only matrix as the
+    right-only problem of G^T), the others on CUDA cores; 1028 spans several 128-row
+    tiles with a ragged tail."""
     rows, cols, left, right = shape
     hp = S.default_hparams()
     opt = S.SoapOptimizer([shape], hp)
@@ -169,7 +173,9 @@ def test_dense_block_full_size(cuda):
 def test_checkpoint_resume_is_bit_exact(cuda):
     """state_get/state_set of every piece (M_hat, v, L, Q_L, R, Q_R, skip flags, t) round-trips:
     3 steps, save, 3 more steps == restore into a new handle and run the same 3 steps."""
-    shapes = [(40, 72, True, True), (72, 40, True, False)]
+    # two-sided, left-only and right-only tensor-core classes (the left-only one stores M_hat
+    # and v transposed) and a CUDA-core class (30 columns: not a multiple of 4)
+    shapes = [(40, 72, True, True), (72, 40, True, False), (44, 36, False, True), (32, 30, True, False)]
     hp = S.default_hparams()
     g = torch.Generator(device=cuda).manual_seed(7)
     Ws = [(0.02 * torch.randn(r, c, device=cuda, generator=g)).contiguous() for r, c, _, _ in shapes]
@@ -178,7 +184,8 @@ def test_checkpoint_resume_is_bit_exact(cuda):
     for t in range(3):
         a.step(Ws, Gs[t])
     pieces = (S.STATE_MHAT, S.STATE_V, S.STATE_L, S.STATE_QL, S.STATE_R, S.STATE_QR, S.STATE_SKIP_L, S.STATE_SKIP_R)
-    saved = {(i, w): a.state_get(i, w).clone() for i in range(2) for w in pieces if a.state_bytes(i, w) > 0}
+    saved = {(i, w): a.state_get(i, w).clone() for i in range(len(shapes)) for w in pieces
+             if a.state_bytes(i, w) > 0}
     W_saved = [w.clone() for w in Ws]
     t_saved = a.t
     for t in range(3, 6):
@@ -194,9 +201,10 @@ def test_checkpoint_resume_is_bit_exact(cuda):
     for x, y in zip(Ws, Wb):
         assert torch.equal(x, y)
     # the rotated-basis first moment round-trips to fp32 rounding
-    m = a.state_get(0, S.STATE_M)
-    b.state_set(0, S.STATE_M, m)
-    assert (b.state_get(0, S.STATE_MHAT) - a.state_get(0, S.STATE_MHAT)).abs().max().item() < 1e-6
+    for i in range(len(shapes)):
+        m = a.state_get(i, S.STATE_M)
+        b.state_set(i, S.STATE_M, m)
+        assert (b.state_get(i, S.STATE_MHAT) - a.state_get(i, S.STATE_MHAT)).abs().max().item() < 1e-6
     a.destroy()
     b.destroy()
 
