@@ -150,7 +150,7 @@ void soap_destroy(soap_handle h);
 /* Kernel families the library launches. */
 typedef enum {
   SOAP_KERNEL_GEMM_SIMT = 0,   /* CUDA-core fp32 batched GEMM */
-  SOAP_KERNEL_GEMM_TC = 1,     /* tcgen05 3xTF32 batched GEMM */
+  SOAP_KERNEL_GEMM_TC = 1,     /* tcgen05 fp32-accurate batched GEMM (four TF32 products) */
   SOAP_KERNEL_QR_PANEL = 2,    /* cluster panel factorisation of the QR */
   SOAP_KERNEL_ELEMENTWISE = 3, /* momentum, Adam, weight update */
   SOAP_KERNEL_OTHER = 4,       /* norms, identity fills */
@@ -216,25 +216,26 @@ soap_status_t soap_gemm(int32_t trans_a, int32_t trans_b, int32_t M, int32_t N, 
                         const float* B, int64_t ldb, int64_t stride_b, float beta, float* C,
                         int64_t ldc, int64_t stride_c, int32_t batch, soap_stream_t stream);
 
-/* The tensor-core form of that product (tcgen05, 3xTF32): for b < batch,
+/* The tensor-core form of that product (tcgen05, four TF32 products): for b < batch,
  *   C_b = alpha * A_b * B_(b mod b_batch)^T + beta * C_b        (or C_b^T if transpose_c)
- * with A_b (M x K) and B (N x K) row-major, each given as hi and lo = x - hi where hi is x
- * with its 13 low mantissa bits cleared (the tf32 value the tensor core reads from an fp32
- * word, so hi may be x itself; see soap_split_tf32); the accumulator adds
- * a_lo b_hi + a_hi b_lo + a_hi b_hi in fp32.
+ * with A_b (M x K) and B (N x K) row-major, each given as hi and lo, where hi is x with its
+ * 13 low mantissa bits cleared (the tf32 value the tensor core reads from an fp32 word, so
+ * hi may be x itself) and lo is x - hi rounded to the nearest tf32 (see soap_split_tf32);
+ * the accumulator adds a_lo b_lo + a_lo b_hi + a_hi b_lo + a_hi b_hi in fp32, each 32-wide
+ * K block summed afresh and added in fp32 registers (fp32-level accuracy at any K).
  * lda, ldb, ldc and every batch stride must be multiples of 4 elements and every
  * pointer 16-byte aligned. C_lo, if non-NULL, receives out - tf32(out) in C's layout
  * (leading dimension ldc). status, if non-NULL, is a device int that gets bit 4 set if
  * a bounded internal wait gave up. */
-soap_status_t soap_gemm_tf32x3(int32_t M, int32_t N, int32_t K, int32_t batch, const float* A_hi,
+soap_status_t soap_gemm_tf32x4(int32_t M, int32_t N, int32_t K, int32_t batch, const float* A_hi,
                                const float* A_lo, int64_t lda, int64_t stride_a, const float* B_hi,
                                const float* B_lo, int64_t ldb, int64_t stride_b, int32_t b_batch,
                                float alpha, float beta, float* C, int64_t ldc, int64_t stride_c,
                                int32_t transpose_c, float* C_lo, int32_t* status,
                                soap_stream_t stream);
 
-/* hi = x with its 13 low mantissa bits cleared (tf32 by truncation), lo = x - hi (exact),
- * for n values on the device; hi may be NULL. */
+/* hi = x with its 13 low mantissa bits cleared (tf32 by truncation), lo = x - hi (exact in
+ * fp32) rounded to the nearest tf32, for n values on the device; hi may be NULL. */
 soap_status_t soap_split_tf32(const float* x, float* hi, float* lo, int64_t n, soap_stream_t stream);
 
 #ifdef __cplusplus

@@ -20,19 +20,22 @@
 // round-to-nearest adds; the drain of block k overlaps the MMAs of block k+1, and the
 // error stays at the level of an fp32 dot product.
 //
-// CTA: 192 threads. Warp 0 issues the TMA loads (one elected lane), warp 1 allocates
-// tensor memory and issues the MMAs (one elected lane), warps 2-5 drain the
-// accumulators and run the epilogue: tensor memory -> registers (each warp owns 32 of
-// the 128 accumulator lanes) -> alpha/beta -> global, optionally transposed and optionally also writing the lo part
-// of the result for a later product. When the epilogue reads C (beta != 0), the
-// epilogue warps copy their part of the C tile into shared memory with cp.async while
-// the MMAs run, so the epilogue does not wait on one global load per output row.
-// Stages are handed over with mbarriers; every
-// wait gives up after ~2 s of %globaltimer time, records kStatusTimeout and lets the
-// CTA drain and free its tensor memory instead of hanging.
+// CTA: warp 0 issues the TMA loads (one elected lane), warp 1 allocates tensor memory and
+// issues the MMAs (one elected lane), and 8 epilogue warps (4 for BN = 32) drain the
+// accumulators: tensor memory -> registers (a warp reads the 32 accumulator lanes of its
+// quadrant, two warps split a quadrant's columns) -> alpha/beta -> a swizzled 32 x 32
+// block in shared memory -> 16-byte global stores, optionally transposed and optionally
+// also writing the lo part of the result for a later product. When the epilogue reads C
+// (beta != 0), the epilogue warps copy their part of the C tile into shared memory with
+// cp.async while the MMAs run. For short K a CTA runs several consecutive tiles, so that
+// the next tile's loads and MMAs proceed while the epilogue stores the current one.
+// Stages are handed over with mbarriers; every wait gives up after ~2 s of %globaltimer
+// time, records kStatusTimeout and lets the CTA drain and free its tensor memory instead
+// of hanging.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "profile.h"
@@ -43,18 +46,23 @@ namespace tc {
 
 constexpr int BM = 128;
 constexpr int BK = 32;  // fp32 elements per K block = one 128-byte swizzle row
-constexpr int THREADS = 192;
 constexpr uint64_t kWaitNs = 2000000000ull;
 
 template <int BN, int STAGES, bool PRE>
 struct Cfg {
+  static constexpr int EPI = BN >= 64 ? 8 : 4;      // epilogue warps (two per TMEM lane quadrant if 8)
+  static constexpr int THREADS = 64 + 32 * EPI;
+  static constexpr int CPW = BN * 4 / EPI;          // accumulator columns drained by one epilogue warp
+  static constexpr int NCH = CPW / 32;              // 32-column chunks per epilogue warp
   static constexpr int TILE_A = BM * BK * 4;
   static constexpr int TILE_B = BN * BK * 4;
   static constexpr int STAGE = 2 * TILE_A + 2 * TILE_B;
-  static constexpr int STAGING = 4 * 32 * 33 * 4;  // per epilogue warp: one 32 x 32 block (+pad)
-  static constexpr int CPRE = PRE ? 4 * 32 * BN * 4 : 0;  // prefetched C tile (32 rows per warp)
-  static constexpr int SMEM = STAGES * STAGE + STAGING + CPRE + 1024 + 256;
+  // per epilogue warp: its whole 32 x CPW block of C when C is prefetched, else one 32 x 32
+  // staging block (both swizzled in 16-byte units)
+  static constexpr int OBUF = PRE ? 32 * CPW : 32 * 32;
+  static constexpr int SMEM = STAGES * STAGE + EPI * OBUF * 4 + 1024 + 256;
   static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators, used alternately
+  static_assert(CPW % 32 == 0, "epilogue chunking");
   static_assert(SMEM <= 232448, "shared memory budget");
 };
 
@@ -174,17 +182,23 @@ __device__ __forceinline__ void cp_async16(float* smem_dst, const float* gmem_sr
                : "memory");
 }
 
+// Word offset of element (r, j) of a 32 x 32 block stored row-major with its 16-byte units
+// XOR-swizzled by r mod 8: a warp touching one 16-byte unit per row, or one row, is
+// conflict-free.
+__device__ __forceinline__ int swz(int r, int j) { return r * 32 + ((((j >> 2) ^ (r & 7))) << 2) + (j & 3); }
+
+// Tiles are numbered n-fastest, then m, then batch; a CTA takes `tpc` consecutive tiles, so
+// that the loads and MMAs of its next tile overlap the epilogue of the current one.
 template <int BN, int STAGES, bool PRE>
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap ta_hi, const __grid_constant__ CUtensorMap ta_lo,
                    const __grid_constant__ CUtensorMap tb_hi, const __grid_constant__ CUtensorMap tb_lo, int M,
-                   int N, int K, int a_mod, int b_mod, TcEpilogue ep) {
+                   int N, int K, int batch, int a_mod, int b_mod, int tpc, TcEpilogue ep) {
   using C = Cfg<BN, STAGES, PRE>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  float* staging = reinterpret_cast<float*>(smem + STAGES * C::STAGE);
-  float* cpre_all = reinterpret_cast<float*>(smem + STAGES * C::STAGE + C::STAGING);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE + C::STAGING + C::CPRE);
+  float* obuf_all = reinterpret_cast<float*>(smem + STAGES * C::STAGE);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE + C::EPI * C::OBUF * 4);
   uint64_t* empty = full + STAGES;
   uint64_t* acc_full = empty + STAGES;  // [2] accumulator a holds a finished K block
   uint64_t* acc_empty = acc_full + 2;   // [2] accumulator a has been drained
@@ -193,8 +207,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   volatile int* consumed = abort_flag + 1;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM, b = blockIdx.z;
   const int kblocks = (K + BK - 1) / BK;
+  const int ntn = (N + BN - 1) / BN, ntm = (M + BM - 1) / BM;
+  const int ntiles = ntn * ntm * batch;
+  const int t_begin = blockIdx.x * tpc;
+  const int t_end = min(ntiles, t_begin + tpc);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -203,7 +220,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&acc_full[a], 1);
-      mbar_init(&acc_empty[a], 4);  // one arrival per epilogue warp
+      mbar_init(&acc_empty[a], C::EPI);  // one arrival per epilogue warp
     }
     *abort_flag = 0;
     *consumed = 0;
@@ -227,167 +244,232 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      int issued = 0;
-      for (int kb = 0; kb < kblocks; ++kb) {
-        const int s = kb % STAGES;
-        const uint32_t ph = (kb / STAGES) & 1;
-        if (!mbar_wait(&empty[s], ph ^ 1) || *abort_flag) {
-          *abort_flag = 1;
-          break;
+      int g = 0, issued = 0;  // k blocks over all of this CTA's tiles
+      for (int t = t_begin; t < t_end && !*abort_flag; ++t) {
+        const int n0 = (t % ntn) * BN, m0 = ((t / ntn) % ntm) * BM, b = t / (ntn * ntm);
+        for (int kb = 0; kb < kblocks; ++kb, ++g) {
+          const int s = g % STAGES;
+          const uint32_t ph = (g / STAGES) & 1;
+          if (!mbar_wait(&empty[s], ph ^ 1) || *abort_flag) {
+            *abort_flag = 1;
+            break;
+          }
+          mbar_expect_tx(&full[s], C::STAGE);
+          const uint32_t st = smem_u32(smem + s * C::STAGE);
+          const int kc = kb * BK;
+          tma_load_3d(st, &ta_hi, &full[s], kc, m0, b % a_mod);
+          tma_load_3d(st + C::TILE_A, &ta_lo, &full[s], kc, m0, b % a_mod);
+          tma_load_3d(st + 2 * C::TILE_A, &tb_hi, &full[s], kc, n0, b % b_mod);
+          tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &tb_lo, &full[s], kc, n0, b % b_mod);
+          issued = g + 1;
         }
-        mbar_expect_tx(&full[s], C::STAGE);
-        const uint32_t st = smem_u32(smem + s * C::STAGE);
-        const int kc = kb * BK;
-        tma_load_3d(st, &ta_hi, &full[s], kc, m0, b % a_mod);
-        tma_load_3d(st + C::TILE_A, &ta_lo, &full[s], kc, m0, b % a_mod);
-        tma_load_3d(st + 2 * C::TILE_A, &tb_hi, &full[s], kc, n0, b % b_mod);
-        tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &tb_lo, &full[s], kc, n0, b % b_mod);
-        issued = kb + 1;
       }
       if (*abort_flag) {
         // let copies already in flight land before the CTA's shared memory goes away
-        for (int kb = *consumed; kb < issued; ++kb) mbar_wait(&full[kb % STAGES], (kb / STAGES) & 1);
+        for (int gg = *consumed; gg < issued; ++gg) mbar_wait(&full[gg % STAGES], (gg / STAGES) & 1);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_tf32(BM, BN);
-      for (int kb = 0; kb < kblocks; ++kb) {
-        const int s = kb % STAGES;
-        const uint32_t ph = (kb / STAGES) & 1;
-        const int a = kb & 1;
-        if (!mbar_wait(&full[s], ph) || (kb >= 2 && !mbar_wait(&acc_empty[a], ((kb >> 1) & 1) ^ 1)) ||
-            *abort_flag) {
-          *abort_flag = 1;
-          break;
-        }
-        *consumed = kb + 1;
-        tc_fence_after();
-        const uint32_t d = tmem + static_cast<uint32_t>(a * BN);
-        const uint32_t a_hi = smem_u32(smem + s * C::STAGE);
-        const uint32_t a_lo = a_hi + C::TILE_A;
-        const uint32_t b_hi = a_hi + 2 * C::TILE_A;
-        const uint32_t b_lo = b_hi + C::TILE_B;
+      int g = 0;
+      for (int t = t_begin; t < t_end && !*abort_flag; ++t) {
+        for (int kb = 0; kb < kblocks; ++kb, ++g) {
+          const int s = g % STAGES;
+          const uint32_t ph = (g / STAGES) & 1;
+          const int a = g & 1;
+          if (!mbar_wait(&full[s], ph) || (g >= 2 && !mbar_wait(&acc_empty[a], ((g >> 1) & 1) ^ 1)) ||
+              *abort_flag) {
+            *abort_flag = 1;
+            break;
+          }
+          *consumed = g + 1;
+          tc_fence_after();
+          const uint32_t d = tmem + static_cast<uint32_t>(a * BN);
+          const uint32_t a_hi = smem_u32(smem + s * C::STAGE);
+          const uint32_t a_lo = a_hi + C::TILE_A;
+          const uint32_t b_hi = a_hi + 2 * C::TILE_A;
+          const uint32_t b_lo = b_hi + C::TILE_B;
 #pragma unroll
-        for (int kk = 0; kk < BK / 8; ++kk) {
-          const uint32_t off = kk * 32;  // 8 tf32 = 32 bytes along K inside the swizzle row
-          umma_tf32(d, desc_sw128(a_lo + off), desc_sw128(b_lo + off), idesc, kk != 0);
-          umma_tf32(d, desc_sw128(a_lo + off), desc_sw128(b_hi + off), idesc, 1u);
-          umma_tf32(d, desc_sw128(a_hi + off), desc_sw128(b_lo + off), idesc, 1u);
-          umma_tf32(d, desc_sw128(a_hi + off), desc_sw128(b_hi + off), idesc, 1u);
+          for (int kk = 0; kk < BK / 8; ++kk) {
+            const uint32_t off = kk * 32;  // 8 tf32 = 32 bytes along K inside the swizzle row
+            umma_tf32(d, desc_sw128(a_lo + off), desc_sw128(b_lo + off), idesc, kk != 0);
+            umma_tf32(d, desc_sw128(a_lo + off), desc_sw128(b_hi + off), idesc, 1u);
+            umma_tf32(d, desc_sw128(a_hi + off), desc_sw128(b_lo + off), idesc, 1u);
+            umma_tf32(d, desc_sw128(a_hi + off), desc_sw128(b_hi + off), idesc, 1u);
+          }
+          umma_commit(&empty[s]);     // frees the stage once these MMAs have read it
+          umma_commit(&acc_full[a]);  // hands the K block's sum to the epilogue warps
         }
-        umma_commit(&empty[s]);     // frees the stage once these MMAs have read it
-        umma_commit(&acc_full[a]);  // hands the K block's sum to the epilogue warps
       }
     }
   } else {
     const int q = warp & 3;  // this warp may read accumulator lanes 32q .. 32q+31
+    const int colbase = ((warp - 2) / 4) * C::CPW;
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * q) << 16);
-    float* Cb = ep.C_ptrs ? ep.C_ptrs[b] : (ep.C ? ep.C + (int64_t)b * ep.c_stride : nullptr);
-    const int row0 = m0 + 32 * q;  // first of this warp's 32 rows
-    // this warp's part of the C tile, copied in while the MMAs run: rows row0.. x BN columns
-    // ([row][col]), or for a transposed C the BN columns' 32 entries each ([col][row]);
-    // only 16-byte chunks wholly inside C are copied, so partial chunks disable it
-    float* cpre = cpre_all + q * 32 * BN;
-    const bool pre = PRE && Cb && ep.beta != 0.f && (ep.ldc & 3) == 0 &&
-                     (reinterpret_cast<uintptr_t>(Cb) & 15) == 0 && ((ep.transpose ? M : N) & 3) == 0;
-    if (pre) {
-      if (!ep.transpose) {
-        for (int i = lane; i < 32 * (BN / 4); i += 32) {
-          const int rr = i / (BN / 4), ch = i % (BN / 4);
-          const int r = row0 + rr, col = n0 + 4 * ch;
-          const bool ok = r < M && col < N;
-          cp_async16(cpre + rr * BN + 4 * ch, ok ? Cb + (int64_t)r * ep.ldc + col : Cb, ok);
-        }
-      } else {
-        for (int i = lane; i < BN * 8; i += 32) {
-          const int cc = i / 8, ch = i % 8;
-          const int col = n0 + cc, r = row0 + 4 * ch;
-          const bool ok = r < M && col < N;
-          cp_async16(cpre + cc * 32 + 4 * ch, ok ? Cb + (int64_t)col * ep.ldc + r : Cb, ok);
-        }
-      }
-      asm volatile("cp.async.commit_group;" ::: "memory");
-    }
-    float acc[BN / 32][32];
-#pragma unroll
-    for (int c = 0; c < BN / 32; ++c)
-#pragma unroll
-      for (int j = 0; j < 32; ++j) acc[c][j] = 0.f;
+    float* obuf = obuf_all + (warp - 2) * C::OBUF;
+    int g = 0;
     bool valid = true;
-    for (int kb = 0; kb < kblocks; ++kb) {
-      const int a = kb & 1;
-      if (!mbar_wait(&acc_full[a], (kb >> 1) & 1) || *abort_flag) {
-        valid = false;
+    for (int t = t_begin; t < t_end && valid; ++t) {
+      const int n0 = (t % ntn) * BN, m0 = ((t / ntn) % ntm) * BM, b = t / (ntn * ntm);
+      float* Cb = ep.C_ptrs ? ep.C_ptrs[b] : (ep.C ? ep.C + (int64_t)b * ep.c_stride : nullptr);
+      float* Lb = ep.C_lo ? ep.C_lo + (int64_t)b * ep.lo_stride : nullptr;
+      const int row0 = m0 + 32 * q;   // first of this warp's 32 rows
+      const int col0 = n0 + colbase;  // first of its CPW columns
+      // 16-byte vector access to C (and C_lo) needs 16-byte aligned rows
+      const bool vec = Cb && (ep.ldc & 3) == 0 && (reinterpret_cast<uintptr_t>(Cb) & 15) == 0 &&
+                       (!Lb || ((ep.ld_lo & 3) == 0 && (reinterpret_cast<uintptr_t>(Lb) & 15) == 0));
+      // the prefetch copies whole 16-byte units: the dimension they run along must be a multiple of 4
+      const bool pre = PRE && vec && ep.beta != 0.f && ((ep.transpose ? M : N) & 3) == 0;
+      if (pre) {
+        // this warp's C block, copied in while the MMAs run; only 16-byte units wholly inside C
+        for (int c = 0; c < C::NCH; ++c) {
+          float* cb = obuf + 1024 * c;
+          for (int u = lane; u < 256; u += 32) {
+            const int x = u >> 3, y4 = u & 7;  // x: row (or column if transposed), y4: 16-byte unit
+            int r, col;
+            if (!ep.transpose) {
+              r = row0 + x;
+              col = col0 + 32 * c + 4 * y4;
+            } else {
+              col = col0 + 32 * c + x;
+              r = row0 + 4 * y4;
+            }
+            const bool ok = ep.transpose ? (col < N && r + 3 < M) : (r < M && col + 3 < N);
+            const float* src = !ok ? Cb : ep.transpose ? Cb + (int64_t)col * ep.ldc + r : Cb + (int64_t)r * ep.ldc + col;
+            cp_async16(cb + x * 32 + ((y4 ^ (x & 7)) << 2), src, ok);
+          }
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+      }
+      float acc[C::NCH][32];
+#pragma unroll
+      for (int c = 0; c < C::NCH; ++c)
+#pragma unroll
+        for (int j = 0; j < 32; ++j) acc[c][j] = 0.f;
+      for (int kb = 0; kb < kblocks; ++kb, ++g) {
+        const int a = g & 1;
+        if (!mbar_wait(&acc_full[a], (g >> 1) & 1) || *abort_flag) {
+          valid = false;
+          break;
+        }
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < C::NCH; ++c) {
+          float v[32];
+          tmem_ld32(lane_base + static_cast<uint32_t>(a * BN + colbase + 32 * c), v);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) acc[c][j] += v[j];
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0)
+          asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&acc_empty[a])) : "memory");
+      }
+      if (pre) {
+        asm volatile("cp.async.wait_all;" ::: "memory");
+        __syncwarp();
+      }
+      if (!valid) {
+        if (lane == 0 && ep.status) atomicOr(ep.status, kStatusTimeout);
         break;
       }
-      tc_fence_after();
+      // out = alpha acc + beta C through the warp's shared block, then 16-byte stores
 #pragma unroll
-      for (int c = 0; c < BN / 32; ++c) {
-        float v[32];
-        tmem_ld32(lane_base + static_cast<uint32_t>(a * BN + 32 * c), v);
+      for (int c = 0; c < C::NCH; ++c) {
+        float* cb = obuf + (PRE ? 1024 * c : 0);
+        const int cc0 = col0 + 32 * c;
+        if (!ep.transpose) {
+          const int r = row0 + lane;  // this lane's row
 #pragma unroll
-        for (int j = 0; j < 32; ++j) acc[c][j] += v[j];
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0)
-        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&acc_empty[a])) : "memory");
-    }
-    if (!valid && lane == 0 && ep.status) atomicOr(ep.status, kStatusTimeout);
-    if (pre) {
-      // the copies complete even when a wait gave up, before the CTA's shared memory goes away
-      asm volatile("cp.async.wait_all;" ::: "memory");
-      __syncwarp();
-    }
-    float* Lb = ep.C_lo ? ep.C_lo + (int64_t)b * ep.lo_stride : nullptr;
-    if (valid && ep.transpose) {
-      // C^T: for a fixed column the 32 lanes (32 consecutive rows) write 128 contiguous bytes
-      const int r = row0 + lane;
-#pragma unroll
-      for (int c = 0; c < BN / 32; ++c) {
-        const int col0 = n0 + 32 * c;
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const int col = col0 + j;
-          if (col >= N || r >= M) continue;
-          const int64_t off = (int64_t)col * ep.ldc + r;
-          float out = ep.alpha * acc[c][j];
-          if (Cb) {
-            if (ep.beta != 0.f) out = fmaf(ep.beta, pre ? cpre[(32 * c + j) * 32 + lane] : Cb[off], out);
-            Cb[off] = out;
-          }
-          if (Lb) Lb[(int64_t)col * ep.ld_lo + r] = tf32_lo(out);
-        }
-      }
-    } else if (valid) {
-      // C: each lane holds one row; stage the warp's 32 x 32 block in shared memory so that
-      // every global access instruction covers 32 consecutive columns of one row
-      float* st = staging + q * (32 * 33);
-#pragma unroll
-      for (int c = 0; c < BN / 32; ++c) {
-        const int col0 = n0 + 32 * c;
-        if (col0 >= N) break;  // warp-uniform
-#pragma unroll
-        for (int j = 0; j < 32; ++j) st[lane * 33 + j] = acc[c][j];
-        __syncwarp();
-        const int col = col0 + lane;
-        for (int rr = 0; rr < 32; ++rr) {
-          const int r = row0 + rr;
-          if (r >= M) break;  // warp-uniform
-          if (col < N) {
-            float out = ep.alpha * st[rr * 33 + lane];
-            if (Cb) {
-              const int64_t off = (int64_t)r * ep.ldc + col;
-              if (ep.beta != 0.f) out = fmaf(ep.beta, pre ? cpre[rr * BN + 32 * c + lane] : Cb[off], out);
-              Cb[off] = out;
+          for (int j4 = 0; j4 < 8; ++j4) {
+            float4 o;
+            o.x = ep.alpha * acc[c][4 * j4];
+            o.y = ep.alpha * acc[c][4 * j4 + 1];
+            o.z = ep.alpha * acc[c][4 * j4 + 2];
+            o.w = ep.alpha * acc[c][4 * j4 + 3];
+            float4* slot = reinterpret_cast<float4*>(cb + swz(lane, 4 * j4));
+            if (ep.beta != 0.f) {
+              float4 cv;
+              if (pre) {
+                cv = *slot;
+              } else {
+                const int col = cc0 + 4 * j4;
+                const float* src = Cb + (int64_t)r * ep.ldc + col;
+                const bool in = Cb && r < M;
+                cv.x = (in && col < N) ? src[0] : 0.f;
+                cv.y = (in && col + 1 < N) ? src[1] : 0.f;
+                cv.z = (in && col + 2 < N) ? src[2] : 0.f;
+                cv.w = (in && col + 3 < N) ? src[3] : 0.f;
+              }
+              o.x = fmaf(ep.beta, cv.x, o.x);
+              o.y = fmaf(ep.beta, cv.y, o.y);
+              o.z = fmaf(ep.beta, cv.z, o.z);
+              o.w = fmaf(ep.beta, cv.w, o.w);
             }
-            if (Lb) Lb[(int64_t)r * ep.ld_lo + col] = tf32_lo(out);
+            *slot = o;
           }
+          __syncwarp();
+#pragma unroll
+          for (int it = 0; it < 8; ++it) {
+            const int rr = 4 * it + (lane >> 3), j4 = lane & 7;
+            const int r2 = row0 + rr, col = cc0 + 4 * j4;
+            if (r2 >= M || col >= N) continue;
+            const float4 o = *reinterpret_cast<const float4*>(cb + swz(rr, 4 * j4));
+            const float ov[4] = {o.x, o.y, o.z, o.w};
+            if (vec && col + 3 < N) {
+              if (Cb) *reinterpret_cast<float4*>(Cb + (int64_t)r2 * ep.ldc + col) = o;
+              if (Lb)
+                *reinterpret_cast<float4*>(Lb + (int64_t)r2 * ep.ld_lo + col) =
+                    make_float4(tf32_lo(o.x), tf32_lo(o.y), tf32_lo(o.z), tf32_lo(o.w));
+            } else {
+              for (int e = 0; e < 4 && col + e < N; ++e) {
+                if (Cb) Cb[(int64_t)r2 * ep.ldc + col + e] = ov[e];
+                if (Lb) Lb[(int64_t)r2 * ep.ld_lo + col + e] = tf32_lo(ov[e]);
+              }
+            }
+          }
+          __syncwarp();
+        } else {
+          // C^T: element (row r = this lane, column j) is stored at column-major block position (j, r)
+          const int r = row0 + lane;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            float o = ep.alpha * acc[c][j];
+            float* slot = cb + swz(j, lane);
+            if (ep.beta != 0.f) {
+              const int col = cc0 + j;
+              const float cv = pre ? *slot : ((Cb && r < M && col < N) ? Cb[(int64_t)col * ep.ldc + r] : 0.f);
+              o = fmaf(ep.beta, cv, o);
+            }
+            *slot = o;
+          }
+          __syncwarp();
+#pragma unroll
+          for (int it = 0; it < 8; ++it) {
+            const int jj = 4 * it + (lane >> 3), r4 = lane & 7;
+            const int col = cc0 + jj, r2 = row0 + 4 * r4;
+            if (col >= N || r2 >= M) continue;
+            const float4 o = *reinterpret_cast<const float4*>(cb + swz(jj, 4 * r4));
+            const float ov[4] = {o.x, o.y, o.z, o.w};
+            if (vec && r2 + 3 < M) {
+              if (Cb) *reinterpret_cast<float4*>(Cb + (int64_t)col * ep.ldc + r2) = o;
+              if (Lb)
+                *reinterpret_cast<float4*>(Lb + (int64_t)col * ep.ld_lo + r2) =
+                    make_float4(tf32_lo(o.x), tf32_lo(o.y), tf32_lo(o.z), tf32_lo(o.w));
+            } else {
+              for (int e = 0; e < 4 && r2 + e < M; ++e) {
+                if (Cb) Cb[(int64_t)col * ep.ldc + r2 + e] = ov[e];
+                if (Lb) Lb[(int64_t)col * ep.ld_lo + r2 + e] = tf32_lo(ov[e]);
+              }
+            }
+          }
+          __syncwarp();
         }
-        __syncwarp();
       }
     }
+    // copies of a tile abandoned after a timeout still land before shared memory goes away
+    if (PRE) asm volatile("cp.async.wait_all;" ::: "memory");
   }
 
   tc_fence_before();
@@ -448,8 +530,15 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM, batch);
-  gemm_tc_kernel<BN, STAGES, PRE><<<grid, THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, amod, bmod, ep);
+  const int64_t ntiles = (int64_t)((N + BN - 1) / BN) * ((M + BM - 1) / BM) * batch;
+  if (ntiles > (int64_t)1 << 30) return cudaErrorInvalidValue;
+  // short K: a CTA runs several tiles so that the next tile's loads and MMAs overlap the
+  // current epilogue, keeping about four waves of CTAs over the 152 SMs
+  const int kblocks = (K + BK - 1) / BK;
+  const int tpc = kblocks > 16 ? 1 : (int)std::max<int64_t>(1, std::min<int64_t>(8, ntiles / (4 * 152)));
+  const int grid = (int)((ntiles + tpc - 1) / tpc);
+  gemm_tc_kernel<BN, STAGES, PRE><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
+                                                                     bmod, tpc, ep);
   return cudaGetLastError();
 }
 
@@ -458,7 +547,7 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
 cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const TcOperand& B, const TcEpilogue& ep,
                        cudaStream_t s, int family) {
   if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
-  if (batch > 65535 || (M + tc::BM - 1) / tc::BM > 65535) return cudaErrorInvalidValue;
+  if (batch > 65535) return cudaErrorInvalidValue;
   const double flops = 2.0 * M * N * (double)K * batch;  // algorithmic (4 tf32 products each on the pipe)
   const double bytes = 4.0 * (2.0 * (double)M * K * (A.batch > 0 ? A.batch : batch) +
                               2.0 * (double)N * K * (B.batch > 0 ? B.batch : batch) +

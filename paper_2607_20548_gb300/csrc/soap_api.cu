@@ -957,7 +957,7 @@ soap_status_t soap_gemm(int32_t trans_a, int32_t trans_b, int32_t M, int32_t N, 
   return e == cudaSuccess ? SOAP_OK : SOAP_ERR_CUDA;
 }
 
-soap_status_t soap_gemm_tf32x3(int32_t M, int32_t N, int32_t K, int32_t batch, const float* A_hi, const float* A_lo,
+soap_status_t soap_gemm_tf32x4(int32_t M, int32_t N, int32_t K, int32_t batch, const float* A_hi, const float* A_lo,
                                int64_t lda, int64_t stride_a, const float* B_hi, const float* B_lo, int64_t ldb,
                                int64_t stride_b, int32_t b_batch, float alpha, float beta, float* C, int64_t ldc,
                                int64_t stride_c, int32_t transpose_c, float* C_lo, int32_t* status,

@@ -25,7 +25,7 @@ STATE_M, STATE_V, STATE_L, STATE_QL, STATE_R, STATE_QR, STATE_MHAT, STATE_SKIP_L
 EXPORTS = ("soap_default_hparams", "soap_create", "soap_step", "soap_set_lr", "soap_state_bytes",
            "soap_state_get", "soap_state_set", "soap_get_step", "soap_set_step", "soap_status",
            "soap_clear_status", "soap_last_error", "soap_destroy", "soap_qr_workspace_bytes",
-           "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_gemm_tf32x3",
+           "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_gemm_tf32x4",
            "soap_split_tf32", "soap_qr_static")
 KERNEL_FAMILIES = ("gemm_simt", "gemm_tc", "qr_panel", "elementwise", "other", "qr_update")
 
@@ -85,7 +85,7 @@ def load_library(path: str = LIB_PATH):
         "soap_profile_begin": (I32, [P, I64]),
         "soap_profile_end": (I32, [P, P, ctypes.POINTER(soap_kernel_stats), ctypes.POINTER(I32)]),
         "soap_gemm": (I32, [I32, I32, I32, I32, I32, F, P, I64, I64, P, I64, I64, F, P, I64, I64, I32, P]),
-        "soap_gemm_tf32x3": (I32, [I32, I32, I32, I32, P, P, I64, I64, P, P, I64, I64, I32, F, F, P, I64, I64,
+        "soap_gemm_tf32x4": (I32, [I32, I32, I32, I32, P, P, I64, I64, P, P, I64, I64, I32, F, F, P, I64, I64,
                                    I32, P, P, P]),
         "soap_split_tf32": (I32, [P, P, P, I64, P]),
         "soap_qr_static": (I32, [I32, I32, P, P, P, F, P]),
@@ -328,7 +328,7 @@ def soap_split_tf32(x: torch.Tensor, stream=None):
     return hi, lo
 
 
-def soap_gemm_tf32x3(A, B, alpha=1.0, beta=0.0, C=None, transpose_c=False, A_split=None, B_split=None,
+def soap_gemm_tf32x4(A, B, alpha=1.0, beta=0.0, C=None, transpose_c=False, A_split=None, B_split=None,
                      with_lo=False, status=None, stream=None):
     """Tensor-core C = alpha A B^T + beta C for [batch, M, K] x [b_batch, N, K] fp32 CUDA tensors.
 
@@ -347,7 +347,7 @@ def soap_gemm_tf32x3(A, B, alpha=1.0, beta=0.0, C=None, transpose_c=False, A_spl
         (C.unsqueeze(0) if C.dim() == 2 else C)
     lo = torch.zeros_like(C3) if with_lo else None
     ldc = shape[2]
-    _check(lib.soap_gemm_tf32x3(M, N, K, batch, ctypes.c_void_p(ahi.data_ptr()), ctypes.c_void_p(alo.data_ptr()),
+    _check(lib.soap_gemm_tf32x4(M, N, K, batch, ctypes.c_void_p(ahi.data_ptr()), ctypes.c_void_p(alo.data_ptr()),
                                 K, M * K, ctypes.c_void_p(bhi.data_ptr()), ctypes.c_void_p(blo.data_ptr()), K,
                                 N * K, bb, float(alpha), float(beta), ctypes.c_void_p(C3.data_ptr()), ldc,
                                 shape[1] * shape[2], int(transpose_c),
