@@ -194,7 +194,7 @@ soap_status_t soap_qr(int32_t n, int32_t batch, const float* P, float* Q, uint8_
  * handed out at start-up, owns it). Same arguments and results as soap_qr, without the
  * workspace: it uses a 32 MiB array compiled into libsoap.so, which every GPU that
  * loads the library keeps until the process exits. That is room for one 1024 x 1024
- * matrix or, e.g., four of 512 x 512; a (n, batch) whose soap_qr_workspace_bytes()
+ * matrix or, e.g., three of 512 x 512; a (n, batch) whose soap_qr_workspace_bytes()
  * exceeds 32 MiB - 256 B is refused with SOAP_ERR_INVALID_ARG before anything is
  * enqueued. It never calls cudaMalloc, cudaFree or any allocating routine.
  * The first call on each device looks up the array's device address with that device

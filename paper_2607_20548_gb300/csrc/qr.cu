@@ -25,7 +25,8 @@
 //   and Q = (Q^T)^T is written with its lo part.
 //
 // The panel of an n x n matrix spans up to n positions; it is spread over a thread-block
-// cluster of ceil((n-k)/1024) CTAs (<= 8 for n <= 8192), 1024 positions each. Each
+// cluster of ceil((n-k)/512) CTAs (<= 16 for n <= 8192), 512 positions each, or, on a
+// device that cannot run 16-CTA clusters of it, 1024 positions in clusters of <= 8. Each
 // Householder step needs one cluster-wide reduction: the squared norm of the column
 // below the pivot and its dot products with the later panel columns are reduced
 // together (the dot products with v follow from them once the reflector is known), and
@@ -57,11 +58,10 @@ namespace {
 
 constexpr int NB = 32;            // panel width
 constexpr int NBO = 128;          // block width: the trailing matrix is updated once per block
-constexpr int COLS = 1024;        // panel positions held by one CTA
 constexpr int PT = 512;           // threads per panel CTA
-constexpr int LDS = COLS + 1;     // row stride of the shared panel (bank-conflict padding)
-constexpr int MAXC = 8;           // largest cluster (portable limit) -> n <= 8192
+constexpr int MAXC = 16;          // largest cluster (16 needs the non-portable cluster size)
 constexpr int NWARP = PT / 32;
+constexpr int NREST = NBO - NB;   // most block rows after a panel
 
 // lo part of x for the tensor-core products: x - trunc_tf32(x) rounded to the nearest tf32
 __device__ __forceinline__ float tf32_lo(float x) {
@@ -94,24 +94,31 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// One 32-column panel, spread over a cluster: CTA c holds positions k + c*COLS .. of the
+// panel rows in shared memory (row stride LDS, 16-byte aligned rows).
+template <int COLS>
 __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
+  constexpr int LDS = COLS + 4;
   cg::cluster_group cluster = cg::this_cluster();
   const int c = (int)cluster.block_rank();
   const int C = (int)cluster.num_blocks();
   const int b = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
-  extern __shared__ float sA[];  // [NB][LDS]: panel row jj (a column of P), position offset i
+  extern __shared__ float4 smem_dyn[];
+  float* sA = reinterpret_cast<float*>(smem_dyn);  // [NB][LDS]: panel row jj, position offset i
   __shared__ float s_part[2][MAXC][NB];  // per-CTA partial [sigma | x . a_c], by source CTA
-  __shared__ float s_piv[2][NB];         // pivot-row values held by rank 0: [alpha | a_c,pivot]
+  __shared__ float s_piv[2][NB];         // rank 0: pivot-row values [alpha | a_c,pivot]
   __shared__ float s_sum[NB];
+  __shared__ float s_pv[NB];             // every CTA's copy of the pivot-row values
   __shared__ float s_w[NB];              // v^T a_c
   __shared__ float s_tau[NB];
   __shared__ int s_skip[NB];
   __shared__ float s_dsign[NB];
   __shared__ float s_T[NB][NB + 1];
   __shared__ float s_Y[NBO][NB + 1];     // rank 0: S V_panel summed over the cluster
-  __shared__ float s_Z[NBO - NB][NB];    // (S_rest V_panel) T_panel for the in-block update
+  __shared__ __align__(16) float s_Z[NREST][NB];  // (S_rest V_panel) T_panel, the in-block update
+  __shared__ float s_Tb[NREST][NREST + 1];        // rank 0: the block's T so far
 
   const int n = p.n, k = p.k, kb = p.kb, k0 = p.k0, kbo = p.kbo;
   const int jb = k - k0;                // panel offset inside its block
@@ -119,11 +126,11 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   const int64_t nn = (int64_t)n * n;
   float* At = p.At + (int64_t)b * nn;
   const int pos0 = k + c * COLS;  // first position held by this CTA
-  const int npos = max(0, min(COLS, n - pos0));
+  const int npos = max(0, min(COLS, n - pos0));  // a multiple of 4
 
-  for (int e = tid; e < npos * NB; e += PT) {
-    const int jj = e / npos, i = e % npos;
-    sA[jj * LDS + i] = jj < kb ? At[(int64_t)(k + jj) * n + pos0 + i] : 0.f;
+  for (int jj = 0; jj < NB; ++jj) {
+    const float* src = At + (int64_t)(k + jj) * n + pos0;
+    for (int i = tid; i < npos; i += PT) sA[jj * LDS + i] = jj < kb ? src[i] : 0.f;
   }
   __syncthreads();
   const float thresh = p.thresh[b];
@@ -133,28 +140,26 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     const int par = j & 1;
     // positions strictly after the pivot (pivot = local position j of rank 0)
     const int ibeg = (c == 0) ? j + 1 : 0;
-    // partial sums over this CTA: sigma (cc = j) and x . a_cc (cc > j)
+    // partial sums over this CTA: sigma (cc = j) and x . a_cc (cc > j), sent to every CTA
     for (int cc = j + warp; cc < kb; cc += NWARP) {
       float d = 0.f;
       for (int i = ibeg + lane; i < npos; i += 32) d = fmaf(sA[j * LDS + i], sA[cc * LDS + i], d);
       d = warp_sum(d);
       if (lane < C) cluster.map_shared_rank(&s_part[par][0][0], lane)[c * NB + cc] = d;
     }
-    if (c == 0 && tid >= j && tid < kb) {
-      const float v = sA[tid * LDS + j];  // alpha (tid == j) or a_tid at the pivot
-      for (int q = 0; q < C; ++q) cluster.map_shared_rank(&s_piv[par][0], q)[tid] = v;
-    }
+    if (c == 0 && tid >= j && tid < kb) s_piv[par][tid] = sA[tid * LDS + j];  // alpha, a_tid at the pivot
     cluster.sync();
     if (tid >= j && tid < kb) {
       float d = 0.f;
       for (int q = 0; q < C; ++q) d += s_part[par][q][tid];
       s_sum[tid] = d;
+      s_pv[tid] = *cluster.map_shared_rank(&s_piv[par][tid], 0);
     }
     __syncthreads();
 
     // every thread derives the same reflector from the same reduced values
     const float sigma = s_sum[j];
-    const float alpha = s_piv[par][j];
+    const float alpha = s_pv[j];
     const float xnorm = sqrtf(fmaf(alpha, alpha, sigma));
     if (!isfinite(xnorm)) nonfinite = 1;
     const bool skip = !(xnorm > thresh);
@@ -170,7 +175,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       }
     }
     // v^T a_cc = a_cc,pivot + (x . a_cc) / v0, with v = x / v0 after the pivot
-    if (tau != 0.f && tid > j && tid < kb) s_w[tid] = s_piv[par][tid] + s_sum[tid] / v0;
+    if (tau != 0.f && tid > j && tid < kb) s_w[tid] = s_pv[tid] + s_sum[tid] / v0;
     if (tid == 0) {
       s_tau[j] = tau;
       s_skip[j] = skip ? 1 : 0;
@@ -181,9 +186,10 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     // v after the pivot (x / v0, or 0 where H = I), and H_j = I - tau v v^T on the later
     // panel rows; every thread owns its positions
     const int piv = (c == 0) ? j : 0;  // local positions >= this take part
+    const float rv0 = tau != 0.f ? 1.f / v0 : 0.f;
     for (int i = piv + tid; i < npos; i += PT) {
       const bool at_pivot = (c == 0 && i == j);
-      const float vi = at_pivot ? 1.f : (tau != 0.f ? sA[j * LDS + i] / v0 : 0.f);
+      const float vi = at_pivot ? 1.f : sA[j * LDS + i] * rv0;
       if (!at_pivot) sA[j * LDS + i] = vi;
       if (tau != 0.f) {
         const float tv = tau * vi;
@@ -210,12 +216,13 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   float* Vt_lo = p.Vt_lo + (int64_t)b * nn;
   float* Vpos = p.Vpos + (int64_t)b * n * NBO;
   float* Vpos_lo = p.Vpos_lo + (int64_t)b * n * NBO;
-  for (int e = tid; e < npos * kb; e += PT) {
-    const int jj = e / npos, i = e % npos;
-    const float v = sA[jj * LDS + i];
-    const int64_t o = (int64_t)(k + jj) * n + pos0 + i;
-    Vt[o] = v;
-    Vt_lo[o] = tf32_lo(v);
+  for (int jj = 0; jj < kb; ++jj) {
+    const int64_t o = (int64_t)(k + jj) * n + pos0;
+    for (int i = tid; i < npos; i += PT) {
+      const float v = sA[jj * LDS + i];
+      Vt[o + i] = v;
+      Vt_lo[o + i] = tf32_lo(v);
+    }
   }
   for (int i = warp; i < npos; i += NWARP) {
     const float v = sA[lane * LDS + i];  // rows kb.. of sA are zero
@@ -224,12 +231,12 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     Vpos_lo[o] = tf32_lo(v);
   }
   if (c == 0) {
-    for (int e = tid; e < kb * jb; e += PT) {
-      const int jj = e / jb, i = e % jb;
-      const int64_t o = (int64_t)(k + jj) * n + k0 + i;
-      Vt[o] = 0.f;
-      Vt_lo[o] = 0.f;
-    }
+    for (int jj = 0; jj < kb; ++jj)
+      for (int i = tid; i < jb; i += PT) {
+        const int64_t o = (int64_t)(k + jj) * n + k0 + i;
+        Vt[o] = 0.f;
+        Vt_lo[o] = 0.f;
+      }
     for (int e = tid; e < jb * NB; e += PT) {
       const int64_t o = (int64_t)(k0 + e / NB) * NBO + jb + e % NB;
       Vpos[o] = 0.f;
@@ -242,76 +249,80 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   // Householder vectors so far (rows before the panel's end, from Vt) and the block rows
   // still to be factored (from At). Warp w takes rows w, w+16, ...; lane jj column jj.
   {
-    float y[NBO / NWARP];
-    const float* srow[NBO / NWARP];
+    constexpr int RW = NBO / NWARP;
+    float y[RW];
+    const float* srow[RW];
+    const int nr = (kbo - warp + NWARP - 1) / NWARP;  // rows of this warp
 #pragma unroll
-    for (int u = 0; u < NBO / NWARP; ++u) {
-      const int r = warp + NWARP * u;
-      const int row = k0 + r;
+    for (int u = 0; u < RW; ++u) {
+      const int row = k0 + warp + NWARP * u;
       y[u] = 0.f;
-      srow[u] = r < kbo ? ((row < k + kb) ? Vt : At) + (int64_t)row * n + pos0 : nullptr;
+      srow[u] = ((row < k + kb) ? Vt : At) + (int64_t)min(row, n - 1) * n + pos0;
     }
-    for (int i = 0; i < npos; i += 4) {  // npos is a multiple of 4
-      const float v0 = sA[lane * LDS + i], v1 = sA[lane * LDS + i + 1];
-      const float v2 = sA[lane * LDS + i + 2], v3 = sA[lane * LDS + i + 3];
+    for (int i = 0; i < npos; i += 4) {
+      const float4 v = *reinterpret_cast<const float4*>(&sA[lane * LDS + i]);
 #pragma unroll
-      for (int u = 0; u < NBO / NWARP; ++u) {
-        if (!srow[u]) continue;
-        const float4 x = *reinterpret_cast<const float4*>(srow[u] + i);
-        y[u] = fmaf(x.w, v3, fmaf(x.z, v2, fmaf(x.y, v1, fmaf(x.x, v0, y[u]))));
+      for (int u = 0; u < RW; ++u) {
+        if (u < nr) {
+          const float4 x = *reinterpret_cast<const float4*>(srow[u] + i);
+          y[u] = fmaf(x.w, v.w, fmaf(x.z, v.z, fmaf(x.y, v.y, fmaf(x.x, v.x, y[u]))));
+        }
       }
     }
     float* yp = p.Ypart + ((int64_t)b * MAXC + c) * NBO * NB;
 #pragma unroll
-    for (int u = 0; u < NBO / NWARP; ++u) {
-      const int r = warp + NWARP * u;
-      if (r < kbo) yp[r * NB + lane] = y[u];
-    }
+    for (int u = 0; u < RW; ++u)
+      if (u < nr) yp[(warp + NWARP * u) * NB + lane] = y[u];
   }
   cluster.sync();  // orders the partials in global memory before rank 0 reads them
 
   if (c == 0) {
-    // sum the partials in a fixed order
+    // sum the partials in a fixed order; stage the block's T so far
     const float* yp = p.Ypart + (int64_t)b * MAXC * NBO * NB;
     for (int e = tid; e < kbo * NB; e += PT) {
+      float part[MAXC];
+#pragma unroll
+      for (int q = 0; q < MAXC; ++q) part[q] = q < C ? yp[(int64_t)q * NBO * NB + e] : 0.f;
       float sum = 0.f;
-      for (int q = 0; q < C; ++q) sum += yp[(int64_t)q * NBO * NB + e];
+#pragma unroll
+      for (int q = 0; q < MAXC; ++q) sum += part[q];
       s_Y[e / NB][e % NB] = sum;
     }
+    const float* Tg = p.T + (int64_t)b * NBO * NBO;
+    for (int e = tid; e < jb * jb; e += PT) s_Tb[e / jb][e % jb] = Tg[(e / jb) * NBO + e % jb];
     __syncthreads();
-    // T of the panel from its Gram matrix (rows jb.. of Y): T_jj = tau_j,
-    // T(0:j, j) = -tau_j T(0:j, 0:j) g(0:j, j)
-    for (int j = 0; j < kb; ++j) {
-      if (tid < kb) {
-        const int i = tid;
+    // T of the panel from its Gram matrix g (rows jb.. of Y): T^-1 = diag(1/tau) + striu(g)
+    // (H_1 ... H_kb = I - V T V^T); a reflector with tau = 0 (v = 0) gets a zero row and column
+    if (tid < kb) {
+      const int cc = tid;
+      float x[NB];
+      // back substitution for column cc of T: (diag(1/tau) + striu(g)) x = e_cc
+      for (int i = NB - 1; i >= 0; --i) {
         float t = 0.f;
-        if (i < j) {
-          float acc = 0.f;
-          for (int l = i; l < j; ++l) acc = fmaf(s_T[i][l], s_Y[jb + l][j], acc);
-          t = -s_tau[j] * acc;
-        } else if (i == j) {
-          t = s_tau[j];
+        if (i <= cc) {
+          float acc = (i == cc) ? 1.f : 0.f;
+          for (int l = i + 1; l <= cc; ++l) acc = fmaf(-s_Y[jb + i][l], x[l], acc);
+          t = acc * (s_tau[i] != 0.f ? s_tau[i] : 1.f);
         }
-        s_T[i][j] = t;
+        x[i] = t;
       }
-      __syncthreads();
+      for (int i = 0; i < NB; ++i) s_T[i][cc] = (s_tau[i] != 0.f && s_tau[cc] != 0.f && i <= cc) ? x[i] : 0.f;
+    } else if (tid < NB) {
+      for (int i = 0; i < NB; ++i) s_T[i][tid] = 0.f;
     }
+    __syncthreads();
     // U = X T_panel with X = V_before^T V_panel (rows 0..jb-1 of Y), in place, and
-    // Z = (S_rest V_panel) T_panel for the block rows after the panel, sent to every CTA
+    // Z = (S_rest V_panel) T_panel for the block rows after the panel
     for (int r = tid; r < kbo; r += PT) {
       if (r >= jb && r < jb + kb) continue;
       float x[NB];
 #pragma unroll
-      for (int l = 0; l < NB; ++l) x[l] = l < kb ? s_Y[r][l] : 0.f;
+      for (int l = 0; l < NB; ++l) x[l] = s_Y[r][l];
       for (int cc = 0; cc < NB; ++cc) {
         float acc = 0.f;
-        for (int l = 0; l <= cc && l < kb; ++l) acc = fmaf(x[l], s_T[l][cc], acc);
-        if (cc >= kb) acc = 0.f;
-        if (r < jb) {
-          s_Y[r][cc] = acc;
-        } else {
-          for (int q = 0; q < C; ++q) cluster.map_shared_rank(&s_Z[0][0], q)[(r - jb - kb) * NB + cc] = acc;
-        }
+        for (int l = 0; l <= cc; ++l) acc = fmaf(x[l], s_T[l][cc], acc);
+        if (r < jb) s_Y[r][cc] = acc;
+        else s_Z[r - jb - kb][cc] = acc;
       }
     }
     __syncthreads();
@@ -323,14 +334,12 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     for (int e = tid; e < NBO * NB; e += PT) {
       const int r = e / NB, cc = e % NB;
       float t = 0.f;
-      if (cc < kb) {
-        if (r < jb) {
-          float acc = 0.f;
-          for (int l = r; l < jb; ++l) acc = fmaf(T[r * NBO + l], s_Y[l][cc], acc);
-          t = -acc;
-        } else if (r < jb + kb && r - jb <= cc) {
-          t = s_T[r - jb][cc];
-        }
+      if (r < jb) {
+        float acc = 0.f;
+        for (int l = r; l < jb; ++l) acc = fmaf(s_Tb[r][l], s_Y[l][cc], acc);
+        t = -acc;
+      } else if (r < jb + NB) {
+        t = s_T[r - jb][cc];
       }
       const int col = jb + cc;
       T[r * NBO + col] = t;
@@ -351,17 +360,41 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     }
   }
   cluster.sync();
+  // every CTA takes Z from rank 0
+  if (c != 0) {
+    const float4* z0 = reinterpret_cast<const float4*>(cluster.map_shared_rank(&s_Z[0][0], 0));
+    for (int e = tid; e < nrest * (NB / 4); e += PT) reinterpret_cast<float4*>(&s_Z[0][0])[e] = z0[e];
+  }
+  cluster.sync();  // rank 0's s_Z stays in place until every CTA has its copy
 
-  // the panel's reflectors on the block rows after it: a_r -= Z_r V^T at this CTA's positions
+  // the panel's reflectors on the block rows after it: a_r -= Z_r V^T at this CTA's
+  // positions, four rows at a time
   for (int i = tid; i < npos; i += PT) {
     float v[NB];
 #pragma unroll
     for (int jj = 0; jj < NB; ++jj) v[jj] = sA[jj * LDS + i];
-    for (int r = 0; r < nrest; ++r) {
+    float* a = At + (int64_t)(k + kb) * n + pos0 + i;
+    int r = 0;
+    for (; r + 4 <= nrest; r += 4) {
+      float x[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) x[u] = a[(int64_t)(r + u) * n];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        float acc = 0.f;
+#pragma unroll
+        for (int j4 = 0; j4 < NB / 4; ++j4) {
+          const float4 z = *reinterpret_cast<const float4*>(&s_Z[r + u][4 * j4]);
+          acc = fmaf(z.x, v[4 * j4], fmaf(z.y, v[4 * j4 + 1], fmaf(z.z, v[4 * j4 + 2], fmaf(z.w, v[4 * j4 + 3], acc))));
+        }
+        a[(int64_t)(r + u) * n] = x[u] - acc;
+      }
+    }
+    for (; r < nrest; ++r) {
       float acc = 0.f;
 #pragma unroll
       for (int jj = 0; jj < NB; ++jj) acc = fmaf(s_Z[r][jj], v[jj], acc);
-      At[(int64_t)(k + kb + r) * n + pos0 + i] -= acc;
+      a[(int64_t)r * n] -= acc;
     }
   }
 }
@@ -428,6 +461,49 @@ __global__ void transpose_out_kernel(const float* Qt, float* Q, float* Q_lo, int
       if (Q_lo) Q_lo[o] = tf32_lo(x);
     }
   }
+}
+
+// The panel kernel variant for this device: 512 positions per CTA in clusters of up to 16
+// where the device runs 16-CTA clusters of it, else 1024 positions in clusters of up to 8.
+struct PanelKernel {
+  void (*fn)(PanelArgs);
+  int cols;
+  size_t smem;
+};
+
+template <int COLS>
+cudaError_t prepare_panel(PanelKernel* pk, bool wide) {
+  pk->fn = qr_panel_kernel<COLS>;
+  pk->cols = COLS;
+  pk->smem = (size_t)NB * (COLS + 4) * sizeof(float);
+  cudaError_t e = cudaFuncSetAttribute(pk->fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pk->smem);
+  if (e == cudaSuccess && wide) e = cudaFuncSetAttribute(pk->fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  return e;
+}
+
+cudaError_t panel_kernel(PanelKernel* pk) {
+  static int choice = 0;  // 0 unknown, 1 clusters of 16 x 512 positions, 2 clusters of 8 x 1024
+  if (choice == 0) {
+    int ok = 0;
+    if (prepare_panel<512>(pk, true) == cudaSuccess) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(16, 1, 1);
+      cfg.blockDim = dim3(PT, 1, 1);
+      cfg.dynamicSmemBytes = pk->smem;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = 16;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int clusters = 0;
+      if (cudaOccupancyMaxActiveClusters(&clusters, pk->fn, &cfg) == cudaSuccess && clusters > 0) ok = 1;
+    }
+    cudaGetLastError();
+    choice = ok ? 1 : 2;
+  }
+  return choice == 1 ? prepare_panel<512>(pk, true) : prepare_panel<1024>(pk, false);
 }
 
 struct Workspace {
@@ -507,7 +583,7 @@ void qr_input_buffers(void* workspace, int n, int batch, float** At, float** At_
 cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q_lo, uint8_t* skip, float tol,
                    void* workspace, size_t workspace_bytes, int* status, cudaStream_t s) {
   if (n <= 0 || batch <= 0) return cudaSuccess;
-  if (n > MAXC * COLS || batch > 65535 || (n & 3)) return cudaErrorInvalidValue;
+  if (n > 8192 || batch > 65535 || (n & 3)) return cudaErrorInvalidValue;
   size_t need = 0;
   Workspace w = carve(workspace, n, batch, &need);
   if (workspace_bytes < need) return cudaErrorInvalidValue;
@@ -527,21 +603,21 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     ProfScope prof(kFamOther, 0, 8.0 * NORM_CHUNKS * batch, s);
     thresh_kernel<<<(batch + 127) / 128, 128, 0, s>>>(w.part, tol, batch, w.thresh);
   }
-  const size_t smem = (size_t)NB * LDS * sizeof(float);
-  e = cudaFuncSetAttribute(qr_panel_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  PanelKernel pk;
+  e = panel_kernel(&pk);
   if (e != cudaSuccess) return e;
 
   for (int blk = 0; blk < nblock; ++blk) {
     const int k0 = blk * NBO, kbo = std::min(NBO, n - k0), m = n - k0;
     for (int k = k0; k < k0 + kbo; k += NB) {
       const int kb = std::min(NB, n - k);
-      const int C = (n - k + COLS - 1) / COLS;
+      const int C = (n - k + pk.cols - 1) / pk.cols;
       PanelArgs a{w.At, w.Vt, w.Vt_lo, w.Vpos, w.Vpos_lo, w.T, w.T_lo, w.Tt, w.Tt_lo, w.Ypart, skip, w.dsign,
                   w.thresh, status, n, k0, kbo, k, kb};
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(C, batch, 1);
       cfg.blockDim = dim3(PT, 1, 1);
-      cfg.dynamicSmemBytes = smem;
+      cfg.dynamicSmemBytes = pk.smem;
       cfg.stream = s;
       cudaLaunchAttribute attr[1];
       attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -555,7 +631,7 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
         // (2 kbo kb (n-k)) and the in-block update (2 kb (kbo-kb) (n-k))
         const double mk = (double)(n - k) * batch;
         ProfScope prof(kFamQrPanel, (4.0 * kb * kb + 4.0 * kbo * kb) * mk, 4.0 * (3.0 * kb + 2.0 * kbo) * mk, s);
-        e = cudaLaunchKernelEx(&cfg, qr_panel_kernel, a);
+        e = cudaLaunchKernelEx(&cfg, pk.fn, a);
       }
       if (e != cudaSuccess) return e;
     }

@@ -14,8 +14,8 @@
 
 namespace {
 
-// 32 MiB: room for the workspace of one 1024 x 1024 matrix (about 25 MB) or of several
-// smaller ones (e.g. 4 of 512 x 512). Every GPU that loads the library keeps this array
+// 32 MiB: room for the workspace of one 1024 x 1024 matrix (about 29 MB) or of several
+// smaller ones (e.g. 3 of 512 x 512). Every GPU that loads the library keeps this array
 // until the process exits.
 constexpr size_t kScratchBytes = size_t(32) << 20;
 __device__ __align__(256) unsigned char g_qr_scratch[kScratchBytes];
