@@ -107,10 +107,9 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
 
   extern __shared__ float4 smem_dyn[];
   float* sA = reinterpret_cast<float*>(smem_dyn);  // [NB][LDS]: panel row jj, position offset i
-  __shared__ float s_part[2][MAXC][NB];  // per-CTA partial [sigma | x . a_c], by source CTA
-  __shared__ float s_piv[2][NB];         // rank 0: pivot-row values [alpha | a_c,pivot]
-  __shared__ float s_sum[NB];
-  __shared__ float s_pv[NB];             // every CTA's copy of the pivot-row values
+  __shared__ float s_part[2][NB];        // this CTA's partial [sigma | x . a_c]
+  __shared__ float s_pv[2][NB];          // rank 0: pivot-row values [alpha | a_c,pivot]
+  __shared__ float s_scal[2];            // tau and 1 / v0 of the current reflector
   __shared__ float s_w[NB];              // v^T a_c
   __shared__ float s_tau[NB];
   __shared__ int s_skip[NB];
@@ -118,7 +117,12 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   __shared__ float s_T[NB][NB + 1];
   __shared__ float s_Y[NBO][NB + 1];     // rank 0: S V_panel summed over the cluster
   __shared__ __align__(16) float s_Z[NREST][NB];  // (S_rest V_panel) T_panel, the in-block update
-  __shared__ float s_Tb[NREST][NREST + 1];        // rank 0: the block's T so far
+  // staging of S (STG chunks of 128 x 32) while Y is formed; afterwards rank 0's copy of the
+  // block's T so far (96 x 97)
+  constexpr int STG = COLS <= 512 ? 4 : 2;
+  constexpr int SCRATCH = STG * NBO * 32 > NREST * (NREST + 1) ? STG * NBO * 32 : NREST * (NREST + 1);
+  __shared__ __align__(16) float s_scratch[SCRATCH];
+  float (*s_Tb)[NREST + 1] = reinterpret_cast<float (*)[NREST + 1]>(s_scratch);
 
   const int n = p.n, k = p.k, kb = p.kb, k0 = p.k0, kbo = p.kbo;
   const int jb = k - k0;                // panel offset inside its block
@@ -128,9 +132,18 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   const int pos0 = k + c * COLS;  // first position held by this CTA
   const int npos = max(0, min(COLS, n - pos0));  // a multiple of 4
 
-  for (int jj = 0; jj < NB; ++jj) {
-    const float* src = At + (int64_t)(k + jj) * n + pos0;
-    for (int i = tid; i < npos; i += PT) sA[jj * LDS + i] = jj < kb ? src[i] : 0.f;
+  const int npad = (npos + 31) & ~31;  // positions read by the chunked S V product
+  {
+    const int q4n = npad / 4;
+    for (int e = tid; e < NB * q4n; e += PT) {
+      const int jj = e / q4n, i = 4 * (e % q4n);
+      const bool ok = jj < kb && i < npos;
+      const float* src = ok ? At + (int64_t)(k + jj) * n + pos0 + i : At;
+      const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(&sA[jj * LDS + i]));
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(ok ? 16 : 0) : "memory");
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
   }
   __syncthreads();
   const float thresh = p.thresh[b];
@@ -140,53 +153,75 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     const int par = j & 1;
     // positions strictly after the pivot (pivot = local position j of rank 0)
     const int ibeg = (c == 0) ? j + 1 : 0;
-    // partial sums over this CTA: sigma (cc = j) and x . a_cc (cc > j), sent to every CTA
+    // partial sums over this CTA: sigma (cc = j) and x . a_cc (cc > j), kept locally; after
+    // the cluster barrier the threads that need them read every CTA's copy
     for (int cc = j + warp; cc < kb; cc += NWARP) {
-      float d = 0.f;
-      for (int i = ibeg + lane; i < npos; i += 32) d = fmaf(sA[j * LDS + i], sA[cc * LDS + i], d);
-      d = warp_sum(d);
-      if (lane < C) cluster.map_shared_rank(&s_part[par][0][0], lane)[c * NB + cc] = d;
+      float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
+      int i = ibeg + lane;
+      for (; i + 96 < npos; i += 128) {
+        d0 = fmaf(sA[j * LDS + i], sA[cc * LDS + i], d0);
+        d1 = fmaf(sA[j * LDS + i + 32], sA[cc * LDS + i + 32], d1);
+        d2 = fmaf(sA[j * LDS + i + 64], sA[cc * LDS + i + 64], d2);
+        d3 = fmaf(sA[j * LDS + i + 96], sA[cc * LDS + i + 96], d3);
+      }
+      for (; i < npos; i += 32) d0 = fmaf(sA[j * LDS + i], sA[cc * LDS + i], d0);
+      const float d = warp_sum((d0 + d1) + (d2 + d3));
+      if (lane == 0) s_part[par][cc] = d;
     }
-    if (c == 0 && tid >= j && tid < kb) s_piv[par][tid] = sA[tid * LDS + j];  // alpha, a_tid at the pivot
+    if (c == 0 && tid >= j && tid < kb) s_pv[par][tid] = sA[tid * LDS + j];  // alpha (tid == j), a_tid at the pivot
     cluster.sync();
+    // threads j..kb-1 reduce sigma and their own column's sum (in the same fixed order, so
+    // they all derive the same reflector) and form v^T a_tid
     if (tid >= j && tid < kb) {
-      float d = 0.f;
-      for (int q = 0; q < C; ++q) d += s_part[par][q][tid];
-      s_sum[tid] = d;
-      s_pv[tid] = *cluster.map_shared_rank(&s_piv[par][tid], 0);
-    }
-    __syncthreads();
-
-    // every thread derives the same reflector from the same reduced values
-    const float sigma = s_sum[j];
-    const float alpha = s_pv[j];
-    const float xnorm = sqrtf(fmaf(alpha, alpha, sigma));
-    if (!isfinite(xnorm)) nonfinite = 1;
-    const bool skip = !(xnorm > thresh);
-    float tau = 0.f, v0 = 1.f, rsign = 1.f;
-    if (!skip) {
-      if (sigma == 0.f) {
-        rsign = alpha < 0.f ? -1.f : 1.f;   // H = I, R_pp = alpha
-      } else {
-        const float beta = alpha >= 0.f ? -xnorm : xnorm;
-        v0 = alpha - beta;                   // same sign as alpha: no cancellation
-        tau = (beta - alpha) / beta;
-        rsign = beta < 0.f ? -1.f : 1.f;
+      float ps[MAXC], pd[MAXC];
+#pragma unroll
+      for (int q = 0; q < MAXC; ++q) {
+        if (q < C) {
+          const float* rp = cluster.map_shared_rank(&s_part[par][0], q);
+          ps[q] = rp[j];
+          pd[q] = rp[tid];
+        }
+      }
+      const float* pv0 = cluster.map_shared_rank(&s_pv[par][0], 0);
+      const float alpha = pv0[j], apiv = pv0[tid];
+      float d = 0.f, sigma = 0.f;
+#pragma unroll
+      for (int q = 0; q < MAXC; ++q) {
+        if (q < C) {
+          sigma += ps[q];
+          d += pd[q];
+        }
+      }
+      const float xnorm = sqrtf(fmaf(alpha, alpha, sigma));
+      const bool skip = !(xnorm > thresh);
+      float tau = 0.f, v0 = 1.f, rsign = 1.f;
+      if (!skip) {
+        if (sigma == 0.f) {
+          rsign = alpha < 0.f ? -1.f : 1.f;   // H = I, R_pp = alpha
+        } else {
+          const float beta = alpha >= 0.f ? -xnorm : xnorm;
+          v0 = alpha - beta;                   // same sign as alpha: no cancellation
+          tau = (beta - alpha) / beta;
+          rsign = beta < 0.f ? -1.f : 1.f;
+        }
+      }
+      if (tid == j) {
+        if (!isfinite(xnorm)) nonfinite = 1;
+        s_tau[j] = tau;
+        s_skip[j] = skip ? 1 : 0;
+        s_dsign[j] = rsign;
+        s_scal[0] = tau;
+        s_scal[1] = tau != 0.f ? 1.f / v0 : 0.f;
+      } else if (tau != 0.f) {
+        s_w[tid] = apiv + d / v0;  // v^T a_tid, with v = x / v0 after the pivot
       }
     }
-    // v^T a_cc = a_cc,pivot + (x . a_cc) / v0, with v = x / v0 after the pivot
-    if (tau != 0.f && tid > j && tid < kb) s_w[tid] = s_pv[tid] + s_sum[tid] / v0;
-    if (tid == 0) {
-      s_tau[j] = tau;
-      s_skip[j] = skip ? 1 : 0;
-      s_dsign[j] = rsign;
-    }
     __syncthreads();
+    const float tau = s_scal[0], rv0 = s_scal[1];
 
     // v after the pivot (x / v0, or 0 where H = I), and H_j = I - tau v v^T on the later
     // panel rows; every thread owns its positions
     const int piv = (c == 0) ? j : 0;  // local positions >= this take part
-    const float rv0 = tau != 0.f ? 1.f / v0 : 0.f;
     for (int i = piv + tid; i < npos; i += PT) {
       const bool at_pivot = (c == 0 && i == j);
       const float vi = at_pivot ? 1.f : sA[j * LDS + i] * rv0;
@@ -198,7 +233,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     }
     __syncthreads();
   }
-  if (nonfinite && tid == 0) atomicOr(p.status, kStatusQrBreakdown);
+  if (nonfinite) atomicOr(p.status, kStatusQrBreakdown);
 
   // V with its unit diagonal and zeros before it (rank 0 holds the first kb positions)
   if (c == 0) {
@@ -217,18 +252,20 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   float* Vpos = p.Vpos + (int64_t)b * n * NBO;
   float* Vpos_lo = p.Vpos_lo + (int64_t)b * n * NBO;
   for (int jj = 0; jj < kb; ++jj) {
-    const int64_t o = (int64_t)(k + jj) * n + pos0;
-    for (int i = tid; i < npos; i += PT) {
-      const float v = sA[jj * LDS + i];
-      Vt[o + i] = v;
-      Vt_lo[o + i] = tf32_lo(v);
+    float* vt = Vt + (int64_t)(k + jj) * n + pos0;
+    float* vl = Vt_lo + (int64_t)(k + jj) * n + pos0;
+    for (int q = tid; q < npos / 4; q += PT) {
+      const float4 v = *reinterpret_cast<const float4*>(&sA[jj * LDS + 4 * q]);
+      reinterpret_cast<float4*>(vt)[q] = v;
+      reinterpret_cast<float4*>(vl)[q] = make_float4(tf32_lo(v.x), tf32_lo(v.y), tf32_lo(v.z), tf32_lo(v.w));
     }
   }
-  for (int i = warp; i < npos; i += NWARP) {
-    const float v = sA[lane * LDS + i];  // rows kb.. of sA are zero
-    const int64_t o = (int64_t)(pos0 + i) * NBO + jb + lane;
-    Vpos[o] = v;
-    Vpos_lo[o] = tf32_lo(v);
+  for (int e = tid; e < npos * (NB / 4); e += PT) {
+    const int i = e >> 3, g4 = 4 * (e & 7);  // rows kb.. of sA are zero
+    const float4 v = make_float4(sA[g4 * LDS + i], sA[(g4 + 1) * LDS + i], sA[(g4 + 2) * LDS + i], sA[(g4 + 3) * LDS + i]);
+    const int64_t o = (int64_t)(pos0 + i) * NBO + jb + g4;
+    *reinterpret_cast<float4*>(Vpos + o) = v;
+    *reinterpret_cast<float4*>(Vpos_lo + o) = make_float4(tf32_lo(v.x), tf32_lo(v.y), tf32_lo(v.z), tf32_lo(v.w));
   }
   if (c == 0) {
     for (int jj = 0; jj < kb; ++jj)
@@ -247,27 +284,52 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
 
   // Y = S V_panel over this CTA's positions, S = the block's rows k0 .. k0+kbo-1: the block's
   // Householder vectors so far (rows before the panel's end, from Vt) and the block rows
-  // still to be factored (from At). Warp w takes rows w, w+16, ...; lane jj column jj.
+  // still to be factored (from At). S is streamed through shared memory in 32-position
+  // chunks (cp.async, double-buffered); warp w takes rows w, w+16, ...; lane jj column jj.
   {
     constexpr int RW = NBO / NWARP;
+    constexpr int CH = 32;  // positions per chunk
     float y[RW];
-    const float* srow[RW];
+#pragma unroll
+    for (int u = 0; u < RW; ++u) y[u] = 0.f;
     const int nr = (kbo - warp + NWARP - 1) / NWARP;  // rows of this warp
-#pragma unroll
-    for (int u = 0; u < RW; ++u) {
-      const int row = k0 + warp + NWARP * u;
-      y[u] = 0.f;
-      srow[u] = ((row < k + kb) ? Vt : At) + (int64_t)min(row, n - 1) * n + pos0;
+    const int nchunk = (npos + CH - 1) / CH;
+    auto issue = [&](int ch, int buf) {
+      float* dst = s_scratch + buf * NBO * CH;
+      for (int e = tid; e < NBO * (CH / 4); e += PT) {
+        const int r = e / (CH / 4), q4 = e % (CH / 4);
+        const int row = k0 + r, i = ch * CH + 4 * q4;
+        const bool ok = r < kbo && i < npos;
+        const float* src = ok ? ((row < k + kb) ? Vt : At) + (int64_t)row * n + pos0 + i : At;
+        const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst + r * CH + 4 * q4));
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(ok ? 16 : 0) : "memory");
+      }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    for (int st0 = 0; st0 < STG - 1; ++st0) {
+      if (st0 < nchunk) issue(st0, st0);
+      else asm volatile("cp.async.commit_group;" ::: "memory");
     }
-    for (int i = 0; i < npos; i += 4) {
-      const float4 v = *reinterpret_cast<const float4*>(&sA[lane * LDS + i]);
+    for (int ch = 0; ch < nchunk; ++ch) {
+      if (ch + STG - 1 < nchunk) issue(ch + STG - 1, (ch + STG - 1) % STG);
+      else asm volatile("cp.async.commit_group;" ::: "memory");  // keeps the group count uniform
+      asm volatile("cp.async.wait_group %0;" ::"n"(STG - 1) : "memory");
+      __syncthreads();
+      const float* st = s_scratch + (ch % STG) * NBO * CH;
+      const int i0 = ch * CH;
 #pragma unroll
-      for (int u = 0; u < RW; ++u) {
-        if (u < nr) {
-          const float4 x = *reinterpret_cast<const float4*>(srow[u] + i);
-          y[u] = fmaf(x.w, v.w, fmaf(x.z, v.z, fmaf(x.y, v.y, fmaf(x.x, v.x, y[u]))));
+      for (int q4 = 0; q4 < CH / 4; ++q4) {
+        // positions past npos are zero in the staged chunk (zero-filled copies)
+        const float4 v = *reinterpret_cast<const float4*>(&sA[lane * LDS + i0 + 4 * q4]);
+#pragma unroll
+        for (int u = 0; u < RW; ++u) {
+          if (u < nr) {
+            const float4 x = *reinterpret_cast<const float4*>(st + (warp + NWARP * u) * CH + 4 * q4);
+            y[u] = fmaf(x.w, v.w, fmaf(x.z, v.z, fmaf(x.y, v.y, fmaf(x.x, v.x, y[u]))));
+          }
         }
       }
+      __syncthreads();  // this buffer is refilled STG - 1 chunks later
     }
     float* yp = p.Ypart + ((int64_t)b * MAXC + c) * NBO * NB;
 #pragma unroll
@@ -292,60 +354,78 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     for (int e = tid; e < jb * jb; e += PT) s_Tb[e / jb][e % jb] = Tg[(e / jb) * NBO + e % jb];
     __syncthreads();
     // T of the panel from its Gram matrix g (rows jb.. of Y): T^-1 = diag(1/tau) + striu(g)
-    // (H_1 ... H_kb = I - V T V^T); a reflector with tau = 0 (v = 0) gets a zero row and column
-    if (tid < kb) {
+    // (H_1 ... H_kb = I - V T V^T); a reflector with tau = 0 (v = 0) gets a zero row and column.
+    // Thread cc solves for column cc by back substitution (fully unrolled, in registers).
+    if (tid < NB) {
       const int cc = tid;
       float x[NB];
-      // back substitution for column cc of T: (diag(1/tau) + striu(g)) x = e_cc
+#pragma unroll
       for (int i = NB - 1; i >= 0; --i) {
-        float t = 0.f;
-        if (i <= cc) {
-          float acc = (i == cc) ? 1.f : 0.f;
-          for (int l = i + 1; l <= cc; ++l) acc = fmaf(-s_Y[jb + i][l], x[l], acc);
-          t = acc * (s_tau[i] != 0.f ? s_tau[i] : 1.f);
-        }
-        x[i] = t;
+        float acc = (i == cc) ? 1.f : 0.f;
+#pragma unroll
+        for (int l = i + 1; l < NB; ++l)
+          if (l <= cc) acc = fmaf(-s_Y[jb + i][l], x[l], acc);
+        const float ti = i < kb ? s_tau[i] : 0.f;
+        x[i] = (i <= cc) ? acc * (ti != 0.f ? ti : 1.f) : 0.f;
       }
-      for (int i = 0; i < NB; ++i) s_T[i][cc] = (s_tau[i] != 0.f && s_tau[cc] != 0.f && i <= cc) ? x[i] : 0.f;
-    } else if (tid < NB) {
-      for (int i = 0; i < NB; ++i) s_T[i][tid] = 0.f;
+      const bool live = cc < kb && s_tau[cc] != 0.f;
+#pragma unroll
+      for (int i = 0; i < NB; ++i) s_T[i][cc] = (live && i < kb && s_tau[i] != 0.f) ? x[i] : 0.f;
     }
     __syncthreads();
     // U = X T_panel with X = V_before^T V_panel (rows 0..jb-1 of Y), in place, and
-    // Z = (S_rest V_panel) T_panel for the block rows after the panel
-    for (int r = tid; r < kbo; r += PT) {
-      if (r >= jb && r < jb + kb) continue;
+    // Z = (S_rest V_panel) T_panel for the block rows after the panel: thread (r, g) forms
+    // columns 8g .. 8g+7 of row r
+    {
+      const int r = tid >> 2, g8 = (tid & 3) * 8;
+      const bool act = r < kbo && (r < jb || r >= jb + kb);
       float x[NB];
 #pragma unroll
-      for (int l = 0; l < NB; ++l) x[l] = s_Y[r][l];
-      for (int cc = 0; cc < NB; ++cc) {
-        float acc = 0.f;
-        for (int l = 0; l <= cc; ++l) acc = fmaf(x[l], s_T[l][cc], acc);
-        if (r < jb) s_Y[r][cc] = acc;
-        else s_Z[r - jb - kb][cc] = acc;
+      for (int l = 0; l < NB; ++l) x[l] = act ? s_Y[r][l] : 0.f;
+      __syncthreads();  // every row is read before U overwrites it
+      if (act) {
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int cc = g8 + u;
+          float acc = 0.f;
+#pragma unroll
+          for (int l = 0; l < NB; ++l)
+            if (l <= cc) acc = fmaf(x[l], s_T[l][cc], acc);
+          if (r < jb) s_Y[r][cc] = acc;
+          else s_Z[r - jb - kb][cc] = acc;
+        }
       }
     }
     __syncthreads();
-    // the block's T: column block jb = [-T_before U ; T_panel ; 0], row block jb left of it = 0
+    // the block's T: column block jb = [-T_before U ; T_panel ; 0], row block jb left of it = 0;
+    // thread (r, g) writes columns jb + 8g .. jb + 8g+7 of row r
     float* T = p.T + (int64_t)b * NBO * NBO;
     float* T_lo = p.T_lo + (int64_t)b * NBO * NBO;
     float* Tt = p.Tt + (int64_t)b * NBO * NBO;
     float* Tt_lo = p.Tt_lo + (int64_t)b * NBO * NBO;
-    for (int e = tid; e < NBO * NB; e += PT) {
-      const int r = e / NB, cc = e % NB;
-      float t = 0.f;
+    {
+      const int r = tid >> 2, g8 = (tid & 3) * 8;
+      float t[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) t[u] = 0.f;
       if (r < jb) {
-        float acc = 0.f;
-        for (int l = r; l < jb; ++l) acc = fmaf(s_Tb[r][l], s_Y[l][cc], acc);
-        t = -acc;
+        for (int l = r; l < jb; ++l) {
+          const float tb = s_Tb[r][l];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) t[u] = fmaf(-tb, s_Y[l][g8 + u], t[u]);
+        }
       } else if (r < jb + NB) {
-        t = s_T[r - jb][cc];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) t[u] = s_T[r - jb][g8 + u];
       }
-      const int col = jb + cc;
-      T[r * NBO + col] = t;
-      T_lo[r * NBO + col] = tf32_lo(t);
-      Tt[col * NBO + r] = t;
-      Tt_lo[col * NBO + r] = tf32_lo(t);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int col = jb + g8 + u;
+        T[r * NBO + col] = t[u];
+        T_lo[r * NBO + col] = tf32_lo(t[u]);
+        Tt[col * NBO + r] = t[u];
+        Tt_lo[col * NBO + r] = tf32_lo(t[u]);
+      }
     }
     for (int e = tid; e < NB * jb; e += PT) {
       const int r = jb + e / jb, col = e % jb;
