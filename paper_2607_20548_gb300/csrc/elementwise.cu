@@ -11,6 +11,8 @@
 //    guard.
 //  * weight_update: W <- (1 - lr wd) W - lr N for a matrix with no preconditioned
 //    side (Alg. 1 "Weight decay and update" with Q_L = Q_R = I).
+#include <algorithm>
+
 #include "profile.h"
 #include "soap_internal.h"
 
@@ -33,7 +35,8 @@ __device__ __forceinline__ float lo_part(float x) {
 inline int blocks_for(int64_t elems, int batch) {
   int64_t want = (elems / 4 + kThreads - 1) / kThreads;
   if (want < 1) want = 1;
-  const int64_t cap = batch >= 64 ? 4 : (batch >= 8 ? 32 : 256);
+  // about 8 blocks of 256 threads per SM over the whole launch (152 SMs)
+  const int64_t cap = std::max<int64_t>(4, (8 * 152) / std::max(1, batch));
   return (int)(want < cap ? want : cap);
 }
 
@@ -74,6 +77,14 @@ __global__ void momentum_copy_kernel(const float* const* grads, float* Gc, float
   if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(status, kStatusNonFinite);
 }
 
+// One Adam step in the basis for one element (v updated, N returned).
+__device__ __forceinline__ float adam_one(float g, float m, float& v, float beta2, float c2, float eps, float inv_bc1,
+                                          float inv_sqrt_bc2) {
+  const float vn = fmaf(beta2, v, c2 * g * g);
+  v = vn;
+  return (m * inv_bc1) / (sqrtf(vn) * inv_sqrt_bc2 + eps);
+}
+
 __global__ void adam_kernel(float* Gp, const float* Mp, float* V, int rows, int cols, float beta2,
                             float eps, float inv_bc1, float inv_sqrt_bc2, const uint8_t* skipL,
                             const uint8_t* skipR, float* N_lo, int* status) {
@@ -82,21 +93,51 @@ __global__ void adam_kernel(float* Gp, const float* Mp, float* V, int rows, int 
   float* gp = Gp + (int64_t)b * elems;
   const float* mp = Mp + (int64_t)b * elems;
   float* v = V + (int64_t)b * elems;
+  float* nl = N_lo ? N_lo + (int64_t)b * elems : nullptr;
   const uint8_t* sl = skipL ? skipL + (int64_t)b * rows : nullptr;
   const uint8_t* sr = skipR ? skipR + (int64_t)b * cols : nullptr;
   const float c2 = 1.f - beta2;
   int bad = 0;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < elems; i += stride) {
-    const float g = gp[i];
-    const float m = mp[i];
-    const float vn = fmaf(beta2, v[i], c2 * g * g);
-    v[i] = vn;
-    float nv = (m * inv_bc1) / (sqrtf(vn) * inv_sqrt_bc2 + eps);
-    if ((sl && sl[i / cols]) || (sr && sr[i % cols])) nv = 0.f;
-    bad |= !isfinite(nv);
-    gp[i] = nv;
-    if (N_lo) N_lo[(int64_t)b * elems + i] = lo_part(nv);
+  const int64_t start = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if ((cols & 3) == 0) {
+    // four elements of one row per thread and step, 16-byte accesses (every matrix of the
+    // arena starts on a 16-byte boundary when cols is a multiple of 4)
+    for (int64_t i4 = start; i4 < elems / 4; i4 += stride) {
+      const float4 g = reinterpret_cast<const float4*>(gp)[i4];
+      const float4 m = reinterpret_cast<const float4*>(mp)[i4];
+      float4 vv = reinterpret_cast<const float4*>(v)[i4];
+      float4 o;
+      o.x = adam_one(g.x, m.x, vv.x, beta2, c2, eps, inv_bc1, inv_sqrt_bc2);
+      o.y = adam_one(g.y, m.y, vv.y, beta2, c2, eps, inv_bc1, inv_sqrt_bc2);
+      o.z = adam_one(g.z, m.z, vv.z, beta2, c2, eps, inv_bc1, inv_sqrt_bc2);
+      o.w = adam_one(g.w, m.w, vv.w, beta2, c2, eps, inv_bc1, inv_sqrt_bc2);
+      if (sl || sr) {
+        const int64_t row = (4 * i4) / cols;
+        const int col = (int)(4 * i4 - row * cols);
+        if (sl && sl[row]) o = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (sr) {
+          if (sr[col]) o.x = 0.f;
+          if (sr[col + 1]) o.y = 0.f;
+          if (sr[col + 2]) o.z = 0.f;
+          if (sr[col + 3]) o.w = 0.f;
+        }
+      }
+      bad |= !isfinite(o.x) | !isfinite(o.y) | !isfinite(o.z) | !isfinite(o.w);
+      reinterpret_cast<float4*>(v)[i4] = vv;
+      reinterpret_cast<float4*>(gp)[i4] = o;
+      if (nl) reinterpret_cast<float4*>(nl)[i4] = make_float4(lo_part(o.x), lo_part(o.y), lo_part(o.z), lo_part(o.w));
+    }
+  } else {
+    for (int64_t i = start; i < elems; i += stride) {
+      float vi = v[i];
+      float nv = adam_one(gp[i], mp[i], vi, beta2, c2, eps, inv_bc1, inv_sqrt_bc2);
+      v[i] = vi;
+      if ((sl && sl[i / cols]) || (sr && sr[i % cols])) nv = 0.f;
+      bad |= !isfinite(nv);
+      gp[i] = nv;
+      if (nl) nl[i] = lo_part(nv);
+    }
   }
   if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(status, kStatusNonFinite);
 }

@@ -15,10 +15,10 @@
 //
 // The tensor core's own accumulation rounds toward zero at every MMA, so a long chain
 // of MMAs into one accumulator drifts (relative error growing ~linearly in K: 6e-5 at
-// K = 8192). Each 32-wide K block is therefore accumulated afresh in one of two TMEM
-// accumulators while the epilogue warps drain the other into fp32 registers with
-// round-to-nearest adds; the drain of block k overlaps the MMAs of block k+1, and the
-// error stays at the level of an fp32 dot product.
+// K = 8192). Each 32-wide K block is therefore accumulated afresh in one of four TMEM
+// accumulators, used in turn, while the epilogue warps drain finished ones into fp32
+// registers with round-to-nearest adds; the drain of block k overlaps the MMAs of the
+// next blocks, and the error stays at the level of an fp32 dot product.
 //
 // CTA: warp 0 issues the TMA loads (one elected lane), warp 1 allocates tensor memory and
 // issues the MMAs (one elected lane), and 8 epilogue warps (4 for BN = 32) drain the
@@ -61,7 +61,10 @@ struct Cfg {
   // staging block (both swizzled in 16-byte units)
   static constexpr int OBUF = PRE ? 32 * CPW : 32 * 32;
   static constexpr int SMEM = STAGES * STAGE + EPI * OBUF * 4 + 1024 + 256;
-  static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators, used alternately
+  // four accumulators used in turn: a K block's partial sum may wait three K blocks of MMAs
+  // for the epilogue warps to drain it
+  static constexpr int NACC = 4;
+  static constexpr uint32_t TMEM_COLS = NACC * BN;
   static_assert(CPW % 32 == 0, "epilogue chunking");
   static_assert(SMEM <= 232448, "shared memory budget");
 };
@@ -187,8 +190,25 @@ __device__ __forceinline__ void cp_async16(float* smem_dst, const float* gmem_sr
 // conflict-free.
 __device__ __forceinline__ int swz(int r, int j) { return r * 32 + ((((j >> 2) ^ (r & 7))) << 2) + (j & 3); }
 
-// Tiles are numbered n-fastest, then m, then batch; a CTA takes `tpc` consecutive tiles, so
-// that the loads and MMAs of its next tile overlap the epilogue of the current one.
+// Tile t of a launch -> (m0, n0, batch index). Within a matrix the tiles go in groups of GM
+// row tiles: m fastest inside a group, then n, then the next group. The ~152 tiles in flight
+// at a time then read about GM A row panels and 152/GM B column panels, whose current K
+// slices stay in L2, instead of all of B once per row of tiles.
+constexpr int GM = 8;
+__device__ __forceinline__ void tile_coords(int t, int ntm, int ntn, int BN_, int& m0, int& n0, int& b) {
+  const int per = ntm * ntn;
+  b = t / per;
+  const int r = t - b * per;
+  const int g = r / (GM * ntn);
+  const int first = g * GM;
+  const int gsz = min(GM, ntm - first);
+  const int w = r - g * GM * ntn;
+  m0 = (first + w % gsz) * BM;
+  n0 = (w / gsz) * BN_;
+}
+
+// A CTA takes `tpc` consecutive tiles, so that the loads and MMAs of its next tile overlap
+// the epilogue of the current one.
 template <int BN, int STAGES, bool PRE>
 __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap ta_hi, const __grid_constant__ CUtensorMap ta_lo,
@@ -200,9 +220,9 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
   float* obuf_all = reinterpret_cast<float*>(smem + STAGES * C::STAGE);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE + C::EPI * C::OBUF * 4);
   uint64_t* empty = full + STAGES;
-  uint64_t* acc_full = empty + STAGES;  // [2] accumulator a holds a finished K block
-  uint64_t* acc_empty = acc_full + 2;   // [2] accumulator a has been drained
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  uint64_t* acc_full = empty + STAGES;      // [NACC] accumulator a holds a finished K block
+  uint64_t* acc_empty = acc_full + C::NACC;  // [NACC] accumulator a has been drained
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acc_empty + C::NACC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
   volatile int* consumed = abort_flag + 1;
 
@@ -218,7 +238,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    for (int a = 0; a < 2; ++a) {
+    for (int a = 0; a < C::NACC; ++a) {
       mbar_init(&acc_full[a], 1);
       mbar_init(&acc_empty[a], C::EPI);  // one arrival per epilogue warp
     }
@@ -246,7 +266,8 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     if (lane == 0) {
       int g = 0, issued = 0;  // k blocks over all of this CTA's tiles
       for (int t = t_begin; t < t_end && !*abort_flag; ++t) {
-        const int n0 = (t % ntn) * BN, m0 = ((t / ntn) % ntm) * BM, b = t / (ntn * ntm);
+        int m0, n0, b;
+        tile_coords(t, ntm, ntn, BN, m0, n0, b);
         for (int kb = 0; kb < kblocks; ++kb, ++g) {
           const int s = g % STAGES;
           const uint32_t ph = (g / STAGES) & 1;
@@ -277,8 +298,9 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
         for (int kb = 0; kb < kblocks; ++kb, ++g) {
           const int s = g % STAGES;
           const uint32_t ph = (g / STAGES) & 1;
-          const int a = g & 1;
-          if (!mbar_wait(&full[s], ph) || (g >= 2 && !mbar_wait(&acc_empty[a], ((g >> 1) & 1) ^ 1)) ||
+          const int a = g % C::NACC;
+          if (!mbar_wait(&full[s], ph) ||
+              (g >= C::NACC && !mbar_wait(&acc_empty[a], ((g / C::NACC) & 1) ^ 1)) ||
               *abort_flag) {
             *abort_flag = 1;
             break;
@@ -311,7 +333,8 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     int g = 0;
     bool valid = true;
     for (int t = t_begin; t < t_end && valid; ++t) {
-      const int n0 = (t % ntn) * BN, m0 = ((t / ntn) % ntm) * BM, b = t / (ntn * ntm);
+      int m0, n0, b;
+      tile_coords(t, ntm, ntn, BN, m0, n0, b);
       float* Cb = ep.C_ptrs ? ep.C_ptrs[b] : (ep.C ? ep.C + (int64_t)b * ep.c_stride : nullptr);
       float* Lb = ep.C_lo ? ep.C_lo + (int64_t)b * ep.lo_stride : nullptr;
       const int row0 = m0 + 32 * q;   // first of this warp's 32 rows
@@ -348,8 +371,8 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
 #pragma unroll
         for (int j = 0; j < 32; ++j) acc[c][j] = 0.f;
       for (int kb = 0; kb < kblocks; ++kb, ++g) {
-        const int a = g & 1;
-        if (!mbar_wait(&acc_full[a], (g >> 1) & 1) || *abort_flag) {
+        const int a = g % C::NACC;
+        if (!mbar_wait(&acc_full[a], (g / C::NACC) & 1) || *abort_flag) {
           valid = false;
           break;
         }
