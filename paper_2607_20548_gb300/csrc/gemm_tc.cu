@@ -208,12 +208,14 @@ __device__ __forceinline__ void tile_coords(int t, int ntm, int ntn, int BN_, in
 }
 
 // A CTA takes `tpc` consecutive tiles, so that the loads and MMAs of its next tile overlap
-// the epilogue of the current one.
+// the epilogue of the current one. With ksplit > 1 the K blocks are split into ksplit
+// consecutive ranges; split s of matrix b is written as output matrix s * batch + b (partial
+// sums that the caller adds up).
 template <int BN, int STAGES, bool PRE>
 __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap ta_hi, const __grid_constant__ CUtensorMap ta_lo,
                    const __grid_constant__ CUtensorMap tb_hi, const __grid_constant__ CUtensorMap tb_lo, int M,
-                   int N, int K, int batch, int a_mod, int b_mod, int tpc, TcEpilogue ep) {
+                   int N, int K, int batch, int a_mod, int b_mod, int tpc, int ksplit, TcEpilogue ep) {
   using C = Cfg<BN, STAGES, PRE>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -228,8 +230,14 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int kblocks = (K + BK - 1) / BK;
+  const int kper = (kblocks + ksplit - 1) / ksplit;  // K blocks of one split
   const int ntn = (N + BN - 1) / BN, ntm = (M + BM - 1) / BM;
-  const int ntiles = ntn * ntm * batch;
+  const int ntiles = ntn * ntm * batch * ksplit;
+  // the K blocks [kb0, kb1) of tile t, and its operand and output matrix indices
+  auto krange = [&](int bo, int& kb0, int& kb1) {
+    kb0 = (bo / batch) * kper;
+    kb1 = min(kblocks, kb0 + kper);
+  };
   const int t_begin = blockIdx.x * tpc;
   const int t_end = min(ntiles, t_begin + tpc);
 
@@ -266,9 +274,11 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     if (lane == 0) {
       int g = 0, issued = 0;  // k blocks over all of this CTA's tiles
       for (int t = t_begin; t < t_end && !*abort_flag; ++t) {
-        int m0, n0, b;
-        tile_coords(t, ntm, ntn, BN, m0, n0, b);
-        for (int kb = 0; kb < kblocks; ++kb, ++g) {
+        int m0, n0, bo, kb0, kb1;
+        tile_coords(t, ntm, ntn, BN, m0, n0, bo);
+        krange(bo, kb0, kb1);
+        const int b = bo % batch;
+        for (int kb = kb0; kb < kb1; ++kb, ++g) {
           const int s = g % STAGES;
           const uint32_t ph = (g / STAGES) & 1;
           if (!mbar_wait(&empty[s], ph ^ 1) || *abort_flag) {
@@ -295,7 +305,10 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
       constexpr uint32_t idesc = idesc_tf32(BM, BN);
       int g = 0;
       for (int t = t_begin; t < t_end && !*abort_flag; ++t) {
-        for (int kb = 0; kb < kblocks; ++kb, ++g) {
+        int m0, n0, bo, kb0, kb1;
+        tile_coords(t, ntm, ntn, BN, m0, n0, bo);
+        krange(bo, kb0, kb1);
+        for (int kb = kb0; kb < kb1; ++kb, ++g) {
           const int s = g % STAGES;
           const uint32_t ph = (g / STAGES) & 1;
           const int a = g % C::NACC;
@@ -333,8 +346,9 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     int g = 0;
     bool valid = true;
     for (int t = t_begin; t < t_end && valid; ++t) {
-      int m0, n0, b;
+      int m0, n0, b, kb0, kb1;  // b: output matrix (split * batch + operand matrix)
       tile_coords(t, ntm, ntn, BN, m0, n0, b);
+      krange(b, kb0, kb1);
       float* Cb = ep.C_ptrs ? ep.C_ptrs[b] : (ep.C ? ep.C + (int64_t)b * ep.c_stride : nullptr);
       float* Lb = ep.C_lo ? ep.C_lo + (int64_t)b * ep.lo_stride : nullptr;
       const int row0 = m0 + 32 * q;   // first of this warp's 32 rows
@@ -370,7 +384,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
       for (int c = 0; c < C::NCH; ++c)
 #pragma unroll
         for (int j = 0; j < 32; ++j) acc[c][j] = 0.f;
-      for (int kb = 0; kb < kblocks; ++kb, ++g) {
+      for (int kb = kb0; kb < kb1; ++kb, ++g) {
         const int a = g % C::NACC;
         if (!mbar_wait(&acc_full[a], (g / C::NACC) & 1) || *abort_flag) {
           valid = false;
@@ -538,7 +552,7 @@ bool make_map(CUtensorMap* map, const float* base, int rows, int K, int64_t ld, 
 
 template <int BN, int STAGES, bool PRE>
 cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, int batch, const TcEpilogue& ep,
-                   cudaStream_t s) {
+                   cudaStream_t s, int ksplit = 1) {
   using C = Cfg<BN, STAGES, PRE>;
   CUtensorMap m[4];
   const int amod = A.batch > 0 ? A.batch : batch;
@@ -553,7 +567,7 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  const int64_t ntiles = (int64_t)((N + BN - 1) / BN) * ((M + BM - 1) / BM) * batch;
+  const int64_t ntiles = (int64_t)((N + BN - 1) / BN) * ((M + BM - 1) / BM) * batch * ksplit;
   if (ntiles > (int64_t)1 << 30) return cudaErrorInvalidValue;
   // short K: a CTA runs several tiles so that the next tile's loads and MMAs overlap the
   // current epilogue, keeping about four waves of CTAs over the 152 SMs
@@ -561,14 +575,56 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
   const int tpc = kblocks > 16 ? 1 : (int)std::max<int64_t>(1, std::min<int64_t>(8, ntiles / (4 * 152)));
   const int grid = (int)((ntiles + tpc - 1) / tpc);
   gemm_tc_kernel<BN, STAGES, PRE><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
-                                                                     bmod, tpc, ep);
+                                                                     bmod, tpc, ksplit, ep);
   return cudaGetLastError();
+}
+
+// C_b = alpha * sum_s P_(s*batch+b) (M x N partial sums, contiguous) and its lo part,
+// 16-byte units along N (N a multiple of 4).
+__global__ void split_reduce_kernel(const float* P, int ksplit, int batch, int M, int N, float alpha, float* C,
+                                    int64_t ldc, int64_t c_stride, float* C_lo) {
+  const int b = blockIdx.y;
+  const int64_t mn = (int64_t)M * N, n4 = mn / 4;
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n4; u += (int64_t)gridDim.x * blockDim.x) {
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int sp = 0; sp < ksplit; ++sp) {
+      const float4 v = reinterpret_cast<const float4*>(P + ((int64_t)sp * batch + b) * mn)[u];
+      acc.x += v.x;
+      acc.y += v.y;
+      acc.z += v.z;
+      acc.w += v.w;
+    }
+    const float4 o = make_float4(alpha * acc.x, alpha * acc.y, alpha * acc.z, alpha * acc.w);
+    const int64_t e = 4 * u, i = e / N, j = e - i * N;
+    *reinterpret_cast<float4*>(C + (int64_t)b * c_stride + i * ldc + j) = o;
+    if (C_lo)
+      *reinterpret_cast<float4*>(C_lo + (int64_t)b * c_stride + i * ldc + j) =
+          make_float4(tf32_lo(o.x), tf32_lo(o.y), tf32_lo(o.z), tf32_lo(o.w));
+  }
+}
+
+// How many K splits give the fewest idle SMs in the last wave, for a launch of `tiles` tiles
+// with kblocks K blocks (each split keeps at least 16 K blocks), within `cap` partial matrices.
+int choose_ksplit(int64_t tiles, int kblocks, int64_t cap) {
+  if (kblocks < 32 || tiles >= 2 * 152) return 1;
+  int best = 1;
+  double best_eff = 0.0;
+  for (int sp = 1; sp <= 8 && kblocks / sp >= 16 && sp <= cap; ++sp) {
+    const int64_t ctas = tiles * sp;
+    const double eff = (double)ctas / (double)(((ctas + 151) / 152) * 152);
+    if (eff > best_eff + 0.02) {
+      best_eff = eff;
+      best = sp;
+    }
+  }
+  const int kper = (kblocks + best - 1) / best;
+  return (kblocks + kper - 1) / kper;  // no empty split
 }
 
 }  // namespace tc
 
 cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const TcOperand& B, const TcEpilogue& ep,
-                       cudaStream_t s, int family) {
+                       cudaStream_t s, int family, float* split_ws, size_t split_ws_floats) {
   if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
   if (batch > 65535) return cudaErrorInvalidValue;
   const double flops = 2.0 * M * N * (double)K * batch;  // algorithmic (4 tf32 products each on the pipe)
@@ -578,6 +634,27 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
   ProfScope prof(family, flops, bytes, s);
   // an epilogue that reads C gives one pipeline stage's shared memory to the C tile
   const bool pre = ep.beta != 0.f && (ep.C || ep.C_ptrs);
+  // few tiles and a long K: split K over more CTAs (plain row-major outputs only)
+  int ksplit = 1;
+  const bool splittable = split_ws && ep.C && !ep.C_ptrs && !ep.transpose && ep.beta == 0.f && (N & 3) == 0 &&
+                          (ep.ldc & 3) == 0 && (ep.c_stride & 3) == 0 && (!ep.C_lo || (ep.ld_lo == ep.ldc && ep.lo_stride == ep.c_stride)) &&
+                          (reinterpret_cast<uintptr_t>(ep.C) & 15) == 0;
+  if (splittable) {
+    const int bn = N <= 32 ? 32 : 128;
+    const int64_t tiles = (int64_t)((N + bn - 1) / bn) * ((M + tc::BM - 1) / tc::BM) * batch;
+    ksplit = tc::choose_ksplit(tiles, (K + tc::BK - 1) / tc::BK, (int64_t)(split_ws_floats / ((size_t)M * N * batch)));
+  }
+  if (ksplit > 1) {
+    const TcEpilogue pe{split_ws, nullptr, N, (int64_t)M * N, nullptr, N, (int64_t)M * N, 0, 1.f, 0.f, ep.status};
+    cudaError_t e = N <= 32 ? tc::launch<32, 5, false>(A, B, M, N, K, batch, pe, s, ksplit)
+                            : tc::launch<128, 3, false>(A, B, M, N, K, batch, pe, s, ksplit);
+    if (e != cudaSuccess) return e;
+    const int64_t n4 = (int64_t)M * N / 4;
+    const int blocks = (int)std::min<int64_t>((n4 + 255) / 256, std::max(1, 1216 / batch));
+    tc::split_reduce_kernel<<<dim3(blocks, batch), 256, 0, s>>>(split_ws, ksplit, batch, M, N, ep.alpha, ep.C, ep.ldc,
+                                                                ep.c_stride, ep.C_lo);
+    return cudaGetLastError();
+  }
   if (N <= 32) return pre ? tc::launch<32, 4, true>(A, B, M, N, K, batch, ep, s)
                           : tc::launch<32, 5, false>(A, B, M, N, K, batch, ep, s);
   return pre ? tc::launch<128, 2, true>(A, B, M, N, K, batch, ep, s)

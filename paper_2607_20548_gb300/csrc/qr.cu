@@ -62,6 +62,7 @@ constexpr int PT = 512;           // threads per panel CTA
 constexpr int MAXC = 16;          // largest cluster (16 needs the non-portable cluster size)
 constexpr int NWARP = PT / 32;
 constexpr int NREST = NBO - NB;   // most block rows after a panel
+constexpr int KSPLIT = 8;         // most K splits of the block products W = At Vt^T
 
 // lo part of x for the tensor-core products: x - trunc_tf32(x) rounded to the nearest tf32
 __device__ __forceinline__ float tf32_lo(float x) {
@@ -479,16 +480,21 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   }
 }
 
-// ||P_b||_F: per-chunk partial sums in double, then tol * sqrt(sum)
-constexpr int NORM_CHUNKS = 64;
+// ||P_b||_F: per-chunk partial sums in double (chunks of whole 16-byte units: nn is a
+// multiple of 16), then tol * sqrt(sum)
+constexpr int NORM_CHUNKS = 512;
 
 __global__ void frob_partial_kernel(const float* P, int64_t nn, double* part) {
   const int b = blockIdx.y;
-  const float* x = P + (int64_t)b * nn;
-  const int64_t per = (nn + NORM_CHUNKS - 1) / NORM_CHUNKS;
-  const int64_t beg = blockIdx.x * per, end = min(nn, beg + per);
+  const float4* x = reinterpret_cast<const float4*>(P + (int64_t)b * nn);
+  const int64_t n4 = nn / 4;
+  const int64_t per = (n4 + NORM_CHUNKS - 1) / NORM_CHUNKS;
+  const int64_t beg = blockIdx.x * per, end = min(n4, beg + per);
   double s = 0.0;
-  for (int64_t i = beg + threadIdx.x; i < end; i += blockDim.x) s += (double)x[i] * (double)x[i];
+  for (int64_t i = beg + threadIdx.x; i < end; i += blockDim.x) {
+    const float4 v = x[i];
+    s += (double)v.x * v.x + (double)v.y * v.y + (double)v.z * v.z + (double)v.w * v.w;
+  }
   __shared__ double red[256];
   red[threadIdx.x] = s;
   __syncthreads();
@@ -604,6 +610,7 @@ struct Workspace {
   float* Tt;
   float* Tt_lo;
   float* Ypart;   // [batch][MAXC][NBO][NB]
+  float* Wsplit;  // [KSPLIT][batch][n][NBO] partial sums of split-K products
   float* thresh;
   float* dsign;
   double* part;
@@ -628,6 +635,7 @@ Workspace carve(void* base, int n, int batch, size_t* total) {
   const size_t oVp = take(thin), oVpl = take(thin), oW = take(thin), oWl = take(thin);
   const size_t oT = take(tsq), oTl = take(tsq), oTt = take(tsq), oTtl = take(tsq);
   const size_t oY = take((size_t)batch * MAXC * NBO * NB * sizeof(float));
+  const size_t oWs = take((size_t)KSPLIT * thin);
   const size_t oth = take((size_t)batch * sizeof(float));
   const size_t osg = take((size_t)batch * n * sizeof(float));
   const size_t opart = take((size_t)batch * NORM_CHUNKS * sizeof(double));
@@ -635,7 +643,8 @@ Workspace carve(void* base, int n, int batch, size_t* total) {
   char* c = (char*)base;
   auto f = [&](size_t o) { return (float*)(c + o); };
   return Workspace{f(oAt), f(oAtl), f(oVt), f(oVtl), f(oVq), f(oVql), f(oVr), f(oVrl), f(oVp), f(oVpl),
-                   f(oW),  f(oWl),  f(oT),  f(oTl),  f(oTt), f(oTtl), f(oY),  f(oth),  f(osg), (double*)(c + opart)};
+                   f(oW),  f(oWl),  f(oT),  f(oTl),  f(oTt), f(oTtl), f(oY),  f(oWs), f(oth),  f(osg),
+                   (double*)(c + opart)};
 }
 
 TcOperand op(const float* hi, const float* lo, int64_t ld, int64_t stride, int batch) {
@@ -732,7 +741,8 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     const int64_t tr = (int64_t)(k0 + kbo) * n;
     e = gemm_tc_nt(nc, kbo, m, batch, op(w.At + tr + k0, w.At_lo + tr + k0, n, nn, batch),
                    op(w.Vt + (int64_t)k0 * n + k0, w.Vt_lo + (int64_t)k0 * n + k0, n, nn, batch),
-                   out(w.W, w.W_lo, NBO, thin, 1.f, 0.f, status), s, kFamQrUpdate);
+                   out(w.W, w.W_lo, NBO, thin, 1.f, 0.f, status), s, kFamQrUpdate, w.Wsplit,
+                   (size_t)KSPLIT * batch * n * NBO);
     if (e != cudaSuccess) return e;
     // At_trail -= W VTr^T at positions k0+kbo.. (the earlier positions of these rows are R's)
     e = gemm_tc_nt(nc, nc, kbo, batch, op(w.W, w.W_lo, NBO, thin, batch),
@@ -755,7 +765,7 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     // W = Qt_sub Vt^T  (m x kbo)
     e = gemm_tc_nt(m, kbo, m, batch, op(Qt + sub, Qt_lo + sub, n, nn, batch),
                    op(w.Vt + sub, w.Vt_lo + sub, n, nn, batch), out(w.W, w.W_lo, NBO, thin, 1.f, 0.f, status), s,
-                   kFamQrUpdate);
+                   kFamQrUpdate, w.Wsplit, (size_t)KSPLIT * batch * n * NBO);
     if (e != cudaSuccess) return e;
     // Qt_sub -= W VTq^T
     const int64_t vq = (int64_t)blk * thin + (int64_t)k0 * NBO;

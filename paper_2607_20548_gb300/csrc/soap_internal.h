@@ -71,9 +71,12 @@ struct TcEpilogue {
   float alpha, beta;     // beta != 0 reads C
   int* status;           // device status word for a timed-out wait (may be nullptr)
 };
-// `family` tags the launch for the library's profiler.
+// `family` tags the launch for the library's profiler. With a split workspace (room for
+// ksplit * batch * M * N floats) a launch of few tiles and long K may split K over more CTAs
+// and add the partial sums in a second kernel (row-major C with beta = 0 only).
 cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const TcOperand& B,
-                       const TcEpilogue& ep, cudaStream_t stream, int family = kFamGemmTc);
+                       const TcEpilogue& ep, cudaStream_t stream, int family = kFamGemmTc,
+                       float* split_ws = nullptr, size_t split_ws_floats = 0);
 // hi = trunc_tf32(x), lo = x - hi (exact), elementwise over n values.
 cudaError_t split_tf32(const float* x, float* hi, float* lo, int64_t n, cudaStream_t stream);
 
