@@ -175,6 +175,20 @@ soap_status_t soap_profile_begin(soap_handle h, int64_t max_launches);
 soap_status_t soap_profile_end(soap_handle h, soap_stream_t stream, soap_kernel_stats* out,
                                int32_t* overflow);
 
+/* One timed launch: its family and its start and end, in ms after the first timed launch
+ * started (CUDA events on the launch's stream). */
+typedef struct {
+  int32_t family;   /* soap_kernel_family */
+  double start_ms;
+  double end_ms;
+} soap_launch_record;
+
+/* Synchronises the device and copies the launches timed since soap_profile_begin, in launch
+ * order, to out[] (at most max of them; *count receives how many were written). Call it
+ * before soap_profile_end, which discards them. The library's QR streams run concurrently
+ * with each other and with the caller's stream, so records may overlap in time. */
+soap_status_t soap_profile_records(soap_handle h, soap_launch_record* out, int64_t max, int64_t* count);
+
 /* ---- stand-alone sub-steps (the same kernels soap_step runs) ------------------- */
 
 /* S3, Alg. 1 "QR(L_t Q_L).Q": for `batch` square n x n matrices P (device,

@@ -273,7 +273,7 @@ __global__ void basis_from_qt_kernel(const float* Qt, const float* Qt_lo, float*
       const int64_t o = (int64_t)b * nn + (int64_t)r * n + c;
       x = Qt[o];
       if (Qt_out) Qt_out[o] = x;
-      if (Qt_lo_out) Qt_lo_out[o] = Qt_lo[o];
+      if (Qt_lo_out) Qt_lo_out[o] = lo_part(x);
     }
     tile[i][threadIdx.x] = x;
   }

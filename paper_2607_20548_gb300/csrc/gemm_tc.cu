@@ -211,7 +211,10 @@ __device__ __forceinline__ void tile_coords(int t, int ntm, int ntn, int BN_, in
 // the epilogue of the current one. With ksplit > 1 the K blocks are split into ksplit
 // consecutive ranges; split s of matrix b is written as output matrix s * batch + b (partial
 // sums that the caller adds up).
-template <int BN, int STAGES, bool PRE>
+// With CVTA the A operand comes as fp32 only: the epilogue warps form its lo part in shared
+// memory, beside the tile TMA brought in (for HBM-bound products whose A is read once; the
+// extra shared-memory traffic would slow a compute-bound product).
+template <int BN, int STAGES, bool PRE, bool CVTA>
 __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap ta_hi, const __grid_constant__ CUtensorMap ta_lo,
                    const __grid_constant__ CUtensorMap tb_hi, const __grid_constant__ CUtensorMap tb_lo, int M,
@@ -222,7 +225,8 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
   float* obuf_all = reinterpret_cast<float*>(smem + STAGES * C::STAGE);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE + C::EPI * C::OBUF * 4);
   uint64_t* empty = full + STAGES;
-  uint64_t* acc_full = empty + STAGES;      // [NACC] accumulator a holds a finished K block
+  uint64_t* conv = empty + STAGES;          // [STAGES] CVTA: the stage's A lo part is in place
+  uint64_t* acc_full = conv + STAGES;       // [NACC] accumulator a holds a finished K block
   uint64_t* acc_empty = acc_full + C::NACC;  // [NACC] accumulator a has been drained
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acc_empty + C::NACC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
@@ -245,6 +249,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
+      mbar_init(&conv[s], C::EPI);  // one arrival per epilogue warp
     }
     for (int a = 0; a < C::NACC; ++a) {
       mbar_init(&acc_full[a], 1);
@@ -285,11 +290,11 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
             *abort_flag = 1;
             break;
           }
-          mbar_expect_tx(&full[s], C::STAGE);
+          mbar_expect_tx(&full[s], CVTA ? C::STAGE - C::TILE_A : C::STAGE);
           const uint32_t st = smem_u32(smem + s * C::STAGE);
           const int kc = kb * BK;
           tma_load_3d(st, &ta_hi, &full[s], kc, m0, b % a_mod);
-          tma_load_3d(st + C::TILE_A, &ta_lo, &full[s], kc, m0, b % a_mod);
+          if (!CVTA) tma_load_3d(st + C::TILE_A, &ta_lo, &full[s], kc, m0, b % a_mod);
           tma_load_3d(st + 2 * C::TILE_A, &tb_hi, &full[s], kc, n0, b % b_mod);
           tma_load_3d(st + 2 * C::TILE_A + C::TILE_B, &tb_lo, &full[s], kc, n0, b % b_mod);
           issued = g + 1;
@@ -312,7 +317,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
           const int s = g % STAGES;
           const uint32_t ph = (g / STAGES) & 1;
           const int a = g % C::NACC;
-          if (!mbar_wait(&full[s], ph) ||
+          if (!mbar_wait(CVTA ? &conv[s] : &full[s], ph) ||
               (g >= C::NACC && !mbar_wait(&acc_empty[a], ((g / C::NACC) & 1) ^ 1)) ||
               *abort_flag) {
             *abort_flag = 1;
@@ -343,6 +348,31 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     const int colbase = ((warp - 2) / 4) * C::CPW;
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * q) << 16);
     float* obuf = obuf_all + (warp - 2) * C::OBUF;
+    // CVTA: the lo part of k block gc's A tile, x - trunc_tf32(x) rounded to the nearest tf32,
+    // written beside it for the tensor core (which reads it through the async proxy)
+    auto convert = [&](int gc) -> bool {
+      const int s = gc % STAGES;
+      if (!mbar_wait(&full[s], (gc / STAGES) & 1) || *abort_flag) return false;
+      const float4* src = reinterpret_cast<const float4*>(smem + s * C::STAGE);
+      float4* dst = reinterpret_cast<float4*>(smem + s * C::STAGE + C::TILE_A);
+      for (int u = (warp - 2) * 32 + lane; u < C::TILE_A / 16; u += C::EPI * 32) {
+        const float4 v = src[u];
+        dst[u] = make_float4(tf32_lo(v.x), tf32_lo(v.y), tf32_lo(v.z), tf32_lo(v.w));
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&conv[s])) : "memory");
+      return true;
+    };
+    int gtotal = 0;  // K blocks over this CTA's tiles
+    if (CVTA)
+      for (int t = t_begin; t < t_end; ++t) {
+        int m0, n0, bo, kb0, kb1;
+        tile_coords(t, ntm, ntn, BN, m0, n0, bo);
+        krange(bo, kb0, kb1);
+        gtotal += kb1 - kb0;
+      }
+    int gconv = 0;  // next K block to convert, kept STAGES - 1 ahead of the drains
     int g = 0;
     bool valid = true;
     for (int t = t_begin; t < t_end && valid; ++t) {
@@ -385,8 +415,10 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
 #pragma unroll
         for (int j = 0; j < 32; ++j) acc[c][j] = 0.f;
       for (int kb = kb0; kb < kb1; ++kb, ++g) {
+        if (CVTA)
+          while (valid && gconv < gtotal && gconv <= g + STAGES - 1) valid = convert(gconv++);
         const int a = g % C::NACC;
-        if (!mbar_wait(&acc_full[a], (g / C::NACC) & 1) || *abort_flag) {
+        if (!valid || !mbar_wait(&acc_full[a], (g / C::NACC) & 1) || *abort_flag) {
           valid = false;
           break;
         }
@@ -550,20 +582,21 @@ bool make_map(CUtensorMap* map, const float* base, int rows, int K, int64_t ld, 
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES, bool PRE>
+template <int BN, int STAGES, bool PRE, bool CVTA = false>
 cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, int batch, const TcEpilogue& ep,
                    cudaStream_t s, int ksplit = 1) {
   using C = Cfg<BN, STAGES, PRE>;
   CUtensorMap m[4];
   const int amod = A.batch > 0 ? A.batch : batch;
   const int bmod = B.batch > 0 ? B.batch : batch;
-  if (!make_map(&m[0], A.hi, M, K, A.ld, A.stride, amod, BM) || !make_map(&m[1], A.lo, M, K, A.ld, A.stride, amod, BM) ||
+  if (!make_map(&m[0], A.hi, M, K, A.ld, A.stride, amod, BM) ||
+      !make_map(&m[1], CVTA ? A.hi : A.lo, M, K, A.ld, A.stride, amod, BM) ||
       !make_map(&m[2], B.hi, N, K, B.ld, B.stride, bmod, BN) || !make_map(&m[3], B.lo, N, K, B.ld, B.stride, bmod, BN))
     return cudaErrorInvalidValue;
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e =
-        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE, CVTA>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
@@ -574,7 +607,7 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
   const int kblocks = (K + BK - 1) / BK;
   const int tpc = kblocks > 16 ? 1 : (int)std::max<int64_t>(1, std::min<int64_t>(8, ntiles / (4 * 152)));
   const int grid = (int)((ntiles + tpc - 1) / tpc);
-  gemm_tc_kernel<BN, STAGES, PRE><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
+  gemm_tc_kernel<BN, STAGES, PRE, CVTA><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
                                                                      bmod, tpc, ksplit, ep);
   return cudaGetLastError();
 }
@@ -628,7 +661,7 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
   if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
   if (batch > 65535) return cudaErrorInvalidValue;
   const double flops = 2.0 * M * N * (double)K * batch;  // algorithmic (4 tf32 products each on the pipe)
-  const double bytes = 4.0 * (2.0 * (double)M * K * (A.batch > 0 ? A.batch : batch) +
+  const double bytes = 4.0 * ((A.lo ? 2.0 : 1.0) * (double)M * K * (A.batch > 0 ? A.batch : batch) +
                               2.0 * (double)N * K * (B.batch > 0 ? B.batch : batch) +
                               (double)M * N * batch * ((ep.beta != 0.f ? 2 : 1) + (ep.C_lo ? 1 : 0)));
   ProfScope prof(family, flops, bytes, s);
@@ -644,10 +677,16 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
     const int64_t tiles = (int64_t)((N + bn - 1) / bn) * ((M + tc::BM - 1) / tc::BM) * batch;
     ksplit = tc::choose_ksplit(tiles, (K + tc::BK - 1) / tc::BK, (int64_t)(split_ws_floats / ((size_t)M * N * batch)));
   }
+  // an A given without its lo part gets it formed in the kernel (products whose C is not read)
+  const bool cvt = A.lo == nullptr;
+  if (cvt && pre) return cudaErrorInvalidValue;
+  if (B.lo == nullptr) return cudaErrorInvalidValue;
   if (ksplit > 1) {
     const TcEpilogue pe{split_ws, nullptr, N, (int64_t)M * N, nullptr, N, (int64_t)M * N, 0, 1.f, 0.f, ep.status};
-    cudaError_t e = N <= 32 ? tc::launch<32, 5, false>(A, B, M, N, K, batch, pe, s, ksplit)
-                            : tc::launch<128, 3, false>(A, B, M, N, K, batch, pe, s, ksplit);
+    cudaError_t e = N <= 32 ? (cvt ? tc::launch<32, 5, false, true>(A, B, M, N, K, batch, pe, s, ksplit)
+                                   : tc::launch<32, 5, false>(A, B, M, N, K, batch, pe, s, ksplit))
+                            : (cvt ? tc::launch<128, 3, false, true>(A, B, M, N, K, batch, pe, s, ksplit)
+                                   : tc::launch<128, 3, false>(A, B, M, N, K, batch, pe, s, ksplit));
     if (e != cudaSuccess) return e;
     const int64_t n4 = (int64_t)M * N / 4;
     const int blocks = (int)std::min<int64_t>((n4 + 255) / 256, std::max(1, 1216 / batch));
@@ -655,6 +694,9 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
                                                                 ep.c_stride, ep.C_lo);
     return cudaGetLastError();
   }
+  if (cvt)
+    return N <= 32 ? tc::launch<32, 5, false, true>(A, B, M, N, K, batch, ep, s)
+                   : tc::launch<128, 3, false, true>(A, B, M, N, K, batch, ep, s);
   if (N <= 32) return pre ? tc::launch<32, 4, true>(A, B, M, N, K, batch, ep, s)
                           : tc::launch<32, 5, false>(A, B, M, N, K, batch, ep, s);
   return pre ? tc::launch<128, 2, true>(A, B, M, N, K, batch, ep, s)

@@ -513,17 +513,15 @@ __global__ void thresh_kernel(const double* part, float tol, int batch, float* t
   thresh[b] = (float)((double)tol * sqrt(s));
 }
 
-// Q^T <- diag(d) (its lo part is zero: +-1 are tf32 values)
-__global__ void signed_identity_kernel(float* Qt, float* Qt_lo, const float* d, int n) {
+// Q^T <- diag(d)
+__global__ void signed_identity_kernel(float* Qt, const float* d, int n) {
   const int b = blockIdx.y;
   const int64_t nn = (int64_t)n * n;
   float* q = Qt + (int64_t)b * nn;
-  float* ql = Qt_lo + (int64_t)b * nn;
   const float* db = d + (int64_t)b * n;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nn; i += (int64_t)gridDim.x * blockDim.x) {
     const int64_t r = i / n, cc = i % n;
     q[i] = r == cc ? db[r] : 0.f;
-    ql[i] = 0.f;
   }
 }
 
@@ -594,7 +592,7 @@ cudaError_t panel_kernel(PanelKernel* pk) {
 
 struct Workspace {
   float* At;
-  float* At_lo;
+  float* At_lo;   // unused (null): the products form A's lo part themselves
   float* Vt;
   float* Vt_lo;
   float* VTq;     // [batch][nblock][n][NBO] V T of every block (kept for the Q accumulation)
@@ -611,6 +609,13 @@ struct Workspace {
   float* Tt_lo;
   float* Ypart;   // [batch][MAXC][NBO][NB]
   float* Wsplit;  // [KSPLIT][batch][n][NBO] partial sums of split-K products
+  // for the look-ahead schedule only (null otherwise): the far update's own W and split-K
+  // buffers, and a second V T^T buffer (blocks alternate)
+  float* W2;
+  float* W2_lo;
+  float* Wsplit2;
+  float* VTr2;
+  float* VTr2_lo;
   float* thresh;
   float* dsign;
   double* part;
@@ -618,7 +623,7 @@ struct Workspace {
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-Workspace carve(void* base, int n, int batch, size_t* total) {
+Workspace carve(void* base, int n, int batch, size_t* total, bool lookahead) {
   const int nblock = (n + NBO - 1) / NBO;
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -630,21 +635,25 @@ Workspace carve(void* base, int n, int batch, size_t* total) {
   const size_t blocks = (size_t)batch * nblock * n * NBO * sizeof(float);
   const size_t thin = (size_t)batch * n * NBO * sizeof(float);
   const size_t tsq = (size_t)batch * NBO * NBO * sizeof(float);
-  const size_t oAt = take(mat), oAtl = take(mat), oVt = take(mat), oVtl = take(mat);
+  const size_t oAt = take(mat), oVt = take(mat), oVtl = take(mat);
   const size_t oVq = take(blocks), oVql = take(blocks), oVr = take(thin), oVrl = take(thin);
   const size_t oVp = take(thin), oVpl = take(thin), oW = take(thin), oWl = take(thin);
   const size_t oT = take(tsq), oTl = take(tsq), oTt = take(tsq), oTtl = take(tsq);
   const size_t oY = take((size_t)batch * MAXC * NBO * NB * sizeof(float));
   const size_t oWs = take((size_t)KSPLIT * thin);
+  const size_t oW2 = lookahead ? take(thin) : 0, oW2l = lookahead ? take(thin) : 0;
+  const size_t oWs2 = lookahead ? take((size_t)KSPLIT * thin) : 0;
+  const size_t oVr2 = lookahead ? take(thin) : 0, oVr2l = lookahead ? take(thin) : 0;
   const size_t oth = take((size_t)batch * sizeof(float));
   const size_t osg = take((size_t)batch * n * sizeof(float));
   const size_t opart = take((size_t)batch * NORM_CHUNKS * sizeof(double));
   if (total) *total = off;
   char* c = (char*)base;
   auto f = [&](size_t o) { return (float*)(c + o); };
-  return Workspace{f(oAt), f(oAtl), f(oVt), f(oVtl), f(oVq), f(oVql), f(oVr), f(oVrl), f(oVp), f(oVpl),
-                   f(oW),  f(oWl),  f(oT),  f(oTl),  f(oTt), f(oTtl), f(oY),  f(oWs), f(oth),  f(osg),
-                   (double*)(c + opart)};
+  auto g = [&](size_t o) { return lookahead ? (float*)(c + o) : nullptr; };
+  return Workspace{f(oAt), nullptr, f(oVt), f(oVtl), f(oVq), f(oVql), f(oVr), f(oVrl), f(oVp),  f(oVpl),
+                   f(oW),  f(oWl),  f(oT),  f(oTl),  f(oTt), f(oTtl), f(oY),  f(oWs), g(oW2),  g(oW2l),
+                   g(oWs2), g(oVr2), g(oVr2l), f(oth), f(osg), (double*)(c + opart)};
 }
 
 TcOperand op(const float* hi, const float* lo, int64_t ld, int64_t stride, int batch) {
@@ -657,29 +666,28 @@ TcEpilogue out(float* C, float* C_lo, int64_t ldc, int64_t stride, float alpha, 
 
 }  // namespace
 
-size_t qr_workspace_bytes(int n, int batch) {
+size_t qr_workspace_bytes(int n, int batch, bool lookahead) {
   size_t total = 0;
-  carve(nullptr, n, batch, &total);
+  carve(nullptr, n, batch, &total, lookahead);
   return total;
 }
 
-void qr_input_buffers(void* workspace, int n, int batch, float** At, float** At_lo) {
-  Workspace w = carve(workspace, n, batch, nullptr);
+void qr_input_buffers(void* workspace, int n, int batch, float** At) {
+  Workspace w = carve(workspace, n, batch, nullptr, false);  // the input buffer comes first either way
   *At = w.At;
-  *At_lo = w.At_lo;
 }
 
 cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q_lo, uint8_t* skip, float tol,
-                   void* workspace, size_t workspace_bytes, int* status, cudaStream_t s) {
+                   void* workspace, size_t workspace_bytes, int* status, cudaStream_t s, cudaStream_t far,
+                   cudaEvent_t ev_vt, cudaEvent_t ev_far) {
   if (n <= 0 || batch <= 0) return cudaSuccess;
   if (n > 8192 || batch > 65535 || (n & 3)) return cudaErrorInvalidValue;
+  // look-ahead: a second stream and two events given, and a workspace sized for it
+  const bool la = far && ev_vt && ev_far && workspace_bytes >= qr_workspace_bytes(n, batch, true);
   size_t need = 0;
-  Workspace w = carve(workspace, n, batch, &need);
+  Workspace w = carve(workspace, n, batch, &need, la);
   if (workspace_bytes < need) return cudaErrorInvalidValue;
-  if (!Qt) {  // the Q accumulation may reuse the factored matrix's buffers
-    Qt = w.At;
-    Qt_lo = w.At_lo;
-  }
+  if (!Qt) Qt = w.At;  // the Q accumulation may reuse the factored matrix's buffer
   const int nblock = (n + NBO - 1) / NBO;
   const int64_t nn = (int64_t)n * n, thin = (int64_t)n * NBO, vq_stride = (int64_t)nblock * thin;
   cudaError_t e;
@@ -696,6 +704,13 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
   e = panel_kernel(&pk);
   if (e != cudaSuccess) return e;
 
+  if (la) {
+    // the far stream starts after everything enqueued on s so far; ev_far stands for "the
+    // previous far update is done" and starts out recorded
+    e = cudaEventRecord(ev_far, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(far, ev_far, 0);
+    if (e != cudaSuccess) return e;
+  }
   for (int blk = 0; blk < nblock; ++blk) {
     const int k0 = blk * NBO, kbo = std::min(NBO, n - k0), m = n - k0;
     for (int k = k0; k < k0 + kbo; k += NB) {
@@ -724,7 +739,11 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
       }
       if (e != cudaSuccess) return e;
     }
-    // VTq = V T (the Q accumulation) and VTr = V T^T (this block's trailing update)
+    // VTq = V T (the Q accumulation) and VTr = V T^T (this block's trailing update); with the
+    // look-ahead the V T^T buffers alternate between blocks, since the far update of block b
+    // still reads its V T^T while block b+1 forms its own
+    float* vtr = (la && (blk & 1)) ? w.VTr2 : w.VTr;
+    float* vtr_lo = (la && (blk & 1)) ? w.VTr2_lo : w.VTr_lo;
     float* vq = w.VTq + (int64_t)blk * thin + (int64_t)k0 * NBO;
     float* vq_lo = w.VTq_lo + (int64_t)blk * thin + (int64_t)k0 * NBO;
     const TcOperand vpos = op(w.Vpos + (int64_t)k0 * NBO, w.Vpos_lo + (int64_t)k0 * NBO, NBO, thin, batch);
@@ -734,28 +753,52 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     const int nc = n - k0 - kbo;  // trailing rows of At (columns of P)
     if (nc <= 0) continue;
     e = gemm_tc_nt(m, kbo, kbo, batch, vpos, op(w.T, w.T_lo, NBO, NBO * NBO, batch),
-                   out(w.VTr + (int64_t)k0 * NBO, w.VTr_lo + (int64_t)k0 * NBO, NBO, thin, 1.f, 0.f, status), s,
+                   out(vtr + (int64_t)k0 * NBO, vtr_lo + (int64_t)k0 * NBO, NBO, thin, 1.f, 0.f, status), s,
                    kFamQrUpdate);
     if (e != cudaSuccess) return e;
-    // W = At_trail Vt^T over positions k0.. (nc x kbo)
-    const int64_t tr = (int64_t)(k0 + kbo) * n;
-    e = gemm_tc_nt(nc, kbo, m, batch, op(w.At + tr + k0, w.At_lo + tr + k0, n, nn, batch),
-                   op(w.Vt + (int64_t)k0 * n + k0, w.Vt_lo + (int64_t)k0 * n + k0, n, nn, batch),
-                   out(w.W, w.W_lo, NBO, thin, 1.f, 0.f, status), s, kFamQrUpdate, w.Wsplit,
-                   (size_t)KSPLIT * batch * n * NBO);
+    const TcOperand vtr_trail =
+        op(vtr + (int64_t)(k0 + kbo) * NBO, vtr_lo + (int64_t)(k0 + kbo) * NBO, NBO, thin, batch);
+    const TcOperand vt_blk = op(w.Vt + (int64_t)k0 * n + k0, w.Vt_lo + (int64_t)k0 * n + k0, n, nn, batch);
+    // rows [r0, r0 + rows) of the trailing matrix: a_r -= (a_r V) T V^T, i.e.
+    //   W = At_rows Vt^T over positions k0.. ; At_rows -= W VTr^T at positions k0+kbo.. (the
+    //   earlier positions of these rows are R's entries, never read again)
+    auto update_rows = [&](int r0, int rows, float* Wb, float* Wb_lo, float* ws, cudaStream_t st) -> cudaError_t {
+      const int64_t tr = (int64_t)r0 * n;
+      cudaError_t e2 = gemm_tc_nt(rows, kbo, m, batch, op(w.At + tr + k0, nullptr, n, nn, batch), vt_blk,
+                                  out(Wb, Wb_lo, NBO, thin, 1.f, 0.f, status), st, kFamQrUpdate, ws,
+                                  (size_t)KSPLIT * batch * n * NBO);
+      if (e2 != cudaSuccess) return e2;
+      return gemm_tc_nt(rows, nc, kbo, batch, op(Wb, Wb_lo, NBO, thin, batch), vtr_trail,
+                        out(w.At + tr + k0 + kbo, nullptr, n, nn, -1.f, 1.f, status), st,
+                        kFamQrUpdate);
+    };
+    if (!la) {
+      e = update_rows(k0 + kbo, nc, w.W, w.W_lo, w.Wsplit, s);
+      if (e != cudaSuccess) return e;
+      continue;
+    }
+    // look-ahead: the next block's rows now (they gate its panels), the rest on the far stream,
+    // where it overlaps the next block's panels; the next block's rows wait for the previous
+    // far update, which covered them
+    const int knext = std::min(NBO, nc);
+    e = cudaEventRecord(ev_vt, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev_far, 0);
+    if (e == cudaSuccess) e = update_rows(k0 + kbo, knext, w.W, w.W_lo, w.Wsplit, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(far, ev_vt, 0);
+    if (e == cudaSuccess && nc > knext) e = update_rows(k0 + kbo + knext, nc - knext, w.W2, w.W2_lo, w.Wsplit2, far);
+    if (e == cudaSuccess) e = cudaEventRecord(ev_far, far);
     if (e != cudaSuccess) return e;
-    // At_trail -= W VTr^T at positions k0+kbo.. (the earlier positions of these rows are R's)
-    e = gemm_tc_nt(nc, nc, kbo, batch, op(w.W, w.W_lo, NBO, thin, batch),
-                   op(w.VTr + (int64_t)(k0 + kbo) * NBO, w.VTr_lo + (int64_t)(k0 + kbo) * NBO, NBO, thin, batch),
-                   out(w.At + tr + k0 + kbo, w.At_lo + tr + k0 + kbo, n, nn, -1.f, 1.f, status), s, kFamQrUpdate);
+  }
+  if (la) {
+    e = cudaStreamWaitEvent(s, ev_far, 0);  // the last far update before the Q accumulation
     if (e != cudaSuccess) return e;
   }
 
   {
     // Q^T = diag(d) H_n ... H_1 accumulated backwards: start from diag(d)
-    ProfScope prof(kFamOther, 0, 8.0 * nn * batch, s);
+    ProfScope prof(kFamOther, 0, 4.0 * nn * batch, s);
     const int blocks = (int)std::min<int64_t>((nn + 255) / 256, 1024);
-    signed_identity_kernel<<<dim3(blocks, batch), 256, 0, s>>>(Qt, Qt_lo, w.dsign, n);
+    signed_identity_kernel<<<dim3(blocks, batch), 256, 0, s>>>(Qt, w.dsign, n);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -763,7 +806,7 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     const int k0 = blk * NBO, kbo = std::min(NBO, n - k0), m = n - k0;
     const int64_t sub = (int64_t)k0 * n + k0;
     // W = Qt_sub Vt^T  (m x kbo)
-    e = gemm_tc_nt(m, kbo, m, batch, op(Qt + sub, Qt_lo + sub, n, nn, batch),
+    e = gemm_tc_nt(m, kbo, m, batch, op(Qt + sub, nullptr, n, nn, batch),
                    op(w.Vt + sub, w.Vt_lo + sub, n, nn, batch), out(w.W, w.W_lo, NBO, thin, 1.f, 0.f, status), s,
                    kFamQrUpdate, w.Wsplit, (size_t)KSPLIT * batch * n * NBO);
     if (e != cudaSuccess) return e;
@@ -771,7 +814,7 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     const int64_t vq = (int64_t)blk * thin + (int64_t)k0 * NBO;
     e = gemm_tc_nt(m, m, kbo, batch, op(w.W, w.W_lo, NBO, thin, batch),
                    op(w.VTq + vq, w.VTq_lo + vq, NBO, vq_stride, batch),
-                   out(Qt + sub, Qt_lo + sub, n, nn, -1.f, 1.f, status), s, kFamQrUpdate);
+                   out(Qt + sub, nullptr, n, nn, -1.f, 1.f, status), s, kFamQrUpdate);
     if (e != cudaSuccess) return e;
   }
   if (Q) {
@@ -788,12 +831,13 @@ cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, floa
                  size_t workspace_bytes, int* status, cudaStream_t s) {
   if (n <= 0 || batch <= 0) return cudaSuccess;
   size_t need = 0;
-  Workspace w = carve(workspace, n, batch, &need);
+  Workspace w = carve(workspace, n, batch, &need, false);
   if (workspace_bytes < need || (n & 3)) return cudaErrorInvalidValue;
   // At = P^T and its lo part
-  cudaError_t e = basis_split(P, nullptr, w.At, w.At_lo, n, batch, s);
+  cudaError_t e = transpose(P, w.At, n, n, batch, s);
   if (e != cudaSuccess) return e;
-  return qr_q_t(n, batch, nullptr, nullptr, Q, nullptr, skip, tol, workspace, workspace_bytes, status, s);
+  return qr_q_t(n, batch, nullptr, nullptr, Q, nullptr, skip, tol, workspace, workspace_bytes, status, s, nullptr,
+                nullptr, nullptr);
 }
 
 }  // namespace soap

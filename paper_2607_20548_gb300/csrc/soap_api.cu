@@ -14,6 +14,7 @@
 //   G' = X1 Q_R, m = X2 Q_R
 //   v <- b2 v + (1-b2) G'^2, N = m / (sqrt(v) + eps)        S6
 //   X1 = Q_L N; W <- (1 - lr wd) W - lr X1 Q_R^T           S7, S8 (fused in the GEMM epilogue)
+#include <algorithm>
 #include <cstdio>
 #include <cstring>
 #include <map>
@@ -76,7 +77,9 @@ struct QrGroup {
   void* ws = nullptr;
   size_t ws_bytes = 0;
   uint8_t* skip = nullptr;  // [batch][n]
-  cudaStream_t stream = nullptr;
+  cudaStream_t stream = nullptr;  // panels and the rows that gate them (high priority)
+  cudaStream_t far = nullptr;     // the rest of each block's trailing update (low priority)
+  cudaEvent_t ev_vt = nullptr, ev_far = nullptr;
   cudaEvent_t done = nullptr;
 };
 
@@ -177,9 +180,12 @@ void free_all(soap_handle h) {
   h->fork_ev = nullptr;
   for (auto& g : h->groups) {
     if (g.stream) cudaStreamDestroy(g.stream);
+    if (g.far) cudaStreamDestroy(g.far);
     if (g.done) cudaEventDestroy(g.done);
-    g.stream = nullptr;
-    g.done = nullptr;
+    if (g.ev_vt) cudaEventDestroy(g.ev_vt);
+    if (g.ev_far) cudaEventDestroy(g.ev_far);
+    g.stream = g.far = nullptr;
+    g.done = g.ev_vt = g.ev_far = nullptr;
   }
   h->h_status = nullptr;
   h->h_ptrs = nullptr;
@@ -260,37 +266,34 @@ soap_status_t refresh_bases(soap_handle h, cudaStream_t s) {
     SOAP_CUDA(h, cudaStreamWaitEvent(gs, h->fork_ev, 0));
     const int n = g.n;
     const int64_t nn = (int64_t)n * n;
-    float *At, *At_lo;
-    soap::qr_input_buffers(g.ws, n, g.batch, &At, &At_lo);
+    float* At;
+    soap::qr_input_buffers(g.ws, n, g.batch, &At);
     for (const QrJob& j : g.jobs) {
       ClassState& c = h->classes[j.cls];
       float* F = j.left ? c.L : c.R;
       float* at = At + (int64_t)j.offset * nn;
-      float* at_lo = At_lo + (int64_t)j.offset * nn;
       if (c.tc) {
         SOAP_CUDA(h, soap::gemm_tc_nt(n, n, n, c.count, opnd(j.left ? c.QLt : c.QRt, j.left ? c.QLt_lo : c.QRt_lo, n, nn,
                                                              c.count),
                                       opnd(F, j.left ? c.L_lo : c.R_lo, n, nn, c.count),
-                                      epi(h, at, n, nn, at_lo, 0, 1.f, 0.f), gs));
+                                      epi(h, at, n, nn, nullptr, 0, 1.f, 0.f), gs));
       } else {
         SOAP_CUDA(h, soap::gemm(true, false, n, n, n, 1.f, strided(j.left ? c.QL : c.QR, n, nn), strided(F, n, nn), 0.f,
                                 strided_mut(at, n, nn), c.count, gs));
-        SOAP_CUDA(h, soap::split_tf32(at, nullptr, at_lo, (int64_t)c.count * nn, gs));
       }
     }
     // the Q accumulation ends with Q^T and its lo part in the input buffers
     SOAP_CUDA(h, soap::qr_q_t(n, g.batch, nullptr, nullptr, nullptr, nullptr, g.skip, hp.qr_tol, g.ws, g.ws_bytes,
-                              h->d_status, gs));
+                              h->d_status, gs, g.far, g.ev_vt, g.ev_far));
     for (const QrJob& j : g.jobs) {
       ClassState& c = h->classes[j.cls];
       const float* qt = At + (int64_t)j.offset * nn;
-      const float* qt_lo = At_lo + (int64_t)j.offset * nn;
       float* Q = j.left ? c.QL : c.QR;
       if (c.tc)
-        SOAP_CUDA(h, soap::basis_from_qt(qt, qt_lo, j.left ? c.QLt : c.QRt, j.left ? c.QLt_lo : c.QRt_lo, Q,
+        SOAP_CUDA(h, soap::basis_from_qt(qt, nullptr, j.left ? c.QLt : c.QRt, j.left ? c.QLt_lo : c.QRt_lo, Q,
                                          j.left ? c.QL_lo : c.QR_lo, n, c.count, gs));
       else
-        SOAP_CUDA(h, soap::basis_from_qt(qt, qt_lo, nullptr, nullptr, Q, nullptr, n, c.count, gs));
+        SOAP_CUDA(h, soap::basis_from_qt(qt, nullptr, nullptr, nullptr, Q, nullptr, n, c.count, gs));
       SOAP_CUDA(h, cudaMemcpyAsync(j.left ? c.skipL : c.skipR, g.skip + (int64_t)j.offset * n, (size_t)c.count * n,
                                    cudaMemcpyDeviceToDevice, gs));
     }
@@ -546,11 +549,17 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
     }
     for (auto& g : h->groups) {
       if (g.batch > 65535) e = cudaErrorInvalidValue;
-      g.ws_bytes = soap::qr_workspace_bytes(g.n, g.batch);
+      g.ws_bytes = soap::qr_workspace_bytes(g.n, g.batch, true);
       if (e == cudaSuccess) e = dalloc(h, &g.ws, g.ws_bytes);
       if (e == cudaSuccess) e = dalloc(h, (void**)&g.skip, (size_t)g.batch * g.n);
-      if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&g.stream, cudaStreamNonBlocking);
+      // the panel chain is latency-bound: its stream goes first when SMs free up
+      int prio_lo = 0, prio_hi = 0;
+      if (e == cudaSuccess) e = cudaDeviceGetStreamPriorityRange(&prio_lo, &prio_hi);
+      if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&g.stream, cudaStreamNonBlocking, prio_hi);
+      if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&g.far, cudaStreamNonBlocking, prio_lo);
       if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.done, cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.ev_vt, cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.ev_far, cudaEventDisableTiming);
     }
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->fork_ev, cudaEventDisableTiming);
   }
@@ -915,6 +924,22 @@ soap_status_t soap_profile_end(soap_handle h, soap_stream_t stream, soap_kernel_
   }
   if (overflow) *overflow = p.overflow ? 1 : 0;
   h->prof.recs.clear();
+  return SOAP_OK;
+}
+
+soap_status_t soap_profile_records(soap_handle h, soap_launch_record* out, int64_t max, int64_t* count) {
+  if (!h || !count || max < 0 || (max > 0 && !out)) return SOAP_ERR_INVALID_ARG;
+  DeviceGuard g(h->device);
+  SOAP_CUDA(h, cudaDeviceSynchronize());
+  const soap::Profiler& p = h->prof;
+  const int64_t n = std::min<int64_t>(max, (int64_t)p.recs.size());
+  for (int64_t i = 0; i < n; ++i) {
+    float t0 = 0.f, t1 = 0.f;
+    SOAP_CUDA(h, cudaEventElapsedTime(&t0, p.events[0], p.events[2 * i]));
+    SOAP_CUDA(h, cudaEventElapsedTime(&t1, p.events[0], p.events[2 * i + 1]));
+    out[i] = soap_launch_record{p.recs[i].family, (double)t0, (double)t1};
+  }
+  *count = n;
   return SOAP_OK;
 }
 

@@ -81,18 +81,23 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
 cudaError_t split_tf32(const float* x, float* hi, float* lo, int64_t n, cudaStream_t stream);
 
 // Householder QR (explicit Q) of `batch` contiguous n x n matrices (n a multiple of 4).
-size_t qr_workspace_bytes(int n, int batch);
+// Workspace of qr_q / qr_q_t; `lookahead` adds the buffers of the two-stream schedule.
+size_t qr_workspace_bytes(int n, int batch, bool lookahead = false);
 // P read only; Q written. Uses the tensor-core QR on P^T (staged in the workspace).
 cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, float tol,
                  void* workspace, size_t workspace_bytes, int* status, cudaStream_t stream);
-// Where the factored matrix P^T and its tf32 lo part must be placed before qr_q_t.
-void qr_input_buffers(void* workspace, int n, int batch, float** At, float** At_lo);
-// QR of P whose transpose (and lo part) is already in qr_input_buffers(). Writes Q^T and its
-// lo part into Qt/Qt_lo (or, if Qt is nullptr, into the workspace) and, if Q is given, Q and
-// (if Q_lo is given) its lo part.
+// Where the factored matrix P^T must be placed before qr_q_t.
+void qr_input_buffers(void* workspace, int n, int batch, float** At);
+// QR of P whose transpose is already in qr_input_buffers(). Writes Q^T into Qt (or, if Qt is
+// nullptr, into the workspace) and, if Q is given, Q and (if Q_lo is given) its lo part.
+// Qt_lo is not written.
+// With `far`, ev_vt and ev_far (and a workspace sized with lookahead) the trailing update of
+// each 128-column block, except the next block's rows, runs on `far` and overlaps the next
+// block's panels; everything is joined back on `stream` before return.
 cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q_lo, uint8_t* skip,
                    float tol, void* workspace, size_t workspace_bytes, int* status,
-                   cudaStream_t stream);
+                   cudaStream_t stream, cudaStream_t far = nullptr, cudaEvent_t ev_vt = nullptr,
+                   cudaEvent_t ev_far = nullptr);
 
 // Elementwise kernels of the step.
 // M_hat <- b1 M_hat + (1-b1) G and Gc <- G for each matrix of a class.
@@ -112,7 +117,8 @@ cudaError_t momentum_split(const float* const* grads, float* Gn, float* Gn_lo, f
                            bool mhat_transposed, int* status, cudaStream_t stream);
 // dst_b = src_b^T for `batch` contiguous rows x cols matrices.
 cudaError_t transpose(const float* src, float* dst, int rows, int cols, int batch, cudaStream_t stream);
-// From Q^T and its lo part: copies of both and Q with its lo part (any output may be null).
+// From Q^T: a copy of it with its lo part, and Q with its lo part (any output may be null;
+// the lo parts are formed from the values, Qt_lo is not read).
 cudaError_t basis_from_qt(const float* Qt, const float* Qt_lo, float* Qt_out, float* Qt_lo_out, float* Q,
                           float* Q_lo, int n, int batch, cudaStream_t stream);
 // Q -> lo part, Q^T, lo part of Q^T for `batch` n x n bases.

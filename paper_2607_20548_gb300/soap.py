@@ -25,7 +25,8 @@ STATE_M, STATE_V, STATE_L, STATE_QL, STATE_R, STATE_QR, STATE_MHAT, STATE_SKIP_L
 EXPORTS = ("soap_default_hparams", "soap_create", "soap_step", "soap_set_lr", "soap_state_bytes",
            "soap_state_get", "soap_state_set", "soap_get_step", "soap_set_step", "soap_status",
            "soap_clear_status", "soap_last_error", "soap_destroy", "soap_qr_workspace_bytes",
-           "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_gemm_tf32x4",
+           "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_profile_records",
+           "soap_gemm_tf32x4",
            "soap_split_tf32", "soap_qr_static")
 KERNEL_FAMILIES = ("gemm_simt", "gemm_tc", "qr_panel", "elementwise", "other", "qr_update")
 
@@ -46,6 +47,10 @@ class soap_hparams(ctypes.Structure):
 class soap_kernel_stats(ctypes.Structure):
     _fields_ = [("family", ctypes.c_int32), ("launches", ctypes.c_int64), ("ms", ctypes.c_double),
                 ("flops", ctypes.c_double), ("bytes", ctypes.c_double)]
+
+
+class soap_launch_record(ctypes.Structure):
+    _fields_ = [("family", ctypes.c_int32), ("start_ms", ctypes.c_double), ("end_ms", ctypes.c_double)]
 
 
 class SoapError(RuntimeError):
@@ -84,6 +89,7 @@ def load_library(path: str = LIB_PATH):
         "soap_qr": (I32, [I32, I32, P, P, P, F, P, SZ, P]),
         "soap_profile_begin": (I32, [P, I64]),
         "soap_profile_end": (I32, [P, P, ctypes.POINTER(soap_kernel_stats), ctypes.POINTER(I32)]),
+        "soap_profile_records": (I32, [P, ctypes.POINTER(soap_launch_record), I64, ctypes.POINTER(I64)]),
         "soap_gemm": (I32, [I32, I32, I32, I32, I32, F, P, I64, I64, P, I64, I64, F, P, I64, I64, I32, P]),
         "soap_gemm_tf32x4": (I32, [I32, I32, I32, I32, P, P, I64, I64, P, P, I64, I64, I32, F, F, P, I64, I64,
                                    I32, P, P, P]),
@@ -218,6 +224,14 @@ class SoapOptimizer:
                for o in out}
         res["overflow"] = bool(ov.value)
         return res
+
+    def profile_records(self, max_records=1 << 20) -> list:
+        """The launches timed since profile_begin as (family, start_ms, end_ms), in launch order
+        (call before profile_end)."""
+        out = (soap_launch_record * max_records)()
+        cnt = ctypes.c_int64(0)
+        _check(load_library().soap_profile_records(self._handle(), out, max_records, ctypes.byref(cnt)), self._h)
+        return [(KERNEL_FAMILIES[out[i].family], out[i].start_ms, out[i].end_ms) for i in range(cnt.value)]
 
     def last_error(self) -> str:
         return load_library().soap_last_error(self._handle()).decode()
