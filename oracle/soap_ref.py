@@ -130,6 +130,7 @@ class HParams:
     bias_correction: bool = False
     guard: bool = True
     qr_tol: float = 1e-4
+    kl: bool = False              # KL-Shampoo factor form (Alg. 1's "Accumulate Kronecker Factors")
 
 
 @dataclass
@@ -174,6 +175,38 @@ class MatrixState:
 
 
 # ---- sub-steps, each a plain transcription of one line group of Alg. 1 ----------
+
+def approx_eigenvalues(F: np.ndarray, Q: np.ndarray) -> np.ndarray:
+    """lambda = diag(Q^T F Q): Alg. 1's approximate eigenvalues of a factor in its current basis."""
+    return np.diag(Q.T @ F @ Q).copy()
+
+
+def factor_ema_kl(st: "MatrixState", G: np.ndarray, b: float, eps: float):
+    """KL-Shampoo factor EMAs (Alg. 1, "Accumulate Kronecker Factors (KL-Shampoo)"; section
+    on the SVD view of KL-Shampoo):
+
+        L <- b L + (1-b)/out * G S_R^-1 G^T,   R <- b R + (1-b)/in * G^T S_L^-1 G,
+
+    with S^-1 = Q diag(1/(lambda + eps)) Q^T, lambda = diag(Q^T F Q) taken from the factors and
+    bases before this step's update (the exponent is read as -1, the inverse of the other
+    factor; beta weights the old state as in the standard form). A side without a factor
+    (identity side) counts as S = I, i.e. lambda = 1 and Q = I. Returns (L_new, R_new)."""
+    rows, cols = G.shape
+    d = G.dtype.type
+    if st.right:
+        wR = 1.0 / (approx_eigenvalues(st.R, st.QR) + eps)
+        SR_inv = st.QR @ np.diag(wR) @ st.QR.T
+    else:
+        SR_inv = np.eye(cols, dtype=G.dtype) / d(1.0 + eps)
+    if st.left:
+        wL = 1.0 / (approx_eigenvalues(st.L, st.QL) + eps)
+        SL_inv = st.QL @ np.diag(wL) @ st.QL.T
+    else:
+        SL_inv = np.eye(rows, dtype=G.dtype) / d(1.0 + eps)
+    L = b * st.L + (1 - b) / cols * (G @ SR_inv @ G.T) if st.left else None
+    R = b * st.R + (1 - b) / rows * (G.T @ SL_inv @ G) if st.right else None
+    return L, R
+
 
 def factor_ema(F: np.ndarray, G: np.ndarray, b: float, side: str) -> np.ndarray:
     """S1: L <- b L + (1-b) G G^T (side 'L') or R <- b R + (1-b) G^T G (side 'R').
@@ -239,10 +272,17 @@ def soap_step(st: MatrixState, W: np.ndarray, G: np.ndarray, hp: HParams,
     st.t += 1
     t = st.t
     # S1: accumulate the Kronecker factors with the current gradient
-    if st.left:
-        st.L = factor_ema(st.L, G, hp.factor_beta, "L")
-    if st.right:
-        st.R = factor_ema(st.R, G, hp.factor_beta, "R")
+    if hp.kl:
+        L, R = factor_ema_kl(st, G, d(hp.factor_beta), d(hp.eps))
+        if st.left:
+            st.L = L
+        if st.right:
+            st.R = R
+    else:
+        if st.left:
+            st.L = factor_ema(st.L, G, hp.factor_beta, "L")
+        if st.right:
+            st.R = factor_ema(st.R, G, hp.factor_beta, "R")
     # S2-S4: eigenbasis re-computation every F steps
     if t % hp.eig_every == 0:
         M_hat = rotate_out(st.QL if st.left else None, st.m, st.QR if st.right else None)

@@ -245,3 +245,80 @@ def test_first_step_of_rectangular_matrix_is_null_space_free():
     assert st.skipR.sum() == 4
     assert np.abs(G @ st.QR[:, st.skipR]).max() < 1e-12
     assert np.abs(G @ st.QR[:, ~st.skipR]).min(axis=0).max() > 1e-3
+
+
+# ---- KL-Shampoo factor form (Alg. 1 "Accumulate Kronecker Factors (KL-Shampoo)") ----------
+
+def test_kl_first_step_closed_form():
+    """From L = R = 0 and Q = I every approximate eigenvalue is 0, so the first KL update is
+    the standard one scaled by 1/((in or out) * eps)."""
+    rng = np.random.default_rng(31)
+    rows, cols = 6, 9
+    G = rng.standard_normal((rows, cols))
+    hp = HParams(kl=True, eps=1e-3)
+    st = MatrixState(rows, cols, True, True)
+    soap_step(st, np.zeros((rows, cols)), G, hp)
+    b = hp.factor_beta
+    L_expect = (1 - b) / (cols * hp.eps) * np.einsum("ik,jk->ij", G, G)
+    R_expect = (1 - b) / (rows * hp.eps) * np.einsum("ki,kj->ij", G, G)
+    np.testing.assert_allclose(st.L, L_expect, rtol=1e-12)
+    np.testing.assert_allclose(st.R, R_expect, rtol=1e-12)
+
+
+def test_kl_update_uses_the_regularised_inverse_of_the_other_factor():
+    """When the basis diagonalises the other factor exactly, Q diag(1/(lambda + eps)) Q^T is
+    (F + eps I)^-1, so the KL update equals b L + (1-b)/out G (R + eps I)^-1 G^T computed with
+    a library inverse (and likewise for R)."""
+    rng = np.random.default_rng(32)
+    rows, cols = 5, 7
+    G = rng.standard_normal((rows, cols))
+    QL = np.linalg.qr(rng.standard_normal((rows, rows)))[0]
+    QR = np.linalg.qr(rng.standard_normal((cols, cols)))[0]
+    muL = rng.uniform(0.5, 2.0, rows)
+    muR = rng.uniform(0.5, 2.0, cols)
+    st = MatrixState(rows, cols, True, True)
+    st.L, st.QL = QL @ np.diag(muL) @ QL.T, QL
+    st.R, st.QR = QR @ np.diag(muR) @ QR.T, QR
+    L0, R0 = st.L.copy(), st.R.copy()
+    from oracle.soap_ref import factor_ema_kl
+    b, eps = 0.9, 0.05
+    L, R = factor_ema_kl(st, G, b, eps)
+    L_expect = b * L0 + (1 - b) / cols * G @ np.linalg.inv(R0 + eps * np.eye(cols)) @ G.T
+    R_expect = b * R0 + (1 - b) / rows * G.T @ np.linalg.inv(L0 + eps * np.eye(rows)) @ G
+    np.testing.assert_allclose(L, L_expect, rtol=1e-10)
+    np.testing.assert_allclose(R, R_expect, rtol=1e-10)
+
+
+def test_kl_identity_side_counts_as_identity_factor():
+    """A one-sided matrix: the missing factor is S = I (lambda = 1)."""
+    rng = np.random.default_rng(33)
+    rows, cols = 4, 6
+    G = rng.standard_normal((rows, cols))
+    st = MatrixState(rows, cols, True, False)
+    from oracle.soap_ref import factor_ema_kl
+    L, R = factor_ema_kl(st, G, 0.9, 1e-3)
+    assert R is None
+    np.testing.assert_allclose(L, 0.1 / cols / (1 + 1e-3) * G @ G.T, rtol=1e-12)
+
+
+def test_kl_factors_track_singular_values_at_the_fixed_point():
+    """The appendix's fixed point: for a constant square gradient G = U diag(s) V^T and balanced
+    factors, KL-Shampoo's factor eigenvalues settle at s / sqrt(n) (with the 1/out and 1/in
+    scalings), not at s^2 / n as Shampoo's do, so kappa(L_KL) = sqrt(kappa(L_Shampoo))."""
+    rng = np.random.default_rng(34)
+    n = 6
+    U = np.linalg.qr(rng.standard_normal((n, n)))[0]
+    V = np.linalg.qr(rng.standard_normal((n, n)))[0]
+    s = np.array([4.0, 2.5, 1.5, 1.0, 0.6, 0.3])
+    G = U @ np.diag(s) @ V.T
+    hp = HParams(kl=True, factor_beta=0.5, eps=1e-8, lr=0.0, weight_decay=0.0)
+    st = MatrixState(n, n, True, True)
+    for _ in range(120):
+        soap_step(st, np.zeros((n, n)), G, hp)
+    evL = np.sort(np.linalg.eigvalsh(st.L))[::-1]
+    evR = np.sort(np.linalg.eigvalsh(st.R))[::-1]
+    np.testing.assert_allclose(evL, s / np.sqrt(n), rtol=1e-6)
+    np.testing.assert_allclose(evR, s / np.sqrt(n), rtol=1e-6)
+    kappa_kl = evL[0] / evL[-1]
+    kappa_shampoo = (s[0] / s[-1]) ** 2
+    assert abs(kappa_kl - np.sqrt(kappa_shampoo)) < 1e-5 * kappa_kl
