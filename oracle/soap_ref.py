@@ -190,16 +190,19 @@ def factor_ema_kl(st: "MatrixState", G: np.ndarray, b: float, eps: float):
     with S^-1 = Q diag(1/(lambda + eps)) Q^T, lambda = diag(Q^T F Q) taken from the factors and
     bases before this step's update (the exponent is read as -1, the inverse of the other
     factor; beta weights the old state as in the standard form). A side without a factor
-    (identity side) counts as S = I, i.e. lambda = 1 and Q = I. Returns (L_new, R_new)."""
+    (identity side) counts as S = I, i.e. lambda = 1 and Q = I. The factor is positive
+    semi-definite, so lambda >= 0 in exact arithmetic; a lambda that rounding made negative is
+    taken as 0, which keeps every weight 1/(lambda + eps) positive and finite for eps > 0.
+    Returns (L_new, R_new)."""
     rows, cols = G.shape
     d = G.dtype.type
     if st.right:
-        wR = 1.0 / (approx_eigenvalues(st.R, st.QR) + eps)
+        wR = 1.0 / (np.maximum(approx_eigenvalues(st.R, st.QR), 0) + eps)
         SR_inv = st.QR @ np.diag(wR) @ st.QR.T
     else:
         SR_inv = np.eye(cols, dtype=G.dtype) / d(1.0 + eps)
     if st.left:
-        wL = 1.0 / (approx_eigenvalues(st.L, st.QL) + eps)
+        wL = 1.0 / (np.maximum(approx_eigenvalues(st.L, st.QL), 0) + eps)
         SL_inv = st.QL @ np.diag(wL) @ st.QL.T
     else:
         SL_inv = np.eye(rows, dtype=G.dtype) / d(1.0 + eps)

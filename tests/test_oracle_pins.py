@@ -322,3 +322,26 @@ def test_kl_factors_track_singular_values_at_the_fixed_point():
     kappa_kl = evL[0] / evL[-1]
     kappa_shampoo = (s[0] / s[-1]) ** 2
     assert abs(kappa_kl - np.sqrt(kappa_shampoo)) < 1e-5 * kappa_kl
+
+
+def test_kl_rounding_negative_eigenvalue_counts_as_zero():
+    """lambda = diag(Q^T F Q) of a positive semi-definite factor is >= 0; a value that rounding
+    pushed below 0 is read as 0, so the weight there is 1/eps (positive, finite) rather than a
+    negative or unbounded 1/(lambda + eps). Checked against the closed form with F's null
+    direction given weight 1/eps and the others 1/(mu + eps)."""
+    rng = np.random.default_rng(35)
+    rows, cols = 4, 5
+    G = rng.standard_normal((rows, cols))
+    QR = np.linalg.qr(rng.standard_normal((cols, cols)))[0]
+    mu = np.array([3.0, 1.0, 0.5, 0.25, -1e-9])  # the last: a rounding artefact of a null direction
+    st = MatrixState(rows, cols, False, True)
+    st.R, st.QR = QR @ np.diag(mu) @ QR.T, QR
+    st2 = MatrixState(rows, cols, True, True)
+    st2.R, st2.QR = st.R, QR
+    from oracle.soap_ref import factor_ema_kl
+    eps = 1e-8
+    L, _ = factor_ema_kl(st2, G, 0.5, eps)
+    w = 1.0 / (np.array([3.0, 1.0, 0.5, 0.25, 0.0]) + eps)
+    L_expect = 0.5 / cols * G @ QR @ np.diag(w) @ QR.T @ G.T
+    np.testing.assert_allclose(L, L_expect, rtol=1e-9)
+    assert np.all(np.linalg.eigvalsh(L) > -1e-6 * np.abs(L).max())
