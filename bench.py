@@ -8,11 +8,12 @@ all 7 matrices. Metric: SOAP steps/s for the whole block, plus effective TFLOP/s
 fixed FLOP model of Alg. 1 (S1 as a SYRK, S2 power step, S3 Householder QR with explicit
 Q, S4 re-projection with four two-sided products, S5/S7 rotations).
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {soap,reference}]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {soap,reference}] [--kl]
 
 N > 1 (torchrun, one rank per GPU) runs N independent replicas of the block: the step
 has no exchange, so value = N * K / max-over-ranks time. --impl reference times the
-fp64 CPU oracle on the host cores instead (rank 0 only).
+fp64 CPU oracle on the host cores instead (rank 0 only). --kl runs Alg. 1's KL-Shampoo
+factor form instead of the standard factor EMAs (a separate line, not the headline).
 """
 from __future__ import annotations
 
@@ -37,10 +38,14 @@ METRIC = "SOAP steps/sec per model + effective TFLOP/s (fraction of dense peak)"
 FP32_SIMT_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 
 
-def model_flops(rows, cols, left, right) -> float:
-    """FLOPs of one literal Alg. 1 step for one matrix (2 per multiply-add)."""
+def model_flops(rows, cols, left, right, kl=False) -> float:
+    """FLOPs of one literal Alg. 1 step for one matrix (2 per multiply-add). The KL-Shampoo
+    factor form of a two-sided matrix adds lambda = diag(Q^T F Q) for both factors (Q^T F)
+    and the rotations G Q_R, G^T Q_L that its weighted EMA terms are built from."""
     m, n = float(rows), float(cols)
     f = 0.0
+    if kl and left and right:
+        f += 2 * m ** 3 + 2 * n ** 3 + 2 * m * n * n + 2 * n * m * m
     if left:
         f += m * m * n + 2 * m ** 3 + (8.0 / 3.0) * m ** 3      # S1 (SYRK), S2, S3
     if right:
@@ -161,7 +166,7 @@ def roofline(family, st, peaks, peak_src):
                 peak_source=peak_src)
 
 
-def oracle_sample(steps: int, warmup: int):
+def oracle_sample(steps: int, warmup: int, kl: bool = False):
     """Times the fp64 oracle's SOAP step on Wq (2048x2048) of the block, on the host cores.
     Returns (seconds per sampled step, block steps/s extrapolated by the FLOP model, threads)."""
     from oracle.soap_ref import HParams, MatrixState, soap_step
@@ -171,7 +176,7 @@ def oracle_sample(steps: int, warmup: int):
     stream = make_stream(WORKLOAD, seed=0, device="cpu", specs=[0])
     W = stream.weights()[0][0].numpy().astype(np.float64)
     st = MatrixState(2048, 2048, True, True, np.float64)
-    hp = HParams()
+    hp = HParams(kl=kl)
     times = []
     for t in range(1, steps + warmup + 1):
         G = stream.grads(t)[0][0].numpy()
@@ -180,8 +185,8 @@ def oracle_sample(steps: int, warmup: int):
         if t > warmup:
             times.append(time.perf_counter() - t0)
     per = float(np.mean(times))
-    block = sum(model_flops(s.rows, s.cols, s.left, s.right) for s in specs)
-    scale = block / model_flops(2048, 2048, True, True)
+    block = sum(model_flops(s.rows, s.cols, s.left, s.right, kl) for s in specs)
+    scale = block / model_flops(2048, 2048, True, True, kl)
     threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
     return per, 1.0 / (per * scale), threads, scale
 
@@ -220,7 +225,8 @@ def run_soap(args):
     if subset:
         specs = [specs[j] for j in subset]
     gen = make_stream(WORKLOAD, seed=rank, device=dev, specs=subset)
-    opt = SoapOptimizer([(s.rows, s.cols, s.left, s.right) for s in specs], default_hparams(), device=local)
+    opt = SoapOptimizer([(s.rows, s.cols, s.left, s.right) for s in specs], default_hparams(kl=int(args.kl)),
+                        device=local)
 
     def flat(tensors):
         out = [None] * len(specs)
@@ -299,14 +305,14 @@ def run_soap(args):
     if rank != 0:
         opt.destroy()
         return
-    block_flops = sum(model_flops(s.rows, s.cols, s.left, s.right) for s in specs)
+    block_flops = sum(model_flops(s.rows, s.cols, s.left, s.right, args.kl) for s in specs)
     peaks, peak_src = measured_peaks()
     fams = {k: v for k, v in prof.items() if k != "overflow"}
     top = max(fams, key=lambda k: fams[k]["ms"])
     st = fams[top]
     launches = sum(v["launches"] for v in fams.values())
     roof = roofline(top, st, peaks, peak_src)
-    per, sps, threads, scale = oracle_sample(1, 0)
+    per, sps, threads, scale = oracle_sample(1, 0, args.kl)
     line = {
         "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True,
@@ -315,6 +321,7 @@ def run_soap(args):
                    "matrices": len(specs),
                    "shapes": "4x 2048x2048, 2x 2048x8192, 1x 8192x2048, all sides preconditioned",
                    "parallelism": "replicas" if world > 1 else "single",
+                   "factor_form": "kl" if args.kl else "standard",
                    "l2": "inputs larger than L2 (3 GB of optimizer state per step)"},
         "effective_tflops": block_flops * value / world / 1e12,
         "effective_frac_of_tensor_fp32_peak": block_flops * value / world / 1e12 /
@@ -348,6 +355,8 @@ def main():
     ap.add_argument("--matrices", default="",
                     help="comma-separated matrix indices of the block to run (a smaller case for profiling); "
                          "default: all 7")
+    ap.add_argument("--kl", action="store_true",
+                    help="KL-Shampoo factor form (Alg. 1's factor accumulation) instead of the standard EMAs")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)

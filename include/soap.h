@@ -62,24 +62,32 @@ typedef struct {
  *   bias_correction:  0 = literal Alg. 1 (none); 1 = divide m, v by (1 - beta^t)
  *   qr_tol:           a Householder column whose remaining norm is <= qr_tol*||P||_F
  *                     is treated as exactly zero (no reflector, R_kk = 0, sign +1)
- *   guard:            1 = rows/cols of N that belong to such zero columns are 0 */
+ *   guard:            1 = rows/cols of N that belong to such zero columns are 0
+ *   kl:               0 = standard Shampoo factor EMAs (above); 1 = Alg. 1's KL-Shampoo form
+ *                       L <- b L + (1-b)/cols * G Q_R diag(1/(lam_R + eps)) Q_R^T G^T
+ *                       R <- b R + (1-b)/rows * G^T Q_L diag(1/(lam_L + eps)) Q_L^T G
+ *                     with lam = diag(Q^T F Q) from the factor and basis held before the
+ *                     step (a negative lam, which only rounding produces, counts as 0); an
+ *                     identity side counts as Q = I, lam = 1. Requires eps > 0. */
 typedef struct {
   float lr, beta1, beta2, factor_beta, eps, weight_decay;
   int32_t eig_every;
   int32_t bias_correction;
   float qr_tol;
   int32_t guard;
+  int32_t kl;
 } soap_hparams;
 
 /* Fills *hp with the defaults used for the paper's workloads: lr 3e-3,
  * beta1 = beta2 = factor_beta = 0.95, eps 1e-8, weight_decay 0.1, F = 1, no bias
- * correction, qr_tol 1e-4, guard on. */
+ * correction, qr_tol 1e-4, guard on, standard factor EMAs (kl 0). */
 void soap_default_hparams(soap_hparams* hp);
 
 /* Creates the optimizer for n matrices on CUDA device `device` and allocates all
  * state (Alg. 1 "Optimizer States") and workspace up front: L = R = 0, Q = I,
  * m = v = 0, t = 0. shapes[] is copied. Returns SOAP_ERR_OOM if the state does
- * not fit; *out is then NULL. The device becomes current for the calling thread. */
+ * not fit; *out is then NULL; SOAP_ERR_INVALID_ARG for kl = 1 with eps <= 0 (the first
+ * KL step weighs by 1/eps). The device becomes current for the calling thread. */
 soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparams* hp,
                           int32_t device, soap_handle* out);
 
@@ -108,7 +116,11 @@ typedef enum {
   SOAP_STATE_MHAT = 6,  /* first moment in the original basis, Q_L m Q_R^T (rows x cols);
                            the library's own storage, bit-exact for checkpoints */
   SOAP_STATE_SKIP_L = 7,/* uint8 per row: 1 where Q_L's column came from a zero QR column */
-  SOAP_STATE_SKIP_R = 8 /* uint8 per col: same for Q_R */
+  SOAP_STATE_SKIP_R = 8,/* uint8 per col: same for Q_R */
+  SOAP_STATE_LAMBDA_L = 9, /* fp32 per row: lam_L = diag(Q_L^T L Q_L) as the last KL step
+                              computed it (before the clamp at 0); read-only, present only
+                              with kl = 1 on a matrix preconditioned on both sides */
+  SOAP_STATE_LAMBDA_R = 10 /* fp32 per col: lam_R likewise */
 } soap_state_which;
 
 /* Number of bytes soap_state_get/set move for (idx, which); 0 if that piece does not
@@ -125,7 +137,8 @@ soap_status_t soap_state_get(soap_handle h, int32_t idx, int32_t which, void* ds
 
 /* Copies src (host or device) into one piece of matrix idx's state, ordered on
  * `stream`. Setting SOAP_STATE_M stores Q_L m Q_R^T with the Q_L, Q_R held at that
- * moment, so set Q_L and Q_R first. */
+ * moment, so set Q_L and Q_R first. SOAP_STATE_LAMBDA_L/R are read-only (each KL step
+ * recomputes them): setting one returns SOAP_ERR_INVALID_ARG. */
 soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const void* src,
                              soap_stream_t stream);
 

@@ -11,6 +11,9 @@
 //    guard.
 //  * weight_update: W <- (1 - lr wd) W - lr N for a matrix with no preconditioned
 //    side (Alg. 1 "Weight decay and update" with Q_L = Q_R = I).
+//  * diag_dot, scale_cols_split: the KL-Shampoo factor form's approximate eigenvalues
+//    lam = diag(Q^T F Q) and the column weights sqrt(coef / (lam + eps)) applied to G Q
+//    (Alg. 1 "Accumulate Kronecker Factors (KL-Shampoo)").
 #include <algorithm>
 
 #include "profile.h"
@@ -290,6 +293,49 @@ __global__ void basis_from_qt_kernel(const float* Qt, const float* Qt_lo, float*
   }
 }
 
+// lam[b][i] = sum_k C[b][i][k] Qt[b][i][k] = (Q^T F Q)_ii for C = Q^T F: one warp per row.
+__global__ void diag_dot_kernel(const float* C, const float* Qt, float* lam, int n) {
+  const int b = blockIdx.y;
+  const int row = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (row >= n) return;
+  const int64_t off = (int64_t)b * n * n + (int64_t)row * n;
+  const float4* c = reinterpret_cast<const float4*>(C + off);
+  const float4* q = reinterpret_cast<const float4*>(Qt + off);
+  float acc = 0.f;
+  for (int k = lane; k < n / 4; k += 32) {
+    const float4 x = c[k], y = q[k];
+    acc = fmaf(x.x, y.x, acc);
+    acc = fmaf(x.y, y.y, acc);
+    acc = fmaf(x.z, y.z, acc);
+    acc = fmaf(x.w, y.w, acc);
+  }
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (lane == 0) lam[(int64_t)b * n + row] = acc;
+}
+
+// X[b][i][j] <- X[b][i][j] * sqrt(coef / (max(lam[b][j], 0) + eps)) and its lo part (cols a
+// multiple of 4, rows of 16-byte multiples).
+__global__ void scale_cols_split_kernel(float* X, float* X_lo, const float* lam, int rows, int cols, float coef,
+                                        float eps) {
+  const int b = blockIdx.y;
+  const int64_t e4 = (int64_t)rows * cols / 4;
+  float4* x = reinterpret_cast<float4*>(X + (int64_t)b * rows * cols);
+  float4* xl = reinterpret_cast<float4*>(X_lo + (int64_t)b * rows * cols);
+  const float* l = lam + (int64_t)b * cols;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < e4; i += stride) {
+    const int j = (int)((i * 4) % cols);
+    float4 v = x[i];
+    v.x *= sqrtf(coef / (fmaxf(l[j], 0.f) + eps));
+    v.y *= sqrtf(coef / (fmaxf(l[j + 1], 0.f) + eps));
+    v.z *= sqrtf(coef / (fmaxf(l[j + 2], 0.f) + eps));
+    v.w *= sqrtf(coef / (fmaxf(l[j + 3], 0.f) + eps));
+    x[i] = v;
+    xl[i] = make_float4(lo_part(v.x), lo_part(v.y), lo_part(v.z), lo_part(v.w));
+  }
+}
+
 __global__ void split_kernel(const float* x, float* hi, float* lo, int64_t n) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
@@ -346,6 +392,26 @@ cudaError_t split_tf32(const float* x, float* hi, float* lo, int64_t n, cudaStre
   ProfScope prof(kFamElementwise, 2.0 * n, 12.0 * n, s);
   const int64_t want = (n + kThreads - 1) / kThreads;
   split_kernel<<<(int)(want < 4096 ? want : 4096), kThreads, 0, s>>>(x, hi, lo, n);
+  return cudaGetLastError();
+}
+
+cudaError_t diag_dot(const float* C, const float* Qt, float* lam, int n, int batch, cudaStream_t s) {
+  if (n <= 0 || batch <= 0) return cudaSuccess;
+  if ((n & 3) || batch > 65535) return cudaErrorInvalidValue;
+  const double e = (double)n * n * batch;
+  ProfScope prof(kFamElementwise, 2.0 * e, 8.0 * e, s);
+  diag_dot_kernel<<<dim3((n + 7) / 8, batch), 256, 0, s>>>(C, Qt, lam, n);
+  return cudaGetLastError();
+}
+
+cudaError_t scale_cols_split(float* X, float* X_lo, const float* lam, int rows, int cols, int batch, float coef,
+                             float eps, cudaStream_t s) {
+  const int64_t elems = (int64_t)rows * cols;
+  if (elems <= 0 || batch <= 0) return cudaSuccess;
+  if ((cols & 3) || batch > 65535) return cudaErrorInvalidValue;
+  ProfScope prof(kFamElementwise, 4.0 * elems * batch, 12.0 * elems * batch, s);
+  scale_cols_split_kernel<<<dim3(blocks_for(elems, batch), batch), kThreads, 0, s>>>(X, X_lo, lam, rows, cols, coef,
+                                                                                     eps);
   return cudaGetLastError();
 }
 

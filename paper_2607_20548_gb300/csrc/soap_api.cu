@@ -14,6 +14,9 @@
 //   G' = X1 Q_R, m = X2 Q_R
 //   v <- b2 v + (1-b2) G'^2, N = m / (sqrt(v) + eps)        S6
 //   X1 = Q_L N; W <- (1 - lr wd) W - lr X1 Q_R^T           S7, S8 (fused in the GEMM epilogue)
+// With hparams.kl, S1 takes Alg. 1's KL-Shampoo form instead: each factor's EMA term is
+// weighed by the other factor's inverse, Q diag(1/(lam + eps)) Q^T with lam = diag(Q^T F Q)
+// (an identity side as lam = 1); see prepare_class.
 #include <algorithm>
 #include <cstdio>
 #include <cstring>
@@ -60,6 +63,9 @@ struct ClassState {
   float* QRt = nullptr;
   float* QRt_lo = nullptr;
   bool basis_dirty = true;  // Q^T and lo parts must be rebuilt from Q before use
+  // KL-Shampoo factor form, two-sided classes: the approximate eigenvalues of the last step
+  float* lamL = nullptr;  // [count][rows]
+  float* lamR = nullptr;  // [count][cols]
 };
 
 // One preconditioned side of one class: `count` factors of size n in a QR group.
@@ -114,6 +120,7 @@ struct soap_s {
   float* N_lo = nullptr;
   float* Zt = nullptr;   // (N Q_R^T)^T
   float* Zt_lo = nullptr;
+  float* lam_ws = nullptr;  // Q^T F of the KL form's eigenvalue estimate (two-sided classes)
   std::vector<QrGroup> groups;  // largest n first
   cudaEvent_t fork_ev = nullptr;
   int* d_status = nullptr;
@@ -225,15 +232,20 @@ soap_status_t prepare_class(soap_handle h, ClassState& c, const float* const* d_
   const int B = c.count, m = (int)c.rows, n = (int)c.cols;
   const int64_t mn = (int64_t)m * n, mm = (int64_t)m * m, nn = (int64_t)n * n;
   const float fb = hp.factor_beta;
+  // S1 weights. Standard form: 1 - b. KL form with an identity side (S = I, lambda = 1):
+  // (1 - b) / (other dimension * (1 + eps)); a two-sided KL class weighs G's columns (rows)
+  // by the other factor's eigenvalues instead (below).
+  const float aL = hp.kl ? (float)((1.0 - fb) / ((double)n * (1.0 + hp.eps))) : 1.f - fb;
+  const float aR = hp.kl ? (float)((1.0 - fb) / ((double)m * (1.0 + hp.eps))) : 1.f - fb;
   using soap::strided;
   using soap::strided_mut;
   if (!c.tc) {
     SOAP_CUDA(h, soap::momentum_and_copy(d_grads, c.Gc, c.Mhat, mn, B, hp.beta1, h->d_status, s));
     if (c.left)  // S1: L <- b L + (1-b) G G^T
-      SOAP_CUDA(h, soap::gemm(false, true, m, m, n, 1.f - fb, strided(c.Gc, n, mn), strided(c.Gc, n, mn), fb,
+      SOAP_CUDA(h, soap::gemm(false, true, m, m, n, aL, strided(c.Gc, n, mn), strided(c.Gc, n, mn), fb,
                               strided_mut(c.L, m, mm), B, s));
     if (c.right)  // S1: R <- b R + (1-b) G^T G
-      SOAP_CUDA(h, soap::gemm(true, false, n, n, m, 1.f - fb, strided(c.Gc, n, mn), strided(c.Gc, n, mn), fb,
+      SOAP_CUDA(h, soap::gemm(true, false, n, n, m, aR, strided(c.Gc, n, mn), strided(c.Gc, n, mn), fb,
                               strided_mut(c.R, n, nn), B, s));
     return SOAP_OK;
   }
@@ -244,12 +256,43 @@ soap_status_t prepare_class(soap_handle h, ClassState& c, const float* const* d_
     if (c.right) SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, n, B, s));
     c.basis_dirty = false;
   }
+  if (hp.kl && c.left && c.right) {
+    // KL-Shampoo factor form (Alg. 1), from the factors and bases held before this step:
+    //   lam_L = diag(Q_L^T L Q_L), lam_R = diag(Q_R^T R Q_R)       (C = Q^T F, then row dots)
+    //   Y = G Q_R diag(sqrt(w_R)),  w_R = (1-b) / (cols (lam_R + eps))
+    //   X = G^T Q_L diag(sqrt(w_L)), w_L = (1-b) / (rows (lam_L + eps))
+    //   L <- b L + Y Y^T,  R <- b R + X X^T
+    // Y and X (with their lo parts) live in the rotation workspace, free until phase C.
+    const int64_t cls = (int64_t)B * mn;
+    float* C = h->lam_ws;
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, m, m, B, opnd(c.QLt, c.QLt_lo, m, mm, B), opnd(c.L, c.L_lo, m, mm, B),
+                                  epi(h, C, m, mm, nullptr, 0, 1.f, 0.f), s));
+    SOAP_CUDA(h, soap::diag_dot(C, c.QLt, c.lamL, m, B, s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(n, n, n, B, opnd(c.QRt, c.QRt_lo, n, nn, B), opnd(c.R, c.R_lo, n, nn, B),
+                                  epi(h, C, n, nn, nullptr, 0, 1.f, 0.f), s));
+    SOAP_CUDA(h, soap::diag_dot(C, c.QRt, c.lamR, n, B, s));
+    float* Y = h->YMt;
+    float* Y_lo = h->YMt_lo;
+    float* X = h->YMt + cls;
+    float* X_lo = h->YMt_lo + cls;
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, B, opnd(c.Gc, c.Gc_lo, n, mn, B), opnd(c.QRt, c.QRt_lo, n, nn, B),
+                                  epi(h, Y, n, mn, nullptr, 0, 1.f, 0.f), s));
+    SOAP_CUDA(h, soap::scale_cols_split(Y, Y_lo, c.lamR, m, n, B, (float)((1.0 - fb) / n), hp.eps, s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(n, m, m, B, opnd(c.Gt, c.Gt_lo, m, mn, B), opnd(c.QLt, c.QLt_lo, m, mm, B),
+                                  epi(h, X, m, mn, nullptr, 0, 1.f, 0.f), s));
+    SOAP_CUDA(h, soap::scale_cols_split(X, X_lo, c.lamL, n, m, B, (float)((1.0 - fb) / m), hp.eps, s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(Y, Y_lo, n, mn, B), opnd(Y, Y_lo, n, mn, B),
+                                  epi(h, c.L, m, mm, c.L_lo, 0, 1.f, fb), s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(X, X_lo, m, mn, B), opnd(X, X_lo, m, mn, B),
+                                  epi(h, c.R, n, nn, c.R_lo, 0, 1.f, fb), s));
+    return SOAP_OK;
+  }
   if (c.left)
     SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(c.Gc, c.Gc_lo, n, mn, B), opnd(c.Gc, c.Gc_lo, n, mn, B),
-                                  epi(h, c.L, m, mm, c.L_lo, 0, 1.f - fb, fb), s));
+                                  epi(h, c.L, m, mm, c.L_lo, 0, aL, fb), s));
   if (c.right)
     SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(c.Gt, c.Gt_lo, m, mn, B), opnd(c.Gt, c.Gt_lo, m, mn, B),
-                                  epi(h, c.R, n, nn, c.R_lo, 0, 1.f - fb, fb), s));
+                                  epi(h, c.R, n, nn, c.R_lo, 0, aR, fb), s));
   return SOAP_OK;
 }
 
@@ -412,6 +455,7 @@ void soap_default_hparams(soap_hparams* hp) {
   hp->bias_correction = 0;
   hp->qr_tol = 1e-4f;
   hp->guard = 1;
+  hp->kl = 0;
 }
 
 soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparams* hp,
@@ -420,6 +464,8 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
   *out = nullptr;
   if (!shapes || n <= 0 || !hp) return SOAP_ERR_INVALID_ARG;
   if (hp->eig_every < 1 || !(hp->eps >= 0.f) || !(hp->qr_tol >= 0.f)) return SOAP_ERR_INVALID_ARG;
+  if (hp->kl != 0 && hp->kl != 1) return SOAP_ERR_INVALID_ARG;
+  if (hp->kl && !(hp->eps > 0.f)) return SOAP_ERR_INVALID_ARG;
   for (int i = 0; i < n; ++i) {
     const soap_shape& s = shapes[i];
     if (s.rows < 1 || s.cols < 1 || s.rows > (1 << 20) || s.cols > (1 << 20)) return SOAP_ERR_INVALID_ARG;
@@ -515,6 +561,12 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
         if (e == cudaSuccess) e = dalloc(h, (void**)&c.QRt_lo, nn * 4);
       }
     }
+    if (hp->kl && c.left && c.right) {
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.lamL, (size_t)c.count * c.rows * 4);
+      if (e == cudaSuccess) e = dalloc(h, (void**)&c.lamR, (size_t)c.count * c.cols * 4);
+      if (e == cudaSuccess) e = cudaMemset(c.lamL, 0, (size_t)c.count * c.rows * 4);
+      if (e == cudaSuccess) e = cudaMemset(c.lamR, 0, (size_t)c.count * c.cols * 4);
+    }
     ws_mat = std::max(ws_mat, mn);
   }
   // QR groups: every preconditioned side, grouped by size
@@ -567,11 +619,13 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
   // workspaces: [G' | m'] for every class; N's lo part for tensor-core classes; the
   // intermediate products of two-sided tensor-core classes; X1/X2 for CUDA-core classes and
   // for single-matrix state reads and writes
-  size_t ws_tc = 0, ws_two = 0, ws_x = 0;
+  size_t ws_tc = 0, ws_two = 0, ws_x = 0, ws_lam = 0;
   for (auto& c : h->classes) {
     const size_t mn = (size_t)c.count * c.rows * c.cols;
     if (c.tc) ws_tc = std::max(ws_tc, mn);
     if (c.tc && c.left && c.right) ws_two = std::max(ws_two, mn);
+    if (hp->kl && c.left && c.right)
+      ws_lam = std::max(ws_lam, (size_t)c.count * std::max(c.rows * c.rows, c.cols * c.cols));
     ws_x = std::max(ws_x, c.tc ? (size_t)(c.rows * c.cols) : mn);
   }
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->X1, ws_x * 4);
@@ -583,6 +637,7 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt_lo, 2 * ws_two * 4);
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt, ws_two * 4);
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt_lo, ws_two * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->lam_ws, ws_lam * 4);
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_status, sizeof(int));
   if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_ptrs, h->nptrs * sizeof(void*));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&h->h_status, sizeof(int));
@@ -605,11 +660,13 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
     if (e == cudaSuccess) e = cudaMemset(c.V, 0, mn * 4);
     if (c.left) {
       if (e == cudaSuccess) e = cudaMemset(c.L, 0, (size_t)c.count * c.rows * c.rows * 4);
+      if (c.tc && e == cudaSuccess) e = cudaMemset(c.L_lo, 0, (size_t)c.count * c.rows * c.rows * 4);
       if (e == cudaSuccess) e = soap::set_identity(c.QL, (int)c.rows, c.count, 0);
       if (e == cudaSuccess) e = cudaMemset(c.skipL, 0, (size_t)c.count * c.rows);
     }
     if (c.right) {
       if (e == cudaSuccess) e = cudaMemset(c.R, 0, (size_t)c.count * c.cols * c.cols * 4);
+      if (c.tc && e == cudaSuccess) e = cudaMemset(c.R_lo, 0, (size_t)c.count * c.cols * c.cols * 4);
       if (e == cudaSuccess) e = soap::set_identity(c.QR, (int)c.cols, c.count, 0);
       if (e == cudaSuccess) e = cudaMemset(c.skipR, 0, (size_t)c.count * c.cols);
     }
@@ -713,6 +770,10 @@ size_t soap_state_bytes(soap_handle h, int32_t idx, int32_t which) {
     case SOAP_STATE_QR: return s.precond_right ? (size_t)s.cols * s.cols * 4 : 0;
     case SOAP_STATE_SKIP_L: return s.precond_left ? (size_t)s.rows : 0;
     case SOAP_STATE_SKIP_R: return s.precond_right ? (size_t)s.cols : 0;
+    case SOAP_STATE_LAMBDA_L:
+      return h->hp.kl && s.precond_left && s.precond_right ? (size_t)s.rows * 4 : 0;
+    case SOAP_STATE_LAMBDA_R:
+      return h->hp.kl && s.precond_left && s.precond_right ? (size_t)s.cols * 4 : 0;
     default: return 0;
   }
 }
@@ -732,6 +793,8 @@ void* state_ptr(soap_handle h, int idx, int which) {
     case SOAP_STATE_QR: return c.QR ? c.QR + slot * nn : nullptr;
     case SOAP_STATE_SKIP_L: return c.skipL ? c.skipL + slot * c.rows : nullptr;
     case SOAP_STATE_SKIP_R: return c.skipR ? c.skipR + slot * c.cols : nullptr;
+    case SOAP_STATE_LAMBDA_L: return c.lamL ? c.lamL + slot * c.rows : nullptr;
+    case SOAP_STATE_LAMBDA_R: return c.lamR ? c.lamR + slot * c.cols : nullptr;
     default: return nullptr;
   }
 }
@@ -808,6 +871,8 @@ soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const vo
   if (!h) return SOAP_ERR_INVALID_ARG;
   const size_t bytes = soap_state_bytes(h, idx, which);
   if (bytes == 0 || !src) return fail(h, SOAP_ERR_INVALID_ARG, "soap_state_set: no such state piece");
+  if (which == SOAP_STATE_LAMBDA_L || which == SOAP_STATE_LAMBDA_R)
+    return fail(h, SOAP_ERR_INVALID_ARG, "soap_state_set: the KL eigenvalue estimates are read-only");
   DeviceGuard g(h->device);
   cudaStream_t s = (cudaStream_t)stream_;
   const auto [ci, slot] = h->loc[idx];
@@ -826,6 +891,13 @@ soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const vo
     if (which == SOAP_STATE_QL || which == SOAP_STATE_QR) c.basis_dirty = true;
     if (which == SOAP_STATE_MHAT && c.tc)
       SOAP_CUDA(h, soap::split_tf32(dstm, nullptr, c.Mhat_lo + slot * mn, mn, s));
+    // the factors' lo parts: the KL form reads them (lambda = diag(Q^T F Q)) before S1 rewrites them
+    if (which == SOAP_STATE_L && c.tc)
+      SOAP_CUDA(h, soap::split_tf32(c.L + slot * (int64_t)m * m, nullptr, c.L_lo + slot * (int64_t)m * m,
+                                    (int64_t)m * m, s));
+    if (which == SOAP_STATE_R && c.tc)
+      SOAP_CUDA(h, soap::split_tf32(c.R + slot * (int64_t)nc * nc, nullptr, c.R_lo + slot * (int64_t)nc * nc,
+                                    (int64_t)nc * nc, s));
     return SOAP_OK;
   }
   // M_hat = Q_L m Q_R^T

@@ -127,6 +127,13 @@ cudaError_t basis_split(const float* Q, float* Q_lo, float* Qt, float* Qt_lo, in
 // W <- (1 - lr*wd) W - lr * D (both sides identity).
 cudaError_t weight_update(float* const* params, const float* D, int64_t elems, int batch,
                           float lr, float wd, cudaStream_t stream);
+// KL-Shampoo factor form: lam[b][i] = sum_k C[b][i][k] Qt[b][i][k], the diagonal of Q^T F Q
+// from C = Q^T F (n a multiple of 4).
+cudaError_t diag_dot(const float* C, const float* Qt, float* lam, int n, int batch, cudaStream_t stream);
+// X[b][:, j] *= sqrt(coef / (max(lam[b][j], 0) + eps)) in place, with the lo part into X_lo
+// (cols a multiple of 4).
+cudaError_t scale_cols_split(float* X, float* X_lo, const float* lam, int rows, int cols, int batch,
+                             float coef, float eps, cudaStream_t stream);
 // Sets `batch` n x n matrices to the identity.
 cudaError_t set_identity(float* Q, int n, int batch, cudaStream_t stream);
 

@@ -19,7 +19,8 @@ LIB_PATH = os.path.join(_HERE, "_lib", platform.machine(), "libsoap.so")
 SOAP_OK = 0
 STATUS_NAMES = {0: "SOAP_OK", 1: "SOAP_ERR_INVALID_ARG", 2: "SOAP_ERR_CUDA", 3: "SOAP_ERR_OOM",
                 4: "SOAP_ERR_NONFINITE", 5: "SOAP_ERR_QR_BREAKDOWN", 6: "SOAP_ERR_TIMEOUT"}
-STATE_M, STATE_V, STATE_L, STATE_QL, STATE_R, STATE_QR, STATE_MHAT, STATE_SKIP_L, STATE_SKIP_R = range(9)
+(STATE_M, STATE_V, STATE_L, STATE_QL, STATE_R, STATE_QR, STATE_MHAT, STATE_SKIP_L, STATE_SKIP_R,
+ STATE_LAMBDA_L, STATE_LAMBDA_R) = range(11)
 
 # every symbol include/soap.h declares
 EXPORTS = ("soap_default_hparams", "soap_create", "soap_step", "soap_set_lr", "soap_state_bytes",
@@ -41,7 +42,7 @@ class soap_hparams(ctypes.Structure):
                 ("factor_beta", ctypes.c_float), ("eps", ctypes.c_float),
                 ("weight_decay", ctypes.c_float), ("eig_every", ctypes.c_int32),
                 ("bias_correction", ctypes.c_int32), ("qr_tol", ctypes.c_float),
-                ("guard", ctypes.c_int32)]
+                ("guard", ctypes.c_int32), ("kl", ctypes.c_int32)]
 
 
 class soap_kernel_stats(ctypes.Structure):
@@ -181,7 +182,8 @@ class SoapOptimizer:
         s = self.shapes[idx]
         shape = {STATE_M: (s.rows, s.cols), STATE_V: (s.rows, s.cols), STATE_MHAT: (s.rows, s.cols),
                  STATE_L: (s.rows, s.rows), STATE_QL: (s.rows, s.rows), STATE_R: (s.cols, s.cols),
-                 STATE_QR: (s.cols, s.cols), STATE_SKIP_L: (s.rows,), STATE_SKIP_R: (s.cols,)}.get(which)
+                 STATE_QR: (s.cols, s.cols), STATE_SKIP_L: (s.rows,), STATE_SKIP_R: (s.cols,),
+                 STATE_LAMBDA_L: (s.rows,), STATE_LAMBDA_R: (s.cols,)}.get(which)
         if shape is None or self.state_bytes(idx, which) == 0:
             raise SoapError(1, f"no state piece {which} for matrix {idx}")
         dtype = torch.uint8 if which in (STATE_SKIP_L, STATE_SKIP_R) else torch.float32

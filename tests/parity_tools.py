@@ -41,7 +41,8 @@ def rel(a, b):
 def oracle_hparams(hp: S.soap_hparams) -> HParams:
     return HParams(lr=hp.lr, beta1=hp.beta1, beta2=hp.beta2, factor_beta=hp.factor_beta, eps=hp.eps,
                    weight_decay=hp.weight_decay, eig_every=hp.eig_every,
-                   bias_correction=bool(hp.bias_correction), guard=bool(hp.guard), qr_tol=hp.qr_tol)
+                   bias_correction=bool(hp.bias_correction), guard=bool(hp.guard), qr_tol=hp.qr_tol,
+                   kl=bool(hp.kl))
 
 
 def gpu_state(opt: S.SoapOptimizer, idx: int, dtype) -> MatrixState:

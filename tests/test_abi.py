@@ -42,6 +42,14 @@ def test_host_side_validation_needs_no_gpu():
     bad_hp.eig_every = 0
     ok_shape = (S.soap_shape * 1)(S.soap_shape(4, 5, 1, 1))
     assert lib.soap_create(ok_shape, 1, ctypes.byref(bad_hp), 0, ctypes.byref(h)) == 1
+    # the KL-Shampoo factor form is off by default and needs eps > 0 (its first step weighs by 1/eps)
+    assert hp.kl == 0
+    kl_hp = S.soap_hparams()
+    lib.soap_default_hparams(ctypes.byref(kl_hp))
+    kl_hp.kl, kl_hp.eps = 1, 0.0
+    assert lib.soap_create(ok_shape, 1, ctypes.byref(kl_hp), 0, ctypes.byref(h)) == 1
+    kl_hp.kl, kl_hp.eps = 2, 1e-8
+    assert lib.soap_create(ok_shape, 1, ctypes.byref(kl_hp), 0, ctypes.byref(h)) == 1
     assert lib.soap_gemm(0, 0, -1, 1, 1, 1.0, None, 1, 0, None, 1, 0, 0.0, None, 1, 0, 1, None) == 1
     assert lib.soap_gemm(0, 0, 0, 1, 1, 1.0, None, 1, 0, None, 1, 0, 0.0, None, 1, 0, 1, None) == 0
     assert lib.soap_qr(0, 1, None, None, None, 0.0, None, 0, None) == 1
