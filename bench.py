@@ -157,7 +157,9 @@ def roofline(family, st, peaks, peak_src):
     # the kernels run inside a long step: the sustained tensor peak
     tc_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]) / 2.0 / TC_PRODUCTS
     ridge = tc_peak * 1e12 / (peaks["hbm_gbs"] * 1e9)  # FLOP per byte where the two bounds meet
-    if family == "gemm_tc" and st["flops"] / max(1.0, st["bytes"]) >= ridge:
+    # a tensor-core family whose FLOPs per algorithmic byte reach the ridge is bound by the tensor
+    # pipe (the QR's block products sit at the ridge: 2 x 128 fp32 FLOP per 4-8 bytes of C)
+    if family in ("gemm_tc", "qr_update") and st["flops"] / max(1.0, st["bytes"]) >= ridge:
         ach = st["flops"] / secs / 1e12
         return dict(base, bound="tensor", achieved=ach, peak=tc_peak, unit="TFLOP/s", frac=ach / tc_peak,
                     peak_source=f"{peak_src} sustained bf16 dense / 2 (tf32) / {TC_PRODUCTS} (tf32 products per fp32 product)")
