@@ -637,12 +637,13 @@ __global__ void split_reduce_kernel(const float* P, int ksplit, int batch, int M
 }
 
 // How many K splits give the fewest idle SMs in the last wave, for a launch of `tiles` tiles
-// with kblocks K blocks (each split keeps at least 16 K blocks), within `cap` partial matrices.
+// with kblocks K blocks (each split keeps at least 16 K blocks, at most 16 splits), within `cap`
+// partial matrices.
 int choose_ksplit(int64_t tiles, int kblocks, int64_t cap) {
   if (kblocks < 32 || tiles >= 2 * 152) return 1;
   int best = 1;
   double best_eff = 0.0;
-  for (int sp = 1; sp <= 8 && kblocks / sp >= 16 && sp <= cap; ++sp) {
+  for (int sp = 1; sp <= 16 && kblocks / sp >= 16 && sp <= cap; ++sp) {
     const int64_t ctas = tiles * sp;
     const double eff = (double)ctas / (double)(((ctas + 151) / 152) * 152);
     if (eff > best_eff + 0.02) {

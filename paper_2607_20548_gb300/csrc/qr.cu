@@ -610,12 +610,19 @@ struct Workspace {
   float* Ypart;   // [batch][MAXC][NBO][NB]
   float* Wsplit;  // [KSPLIT][batch][n][NBO] partial sums of split-K products
   // for the look-ahead schedule only (null otherwise): the far update's own W and split-K
-  // buffers, and a second V T^T buffer (blocks alternate)
+  // buffers, and second V T^T, Vpos and T buffers (blocks alternate: a block's V T^T is read
+  // by its far update and its Vpos and T by its V T while the next block is factored)
   float* W2;
   float* W2_lo;
   float* Wsplit2;
   float* VTr2;
   float* VTr2_lo;
+  float* Vpos2;
+  float* Vpos2_lo;
+  float* T2;
+  float* T2_lo;
+  float* Tt2;
+  float* Tt2_lo;
   float* thresh;
   float* dsign;
   double* part;
@@ -644,6 +651,9 @@ Workspace carve(void* base, int n, int batch, size_t* total, bool lookahead) {
   const size_t oW2 = lookahead ? take(thin) : 0, oW2l = lookahead ? take(thin) : 0;
   const size_t oWs2 = lookahead ? take((size_t)KSPLIT * thin) : 0;
   const size_t oVr2 = lookahead ? take(thin) : 0, oVr2l = lookahead ? take(thin) : 0;
+  const size_t oVp2 = lookahead ? take(thin) : 0, oVp2l = lookahead ? take(thin) : 0;
+  const size_t oT2 = lookahead ? take(tsq) : 0, oT2l = lookahead ? take(tsq) : 0;
+  const size_t oTt2 = lookahead ? take(tsq) : 0, oTt2l = lookahead ? take(tsq) : 0;
   const size_t oth = take((size_t)batch * sizeof(float));
   const size_t osg = take((size_t)batch * n * sizeof(float));
   const size_t opart = take((size_t)batch * NORM_CHUNKS * sizeof(double));
@@ -653,7 +663,8 @@ Workspace carve(void* base, int n, int batch, size_t* total, bool lookahead) {
   auto g = [&](size_t o) { return lookahead ? (float*)(c + o) : nullptr; };
   return Workspace{f(oAt), nullptr, f(oVt), f(oVtl), f(oVq), f(oVql), f(oVr), f(oVrl), f(oVp),  f(oVpl),
                    f(oW),  f(oWl),  f(oT),  f(oTl),  f(oTt), f(oTtl), f(oY),  f(oWs), g(oW2),  g(oW2l),
-                   g(oWs2), g(oVr2), g(oVr2l), f(oth), f(osg), (double*)(c + opart)};
+                   g(oWs2), g(oVr2), g(oVr2l), g(oVp2), g(oVp2l), g(oT2),  g(oT2l),  g(oTt2), g(oTt2l),
+                   f(oth), f(osg), (double*)(c + opart)};
 }
 
 TcOperand op(const float* hi, const float* lo, int64_t ld, int64_t stride, int batch) {
@@ -678,12 +689,14 @@ void qr_input_buffers(void* workspace, int n, int batch, float** At) {
 }
 
 cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q_lo, uint8_t* skip, float tol,
-                   void* workspace, size_t workspace_bytes, int* status, cudaStream_t s, cudaStream_t far,
-                   cudaEvent_t ev_vt, cudaEvent_t ev_far) {
+                   void* workspace, size_t workspace_bytes, int* status, cudaStream_t s, const QrLookahead* lah) {
   if (n <= 0 || batch <= 0) return cudaSuccess;
   if (n > 8192 || batch > 65535 || (n & 3)) return cudaErrorInvalidValue;
-  // look-ahead: a second stream and two events given, and a workspace sized for it
-  const bool la = far && ev_vt && ev_far && workspace_bytes >= qr_workspace_bytes(n, batch, true);
+  // look-ahead: a second stream and its events given, and a workspace sized for it
+  const bool la = lah && lah->far && lah->vt && lah->far_done && lah->vq[0] && lah->vq[1] &&
+                  workspace_bytes >= qr_workspace_bytes(n, batch, true);
+  cudaStream_t far = la ? lah->far : nullptr;
+  cudaEvent_t ev_vt = la ? lah->vt : nullptr, ev_far = la ? lah->far_done : nullptr;
   size_t need = 0;
   Workspace w = carve(workspace, n, batch, &need, la);
   if (workspace_bytes < need) return cudaErrorInvalidValue;
@@ -713,10 +726,24 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
   }
   for (int blk = 0; blk < nblock; ++blk) {
     const int k0 = blk * NBO, kbo = std::min(NBO, n - k0), m = n - k0;
+    const int par = blk & 1;
+    const bool alt = la && par;
+    float* vp = alt ? w.Vpos2 : w.Vpos;
+    float* vp_lo = alt ? w.Vpos2_lo : w.Vpos_lo;
+    float* Tb = alt ? w.T2 : w.T;
+    float* Tb_lo = alt ? w.T2_lo : w.T_lo;
+    float* Ttb = alt ? w.Tt2 : w.Tt;
+    float* Ttb_lo = alt ? w.Tt2_lo : w.Tt_lo;
+    // with the look-ahead, this block's Vpos and T buffers were last read by the V T of the
+    // block two before, on the far stream
+    if (la && blk >= 2) {
+      e = cudaStreamWaitEvent(s, lah->vq[par], 0);
+      if (e != cudaSuccess) return e;
+    }
     for (int k = k0; k < k0 + kbo; k += NB) {
       const int kb = std::min(NB, n - k);
       const int C = (n - k + pk.cols - 1) / pk.cols;
-      PanelArgs a{w.At, w.Vt, w.Vt_lo, w.Vpos, w.Vpos_lo, w.T, w.T_lo, w.Tt, w.Tt_lo, w.Ypart, skip, w.dsign,
+      PanelArgs a{w.At, w.Vt, w.Vt_lo, vp, vp_lo, Tb, Tb_lo, Ttb, Ttb_lo, w.Ypart, skip, w.dsign,
                   w.thresh, status, n, k0, kbo, k, kb};
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(C, batch, 1);
@@ -742,20 +769,27 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     // VTq = V T (the Q accumulation) and VTr = V T^T (this block's trailing update); with the
     // look-ahead the V T^T buffers alternate between blocks, since the far update of block b
     // still reads its V T^T while block b+1 forms its own
-    float* vtr = (la && (blk & 1)) ? w.VTr2 : w.VTr;
-    float* vtr_lo = (la && (blk & 1)) ? w.VTr2_lo : w.VTr_lo;
+    float* vtr = alt ? w.VTr2 : w.VTr;
+    float* vtr_lo = alt ? w.VTr2_lo : w.VTr_lo;
     float* vq = w.VTq + (int64_t)blk * thin + (int64_t)k0 * NBO;
     float* vq_lo = w.VTq_lo + (int64_t)blk * thin + (int64_t)k0 * NBO;
-    const TcOperand vpos = op(w.Vpos + (int64_t)k0 * NBO, w.Vpos_lo + (int64_t)k0 * NBO, NBO, thin, batch);
-    e = gemm_tc_nt(m, kbo, kbo, batch, vpos, op(w.Tt, w.Tt_lo, NBO, NBO * NBO, batch),
-                   out(vq, vq_lo, NBO, vq_stride, 1.f, 0.f, status), s, kFamQrUpdate);
-    if (e != cudaSuccess) return e;
+    const TcOperand vpos = op(vp + (int64_t)k0 * NBO, vp_lo + (int64_t)k0 * NBO, NBO, thin, batch);
+    auto form_vtq = [&](cudaStream_t st) {
+      return gemm_tc_nt(m, kbo, kbo, batch, vpos, op(Ttb, Ttb_lo, NBO, NBO * NBO, batch),
+                        out(vq, vq_lo, NBO, vq_stride, 1.f, 0.f, status), st, kFamQrUpdate);
+    };
+    if (!la) {
+      e = form_vtq(s);
+      if (e != cudaSuccess) return e;
+    }
     const int nc = n - k0 - kbo;  // trailing rows of At (columns of P)
-    if (nc <= 0) continue;
-    e = gemm_tc_nt(m, kbo, kbo, batch, vpos, op(w.T, w.T_lo, NBO, NBO * NBO, batch),
-                   out(vtr + (int64_t)k0 * NBO, vtr_lo + (int64_t)k0 * NBO, NBO, thin, 1.f, 0.f, status), s,
-                   kFamQrUpdate);
-    if (e != cudaSuccess) return e;
+    if (nc > 0) {
+      e = gemm_tc_nt(m, kbo, kbo, batch, vpos, op(Tb, Tb_lo, NBO, NBO * NBO, batch),
+                     out(vtr + (int64_t)k0 * NBO, vtr_lo + (int64_t)k0 * NBO, NBO, thin, 1.f, 0.f, status), s,
+                     kFamQrUpdate);
+      if (e != cudaSuccess) return e;
+    }
+    if (nc <= 0 && !la) continue;
     const TcOperand vtr_trail =
         op(vtr + (int64_t)(k0 + kbo) * NBO, vtr_lo + (int64_t)(k0 + kbo) * NBO, NBO, thin, batch);
     const TcOperand vt_blk = op(w.Vt + (int64_t)k0 * n + k0, w.Vt_lo + (int64_t)k0 * n + k0, n, nn, batch);
@@ -779,18 +813,22 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     }
     // look-ahead: the next block's rows now (they gate its panels), the rest on the far stream,
     // where it overlaps the next block's panels; the next block's rows wait for the previous
-    // far update, which covered them
-    const int knext = std::min(NBO, nc);
+    // far update, which covered them. The block's V T follows its far update on the far stream.
+    const int knext = std::min(NBO, std::max(nc, 0));
     e = cudaEventRecord(ev_vt, s);
-    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev_far, 0);
-    if (e == cudaSuccess) e = update_rows(k0 + kbo, knext, w.W, w.W_lo, w.Wsplit, s);
+    if (e == cudaSuccess && nc > 0) e = cudaStreamWaitEvent(s, ev_far, 0);
+    if (e == cudaSuccess && nc > 0) e = update_rows(k0 + kbo, knext, w.W, w.W_lo, w.Wsplit, s);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(far, ev_vt, 0);
     if (e == cudaSuccess && nc > knext) e = update_rows(k0 + kbo + knext, nc - knext, w.W2, w.W2_lo, w.Wsplit2, far);
     if (e == cudaSuccess) e = cudaEventRecord(ev_far, far);
+    if (e == cudaSuccess) e = form_vtq(far);
+    if (e == cudaSuccess) e = cudaEventRecord(lah->vq[par], far);
     if (e != cudaSuccess) return e;
   }
   if (la) {
-    e = cudaStreamWaitEvent(s, ev_far, 0);  // the last far update before the Q accumulation
+    // the last far update and the last V T before the Q accumulation
+    e = cudaEventRecord(ev_far, far);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev_far, 0);
     if (e != cudaSuccess) return e;
   }
 
@@ -836,8 +874,7 @@ cudaError_t qr_q(int n, int batch, const float* P, float* Q, uint8_t* skip, floa
   // At = P^T and its lo part
   cudaError_t e = transpose(P, w.At, n, n, batch, s);
   if (e != cudaSuccess) return e;
-  return qr_q_t(n, batch, nullptr, nullptr, Q, nullptr, skip, tol, workspace, workspace_bytes, status, s, nullptr,
-                nullptr, nullptr);
+  return qr_q_t(n, batch, nullptr, nullptr, Q, nullptr, skip, tol, workspace, workspace_bytes, status, s, nullptr);
 }
 
 }  // namespace soap

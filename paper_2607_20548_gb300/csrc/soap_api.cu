@@ -85,7 +85,7 @@ struct QrGroup {
   uint8_t* skip = nullptr;  // [batch][n]
   cudaStream_t stream = nullptr;  // panels and the rows that gate them (high priority)
   cudaStream_t far = nullptr;     // the rest of each block's trailing update (low priority)
-  cudaEvent_t ev_vt = nullptr, ev_far = nullptr;
+  cudaEvent_t ev_vt = nullptr, ev_far = nullptr, ev_vq[2] = {nullptr, nullptr};
   cudaEvent_t done = nullptr;
 };
 
@@ -191,6 +191,10 @@ void free_all(soap_handle h) {
     if (g.done) cudaEventDestroy(g.done);
     if (g.ev_vt) cudaEventDestroy(g.ev_vt);
     if (g.ev_far) cudaEventDestroy(g.ev_far);
+    for (cudaEvent_t& ev : g.ev_vq) {
+      if (ev) cudaEventDestroy(ev);
+      ev = nullptr;
+    }
     g.stream = g.far = nullptr;
     g.done = g.ev_vt = g.ev_far = nullptr;
   }
@@ -326,8 +330,9 @@ soap_status_t refresh_bases(soap_handle h, cudaStream_t s) {
       }
     }
     // the Q accumulation ends with Q^T and its lo part in the input buffers
+    const soap::QrLookahead la{g.far, g.ev_vt, g.ev_far, {g.ev_vq[0], g.ev_vq[1]}};
     SOAP_CUDA(h, soap::qr_q_t(n, g.batch, nullptr, nullptr, nullptr, nullptr, g.skip, hp.qr_tol, g.ws, g.ws_bytes,
-                              h->d_status, gs, g.far, g.ev_vt, g.ev_far));
+                              h->d_status, gs, &la));
     for (const QrJob& j : g.jobs) {
       ClassState& c = h->classes[j.cls];
       const float* qt = At + (int64_t)j.offset * nn;
@@ -612,6 +617,8 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
       if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.done, cudaEventDisableTiming);
       if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.ev_vt, cudaEventDisableTiming);
       if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.ev_far, cudaEventDisableTiming);
+      for (cudaEvent_t& ev : g.ev_vq)
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
     }
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->fork_ev, cudaEventDisableTiming);
   }

@@ -91,13 +91,19 @@ void qr_input_buffers(void* workspace, int n, int batch, float** At);
 // QR of P whose transpose is already in qr_input_buffers(). Writes Q^T into Qt (or, if Qt is
 // nullptr, into the workspace) and, if Q is given, Q and (if Q_lo is given) its lo part.
 // Qt_lo is not written.
-// With `far`, ev_vt and ev_far (and a workspace sized with lookahead) the trailing update of
-// each 128-column block, except the next block's rows, runs on `far` and overlaps the next
-// block's panels; everything is joined back on `stream` before return.
+// The look-ahead schedule of qr_q_t: a second (low-priority) stream and its events.
+struct QrLookahead {
+  cudaStream_t far;     // trailing updates beyond the next block, and V T for the Q accumulation
+  cudaEvent_t vt;       // this block's V T^T is ready (recorded on the caller's stream)
+  cudaEvent_t far_done; // the far update of the previous block is done (recorded on `far`)
+  cudaEvent_t vq[2];    // V T of the block using buffer 0 / 1 is done (recorded on `far`)
+};
+// With `la` (all members set, and a workspace sized with lookahead) the trailing update of each
+// 128-column block, except the next block's rows, and the block's V T run on la->far and
+// overlap the next block's panels; everything is joined back on `stream` before return.
 cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q_lo, uint8_t* skip,
                    float tol, void* workspace, size_t workspace_bytes, int* status,
-                   cudaStream_t stream, cudaStream_t far = nullptr, cudaEvent_t ev_vt = nullptr,
-                   cudaEvent_t ev_far = nullptr);
+                   cudaStream_t stream, const QrLookahead* la = nullptr);
 
 // Elementwise kernels of the step.
 // M_hat <- b1 M_hat + (1-b1) G and Gc <- G for each matrix of a class.
