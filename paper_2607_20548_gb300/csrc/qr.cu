@@ -112,6 +112,8 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   __shared__ float s_pv[2][NB];          // rank 0: pivot-row values [alpha | a_c,pivot]
   __shared__ float s_scal[2];            // tau and 1 / v0 of the current reflector
   __shared__ float s_w[NB];              // v^T a_c
+  __shared__ __align__(16) float s_wl[NB];  // v^T a_(j+l) by offset l from the current row j
+  __shared__ float s_red[NWARP][NB];     // per-warp partial sums of the register path
   __shared__ float s_tau[NB];
   __shared__ int s_skip[NB];
   __shared__ float s_dsign[NB];
@@ -150,29 +152,61 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   const float thresh = p.thresh[b];
   int nonfinite = 0;
 
-  for (int j = 0; j < kb; ++j) {
-    const int par = j & 1;
-    // positions strictly after the pivot (pivot = local position j of rank 0)
-    const int ibeg = (c == 0) ? j + 1 : 0;
-    // partial sums over this CTA: sigma (cc = j) and x . a_cc (cc > j), kept locally; after
-    // the cluster barrier the threads that need them read every CTA's copy
-    for (int cc = j + warp; cc < kb; cc += NWARP) {
-      float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
-      int i = ibeg + lane;
-      for (; i + 96 < npos; i += 128) {
-        d0 = fmaf(sA[j * LDS + i], sA[cc * LDS + i], d0);
-        d1 = fmaf(sA[j * LDS + i + 32], sA[cc * LDS + i + 32], d1);
-        d2 = fmaf(sA[j * LDS + i + 64], sA[cc * LDS + i + 64], d2);
-        d3 = fmaf(sA[j * LDS + i + 96], sA[cc * LDS + i + 96], d3);
+  if constexpr (COLS == PT) {
+    // One position per thread: thread tid holds the panel rows' values at position tid in
+    // registers, the current row first (a[l] = row j + l; rows past the panel are zero), so
+    // that the per-column dot products and the reflector's update never touch shared memory;
+    // only v (row j) is written back, for the phases after the loop.
+    const int i = tid;
+    const bool have = i < npos;
+    float a[NB];
+#pragma unroll
+    for (int l = 0; l < NB; ++l) a[l] = (have && l < kb) ? sA[l * LDS + i] : 0.f;
+    for (int j = 0; j < kb; ++j) {
+      const int par = j & 1;
+      // this position's share of sigma (l = 0) and of x . a_(j+l) (l > 0), for positions
+      // strictly after the pivot (pivot = local position j of rank 0)
+      const float x = (have && (c != 0 || i > j)) ? a[0] : 0.f;
+      float v[NB];
+#pragma unroll
+      for (int l = 0; l < NB; ++l) v[l] = x * a[l];
+      // transposing butterfly over the warp: lane l ends with the warp's sum for row j + l
+#define SOAP_BFLY(o, nh)                                                   \
+  {                                                                        \
+    const bool up = (lane & (o)) != 0;                                     \
+    _Pragma("unroll") for (int q = 0; q < (nh); ++q) {                     \
+      const float keep = up ? v[q + (nh)] : v[q];                          \
+      const float send = up ? v[q] : v[q + (nh)];                          \
+      v[q] = keep + __shfl_xor_sync(0xffffffffu, send, (o));               \
+    }                                                                      \
+  }
+      SOAP_BFLY(16, 16)
+      SOAP_BFLY(8, 8)
+      SOAP_BFLY(4, 4)
+      SOAP_BFLY(2, 2)
+      SOAP_BFLY(1, 1)
+#undef SOAP_BFLY
+      s_red[warp][lane] = v[0];
+      // rank 0's pivot position: alpha and the later rows' values there
+      if (c == 0 && i == j) {
+#pragma unroll
+        for (int l = 0; l < NB; ++l)
+          if (j + l < kb) s_pv[par][j + l] = a[l];
       }
-      for (; i < npos; i += 32) d0 = fmaf(sA[j * LDS + i], sA[cc * LDS + i], d0);
-      const float d = warp_sum((d0 + d1) + (d2 + d3));
-      if (lane == 0) s_part[par][cc] = d;
-    }
-    if (c == 0 && tid >= j && tid < kb) s_pv[par][tid] = sA[tid * LDS + j];  // alpha (tid == j), a_tid at the pivot
-    cluster.sync();
+      __syncthreads();
+      if (warp == 0) {
+        float sum = 0.f;
+#pragma unroll
+        for (int w = 0; w < NWARP; ++w) sum += s_red[w][lane];
+        if (j + lane < kb) s_part[par][j + lane] = sum;
+      }
+      cluster.sync();
     // threads j..kb-1 reduce sigma and their own column's sum (in the same fixed order, so
     // they all derive the same reflector) and form v^T a_tid
+    if (warp == 0) {
+      s_wl[lane] = 0.f;
+      __syncwarp();
+    }
     if (tid >= j && tid < kb) {
       float ps[MAXC], pd[MAXC];
 #pragma unroll
@@ -213,26 +247,151 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
         s_dsign[j] = rsign;
         s_scal[0] = tau;
         s_scal[1] = tau != 0.f ? 1.f / v0 : 0.f;
-      } else if (tau != 0.f) {
-        s_w[tid] = apiv + d / v0;  // v^T a_tid, with v = x / v0 after the pivot
+      } else {
+        s_wl[tid - j] = tau != 0.f ? apiv + d / v0 : 0.f;  // v^T a_tid, with v = x / v0 after the pivot
       }
     }
-    __syncthreads();
-    const float tau = s_scal[0], rv0 = s_scal[1];
+      __syncthreads();
+      const float tau = s_scal[0], rv0 = s_scal[1];
+      // v at this position (x / v0 after the pivot, 1 at it) and H_j = I - tau v v^T on the
+      // later rows, shifting them down one register; positions before the pivot only shift
+      if (have && (c != 0 || i >= j)) {
+        const bool at_pivot = (c == 0 && i == j);
+        const float vi = at_pivot ? 1.f : a[0] * rv0;
+        if (!at_pivot) sA[j * LDS + i] = vi;
+        if (tau != 0.f) {
+          const float tv = tau * vi;
+#pragma unroll
+          for (int l4 = 0; l4 < NB / 4; ++l4) {
+            const float4 w4 = reinterpret_cast<const float4*>(s_wl)[l4];
+            if (l4 > 0) a[4 * l4 - 1] = fmaf(-tv, w4.x, a[4 * l4]);
+            a[4 * l4] = fmaf(-tv, w4.y, a[4 * l4 + 1]);
+            a[4 * l4 + 1] = fmaf(-tv, w4.z, a[4 * l4 + 2]);
+            a[4 * l4 + 2] = fmaf(-tv, w4.w, a[4 * l4 + 3]);
+          }
+          a[NB - 1] = 0.f;
+        } else {
+#pragma unroll
+          for (int l = 0; l < NB - 1; ++l) a[l] = a[l + 1];
+          a[NB - 1] = 0.f;
+        }
+      } else {
+#pragma unroll
+        for (int l = 0; l < NB - 1; ++l) a[l] = a[l + 1];
+        a[NB - 1] = 0.f;
+      }
+      __syncthreads();  // s_wl, s_red and s_scal are rewritten by the next column
+    }
+  } else {
+    for (int j = 0; j < kb; ++j) {
+      const int par = j & 1;
+      // positions strictly after the pivot (pivot = local position j of rank 0)
+      const int ibeg = (c == 0) ? j + 1 : 0;
+      // partial sums over this CTA: sigma (cc = j) and x . a_cc (cc > j), kept locally; after
+      // the cluster barrier the threads that need them read every CTA's copy. Warp w takes
+      // columns j + w and j + w + 16 in one pass over x (kb - j <= 32 columns).
+      {
+        const int c1 = j + warp, c2 = c1 + NWARP;
+        if (c1 < kb) {
+          const bool h2 = c2 < kb;
+          float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f, b0 = 0.f, b1 = 0.f, b2 = 0.f, b3 = 0.f;
+          const float* xr = sA + j * LDS;
+          const float* r1 = sA + c1 * LDS;
+          const float* r2 = sA + (h2 ? c2 : c1) * LDS;
+          int i = ibeg + lane;
+          for (; i + 96 < npos; i += 128) {
+            const float x0 = xr[i], x1 = xr[i + 32], x2 = xr[i + 64], x3 = xr[i + 96];
+            a0 = fmaf(x0, r1[i], a0);
+            a1 = fmaf(x1, r1[i + 32], a1);
+            a2 = fmaf(x2, r1[i + 64], a2);
+            a3 = fmaf(x3, r1[i + 96], a3);
+            b0 = fmaf(x0, r2[i], b0);
+            b1 = fmaf(x1, r2[i + 32], b1);
+            b2 = fmaf(x2, r2[i + 64], b2);
+            b3 = fmaf(x3, r2[i + 96], b3);
+          }
+          for (; i < npos; i += 32) {
+            const float x0 = xr[i];
+            a0 = fmaf(x0, r1[i], a0);
+            b0 = fmaf(x0, r2[i], b0);
+          }
+          float da = (a0 + a1) + (a2 + a3), db = (b0 + b1) + (b2 + b3);
+  #pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+            da += __shfl_xor_sync(0xffffffffu, da, o);
+            db += __shfl_xor_sync(0xffffffffu, db, o);
+          }
+          if (lane == 0) {
+            s_part[par][c1] = da;
+            if (h2) s_part[par][c2] = db;
+          }
+        }
+      }
+      if (c == 0 && tid >= j && tid < kb) s_pv[par][tid] = sA[tid * LDS + j];  // alpha (tid == j), a_tid at the pivot
+      cluster.sync();
+      // threads j..kb-1 reduce sigma and their own column's sum (in the same fixed order, so
+      // they all derive the same reflector) and form v^T a_tid
+      if (tid >= j && tid < kb) {
+        float ps[MAXC], pd[MAXC];
+  #pragma unroll
+        for (int q = 0; q < MAXC; ++q) {
+          if (q < C) {
+            const float* rp = cluster.map_shared_rank(&s_part[par][0], q);
+            ps[q] = rp[j];
+            pd[q] = rp[tid];
+          }
+        }
+        const float* pv0 = cluster.map_shared_rank(&s_pv[par][0], 0);
+        const float alpha = pv0[j], apiv = pv0[tid];
+        float d = 0.f, sigma = 0.f;
+  #pragma unroll
+        for (int q = 0; q < MAXC; ++q) {
+          if (q < C) {
+            sigma += ps[q];
+            d += pd[q];
+          }
+        }
+        const float xnorm = sqrtf(fmaf(alpha, alpha, sigma));
+        const bool skip = !(xnorm > thresh);
+        float tau = 0.f, v0 = 1.f, rsign = 1.f;
+        if (!skip) {
+          if (sigma == 0.f) {
+            rsign = alpha < 0.f ? -1.f : 1.f;   // H = I, R_pp = alpha
+          } else {
+            const float beta = alpha >= 0.f ? -xnorm : xnorm;
+            v0 = alpha - beta;                   // same sign as alpha: no cancellation
+            tau = (beta - alpha) / beta;
+            rsign = beta < 0.f ? -1.f : 1.f;
+          }
+        }
+        if (tid == j) {
+          if (!isfinite(xnorm)) nonfinite = 1;
+          s_tau[j] = tau;
+          s_skip[j] = skip ? 1 : 0;
+          s_dsign[j] = rsign;
+          s_scal[0] = tau;
+          s_scal[1] = tau != 0.f ? 1.f / v0 : 0.f;
+        } else if (tau != 0.f) {
+          s_w[tid] = apiv + d / v0;  // v^T a_tid, with v = x / v0 after the pivot
+        }
+      }
+      __syncthreads();
+      const float tau = s_scal[0], rv0 = s_scal[1];
 
-    // v after the pivot (x / v0, or 0 where H = I), and H_j = I - tau v v^T on the later
-    // panel rows; every thread owns its positions
-    const int piv = (c == 0) ? j : 0;  // local positions >= this take part
-    for (int i = piv + tid; i < npos; i += PT) {
-      const bool at_pivot = (c == 0 && i == j);
-      const float vi = at_pivot ? 1.f : sA[j * LDS + i] * rv0;
-      if (!at_pivot) sA[j * LDS + i] = vi;
-      if (tau != 0.f) {
-        const float tv = tau * vi;
-        for (int cc = j + 1; cc < kb; ++cc) sA[cc * LDS + i] = fmaf(-tv, s_w[cc], sA[cc * LDS + i]);
+      // v after the pivot (x / v0, or 0 where H = I), and H_j = I - tau v v^T on the later
+      // panel rows; every thread owns its positions
+      const int piv = (c == 0) ? j : 0;  // local positions >= this take part
+      for (int i = piv + tid; i < npos; i += PT) {
+        const bool at_pivot = (c == 0 && i == j);
+        const float vi = at_pivot ? 1.f : sA[j * LDS + i] * rv0;
+        if (!at_pivot) sA[j * LDS + i] = vi;
+        if (tau != 0.f) {
+          const float tv = tau * vi;
+          for (int cc = j + 1; cc < kb; ++cc) sA[cc * LDS + i] = fmaf(-tv, s_w[cc], sA[cc * LDS + i]);
+        }
       }
+      __syncthreads();
     }
-    __syncthreads();
   }
   if (nonfinite) atomicOr(p.status, kStatusQrBreakdown);
 
@@ -252,13 +411,14 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   float* Vt_lo = p.Vt_lo + (int64_t)b * nn;
   float* Vpos = p.Vpos + (int64_t)b * n * NBO;
   float* Vpos_lo = p.Vpos_lo + (int64_t)b * n * NBO;
-  for (int jj = 0; jj < kb; ++jj) {
-    float* vt = Vt + (int64_t)(k + jj) * n + pos0;
-    float* vl = Vt_lo + (int64_t)(k + jj) * n + pos0;
-    for (int q = tid; q < npos / 4; q += PT) {
+  {
+    const int q4n = npos / 4;
+    for (int e = tid; e < kb * q4n; e += PT) {
+      const int jj = e / q4n, q = e - jj * q4n;
+      const int64_t o = (int64_t)(k + jj) * n + pos0 + 4 * q;
       const float4 v = *reinterpret_cast<const float4*>(&sA[jj * LDS + 4 * q]);
-      reinterpret_cast<float4*>(vt)[q] = v;
-      reinterpret_cast<float4*>(vl)[q] = make_float4(tf32_lo(v.x), tf32_lo(v.y), tf32_lo(v.z), tf32_lo(v.w));
+      *reinterpret_cast<float4*>(Vt + o) = v;
+      *reinterpret_cast<float4*>(Vt_lo + o) = make_float4(tf32_lo(v.x), tf32_lo(v.y), tf32_lo(v.z), tf32_lo(v.w));
     }
   }
   for (int e = tid; e < npos * (NB / 4); e += PT) {
@@ -356,22 +516,19 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     __syncthreads();
     // T of the panel from its Gram matrix g (rows jb.. of Y): T^-1 = diag(1/tau) + striu(g)
     // (H_1 ... H_kb = I - V T V^T); a reflector with tau = 0 (v = 0) gets a zero row and column.
-    // Thread cc solves for column cc by back substitution (fully unrolled, in registers).
-    if (tid < NB) {
-      const int cc = tid;
-      float x[NB];
-#pragma unroll
-      for (int i = NB - 1; i >= 0; --i) {
-        float acc = (i == cc) ? 1.f : 0.f;
-#pragma unroll
-        for (int l = i + 1; l < NB; ++l)
-          if (l <= cc) acc = fmaf(-s_Y[jb + i][l], x[l], acc);
-        const float ti = i < kb ? s_tau[i] : 0.f;
-        x[i] = (i <= cc) ? acc * (ti != 0.f ? ti : 1.f) : 0.f;
+    // Warp w solves columns w and w + 16 by back substitution, lane l holding x_l:
+    //   x_i = tau_i (delta_{i,cc} - sum_{i < l <= cc} g_il x_l)   (tau_i read as 1 where it is 0)
+    for (int cc = warp; cc < NB; cc += NWARP) {
+      float x = 0.f;
+      for (int i = cc; i >= 0; --i) {
+        const float part = warp_sum((lane > i && lane <= cc) ? s_Y[jb + i][lane] * x : 0.f);
+        if (lane == i) {
+          const float ti = i < kb ? s_tau[i] : 0.f;
+          x = ((i == cc ? 1.f : 0.f) - part) * (ti != 0.f ? ti : 1.f);
+        }
       }
       const bool live = cc < kb && s_tau[cc] != 0.f;
-#pragma unroll
-      for (int i = 0; i < NB; ++i) s_T[i][cc] = (live && i < kb && s_tau[i] != 0.f) ? x[i] : 0.f;
+      s_T[lane][cc] = (live && lane <= cc && lane < kb && s_tau[lane] != 0.f) ? x : 0.f;
     }
     __syncthreads();
     // U = X T_panel with X = V_before^T V_panel (rows 0..jb-1 of Y), in place, and
