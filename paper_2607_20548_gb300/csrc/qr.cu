@@ -89,6 +89,21 @@ struct PanelArgs {
   int n, k0, kbo, k, kb;  // block start and width, panel start and width
 };
 
+// x = hi + lo with hi = tf32(x) rounded to nearest and lo = tf32(x - hi): both as tf32 bits
+__device__ __forceinline__ void tf32_split(float x, uint32_t& hi, uint32_t& lo) {
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(hi) : "f"(x));
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(lo) : "f"(x - __uint_as_float(hi)));
+}
+
+// d += a b for a 16 x 8 (rows) tf32 A fragment and an 8 x 8 (columns) B fragment, fp32 d
+__device__ __forceinline__ void mma_tf32_16x8x8(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -120,12 +135,9 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   __shared__ float s_T[NB][NB + 1];
   __shared__ float s_Y[NBO][NB + 1];     // rank 0: S V_panel summed over the cluster
   __shared__ __align__(16) float s_Z[NREST][NB];  // (S_rest V_panel) T_panel, the in-block update
-  // staging of S (STG chunks of 128 x 32) while Y is formed; afterwards rank 0's copy of the
-  // block's T so far (96 x 97)
+  // staging of S (STG chunks of 128 x 36) while Y is formed
   constexpr int STG = COLS <= 512 ? 4 : 2;
-  constexpr int SCRATCH = STG * NBO * 32 > NREST * (NREST + 1) ? STG * NBO * 32 : NREST * (NREST + 1);
-  __shared__ __align__(16) float s_scratch[SCRATCH];
-  float (*s_Tb)[NREST + 1] = reinterpret_cast<float (*)[NREST + 1]>(s_scratch);
+  __shared__ __align__(16) float s_scratch[STG * NBO * 36];
 
   const int n = p.n, k = p.k, kb = p.kb, k0 = p.k0, kbo = p.kbo;
   const int jb = k - k0;                // panel offset inside its block
@@ -201,56 +213,56 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
         if (j + lane < kb) s_part[par][j + lane] = sum;
       }
       cluster.sync();
-    // threads j..kb-1 reduce sigma and their own column's sum (in the same fixed order, so
-    // they all derive the same reflector) and form v^T a_tid
-    if (warp == 0) {
-      s_wl[lane] = 0.f;
-      __syncwarp();
-    }
-    if (tid >= j && tid < kb) {
-      float ps[MAXC], pd[MAXC];
-#pragma unroll
-      for (int q = 0; q < MAXC; ++q) {
-        if (q < C) {
-          const float* rp = cluster.map_shared_rank(&s_part[par][0], q);
-          ps[q] = rp[j];
-          pd[q] = rp[tid];
-        }
+      // threads j..kb-1 reduce sigma and their own column's sum (in the same fixed order, so
+      // they all derive the same reflector) and form v^T a_tid
+      if (warp == 0) {
+        s_wl[lane] = 0.f;
+        __syncwarp();
       }
-      const float* pv0 = cluster.map_shared_rank(&s_pv[par][0], 0);
-      const float alpha = pv0[j], apiv = pv0[tid];
-      float d = 0.f, sigma = 0.f;
+      if (tid >= j && tid < kb) {
+        float ps[MAXC], pd[MAXC];
 #pragma unroll
-      for (int q = 0; q < MAXC; ++q) {
-        if (q < C) {
-          sigma += ps[q];
-          d += pd[q];
+        for (int q = 0; q < MAXC; ++q) {
+          if (q < C) {
+            const float* rp = cluster.map_shared_rank(&s_part[par][0], q);
+            ps[q] = rp[j];
+            pd[q] = rp[tid];
+          }
         }
-      }
-      const float xnorm = sqrtf(fmaf(alpha, alpha, sigma));
-      const bool skip = !(xnorm > thresh);
-      float tau = 0.f, v0 = 1.f, rsign = 1.f;
-      if (!skip) {
-        if (sigma == 0.f) {
-          rsign = alpha < 0.f ? -1.f : 1.f;   // H = I, R_pp = alpha
+        const float* pv0 = cluster.map_shared_rank(&s_pv[par][0], 0);
+        const float alpha = pv0[j], apiv = pv0[tid];
+        float d = 0.f, sigma = 0.f;
+#pragma unroll
+        for (int q = 0; q < MAXC; ++q) {
+          if (q < C) {
+            sigma += ps[q];
+            d += pd[q];
+          }
+        }
+        const float xnorm = sqrtf(fmaf(alpha, alpha, sigma));
+        const bool skip = !(xnorm > thresh);
+        float tau = 0.f, v0 = 1.f, rsign = 1.f;
+        if (!skip) {
+          if (sigma == 0.f) {
+            rsign = alpha < 0.f ? -1.f : 1.f;   // H = I, R_pp = alpha
+          } else {
+            const float beta = alpha >= 0.f ? -xnorm : xnorm;
+            v0 = alpha - beta;                   // same sign as alpha: no cancellation
+            tau = (beta - alpha) / beta;
+            rsign = beta < 0.f ? -1.f : 1.f;
+          }
+        }
+        if (tid == j) {
+          if (!isfinite(xnorm)) nonfinite = 1;
+          s_tau[j] = tau;
+          s_skip[j] = skip ? 1 : 0;
+          s_dsign[j] = rsign;
+          s_scal[0] = tau;
+          s_scal[1] = tau != 0.f ? 1.f / v0 : 0.f;
         } else {
-          const float beta = alpha >= 0.f ? -xnorm : xnorm;
-          v0 = alpha - beta;                   // same sign as alpha: no cancellation
-          tau = (beta - alpha) / beta;
-          rsign = beta < 0.f ? -1.f : 1.f;
+          s_wl[tid - j] = tau != 0.f ? apiv + d / v0 : 0.f;  // v^T a_tid, with v = x / v0 after the pivot
         }
       }
-      if (tid == j) {
-        if (!isfinite(xnorm)) nonfinite = 1;
-        s_tau[j] = tau;
-        s_skip[j] = skip ? 1 : 0;
-        s_dsign[j] = rsign;
-        s_scal[0] = tau;
-        s_scal[1] = tau != 0.f ? 1.f / v0 : 0.f;
-      } else {
-        s_wl[tid - j] = tau != 0.f ? apiv + d / v0 : 0.f;  // v^T a_tid, with v = x / v0 after the pivot
-      }
-    }
       __syncthreads();
       const float tau = s_scal[0], rv0 = s_scal[1];
       // v at this position (x / v0 after the pivot, 1 at it) and H_j = I - tau v v^T on the
@@ -316,7 +328,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
             b0 = fmaf(x0, r2[i], b0);
           }
           float da = (a0 + a1) + (a2 + a3), db = (b0 + b1) + (b2 + b3);
-  #pragma unroll
+#pragma unroll
           for (int o = 16; o > 0; o >>= 1) {
             da += __shfl_xor_sync(0xffffffffu, da, o);
             db += __shfl_xor_sync(0xffffffffu, db, o);
@@ -333,7 +345,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       // they all derive the same reflector) and form v^T a_tid
       if (tid >= j && tid < kb) {
         float ps[MAXC], pd[MAXC];
-  #pragma unroll
+#pragma unroll
         for (int q = 0; q < MAXC; ++q) {
           if (q < C) {
             const float* rp = cluster.map_shared_rank(&s_part[par][0], q);
@@ -344,7 +356,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
         const float* pv0 = cluster.map_shared_rank(&s_pv[par][0], 0);
         const float alpha = pv0[j], apiv = pv0[tid];
         float d = 0.f, sigma = 0.f;
-  #pragma unroll
+#pragma unroll
         for (int q = 0; q < MAXC; ++q) {
           if (q < C) {
             sigma += ps[q];
@@ -446,23 +458,29 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   // Y = S V_panel over this CTA's positions, S = the block's rows k0 .. k0+kbo-1: the block's
   // Householder vectors so far (rows before the panel's end, from Vt) and the block rows
   // still to be factored (from At). S is streamed through shared memory in 32-position
-  // chunks (cp.async, double-buffered); warp w takes rows w, w+16, ...; lane jj column jj.
+  // chunks (cp.async, STG buffers, rows padded to 36 floats), and the product runs on the
+  // tensor cores as warp-level m16n8k8 TF32 MMAs with both operands split into tf32 hi and lo
+  // parts (four products: fp32 accuracy). Warp w owns rows 16 (w mod 8) .. +15 and columns
+  // 16 (w / 8) .. +15; each chunk is accumulated afresh and added to fp32 registers, so the
+  // tensor core's own accumulation never runs longer than 32 positions.
   {
-    constexpr int RW = NBO / NWARP;
-    constexpr int CH = 32;  // positions per chunk
-    float y[RW];
+    static_assert(NBO == 128 && NB == 32 && NWARP == 16, "8 x 2 warp tiles of 16 x 16");
+    constexpr int CH = 32;       // positions per chunk
+    constexpr int CHP = CH + 4;  // padded row stride of a staged chunk
+    const int gq = lane >> 2, tg = lane & 3;
+    const int m0 = 16 * (warp & 7), nb = 16 * (warp >> 3);
+    float y[2][4];
 #pragma unroll
-    for (int u = 0; u < RW; ++u) y[u] = 0.f;
-    const int nr = (kbo - warp + NWARP - 1) / NWARP;  // rows of this warp
+    for (int e = 0; e < 4; ++e) y[0][e] = y[1][e] = 0.f;
     const int nchunk = (npos + CH - 1) / CH;
     auto issue = [&](int ch, int buf) {
-      float* dst = s_scratch + buf * NBO * CH;
+      float* dst = s_scratch + buf * NBO * CHP;
       for (int e = tid; e < NBO * (CH / 4); e += PT) {
         const int r = e / (CH / 4), q4 = e % (CH / 4);
         const int row = k0 + r, i = ch * CH + 4 * q4;
         const bool ok = r < kbo && i < npos;
         const float* src = ok ? ((row < k + kb) ? Vt : At) + (int64_t)row * n + pos0 + i : At;
-        const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst + r * CH + 4 * q4));
+        const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst + r * CHP + 4 * q4));
         asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(ok ? 16 : 0) : "memory");
       }
       asm volatile("cp.async.commit_group;" ::: "memory");
@@ -476,31 +494,56 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       else asm volatile("cp.async.commit_group;" ::: "memory");  // keeps the group count uniform
       asm volatile("cp.async.wait_group %0;" ::"n"(STG - 1) : "memory");
       __syncthreads();
-      const float* st = s_scratch + (ch % STG) * NBO * CH;
+      const float* st = s_scratch + (ch % STG) * NBO * CHP;
       const int i0 = ch * CH;
+      float d[2][4];
 #pragma unroll
-      for (int q4 = 0; q4 < CH / 4; ++q4) {
-        // positions past npos are zero in the staged chunk (zero-filled copies)
-        const float4 v = *reinterpret_cast<const float4*>(&sA[lane * LDS + i0 + 4 * q4]);
+      for (int e = 0; e < 4; ++e) d[0][e] = d[1][e] = 0.f;
 #pragma unroll
-        for (int u = 0; u < RW; ++u) {
-          if (u < nr) {
-            const float4 x = *reinterpret_cast<const float4*>(st + (warp + NWARP * u) * CH + 4 * q4);
-            y[u] = fmaf(x.w, v.w, fmaf(x.z, v.z, fmaf(x.y, v.y, fmaf(x.x, v.x, y[u]))));
-          }
+      for (int ks = 0; ks < CH / 8; ++ks) {
+        // positions past npos are zero in the staged chunk and in V (zero-filled copies)
+        const int kk = 8 * ks;
+        const float av[4] = {st[(m0 + gq) * CHP + kk + tg], st[(m0 + gq + 8) * CHP + kk + tg],
+                             st[(m0 + gq) * CHP + kk + tg + 4], st[(m0 + gq + 8) * CHP + kk + tg + 4]};
+        uint32_t ah[4], al[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) tf32_split(av[e], ah[e], al[e]);
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt) {
+          const float* vr = sA + (nb + 8 * nt + gq) * LDS + i0 + kk + tg;
+          uint32_t bh[2], bl[2];
+          tf32_split(vr[0], bh[0], bl[0]);
+          tf32_split(vr[4], bh[1], bl[1]);
+          mma_tf32_16x8x8(d[nt], al, bl);
+          mma_tf32_16x8x8(d[nt], al, bh);
+          mma_tf32_16x8x8(d[nt], ah, bl);
+          mma_tf32_16x8x8(d[nt], ah, bh);
         }
       }
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) y[nt][e] += d[nt][e];
       __syncthreads();  // this buffer is refilled STG - 1 chunks later
     }
     float* yp = p.Ypart + ((int64_t)b * MAXC + c) * NBO * NB;
 #pragma unroll
-    for (int u = 0; u < RW; ++u)
-      if (u < nr) yp[(warp + NWARP * u) * NB + lane] = y[u];
+    for (int nt = 0; nt < 2; ++nt) {
+      const int col = nb + 8 * nt + 2 * tg;
+      *reinterpret_cast<float2*>(yp + (m0 + gq) * NB + col) = make_float2(y[nt][0], y[nt][1]);
+      *reinterpret_cast<float2*>(yp + (m0 + gq + 8) * NB + col) = make_float2(y[nt][2], y[nt][3]);
+    }
   }
   cluster.sync();  // orders the partials in global memory before rank 0 reads them
 
+  // rank 0 sums the partials, forms T_panel, U = X T_panel and Z, and hands Z, U and T_panel
+  // to the cluster through global memory (rank 0's slots of Ypart, free once it has summed
+  // them): Z at 0, U at 3072 (jb <= 96 rows), T_panel at 6144 floats
+  float* xg = p.Ypart + (int64_t)b * MAXC * NBO * NB;
+  float* Ug = xg + NREST * NB;
+  float* Tpg = xg + 2 * NREST * NB;
   if (c == 0) {
-    // sum the partials in a fixed order; stage the block's T so far
+    // sum the partials in a fixed order
     const float* yp = p.Ypart + (int64_t)b * MAXC * NBO * NB;
     for (int e = tid; e < kbo * NB; e += PT) {
       float part[MAXC];
@@ -511,8 +554,6 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       for (int q = 0; q < MAXC; ++q) sum += part[q];
       s_Y[e / NB][e % NB] = sum;
     }
-    const float* Tg = p.T + (int64_t)b * NBO * NBO;
-    for (int e = tid; e < jb * jb; e += PT) s_Tb[e / jb][e % jb] = Tg[(e / jb) * NBO + e % jb];
     __syncthreads();
     // T of the panel from its Gram matrix g (rows jb.. of Y): T^-1 = diag(1/tau) + striu(g)
     // (H_1 ... H_kb = I - V T V^T); a reflector with tau = 0 (v = 0) gets a zero row and column.
@@ -555,20 +596,37 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       }
     }
     __syncthreads();
-    // the block's T: column block jb = [-T_before U ; T_panel ; 0], row block jb left of it = 0;
-    // thread (r, g) writes columns jb + 8g .. jb + 8g+7 of row r
+    for (int e = tid; e < nrest * NB; e += PT) xg[e] = s_Z[e / NB][e % NB];
+    for (int e = tid; e < jb * NB; e += PT) Ug[e] = s_Y[e / NB][e % NB];
+    for (int e = tid; e < NB * NB; e += PT) Tpg[e] = s_T[e / NB][e % NB];
+    if (tid < kb) {
+      p.skip[(int64_t)b * n + k + tid] = (uint8_t)s_skip[tid];
+      p.dsign[(int64_t)b * n + k + tid] = s_dsign[tid];
+    }
+  }
+  cluster.sync();  // Z, U and T_panel in global memory are visible to the cluster
+  if (c != 0) {
+    for (int e = tid; e < nrest * NB; e += PT) s_Z[e / NB][e % NB] = xg[e];
+    for (int e = tid; e < jb * NB; e += PT) s_Y[e / NB][e % NB] = Ug[e];
+    for (int e = tid; e < NB * NB; e += PT) s_T[e / NB][e % NB] = Tpg[e];
+  }
+  __syncthreads();
+  // the block's T, rows spread over the cluster (row r by CTA r mod C): column block jb =
+  // [-T_before U ; T_panel ; 0] and the row block jb left of it = 0; thread (rl, g) writes
+  // columns jb + 8g .. jb + 8g+7 of row r = c + C rl
+  {
     float* T = p.T + (int64_t)b * NBO * NBO;
     float* T_lo = p.T_lo + (int64_t)b * NBO * NBO;
     float* Tt = p.Tt + (int64_t)b * NBO * NBO;
     float* Tt_lo = p.Tt_lo + (int64_t)b * NBO * NBO;
-    {
-      const int r = tid >> 2, g8 = (tid & 3) * 8;
+    const int r = c + C * (tid >> 2), g8 = (tid & 3) * 8;
+    if (r < NBO) {
       float t[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) t[u] = 0.f;
       if (r < jb) {
         for (int l = r; l < jb; ++l) {
-          const float tb = s_Tb[r][l];
+          const float tb = T[r * NBO + l];  // T_before, written by the block's earlier panels
 #pragma unroll
           for (int u = 0; u < 8; ++u) t[u] = fmaf(-tb, s_Y[l][g8 + u], t[u]);
         }
@@ -586,24 +644,14 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       }
     }
     for (int e = tid; e < NB * jb; e += PT) {
-      const int r = jb + e / jb, col = e % jb;
-      T[r * NBO + col] = 0.f;
-      T_lo[r * NBO + col] = 0.f;
-      Tt[col * NBO + r] = 0.f;
-      Tt_lo[col * NBO + r] = 0.f;
-    }
-    if (tid < kb) {
-      p.skip[(int64_t)b * n + k + tid] = (uint8_t)s_skip[tid];
-      p.dsign[(int64_t)b * n + k + tid] = s_dsign[tid];
+      const int rr = jb + e / jb, col = e % jb;
+      if (rr % C != c) continue;
+      T[rr * NBO + col] = 0.f;
+      T_lo[rr * NBO + col] = 0.f;
+      Tt[col * NBO + rr] = 0.f;
+      Tt_lo[col * NBO + rr] = 0.f;
     }
   }
-  cluster.sync();
-  // every CTA takes Z from rank 0
-  if (c != 0) {
-    const float4* z0 = reinterpret_cast<const float4*>(cluster.map_shared_rank(&s_Z[0][0], 0));
-    for (int e = tid; e < nrest * (NB / 4); e += PT) reinterpret_cast<float4*>(&s_Z[0][0])[e] = z0[e];
-  }
-  cluster.sync();  // rank 0's s_Z stays in place until every CTA has its copy
 
   // the panel's reflectors on the block rows after it: a_r -= Z_r V^T at this CTA's
   // positions, four rows at a time

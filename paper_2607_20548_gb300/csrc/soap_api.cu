@@ -87,6 +87,7 @@ struct QrGroup {
   cudaStream_t far = nullptr;     // the rest of each block's trailing update (low priority)
   cudaEvent_t ev_vt = nullptr, ev_far = nullptr, ev_vq[2] = {nullptr, nullptr};
   cudaEvent_t done = nullptr;
+  cudaEvent_t fork = nullptr;  // recorded on the caller's stream once the group's inputs are ready
 };
 
 struct DeviceGuard {
@@ -122,7 +123,10 @@ struct soap_s {
   float* Zt_lo = nullptr;
   float* lam_ws = nullptr;  // Q^T F of the KL form's eigenvalue estimate (two-sided classes)
   std::vector<QrGroup> groups;  // largest n first
-  cudaEvent_t fork_ev = nullptr;
+  std::vector<int> prep_order;               // classes, largest factor first
+  std::vector<int> update_order;             // classes, smallest largest-factor first
+  std::vector<std::vector<int>> fork_after;  // per class: groups whose last feeding class it is
+  std::vector<std::vector<int>> groups_of;   // per class: the groups its bases come from
   int* d_status = nullptr;
   int* h_status = nullptr;          // pinned mirror, refreshed after every step
   cudaEvent_t status_ev = nullptr;
@@ -183,12 +187,12 @@ void free_all(soap_handle h) {
   if (h->h_ptrs) cudaFreeHost(h->h_ptrs);
   if (h->status_ev) cudaEventDestroy(h->status_ev);
   if (h->stage_ev) cudaEventDestroy(h->stage_ev);
-  if (h->fork_ev) cudaEventDestroy(h->fork_ev);
-  h->fork_ev = nullptr;
   for (auto& g : h->groups) {
     if (g.stream) cudaStreamDestroy(g.stream);
     if (g.far) cudaStreamDestroy(g.far);
     if (g.done) cudaEventDestroy(g.done);
+    if (g.fork) cudaEventDestroy(g.fork);
+    g.fork = nullptr;
     if (g.ev_vt) cudaEventDestroy(g.ev_vt);
     if (g.ev_far) cudaEventDestroy(g.ev_far);
     for (cudaEvent_t& ev : g.ev_vq) {
@@ -300,17 +304,18 @@ soap_status_t prepare_class(soap_handle h, ClassState& c, const float* const* d_
   return SOAP_OK;
 }
 
-// S2 + S3 for every preconditioned side: per size group, P^T = Q^T F for each member (F the
+// S2 + S3 for the preconditioned sides of one size group: P^T = Q^T F for each member (F the
 // factor, symmetric) into one batched input, one QR, then Q^T, Q (and lo parts) and the
-// zero-column flags back to the classes. Groups run concurrently on their own streams.
-soap_status_t refresh_bases(soap_handle h, cudaStream_t s) {
+// zero-column flags back to the classes. The group runs on its own stream from the moment
+// its members' factors are updated on the caller's stream, concurrently with other groups.
+soap_status_t refresh_group(soap_handle h, QrGroup& g, cudaStream_t s) {
   const soap_hparams& hp = h->hp;
   using soap::strided;
   using soap::strided_mut;
-  SOAP_CUDA(h, cudaEventRecord(h->fork_ev, s));
-  for (auto& g : h->groups) {
+  SOAP_CUDA(h, cudaEventRecord(g.fork, s));
+  {
     cudaStream_t gs = g.stream;
-    SOAP_CUDA(h, cudaStreamWaitEvent(gs, h->fork_ev, 0));
+    SOAP_CUDA(h, cudaStreamWaitEvent(gs, g.fork, 0));
     const int n = g.n;
     const int64_t nn = (int64_t)n * n;
     float* At;
@@ -347,7 +352,6 @@ soap_status_t refresh_bases(soap_handle h, cudaStream_t s) {
     }
     SOAP_CUDA(h, cudaEventRecord(g.done, gs));
   }
-  for (auto& g : h->groups) SOAP_CUDA(h, cudaStreamWaitEvent(s, g.done, 0));
   return SOAP_OK;
 }
 
@@ -615,12 +619,36 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
       if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&g.stream, cudaStreamNonBlocking, prio_hi);
       if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&g.far, cudaStreamNonBlocking, prio_lo);
       if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.done, cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.fork, cudaEventDisableTiming);
       if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.ev_vt, cudaEventDisableTiming);
       if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.ev_far, cudaEventDisableTiming);
       for (cudaEvent_t& ev : g.ev_vq)
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
     }
-    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->fork_ev, cudaEventDisableTiming);
+    // step order: see soap_step
+    const int nc = (int)h->classes.size();
+    auto largest = [&](int ci) {
+      const ClassState& c = h->classes[ci];
+      return std::max(c.left ? c.rows : (int64_t)0, c.right ? c.cols : (int64_t)0);
+    };
+    h->prep_order.resize(nc);
+    for (int ci = 0; ci < nc; ++ci) h->prep_order[ci] = ci;
+    h->update_order = h->prep_order;
+    std::stable_sort(h->prep_order.begin(), h->prep_order.end(), [&](int x, int y) { return largest(x) > largest(y); });
+    std::stable_sort(h->update_order.begin(), h->update_order.end(),
+                     [&](int x, int y) { return largest(x) < largest(y); });
+    h->fork_after.assign(nc, {});
+    h->groups_of.assign(nc, {});
+    std::vector<int> pos(nc);
+    for (int q = 0; q < nc; ++q) pos[h->prep_order[q]] = q;
+    for (int gi = 0; gi < (int)h->groups.size(); ++gi) {
+      int last = -1;
+      for (const QrJob& j : h->groups[gi].jobs) {
+        h->groups_of[j.cls].push_back(gi);
+        if (last < 0 || pos[j.cls] > pos[last]) last = j.cls;
+      }
+      if (last >= 0) h->fork_after[last].push_back(gi);
+    }
   }
   h->nptrs = off;
   // workspaces: [G' | m'] for every class; N's lo part for tensor-core classes; the
@@ -746,18 +774,31 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
   auto grads_of = [&](const ClassState& c) {
     return reinterpret_cast<const float* const*>(h->d_ptrs + c.ptr_offset + c.count);
   };
-  for (auto& c : h->classes) {
-    soap_status_t st = prepare_class(h, c, grads_of(c), s);
+  // Phase A class by class, each size group's refresh forked as soon as the last class feeding
+  // it is prepared (classes with the largest factors first, so the longest refresh starts
+  // earliest); phase C class by class, each waiting only for the groups its bases come from
+  // (classes with the smallest factors first, whose refreshes finish earliest).
+  for (int ci : h->prep_order) {
+    soap_status_t st = prepare_class(h, h->classes[ci], grads_of(h->classes[ci]), s);
+    if (st != SOAP_OK) return st;
+    if (refresh)
+      for (int gi : h->fork_after[ci]) {
+        st = refresh_group(h, h->groups[gi], s);
+        if (st != SOAP_OK) return st;
+      }
+  }
+  std::vector<bool> joined(h->groups.size(), !refresh);
+  for (int ci : h->update_order) {
+    for (int gi : h->groups_of[ci])
+      if (!joined[gi]) {
+        SOAP_CUDA(h, cudaStreamWaitEvent(s, h->groups[gi].done, 0));
+        joined[gi] = true;
+      }
+    soap_status_t st = rotate_update_class(h, h->classes[ci], params_of(h->classes[ci]), bc1, bc2, s);
     if (st != SOAP_OK) return st;
   }
-  if (refresh) {
-    soap_status_t st = refresh_bases(h, s);
-    if (st != SOAP_OK) return st;
-  }
-  for (auto& c : h->classes) {
-    soap_status_t st = rotate_update_class(h, c, params_of(c), bc1, bc2, s);
-    if (st != SOAP_OK) return st;
-  }
+  for (size_t gi = 0; gi < h->groups.size(); ++gi)
+    if (!joined[gi]) SOAP_CUDA(h, cudaStreamWaitEvent(s, h->groups[gi].done, 0));
   SOAP_CUDA(h, cudaMemcpyAsync(h->h_status, h->d_status, sizeof(int), cudaMemcpyDeviceToHost, s));
   SOAP_CUDA(h, cudaEventRecord(h->status_ev, s));
   h->status_pending = true;
