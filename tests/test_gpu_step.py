@@ -139,6 +139,27 @@ def test_moe_layer_all_193_matrices(cuda):
     opt.destroy()
 
 
+def test_moe_stack_24x_sample(cuda):
+    """The 24-layer MoE stack (4706 matrices) does not fit one GPU's HBM with every matrix's
+    state resident, and its matrices are independent, so a deterministic sample is stepped as
+    one batch for the workload's 10 steps: layers 0 and 23 (Wq, Wk, Wv, Wo and experts 0, 31, 63
+    with gate, up and down each) plus the embedding and the LM head (2048x32768, left side only).
+    Teacher-forced against the oracle on steps 1, 2 and 10 for one matrix of each shape class."""
+    per_layer = 4 + 192
+    sample = []
+    for layer in (0, 23):
+        base = layer * per_layer
+        sample += [base + j for j in range(4)]
+        for e in (0, 31, 63):
+            sample += [base + 4 + e, base + 4 + 64 + e, base + 4 + 128 + e]
+    sample += [24 * per_layer, 24 * per_layer + 1]
+    checked = [0, 4, 6, len(sample) - 1]  # Wq of layer 0, gate and down of expert 0, LM head
+    opt, chk = _run_teacher_forced(cuda, "moe_stack_24x_h2048", 10, checked, specs=sample,
+                                   check_steps={1, 2, 10})
+    chk.assert_ok()
+    opt.destroy()
+
+
 def test_dense_block_full_size(cuda):
     """The dense block (hidden 2048, FFN 8192) at full size for 20 steps. Wq is teacher-forced
     against the oracle on steps 1-3 and 20; every matrix's refreshed bases are orthogonal to 1e-5
