@@ -21,7 +21,7 @@ with the Kronecker factors accumulated in the standard Shampoo form of the prime
   S7  dW = Q_L N Q_R^T                                          (Alg. 1, rotate update out)
   S8  W <- (1 - lr*wd) W - lr*dW                                (Alg. 1, weight decay and update)
 
-Readings of points the paper leaves open (each is listed in the design doc):
+Readings of points the paper leaves open:
   * EMA convention: the coefficient multiplies the OLD state (primer, section 2).
     Alg. 1 prints (1-beta) old + beta new; with beta = 0.95 for every EMA here the
     primer's form is used.
@@ -131,6 +131,7 @@ class HParams:
     guard: bool = True
     qr_tol: float = 1e-4
     kl: bool = False              # KL-Shampoo factor form (Alg. 1's "Accumulate Kronecker Factors")
+    stale: bool = False           # factors updated after the refresh (the stale variant of section 5)
 
 
 @dataclass
@@ -274,6 +275,18 @@ def soap_step(st: MatrixState, W: np.ndarray, G: np.ndarray, hp: HParams,
     wd = hp.weight_decay if wd is None else wd
     st.t += 1
     t = st.t
+    if hp.stale:
+        # section 5's "stale preconditioner" variant: the refresh sees the factors of the earlier
+        # steps only, and the current gradient enters them after the update. Its zero QR
+        # columns are not null directions of the current gradient, so the guard does not apply.
+        if hp.kl or hp.guard:
+            raise ValueError("the stale variant is defined for the standard factors without the guard")
+        W_new, dW = _rotate_adam_update(st, W, G, hp, t, d, lr, wd)
+        if st.left:
+            st.L = factor_ema(st.L, G, hp.factor_beta, "L")
+        if st.right:
+            st.R = factor_ema(st.R, G, hp.factor_beta, "R")
+        return W_new, dW
     # S1: accumulate the Kronecker factors with the current gradient
     if hp.kl:
         L, R = factor_ema_kl(st, G, d(hp.factor_beta), d(hp.eps))
@@ -286,6 +299,12 @@ def soap_step(st: MatrixState, W: np.ndarray, G: np.ndarray, hp: HParams,
             st.L = factor_ema(st.L, G, hp.factor_beta, "L")
         if st.right:
             st.R = factor_ema(st.R, G, hp.factor_beta, "R")
+    return _rotate_adam_update(st, W, G, hp, t, d, lr, wd)
+
+
+def _rotate_adam_update(st: MatrixState, W, G, hp: HParams, t: int, d, lr, wd):
+    """S2-S8 of one step (the factors as they stand): refresh every F steps, re-projection,
+    rotation, Adam in the basis, back-rotation and update. Returns (W_new, dW)."""
     # S2-S4: eigenbasis re-computation every F steps
     if t % hp.eig_every == 0:
         M_hat = rotate_out(st.QL if st.left else None, st.m, st.QR if st.right else None)

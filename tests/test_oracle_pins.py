@@ -345,3 +345,54 @@ def test_kl_rounding_negative_eigenvalue_counts_as_zero():
     L_expect = 0.5 / cols * G @ QR @ np.diag(w) @ QR.T @ G.T
     np.testing.assert_allclose(L, L_expect, rtol=1e-9)
     assert np.all(np.linalg.eigvalsh(L) > -1e-6 * np.abs(L).max())
+
+
+# ---- the stale variant (section 5, "Diagnosing the Slingshot Instability") -----------------
+
+def test_stale_first_step_is_plain_adam():
+    """With the current gradient left out of the refresh, step 1 factors P = 0 Q = 0: every QR
+    column is zero, Q stays I, and (without the guard) the step is elementwise Adam with
+    decoupled weight decay; the factors take the gradient only afterwards."""
+    rng = np.random.default_rng(41)
+    rows, cols = 5, 7
+    G = rng.standard_normal((rows, cols))
+    W0 = rng.standard_normal((rows, cols))
+    hp = HParams(stale=True, guard=False)
+    st = MatrixState(rows, cols, True, True)
+    W1, _ = soap_step(st, W0, G, hp)
+    m = (1 - hp.beta1) * G
+    v = (1 - hp.beta2) * G * G
+    N = m / (np.sqrt(v) + hp.eps)
+    np.testing.assert_allclose(W1, (1 - hp.lr * hp.weight_decay) * W0 - hp.lr * N, rtol=1e-12, atol=1e-15)
+    np.testing.assert_array_equal(st.QL, np.eye(rows))
+    np.testing.assert_array_equal(st.QR, np.eye(cols))
+    np.testing.assert_allclose(st.L, (1 - hp.factor_beta) * G @ G.T, rtol=1e-12)
+    np.testing.assert_allclose(st.R, (1 - hp.factor_beta) * G.T @ G, rtol=1e-12)
+
+
+def test_stale_basis_lags_one_gradient():
+    """Step 2 of the stale variant refreshes from L_1 = (1-b) G_1 G_1^T alone: Q_L equals a
+    library QR of L_1 (Q_L = I before it) with the sign fix, and differs from the real-time
+    basis, which also sees G_2."""
+    rng = np.random.default_rng(42)
+    rows, cols = 5, 9
+    G1, G2 = rng.standard_normal((rows, cols)), rng.standard_normal((rows, cols))
+    W = np.zeros((rows, cols))
+    hp = HParams(stale=True, guard=False)
+    st = MatrixState(rows, cols, True, True)
+    soap_step(st, W, G1, hp)
+    soap_step(st, W, G2, hp)
+    Q, Rm = np.linalg.qr((1 - hp.factor_beta) * G1 @ G1.T)
+    Q = Q * np.where(np.diag(Rm) < 0, -1.0, 1.0)
+    np.testing.assert_allclose(st.QL, Q, atol=1e-12)
+    rt = MatrixState(rows, cols, True, True)
+    soap_step(rt, W, G1, HParams(guard=False))
+    soap_step(rt, W, G2, HParams(guard=False))
+    assert np.abs(rt.QL - st.QL).max() > 1e-3
+
+
+def test_stale_rejects_kl_and_guard():
+    st = MatrixState(3, 4, True, True)
+    for hp in (HParams(stale=True), HParams(stale=True, guard=False, kl=True)):
+        with pytest.raises(ValueError):
+            soap_step(st, np.zeros((3, 4)), np.ones((3, 4)), hp)
