@@ -68,7 +68,12 @@ typedef struct {
  *                       R <- b R + (1-b)/rows * G^T Q_L diag(1/(lam_L + eps)) Q_L^T G
  *                     with lam = diag(Q^T F Q) from the factor and basis held before the
  *                     step (a negative lam, which only rounding produces, counts as 0); an
- *                     identity side counts as Q = I, lam = 1. Requires eps > 0. */
+ *                     identity side counts as Q = I, lam = 1. Requires eps > 0.
+ *   stale:            0 = the refresh sees the current gradient (section 5's real-time
+ *                     update); 1 = the stale variant section 5 diagnoses: the refresh uses the
+ *                     factors of the earlier steps and G enters them after the step's update.
+ *                     Requires kl = 0 and guard = 0 (the factors' zero QR columns are then not
+ *                     null directions of the current gradient). */
 typedef struct {
   float lr, beta1, beta2, factor_beta, eps, weight_decay;
   int32_t eig_every;
@@ -76,18 +81,21 @@ typedef struct {
   float qr_tol;
   int32_t guard;
   int32_t kl;
+  int32_t stale;
 } soap_hparams;
 
 /* Fills *hp with the defaults used for the paper's workloads: lr 3e-3,
  * beta1 = beta2 = factor_beta = 0.95, eps 1e-8, weight_decay 0.1, F = 1, no bias
- * correction, qr_tol 1e-4, guard on, standard factor EMAs (kl 0). */
+ * correction, qr_tol 1e-4, guard on, standard factor EMAs (kl 0) with the current gradient
+ * (stale 0). */
 void soap_default_hparams(soap_hparams* hp);
 
 /* Creates the optimizer for n matrices on CUDA device `device` and allocates all
  * state (Alg. 1 "Optimizer States") and workspace up front: L = R = 0, Q = I,
  * m = v = 0, t = 0. shapes[] is copied. Returns SOAP_ERR_OOM if the state does
  * not fit; *out is then NULL; SOAP_ERR_INVALID_ARG for kl = 1 with eps <= 0 (the first
- * KL step weighs by 1/eps). The device becomes current for the calling thread. */
+ * KL step weighs by 1/eps) and for stale = 1 with kl or guard set. The device becomes
+ * current for the calling thread. */
 soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparams* hp,
                           int32_t device, soap_handle* out);
 

@@ -14,7 +14,8 @@
 //   G' = X1 Q_R, m = X2 Q_R
 //   v <- b2 v + (1-b2) G'^2, N = m / (sqrt(v) + eps)        S6
 //   X1 = Q_L N; W <- (1 - lr wd) W - lr X1 Q_R^T           S7, S8 (fused in the GEMM epilogue)
-// With hparams.kl, S1 takes Alg. 1's KL-Shampoo form instead: each factor's EMA term is
+// With hparams.stale, S1 moves to the end of the step (the refresh sees the earlier gradients
+// only). With hparams.kl, S1 takes Alg. 1's KL-Shampoo form instead: each factor's EMA term is
 // weighed by the other factor's inverse, Q diag(1/(lam + eps)) Q^T with lam = diag(Q^T F Q)
 // (an identity side as lam = 1); see prepare_class.
 #include <algorithm>
@@ -238,6 +239,25 @@ soap::TcEpilogue epi(soap_handle h, float* C, int64_t ldc, int64_t c_stride, flo
 soap_status_t prepare_class(soap_handle h, ClassState& c, const float* const* d_grads, cudaStream_t s) {
   const soap_hparams& hp = h->hp;
   const int B = c.count, m = (int)c.rows, n = (int)c.cols;
+  const int64_t mn = (int64_t)m * n;
+  if (!c.tc) {
+    SOAP_CUDA(h, soap::momentum_and_copy(d_grads, c.Gc, c.Mhat, mn, B, hp.beta1, h->d_status, s));
+    return SOAP_OK;
+  }
+  SOAP_CUDA(h, soap::momentum_split(d_grads, c.Gc, c.Gc_lo, c.Gt, c.Gt_lo, c.Mhat, c.Mhat_lo, m, n, B, hp.beta1, c.tr,
+                                    h->d_status, s));
+  if (c.basis_dirty) {
+    if (c.left) SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, B, s));
+    if (c.right) SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, n, B, s));
+    c.basis_dirty = false;
+  }
+  return SOAP_OK;
+}
+
+// S1 for one class (after prepare_class): the standard factor EMAs, or Alg. 1's KL form.
+soap_status_t accumulate_factors(soap_handle h, ClassState& c, cudaStream_t s) {
+  const soap_hparams& hp = h->hp;
+  const int B = c.count, m = (int)c.rows, n = (int)c.cols;
   const int64_t mn = (int64_t)m * n, mm = (int64_t)m * m, nn = (int64_t)n * n;
   const float fb = hp.factor_beta;
   // S1 weights. Standard form: 1 - b. KL form with an identity side (S = I, lambda = 1):
@@ -248,7 +268,6 @@ soap_status_t prepare_class(soap_handle h, ClassState& c, const float* const* d_
   using soap::strided;
   using soap::strided_mut;
   if (!c.tc) {
-    SOAP_CUDA(h, soap::momentum_and_copy(d_grads, c.Gc, c.Mhat, mn, B, hp.beta1, h->d_status, s));
     if (c.left)  // S1: L <- b L + (1-b) G G^T
       SOAP_CUDA(h, soap::gemm(false, true, m, m, n, aL, strided(c.Gc, n, mn), strided(c.Gc, n, mn), fb,
                               strided_mut(c.L, m, mm), B, s));
@@ -256,13 +275,6 @@ soap_status_t prepare_class(soap_handle h, ClassState& c, const float* const* d_
       SOAP_CUDA(h, soap::gemm(true, false, n, n, m, aR, strided(c.Gc, n, mn), strided(c.Gc, n, mn), fb,
                               strided_mut(c.R, n, nn), B, s));
     return SOAP_OK;
-  }
-  SOAP_CUDA(h, soap::momentum_split(d_grads, c.Gc, c.Gc_lo, c.Gt, c.Gt_lo, c.Mhat, c.Mhat_lo, m, n, B, hp.beta1, c.tr,
-                                    h->d_status, s));
-  if (c.basis_dirty) {
-    if (c.left) SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, B, s));
-    if (c.right) SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, n, B, s));
-    c.basis_dirty = false;
   }
   if (hp.kl && c.left && c.right) {
     // KL-Shampoo factor form (Alg. 1), from the factors and bases held before this step:
@@ -465,6 +477,7 @@ void soap_default_hparams(soap_hparams* hp) {
   hp->qr_tol = 1e-4f;
   hp->guard = 1;
   hp->kl = 0;
+  hp->stale = 0;
 }
 
 soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparams* hp,
@@ -475,6 +488,7 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
   if (hp->eig_every < 1 || !(hp->eps >= 0.f) || !(hp->qr_tol >= 0.f)) return SOAP_ERR_INVALID_ARG;
   if (hp->kl != 0 && hp->kl != 1) return SOAP_ERR_INVALID_ARG;
   if (hp->kl && !(hp->eps > 0.f)) return SOAP_ERR_INVALID_ARG;
+  if ((hp->stale != 0 && hp->stale != 1) || (hp->stale && (hp->kl || hp->guard))) return SOAP_ERR_INVALID_ARG;
   for (int i = 0; i < n; ++i) {
     const soap_shape& s = shapes[i];
     if (s.rows < 1 || s.cols < 1 || s.rows > (1 << 20) || s.cols > (1 << 20)) return SOAP_ERR_INVALID_ARG;
@@ -778,8 +792,11 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
   // it is prepared (classes with the largest factors first, so the longest refresh starts
   // earliest); phase C class by class, each waiting only for the groups its bases come from
   // (classes with the smallest factors first, whose refreshes finish earliest).
+  // The stale variant refreshes from the factors as they stand and accumulates G_t into them
+  // at the end of the step.
   for (int ci : h->prep_order) {
     soap_status_t st = prepare_class(h, h->classes[ci], grads_of(h->classes[ci]), s);
+    if (st == SOAP_OK && !hp.stale) st = accumulate_factors(h, h->classes[ci], s);
     if (st != SOAP_OK) return st;
     if (refresh)
       for (int gi : h->fork_after[ci]) {
@@ -799,6 +816,11 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
   }
   for (size_t gi = 0; gi < h->groups.size(); ++gi)
     if (!joined[gi]) SOAP_CUDA(h, cudaStreamWaitEvent(s, h->groups[gi].done, 0));
+  if (hp.stale)
+    for (auto& c : h->classes) {
+      soap_status_t st = accumulate_factors(h, c, s);
+      if (st != SOAP_OK) return st;
+    }
   SOAP_CUDA(h, cudaMemcpyAsync(h->h_status, h->d_status, sizeof(int), cudaMemcpyDeviceToHost, s));
   SOAP_CUDA(h, cudaEventRecord(h->status_ev, s));
   h->status_pending = true;

@@ -42,7 +42,8 @@ class soap_hparams(ctypes.Structure):
                 ("factor_beta", ctypes.c_float), ("eps", ctypes.c_float),
                 ("weight_decay", ctypes.c_float), ("eig_every", ctypes.c_int32),
                 ("bias_correction", ctypes.c_int32), ("qr_tol", ctypes.c_float),
-                ("guard", ctypes.c_int32), ("kl", ctypes.c_int32)]
+                ("guard", ctypes.c_int32), ("kl", ctypes.c_int32),
+                ("stale", ctypes.c_int32)]
 
 
 class soap_kernel_stats(ctypes.Structure):

@@ -42,7 +42,7 @@ def oracle_hparams(hp: S.soap_hparams) -> HParams:
     return HParams(lr=hp.lr, beta1=hp.beta1, beta2=hp.beta2, factor_beta=hp.factor_beta, eps=hp.eps,
                    weight_decay=hp.weight_decay, eig_every=hp.eig_every,
                    bias_correction=bool(hp.bias_correction), guard=bool(hp.guard), qr_tol=hp.qr_tol,
-                   kl=bool(hp.kl))
+                   kl=bool(hp.kl), stale=bool(hp.stale))
 
 
 def gpu_state(opt: S.SoapOptimizer, idx: int, dtype) -> MatrixState:

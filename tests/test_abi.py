@@ -50,6 +50,14 @@ def test_host_side_validation_needs_no_gpu():
     assert lib.soap_create(ok_shape, 1, ctypes.byref(kl_hp), 0, ctypes.byref(h)) == 1
     kl_hp.kl, kl_hp.eps = 2, 1e-8
     assert lib.soap_create(ok_shape, 1, ctypes.byref(kl_hp), 0, ctypes.byref(h)) == 1
+    # the stale variant needs the guard off and the standard factor form
+    assert hp.stale == 0
+    st_hp = S.soap_hparams()
+    lib.soap_default_hparams(ctypes.byref(st_hp))
+    st_hp.stale = 1
+    assert lib.soap_create(ok_shape, 1, ctypes.byref(st_hp), 0, ctypes.byref(h)) == 1
+    st_hp.guard, st_hp.kl = 0, 1
+    assert lib.soap_create(ok_shape, 1, ctypes.byref(st_hp), 0, ctypes.byref(h)) == 1
     assert lib.soap_gemm(0, 0, -1, 1, 1, 1.0, None, 1, 0, None, 1, 0, 0.0, None, 1, 0, 1, None) == 1
     assert lib.soap_gemm(0, 0, 0, 1, 1, 1.0, None, 1, 0, None, 1, 0, 0.0, None, 1, 0, 1, None) == 0
     assert lib.soap_qr(0, 1, None, None, None, 0.0, None, 0, None) == 1

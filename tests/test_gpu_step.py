@@ -108,9 +108,12 @@ def test_one_sided_and_identity_matrices(cuda, shape):
     chk.assert_ok()
 
 
-@pytest.mark.parametrize("variant", [dict(eig_every=3), dict(bias_correction=1), dict(guard=0, qr_tol=0.0)])
+@pytest.mark.parametrize("variant", [dict(eig_every=3), dict(bias_correction=1), dict(guard=0, qr_tol=0.0),
+                                     dict(stale=1, guard=0), dict(stale=1, guard=0, eig_every=3)])
 def test_variants_against_oracle(cuda, variant):
-    """F > 1 (no refresh on most steps), bias correction, and the guard/zero-column reading off."""
+    """F > 1 (no refresh on most steps), bias correction, the guard/zero-column reading off, and
+    section 5's stale variant (the refresh leaves out the current gradient), every step and every
+    third step."""
     hp = S.default_hparams(**variant)
     opt = S.SoapOptimizer([(96, 160)], hp)
     chk = TeacherForcedCheck(opt, oracle_hparams(hp))
@@ -123,7 +126,7 @@ def test_variants_against_oracle(cuda, variant):
         opt.step([W], [G])
         chk.after(0, W)
     print("\n" + chk.report())
-    if variant.get("guard", 1) == 0:
+    if variant.get("guard", 1) == 0 and not variant.get("stale"):
         # without the guard, fp32 junk in the zero directions decides the update: bound by the twin only
         assert all(np.isfinite(r["e_gpu"]) for r in chk.rows)
     else:
@@ -135,6 +138,27 @@ def test_moe_layer_all_193_matrices(cuda):
     step for 20 steps; sampled matrices teacher-forced against the oracle on chosen steps."""
     sample = [0, 64 + 5, 128 + 9, 192]  # gate of expert 0, up of expert 5, down of expert 9, router
     opt, chk = _run_teacher_forced(cuda, "moe_layer_64x768_h2048", 20, sample, check_steps={1, 2, 3, 20})
+    chk.assert_ok()
+    opt.destroy()
+
+
+@pytest.mark.parametrize("shape", [(64, 304, True, False), (300, 64, False, True), (48, 40, True, True)])
+def test_stale_variant_one_sided_and_small(cuda, shape):
+    """The stale variant on a left-only tensor-core class (run as the right-only problem of G^T),
+    a right-only CUDA-core class and a small two-sided class, 8 steps against the oracle."""
+    rows, cols, left, right = shape
+    hp = S.default_hparams(stale=1, guard=0)
+    opt = S.SoapOptimizer([shape], hp)
+    chk = TeacherForcedCheck(opt, oracle_hparams(hp))
+    g = torch.Generator(device=cuda).manual_seed(13)
+    W = (0.02 * torch.randn(rows, cols, device=cuda, generator=g)).contiguous()
+    A = torch.randn(rows, cols, device=cuda, generator=g) / np.sqrt(rows * cols)
+    for t in range(8):
+        G = (A + 0.3 * torch.randn(rows, cols, device=cuda, generator=g) / np.sqrt(cols)).contiguous()
+        chk.before(0, W, G)
+        opt.step([W], [G])
+        chk.after(0, W)
+    print("\n" + chk.report())
     chk.assert_ok()
     opt.destroy()
 
