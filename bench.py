@@ -55,6 +55,17 @@ def model_flops(rows, cols, left, right, kl=False) -> float:
     return f
 
 
+MUON_NS_STEPS = 16
+MUON_METRIC = "Muon steps/sec per model (bf16 Newton-Schulz) + effective TFLOP/s"
+
+
+def muon_flops(rows, cols, ns=MUON_NS_STEPS) -> float:
+    """FLOPs of one Alg. Muon step for one matrix: per Newton-Schulz iteration A = X X^T,
+    A^2 and (b A + c A^2) X on the min(rows, cols) side (2 per multiply-add)."""
+    r, k = float(min(rows, cols)), float(max(rows, cols))
+    return ns * (2 * r * r * k + 2 * r ** 3 + 2 * r * r * k)
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -140,7 +151,7 @@ TC_PRODUCTS = 4
 TRAFFIC_PER_ALGORITHMIC_BYTE = {"qr_update": 0.884, "qr_panel": 0.390, "gemm_tc": 2.78}
 
 
-def roofline(family, st, peaks, peak_src):
+def roofline(family, st, peaks, peak_src, products=None, dtype_ratio=2.0):
     """Roofline of one kernel family from its CUDA-event time and algorithmic FLOPs/bytes."""
     secs = st["ms"] / 1e3
     ratio = TRAFFIC_PER_ALGORITHMIC_BYTE.get(family)
@@ -154,15 +165,18 @@ def roofline(family, st, peaks, peak_src):
         return dict(base, bound="alu", achieved=ach, peak=FP32_SIMT_PEAK_TFLOPS, unit="TFLOP/s",
                     frac=ach / FP32_SIMT_PEAK_TFLOPS,
                     peak_source="fp32 FMA peak of the CUDA cores, 152 SMs x 128 lanes x 2 x 2.07 GHz")
-    # the kernels run inside a long step: the sustained tensor peak
-    tc_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]) / 2.0 / TC_PRODUCTS
+    # the kernels run inside a long step: the sustained tensor peak; fp32 products take
+    # TC_PRODUCTS tf32 MMAs at half the bf16 rate, bf16 products (Muon) one MMA at the bf16 rate
+    products = TC_PRODUCTS if products is None else products
+    tc_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]) / dtype_ratio / products
     ridge = tc_peak * 1e12 / (peaks["hbm_gbs"] * 1e9)  # FLOP per byte where the two bounds meet
     # a tensor-core family whose FLOPs per algorithmic byte reach the ridge is bound by the tensor
     # pipe (the QR's block products sit at the ridge: 2 x 128 fp32 FLOP per 4-8 bytes of C)
     if family in ("gemm_tc", "qr_update") and st["flops"] / max(1.0, st["bytes"]) >= ridge:
         ach = st["flops"] / secs / 1e12
         return dict(base, bound="tensor", achieved=ach, peak=tc_peak, unit="TFLOP/s", frac=ach / tc_peak,
-                    peak_source=f"{peak_src} sustained bf16 dense / 2 (tf32) / {TC_PRODUCTS} (tf32 products per fp32 product)")
+                    peak_source=f"{peak_src} sustained bf16 dense" + (
+                        f" / 2 (tf32) / {products} (tf32 products per fp32 product)" if products > 1 else ""))
     ach = st["bytes"] / secs / 1e9
     return dict(base, bound="hbm", achieved=ach, peak=peaks["hbm_gbs"], unit="GB/s", frac=ach / peaks["hbm_gbs"],
                 peak_source=peak_src)
@@ -189,6 +203,24 @@ def oracle_sample(steps: int, warmup: int, kl: bool = False):
     per = float(np.mean(times))
     block = sum(model_flops(s.rows, s.cols, s.left, s.right, kl) for s in specs)
     scale = block / model_flops(2048, 2048, True, True, kl)
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return per, 1.0 / (per * scale), threads, scale
+
+
+def muon_oracle_sample():
+    """One fp64 oracle Muon step of Wq (2048x2048) on the host cores, scaled to the block."""
+    from oracle.muon_ref import MuonParams, MuonState, muon_step
+    from paper_2607_20548_gb300.workloads import WORKLOADS, make_stream
+
+    specs, _ = WORKLOADS[WORKLOAD]
+    stream = make_stream(WORKLOAD, seed=0, device="cpu", specs=[0])
+    W = stream.weights()[0][0].numpy().astype(np.float64)
+    G = stream.grads(1)[0][0].numpy()
+    hp = MuonParams(coeffs=[(15 / 8, -10 / 8, 3 / 8)] * MUON_NS_STEPS)
+    t0 = time.perf_counter()
+    muon_step(MuonState(2048, 2048), W, G, hp)
+    per = time.perf_counter() - t0
+    scale = sum(muon_flops(s.rows, s.cols) for s in specs) / muon_flops(2048, 2048)
     threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
     return per, 1.0 / (per * scale), threads, scale
 
@@ -227,8 +259,12 @@ def run_soap(args):
     if subset:
         specs = [specs[j] for j in subset]
     gen = make_stream(WORKLOAD, seed=rank, device=dev, specs=subset)
-    opt = SoapOptimizer([(s.rows, s.cols, s.left, s.right) for s in specs], default_hparams(kl=int(args.kl)),
-                        device=local)
+    muon = args.optimizer == "muon"
+    if muon:
+        opt = S.MuonOptimizer([(s.rows, s.cols) for s in specs], ns_steps=MUON_NS_STEPS, device=local)
+    else:
+        opt = SoapOptimizer([(s.rows, s.cols, s.left, s.right) for s in specs], default_hparams(kl=int(args.kl)),
+                            device=local)
 
     def flat(tensors):
         out = [None] * len(specs)
@@ -307,27 +343,35 @@ def run_soap(args):
     if rank != 0:
         opt.destroy()
         return
-    block_flops = sum(model_flops(s.rows, s.cols, s.left, s.right, args.kl) for s in specs)
+    if muon:
+        block_flops = sum(muon_flops(s.rows, s.cols) for s in specs)
+    else:
+        block_flops = sum(model_flops(s.rows, s.cols, s.left, s.right, args.kl) for s in specs)
     peaks, peak_src = measured_peaks()
     fams = {k: v for k, v in prof.items() if k != "overflow"}
     top = max(fams, key=lambda k: fams[k]["ms"])
     st = fams[top]
     launches = sum(v["launches"] for v in fams.values())
-    roof = roofline(top, st, peaks, peak_src)
-    per, sps, threads, scale = oracle_sample(1, 0, args.kl)
+    roof = roofline(top, st, peaks, peak_src, products=1 if muon else TC_PRODUCTS, dtype_ratio=1.0 if muon else 2.0)
+    if muon:
+        # the DRAM/algorithmic ratios above were measured for the fp32 (tf32 x4) kernels
+        roof["traffic"], roof["traffic_note"] = None, "not measured for the bf16 kernel"
+    per, sps, threads, scale = muon_oracle_sample() if muon else oracle_sample(1, 0, args.kl)
+    tc_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]) / (1.0 if muon else 2.0 * TC_PRODUCTS)
     line = {
-        "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "metric": MUON_METRIC if muon else METRIC, "value": value, "unit": "steps/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if muon else "f32",
+        "data": "synthetic",
         "config": {"workload": WORKLOAD if not subset else f"{WORKLOAD}[matrices {args.matrices}]",
                    "matrices": len(specs),
                    "shapes": "4x 2048x2048, 2x 2048x8192, 1x 8192x2048, all sides preconditioned",
                    "parallelism": "replicas" if world > 1 else "single",
-                   "factor_form": "kl" if args.kl else "standard",
+                   "optimizer": "muon (16 quintic Newton-Schulz steps)" if muon else
+                   ("soap, KL factor form" if args.kl else "soap, standard factor form"),
                    "l2": "inputs larger than L2 (3 GB of optimizer state per step)"},
         "effective_tflops": block_flops * value / world / 1e12,
-        "effective_frac_of_tensor_fp32_peak": block_flops * value / world / 1e12 /
-                                              (peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]) / 2.0 / TC_PRODUCTS),
+        "effective_frac_of_tensor_peak": block_flops * value / world / 1e12 / tc_peak,
         "model_flop_per_step": block_flops,
         "roofline": roof,
         "kernel_time_share": {k: round(v["ms"] / max(1e-9, sum(x["ms"] for x in fams.values())), 4)
@@ -337,8 +381,8 @@ def run_soap(args):
                                 "gbs": v["bytes"] / max(1e-12, v["ms"] / 1e3) / 1e9}
                             for k, v in fams.items() if v["launches"]},
         "cpu_baseline": {"value": sps, "unit": "steps/s", "cores": threads, "kind": "oracle",
-                         "sample": f"one fp64 oracle step of Wq (2048x2048) took {per:.1f} s; whole block "
-                                   f"= {scale:.1f}x that by the FLOP model"},
+                         "sample": f"one fp64 oracle {'Muon' if muon else 'SOAP'} step of Wq (2048x2048) took "
+                                   f"{per:.1f} s; whole block = {scale:.1f}x that by the FLOP model"},
         "e2e": {"value": world * args.steps / e2e_s, "unit": "steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
@@ -357,6 +401,8 @@ def main():
     ap.add_argument("--matrices", default="",
                     help="comma-separated matrix indices of the block to run (a smaller case for profiling); "
                          "default: all 7")
+    ap.add_argument("--optimizer", choices=["soap", "muon"], default="soap",
+                    help="muon: the paper's Muon step on the same block (a separate line, not the headline)")
     ap.add_argument("--kl", action="store_true",
                     help="KL-Shampoo factor form (Alg. 1's factor accumulation) instead of the standard EMAs")
     args = ap.parse_args()

@@ -1,6 +1,7 @@
 // Internal declarations shared by the libsoap translation units (not part of the ABI).
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -104,6 +105,38 @@ struct QrLookahead {
 cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q_lo, uint8_t* skip,
                    float tol, void* workspace, size_t workspace_bytes, int* status,
                    cudaStream_t stream, const QrLookahead* la = nullptr);
+
+// bf16 tensor-core product out_b = alpha A_b B_b^T + beta Cin_b (A_b M x K, B_b N x K, bf16
+// row-major; fp32 accumulation). Outputs (any may be null): out (bf16, ld, stride; Cin has the
+// same layout), out_t (bf16, transposed: element (r, c) at c * ld_t + r) and out_f32.
+// N and K must be multiples of 8.
+struct Bf16Epilogue {
+  __nv_bfloat16* out;
+  int64_t ld, stride;
+  const __nv_bfloat16* cin;
+  __nv_bfloat16* out_t;
+  int64_t ld_t, stride_t;
+  float* out_f32;
+  int64_t ld_f32, stride_f32;
+  float alpha, beta;
+  int* status;
+};
+cudaError_t gemm_bf16_nt(int M, int N, int K, int batch, const __nv_bfloat16* A, int64_t lda, int64_t a_stride,
+                         const __nv_bfloat16* B, int64_t ldb, int64_t b_stride, const Bf16Epilogue& ep,
+                         cudaStream_t stream);
+
+// Muon's elementwise kernels (batched over `batch` rows x cols matrices of a class).
+// M <- beta1 M + (1 - beta1) G and norm2[b] += ||M_b||_F^2 (norm2 zeroed by the caller);
+// non-finite gradients set kStatusNonFinite.
+cudaError_t muon_momentum(const float* const* grads, float* M, double* norm2, int64_t elems, int batch, float beta1,
+                          int* status, cudaStream_t stream);
+// X_0 = M / max(||M||_F, eps) in bf16, as X (r x c) and X^T (c x r) with (r, c) = (rows, cols),
+// or, if `transposed`, (r, c) = (cols, rows) and X = M^T scaled.
+cudaError_t muon_init_x(const float* M, const double* norm2, float eps, __nv_bfloat16* X, __nv_bfloat16* Xt,
+                        int rows, int cols, int batch, bool transposed, cudaStream_t stream);
+// W <- (1 - lr wd) W - lr scale O, O bf16 rows x cols.
+cudaError_t muon_update(float* const* params, const __nv_bfloat16* O, int64_t elems, int batch, float lr, float wd,
+                        float scale, cudaStream_t stream);
 
 // Elementwise kernels of the step.
 // M_hat <- b1 M_hat + (1-b1) G and Gc <- G for each matrix of a class.

@@ -1,4 +1,4 @@
-"""ctypes binding of libsoap (include/soap.h): argument marshalling only.
+"""ctypes binding of libsoap (include/soap.h, include/muon.h): argument marshalling only.
 
 Every step of the optimizer runs in the library's CUDA kernels; this module only
 turns torch tensors into pointers and streams. It never computes anything itself,
@@ -29,7 +29,16 @@ EXPORTS = ("soap_default_hparams", "soap_create", "soap_step", "soap_set_lr", "s
            "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_profile_records",
            "soap_gemm_tf32x4",
            "soap_split_tf32", "soap_qr_static")
+# every symbol include/muon.h declares
+MUON_EXPORTS = ("muon_default_hparams", "muon_create", "muon_step", "muon_set_lr", "muon_state_get",
+                "muon_state_set", "muon_status", "muon_last_error", "muon_destroy", "muon_profile_begin",
+                "muon_profile_end")
 KERNEL_FAMILIES = ("gemm_simt", "gemm_tc", "qr_panel", "elementwise", "other", "qr_update")
+
+
+class muon_hparams(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("weight_decay", ctypes.c_float),
+                ("eps", ctypes.c_float), ("ns_steps", ctypes.c_int32), ("coeffs", ctypes.c_void_p)]
 
 
 class soap_shape(ctypes.Structure):
@@ -97,6 +106,17 @@ def load_library(path: str = LIB_PATH):
                                    I32, P, P, P]),
         "soap_split_tf32": (I32, [P, P, P, I64, P]),
         "soap_qr_static": (I32, [I32, I32, P, P, P, F, P]),
+        "muon_default_hparams": (None, [ctypes.POINTER(muon_hparams)]),
+        "muon_create": (I32, [ctypes.POINTER(soap_shape), I32, ctypes.POINTER(muon_hparams), I32, ctypes.POINTER(P)]),
+        "muon_step": (I32, [P, P, P, P]),
+        "muon_set_lr": (I32, [P, F, F]),
+        "muon_state_get": (I32, [P, I32, P, P]),
+        "muon_state_set": (I32, [P, I32, P, P]),
+        "muon_status": (I32, [P, P]),
+        "muon_last_error": (ctypes.c_char_p, [P]),
+        "muon_destroy": (None, [P]),
+        "muon_profile_begin": (I32, [P, I64]),
+        "muon_profile_end": (I32, [P, P, ctypes.POINTER(soap_kernel_stats), ctypes.POINTER(I32)]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -375,3 +395,106 @@ def soap_gemm_tf32x4(A, B, alpha=1.0, beta=0.0, C=None, transpose_c=False, A_spl
     if with_lo:
         return out, (lo[0] if out.dim() == 2 else lo)
     return out
+
+
+class MuonOptimizer:
+    """One Muon handle (include/muon.h): muon_create / muon_step / muon_state_get / set.
+
+    ``coeffs`` is a list of (a_i, b_i, c_i) Newton-Schulz coefficients (None: the library's
+    default quintic schedule); its length sets the number of iterations."""
+
+    def __init__(self, shapes, lr=3e-3, beta1=0.9, weight_decay=0.1, eps=1e-7, coeffs=None, ns_steps=16,
+                 device: int | None = None):
+        lib = load_library()
+        self.shapes = [(int(s[0]), int(s[1])) for s in shapes]
+        arr = (soap_shape * len(self.shapes))(*[soap_shape(r, c, 0, 0) for r, c in self.shapes])
+        hp = muon_hparams()
+        lib.muon_default_hparams(ctypes.byref(hp))
+        hp.lr, hp.beta1, hp.weight_decay, hp.eps = lr, beta1, weight_decay, eps
+        self._coeffs = None
+        if coeffs is not None:
+            flat = [float(x) for abc in coeffs for x in abc]
+            self._coeffs = (ctypes.c_float * len(flat))(*flat)
+            hp.ns_steps = len(coeffs)
+            hp.coeffs = ctypes.cast(self._coeffs, ctypes.c_void_p)
+        else:
+            hp.ns_steps = ns_steps
+        self.device = torch.cuda.current_device() if device is None else device
+        h = ctypes.c_void_p()
+        code = lib.muon_create(arr, len(self.shapes), ctypes.byref(hp), self.device, ctypes.byref(h))
+        if code != SOAP_OK:
+            raise SoapError(code, "muon_create")
+        self._h = h
+        n = len(self.shapes)
+        self._pp = (ctypes.c_void_p * n)()
+        self._gp = (ctypes.c_void_p * n)()
+
+    def _handle(self):
+        if self._h is None:
+            raise SoapError(1, "handle destroyed")
+        return self._h
+
+    def _check(self, code):
+        if code != SOAP_OK:
+            raise SoapError(code, load_library().muon_last_error(self._h).decode())
+
+    def step(self, params, grads, stream=None):
+        """muon_step on device tensors (fp32, contiguous); params are updated in place."""
+        n = len(self.shapes)
+        if len(params) != n or len(grads) != n:
+            raise ValueError("need one param and one grad per matrix")
+        for i, (p, g, s) in enumerate(zip(params, grads, self.shapes)):
+            if p.dtype != torch.float32 or g.dtype != torch.float32 or not p.is_cuda or not g.is_cuda:
+                raise TypeError(f"matrix {i}: params/grads must be fp32 CUDA tensors")
+            if tuple(p.shape) != s or tuple(g.shape) != s or not p.is_contiguous() or not g.is_contiguous():
+                raise ValueError(f"matrix {i}: expected a contiguous {s} tensor")
+            self._pp[i] = p.data_ptr()
+            self._gp[i] = g.data_ptr()
+        self._check(load_library().muon_step(self._handle(), self._pp, self._gp, _stream(stream)))
+
+    def set_lr(self, lr: float, weight_decay: float):
+        self._check(load_library().muon_set_lr(self._handle(), lr, weight_decay))
+
+    def state_get(self, idx: int, stream=None) -> torch.Tensor:
+        """The momentum M of matrix idx as a new device tensor."""
+        out = torch.empty(self.shapes[idx], dtype=torch.float32, device=f"cuda:{self.device}")
+        self._check(load_library().muon_state_get(self._handle(), idx, ctypes.c_void_p(out.data_ptr()),
+                                                  _stream(stream)))
+        return out
+
+    def state_set(self, idx: int, src: torch.Tensor, stream=None):
+        if tuple(src.shape) != self.shapes[idx] or src.dtype != torch.float32 or not src.is_contiguous():
+            raise ValueError("state_set: wrong shape, dtype or layout")
+        self._check(load_library().muon_state_set(self._handle(), idx, ctypes.c_void_p(src.data_ptr()),
+                                                  _stream(stream)))
+
+    def status(self, stream=None) -> int:
+        return load_library().muon_status(self._handle(), _stream(stream))
+
+    def last_error(self) -> str:
+        return load_library().muon_last_error(self._h).decode() if self._h else "handle destroyed"
+
+    def profile_begin(self, max_launches: int = 1 << 16):
+        """Time every kernel launch of the following calls with CUDA events."""
+        self._check(load_library().muon_profile_begin(self._handle(), max_launches))
+
+    def profile_end(self, stream=None) -> dict:
+        """Synchronise and return {family: {launches, ms, flops, bytes}} plus an overflow flag."""
+        out = (soap_kernel_stats * len(KERNEL_FAMILIES))()
+        ov = ctypes.c_int32(0)
+        self._check(load_library().muon_profile_end(self._handle(), _stream(stream), out, ctypes.byref(ov)))
+        res = {KERNEL_FAMILIES[o.family]: dict(launches=o.launches, ms=o.ms, flops=o.flops, bytes=o.bytes)
+               for o in out}
+        res["overflow"] = bool(ov.value)
+        return res
+
+    def destroy(self):
+        if self._h is not None:
+            load_library().muon_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass

@@ -10,10 +10,10 @@ from paper_2607_20548_gb300 import soap as S
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
-def _declared():
-    text = open(os.path.join(ROOT, "include", "soap.h")).read()
+def _declared(header="soap.h", prefix="soap_"):
+    text = open(os.path.join(ROOT, "include", header)).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(soap_[a-z0-9_]+)\s*\(", text)))
+    return sorted(set(re.findall(r"\b(" + prefix + r"[a-z0-9_]+)\s*\(", text)))
 
 
 def test_library_exports_every_declared_symbol():
@@ -24,6 +24,10 @@ def test_library_exports_every_declared_symbol():
     missing = [n for n in names if not hasattr(lib, n)]
     assert not missing, missing
     assert set(names) == set(S.EXPORTS)
+    muon = _declared("muon.h", "muon_")
+    assert "muon_create" in muon and "muon_step" in muon
+    assert not [n for n in muon if not hasattr(lib, n)]
+    assert set(muon) == set(S.MUON_EXPORTS)
 
 
 def test_host_side_validation_needs_no_gpu():
@@ -66,3 +70,14 @@ def test_host_side_validation_needs_no_gpu():
     assert lib.soap_get_step(None) == -1
     assert lib.soap_last_error(None) == b"null handle"
     lib.soap_destroy(None)
+    # Muon: sides must be multiples of 8, ns_steps in 1..64
+    mh = S.muon_hparams()
+    lib.muon_default_hparams(ctypes.byref(mh))
+    assert mh.ns_steps == 16 and abs(mh.beta1 - 0.9) < 1e-7 and abs(mh.eps - 1e-7) < 1e-12
+    bad = (S.soap_shape * 1)(S.soap_shape(12, 16, 0, 0))
+    assert lib.muon_create(bad, 1, ctypes.byref(mh), 0, ctypes.byref(h)) == 1
+    mh.ns_steps = 0
+    good = (S.soap_shape * 1)(S.soap_shape(16, 16, 0, 0))
+    assert lib.muon_create(good, 1, ctypes.byref(mh), 0, ctypes.byref(h)) == 1
+    assert lib.muon_last_error(None) == b"null handle"
+    lib.muon_destroy(None)
