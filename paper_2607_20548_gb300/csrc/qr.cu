@@ -1020,9 +1020,12 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     // where it overlaps the next block's panels; the next block's rows wait for the previous
     // far update, which covered them. The block's V T follows its far update on the far stream.
     const int knext = std::min(NBO, std::max(nc, 0));
-    e = cudaEventRecord(ev_vt, s);
-    if (e == cudaSuccess && nc > 0) e = cudaStreamWaitEvent(s, ev_far, 0);
+    // (the far update starts once the next block's rows are done, so that those small products
+    // do not wait for SMs behind it)
+    e = cudaSuccess;
+    if (nc > 0) e = cudaStreamWaitEvent(s, ev_far, 0);
     if (e == cudaSuccess && nc > 0) e = update_rows(k0 + kbo, knext, w.W, w.W_lo, w.Wsplit, s);
+    if (e == cudaSuccess) e = cudaEventRecord(ev_vt, s);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(far, ev_vt, 0);
     if (e == cudaSuccess && nc > knext) e = update_rows(k0 + kbo + knext, nc - knext, w.W2, w.W2_lo, w.Wsplit2, far);
     if (e == cudaSuccess) e = cudaEventRecord(ev_far, far);

@@ -95,7 +95,7 @@ void qr_input_buffers(void* workspace, int n, int batch, float** At);
 // The look-ahead schedule of qr_q_t: a second (low-priority) stream and its events.
 struct QrLookahead {
   cudaStream_t far;     // trailing updates beyond the next block, and V T for the Q accumulation
-  cudaEvent_t vt;       // this block's V T^T is ready (recorded on the caller's stream)
+  cudaEvent_t vt;       // this block's V T^T and the next block's rows are ready (caller's stream)
   cudaEvent_t far_done; // the far update of the previous block is done (recorded on `far`)
   cudaEvent_t vq[2];    // V T of the block using buffer 0 / 1 is done (recorded on `far`)
 };
