@@ -145,10 +145,10 @@ TC_PRODUCTS = 4
 
 # DRAM bytes (ncu dram__bytes_read.sum + dram__bytes_write.sum) per algorithmic byte of each
 # kernel family, measured with ncu over one step of the block's 2048x8192 matrix alone
-# (both of its QR sizes) for the current kernels. The QR update products read operands that
-# stay in L2 across tiles (ratio < 1); the large contractions re-read operand panels
-# (ratio > 1); the panel kernel keeps its panel in shared memory.
-TRAFFIC_PER_ALGORITHMIC_BYTE = {"qr_update": 0.884, "qr_panel": 0.390, "gemm_tc": 2.78}
+# (both of its QR sizes) for the current kernels. The QR products read their small operands
+# from L2 across tiles and write split-K partial sums (ratio about 1); the large contractions
+# re-read operand panels (ratio > 1); the panel kernel keeps its panel on chip.
+TRAFFIC_PER_ALGORITHMIC_BYTE = {"qr_update": 1.059, "qr_panel": 0.383, "gemm_tc": 1.617}
 
 
 def roofline(family, st, peaks, peak_src, products=None, dtype_ratio=2.0):
