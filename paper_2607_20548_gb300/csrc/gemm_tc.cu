@@ -214,7 +214,7 @@ __device__ __forceinline__ void tile_coords(int t, int ntm, int ntn, int BN_, in
 // With CVTA the A operand comes as fp32 only: the epilogue warps form its lo part in shared
 // memory, beside the tile TMA brought in (for HBM-bound products whose A is read once; the
 // extra shared-memory traffic would slow a compute-bound product).
-template <int BN, int STAGES, bool PRE, bool CVTA>
+template <int BN, int STAGES, bool PRE, bool CVTA, bool TR>
 __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap ta_hi, const __grid_constant__ CUtensorMap ta_lo,
                    const __grid_constant__ CUtensorMap tb_hi, const __grid_constant__ CUtensorMap tb_lo, int M,
@@ -387,7 +387,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
       const bool vec = Cb && (ep.ldc & 3) == 0 && (reinterpret_cast<uintptr_t>(Cb) & 15) == 0 &&
                        (!Lb || ((ep.ld_lo & 3) == 0 && (reinterpret_cast<uintptr_t>(Lb) & 15) == 0));
       // the prefetch copies whole 16-byte units: the dimension they run along must be a multiple of 4
-      const bool pre = PRE && vec && ep.beta != 0.f && ((ep.transpose ? M : N) & 3) == 0;
+      const bool pre = PRE && vec && ep.beta != 0.f && ((TR ? M : N) & 3) == 0;
       if (pre) {
         // this warp's C block, copied in while the MMAs run; only 16-byte units wholly inside C
         for (int c = 0; c < C::NCH; ++c) {
@@ -395,15 +395,15 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
           for (int u = lane; u < 256; u += 32) {
             const int x = u >> 3, y4 = u & 7;  // x: row (or column if transposed), y4: 16-byte unit
             int r, col;
-            if (!ep.transpose) {
+            if (!TR) {
               r = row0 + x;
               col = col0 + 32 * c + 4 * y4;
             } else {
               col = col0 + 32 * c + x;
               r = row0 + 4 * y4;
             }
-            const bool ok = ep.transpose ? (col < N && r + 3 < M) : (r < M && col + 3 < N);
-            const float* src = !ok ? Cb : ep.transpose ? Cb + (int64_t)col * ep.ldc + r : Cb + (int64_t)r * ep.ldc + col;
+            const bool ok = TR ? (col < N && r + 3 < M) : (r < M && col + 3 < N);
+            const float* src = !ok ? Cb : TR ? Cb + (int64_t)col * ep.ldc + r : Cb + (int64_t)r * ep.ldc + col;
             cp_async16(cb + x * 32 + ((y4 ^ (x & 7)) << 2), src, ok);
           }
         }
@@ -448,7 +448,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
       for (int c = 0; c < C::NCH; ++c) {
         float* cb = obuf + (PRE ? 1024 * c : 0);
         const int cc0 = col0 + 32 * c;
-        if (!ep.transpose) {
+        if (!TR) {
           const int r = row0 + lane;  // this lane's row
 #pragma unroll
           for (int j4 = 0; j4 < 8; ++j4) {
@@ -582,7 +582,7 @@ bool make_map(CUtensorMap* map, const float* base, int rows, int K, int64_t ld, 
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES, bool PRE, bool CVTA = false>
+template <int BN, int STAGES, bool PRE, bool CVTA = false, bool TR = false>
 cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, int batch, const TcEpilogue& ep,
                    cudaStream_t s, int ksplit = 1) {
   using C = Cfg<BN, STAGES, PRE>;
@@ -596,7 +596,8 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e =
-        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE, CVTA>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
@@ -607,7 +608,7 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
   const int kblocks = (K + BK - 1) / BK;
   const int tpc = kblocks > 16 ? 1 : (int)std::max<int64_t>(1, std::min<int64_t>(8, ntiles / (4 * 152)));
   const int grid = (int)((ntiles + tpc - 1) / tpc);
-  gemm_tc_kernel<BN, STAGES, PRE, CVTA><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
+  gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
                                                                      bmod, tpc, ksplit, ep);
   return cudaGetLastError();
 }
@@ -680,7 +681,7 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
   }
   // an A given without its lo part gets it formed in the kernel (products whose C is not read)
   const bool cvt = A.lo == nullptr;
-  if (cvt && pre) return cudaErrorInvalidValue;
+  if (cvt && (pre || ep.transpose)) return cudaErrorInvalidValue;
   if (B.lo == nullptr) return cudaErrorInvalidValue;
   if (ksplit > 1) {
     const TcEpilogue pe{split_ws, nullptr, N, (int64_t)M * N, nullptr, N, (int64_t)M * N, 0, 1.f, 0.f, ep.status};
@@ -698,10 +699,17 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
   if (cvt)
     return N <= 32 ? tc::launch<32, 5, false, true>(A, B, M, N, K, batch, ep, s)
                    : tc::launch<128, 3, false, true>(A, B, M, N, K, batch, ep, s);
-  if (N <= 32) return pre ? tc::launch<32, 4, true>(A, B, M, N, K, batch, ep, s)
-                          : tc::launch<32, 5, false>(A, B, M, N, K, batch, ep, s);
-  return pre ? tc::launch<128, 2, true>(A, B, M, N, K, batch, ep, s)
-             : tc::launch<128, 3, false>(A, B, M, N, K, batch, ep, s);
+  // transposed outputs get their own instantiations (a smaller epilogue for each)
+  const bool tr = ep.transpose != 0;
+  if (N <= 32)
+    return pre ? (tr ? tc::launch<32, 4, true, false, true>(A, B, M, N, K, batch, ep, s)
+                     : tc::launch<32, 4, true>(A, B, M, N, K, batch, ep, s))
+               : (tr ? tc::launch<32, 5, false, false, true>(A, B, M, N, K, batch, ep, s)
+                     : tc::launch<32, 5, false>(A, B, M, N, K, batch, ep, s));
+  return pre ? (tr ? tc::launch<128, 2, true, false, true>(A, B, M, N, K, batch, ep, s)
+                   : tc::launch<128, 2, true>(A, B, M, N, K, batch, ep, s))
+             : (tr ? tc::launch<128, 3, false, false, true>(A, B, M, N, K, batch, ep, s)
+                   : tc::launch<128, 3, false>(A, B, M, N, K, batch, ep, s));
 }
 
 }  // namespace soap
