@@ -214,7 +214,7 @@ __device__ __forceinline__ void tile_coords(int t, int ntm, int ntn, int BN_, in
 // With CVTA the A operand comes as fp32 only: the epilogue warps form its lo part in shared
 // memory, beside the tile TMA brought in (for HBM-bound products whose A is read once; the
 // extra shared-memory traffic would slow a compute-bound product).
-template <int BN, int STAGES, bool PRE, bool CVTA, bool TR>
+template <int BN, int STAGES, bool PRE, bool CVTA, bool TR, bool LO>
 __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap ta_hi, const __grid_constant__ CUtensorMap ta_lo,
                    const __grid_constant__ CUtensorMap tb_hi, const __grid_constant__ CUtensorMap tb_lo, int M,
@@ -380,14 +380,15 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
       tile_coords(t, ntm, ntn, BN, m0, n0, b);
       krange(b, kb0, kb1);
       float* Cb = ep.C_ptrs ? ep.C_ptrs[b] : (ep.C ? ep.C + (int64_t)b * ep.c_stride : nullptr);
-      float* Lb = ep.C_lo ? ep.C_lo + (int64_t)b * ep.lo_stride : nullptr;
+      float* Lb = LO && ep.C_lo ? ep.C_lo + (int64_t)b * ep.lo_stride : nullptr;
       const int row0 = m0 + 32 * q;   // first of this warp's 32 rows
       const int col0 = n0 + colbase;  // first of its CPW columns
       // 16-byte vector access to C (and C_lo) needs 16-byte aligned rows
-      const bool vec = Cb && (ep.ldc & 3) == 0 && (reinterpret_cast<uintptr_t>(Cb) & 15) == 0 &&
+      // (a kernel that prefetches C is only launched on 16-byte aligned C, lo part and rows)
+      const bool vec = PRE || Cb && (ep.ldc & 3) == 0 && (reinterpret_cast<uintptr_t>(Cb) & 15) == 0 &&
                        (!Lb || ((ep.ld_lo & 3) == 0 && (reinterpret_cast<uintptr_t>(Lb) & 15) == 0));
       // the prefetch copies whole 16-byte units: the dimension they run along must be a multiple of 4
-      const bool pre = PRE && vec && ep.beta != 0.f && ((TR ? M : N) & 3) == 0;
+      const bool pre = PRE;
       if (pre) {
         // this warp's C block, copied in while the MMAs run; only 16-byte units wholly inside C
         for (int c = 0; c < C::NCH; ++c) {
@@ -582,7 +583,7 @@ bool make_map(CUtensorMap* map, const float* base, int rows, int K, int64_t ld, 
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES, bool PRE, bool CVTA = false, bool TR = false>
+template <int BN, int STAGES, bool PRE, bool CVTA = false, bool TR = false, bool LO = false>
 cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, int batch, const TcEpilogue& ep,
                    cudaStream_t s, int ksplit = 1) {
   using C = Cfg<BN, STAGES, PRE>;
@@ -596,7 +597,7 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e =
-        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
@@ -608,7 +609,7 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
   const int kblocks = (K + BK - 1) / BK;
   const int tpc = kblocks > 16 ? 1 : (int)std::max<int64_t>(1, std::min<int64_t>(8, ntiles / (4 * 152)));
   const int grid = (int)((ntiles + tpc - 1) / tpc);
-  gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
+  gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
                                                                      bmod, tpc, ksplit, ep);
   return cudaGetLastError();
 }
@@ -635,6 +636,17 @@ __global__ void split_reduce_kernel(const float* P, int ksplit, int batch, int M
       *reinterpret_cast<float4*>(C_lo + (int64_t)b * c_stride + i * ldc + j) =
           make_float4(tf32_lo(o.x), tf32_lo(o.y), tf32_lo(o.z), tf32_lo(o.w));
   }
+}
+
+// One instantiation per (transposed output, lo output): each kernel's epilogue then carries
+// only the store path it uses.
+template <int BN, int STAGES, bool PRE, bool CVTA>
+cudaError_t launch_tl(bool tr, bool lo, const TcOperand& A, const TcOperand& B, int M, int N, int K, int batch,
+                      const TcEpilogue& ep, cudaStream_t s, int ksplit = 1) {
+  if (tr) return lo ? launch<BN, STAGES, PRE, CVTA, true, true>(A, B, M, N, K, batch, ep, s, ksplit)
+                    : launch<BN, STAGES, PRE, CVTA, true, false>(A, B, M, N, K, batch, ep, s, ksplit);
+  return lo ? launch<BN, STAGES, PRE, CVTA, false, true>(A, B, M, N, K, batch, ep, s, ksplit)
+            : launch<BN, STAGES, PRE, CVTA, false, false>(A, B, M, N, K, batch, ep, s, ksplit);
 }
 
 // How many K splits give the fewest idle SMs in the last wave, for a launch of `tiles` tiles
@@ -667,8 +679,13 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
                               2.0 * (double)N * K * (B.batch > 0 ? B.batch : batch) +
                               (double)M * N * batch * ((ep.beta != 0.f ? 2 : 1) + (ep.C_lo ? 1 : 0)));
   ProfScope prof(family, flops, bytes, s);
-  // an epilogue that reads C gives one pipeline stage's shared memory to the C tile
-  const bool pre = ep.beta != 0.f && (ep.C || ep.C_ptrs);
+  // an epilogue that reads C gives one pipeline stage's shared memory to the C tile, which it
+  // prefetches in 16-byte units: C (and its lo part) 16-byte aligned with rows of 16-byte
+  // multiples; otherwise the kernel without the prefetch reads C element by element
+  auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+  const bool pre = ep.beta != 0.f && (ep.C || ep.C_ptrs) && (ep.ldc & 3) == 0 && (ep.c_stride & 3) == 0 &&
+                   (!ep.C || al16(ep.C)) && ((ep.transpose ? M : N) & 3) == 0 &&
+                   (!ep.C_lo || ((ep.ld_lo & 3) == 0 && (ep.lo_stride & 3) == 0 && al16(ep.C_lo)));
   // few tiles and a long K: split K over more CTAs (plain row-major outputs only)
   int ksplit = 1;
   const bool splittable = split_ws && ep.C && !ep.C_ptrs && !ep.transpose && ep.beta == 0.f && (N & 3) == 0 &&
@@ -696,20 +713,15 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
                                                                 ep.c_stride, ep.C_lo);
     return cudaGetLastError();
   }
+  const bool tr = ep.transpose != 0, lo = ep.C_lo != nullptr;
   if (cvt)
-    return N <= 32 ? tc::launch<32, 5, false, true>(A, B, M, N, K, batch, ep, s)
-                   : tc::launch<128, 3, false, true>(A, B, M, N, K, batch, ep, s);
-  // transposed outputs get their own instantiations (a smaller epilogue for each)
-  const bool tr = ep.transpose != 0;
+    return N <= 32 ? tc::launch_tl<32, 5, false, true>(false, lo, A, B, M, N, K, batch, ep, s)
+                   : tc::launch_tl<128, 3, false, true>(false, lo, A, B, M, N, K, batch, ep, s);
   if (N <= 32)
-    return pre ? (tr ? tc::launch<32, 4, true, false, true>(A, B, M, N, K, batch, ep, s)
-                     : tc::launch<32, 4, true>(A, B, M, N, K, batch, ep, s))
-               : (tr ? tc::launch<32, 5, false, false, true>(A, B, M, N, K, batch, ep, s)
-                     : tc::launch<32, 5, false>(A, B, M, N, K, batch, ep, s));
-  return pre ? (tr ? tc::launch<128, 2, true, false, true>(A, B, M, N, K, batch, ep, s)
-                   : tc::launch<128, 2, true>(A, B, M, N, K, batch, ep, s))
-             : (tr ? tc::launch<128, 3, false, false, true>(A, B, M, N, K, batch, ep, s)
-                   : tc::launch<128, 3, false>(A, B, M, N, K, batch, ep, s));
+    return pre ? tc::launch_tl<32, 4, true, false>(tr, lo, A, B, M, N, K, batch, ep, s)
+               : tc::launch_tl<32, 5, false, false>(tr, lo, A, B, M, N, K, batch, ep, s);
+  return pre ? tc::launch_tl<128, 2, true, false>(tr, lo, A, B, M, N, K, batch, ep, s)
+             : tc::launch_tl<128, 3, false, false>(tr, lo, A, B, M, N, K, batch, ep, s);
 }
 
 }  // namespace soap
