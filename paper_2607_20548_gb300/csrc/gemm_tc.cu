@@ -214,7 +214,7 @@ __device__ __forceinline__ void tile_coords(int t, int ntm, int ntn, int BN_, in
 // With CVTA the A operand comes as fp32 only: the epilogue warps form its lo part in shared
 // memory, beside the tile TMA brought in (for HBM-bound products whose A is read once; the
 // extra shared-memory traffic would slow a compute-bound product).
-template <int BN, int STAGES, bool PRE, bool CVTA, bool TR, bool LO>
+template <int BN, int STAGES, bool PRE, bool CVTA, bool TR, bool LO, bool VEC>
 __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap ta_hi, const __grid_constant__ CUtensorMap ta_lo,
                    const __grid_constant__ CUtensorMap tb_hi, const __grid_constant__ CUtensorMap tb_lo, int M,
@@ -385,7 +385,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
       const int col0 = n0 + colbase;  // first of its CPW columns
       // 16-byte vector access to C (and C_lo) needs 16-byte aligned rows
       // (a kernel that prefetches C is only launched on 16-byte aligned C, lo part and rows)
-      const bool vec = PRE || Cb && (ep.ldc & 3) == 0 && (reinterpret_cast<uintptr_t>(Cb) & 15) == 0 &&
+      const bool vec = PRE || VEC || Cb && (ep.ldc & 3) == 0 && (reinterpret_cast<uintptr_t>(Cb) & 15) == 0 &&
                        (!Lb || ((ep.ld_lo & 3) == 0 && (reinterpret_cast<uintptr_t>(Lb) & 15) == 0));
       // the prefetch copies whole 16-byte units: the dimension they run along must be a multiple of 4
       const bool pre = PRE;
@@ -583,7 +583,7 @@ bool make_map(CUtensorMap* map, const float* base, int rows, int K, int64_t ld, 
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES, bool PRE, bool CVTA = false, bool TR = false, bool LO = false>
+template <int BN, int STAGES, bool PRE, bool CVTA = false, bool TR = false, bool LO = false, bool VEC = false>
 cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, int batch, const TcEpilogue& ep,
                    cudaStream_t s, int ksplit = 1) {
   using C = Cfg<BN, STAGES, PRE>;
@@ -597,7 +597,7 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e =
-        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
@@ -609,7 +609,7 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
   const int kblocks = (K + BK - 1) / BK;
   const int tpc = kblocks > 16 ? 1 : (int)std::max<int64_t>(1, std::min<int64_t>(8, ntiles / (4 * 152)));
   const int grid = (int)((ntiles + tpc - 1) / tpc);
-  gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
+  gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO, VEC><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
                                                                      bmod, tpc, ksplit, ep);
   return cudaGetLastError();
 }
@@ -640,13 +640,25 @@ __global__ void split_reduce_kernel(const float* P, int ksplit, int batch, int M
 
 // One instantiation per (transposed output, lo output): each kernel's epilogue then carries
 // only the store path it uses.
+// With `vec` (C and its lo part 16-byte aligned, rows of 16-byte multiples) the kernel has no
+// element-wise store path either.
+template <int BN, int STAGES, bool PRE, bool CVTA, bool VEC>
+cudaError_t launch_tlv(bool tr, bool lo, const TcOperand& A, const TcOperand& B, int M, int N, int K, int batch,
+                       const TcEpilogue& ep, cudaStream_t s) {
+  if (tr) return lo ? launch<BN, STAGES, PRE, CVTA, true, true, VEC>(A, B, M, N, K, batch, ep, s)
+                    : launch<BN, STAGES, PRE, CVTA, true, false, VEC>(A, B, M, N, K, batch, ep, s);
+  return lo ? launch<BN, STAGES, PRE, CVTA, false, true, VEC>(A, B, M, N, K, batch, ep, s)
+            : launch<BN, STAGES, PRE, CVTA, false, false, VEC>(A, B, M, N, K, batch, ep, s);
+}
 template <int BN, int STAGES, bool PRE, bool CVTA>
-cudaError_t launch_tl(bool tr, bool lo, const TcOperand& A, const TcOperand& B, int M, int N, int K, int batch,
-                      const TcEpilogue& ep, cudaStream_t s, int ksplit = 1) {
-  if (tr) return lo ? launch<BN, STAGES, PRE, CVTA, true, true>(A, B, M, N, K, batch, ep, s, ksplit)
-                    : launch<BN, STAGES, PRE, CVTA, true, false>(A, B, M, N, K, batch, ep, s, ksplit);
-  return lo ? launch<BN, STAGES, PRE, CVTA, false, true>(A, B, M, N, K, batch, ep, s, ksplit)
-            : launch<BN, STAGES, PRE, CVTA, false, false>(A, B, M, N, K, batch, ep, s, ksplit);
+cudaError_t launch_tl(bool tr, bool lo, bool vec, const TcOperand& A, const TcOperand& B, int M, int N, int K,
+                      int batch, const TcEpilogue& ep, cudaStream_t s) {
+  if constexpr (PRE) {
+    return launch_tlv<BN, STAGES, PRE, CVTA, true>(tr, lo, A, B, M, N, K, batch, ep, s);
+  } else {
+    if (vec) return launch_tlv<BN, STAGES, PRE, CVTA, true>(tr, lo, A, B, M, N, K, batch, ep, s);
+    return launch_tlv<BN, STAGES, PRE, CVTA, false>(tr, lo, A, B, M, N, K, batch, ep, s);
+  }
 }
 
 // How many K splits give the fewest idle SMs in the last wave, for a launch of `tiles` tiles
@@ -714,14 +726,17 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
     return cudaGetLastError();
   }
   const bool tr = ep.transpose != 0, lo = ep.C_lo != nullptr;
+  const bool vec = !ep.C_ptrs && ep.C && al16(ep.C) && (ep.ldc & 3) == 0 && (ep.c_stride & 3) == 0 &&
+                   ((tr ? M : N) & 3) == 0 &&
+                   (!ep.C_lo || ((ep.ld_lo & 3) == 0 && (ep.lo_stride & 3) == 0 && al16(ep.C_lo)));
   if (cvt)
-    return N <= 32 ? tc::launch_tl<32, 5, false, true>(false, lo, A, B, M, N, K, batch, ep, s)
-                   : tc::launch_tl<128, 3, false, true>(false, lo, A, B, M, N, K, batch, ep, s);
+    return N <= 32 ? tc::launch_tl<32, 5, false, true>(false, lo, vec, A, B, M, N, K, batch, ep, s)
+                   : tc::launch_tl<128, 3, false, true>(false, lo, vec, A, B, M, N, K, batch, ep, s);
   if (N <= 32)
-    return pre ? tc::launch_tl<32, 4, true, false>(tr, lo, A, B, M, N, K, batch, ep, s)
-               : tc::launch_tl<32, 5, false, false>(tr, lo, A, B, M, N, K, batch, ep, s);
-  return pre ? tc::launch_tl<128, 2, true, false>(tr, lo, A, B, M, N, K, batch, ep, s)
-             : tc::launch_tl<128, 3, false, false>(tr, lo, A, B, M, N, K, batch, ep, s);
+    return pre ? tc::launch_tl<32, 4, true, false>(tr, lo, vec, A, B, M, N, K, batch, ep, s)
+               : tc::launch_tl<32, 5, false, false>(tr, lo, vec, A, B, M, N, K, batch, ep, s);
+  return pre ? tc::launch_tl<128, 2, true, false>(tr, lo, vec, A, B, M, N, K, batch, ep, s)
+             : tc::launch_tl<128, 3, false, false>(tr, lo, vec, A, B, M, N, K, batch, ep, s);
 }
 
 }  // namespace soap
