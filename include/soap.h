@@ -273,6 +273,22 @@ soap_status_t soap_gemm_tf32x4(int32_t M, int32_t N, int32_t K, int32_t batch, c
  * fp32) rounded to the nearest tf32, for n values on the device; hi may be NULL. */
 soap_status_t soap_split_tf32(const float* x, float* hi, float* lo, int64_t n, soap_stream_t stream);
 
+/* Layer-wise ownership for data-parallel ranks (section 6, "layer-wise distributed
+ * optimizer"): every matrix is stepped by exactly one of `world` ranks, which then share the
+ * updated weights with the others (an all-gather of variable-size pieces). Host-only; no
+ * device is touched.
+ *   policy 0: the paper's assignment -- matrices sorted by size (rows * cols, largest first,
+ *             ties by index) and dealt round-robin to ranks 0, 1, ..., world-1, 0, ...
+ *   policy 1: longest processing time first on this library's step cost -- the same order,
+ *             each matrix to the rank with the smallest cost so far (ties: lowest rank), the
+ *             cost of a matrix being the FLOPs of its SOAP step (S1 as a symmetric product,
+ *             the power step, the QR, the rotations), identity sides dropped
+ * owner[i] receives matrix i's rank; load[r] (may be NULL) receives rank r's summed cost
+ * (FLOPs, under either policy). SOAP_ERR_INVALID_ARG for n < 1, world < 1, a null shapes or
+ * owner, an unknown policy or a non-positive side. */
+soap_status_t soap_layerwise_assign(const soap_shape* shapes, int32_t n, int32_t world, int32_t policy,
+                                    int32_t* owner, double* load);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1085,6 +1085,42 @@ soap_status_t soap_profile_records(soap_handle h, soap_launch_record* out, int64
   return SOAP_OK;
 }
 
+soap_status_t soap_layerwise_assign(const soap_shape* shapes, int32_t n, int32_t world, int32_t policy,
+                                    int32_t* owner, double* load) {
+  if (!shapes || !owner || n < 1 || world < 1 || (policy != 0 && policy != 1)) return SOAP_ERR_INVALID_ARG;
+  for (int i = 0; i < n; ++i)
+    if (shapes[i].rows < 1 || shapes[i].cols < 1) return SOAP_ERR_INVALID_ARG;
+  // the step's FLOPs for one matrix (2 per multiply-add): S1 as a symmetric product, the power
+  // step, Householder QR with explicit Q, and the rotations of G, m and N per preconditioned side
+  auto cost = [&](const soap_shape& s) {
+    const double m = (double)s.rows, c = (double)s.cols;
+    double f = 0.0;
+    if (s.precond_left) f += m * m * c + 2 * m * m * m + (8.0 / 3.0) * m * m * m + 8 * m * m * c;
+    if (s.precond_right) f += c * c * m + 2 * c * c * c + (8.0 / 3.0) * c * c * c + 8 * m * c * c;
+    return f + 10 * m * c;  // the elementwise work
+  };
+  std::vector<int> order(n);
+  for (int i = 0; i < n; ++i) order[i] = i;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) {
+    return shapes[a].rows * shapes[a].cols > shapes[b].rows * shapes[b].cols;
+  });
+  std::vector<double> l(world, 0.0);
+  for (int q = 0; q < n; ++q) {
+    const int i = order[q];
+    int r = q % world;
+    if (policy == 1) {
+      r = 0;
+      for (int k = 1; k < world; ++k)
+        if (l[k] < l[r]) r = k;
+    }
+    owner[i] = r;
+    l[r] += cost(shapes[i]);
+  }
+  if (load)
+    for (int r = 0; r < world; ++r) load[r] = l[r];
+  return SOAP_OK;
+}
+
 size_t soap_qr_workspace_bytes(int32_t n, int32_t batch) {
   if (n <= 0 || batch <= 0) return 0;
   return soap::qr_workspace_bytes(n, batch) + 256;

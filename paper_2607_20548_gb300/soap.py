@@ -28,7 +28,7 @@ EXPORTS = ("soap_default_hparams", "soap_create", "soap_step", "soap_set_lr", "s
            "soap_clear_status", "soap_last_error", "soap_destroy", "soap_qr_workspace_bytes",
            "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_profile_records",
            "soap_gemm_tf32x4",
-           "soap_split_tf32", "soap_qr_static")
+           "soap_split_tf32", "soap_qr_static", "soap_layerwise_assign")
 # every symbol include/muon.h declares
 MUON_EXPORTS = ("muon_default_hparams", "muon_create", "muon_step", "muon_set_lr", "muon_state_get",
                 "muon_state_set", "muon_status", "muon_last_error", "muon_destroy", "muon_profile_begin",
@@ -106,6 +106,8 @@ def load_library(path: str = LIB_PATH):
                                    I32, P, P, P]),
         "soap_split_tf32": (I32, [P, P, P, I64, P]),
         "soap_qr_static": (I32, [I32, I32, P, P, P, F, P]),
+        "soap_layerwise_assign": (I32, [ctypes.POINTER(soap_shape), I32, I32, I32, ctypes.POINTER(I32),
+                                        ctypes.POINTER(ctypes.c_double)]),
         "muon_default_hparams": (None, [ctypes.POINTER(muon_hparams)]),
         "muon_create": (I32, [ctypes.POINTER(soap_shape), I32, ctypes.POINTER(muon_hparams), I32, ctypes.POINTER(P)]),
         "muon_step": (I32, [P, P, P, P]),
@@ -498,3 +500,16 @@ class MuonOptimizer:
             self.destroy()
         except Exception:
             pass
+
+
+def layerwise_assign(shapes, world: int, policy: int = 0):
+    """soap_layerwise_assign: (owner per matrix, cost per rank) for `world` ranks."""
+    n = len(shapes)
+    arr = (soap_shape * n)(*[soap_shape(int(s[0]), int(s[1]), int(s[2]) if len(s) > 2 else 1,
+                                        int(s[3]) if len(s) > 3 else 1) for s in shapes])
+    owner = (ctypes.c_int32 * n)()
+    load = (ctypes.c_double * world)()
+    code = load_library().soap_layerwise_assign(arr, n, world, policy, owner, load)
+    if code != SOAP_OK:
+        raise SoapError(code, "soap_layerwise_assign")
+    return list(owner), list(load)

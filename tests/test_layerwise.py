@@ -1,0 +1,90 @@
+"""Layer-wise ownership (section 6): the planner (C ABI, host-only) and the all-gather of the
+updated weights across ranks, with world_size 2 on gloo (CPU; no GPU involved)."""
+import ctypes
+import os
+import socket
+
+import numpy as np
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+from paper_2607_20548_gb300 import soap as S
+from paper_2607_20548_gb300.layerwise import LayerwiseOptimizer
+from paper_2607_20548_gb300.workloads import WORKLOADS
+
+BLOCK = [(s.rows, s.cols, int(s.left), int(s.right)) for s in WORKLOADS["dense_block_h2048_ffn8192"][0]]
+
+
+def test_paper_assignment_is_size_sorted_round_robin():
+    """Policy 0: sorted by rows * cols (largest first, ties by index) and dealt round-robin."""
+    shapes = [(4, 4), (8, 8), (2, 2), (8, 8), (6, 6)]
+    owner, _ = S.layerwise_assign(shapes, 2, 0)
+    # order: (8,8)#1, (8,8)#3, (6,6)#4, (4,4)#0, (2,2)#2 -> ranks 0, 1, 0, 1, 0
+    assert owner == [1, 0, 0, 1, 0]
+    owner3, _ = S.layerwise_assign(shapes, 3, 0)
+    assert owner3 == [0, 0, 1, 1, 2]
+
+
+def test_lpt_assignment_balances_cost_and_covers_every_matrix():
+    """Policy 1 gives every matrix one owner and no rank more than the largest single matrix's
+    cost above the lightest rank (the LPT bound); the loads add up to the whole step."""
+    for world in (1, 2, 3, 4, 8):
+        owner, load = S.layerwise_assign(BLOCK, world, 1)
+        assert len(owner) == len(BLOCK) and all(0 <= o < world for o in owner)
+        _, total = S.layerwise_assign(BLOCK, 1, 1)
+        assert abs(sum(load) - total[0]) <= 1e-9 * total[0]
+        _, single = zip(*[S.layerwise_assign([s], 1, 1) for s in BLOCK])
+        assert max(load) - min(load) <= max(x[0] for x in single) * (1 + 1e-12)
+
+
+def test_planner_rejects_bad_arguments():
+    lib = S.load_library()
+    arr = (S.soap_shape * 1)(S.soap_shape(4, 4, 1, 1))
+    own = (ctypes.c_int32 * 1)()
+    assert lib.soap_layerwise_assign(arr, 1, 0, 0, own, None) == 1
+    assert lib.soap_layerwise_assign(arr, 1, 2, 5, own, None) == 1
+    bad = (S.soap_shape * 1)(S.soap_shape(0, 4, 1, 1))
+    assert lib.soap_layerwise_assign(bad, 1, 2, 0, own, None) == 1
+
+
+class _Descent:
+    """A stand-in local optimizer for the exchange test: W <- W - 0.5 G on the owned matrices."""
+
+    def __init__(self, shapes):
+        self.shapes = shapes
+
+    def step(self, params, grads):
+        for p, g in zip(params, grads):
+            p.sub_(0.5 * g)
+
+
+def _worker(rank, world, port, shapes, out):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        g = torch.Generator().manual_seed(0)
+        W = [torch.randn(r, c, generator=g) for r, c in shapes]
+        W0 = [w.clone() for w in W]
+        G = [torch.randn(r, c, generator=g) for r, c in shapes]
+        opt = LayerwiseOptimizer(shapes, _Descent)
+        opt.step(W, G)
+        for w, w0, gg in zip(W, W0, G):
+            # every matrix was stepped exactly once, by its owner, and every rank holds the result
+            assert torch.equal(w, w0 - 0.5 * gg)
+        out[rank] = opt.mine
+    finally:
+        dist.destroy_process_group()
+
+
+def test_exchange_world_size_2_gloo():
+    shapes = [(12, 20), (20, 12), (8, 8), (16, 4), (4, 16), (12, 20)]
+    with socket.socket() as sock:
+        sock.bind(("127.0.0.1", 0))
+        port = sock.getsockname()[1]
+    mgr = mp.Manager()
+    out = mgr.dict()
+    mp.spawn(_worker, args=(2, port, shapes, out), nprocs=2, join=True)
+    owned = sorted(out[0] + out[1])
+    assert owned == list(range(len(shapes)))
