@@ -9,11 +9,15 @@ fixed FLOP model of Alg. 1 (S1 as a SYRK, S2 power step, S3 Householder QR with 
 Q, S4 re-projection with four two-sided products, S5/S7 rotations).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {soap,reference}] [--kl]
+                  [--optimizer {soap,muon}] [--layerwise] [--matrices i,j,...]
 
 N > 1 (torchrun, one rank per GPU) runs N independent replicas of the block: the step
 has no exchange, so value = N * K / max-over-ranks time. --impl reference times the
 fp64 CPU oracle on the host cores instead (rank 0 only). --kl runs Alg. 1's KL-Shampoo
-factor form instead of the standard factor EMAs (a separate line, not the headline).
+factor form instead of the standard factor EMAs, --optimizer muon the paper's Muon step,
+and --layerwise (N > 1) one block stepped by all ranks, each owning whole matrices
+(section 6) and all-gathering the updated weights; these are separate lines, not the
+headline.
 """
 from __future__ import annotations
 
@@ -260,7 +264,17 @@ def run_soap(args):
         specs = [specs[j] for j in subset]
     gen = make_stream(WORKLOAD, seed=rank, device=dev, specs=subset)
     muon = args.optimizer == "muon"
-    if muon:
+    layerwise = args.layerwise and world > 1
+    if layerwise:
+        # one model stepped by all ranks: each owns whole matrices (section 6) and the updated
+        # weights are all-gathered over NCCL after every step
+        from paper_2607_20548_gb300.layerwise import LayerwiseOptimizer
+        nccl = dist.new_group(backend="nccl")
+        gen = make_stream(WORKLOAD, seed=0, device=dev, specs=subset)
+        hp = default_hparams(kl=int(args.kl))
+        opt = LayerwiseOptimizer([(s.rows, s.cols, int(s.left), int(s.right)) for s in specs],
+                                 lambda sh: SoapOptimizer(sh, hp, device=local), group=nccl, policy=1)
+    elif muon:
         opt = S.MuonOptimizer([(s.rows, s.cols) for s in specs], ns_steps=MUON_NS_STEPS, device=local)
     else:
         opt = SoapOptimizer([(s.rows, s.cols, s.left, s.right) for s in specs], default_hparams(kl=int(args.kl)),
@@ -311,7 +325,9 @@ def run_soap(args):
         tt = torch.tensor([elapsed], dtype=torch.float64)
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         elapsed = float(tt.item())
-    value = world * args.steps / elapsed
+    # replicas: N models per step; layer-wise: one model per step, stepped by all ranks
+    units = 1 if layerwise else world
+    value = units * args.steps / elapsed
 
     # end to end through the public API: pinned host gradients in, updated weights out
     host_g = [[g.cpu().pin_memory() for g in pool[i]] for i in range(npool)]
@@ -361,17 +377,19 @@ def run_soap(args):
     line = {
         "metric": MUON_METRIC if muon else METRIC, "value": value, "unit": "steps/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if muon else "f32",
+        "higher_is_better": True, "scaling": "strong" if layerwise else "weak", "vs_baseline": None,
+        "dtype": "bf16" if muon else "f32",
         "data": "synthetic",
         "config": {"workload": WORKLOAD if not subset else f"{WORKLOAD}[matrices {args.matrices}]",
                    "matrices": len(specs),
                    "shapes": "4x 2048x2048, 2x 2048x8192, 1x 8192x2048, all sides preconditioned",
-                   "parallelism": "replicas" if world > 1 else "single",
+                   "parallelism": f"layerwise{world}" if layerwise else ("replicas" if world > 1 else "single"),
                    "optimizer": "muon (16 quintic Newton-Schulz steps)" if muon else
                    ("soap, KL factor form" if args.kl else "soap, standard factor form"),
                    "l2": "inputs larger than L2 (3 GB of optimizer state per step)"},
         "effective_tflops": block_flops * value / world / 1e12,
         "effective_frac_of_tensor_peak": block_flops * value / world / 1e12 / tc_peak,
+        "effective_note": "per GPU (the whole-job FLOP rate divided by the number of GPUs)",
         "model_flop_per_step": block_flops,
         "roofline": roof,
         "kernel_time_share": {k: round(v["ms"] / max(1e-9, sum(x["ms"] for x in fams.values())), 4)
@@ -383,7 +401,7 @@ def run_soap(args):
         "cpu_baseline": {"value": sps, "unit": "steps/s", "cores": threads, "kind": "oracle",
                          "sample": f"one fp64 oracle {'Muon' if muon else 'SOAP'} step of Wq (2048x2048) took "
                                    f"{per:.1f} s; whole block = {scale:.1f}x that by the FLOP model"},
-        "e2e": {"value": world * args.steps / e2e_s, "unit": "steps/s", "h2d_bytes_per_step": h2d,
+        "e2e": {"value": units * args.steps / e2e_s, "unit": "steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
         "clocks": clk.summary(),
@@ -403,6 +421,9 @@ def main():
                          "default: all 7")
     ap.add_argument("--optimizer", choices=["soap", "muon"], default="soap",
                     help="muon: the paper's Muon step on the same block (a separate line, not the headline)")
+    ap.add_argument("--layerwise", action="store_true",
+                    help="with N > 1: one model, each rank stepping its own matrices (section 6) and "
+                         "all-gathering the updated weights over NCCL (strong scaling)")
     ap.add_argument("--kl", action="store_true",
                     help="KL-Shampoo factor form (Alg. 1's factor accumulation) instead of the standard EMAs")
     args = ap.parse_args()

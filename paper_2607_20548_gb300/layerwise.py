@@ -62,3 +62,27 @@ class LayerwiseOptimizer:
                     k = params[i].numel()
                     params[i].copy_(buf[off:off + k].view_as(params[i]))
                     off += k
+
+    # the local optimizer's status and profiling, for a caller that treats this like one handle
+    def status(self) -> int:
+        return self.opt.status() if self.opt is not None else 0
+
+    def last_error(self) -> str:
+        return self.opt.last_error() if self.opt is not None else ""
+
+    def profile_begin(self, max_launches: int = 1 << 16):
+        if self.opt is not None:
+            self.opt.profile_begin(max_launches)
+
+    def profile_end(self) -> dict:
+        if self.opt is not None:
+            return self.opt.profile_end()
+        from .soap import KERNEL_FAMILIES
+        res = {k: dict(launches=0, ms=0.0, flops=0.0, bytes=0.0) for k in KERNEL_FAMILIES}
+        res["overflow"] = False
+        return res
+
+    def destroy(self):
+        if self.opt is not None:
+            self.opt.destroy()
+            self.opt = None
