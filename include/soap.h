@@ -171,7 +171,7 @@ void soap_destroy(soap_handle h);
 /* Kernel families the library launches. */
 typedef enum {
   SOAP_KERNEL_GEMM_SIMT = 0,   /* CUDA-core fp32 batched GEMM */
-  SOAP_KERNEL_GEMM_TC = 1,     /* tcgen05 fp32-accurate batched GEMM (four TF32 products) */
+  SOAP_KERNEL_GEMM_TC = 1,     /* tcgen05 batched GEMM: fp32-accurate (four TF32 products), or bf16 (Muon) */
   SOAP_KERNEL_QR_PANEL = 2,    /* cluster panel factorisation of the QR */
   SOAP_KERNEL_ELEMENTWISE = 3, /* momentum, Adam, weight update */
   SOAP_KERNEL_OTHER = 4,       /* norms, identity fills */

@@ -14,11 +14,11 @@ namespace soap {
 
 enum KernelFamily : int {
   kFamGemmSimt = 0,   // CUDA-core fp32 GEMM
-  kFamGemmTc = 1,     // tcgen05 3xTF32 GEMM
+  kFamGemmTc = 1,     // tcgen05 GEMM: fp32 as four TF32 products, or bf16 (Muon)
   kFamQrPanel = 2,    // cluster panel factorisation of the QR
   kFamElementwise = 3,// momentum / Adam / weight update
   kFamOther = 4,      // norms, identity fills
-  kFamQrUpdate = 5,   // tensor-core products of the QR's block updates (HBM-bound)
+  kFamQrUpdate = 5,   // tensor-core products of the QR's block updates (at the roofline ridge)
   kNumFamilies = 6,
 };
 

@@ -50,7 +50,7 @@ cudaError_t gemm(bool trans_a, bool trans_b, int M, int N, int K, float alpha, O
 cudaError_t gemm_simt(bool trans_a, bool trans_b, int M, int N, int K, float alpha, Operand A,
                       Operand B, float beta, MutOperand C, int batch, cudaStream_t stream);
 
-// ---- tcgen05 3xTF32 engine: C_b = alpha * A_b B_(b mod B.batch)^T + beta * C_b ----------
+// ---- tcgen05 fp32 engine (four TF32 products): C_b = alpha * A_b B_(b mod B.batch)^T + beta * C_b
 // An operand is `batch` row-major (rows x K) matrices split as hi = trunc_tf32(x) (the fp32
 // array itself may serve: the tensor core drops the 13 low mantissa bits) and lo = x - hi.
 struct TcOperand {
