@@ -245,6 +245,58 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def library_sample(specs, pool, dev, steps=2):
+    """Context only: the same standard-form SOAP step written with library calls (torch fp32
+    matmul with TF32 off, cuSOLVER QR through torch.linalg.qr), per matrix, on the same GPU.
+    Returns (steps/s, note) or (None, reason)."""
+    try:
+        prev = torch.backends.cuda.matmul.allow_tf32
+        torch.backends.cuda.matmul.allow_tf32 = False
+        b, b1, b2, eps, lr, wd = 0.95, 0.95, 0.95, 1e-8, 3e-3, 0.1
+        st = []
+        for s_ in specs:
+            m, n = s_.rows, s_.cols
+            st.append(dict(L=torch.zeros(m, m, device=dev), R=torch.zeros(n, n, device=dev),
+                           QL=torch.eye(m, device=dev), QR=torch.eye(n, device=dev),
+                           Mh=torch.zeros(m, n, device=dev), V=torch.zeros(m, n, device=dev),
+                           W=torch.zeros(m, n, device=dev)))
+
+        def qr_pos(P):
+            Q, Rr = torch.linalg.qr(P)
+            d = torch.sign(torch.diagonal(Rr))
+            return Q * torch.where(d == 0, torch.ones_like(d), d)
+
+        def one(G_all):
+            for x, G in zip(st, G_all):
+                x["L"].mul_(b).addmm_(G, G.T, alpha=1 - b)
+                x["R"].mul_(b).addmm_(G.T, G, alpha=1 - b)
+                x["Mh"].mul_(b1).add_(G, alpha=1 - b1)
+                x["QL"] = qr_pos(x["L"] @ x["QL"])
+                x["QR"] = qr_pos(x["R"] @ x["QR"])
+                Gp = x["QL"].T @ G @ x["QR"]
+                mp = x["QL"].T @ x["Mh"] @ x["QR"]
+                x["V"].mul_(b2).addcmul_(Gp, Gp, value=1 - b2)
+                N = mp / (x["V"].sqrt() + eps)
+                x["W"].mul_(1 - lr * wd).sub_(x["QL"] @ N @ x["QR"].T, alpha=lr)
+
+        one(pool[0])
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for t in range(steps):
+            one(pool[(t + 1) % len(pool)])
+        e1.record()
+        torch.cuda.synchronize()
+        torch.backends.cuda.matmul.allow_tf32 = prev
+        del st
+        torch.cuda.empty_cache()
+        return steps / (e0.elapsed_time(e1) / 1e3), (
+            f"the standard-form step per matrix with torch fp32 matmul (TF32 off) and torch.linalg.qr "
+            f"(cuSOLVER), sign-fixed; {steps} steps after one warm-up, same GPU and gradients")
+    except Exception as e:  # context only: never fails the bench
+        return None, f"unavailable: {type(e).__name__}: {str(e)[:200]}"
+
+
 def run_soap(args):
     rank, world, local = dist_env()
     torch.cuda.set_device(local)
@@ -373,6 +425,10 @@ def run_soap(args):
         # the DRAM/algorithmic ratios above were measured for the fp32 (tf32 x4) kernels
         roof["traffic"], roof["traffic_note"] = None, "not measured for the bf16 kernel"
     per, sps, threads, scale = muon_oracle_sample() if muon else oracle_sample(1, 0, args.kl)
+    lib_line = None
+    if not (muon or args.kl or layerwise or subset):
+        lib_v, lib_note = library_sample(specs, pool, dev)
+        lib_line = {"value": lib_v, "unit": "steps/s", "kind": "torch + cuSOLVER", "sample": lib_note}
     tc_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]) / (1.0 if muon else 2.0 * TC_PRODUCTS)
     line = {
         "metric": MUON_METRIC if muon else METRIC, "value": value, "unit": "steps/s", "n_gpus": world,
@@ -405,6 +461,7 @@ def run_soap(args):
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
         "clocks": clk.summary(),
+        "library_baseline": lib_line,
     }
     print(json.dumps(line), flush=True)
     opt.destroy()
