@@ -10,7 +10,7 @@ import torch.distributed as dist
 import torch.multiprocessing as mp
 
 from paper_2607_20548_gb300 import soap as S
-from paper_2607_20548_gb300.layerwise import LayerwiseOptimizer
+from paper_2607_20548_gb300.layerwise import LayerwiseOptimizer, plan_buckets
 from paper_2607_20548_gb300.workloads import WORKLOADS
 
 BLOCK = [(s.rows, s.cols, int(s.left), int(s.right)) for s in WORKLOADS["dense_block_h2048_ffn8192"][0]]
@@ -46,6 +46,19 @@ def test_planner_rejects_bad_arguments():
     assert lib.soap_layerwise_assign(arr, 1, 2, 5, own, None) == 1
     bad = (S.soap_shape * 1)(S.soap_shape(0, 4, 1, 1))
     assert lib.soap_layerwise_assign(bad, 1, 2, 0, own, None) == 1
+
+
+def test_buckets_are_consecutive_and_bounded():
+    shapes = [(4, 4), (4, 4), (8, 8), (2, 2), (16, 16), (2, 2), (2, 2)]   # 64, 64, 256, 16, 1024, 16, 16 B
+    assert plan_buckets(shapes) == [list(range(7))]
+    assert plan_buckets([]) == []
+    b = plan_buckets(shapes, bucket_bytes=256)
+    # in order, nothing skipped or repeated; a bucket only exceeds the bound when it holds one matrix
+    assert [i for bkt in b for i in bkt] == list(range(7))
+    assert b == [[0, 1], [2], [3], [4], [5, 6]]
+    for bkt in b:
+        assert len(bkt) == 1 or sum(shapes[i][0] * shapes[i][1] * 4 for i in bkt) <= 256
+    assert plan_buckets(shapes, bucket_bytes=1) == [[i] for i in range(7)]
 
 
 class _Descent:
@@ -88,3 +101,46 @@ def test_exchange_world_size_2_gloo():
     mp.spawn(_worker, args=(2, port, shapes, out), nprocs=2, join=True)
     owned = sorted(out[0] + out[1])
     assert owned == list(range(len(shapes)))
+
+
+def _overlap_worker(rank, world, port, shapes, policy, bucket_bytes, out):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        g = torch.Generator().manual_seed(1)
+        W = [torch.randn(r, c, generator=g) for r, c in shapes]
+        W0 = [w.clone() for w in W]
+        G = [torch.randn(r, c, generator=g) for r, c in shapes]
+        opt = LayerwiseOptimizer(shapes, _Descent, policy=policy, bucket_bytes=bucket_bytes)
+        assert len(opt.buckets) > 1
+        pending = opt.step(W, G, overlap=True)
+        for b, bkt in enumerate(opt.buckets):
+            for i in bkt:
+                # a matrix another rank owns keeps its old value until its bucket is waited for
+                want_before = W0[i] - 0.5 * G[i] if opt.owner[i] == rank else W0[i]
+                assert torch.equal(W[i], want_before)
+            pending.wait(b)
+            for i in bkt:
+                assert torch.equal(W[i], W0[i] - 0.5 * G[i])
+        pending.wait_all()
+        # a second step through the blocking path agrees with the same rule
+        W1 = [w.clone() for w in W]
+        opt.step(W, G)
+        for w, w1, gg in zip(W, W1, G):
+            assert torch.equal(w, w1 - 0.5 * gg)
+        out[rank] = opt.mine
+    finally:
+        dist.destroy_process_group()
+
+
+def test_bucketed_overlapped_exchange_world_size_2_gloo():
+    shapes = [(12, 20), (20, 12), (8, 8), (16, 4), (4, 16), (12, 20), (30, 2), (2, 30)]
+    for policy in (0, 1):
+        with socket.socket() as sock:
+            sock.bind(("127.0.0.1", 0))
+            port = sock.getsockname()[1]
+        mgr = mp.Manager()
+        out = mgr.dict()
+        mp.spawn(_overlap_worker, args=(2, port, shapes, policy, 1000, out), nprocs=2, join=True)
+        assert sorted(out[0] + out[1]) == list(range(len(shapes)))
