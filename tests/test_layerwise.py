@@ -144,3 +144,50 @@ def test_bucketed_overlapped_exchange_world_size_2_gloo():
         out = mgr.dict()
         mp.spawn(_overlap_worker, args=(2, port, shapes, policy, 1000, out), nprocs=2, join=True)
         assert sorted(out[0] + out[1]) == list(range(len(shapes)))
+
+
+def _departing_worker(rank, world, port, shapes, out):
+    """Rank 1 leaves between steps (no collective of its own in flight); rank 0's next exchange
+    must end with an error from the process group, not wait forever."""
+    import datetime
+    import time
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world, timeout=datetime.timedelta(seconds=10))
+    g = torch.Generator().manual_seed(2)
+    W = [torch.randn(r, c, generator=g) for r, c in shapes]
+    G = [torch.randn(r, c, generator=g) for r, c in shapes]
+    opt = LayerwiseOptimizer(shapes, _Descent)
+    opt.step(W, G)                       # one good step on both ranks
+    if rank == 1:
+        out[rank] = "left"
+        os._exit(0)                      # gone without a goodbye
+    t0 = time.monotonic()
+    try:
+        opt.step(W, G)
+        out[rank] = "no error"
+    except Exception as e:  # noqa: BLE001 - any process-group error is the expected outcome
+        out[rank] = f"raised after {time.monotonic() - t0:.1f} s: {type(e).__name__}"
+    os._exit(0)
+
+
+def test_exchange_with_a_departed_rank_raises_instead_of_hanging():
+    shapes = [(12, 20), (20, 12), (8, 8), (16, 4)]
+    with socket.socket() as sock:
+        sock.bind(("127.0.0.1", 0))
+        port = sock.getsockname()[1]
+    ctx = mp.get_context("spawn")
+    mgr = ctx.Manager()
+    out = mgr.dict()
+    procs = [ctx.Process(target=_departing_worker, args=(r, 2, port, shapes, out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=120)
+    alive = [p for p in procs if p.is_alive()]
+    for p in alive:
+        p.kill()                         # only the processes this test started
+        p.join()
+    assert not alive, "a rank hung in the exchange"
+    assert out.get(1) == "left"
+    assert str(out.get(0, "")).startswith("raised after"), out.get(0)
