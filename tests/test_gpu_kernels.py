@@ -55,7 +55,8 @@ def _qr_case(n, batch, kind, seed):
 
 @pytest.mark.parametrize("n,batch,kind", [(4, 1, "well"), (36, 2, "well"), (32, 1, "gauss"), (36, 3, "gauss"),
                                           (100, 2, "lowrank"), (516, 2, "well"), (1028, 1, "well"),
-                                          (768, 2, "lowrank"), (2048, 1, "well"), (2048, 1, "lowrank")])
+                                          (768, 2, "lowrank"), (2048, 1, "well"), (2048, 1, "lowrank"),
+                                          (200, 2, "lowrank"), (644, 1, "gauss")])
 def test_qr_matches_oracle(cuda, n, batch, kind):
     """S3 on identical fp32 inputs: skip flags equal the oracle's, Q^T Q = I to 1e-5, and Q agrees
     with the fp64 oracle to within 4x the oracle's own fp32 twin (the problem's fp32 resolution)."""
