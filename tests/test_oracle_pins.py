@@ -147,6 +147,48 @@ def test_zero_gradient_is_pure_weight_decay():
     assert st.skipL.all() and st.skipR.all()
 
 
+def test_basis_frequency_refreshes_only_every_f_steps():
+    """Eigenbasis frequency F = 4 (Alg. 1 refreshes when t mod F = 0): steps 1-3 keep Q = I and
+    are AdamW in closed form for any gradients; step 4 takes Q from the library QR of L_4 Q = L_4
+    (and R_4) with the sign fix, re-projects m but not v (Alg. 1 re-projects only m), and rotates;
+    steps 5-7 keep that basis while the factors move on."""
+    rows, cols, F = 6, 5, 4
+    b, b1, b2, eps, lr, wd = 0.95, 0.9, 0.99, 1e-8, 1e-2, 0.1
+    hp = HParams(lr=lr, weight_decay=wd, beta1=b1, beta2=b2, factor_beta=b, eps=eps, eig_every=F)
+    rng = np.random.default_rng(77)
+    st = MatrixState(rows, cols, True, True)
+    W = rng.standard_normal((rows, cols))
+    m, v = np.zeros((rows, cols)), np.zeros((rows, cols))
+    L, R = np.zeros((rows, rows)), np.zeros((cols, cols))
+    QL, QR = np.eye(rows), np.eye(cols)
+
+    def signed_q(P):
+        q, r = np.linalg.qr(P)
+        return q * np.where(np.diag(r) < 0, -1.0, 1.0)
+
+    for t in range(1, 8):
+        G = rng.standard_normal((rows, cols))
+        L = b * L + (1 - b) * G @ G.T
+        R = b * R + (1 - b) * G.T @ G
+        if t % F == 0:
+            newL, newR = signed_q(L @ QL), signed_q(R @ QR)
+            m = newL.T @ (QL @ m @ QR.T) @ newR
+            QL, QR = newL, newR
+        Gp = QL.T @ G @ QR
+        m = b1 * m + (1 - b1) * Gp
+        v = b2 * v + (1 - b2) * Gp * Gp
+        want = (1 - lr * wd) * W - lr * QL @ (m / (np.sqrt(v) + eps)) @ QR.T
+        W, _ = soap_step(st, W, G, hp)
+        np.testing.assert_allclose(W, want, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(st.QL, QL, atol=1e-12)
+        np.testing.assert_allclose(st.QR, QR, atol=1e-12)
+        np.testing.assert_allclose(st.v, v, atol=1e-14)
+        if t < F:
+            assert np.array_equal(st.QL, np.eye(rows)) and np.array_equal(st.QR, np.eye(cols))
+    assert not st.skipL.any() and not st.skipR.any()
+    assert not np.allclose(QL, np.eye(rows))
+
+
 # ---- S7: update-RMS invariance ------------------------------------------------------
 
 def test_update_norm_equals_adam_norm():
