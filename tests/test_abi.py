@@ -81,3 +81,15 @@ def test_host_side_validation_needs_no_gpu():
     assert lib.muon_create(good, 1, ctypes.byref(mh), 0, ctypes.byref(h)) == 1
     assert lib.muon_last_error(None) == b"null handle"
     lib.muon_destroy(None)
+
+
+def test_missing_library_fails_loudly():
+    """Without libsoap.so the binding raises; there is no other path that computes the step."""
+    import pytest
+    saved = S._lib
+    S._lib = None
+    try:
+        with pytest.raises(ImportError, match="libsoap.so not built"):
+            S.load_library(os.path.join(ROOT, "no_such_dir", "libsoap.so"))
+    finally:
+        S._lib = saved
