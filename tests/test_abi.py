@@ -93,3 +93,20 @@ def test_missing_library_fails_loudly():
             S.load_library(os.path.join(ROOT, "no_such_dir", "libsoap.so"))
     finally:
         S._lib = saved
+
+
+def test_product_code_shares_nothing_with_the_oracle():
+    """The package (binding, workloads, CUDA sources) neither imports nor includes anything from
+    oracle/; only tests, the smoke entry and the bench's CPU baseline use the oracle."""
+    pkg = os.path.join(ROOT, "paper_2607_20548_gb300")
+    pat = re.compile(r"^\s*(from\s+oracle\b|import\s+oracle\b|#\s*include\s*[<\"][^>\"]*oracle)", re.M)
+    offenders = []
+    for dirpath, _, files in os.walk(pkg):
+        if "_build" in dirpath or "_lib" in dirpath or "__pycache__" in dirpath:
+            continue
+        for f in files:
+            if f.endswith((".py", ".cu", ".h", ".cuh", ".cpp", ".c")):
+                text = open(os.path.join(dirpath, f)).read()
+                if pat.search(text):
+                    offenders.append(f)
+    assert not offenders, offenders
