@@ -110,3 +110,7 @@ def test_product_code_shares_nothing_with_the_oracle():
                 if pat.search(text):
                     offenders.append(f)
     assert not offenders, offenders
+    for f in os.listdir(os.path.join(ROOT, "oracle")):
+        if f.endswith((".py", ".c", ".h")):
+            text = open(os.path.join(ROOT, "oracle", f)).read()
+            assert "paper_2607_20548_gb300" not in text and "csrc" not in text, f
