@@ -2,9 +2,12 @@
 //
 // Plan: matrices with the same (rows, cols, sides) form a class; each class keeps
 // its state in contiguous arenas ([count][rows][cols], [count][rows][rows], ...)
-// so every contraction of the step is one batched GEMM per class. Classes run one
-// after another on the caller's stream and share one workspace sized for the
-// largest class.
+// so every contraction of the step is one batched GEMM per class. The classes' own
+// launches go to the caller's stream (prepared largest factor first, rotated smallest
+// first) and share one workspace sized for the largest class; the QR refreshes are
+// regrouped by factor size, one batched QR per size on its own pair of streams, forked
+// as soon as the last class feeding it is prepared and joined by events before the
+// classes whose bases it refreshes are rotated.
 //
 // Per class, the step (Alg. 1 with the standard factor EMAs of section 2) is:
 //   M_hat <- b1 M_hat + (1-b1) G, Gc <- G                 momentum in the original basis
