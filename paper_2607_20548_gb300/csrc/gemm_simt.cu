@@ -1,8 +1,9 @@
 // Batched fp32 GEMM on the CUDA cores: C_b = alpha * op(A_b) op(B_b) + beta * C_b.
 //
 // Exact fp32 FMAs, so it is the accuracy reference for the tensor-core path and
-// the engine for shapes too small or too skinny for tcgen05 tiles (the panel
-// updates of the QR with K = 32, the 64-wide router factor).
+// the engine where the tcgen05 path does not apply: the whole step of a class with a
+// side that is not a multiple of 4 (TMA copies 16-byte rows), and the basis changes
+// of the first moment in soap_state_get/set.
 //
 // Tiling: BM x BN output tile per 256-thread CTA, BK = 8, each thread owns a
 // (BM/16) x (BN/16) micro-tile at rows ty + 16 i and columns tx + 16 j, operands
