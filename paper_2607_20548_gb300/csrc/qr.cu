@@ -62,7 +62,7 @@ constexpr int PT = 512;           // threads per panel CTA
 constexpr int MAXC = 16;          // largest cluster (16 needs the non-portable cluster size)
 constexpr int NWARP = PT / 32;
 constexpr int NREST = NBO - NB;   // most block rows after a panel
-constexpr int KSPLIT = 8;         // most K splits of the block products W = At Vt^T
+constexpr int KSPLIT = 8;         // split-K workspace: 8 partial n x NBO products (shorter ones split up to 16 ways)
 
 // lo part of x for the tensor-core products: x - trunc_tf32(x) rounded to the nearest tf32
 __device__ __forceinline__ float tf32_lo(float x) {
