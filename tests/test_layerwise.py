@@ -191,3 +191,15 @@ def test_exchange_with_a_departed_rank_raises_instead_of_hanging():
     assert not alive, "a rank hung in the exchange"
     assert out.get(1) == "left"
     assert str(out.get(0, "")).startswith("raised after"), out.get(0)
+
+
+def test_lpt_cost_model_is_the_step_flop_model():
+    """Policy 1 balances the literal Alg. 1 FLOP count (the bench's model) plus 10 FLOP per
+    weight element for the elementwise work; identity sides cost nothing of their own."""
+    import sys
+    sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+    import bench
+    for shape in [(2048, 2048, 1, 1), (2048, 8192, 1, 1), (8192, 28672, 1, 0), (28672, 8192, 0, 1), (768, 2048, 1, 1)]:
+        _, load = S.layerwise_assign([shape], 1, 1)
+        want = bench.model_flops(*shape) + 10.0 * shape[0] * shape[1]
+        assert abs(load[0] - want) <= 1e-9 * want, (shape, load[0], want)
