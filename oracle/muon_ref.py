@@ -71,6 +71,7 @@ def newton_schulz(M: np.ndarray, coeffs, eps: float, bf16: bool = False) -> np.n
 
 @dataclass
 class MuonState:
+    """Per-matrix state of Alg. Muon: the momentum M (rows x cols, zero at t = 0) and the step count."""
     rows: int
     cols: int
     dtype: type = np.float64
