@@ -39,6 +39,14 @@ Readings of points the paper leaves open:
     column, and columns of N whose Q_R column was, are set to 0. In exact arithmetic
     G' is exactly 0 there, so N = 0 there too; in finite precision G' holds rounding
     noise that Adam's normalisation would blow up to O(1).
+  * ``refresh="eigh"`` (the appendix's alternative to QR, which it finds equivalent at
+    F = 1): Q <- the factor's eigenvectors ordered by decreasing eigenvalue, each column's
+    sign chosen so that q_new . q_old >= 0. That order is the one the QR refresh converges
+    to (subspace iteration orders by decreasing eigenvalue), and that sign rule is the one it
+    follows near its fixed point (R_kk = q_new . L q_old > 0 becomes lambda_k q_new . q_old > 0),
+    so v's coordinates stay aligned from step to step. An eigenvalue at most ``qr_tol * ||F||_F`` counts as a
+    zero direction for the guard, as a zero QR column does (||P||_F = ||F Q||_F = ||F||_F).
+    The CUDA path has no eigh refresh (not built); this reading serves the oracle's pins.
 
 Precision: every array is held in ``dtype`` (float64 by default). ``dtype=np.float32``
 gives the "fp32 twin" used to measure the error any faithful fp32 implementation
@@ -132,6 +140,7 @@ class HParams:
     qr_tol: float = 1e-4
     kl: bool = False              # KL-Shampoo factor form (Alg. 1's "Accumulate Kronecker Factors")
     stale: bool = False           # factors updated after the refresh (the stale variant of section 5)
+    refresh: str = "qr"           # "qr" (Alg. 1) or "eigh" (the appendix's alternative)
 
 
 @dataclass
@@ -176,6 +185,17 @@ class MatrixState:
 
 
 # ---- sub-steps, each a plain transcription of one line group of Alg. 1 ----------
+
+def eigh_basis(F: np.ndarray, Q_old: np.ndarray, tol: float):
+    """The eigh refresh (appendix on eigh vs QR): eigenvectors of the symmetric factor F by
+    decreasing eigenvalue, signs aligned with the previous basis; zero directions flagged as
+    eigenvalues at most tol * ||F||_F. Returns (Q, skipped)."""
+    lam, U = np.linalg.eigh((F + F.T) / 2)
+    order = np.argsort(-lam, kind="stable")
+    lam, U = lam[order], U[:, order]
+    sign = np.where(np.sum(U * Q_old, axis=0) < 0, -1.0, 1.0).astype(F.dtype)
+    return (U * sign).astype(F.dtype), lam <= tol * np.linalg.norm(F)
+
 
 def approx_eigenvalues(F: np.ndarray, Q: np.ndarray) -> np.ndarray:
     """lambda = diag(Q^T F Q): Alg. 1's approximate eigenvalues of a factor in its current basis."""
@@ -305,13 +325,21 @@ def soap_step(st: MatrixState, W: np.ndarray, G: np.ndarray, hp: HParams,
 def _rotate_adam_update(st: MatrixState, W, G, hp: HParams, t: int, d, lr, wd):
     """S2-S8 of one step (the factors as they stand): refresh every F steps, re-projection,
     rotation, Adam in the basis, back-rotation and update. Returns (W_new, dW)."""
+    if hp.refresh not in ("qr", "eigh"):
+        raise ValueError(f"unknown basis refresh {hp.refresh!r}")
     # S2-S4: eigenbasis re-computation every F steps
     if t % hp.eig_every == 0:
         M_hat = rotate_out(st.QL if st.left else None, st.m, st.QR if st.right else None)
-        if st.left:
-            st.QL, st.skipL, _ = householder_q(st.L @ st.QL, hp.qr_tol)
-        if st.right:
-            st.QR, st.skipR, _ = householder_q(st.R @ st.QR, hp.qr_tol)
+        if hp.refresh == "eigh":
+            if st.left:
+                st.QL, st.skipL = eigh_basis(st.L, st.QL, hp.qr_tol)
+            if st.right:
+                st.QR, st.skipR = eigh_basis(st.R, st.QR, hp.qr_tol)
+        else:
+            if st.left:
+                st.QL, st.skipL, _ = householder_q(st.L @ st.QL, hp.qr_tol)
+            if st.right:
+                st.QR, st.skipR, _ = householder_q(st.R @ st.QR, hp.qr_tol)
         st.m = rotate_in(st.QL if st.left else None, M_hat, st.QR if st.right else None)
     # S5: rotate the gradient with the (new) basis
     QL = st.QL if st.left else None

@@ -6,7 +6,7 @@ invariant, a library routine solving the same textbook problem, or brute force.
 import numpy as np
 import pytest
 
-from oracle.soap_ref import (HParams, MatrixState, factor_ema, householder_q, rotate_in,
+from oracle.soap_ref import (HParams, MatrixState, eigh_basis, factor_ema, householder_q, rotate_in,
                              rotate_out, soap_step)
 
 RNG = np.random.default_rng(1234)
@@ -438,3 +438,60 @@ def test_stale_rejects_kl_and_guard():
     for hp in (HParams(stale=True), HParams(stale=True, guard=False, kl=True)):
         with pytest.raises(ValueError):
             soap_step(st, np.zeros((3, 4)), np.ones((3, 4)), hp)
+
+
+# ---- the eigh refresh (appendix on eigh vs QR) ----------------------------------------
+
+def test_eigh_basis_diagonalises_in_decreasing_order_with_aligned_signs():
+    """eigh_basis returns an orthogonal Q with Q^T F Q diagonal and its diagonal decreasing, and
+    every column has a nonnegative overlap with the previous basis's column."""
+    rng = np.random.default_rng(61)
+    n = 9
+    X = rng.standard_normal((n, 4))
+    F = X @ X.T + np.diag(np.linspace(0.1, 0.2, n))
+    Q_old = np.linalg.qr(rng.standard_normal((n, n)))[0]
+    Q, skip = eigh_basis(F, Q_old, 1e-4)
+    assert np.abs(Q.T @ Q - np.eye(n)).max() < 1e-13
+    D = Q.T @ F @ Q
+    assert np.abs(D - np.diag(np.diag(D))).max() < 1e-12 * np.abs(F).max()
+    assert np.all(np.diff(np.diag(D)) <= 1e-14)
+    assert np.all(np.sum(Q * Q_old, axis=0) >= 0)
+    assert not skip.any()
+    # the zero factor: every direction is a zero direction, and the basis stays the old one
+    Q0, skip0 = eigh_basis(np.zeros((n, n)), np.eye(n), 1e-4)
+    assert skip0.all() and np.array_equal(Q0, np.eye(n))
+
+
+def test_eigh_and_qr_refreshes_agree_at_the_fixed_point():
+    """For a constant gradient the QR refresh is subspace iteration and converges to the
+    eigenvectors by decreasing eigenvalue, the basis and order the eigh refresh takes at once
+    (the appendix finds the two refreshes equivalent at F = 1). Column signs may differ (each
+    path keeps the signs its history gave), and the update does not depend on them: once the
+    EMAs have forgotten the steps before convergence, both give the same update. The entries of
+    N off the converged diagonal forget slowest, as (beta1 / sqrt(beta2))^k = 0.974^k, about
+    1e-5 after the 450 steps here."""
+    rng = np.random.default_rng(62)
+    n = 5
+    U = np.linalg.qr(rng.standard_normal((n, n)))[0]
+    V = np.linalg.qr(rng.standard_normal((n, n)))[0]
+    G = U @ np.diag([3.0, 2.0, 1.3, 0.8, 0.5]) @ V.T
+    runs = {}
+    for refresh in ("qr", "eigh"):
+        hp = HParams(refresh=refresh, lr=1e-3)
+        st = MatrixState(n, n, True, True)
+        W = np.zeros((n, n))
+        for _ in range(450):
+            W, dW = soap_step(st, W, G, hp)
+        runs[refresh] = (st, dW)
+    (sq, dq), (se, de) = runs["qr"], runs["eigh"]
+    for A, B in ((sq.QL, se.QL), (sq.QR, se.QR)):
+        s = np.sign(np.sum(A * B, axis=0))
+        np.testing.assert_allclose(A, B * s, atol=1e-9)
+    np.testing.assert_allclose(dq, de, rtol=0, atol=1e-5 * np.abs(de).max())
+    # and the eigenvectors are G's singular vectors, up to sign
+    np.testing.assert_allclose(np.abs(se.QL), np.abs(U), atol=1e-9)
+
+
+def test_unknown_refresh_is_rejected():
+    with pytest.raises(ValueError):
+        soap_step(MatrixState(2, 2, True, True), np.zeros((2, 2)), np.ones((2, 2)), HParams(refresh="svd"))
