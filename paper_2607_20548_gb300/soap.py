@@ -186,6 +186,8 @@ class SoapOptimizer:
         for i, (p, g, s) in enumerate(zip(params, grads, self.shapes)):
             if p.dtype != torch.float32 or g.dtype != torch.float32 or not p.is_cuda or not g.is_cuda:
                 raise TypeError(f"matrix {i}: params/grads must be fp32 CUDA tensors")
+            if p.device.index != self.device or g.device.index != self.device:
+                raise ValueError(f"matrix {i}: tensors must be on cuda:{self.device}, the handle's device")
             if tuple(p.shape) != (s.rows, s.cols) or tuple(g.shape) != (s.rows, s.cols):
                 raise ValueError(f"matrix {i}: expected {(s.rows, s.cols)}")
             if not p.is_contiguous() or not g.is_contiguous():
@@ -448,6 +450,8 @@ class MuonOptimizer:
         for i, (p, g, s) in enumerate(zip(params, grads, self.shapes)):
             if p.dtype != torch.float32 or g.dtype != torch.float32 or not p.is_cuda or not g.is_cuda:
                 raise TypeError(f"matrix {i}: params/grads must be fp32 CUDA tensors")
+            if p.device.index != self.device or g.device.index != self.device:
+                raise ValueError(f"matrix {i}: tensors must be on cuda:{self.device}, the handle's device")
             if tuple(p.shape) != s or tuple(g.shape) != s or not p.is_contiguous() or not g.is_contiguous():
                 raise ValueError(f"matrix {i}: expected a contiguous {s} tensor")
             self._pp[i] = p.data_ptr()

@@ -114,3 +114,37 @@ def test_product_code_shares_nothing_with_the_oracle():
         if f.endswith((".py", ".c", ".h")):
             text = open(os.path.join(ROOT, "oracle", f)).read()
             assert "paper_2607_20548_gb300" not in text and "csrc" not in text, f
+
+
+class _FakeCudaTensor:
+    """Just enough of a CUDA tensor for the binding's argument checks (never reaches the library)."""
+
+    def __init__(self, shape, index):
+        import torch
+        self.shape, self.dtype, self.is_cuda = shape, torch.float32, True
+        self.device = torch.device("cuda", index)
+
+    def is_contiguous(self):
+        return True
+
+    def data_ptr(self):
+        return 1 << 20
+
+
+def test_binding_rejects_tensors_on_another_device():
+    """A handle steps tensors on its own device only; the check happens before any library call."""
+    import ctypes as ct
+
+    import pytest
+    for cls in (S.SoapOptimizer, S.MuonOptimizer):
+        opt = cls.__new__(cls)
+        opt.shapes = [S.Shape(4, 8)] if cls is S.SoapOptimizer else [(4, 8)]
+        opt.device, opt._h = 0, None
+        opt._pp, opt._gp = (ct.c_void_p * 1)(), (ct.c_void_p * 1)()
+        with pytest.raises(ValueError, match="cuda:0"):
+            opt.step([_FakeCudaTensor((4, 8), 1)], [_FakeCudaTensor((4, 8), 1)])
+        with pytest.raises(ValueError, match="cuda:0"):
+            opt.step([_FakeCudaTensor((4, 8), 0)], [_FakeCudaTensor((4, 8), 1)])
+        # tensors on the handle's device pass the checks (and reach the handle, destroyed here)
+        with pytest.raises(S.SoapError, match="handle destroyed"):
+            opt.step([_FakeCudaTensor((4, 8), 0)], [_FakeCudaTensor((4, 8), 0)])
