@@ -134,6 +134,22 @@ def _stream(stream=None):
     return ctypes.c_void_p(stream.cuda_stream)
 
 
+def _one_device(name, *tensors, dtype=torch.float32):
+    """The device the given tensors share; raises unless each is a ``dtype`` CUDA tensor on it
+    (a host or a foreign-device pointer must never reach a kernel)."""
+    dev = None
+    for t in tensors:
+        if t is None:
+            continue
+        if not isinstance(t, torch.Tensor) or not t.is_cuda or t.dtype != dtype:
+            raise TypeError(f"{name}: expected {dtype} CUDA tensors")
+        if dev is None:
+            dev = t.device
+        elif t.device != dev:
+            raise ValueError(f"{name}: tensors on {dev} and {t.device}")
+    return dev
+
+
 def _check(code, h=None):
     if code != SOAP_OK:
         msg = load_library().soap_last_error(h).decode() if h else ""
@@ -306,9 +322,10 @@ def soap_qr(P: torch.Tensor, tol: float = 0.0, stream=None):
     skip = torch.empty(batch, n, dtype=torch.uint8, device=P.device)
     ws_bytes = lib.soap_qr_workspace_bytes(n, batch)
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device=P.device)
-    _check(lib.soap_qr(n, batch, ctypes.c_void_p(P.data_ptr()), ctypes.c_void_p(Q.data_ptr()),
-                       ctypes.c_void_p(skip.data_ptr()), float(tol), ctypes.c_void_p(ws.data_ptr()), ws_bytes,
-                       _stream(stream)))
+    with torch.cuda.device(P.device):
+        _check(lib.soap_qr(n, batch, ctypes.c_void_p(P.data_ptr()), ctypes.c_void_p(Q.data_ptr()),
+                           ctypes.c_void_p(skip.data_ptr()), float(tol), ctypes.c_void_p(ws.data_ptr()), ws_bytes,
+                           _stream(stream)))
     return Q, skip
 
 
@@ -327,8 +344,9 @@ def soap_qr_static(P: torch.Tensor, tol: float = 0.0, stream=None):
     batch, n = P.shape[0], P.shape[1]
     Q = torch.empty_like(P)
     skip = torch.empty(batch, n, dtype=torch.uint8, device=P.device)
-    code = lib.soap_qr_static(n, batch, ctypes.c_void_p(P.data_ptr()), ctypes.c_void_p(Q.data_ptr()),
-                              ctypes.c_void_p(skip.data_ptr()), float(tol), _stream(stream))
+    with torch.cuda.device(P.device):
+        code = lib.soap_qr_static(n, batch, ctypes.c_void_p(P.data_ptr()), ctypes.c_void_p(Q.data_ptr()),
+                                  ctypes.c_void_p(skip.data_ptr()), float(tol), _stream(stream))
     if code != SOAP_OK:
         raise SoapError(code, f"soap_qr_static(n={n}, batch={batch}): needs "
                               f"{lib.soap_qr_workspace_bytes(n, batch)} bytes of workspace; the fixed array "
@@ -347,25 +365,29 @@ def soap_gemm(A: torch.Tensor, B: torch.Tensor, trans_a=False, trans_b=False, al
     M = A3.shape[2] if trans_a else A3.shape[1]
     K = A3.shape[1] if trans_a else A3.shape[2]
     N = B3.shape[1] if trans_b else B3.shape[2]
+    dev = _one_device("soap_gemm", A3, B3, C)
     if C is None:
-        C3 = torch.zeros(batch, M, N, dtype=torch.float32, device=A.device)
+        C3 = torch.zeros(batch, M, N, dtype=torch.float32, device=dev)
     else:
         C3 = C.unsqueeze(0) if C.dim() == 2 else C
         if not C3.is_contiguous():
             raise ValueError("C must be contiguous")
-    _check(lib.soap_gemm(int(trans_a), int(trans_b), M, N, K, float(alpha),
-                         ctypes.c_void_p(A3.data_ptr()), A3.shape[2], A3.shape[1] * A3.shape[2],
-                         ctypes.c_void_p(B3.data_ptr()), B3.shape[2], B3.shape[1] * B3.shape[2], float(beta),
-                         ctypes.c_void_p(C3.data_ptr()), N, M * N, batch, _stream(stream)))
+    with torch.cuda.device(dev):
+        _check(lib.soap_gemm(int(trans_a), int(trans_b), M, N, K, float(alpha),
+                             ctypes.c_void_p(A3.data_ptr()), A3.shape[2], A3.shape[1] * A3.shape[2],
+                             ctypes.c_void_p(B3.data_ptr()), B3.shape[2], B3.shape[1] * B3.shape[2], float(beta),
+                             ctypes.c_void_p(C3.data_ptr()), N, M * N, batch, _stream(stream)))
     return C3[0] if squeeze else C3
 
 
 def soap_split_tf32(x: torch.Tensor, stream=None):
     """(hi, lo) with hi = x truncated to tf32 and lo = x - hi, computed on the device."""
+    dev = _one_device("soap_split_tf32", x)
     x = x.contiguous()
     hi, lo = torch.empty_like(x), torch.empty_like(x)
-    _check(load_library().soap_split_tf32(ctypes.c_void_p(x.data_ptr()), ctypes.c_void_p(hi.data_ptr()),
-                                          ctypes.c_void_p(lo.data_ptr()), x.numel(), _stream(stream)))
+    with torch.cuda.device(dev):
+        _check(load_library().soap_split_tf32(ctypes.c_void_p(x.data_ptr()), ctypes.c_void_p(hi.data_ptr()),
+                                              ctypes.c_void_p(lo.data_ptr()), x.numel(), _stream(stream)))
     return hi, lo
 
 
@@ -380,21 +402,30 @@ def soap_gemm_tf32x4(A, B, alpha=1.0, beta=0.0, C=None, transpose_c=False, A_spl
     B3 = (B.unsqueeze(0) if B.dim() == 2 else B).contiguous()
     batch, M, K = A3.shape
     bb, N, K2 = B3.shape
-    assert K == K2
+    if K != K2:
+        raise ValueError("soap_gemm_tf32x4: A and B need the same K")
+    dev = _one_device("soap_gemm_tf32x4", A3, B3, C)
+    if status is not None:
+        _one_device("soap_gemm_tf32x4 status", status, dtype=torch.int32)
+        if status.device != dev:
+            raise ValueError("soap_gemm_tf32x4: status on another device")
     ahi, alo = A_split if A_split is not None else soap_split_tf32(A3, stream)
     bhi, blo = B_split if B_split is not None else soap_split_tf32(B3, stream)
+    if _one_device("soap_gemm_tf32x4 splits", ahi, alo, bhi, blo) != dev:
+        raise ValueError("soap_gemm_tf32x4: split operands on another device")
     shape = (batch, N, M) if transpose_c else (batch, M, N)
     C3 = torch.zeros(shape, dtype=torch.float32, device=A3.device) if C is None else \
         (C.unsqueeze(0) if C.dim() == 2 else C)
     lo = torch.zeros_like(C3) if with_lo else None
     ldc = shape[2]
-    _check(lib.soap_gemm_tf32x4(M, N, K, batch, ctypes.c_void_p(ahi.data_ptr()), ctypes.c_void_p(alo.data_ptr()),
-                                K, M * K, ctypes.c_void_p(bhi.data_ptr()), ctypes.c_void_p(blo.data_ptr()), K,
-                                N * K, bb, float(alpha), float(beta), ctypes.c_void_p(C3.data_ptr()), ldc,
-                                shape[1] * shape[2], int(transpose_c),
-                                ctypes.c_void_p(lo.data_ptr()) if with_lo else None,
-                                ctypes.c_void_p(status.data_ptr()) if status is not None else None,
-                                _stream(stream)))
+    with torch.cuda.device(dev):
+        _check(lib.soap_gemm_tf32x4(M, N, K, batch, ctypes.c_void_p(ahi.data_ptr()), ctypes.c_void_p(alo.data_ptr()),
+                                    K, M * K, ctypes.c_void_p(bhi.data_ptr()), ctypes.c_void_p(blo.data_ptr()), K,
+                                    N * K, bb, float(alpha), float(beta), ctypes.c_void_p(C3.data_ptr()), ldc,
+                                    shape[1] * shape[2], int(transpose_c),
+                                    ctypes.c_void_p(lo.data_ptr()) if with_lo else None,
+                                    ctypes.c_void_p(status.data_ptr()) if status is not None else None,
+                                    _stream(stream)))
     out = C3[0] if A.dim() == 2 and (C is None or C.dim() == 2) else C3
     if with_lo:
         return out, (lo[0] if out.dim() == 2 else lo)

@@ -148,3 +148,15 @@ def test_binding_rejects_tensors_on_another_device():
         # tensors on the handle's device pass the checks (and reach the handle, destroyed here)
         with pytest.raises(S.SoapError, match="handle destroyed"):
             opt.step([_FakeCudaTensor((4, 8), 0)], [_FakeCudaTensor((4, 8), 0)])
+
+
+def test_standalone_entry_points_reject_host_tensors():
+    """The stand-alone sub-steps hand only CUDA tensors of the right type to the kernels: host
+    tensors are refused on the host, before any launch."""
+    import pytest
+    import torch
+    x = torch.zeros(4, 4)
+    for call in (lambda: S.soap_gemm(x, x), lambda: S.soap_split_tf32(x), lambda: S.soap_gemm_tf32x4(x, x),
+                 lambda: S.soap_qr(x), lambda: S.soap_qr_static(x)):
+        with pytest.raises(TypeError):
+            call()
