@@ -95,9 +95,9 @@ void soap_default_hparams(soap_hparams* hp);
  * m = v = 0, t = 0. shapes[] is copied. Returns SOAP_ERR_OOM if the state does
  * not fit; *out is then NULL; SOAP_ERR_INVALID_ARG for kl = 1 with eps <= 0 (the first
  * KL step weighs by 1/eps) and for stale = 1 with kl or guard set. The device becomes
- * current for the calling thread. All handles of one process must use the same device (one
- * process per GPU): the kernels' launch attributes are set once per process, so steps of a
- * handle on a second device fail with SOAP_ERR_CUDA. */
+ * current for the calling thread. Handles on different devices may coexist in one process
+ * (each kernel's launch attributes are set once per device); the usual layout is one process
+ * per GPU. */
 soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparams* hp,
                           int32_t device, soap_handle* out);
 

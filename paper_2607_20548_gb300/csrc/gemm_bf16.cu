@@ -19,6 +19,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 
 #include "profile.h"
@@ -397,14 +398,17 @@ cudaError_t gemm_bf16_nt(int M, int N, int K, int batch, const __nv_bfloat16* A,
   CUtensorMap ta, tb;
   if (!make_map(&ta, A, M, K, lda, a_stride, batch, BM) || !make_map(&tb, B, N, K, ldb, b_stride, batch, BN))
     return cudaErrorInvalidValue;
-  static bool attr_set = false;
-  if (!attr_set) {
+  // the shared-memory attribute belongs to each device's context: one bit per device that has it
+  static std::atomic<uint64_t> attr_set{0};
+  int dev = 0, sms = 152;
+  if (cudaGetDevice(&dev) != cudaSuccess) dev = 0;
+  const uint64_t bit = (dev >= 0 && dev < 64) ? uint64_t(1) << dev : 0;
+  if (bit == 0 || !(attr_set.load(std::memory_order_relaxed) & bit)) {
     cudaError_t e = cudaFuncSetAttribute(gemm_bf16_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    attr_set.fetch_or(bit, std::memory_order_relaxed);
   }
-  int dev = 0, sms = 152;
-  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int64_t ntiles = (int64_t)((N + BN - 1) / BN) * ((M + BM - 1) / BM) * batch;
   if (ntiles > (int64_t)1 << 30) return cudaErrorInvalidValue;
   const int grid = (int)std::min<int64_t>(ntiles, sms);

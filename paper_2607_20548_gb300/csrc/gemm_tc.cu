@@ -36,6 +36,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 
 #include "profile.h"
@@ -594,13 +595,17 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
       !make_map(&m[1], CVTA ? A.hi : A.lo, M, K, A.ld, A.stride, amod, BM) ||
       !make_map(&m[2], B.hi, N, K, B.ld, B.stride, bmod, BN) || !make_map(&m[3], B.lo, N, K, B.ld, B.stride, bmod, BN))
     return cudaErrorInvalidValue;
-  static bool attr_set = false;
-  if (!attr_set) {
+  // the shared-memory attribute belongs to each device's context: one bit per device that has it
+  static std::atomic<uint64_t> attr_set{0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) dev = 0;
+  const uint64_t bit = (dev >= 0 && dev < 64) ? uint64_t(1) << dev : 0;
+  if (bit == 0 || !(attr_set.load(std::memory_order_relaxed) & bit)) {
     cudaError_t e =
         cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              C::SMEM);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    attr_set.fetch_or(bit, std::memory_order_relaxed);
   }
   const int64_t ntiles = (int64_t)((N + BN - 1) / BN) * ((M + BM - 1) / BM) * batch * ksplit;
   if (ntiles > (int64_t)1 << 30) return cudaErrorInvalidValue;
