@@ -160,3 +160,24 @@ def test_standalone_entry_points_reject_host_tensors():
                  lambda: S.soap_qr(x), lambda: S.soap_qr_static(x)):
         with pytest.raises(TypeError):
             call()
+
+
+def test_plain_c_consumer_builds_and_runs():
+    """include/*.h are plain C: a C99 program compiles against them with gcc alone, links
+    libsoap.so and runs its host-side entry points."""
+    import shutil
+    import subprocess
+    import tempfile
+
+    import pytest
+    if shutil.which("gcc") is None:
+        pytest.skip("no gcc")
+    lib = build.build()
+    with tempfile.TemporaryDirectory() as d:
+        exe = os.path.join(d, "c_abi_host")
+        r = subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", "-I", os.path.join(ROOT, "include"),
+                            os.path.join(ROOT, "tests", "c_abi_host.c"), lib, "-Wl,-rpath," + os.path.dirname(lib),
+                            "-o", exe], capture_output=True, text=True)
+        assert r.returncode == 0, r.stderr
+        r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
+        assert r.returncode == 0 and "c abi ok" in r.stdout, (r.returncode, r.stdout, r.stderr)
