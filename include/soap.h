@@ -101,14 +101,34 @@ void soap_default_hparams(soap_hparams* hp);
 soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparams* hp,
                           int32_t device, soap_handle* out);
 
+/* soap_create with a bound on the workspace. Besides the optimizer state proper (per matrix
+ * M_hat and v, the factors L and R stored as their lower-triangular 32 x 32 tiles, the bases
+ * Q_L and Q_R), a step needs a workspace for the operands it forms (the gradient copy and its
+ * transpose, tf32 lo parts, Q^T, the unpacked factors, the QR's buffers, the rotation
+ * intermediates). Matrices are stepped in waves: runs of matrices whose workspace fits side by
+ * side, the next wave reusing it. workspace_limit = 0 (what soap_create does) takes one wave
+ * holding every matrix if that leaves 1 GiB + 1% of the device's memory free, else waves cut
+ * to the memory free at that moment less that reserve; workspace_limit > 0 caps the workspace
+ * at that many bytes (and at the free memory less the reserve). Returns SOAP_ERR_OOM if the
+ * state does not fit, or if one matrix of some shape needs more workspace than allowed. */
+soap_status_t soap_create_ex(const soap_shape* shapes, int32_t n, const soap_hparams* hp, int32_t device,
+                             size_t workspace_limit, soap_handle* out);
+
+/* The plan soap_create chose: number of waves per step, workspace bytes and state bytes
+ * (device memory held by the handle is their sum). Any pointer may be NULL. */
+soap_status_t soap_plan_info(soap_handle h, int32_t* waves, size_t* workspace_bytes, size_t* state_bytes);
+
 /* One SOAP step (Alg. 1) over all n matrices, enqueued on `stream`:
  * factor EMAs with the current gradient, power step P = L Q and QR refresh with
  * diag(R) >= 0, first-moment re-projection, rotation G' = Q_L^T G Q_R, Adam in the
  * rotated basis, back-rotation dW = Q_L N Q_R^T and W <- (1 - eta lambda) W - eta dW.
  * params[i] / grads[i]: device pointers to matrix i (rows_i x cols_i, fp32); params
  * are updated in place, grads are only read. Both pointer arrays are host arrays
- * and are copied before the call returns. Returns a pending sticky device status
- * from an earlier step, if any, before enqueuing anything. */
+ * and are copied before the call returns (a changed table is written to the device by the
+ * launches themselves; nothing on the host waits for the GPU). Steps, and state reads and
+ * writes, share the handle's workspace: each is ordered after the one enqueued before it,
+ * whatever stream either came on. Returns a pending sticky device status from an earlier
+ * step, if any, before enqueuing anything. */
 soap_status_t soap_step(soap_handle h, float* const* params, const float* const* grads,
                         soap_stream_t stream);
 
@@ -214,14 +234,23 @@ soap_status_t soap_profile_records(soap_handle h, soap_launch_record* out, int64
 
 /* ---- stand-alone sub-steps (the same kernels soap_step runs) ------------------- */
 
+/* Device status bits of the stand-alone sub-steps (the int32 words they take as `status`):
+ * set by the kernels with an atomic OR, never cleared by them. */
+#define SOAP_STATUS_NONFINITE 1     /* a non-finite value in the input */
+#define SOAP_STATUS_QR_BREAKDOWN 2  /* a QR pivot norm was not finite */
+#define SOAP_STATUS_TIMEOUT 4       /* a bounded device-side wait gave up (results invalid) */
+
 /* S3, Alg. 1 "QR(L_t Q_L).Q": for `batch` square n x n matrices P (device,
  * contiguous, batch stride n*n), writes Q with P = Q R and diag(R) >= 0 (blocked
  * Householder QR, explicit Q) and skip[b*n + k] = 1 where column k was treated as
  * exactly zero (remaining norm <= tol * ||P_b||_F). P is read only. `workspace`
- * must hold soap_qr_workspace_bytes(n, batch) bytes of device memory. */
+ * must hold soap_qr_workspace_bytes(n, batch) bytes of device memory (256-byte aligned).
+ * status: NULL, or a device int32 (4-byte aligned) that the call sets to 0 on the stream and
+ * into which its kernels OR SOAP_STATUS_QR_BREAKDOWN / SOAP_STATUS_TIMEOUT; read it once the
+ * stream has passed the call (0 = Q is valid). */
 size_t soap_qr_workspace_bytes(int32_t n, int32_t batch);
 soap_status_t soap_qr(int32_t n, int32_t batch, const float* P, float* Q, uint8_t* skip,
-                      float tol, void* workspace, size_t workspace_bytes,
+                      float tol, void* workspace, size_t workspace_bytes, int32_t* status,
                       soap_stream_t stream);
 
 /* soap_qr for callers that cannot give this library device memory. The paper has no
@@ -234,13 +263,14 @@ soap_status_t soap_qr(int32_t n, int32_t batch, const float* P, float* Q, uint8_
  * matrix or, e.g., three of 512 x 512; a (n, batch) whose soap_qr_workspace_bytes()
  * exceeds 32 MiB - 256 B is refused with SOAP_ERR_INVALID_ARG before anything is
  * enqueued. It never calls cudaMalloc, cudaFree or any allocating routine.
+ * status: as for soap_qr (NULL: the word is kept inside the array, where no one reads it).
  * The first call on each device looks up the array's device address with that device
  * current (cudaGetSymbolAddress); make that first call before any stream capture. All
  * calls in the process share the one array per device and it keeps the last call's
  * contents, so two calls that can overlap on the GPU (different streams without
  * ordering between them) race: order them, e.g. on one stream. */
 soap_status_t soap_qr_static(int32_t n, int32_t batch, const float* P, float* Q, uint8_t* skip,
-                             float tol, soap_stream_t stream);
+                             float tol, int32_t* status, soap_stream_t stream);
 
 /* The fp32-accurate batched product used by every contraction of the step (S1, S2,
  * S4, S5, S7 and the QR updates): for b < batch,
@@ -262,8 +292,8 @@ soap_status_t soap_gemm(int32_t trans_a, int32_t trans_b, int32_t M, int32_t N, 
  * K block summed afresh and added in fp32 registers (fp32-level accuracy at any K).
  * lda, ldb, ldc and every batch stride must be multiples of 4 elements and every
  * pointer 16-byte aligned. C_lo, if non-NULL, receives out - tf32(out) in C's layout
- * (leading dimension ldc). status, if non-NULL, is a device int that gets bit 4 set if
- * a bounded internal wait gave up. */
+ * (leading dimension ldc). status, if non-NULL, is a device int32 into which the kernel ORs
+ * SOAP_STATUS_TIMEOUT if a bounded internal wait gave up (it is not cleared). */
 soap_status_t soap_gemm_tf32x4(int32_t M, int32_t N, int32_t K, int32_t batch, const float* A_hi,
                                const float* A_lo, int64_t lda, int64_t stride_a, const float* B_hi,
                                const float* B_lo, int64_t ldb, int64_t stride_b, int32_t b_batch,

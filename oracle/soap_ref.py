@@ -28,8 +28,8 @@ Readings of points the paper leaves open:
   * Initial state: L = R = 0, Q = I, m = v = 0, t = 1 on the first call, and the
     first call applies an update (Alg. 1 has no warm-up branch).
   * Only m is re-projected when the basis changes; v is not (Alg. 1).
-  * No bias correction unless ``bias_correction`` is set (primer: "ignoring ...
-    bias corrections"; Alg. 1 has none).
+  * No bias correction unless ``bias_correction`` is set (section 2's AdamW primer leaves
+    it out; Alg. 1 has none).
   * eps is added outside the square root (Alg. 1).
   * A side whose dimension is not preconditioned keeps Q = I and stores no factor.
   * QR of a rank-deficient P: a Householder column whose remaining norm is at most

@@ -167,13 +167,14 @@ __global__ void identity_kernel(float* Q, int n) {
 
 
 // One 32 x 32 tile of one matrix per block (32 x 8 threads). Reads G and writes the
-// tensor-core operands: G and its lo part, G^T and its lo part, and the momentum EMA
-// M_hat <- b1 M_hat + (1-b1) G with its lo part. M_hat is kept in G's orientation or, with
-// mh_transposed, as M_hat^T (the working orientation of a matrix preconditioned on its
-// left side only).
+// tensor-core operands into the step's workspace: G and its lo part, G^T and its lo part, and
+// the momentum EMA M_hat <- b1 M_hat + (1-b1) G, stored back into the optimizer state (Mh) and
+// copied with its lo part beside G (Mc, Mc_lo), so that one batched product rotates both.
+// M_hat is kept in G's orientation or, with mh_transposed, as M_hat^T (the working orientation
+// of a matrix preconditioned on its left side only).
 __global__ void momentum_split_kernel(const float* const* grads, float* Gn, float* Gn_lo, float* Gt, float* Gt_lo,
-                                      float* Mh, float* Mh_lo, int rows, int cols, float beta1, int mh_transposed,
-                                      int* status) {
+                                      float* Mh, float* Mc, float* Mc_lo, int rows, int cols, float beta1,
+                                      int mh_transposed, int* status) {
   __shared__ float tile[32][33];
   const int b = blockIdx.z;
   const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
@@ -193,7 +194,8 @@ __global__ void momentum_split_kernel(const float* const* grads, float* Gn, floa
       if (!mh_transposed) {
         const float m = fmaf(beta1, Mh[o], c1 * x);
         Mh[o] = m;
-        Mh_lo[o] = lo_part(m);
+        Mc[o] = m;
+        Mc_lo[o] = lo_part(m);
       }
     }
     tile[i][threadIdx.x] = x;
@@ -209,11 +211,82 @@ __global__ void momentum_split_kernel(const float* const* grads, float* Gn, floa
       if (mh_transposed) {
         const float m = fmaf(beta1, Mh[o], c1 * x);
         Mh[o] = m;
-        Mh_lo[o] = lo_part(m);
+        Mc[o] = m;
+        Mc_lo[o] = lo_part(m);
       }
     }
   }
   if (__syncthreads_or(bad) && threadIdx.x == 0 && threadIdx.y == 0) atomicOr(status, kStatusNonFinite);
+}
+
+// Packed symmetric storage of an n x n factor: only its lower-triangular 32 x 32 tiles, tile
+// (I, J) with I >= J at tile index I (I + 1) / 2 + J, each tile row-major; entries beyond n
+// are zero. A diagonal tile is stored whole (its upper half mirrors its lower half).
+__device__ __forceinline__ void tri_tile(int t, int& I, int& J) {
+  int i = (int)((sqrtf(8.f * (float)t + 1.f) - 1.f) * 0.5f);
+  while ((i + 1) * (i + 2) / 2 <= t) ++i;
+  while (i * (i + 1) / 2 > t) --i;
+  I = i;
+  J = t - i * (i + 1) / 2;
+}
+
+// Full matrix (and, if F_lo is given, its lo part) from packed tiles: one lower tile per
+// block (32 x 8 threads), written in place and, off the diagonal, mirrored through shared
+// memory.
+__global__ void unpack_sym_kernel(const float* P, float* F, float* F_lo, int n, int64_t packed) {
+  __shared__ float tile[32][33];
+  const int b = blockIdx.y;
+  int I, J;
+  tri_tile(blockIdx.x, I, J);
+  const float* p = P + (int64_t)b * packed + (int64_t)blockIdx.x * 1024;
+  float* f = F + (int64_t)b * n * n;
+  float* fl = F_lo ? F_lo + (int64_t)b * n * n : nullptr;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const float x = p[i * 32 + threadIdx.x];
+    tile[i][threadIdx.x] = x;
+    const int r = I * 32 + i, c = J * 32 + threadIdx.x;
+    if (r < n && c < n) {
+      f[(int64_t)r * n + c] = x;
+      if (fl) fl[(int64_t)r * n + c] = lo_part(x);
+    }
+  }
+  if (I == J) return;  // uniform over the block
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = J * 32 + i, c = I * 32 + threadIdx.x;
+    if (r < n && c < n) {
+      const float x = tile[threadIdx.x][i];
+      f[(int64_t)r * n + c] = x;
+      if (fl) fl[(int64_t)r * n + c] = lo_part(x);
+    }
+  }
+}
+
+// Packed tiles from the lower triangle of a full matrix (the upper triangle is not read
+// except inside diagonal tiles, where the lower half is mirrored over it).
+__global__ void pack_sym_kernel(const float* F, float* P, int n, int64_t packed) {
+  __shared__ float tile[32][33];
+  const int b = blockIdx.y;
+  int I, J;
+  tri_tile(blockIdx.x, I, J);
+  const float* f = F + (int64_t)b * n * n;
+  float* p = P + (int64_t)b * packed + (int64_t)blockIdx.x * 1024;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = I * 32 + i, c = J * 32 + threadIdx.x;
+    tile[i][threadIdx.x] = (r < n && c < n) ? f[(int64_t)r * n + c] : 0.f;
+  }
+  if (I == J) __syncthreads();  // uniform over the block
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int j = threadIdx.x;
+    p[i * 32 + j] = (I != J || i >= j) ? tile[i][j] : tile[j][i];
+  }
+}
+
+// Writes n (<= kPtrChunk) device pointers handed over as a kernel parameter (the launch copies
+// them, so the host array may be reused as soon as the launch call returns).
+__global__ void put_ptrs_kernel(void** dst, PtrChunk c, int n) {
+  const int i = threadIdx.x;
+  if (i < n) dst[i] = c.p[i];
 }
 
 // dst_b = src_b^T for `batch` contiguous rows x cols matrices (32 x 32 tiles, 32 x 8 threads).
@@ -348,15 +421,54 @@ __global__ void split_kernel(const float* x, float* hi, float* lo, int64_t n) {
 }  // namespace
 
 cudaError_t momentum_split(const float* const* grads, float* Gn, float* Gn_lo, float* Gt, float* Gt_lo, float* Mhat,
-                           float* Mhat_lo, int rows, int cols, int batch, float beta1, bool mhat_transposed, int* status,
-                           cudaStream_t s) {
+                           float* Mcopy, float* Mcopy_lo, int rows, int cols, int batch, float beta1,
+                           bool mhat_transposed, int* status, cudaStream_t s) {
   if (rows <= 0 || cols <= 0 || batch <= 0) return cudaSuccess;
+  if (batch > 65535 || (rows + 31) / 32 > 65535) return cudaErrorInvalidValue;
   const double e = (double)rows * cols * batch;
-  ProfScope prof(kFamElementwise, 3.0 * e, 32.0 * e, s);
+  ProfScope prof(kFamElementwise, 3.0 * e, 36.0 * e, s);
   dim3 grid((cols + 31) / 32, (rows + 31) / 32, batch);
-  momentum_split_kernel<<<grid, dim3(32, 8), 0, s>>>(grads, Gn, Gn_lo, Gt, Gt_lo, Mhat, Mhat_lo, rows, cols, beta1,
-                                                     mhat_transposed ? 1 : 0, status);
+  momentum_split_kernel<<<grid, dim3(32, 8), 0, s>>>(grads, Gn, Gn_lo, Gt, Gt_lo, Mhat, Mcopy, Mcopy_lo, rows, cols,
+                                                     beta1, mhat_transposed ? 1 : 0, status);
   return cudaGetLastError();
+}
+
+int64_t packed_floats(int n) {
+  const int64_t t = (n + 31) / 32;
+  return t * (t + 1) / 2 * 1024;
+}
+
+cudaError_t unpack_sym(const float* P, float* F, float* F_lo, int n, int batch, cudaStream_t s) {
+  if (n <= 0 || batch <= 0) return cudaSuccess;
+  if (batch > 65535) return cudaErrorInvalidValue;
+  const int64_t tiles = packed_floats(n) / 1024;
+  const double e = (double)n * n * batch;
+  ProfScope prof(kFamElementwise, 0.0, (2.0 + (F_lo ? 8.0 : 4.0)) * e, s);
+  unpack_sym_kernel<<<dim3((unsigned)tiles, batch), dim3(32, 8), 0, s>>>(P, F, F_lo, n, packed_floats(n));
+  return cudaGetLastError();
+}
+
+cudaError_t pack_sym(const float* F, float* P, int n, int batch, cudaStream_t s) {
+  if (n <= 0 || batch <= 0) return cudaSuccess;
+  if (batch > 65535) return cudaErrorInvalidValue;
+  const int64_t tiles = packed_floats(n) / 1024;
+  const double e = (double)n * n * batch;
+  ProfScope prof(kFamElementwise, 0.0, 4.0 * e, s);
+  pack_sym_kernel<<<dim3((unsigned)tiles, batch), dim3(32, 8), 0, s>>>(F, P, n, packed_floats(n));
+  return cudaGetLastError();
+}
+
+cudaError_t put_ptrs(void** dst, void* const* src, int64_t n, cudaStream_t s) {
+  for (int64_t i = 0; i < n; i += kPtrChunk) {
+    PtrChunk c;
+    const int k = (int)std::min<int64_t>(kPtrChunk, n - i);
+    for (int j = 0; j < k; ++j) c.p[j] = src[i + j];
+    ProfScope prof(kFamOther, 0.0, 8.0 * k, s);
+    put_ptrs_kernel<<<1, 512, 0, s>>>(dst + i, c, k);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t transpose(const float* src, float* dst, int rows, int cols, int batch, cudaStream_t s) {

@@ -46,6 +46,7 @@
 #include <cooperative_groups.h>
 
 #include <algorithm>
+#include <atomic>
 
 #include "profile.h"
 #include "soap_internal.h"
@@ -770,8 +771,15 @@ cudaError_t prepare_panel(PanelKernel* pk, bool wide) {
   return e;
 }
 
+// The cluster shape is chosen once per device (with that device current): 1 = clusters of
+// 16 x 512 positions where the device can place them, 2 = clusters of 8 x 1024.
+std::atomic<int> g_panel_choice[64];
+
 cudaError_t panel_kernel(PanelKernel* pk) {
-  static int choice = 0;  // 0 unknown, 1 clusters of 16 x 512 positions, 2 clusters of 8 x 1024
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) dev = 0;
+  std::atomic<int>* slot = dev < 64 ? &g_panel_choice[dev] : nullptr;
+  int choice = slot ? slot->load(std::memory_order_relaxed) : 0;
   if (choice == 0) {
     int ok = 0;
     if (prepare_panel<512>(pk, true) == cudaSuccess) {
@@ -791,6 +799,7 @@ cudaError_t panel_kernel(PanelKernel* pk) {
     }
     cudaGetLastError();
     choice = ok ? 1 : 2;
+    if (slot) slot->store(choice, std::memory_order_relaxed);
   }
   return choice == 1 ? prepare_panel<512>(pk, true) : prepare_panel<1024>(pk, false);
 }

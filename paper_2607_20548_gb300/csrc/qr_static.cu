@@ -28,10 +28,11 @@ void* g_scratch_addr[kMaxDevices] = {};
 }  // namespace
 
 extern "C" soap_status_t soap_qr_static(int32_t n, int32_t batch, const float* P, float* Q, uint8_t* skip,
-                                        float tol, soap_stream_t stream) {
+                                        float tol, int32_t* status, soap_stream_t stream) {
   if (n <= 0 || n > 8192 || (n & 3) || batch <= 0 || batch > 65535 || !P || !Q || !skip || !(tol >= 0.f))
     return SOAP_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(P) | reinterpret_cast<uintptr_t>(Q)) & 15) return SOAP_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(status) & 3) return SOAP_ERR_INVALID_ARG;
   const size_t qb = soap::qr_workspace_bytes(n, batch);
   if (qb + 256 > kScratchBytes) return SOAP_ERR_INVALID_ARG;  // more than the fixed array holds
   int dev = -1;
@@ -49,8 +50,9 @@ extern "C" soap_status_t soap_qr_static(int32_t n, int32_t batch, const float* P
   }
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   // the array keeps the previous call's contents; only the status word must start at zero
-  // (every other region is written before it is read)
-  int* status = reinterpret_cast<int*>(static_cast<char*>(base) + qb);
-  if (cudaMemsetAsync(status, 0, sizeof(int), s) != cudaSuccess) return SOAP_ERR_CUDA;
-  return soap::qr_q(n, batch, P, Q, skip, tol, base, qb, status, s) == cudaSuccess ? SOAP_OK : SOAP_ERR_CUDA;
+  // (every other region is written before it is read). The word is the caller's if given, so
+  // that a breakdown or a wait that gave up can be read back; else it sits in the array.
+  int* word = status ? reinterpret_cast<int*>(status) : reinterpret_cast<int*>(static_cast<char*>(base) + qb);
+  if (cudaMemsetAsync(word, 0, sizeof(int), s) != cudaSuccess) return SOAP_ERR_CUDA;
+  return soap::qr_q(n, batch, P, Q, skip, tol, base, qb, word, s) == cudaSuccess ? SOAP_OK : SOAP_ERR_CUDA;
 }

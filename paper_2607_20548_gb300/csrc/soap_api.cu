@@ -1,17 +1,24 @@
 // libsoap: the C ABI of include/soap.h.
 //
-// Plan: matrices with the same (rows, cols, sides) form a class; each class keeps
-// its state in contiguous arenas ([count][rows][cols], [count][rows][rows], ...)
-// so every contraction of the step is one batched GEMM per class. The classes' own
-// launches go to the caller's stream (prepared largest factor first, rotated smallest
-// first) and share one workspace sized for the largest class; the QR refreshes are
-// regrouped by factor size, one batched QR per size on its own pair of streams, forked
-// as soon as the last class feeding it is prepared and joined by events before the
-// classes whose bases it refreshes are rotated.
+// Memory plan. The optimizer state proper is all that stays resident: per matrix M_hat and v
+// (rows x cols), the factors L and R as packed lower-triangular tiles (half of a full matrix),
+// and the bases Q_L, Q_R. Matrices with the same (rows, cols, sides) form a class, whose state
+// sits in contiguous arenas ([count][...]). Everything a step forms from that state -- the
+// gradient copy G and G^T, every tensor-core operand's tf32 lo part, Q^T, the unpacked
+// factors, the QR's workspace and the rotation intermediates -- lives in one workspace arena.
+// A step walks the classes in slices (runs of consecutive matrices of one class) grouped into
+// waves: a wave's slices are laid out side by side in the arena, and the next wave reuses it.
+// When the whole model fits, there is one wave holding every class whole; otherwise the waves
+// are cut to the free device memory (or to the caller's workspace limit).
 //
-// Per class, the step (Alg. 1 with the standard factor EMAs of section 2) is:
+// Within a wave, the slices' own launches go to the caller's stream (prepared largest factor
+// first, rotated smallest first); the QR refreshes of the wave are regrouped by factor size, one
+// batched QR per size on its own pair of streams, forked as soon as the last slice feeding it is
+// prepared and joined by events before the slices whose bases it refreshes are rotated.
+//
+// Per slice, the step (Alg. 1 with the standard factor EMAs of section 2) is:
 //   M_hat <- b1 M_hat + (1-b1) G, Gc <- G                 momentum in the original basis
-//   L <- b L + (1-b) Gc Gc^T, R <- b R + (1-b) Gc^T Gc     S1
+//   L <- b L + (1-b) Gc Gc^T, R <- b R + (1-b) Gc^T Gc     S1 (on the unpacked factors, then packed)
 //   P = L Q_L -> Q_L = QR(P).Q; same for R                 S2, S3 (when t mod F == 0)
 //   X1 = Q_L^T Gc, X2 = Q_L^T M_hat                        S5, S4 (re-projected m)
 //   G' = X1 Q_R, m = X2 Q_R
@@ -20,7 +27,7 @@
 // With hparams.stale, S1 moves to the end of the step (the refresh sees the earlier gradients
 // only). With hparams.kl, S1 takes Alg. 1's KL-Shampoo form instead: each factor's EMA term is
 // weighed by the other factor's inverse, Q diag(1/(lam + eps)) Q^T with lam = diag(Q^T F Q)
-// (an identity side as lam = 1); see prepare_class.
+// (an identity side as lam = 1); see accumulate_factors.
 #include <algorithm>
 #include <cstdio>
 #include <cstring>
@@ -39,54 +46,142 @@ struct ClassState {
   bool left = false, right = false;
   int count = 0;
   std::vector<int> members;
-  float* Gc = nullptr;    // G (copy of the caller's gradient); [G | M_hat] unless `tr`
-  float* Mhat = nullptr;  // first moment in the original basis, in the working orientation
-  float* V = nullptr;
-  float* L = nullptr;
-  float* QL = nullptr;
-  float* R = nullptr;
-  float* QR = nullptr;
-  uint8_t* skipL = nullptr;
-  uint8_t* skipR = nullptr;
   size_t ptr_offset = 0;  // index of this class's params pointers in the pointer table
-  // tensor-core path: operand copies and their lo parts
+  // tensor-core path (both dimensions multiples of 4): operand copies with lo parts in the
+  // workspace, factors packed; otherwise CUDA cores with full factors
   bool tc = false;
   // working orientation transposed: a class preconditioned on its left only runs as the
   // right-only problem of G^T, and keeps M_hat and v as M_hat^T and v^T
   bool tr = false;
-  float* Gc_lo = nullptr;  // lo parts of the Gc arena
-  float* Gt = nullptr;     // G^T; [G^T | M_hat^T] if `tr`
-  float* Gt_lo = nullptr;
-  float* Mhat_lo = nullptr;
-  float* L_lo = nullptr;
-  float* R_lo = nullptr;
-  float* QL_lo = nullptr;
-  float* QLt = nullptr;
-  float* QLt_lo = nullptr;
-  float* QR_lo = nullptr;
-  float* QRt = nullptr;
-  float* QRt_lo = nullptr;
-  bool basis_dirty = true;  // Q^T and lo parts must be rebuilt from Q before use
+  // persistent state
+  float* Mhat = nullptr;  // first moment in the original basis, in the working orientation
+  float* V = nullptr;
+  float* L = nullptr;     // tc: [count][packed_floats(rows)]; CUDA cores: [count][rows][rows]
+  float* QL = nullptr;    // [count][rows][rows]
+  float* R = nullptr;
+  float* QR = nullptr;
+  uint8_t* skipL = nullptr;
+  uint8_t* skipR = nullptr;
   // KL-Shampoo factor form, two-sided classes: the approximate eigenvalues of the last step
   float* lamL = nullptr;  // [count][rows]
   float* lamR = nullptr;  // [count][cols]
+  int64_t lpk() const { return tc ? soap::packed_floats((int)rows) : rows * rows; }
+  int64_t rpk() const { return tc ? soap::packed_floats((int)cols) : cols * cols; }
 };
 
-// One preconditioned side of one class: `count` factors of size n in a QR group.
+// `count` consecutive matrices of one class, starting at slot `first`: the persistent state
+// offset to that slot, and the slice's operands in the workspace.
+struct View {
+  int cls = 0, first = 0, count = 0;
+  // persistent state of the slice
+  float *Mhat = nullptr, *V = nullptr, *L = nullptr, *QL = nullptr, *R = nullptr, *QR = nullptr;
+  uint8_t *skipL = nullptr, *skipR = nullptr;
+  float *lamL = nullptr, *lamR = nullptr;
+  // workspace: [G | M_hat copy] (or G alone if tr) and [G^T] (or [G^T | M_hat^T copy]), lo parts
+  float *Gc = nullptr, *Gc_lo = nullptr, *Gt = nullptr, *Gt_lo = nullptr;
+  float *Mc = nullptr, *Mc_lo = nullptr;  // the M_hat copy inside Gc or Gt
+  // workspace: unpacked factors with lo parts, and the bases' lo parts and transposes
+  float *Lf = nullptr, *Lf_lo = nullptr, *QL_lo = nullptr, *QLt = nullptr, *QLt_lo = nullptr;
+  float *Rf = nullptr, *Rf_lo = nullptr, *QR_lo = nullptr, *QRt = nullptr, *QRt_lo = nullptr;
+};
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// View of matrices [first, first + count) of class `cls` with its workspace at `base` (null
+// base: only the size is computed); returns the workspace bytes.
+size_t make_view(const ClassState& c, int cls, int first, int count, char* base, View* v) {
+  View w;
+  w.cls = cls;
+  w.first = first;
+  w.count = count;
+  const int64_t m = c.rows, n = c.cols, mn = m * n;
+  w.Mhat = c.Mhat ? c.Mhat + first * mn : nullptr;
+  w.V = c.V ? c.V + first * mn : nullptr;
+  if (c.left) {
+    w.L = c.L ? c.L + first * c.lpk() : nullptr;
+    w.QL = c.QL ? c.QL + first * m * m : nullptr;
+    w.skipL = c.skipL ? c.skipL + first * m : nullptr;
+    w.lamL = c.lamL ? c.lamL + first * m : nullptr;
+  }
+  if (c.right) {
+    w.R = c.R ? c.R + first * c.rpk() : nullptr;
+    w.QR = c.QR ? c.QR + first * n * n : nullptr;
+    w.skipR = c.skipR ? c.skipR + first * n : nullptr;
+    w.lamR = c.lamR ? c.lamR + first * n : nullptr;
+  }
+  size_t off = 0;
+  auto take = [&](size_t floats) -> float* {
+    const size_t o = off;
+    off += align256(floats * sizeof(float));
+    return base ? reinterpret_cast<float*>(base + o) : nullptr;
+  };
+  const size_t cmn = (size_t)count * mn, cmm = (size_t)count * m * m, cnn = (size_t)count * n * n;
+  if (!c.tc) {
+    w.Gc = take(cmn);  // the gradient copy; M_hat stays where it is
+    w.Lf = w.L;
+    w.Rf = w.R;
+  } else {
+    const size_t ga = c.tr ? cmn : 2 * cmn, ta = c.tr ? 2 * cmn : cmn;
+    w.Gc = take(ga);
+    w.Gc_lo = take(ga);
+    w.Gt = take(ta);
+    w.Gt_lo = take(ta);
+    if (base) {
+      w.Mc = c.tr ? w.Gt + cmn : w.Gc + cmn;
+      w.Mc_lo = c.tr ? w.Gt_lo + cmn : w.Gc_lo + cmn;
+    }
+    if (c.left) {
+      w.Lf = take(cmm);
+      w.Lf_lo = take(cmm);
+      w.QL_lo = take(cmm);
+      w.QLt = take(cmm);
+      w.QLt_lo = take(cmm);
+    }
+    if (c.right) {
+      w.Rf = take(cnn);
+      w.Rf_lo = take(cnn);
+      w.QR_lo = take(cnn);
+      w.QRt = take(cnn);
+      w.QRt_lo = take(cnn);
+    }
+  }
+  if (v) *v = w;
+  return off;
+}
+
+// One preconditioned side of one slice: `count` factors of size n in a QR group.
 struct QrJob {
-  int cls;
+  int slice;
   bool left;
   int offset;  // first batch index of this job inside its group
 };
 
-// All factors of one size, refreshed by one batched QR on their own stream.
+// All factors of one size in a wave, refreshed by one batched QR on their own streams.
 struct QrGroup {
   int n = 0;
   int batch = 0;
   std::vector<QrJob> jobs;
-  void* ws = nullptr;
-  size_t ws_bytes = 0;
-  uint8_t* skip = nullptr;  // [batch][n]
+  size_t ws_off = 0, ws_bytes = 0, skip_off = 0;  // in the arena
+  int slot = 0;                                   // which stream pair and events
+};
+
+struct Slice {
+  int cls = 0, first = 0, count = 0;
+  size_t off = 0;  // workspace offset in the arena
+};
+
+struct Wave {
+  std::vector<Slice> slices;
+  std::vector<int> prep_order;               // slices, largest factor first
+  std::vector<int> update_order;             // slices, smallest largest-factor first
+  std::vector<std::vector<int>> fork_after;  // per slice: groups whose last feeding slice it is
+  std::vector<std::vector<int>> groups_of;   // per slice: the groups its bases come from
+  std::vector<QrGroup> groups;
+  size_t bytes = 0;  // arena bytes the wave uses
+};
+
+// Streams and events of one QR group slot (reused by every wave).
+struct GroupStreams {
   cudaStream_t stream = nullptr;  // panels and the rows that gate them (high priority)
   cudaStream_t far = nullptr;     // the rest of each block's trailing update (low priority)
   cudaEvent_t ev_vt = nullptr, ev_far = nullptr, ev_vq[2] = {nullptr, nullptr};
@@ -116,6 +211,13 @@ struct soap_s {
   std::vector<soap_shape> shapes;
   std::vector<std::pair<int, int>> loc;  // matrix index -> (class, slot)
   std::vector<ClassState> classes;
+  std::vector<Wave> waves;
+  std::vector<GroupStreams> slots;
+  char* arena = nullptr;  // workspace of one wave at a time
+  size_t arena_bytes = 0;
+  size_t state_bytes = 0;
+  // rotation intermediates, shared by the slices of a wave (their rotations run one after
+  // another on the caller's stream)
   float* X1 = nullptr;
   float* X2 = nullptr;
   float* Gp = nullptr;   // [G' | m'] for the tensor-core path: Gp .. Gp + 2 * ws_mat
@@ -126,20 +228,16 @@ struct soap_s {
   float* Zt = nullptr;   // (N Q_R^T)^T
   float* Zt_lo = nullptr;
   float* lam_ws = nullptr;  // Q^T F of the KL form's eigenvalue estimate (two-sided classes)
-  std::vector<QrGroup> groups;  // largest n first
-  std::vector<int> prep_order;               // classes, largest factor first
-  std::vector<int> update_order;             // classes, smallest largest-factor first
-  std::vector<std::vector<int>> fork_after;  // per class: groups whose last feeding class it is
-  std::vector<std::vector<int>> groups_of;   // per class: the groups its bases come from
+  size_t ws_mat = 0;
+  size_t rot_bytes = 0;
   int* d_status = nullptr;
-  int* h_status = nullptr;          // pinned mirror, refreshed after every step
+  int* h_status = nullptr;  // pinned mirror, refreshed after every step
   cudaEvent_t status_ev = nullptr;
   bool status_pending = false;
-  void** h_ptrs = nullptr;          // pinned staging for the params/grads pointer table
-  void** d_ptrs = nullptr;
+  cudaEvent_t step_done = nullptr;  // the last enqueued step's end (steps share the workspace)
+  bool step_recorded = false;
+  void** d_ptrs = nullptr;  // params/grads pointer table, [class][params..., grads...]
   size_t nptrs = 0;
-  cudaEvent_t stage_ev = nullptr;
-  bool stage_pending = false;
   std::vector<void*> last_ptrs;
   std::vector<void*> allocs;
   soap::Profiler prof;
@@ -188,27 +286,17 @@ void free_all(soap_handle h) {
   for (void* p : h->allocs) cudaFree(p);
   h->allocs.clear();
   if (h->h_status) cudaFreeHost(h->h_status);
-  if (h->h_ptrs) cudaFreeHost(h->h_ptrs);
   if (h->status_ev) cudaEventDestroy(h->status_ev);
-  if (h->stage_ev) cudaEventDestroy(h->stage_ev);
-  for (auto& g : h->groups) {
+  if (h->step_done) cudaEventDestroy(h->step_done);
+  for (auto& g : h->slots) {
     if (g.stream) cudaStreamDestroy(g.stream);
     if (g.far) cudaStreamDestroy(g.far);
-    if (g.done) cudaEventDestroy(g.done);
-    if (g.fork) cudaEventDestroy(g.fork);
-    g.fork = nullptr;
-    if (g.ev_vt) cudaEventDestroy(g.ev_vt);
-    if (g.ev_far) cudaEventDestroy(g.ev_far);
-    for (cudaEvent_t& ev : g.ev_vq) {
+    for (cudaEvent_t ev : {g.done, g.fork, g.ev_vt, g.ev_far, g.ev_vq[0], g.ev_vq[1]})
       if (ev) cudaEventDestroy(ev);
-      ev = nullptr;
-    }
-    g.stream = g.far = nullptr;
-    g.done = g.ev_vt = g.ev_far = nullptr;
   }
+  h->slots.clear();
   h->h_status = nullptr;
-  h->h_ptrs = nullptr;
-  h->status_ev = h->stage_ev = nullptr;
+  h->status_ev = h->step_done = nullptr;
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
@@ -222,12 +310,18 @@ soap::TcEpilogue epi(soap_handle h, float* C, int64_t ldc, int64_t c_stride, flo
   return soap::TcEpilogue{C, nullptr, ldc, c_stride, C_lo, ldc, c_stride, transpose, alpha, beta, h->d_status};
 }
 
-// A class's step in three phases, so that the QR refreshes of all classes can be batched by size:
-//   A  operand preparation and S1 (per class, caller's stream)
-//   B  S2 + S3 for every preconditioned side, one batched QR per size group (refresh_bases)
-//   C  S5-S8: rotations, Adam in the basis, back-rotation and update (per class)
+View view_of(soap_handle h, const Slice& sl) {
+  View v;
+  make_view(h->classes[sl.cls], sl.cls, sl.first, sl.count, h->arena + sl.off, &v);
+  return v;
+}
+
+// A slice's step in three phases, so that the QR refreshes of a wave can be batched by size:
+//   A  operand preparation and S1 (per slice, caller's stream)
+//   B  S2 + S3 for every preconditioned side, one batched QR per size group (refresh_group)
+//   C  S5-S8: rotations, Adam in the basis, back-rotation and update (per slice)
 //
-// Two-sided classes run every contraction as a tcgen05 product C = A B^T of K-major operands:
+// Two-sided slices run every contraction as a tcgen05 product C = A B^T of K-major operands:
 //   S1  L <- b L + (1-b) G G^T       A = G,     B = G
 //       R <- b R + (1-b) G^T G       A = G^T,   B = G^T
 //   S2  P^T = Q_L^T L                A = Q_L^T, B = L (symmetric)  -> QR -> Q_L, Q_L^T
@@ -236,31 +330,38 @@ soap::TcEpilogue epi(soap_handle h, float* C, int64_t ldc, int64_t c_stride, flo
 //   S6  N = Adam(G', m', v)
 //   S7  Z^T = (N Q_R^T)^T            A = N,     B = Q_R      (transposed epilogue)
 //   S8  W <- (1 - lr wd) W - lr Q_L Z  A = Q_L, B = Z^T      (epilogue into W)
-// One-sided classes take the same route with one rotation on each side of Adam (a left-only
+// One-sided slices take the same route with one rotation on each side of Adam (a left-only
 // class as the right-only problem of G^T). Classes whose rows or columns are not a multiple
 // of 4 (rows of an operand must be 16-byte multiples for TMA) run on CUDA cores.
-soap_status_t prepare_class(soap_handle h, ClassState& c, const float* const* d_grads, cudaStream_t s) {
+soap_status_t prepare(soap_handle h, const ClassState& c, const View& v, const float* const* d_grads, cudaStream_t s) {
   const soap_hparams& hp = h->hp;
-  const int B = c.count, m = (int)c.rows, n = (int)c.cols;
+  const int B = v.count, m = (int)c.rows, n = (int)c.cols;
   const int64_t mn = (int64_t)m * n;
   if (!c.tc) {
-    SOAP_CUDA(h, soap::momentum_and_copy(d_grads, c.Gc, c.Mhat, mn, B, hp.beta1, h->d_status, s));
+    SOAP_CUDA(h, soap::momentum_and_copy(d_grads, v.Gc, v.Mhat, mn, B, hp.beta1, h->d_status, s));
     return SOAP_OK;
   }
-  SOAP_CUDA(h, soap::momentum_split(d_grads, c.Gc, c.Gc_lo, c.Gt, c.Gt_lo, c.Mhat, c.Mhat_lo, m, n, B, hp.beta1, c.tr,
-                                    h->d_status, s));
-  if (c.basis_dirty) {
-    if (c.left) SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, B, s));
-    if (c.right) SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, n, B, s));
-    c.basis_dirty = false;
+  SOAP_CUDA(h, soap::momentum_split(d_grads, v.Gc, v.Gc_lo, v.Gt, v.Gt_lo, v.Mhat, v.Mc, v.Mc_lo, m, n, B, hp.beta1,
+                                    c.tr, h->d_status, s));
+  // the factors' lo parts are read before S1 rewrites them by the KL form's eigenvalue product
+  // and by the stale variant's refresh
+  const bool lo = hp.kl || hp.stale;
+  if (c.left) {
+    SOAP_CUDA(h, soap::basis_split(v.QL, v.QL_lo, v.QLt, v.QLt_lo, m, B, s));
+    SOAP_CUDA(h, soap::unpack_sym(v.L, v.Lf, lo ? v.Lf_lo : nullptr, m, B, s));
+  }
+  if (c.right) {
+    SOAP_CUDA(h, soap::basis_split(v.QR, v.QR_lo, v.QRt, v.QRt_lo, n, B, s));
+    SOAP_CUDA(h, soap::unpack_sym(v.R, v.Rf, lo ? v.Rf_lo : nullptr, n, B, s));
   }
   return SOAP_OK;
 }
 
-// S1 for one class (after prepare_class): the standard factor EMAs, or Alg. 1's KL form.
-soap_status_t accumulate_factors(soap_handle h, ClassState& c, cudaStream_t s) {
+// S1 for one slice (after prepare): the standard factor EMAs, or Alg. 1's KL form, on the
+// unpacked factors, which are then packed back into the state.
+soap_status_t accumulate_factors(soap_handle h, const ClassState& c, const View& v, cudaStream_t s) {
   const soap_hparams& hp = h->hp;
-  const int B = c.count, m = (int)c.rows, n = (int)c.cols;
+  const int B = v.count, m = (int)c.rows, n = (int)c.cols;
   const int64_t mn = (int64_t)m * n, mm = (int64_t)m * m, nn = (int64_t)n * n;
   const float fb = hp.factor_beta;
   // S1 weights. Standard form: 1 - b. KL form with an identity side (S = I, lambda = 1):
@@ -272,11 +373,11 @@ soap_status_t accumulate_factors(soap_handle h, ClassState& c, cudaStream_t s) {
   using soap::strided_mut;
   if (!c.tc) {
     if (c.left)  // S1: L <- b L + (1-b) G G^T
-      SOAP_CUDA(h, soap::gemm(false, true, m, m, n, aL, strided(c.Gc, n, mn), strided(c.Gc, n, mn), fb,
-                              strided_mut(c.L, m, mm), B, s));
+      SOAP_CUDA(h, soap::gemm(false, true, m, m, n, aL, strided(v.Gc, n, mn), strided(v.Gc, n, mn), fb,
+                              strided_mut(v.L, m, mm), B, s));
     if (c.right)  // S1: R <- b R + (1-b) G^T G
-      SOAP_CUDA(h, soap::gemm(true, false, n, n, m, aR, strided(c.Gc, n, mn), strided(c.Gc, n, mn), fb,
-                              strided_mut(c.R, n, nn), B, s));
+      SOAP_CUDA(h, soap::gemm(true, false, n, n, m, aR, strided(v.Gc, n, mn), strided(v.Gc, n, mn), fb,
+                              strided_mut(v.R, n, nn), B, s));
     return SOAP_OK;
   }
   if (hp.kl && c.left && c.right) {
@@ -288,92 +389,98 @@ soap_status_t accumulate_factors(soap_handle h, ClassState& c, cudaStream_t s) {
     // Y and X (with their lo parts) live in the rotation workspace, free until phase C.
     const int64_t cls = (int64_t)B * mn;
     float* C = h->lam_ws;
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, m, m, B, opnd(c.QLt, c.QLt_lo, m, mm, B), opnd(c.L, c.L_lo, m, mm, B),
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, m, m, B, opnd(v.QLt, v.QLt_lo, m, mm, B), opnd(v.Lf, v.Lf_lo, m, mm, B),
                                   epi(h, C, m, mm, nullptr, 0, 1.f, 0.f), s));
-    SOAP_CUDA(h, soap::diag_dot(C, c.QLt, c.lamL, m, B, s));
-    SOAP_CUDA(h, soap::gemm_tc_nt(n, n, n, B, opnd(c.QRt, c.QRt_lo, n, nn, B), opnd(c.R, c.R_lo, n, nn, B),
+    SOAP_CUDA(h, soap::diag_dot(C, v.QLt, v.lamL, m, B, s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(n, n, n, B, opnd(v.QRt, v.QRt_lo, n, nn, B), opnd(v.Rf, v.Rf_lo, n, nn, B),
                                   epi(h, C, n, nn, nullptr, 0, 1.f, 0.f), s));
-    SOAP_CUDA(h, soap::diag_dot(C, c.QRt, c.lamR, n, B, s));
+    SOAP_CUDA(h, soap::diag_dot(C, v.QRt, v.lamR, n, B, s));
     float* Y = h->YMt;
     float* Y_lo = h->YMt_lo;
     float* X = h->YMt + cls;
     float* X_lo = h->YMt_lo + cls;
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, B, opnd(c.Gc, c.Gc_lo, n, mn, B), opnd(c.QRt, c.QRt_lo, n, nn, B),
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, B, opnd(v.Gc, v.Gc_lo, n, mn, B), opnd(v.QRt, v.QRt_lo, n, nn, B),
                                   epi(h, Y, n, mn, nullptr, 0, 1.f, 0.f), s));
-    SOAP_CUDA(h, soap::scale_cols_split(Y, Y_lo, c.lamR, m, n, B, (float)((1.0 - fb) / n), hp.eps, s));
-    SOAP_CUDA(h, soap::gemm_tc_nt(n, m, m, B, opnd(c.Gt, c.Gt_lo, m, mn, B), opnd(c.QLt, c.QLt_lo, m, mm, B),
+    SOAP_CUDA(h, soap::scale_cols_split(Y, Y_lo, v.lamR, m, n, B, (float)((1.0 - fb) / n), hp.eps, s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(n, m, m, B, opnd(v.Gt, v.Gt_lo, m, mn, B), opnd(v.QLt, v.QLt_lo, m, mm, B),
                                   epi(h, X, m, mn, nullptr, 0, 1.f, 0.f), s));
-    SOAP_CUDA(h, soap::scale_cols_split(X, X_lo, c.lamL, n, m, B, (float)((1.0 - fb) / m), hp.eps, s));
+    SOAP_CUDA(h, soap::scale_cols_split(X, X_lo, v.lamL, n, m, B, (float)((1.0 - fb) / m), hp.eps, s));
     SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(Y, Y_lo, n, mn, B), opnd(Y, Y_lo, n, mn, B),
-                                  epi(h, c.L, m, mm, c.L_lo, 0, 1.f, fb), s));
+                                  epi(h, v.Lf, m, mm, v.Lf_lo, 0, 1.f, fb), s));
     SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(X, X_lo, m, mn, B), opnd(X, X_lo, m, mn, B),
-                                  epi(h, c.R, n, nn, c.R_lo, 0, 1.f, fb), s));
-    return SOAP_OK;
+                                  epi(h, v.Rf, n, nn, v.Rf_lo, 0, 1.f, fb), s));
+  } else {
+    if (c.left)
+      SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(v.Gc, v.Gc_lo, n, mn, B), opnd(v.Gc, v.Gc_lo, n, mn, B),
+                                    epi(h, v.Lf, m, mm, v.Lf_lo, 0, aL, fb), s));
+    if (c.right)
+      SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(v.Gt, v.Gt_lo, m, mn, B), opnd(v.Gt, v.Gt_lo, m, mn, B),
+                                    epi(h, v.Rf, n, nn, v.Rf_lo, 0, aR, fb), s));
   }
-  if (c.left)
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(c.Gc, c.Gc_lo, n, mn, B), opnd(c.Gc, c.Gc_lo, n, mn, B),
-                                  epi(h, c.L, m, mm, c.L_lo, 0, aL, fb), s));
-  if (c.right)
-    SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(c.Gt, c.Gt_lo, m, mn, B), opnd(c.Gt, c.Gt_lo, m, mn, B),
-                                  epi(h, c.R, n, nn, c.R_lo, 0, aR, fb), s));
+  if (c.left) SOAP_CUDA(h, soap::pack_sym(v.Lf, v.L, m, B, s));
+  if (c.right) SOAP_CUDA(h, soap::pack_sym(v.Rf, v.R, n, B, s));
   return SOAP_OK;
 }
 
-// S2 + S3 for the preconditioned sides of one size group: P^T = Q^T F for each member (F the
-// factor, symmetric) into one batched input, one QR, then Q^T, Q (and lo parts) and the
-// zero-column flags back to the classes. The group runs on its own stream from the moment
-// its members' factors are updated on the caller's stream, concurrently with other groups.
-soap_status_t refresh_group(soap_handle h, QrGroup& g, cudaStream_t s) {
+// S2 + S3 for the preconditioned sides of one size group of a wave: P^T = Q^T F for each member
+// (F the unpacked factor, symmetric) into one batched input, one QR, then Q (into the state),
+// Q^T and the lo parts (into the slices' workspace) and the zero-column flags. The group runs
+// on its own streams from the moment its members' factors are updated on the caller's stream,
+// concurrently with other groups.
+soap_status_t refresh_group(soap_handle h, const Wave& w, const QrGroup& g, cudaStream_t s) {
   const soap_hparams& hp = h->hp;
   using soap::strided;
   using soap::strided_mut;
-  SOAP_CUDA(h, cudaEventRecord(g.fork, s));
-  {
-    cudaStream_t gs = g.stream;
-    SOAP_CUDA(h, cudaStreamWaitEvent(gs, g.fork, 0));
-    const int n = g.n;
-    const int64_t nn = (int64_t)n * n;
-    float* At;
-    soap::qr_input_buffers(g.ws, n, g.batch, &At);
-    for (const QrJob& j : g.jobs) {
-      ClassState& c = h->classes[j.cls];
-      float* F = j.left ? c.L : c.R;
-      float* at = At + (int64_t)j.offset * nn;
-      if (c.tc) {
-        SOAP_CUDA(h, soap::gemm_tc_nt(n, n, n, c.count, opnd(j.left ? c.QLt : c.QRt, j.left ? c.QLt_lo : c.QRt_lo, n, nn,
-                                                             c.count),
-                                      opnd(F, j.left ? c.L_lo : c.R_lo, n, nn, c.count),
-                                      epi(h, at, n, nn, nullptr, 0, 1.f, 0.f), gs));
-      } else {
-        SOAP_CUDA(h, soap::gemm(true, false, n, n, n, 1.f, strided(j.left ? c.QL : c.QR, n, nn), strided(F, n, nn), 0.f,
-                                strided_mut(at, n, nn), c.count, gs));
-      }
+  GroupStreams& gs = h->slots[g.slot];
+  SOAP_CUDA(h, cudaEventRecord(gs.fork, s));
+  SOAP_CUDA(h, cudaStreamWaitEvent(gs.stream, gs.fork, 0));
+  const int n = g.n;
+  const int64_t nn = (int64_t)n * n;
+  void* ws = h->arena + g.ws_off;
+  uint8_t* skip = reinterpret_cast<uint8_t*>(h->arena + g.skip_off);
+  float* At;
+  soap::qr_input_buffers(ws, n, g.batch, &At);
+  for (const QrJob& j : g.jobs) {
+    const Slice& sl = w.slices[j.slice];
+    const ClassState& c = h->classes[sl.cls];
+    const View v = view_of(h, sl);
+    float* at = At + (int64_t)j.offset * nn;
+    if (c.tc) {
+      SOAP_CUDA(h, soap::gemm_tc_nt(n, n, n, v.count, opnd(j.left ? v.QLt : v.QRt, j.left ? v.QLt_lo : v.QRt_lo, n, nn,
+                                                           v.count),
+                                    opnd(j.left ? v.Lf : v.Rf, j.left ? v.Lf_lo : v.Rf_lo, n, nn, v.count),
+                                    epi(h, at, n, nn, nullptr, 0, 1.f, 0.f), gs.stream));
+    } else {
+      SOAP_CUDA(h, soap::gemm(true, false, n, n, n, 1.f, strided(j.left ? v.QL : v.QR, n, nn),
+                              strided(j.left ? v.L : v.R, n, nn), 0.f, strided_mut(at, n, nn), v.count, gs.stream));
     }
-    // the Q accumulation ends with Q^T and its lo part in the input buffers
-    const soap::QrLookahead la{g.far, g.ev_vt, g.ev_far, {g.ev_vq[0], g.ev_vq[1]}};
-    SOAP_CUDA(h, soap::qr_q_t(n, g.batch, nullptr, nullptr, nullptr, nullptr, g.skip, hp.qr_tol, g.ws, g.ws_bytes,
-                              h->d_status, gs, &la));
-    for (const QrJob& j : g.jobs) {
-      ClassState& c = h->classes[j.cls];
-      const float* qt = At + (int64_t)j.offset * nn;
-      float* Q = j.left ? c.QL : c.QR;
-      if (c.tc)
-        SOAP_CUDA(h, soap::basis_from_qt(qt, nullptr, j.left ? c.QLt : c.QRt, j.left ? c.QLt_lo : c.QRt_lo, Q,
-                                         j.left ? c.QL_lo : c.QR_lo, n, c.count, gs));
-      else
-        SOAP_CUDA(h, soap::basis_from_qt(qt, nullptr, nullptr, nullptr, Q, nullptr, n, c.count, gs));
-      SOAP_CUDA(h, cudaMemcpyAsync(j.left ? c.skipL : c.skipR, g.skip + (int64_t)j.offset * n, (size_t)c.count * n,
-                                   cudaMemcpyDeviceToDevice, gs));
-    }
-    SOAP_CUDA(h, cudaEventRecord(g.done, gs));
   }
+  // the Q accumulation ends with Q^T in the input buffers
+  const soap::QrLookahead la{gs.far, gs.ev_vt, gs.ev_far, {gs.ev_vq[0], gs.ev_vq[1]}};
+  SOAP_CUDA(h, soap::qr_q_t(n, g.batch, nullptr, nullptr, nullptr, nullptr, skip, hp.qr_tol, ws, g.ws_bytes,
+                            h->d_status, gs.stream, &la));
+  for (const QrJob& j : g.jobs) {
+    const Slice& sl = w.slices[j.slice];
+    const ClassState& c = h->classes[sl.cls];
+    const View v = view_of(h, sl);
+    const float* qt = At + (int64_t)j.offset * nn;
+    float* Q = j.left ? v.QL : v.QR;
+    if (c.tc)
+      SOAP_CUDA(h, soap::basis_from_qt(qt, nullptr, j.left ? v.QLt : v.QRt, j.left ? v.QLt_lo : v.QRt_lo, Q,
+                                       j.left ? v.QL_lo : v.QR_lo, n, v.count, gs.stream));
+    else
+      SOAP_CUDA(h, soap::basis_from_qt(qt, nullptr, nullptr, nullptr, Q, nullptr, n, v.count, gs.stream));
+    SOAP_CUDA(h, cudaMemcpyAsync(j.left ? v.skipL : v.skipR, skip + (int64_t)j.offset * n, (size_t)v.count * n,
+                                 cudaMemcpyDeviceToDevice, gs.stream));
+  }
+  SOAP_CUDA(h, cudaEventRecord(gs.done, gs.stream));
   return SOAP_OK;
 }
 
-soap_status_t rotate_update_class(soap_handle h, ClassState& c, float* const* d_params, float bc1, float bc2,
-                                  cudaStream_t s) {
+soap_status_t rotate_update(soap_handle h, const ClassState& c, const View& v, float* const* d_params, float bc1,
+                            float bc2, cudaStream_t s) {
   const soap_hparams& hp = h->hp;
-  const int B = c.count, m = (int)c.rows, n = (int)c.cols;
+  const int B = v.count, m = (int)c.rows, n = (int)c.cols;
   const int64_t mn = (int64_t)m * n, mm = (int64_t)m * m, nn = (int64_t)n * n;
   using soap::strided;
   using soap::strided_mut;
@@ -385,16 +492,16 @@ soap_status_t rotate_update_class(soap_handle h, ClassState& c, float* const* d_
     //   W <- (1 - lr wd) W - lr N Q^T  A = N,  B = Q   (epilogue into W, transposed if c.tr)
     const int rr = c.tr ? n : m, cc = c.tr ? m : n;
     const int64_t cls = (int64_t)B * mn, qq = (int64_t)cc * cc;
-    const float* X = c.tr ? c.Gt : c.Gc;
-    const float* X_lo = c.tr ? c.Gt_lo : c.Gc_lo;
-    const float* Q = c.tr ? c.QL : c.QR;
-    const float* Q_lo = c.tr ? c.QL_lo : c.QR_lo;
-    const float* Qt = c.tr ? c.QLt : c.QRt;
-    const float* Qt_lo = c.tr ? c.QLt_lo : c.QRt_lo;
+    const float* X = c.tr ? v.Gt : v.Gc;
+    const float* X_lo = c.tr ? v.Gt_lo : v.Gc_lo;
+    const float* Q = c.tr ? v.QL : v.QR;
+    const float* Q_lo = c.tr ? v.QL_lo : v.QR_lo;
+    const float* Qt = c.tr ? v.QLt : v.QRt;
+    const float* Qt_lo = c.tr ? v.QLt_lo : v.QRt_lo;
     SOAP_CUDA(h, soap::gemm_tc_nt(rr, cc, cc, 2 * B, opnd(X, X_lo, cc, mn, 2 * B), opnd(Qt, Qt_lo, cc, qq, B),
                                   epi(h, h->Gp, cc, mn, nullptr, 0, 1.f, 0.f), s));
-    const uint8_t* skip = hp.guard ? (c.tr ? c.skipL : c.skipR) : nullptr;
-    SOAP_CUDA(h, soap::adam_in_basis(h->Gp, h->Gp + cls, c.V, rr, cc, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2, nullptr,
+    const uint8_t* skip = hp.guard ? (c.tr ? v.skipL : v.skipR) : nullptr;
+    SOAP_CUDA(h, soap::adam_in_basis(h->Gp, h->Gp + cls, v.V, rr, cc, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2, nullptr,
                                      skip, h->N_lo, h->d_status, s));
     soap::TcEpilogue ew = epi(h, nullptr, n, 0, nullptr, c.tr ? 1 : 0, -h->lr, 1.f - h->lr * h->wd);
     ew.C_ptrs = d_params;
@@ -404,27 +511,27 @@ soap_status_t rotate_update_class(soap_handle h, ClassState& c, float* const* d_
   if (c.tc) {
     const int64_t cls = (int64_t)B * mn;
     // rotations of the gradient and of the momentum in one launch each (batch 2B)
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, 2 * B, opnd(c.Gc, c.Gc_lo, n, mn, 2 * B), opnd(c.QRt, c.QRt_lo, n, nn, B),
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, 2 * B, opnd(v.Gc, v.Gc_lo, n, mn, 2 * B), opnd(v.QRt, v.QRt_lo, n, nn, B),
                                   epi(h, h->YMt, m, mn, h->YMt_lo, 1, 1.f, 0.f), s));
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, 2 * B, opnd(c.QLt, c.QLt_lo, m, mm, B),
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, 2 * B, opnd(v.QLt, v.QLt_lo, m, mm, B),
                                   opnd(h->YMt, h->YMt_lo, m, mn, 2 * B), epi(h, h->Gp, n, mn, nullptr, 0, 1.f, 0.f), s));
-    SOAP_CUDA(h, soap::adam_in_basis(h->Gp, h->Gp + cls, c.V, m, n, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
-                                     hp.guard ? c.skipL : nullptr, hp.guard ? c.skipR : nullptr, h->N_lo, h->d_status,
+    SOAP_CUDA(h, soap::adam_in_basis(h->Gp, h->Gp + cls, v.V, m, n, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
+                                     hp.guard ? v.skipL : nullptr, hp.guard ? v.skipR : nullptr, h->N_lo, h->d_status,
                                      s));
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, B, opnd(h->Gp, h->N_lo, n, mn, B), opnd(c.QR, c.QR_lo, n, nn, B),
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, n, B, opnd(h->Gp, h->N_lo, n, mn, B), opnd(v.QR, v.QR_lo, n, nn, B),
                                   epi(h, h->Zt, m, mn, h->Zt_lo, 1, 1.f, 0.f), s));
     soap::TcEpilogue ew = epi(h, nullptr, n, 0, nullptr, 0, -h->lr, 1.f - h->lr * h->wd);
     ew.C_ptrs = d_params;
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, B, opnd(c.QL, c.QL_lo, m, mm, B), opnd(h->Zt, h->Zt_lo, m, mn, B), ew, s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, n, m, B, opnd(v.QL, v.QL_lo, m, mm, B), opnd(h->Zt, h->Zt_lo, m, mn, B), ew, s));
     return SOAP_OK;
   }
   // S5 and the re-projected first moment: G' = Q_L^T G Q_R, m = Q_L^T M_hat Q_R
-  const float* xg = c.Gc;
-  const float* xm = c.Mhat;
+  const float* xg = v.Gc;
+  const float* xm = v.Mhat;
   if (c.left) {
-    SOAP_CUDA(h, soap::gemm(true, false, m, n, m, 1.f, strided(c.QL, m, mm), strided(c.Gc, n, mn), 0.f,
+    SOAP_CUDA(h, soap::gemm(true, false, m, n, m, 1.f, strided(v.QL, m, mm), strided(v.Gc, n, mn), 0.f,
                             strided_mut(h->X1, n, mn), B, s));
-    SOAP_CUDA(h, soap::gemm(true, false, m, n, m, 1.f, strided(c.QL, m, mm), strided(c.Mhat, n, mn), 0.f,
+    SOAP_CUDA(h, soap::gemm(true, false, m, n, m, 1.f, strided(v.QL, m, mm), strided(v.Mhat, n, mn), 0.f,
                             strided_mut(h->X2, n, mn), B, s));
     xg = h->X1;
     xm = h->X2;
@@ -432,35 +539,201 @@ soap_status_t rotate_update_class(soap_handle h, ClassState& c, float* const* d_
   float* gp;
   const float* mp;
   if (c.right) {
-    SOAP_CUDA(h, soap::gemm(false, false, m, n, n, 1.f, strided(xg, n, mn), strided(c.QR, n, nn), 0.f,
+    SOAP_CUDA(h, soap::gemm(false, false, m, n, n, 1.f, strided(xg, n, mn), strided(v.QR, n, nn), 0.f,
                             strided_mut(h->Gp, n, mn), B, s));
-    SOAP_CUDA(h, soap::gemm(false, false, m, n, n, 1.f, strided(xm, n, mn), strided(c.QR, n, nn), 0.f,
+    SOAP_CUDA(h, soap::gemm(false, false, m, n, n, 1.f, strided(xm, n, mn), strided(v.QR, n, nn), 0.f,
                             strided_mut(h->Mp, n, mn), B, s));
     gp = h->Gp;
     mp = h->Mp;
   } else {
-    gp = const_cast<float*>(xg);  // X1, or the gradient arena copy when no side rotates
+    gp = const_cast<float*>(xg);  // X1, or the gradient copy when no side rotates
     mp = xm;
   }
   // S6
-  SOAP_CUDA(h, soap::adam_in_basis(gp, mp, c.V, m, n, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
-                                   (hp.guard && c.left) ? c.skipL : nullptr, (hp.guard && c.right) ? c.skipR : nullptr,
+  SOAP_CUDA(h, soap::adam_in_basis(gp, mp, v.V, m, n, B, hp.beta1, hp.beta2, hp.eps, bc1, bc2,
+                                   (hp.guard && c.left) ? v.skipL : nullptr, (hp.guard && c.right) ? v.skipR : nullptr,
                                    nullptr, h->d_status, s));
   // S7 + S8: W <- (1 - lr wd) W - lr Q_L N Q_R^T
   const float keep = 1.f - h->lr * h->wd;
   soap::MutOperand W{nullptr, d_params, 0, 0, n};
   if (c.left && c.right) {
-    SOAP_CUDA(h, soap::gemm(false, false, m, n, m, 1.f, strided(c.QL, m, mm), strided(gp, n, mn), 0.f,
+    SOAP_CUDA(h, soap::gemm(false, false, m, n, m, 1.f, strided(v.QL, m, mm), strided(gp, n, mn), 0.f,
                             strided_mut(h->X1, n, mn), B, s));
-    SOAP_CUDA(h, soap::gemm(false, true, m, n, n, -h->lr, strided(h->X1, n, mn), strided(c.QR, n, nn), keep, W, B, s));
+    SOAP_CUDA(h, soap::gemm(false, true, m, n, n, -h->lr, strided(h->X1, n, mn), strided(v.QR, n, nn), keep, W, B, s));
   } else if (c.left) {
-    SOAP_CUDA(h, soap::gemm(false, false, m, n, m, -h->lr, strided(c.QL, m, mm), strided(gp, n, mn), keep, W, B, s));
+    SOAP_CUDA(h, soap::gemm(false, false, m, n, m, -h->lr, strided(v.QL, m, mm), strided(gp, n, mn), keep, W, B, s));
   } else if (c.right) {
-    SOAP_CUDA(h, soap::gemm(false, true, m, n, n, -h->lr, strided(gp, n, mn), strided(c.QR, n, nn), keep, W, B, s));
+    SOAP_CUDA(h, soap::gemm(false, true, m, n, n, -h->lr, strided(gp, n, mn), strided(v.QR, n, nn), keep, W, B, s));
   } else {
     SOAP_CUDA(h, soap::weight_update(d_params, gp, mn, B, h->lr, h->wd, s));
   }
   return SOAP_OK;
+}
+
+// ---- the wave plan ---------------------------------------------------------------------
+
+int largest_side(const ClassState& c) {
+  return (int)std::max(c.left ? c.rows : (int64_t)0, c.right ? c.cols : (int64_t)0);
+}
+
+// Rotation intermediates (floats) that a slice of `count` matrices of class c needs.
+struct RotSizes {
+  size_t mat = 0, tc = 0, two = 0, x = 0, lam = 0;
+  void grow(const RotSizes& o) {
+    mat = std::max(mat, o.mat);
+    tc = std::max(tc, o.tc);
+    two = std::max(two, o.two);
+    x = std::max(x, o.x);
+    lam = std::max(lam, o.lam);
+  }
+  size_t bytes() const { return 4 * (2 * mat + tc + 4 * two + 2 * two + 2 * x + lam) + 16 * 256; }
+};
+RotSizes rot_sizes(const ClassState& c, int count, bool kl) {
+  RotSizes r;
+  const size_t mn = (size_t)count * c.rows * c.cols;
+  r.mat = mn;
+  if (c.tc) r.tc = mn;
+  if (c.tc && c.left && c.right) r.two = mn;
+  // X1/X2: a CUDA-core slice's intermediates, or one matrix (state reads and writes)
+  r.x = c.tc ? (size_t)(c.rows * c.cols) : mn;
+  if (kl && c.tc && c.left && c.right) r.lam = (size_t)count * std::max(c.rows * c.rows, c.cols * c.cols);
+  return r;
+}
+
+// Lays out one wave: its slices' workspaces and its QR groups in the arena (offsets from 0).
+void layout_wave(soap_handle h, Wave& w) {
+  size_t off = 0;
+  for (Slice& sl : w.slices) {
+    sl.off = off;
+    off += make_view(h->classes[sl.cls], sl.cls, sl.first, sl.count, nullptr, nullptr);
+  }
+  // QR groups: every preconditioned side of the wave's slices, grouped by size, largest first
+  w.groups.clear();
+  std::map<int, int, std::greater<int>> by_n;
+  for (const Slice& sl : w.slices) {
+    const ClassState& c = h->classes[sl.cls];
+    if (c.left) by_n.emplace((int)c.rows, 0);
+    if (c.right) by_n.emplace((int)c.cols, 0);
+  }
+  for (auto& kv : by_n) {
+    kv.second = (int)w.groups.size();
+    QrGroup g;
+    g.n = kv.first;
+    g.slot = kv.second;
+    w.groups.push_back(g);
+  }
+  for (int si = 0; si < (int)w.slices.size(); ++si) {
+    const Slice& sl = w.slices[si];
+    const ClassState& c = h->classes[sl.cls];
+    for (int side = 0; side < 2; ++side) {
+      if (side == 0 ? !c.left : !c.right) continue;
+      QrGroup& g = w.groups[by_n[(int)(side == 0 ? c.rows : c.cols)]];
+      g.jobs.push_back(QrJob{si, side == 0, g.batch});
+      g.batch += sl.count;
+    }
+  }
+  for (QrGroup& g : w.groups) {
+    g.ws_bytes = soap::qr_workspace_bytes(g.n, g.batch, true);
+    g.ws_off = off;
+    off += align256(g.ws_bytes);
+    g.skip_off = off;
+    off += align256((size_t)g.batch * g.n);
+  }
+  w.bytes = off;
+  // step order: see soap_step
+  const int ns = (int)w.slices.size();
+  auto largest = [&](int si) { return largest_side(h->classes[w.slices[si].cls]); };
+  w.prep_order.resize(ns);
+  for (int si = 0; si < ns; ++si) w.prep_order[si] = si;
+  w.update_order = w.prep_order;
+  std::stable_sort(w.prep_order.begin(), w.prep_order.end(), [&](int x, int y) { return largest(x) > largest(y); });
+  std::stable_sort(w.update_order.begin(), w.update_order.end(), [&](int x, int y) { return largest(x) < largest(y); });
+  w.fork_after.assign(ns, {});
+  w.groups_of.assign(ns, {});
+  std::vector<int> pos(ns);
+  for (int q = 0; q < ns; ++q) pos[w.prep_order[q]] = q;
+  for (int gi = 0; gi < (int)w.groups.size(); ++gi) {
+    int last = -1;
+    for (const QrJob& j : w.groups[gi].jobs) {
+      w.groups_of[j.slice].push_back(gi);
+      if (last < 0 || pos[j.slice] > pos[last]) last = j.slice;
+    }
+    if (last >= 0) w.fork_after[last].push_back(gi);
+  }
+}
+
+// Largest slice a wave (or a product launch) may hold: batched launches index matrices in a
+// 16-bit grid dimension, and the rotations run [G | M_hat] as one batch of twice the slice.
+constexpr int kMaxSlice = 32767;
+
+// Cuts the classes into waves whose workspace (arena + rotation intermediates) fits `budget`
+// bytes. Returns false if some class cannot fit even one matrix.
+bool plan_waves(soap_handle h, size_t budget, bool single_ok, std::vector<Wave>* out, RotSizes* rot) {
+  const int nc = (int)h->classes.size();
+  std::vector<int> order(nc);
+  for (int ci = 0; ci < nc; ++ci) order[ci] = ci;
+  std::stable_sort(order.begin(), order.end(),
+                   [&](int x, int y) { return largest_side(h->classes[x]) > largest_side(h->classes[y]); });
+  const bool kl = h->hp.kl != 0;
+  if (single_ok) {
+    // every class whole in one wave
+    Wave w;
+    RotSizes r;
+    bool fits = true;
+    for (int ci : order) {
+      const ClassState& c = h->classes[ci];
+      if (c.count > kMaxSlice) fits = false;
+      w.slices.push_back(Slice{ci, 0, c.count, 0});
+      r.grow(rot_sizes(c, c.count, kl));
+    }
+    layout_wave(h, w);
+    for (const QrGroup& g : w.groups)
+      if (g.batch > 65535) fits = false;
+    if (fits && w.bytes + r.bytes() <= budget) {
+      out->assign(1, w);
+      *rot = r;
+      return true;
+    }
+  }
+  // waves cut to the budget: a slice costs its workspace, its share of its QR groups and (as if
+  // every slice needed its own) its rotation intermediates per matrix, so the sum is an upper bound
+  auto per_matrix = [&](const ClassState& c) {
+    size_t b = make_view(c, 0, 0, 1, nullptr, nullptr) + rot_sizes(c, 1, kl).bytes();
+    if (c.left) b += soap::qr_workspace_bytes((int)c.rows, 1, true) + (size_t)c.rows + 64 * 256;
+    if (c.right) b += soap::qr_workspace_bytes((int)c.cols, 1, true) + (size_t)c.cols + 64 * 256;
+    return b + 8 * 256;
+  };
+  std::vector<Wave> waves;
+  Wave cur;
+  size_t used = 0;
+  for (int ci : order) {
+    const ClassState& c = h->classes[ci];
+    const size_t pm = per_matrix(c);
+    if (pm > budget) return false;
+    int first = 0;
+    while (first < c.count) {
+      int k = (int)std::min<size_t>((size_t)(c.count - first), (budget - used) / pm);
+      k = std::min(k, kMaxSlice);
+      if (k <= 0) {
+        waves.push_back(cur);
+        cur = Wave();
+        used = 0;
+        continue;
+      }
+      cur.slices.push_back(Slice{ci, first, k, 0});
+      used += (size_t)k * pm;
+      first += k;
+    }
+  }
+  if (!cur.slices.empty()) waves.push_back(cur);
+  RotSizes r;
+  for (Wave& w : waves) {
+    layout_wave(h, w);
+    for (const Slice& sl : w.slices) r.grow(rot_sizes(h->classes[sl.cls], sl.count, kl));
+  }
+  *out = waves;
+  *rot = r;
+  return true;
 }
 
 }  // namespace
@@ -483,8 +756,8 @@ void soap_default_hparams(soap_hparams* hp) {
   hp->stale = 0;
 }
 
-soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparams* hp,
-                          int32_t device, soap_handle* out) {
+soap_status_t soap_create_ex(const soap_shape* shapes, int32_t n, const soap_hparams* hp, int32_t device,
+                             size_t workspace_limit, soap_handle* out) {
   if (!out) return SOAP_ERR_INVALID_ARG;
   *out = nullptr;
   if (!shapes || n <= 0 || !hp) return SOAP_ERR_INVALID_ARG;
@@ -533,16 +806,14 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
     h->classes[ci].members.push_back(i);
     h->classes[ci].count++;
   }
-  for (auto& c : h->classes) {
-    if (c.count > 65535) {
-      delete h;
-      return SOAP_ERR_INVALID_ARG;
-    }
-  }
 
-  size_t ws_mat = 0;
+  // persistent state
   size_t off = 0;
   cudaError_t e = cudaSuccess;
+  auto take = [&](void** p, size_t bytes) {
+    if (e == cudaSuccess) e = dalloc(h, p, bytes);
+    if (e == cudaSuccess) h->state_bytes += bytes;
+  };
   for (auto& c : h->classes) {
     const size_t mn = (size_t)c.count * c.rows * c.cols;
     c.ptr_offset = off;
@@ -550,152 +821,72 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
     // tensor-core operands are read with TMA: rows of both G and G^T must be 16-byte multiples
     c.tc = (c.left || c.right) && (c.rows % 4 == 0) && (c.cols % 4 == 0);
     c.tr = c.tc && c.left && !c.right;
-    // the arena holding M_hat directly after G (or G^T), so that one batch-2B product rotates both
-    const size_t ga = c.tr ? mn : 2 * mn, ta = c.tr ? 2 * mn : mn;
-    if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gc, (c.tc ? ga : 2 * mn) * 4);
-    if (e == cudaSuccess) e = dalloc(h, (void**)&c.V, mn * 4);
-    if (c.tc) {
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gc_lo, ga * 4);
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gt, ta * 4);
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.Gt_lo, ta * 4);
-    }
-    if (e == cudaSuccess) {
-      c.Mhat = c.tr ? c.Gt + mn : c.Gc + mn;
-      c.Mhat_lo = !c.tc ? nullptr : c.tr ? c.Gt_lo + mn : c.Gc_lo + mn;
-    }
+    take((void**)&c.Mhat, mn * 4);
+    take((void**)&c.V, mn * 4);
     if (c.left) {
-      const size_t mm = (size_t)c.count * c.rows * c.rows;
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.L, mm * 4);
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.QL, mm * 4);
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.skipL, (size_t)c.count * c.rows);
-      if (c.tc) {
-        if (e == cudaSuccess) e = dalloc(h, (void**)&c.L_lo, mm * 4);
-        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QL_lo, mm * 4);
-        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QLt, mm * 4);
-        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QLt_lo, mm * 4);
-      }
+      take((void**)&c.L, (size_t)c.count * c.lpk() * 4);
+      take((void**)&c.QL, (size_t)c.count * c.rows * c.rows * 4);
+      take((void**)&c.skipL, (size_t)c.count * c.rows);
     }
     if (c.right) {
-      const size_t nn = (size_t)c.count * c.cols * c.cols;
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.R, nn * 4);
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.QR, nn * 4);
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.skipR, (size_t)c.count * c.cols);
-      if (c.tc) {
-        if (e == cudaSuccess) e = dalloc(h, (void**)&c.R_lo, nn * 4);
-        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QR_lo, nn * 4);
-        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QRt, nn * 4);
-        if (e == cudaSuccess) e = dalloc(h, (void**)&c.QRt_lo, nn * 4);
-      }
+      take((void**)&c.R, (size_t)c.count * c.rpk() * 4);
+      take((void**)&c.QR, (size_t)c.count * c.cols * c.cols * 4);
+      take((void**)&c.skipR, (size_t)c.count * c.cols);
     }
     if (hp->kl && c.left && c.right) {
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.lamL, (size_t)c.count * c.rows * 4);
-      if (e == cudaSuccess) e = dalloc(h, (void**)&c.lamR, (size_t)c.count * c.cols * 4);
-      if (e == cudaSuccess) e = cudaMemset(c.lamL, 0, (size_t)c.count * c.rows * 4);
-      if (e == cudaSuccess) e = cudaMemset(c.lamR, 0, (size_t)c.count * c.cols * 4);
-    }
-    ws_mat = std::max(ws_mat, mn);
-  }
-  // QR groups: every preconditioned side, grouped by size
-  {
-    std::map<int, int, std::greater<int>> by_n;
-    for (int ci = 0; ci < (int)h->classes.size(); ++ci) {
-      const ClassState& c = h->classes[ci];
-      for (int side = 0; side < 2; ++side) {
-        if (side == 0 ? !c.left : !c.right) continue;
-        const int n = (int)(side == 0 ? c.rows : c.cols);
-        auto it = by_n.find(n);
-        if (it == by_n.end()) it = by_n.emplace(n, (int)by_n.size()).first;
-        (void)it;
-      }
-    }
-    for (auto& kv : by_n) {
-      QrGroup g;
-      g.n = kv.first;
-      h->groups.push_back(g);
-    }
-    for (int ci = 0; ci < (int)h->classes.size(); ++ci) {
-      const ClassState& c = h->classes[ci];
-      for (int side = 0; side < 2; ++side) {
-        if (side == 0 ? !c.left : !c.right) continue;
-        const int n = (int)(side == 0 ? c.rows : c.cols);
-        for (auto& g : h->groups)
-          if (g.n == n) {
-            g.jobs.push_back(QrJob{ci, side == 0, g.batch});
-            g.batch += c.count;
-          }
-      }
-    }
-    for (auto& g : h->groups) {
-      if (g.batch > 65535) e = cudaErrorInvalidValue;
-      g.ws_bytes = soap::qr_workspace_bytes(g.n, g.batch, true);
-      if (e == cudaSuccess) e = dalloc(h, &g.ws, g.ws_bytes);
-      if (e == cudaSuccess) e = dalloc(h, (void**)&g.skip, (size_t)g.batch * g.n);
-      // the panel chain is latency-bound: its stream goes first when SMs free up
-      int prio_lo = 0, prio_hi = 0;
-      if (e == cudaSuccess) e = cudaDeviceGetStreamPriorityRange(&prio_lo, &prio_hi);
-      if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&g.stream, cudaStreamNonBlocking, prio_hi);
-      if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&g.far, cudaStreamNonBlocking, prio_lo);
-      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.done, cudaEventDisableTiming);
-      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.fork, cudaEventDisableTiming);
-      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.ev_vt, cudaEventDisableTiming);
-      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&g.ev_far, cudaEventDisableTiming);
-      for (cudaEvent_t& ev : g.ev_vq)
-        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
-    }
-    // step order: see soap_step
-    const int nc = (int)h->classes.size();
-    auto largest = [&](int ci) {
-      const ClassState& c = h->classes[ci];
-      return std::max(c.left ? c.rows : (int64_t)0, c.right ? c.cols : (int64_t)0);
-    };
-    h->prep_order.resize(nc);
-    for (int ci = 0; ci < nc; ++ci) h->prep_order[ci] = ci;
-    h->update_order = h->prep_order;
-    std::stable_sort(h->prep_order.begin(), h->prep_order.end(), [&](int x, int y) { return largest(x) > largest(y); });
-    std::stable_sort(h->update_order.begin(), h->update_order.end(),
-                     [&](int x, int y) { return largest(x) < largest(y); });
-    h->fork_after.assign(nc, {});
-    h->groups_of.assign(nc, {});
-    std::vector<int> pos(nc);
-    for (int q = 0; q < nc; ++q) pos[h->prep_order[q]] = q;
-    for (int gi = 0; gi < (int)h->groups.size(); ++gi) {
-      int last = -1;
-      for (const QrJob& j : h->groups[gi].jobs) {
-        h->groups_of[j.cls].push_back(gi);
-        if (last < 0 || pos[j.cls] > pos[last]) last = j.cls;
-      }
-      if (last >= 0) h->fork_after[last].push_back(gi);
+      take((void**)&c.lamL, (size_t)c.count * c.rows * 4);
+      take((void**)&c.lamR, (size_t)c.count * c.cols * 4);
     }
   }
   h->nptrs = off;
-  // workspaces: [G' | m'] for every class; N's lo part for tensor-core classes; the
-  // intermediate products of two-sided tensor-core classes; X1/X2 for CUDA-core classes and
-  // for single-matrix state reads and writes
-  size_t ws_tc = 0, ws_two = 0, ws_x = 0, ws_lam = 0;
-  for (auto& c : h->classes) {
-    const size_t mn = (size_t)c.count * c.rows * c.cols;
-    if (c.tc) ws_tc = std::max(ws_tc, mn);
-    if (c.tc && c.left && c.right) ws_two = std::max(ws_two, mn);
-    if (hp->kl && c.left && c.right)
-      ws_lam = std::max(ws_lam, (size_t)c.count * std::max(c.rows * c.rows, c.cols * c.cols));
-    ws_x = std::max(ws_x, c.tc ? (size_t)(c.rows * c.cols) : mn);
-  }
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->X1, ws_x * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->X2, ws_x * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Gp, 2 * ws_mat * 4);
-  h->Mp = h->Gp ? h->Gp + ws_mat : nullptr;
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->N_lo, ws_tc * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt, 2 * ws_two * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt_lo, 2 * ws_two * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt, ws_two * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt_lo, ws_two * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->lam_ws, ws_lam * 4);
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_status, sizeof(int));
-  if (e == cudaSuccess) e = dalloc(h, (void**)&h->d_ptrs, h->nptrs * sizeof(void*));
+  take((void**)&h->d_status, sizeof(int));
+  take((void**)&h->d_ptrs, h->nptrs * sizeof(void*));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&h->h_status, sizeof(int));
-  if (e == cudaSuccess) e = cudaMallocHost((void**)&h->h_ptrs, h->nptrs * sizeof(void*));
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->status_ev, cudaEventDisableTiming);
-  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->stage_ev, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->step_done, cudaEventDisableTiming);
+
+  // the workspace: one wave holding every class if that fits (within the limit, or leaving a
+  // reserve of free memory), else waves cut to what is available
+  RotSizes rot;
+  if (e == cudaSuccess) {
+    size_t free_b = 0, total_b = 0;
+    e = cudaMemGetInfo(&free_b, &total_b);
+    const size_t reserve = (size_t(1) << 30) + total_b / 100;
+    const size_t avail = free_b > reserve ? free_b - reserve : 0;
+    const size_t budget = workspace_limit ? std::min(workspace_limit, avail) : avail;
+    if (e == cudaSuccess && !plan_waves(h, budget, true, &h->waves, &rot)) e = cudaErrorMemoryAllocation;
+  }
+  if (e == cudaSuccess) {
+    for (const Wave& w : h->waves) h->arena_bytes = std::max(h->arena_bytes, w.bytes);
+    e = dalloc(h, (void**)&h->arena, h->arena_bytes);
+  }
+  size_t nslots = 0;
+  for (const Wave& w : h->waves) nslots = std::max(nslots, w.groups.size());
+  h->slots.resize(nslots);
+  for (GroupStreams& gs : h->slots) {
+    // the panel chain is latency-bound: its stream goes first when SMs free up
+    int prio_lo = 0, prio_hi = 0;
+    if (e == cudaSuccess) e = cudaDeviceGetStreamPriorityRange(&prio_lo, &prio_hi);
+    if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&gs.stream, cudaStreamNonBlocking, prio_hi);
+    if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&gs.far, cudaStreamNonBlocking, prio_lo);
+    for (cudaEvent_t* ev : {&gs.done, &gs.fork, &gs.ev_vt, &gs.ev_far, &gs.ev_vq[0], &gs.ev_vq[1]})
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming);
+  }
+  // rotation intermediates: [G' | m'] for every slice; N's lo part for tensor-core slices; the
+  // intermediate products of two-sided tensor-core slices; X1/X2 for CUDA-core slices and for
+  // single-matrix state reads and writes; Q^T F for the KL form's eigenvalues
+  h->ws_mat = rot.mat;
+  h->rot_bytes = rot.bytes();
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->X1, rot.x * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->X2, rot.x * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Gp, 2 * rot.mat * 4);
+  h->Mp = h->Gp ? h->Gp + rot.mat : nullptr;
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->N_lo, rot.tc * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt, 2 * rot.two * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->YMt_lo, 2 * rot.two * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt, rot.two * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->Zt_lo, rot.two * 4);
+  if (e == cudaSuccess) e = dalloc(h, (void**)&h->lam_ws, rot.lam * 4);
   if (e != cudaSuccess) {
     soap_status_t code = e == cudaErrorMemoryAllocation ? SOAP_ERR_OOM : SOAP_ERR_CUDA;
     free_all(h);
@@ -708,20 +899,19 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
   for (auto& c : h->classes) {
     const size_t mn = (size_t)c.count * c.rows * c.cols;
     if (e == cudaSuccess) e = cudaMemset(c.Mhat, 0, mn * 4);
-    if (c.tc && e == cudaSuccess) e = cudaMemset(c.Mhat_lo, 0, mn * 4);
     if (e == cudaSuccess) e = cudaMemset(c.V, 0, mn * 4);
     if (c.left) {
-      if (e == cudaSuccess) e = cudaMemset(c.L, 0, (size_t)c.count * c.rows * c.rows * 4);
-      if (c.tc && e == cudaSuccess) e = cudaMemset(c.L_lo, 0, (size_t)c.count * c.rows * c.rows * 4);
+      if (e == cudaSuccess) e = cudaMemset(c.L, 0, (size_t)c.count * c.lpk() * 4);
       if (e == cudaSuccess) e = soap::set_identity(c.QL, (int)c.rows, c.count, 0);
       if (e == cudaSuccess) e = cudaMemset(c.skipL, 0, (size_t)c.count * c.rows);
     }
     if (c.right) {
-      if (e == cudaSuccess) e = cudaMemset(c.R, 0, (size_t)c.count * c.cols * c.cols * 4);
-      if (c.tc && e == cudaSuccess) e = cudaMemset(c.R_lo, 0, (size_t)c.count * c.cols * c.cols * 4);
+      if (e == cudaSuccess) e = cudaMemset(c.R, 0, (size_t)c.count * c.rpk() * 4);
       if (e == cudaSuccess) e = soap::set_identity(c.QR, (int)c.cols, c.count, 0);
       if (e == cudaSuccess) e = cudaMemset(c.skipR, 0, (size_t)c.count * c.cols);
     }
+    if (c.lamL && e == cudaSuccess) e = cudaMemset(c.lamL, 0, (size_t)c.count * c.rows * 4);
+    if (c.lamR && e == cudaSuccess) e = cudaMemset(c.lamR, 0, (size_t)c.count * c.cols * 4);
   }
   if (e == cudaSuccess) e = cudaMemset(h->d_status, 0, sizeof(int));
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
@@ -733,6 +923,19 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
   }
   h->last_ptrs.assign(h->nptrs, nullptr);
   *out = h;
+  return SOAP_OK;
+}
+
+soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparams* hp, int32_t device,
+                          soap_handle* out) {
+  return soap_create_ex(shapes, n, hp, device, 0, out);
+}
+
+soap_status_t soap_plan_info(soap_handle h, int32_t* waves, size_t* workspace_bytes, size_t* state_bytes) {
+  if (!h) return SOAP_ERR_INVALID_ARG;
+  if (waves) *waves = (int32_t)h->waves.size();
+  if (workspace_bytes) *workspace_bytes = h->arena_bytes + h->rot_bytes;
+  if (state_bytes) *state_bytes = h->state_bytes;
   return SOAP_OK;
 }
 
@@ -761,7 +964,10 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
     soap_status_t st = status_code(*h->h_status);
     if (st != SOAP_OK) return fail(h, st, "soap_step: sticky device status from an earlier step");
   }
-  // pointer table: [class][params..., grads...], uploaded only when it changed
+  // steps share the workspace: a step on another stream starts after the previous one ends
+  if (h->step_recorded) SOAP_CUDA(h, cudaStreamWaitEvent(s, h->step_done, 0));
+  // pointer table: [class][params..., grads...], written on the stream through kernel
+  // parameters when it changed (nothing on the host waits)
   bool changed = false;
   for (auto& c : h->classes) {
     for (int j = 0; j < c.count; ++j) {
@@ -773,13 +979,7 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
       h->last_ptrs[c.ptr_offset + c.count + j] = gp;
     }
   }
-  if (changed) {
-    if (h->stage_pending) SOAP_CUDA(h, cudaEventSynchronize(h->stage_ev));
-    std::memcpy(h->h_ptrs, h->last_ptrs.data(), h->nptrs * sizeof(void*));
-    SOAP_CUDA(h, cudaMemcpyAsync(h->d_ptrs, h->h_ptrs, h->nptrs * sizeof(void*), cudaMemcpyHostToDevice, s));
-    SOAP_CUDA(h, cudaEventRecord(h->stage_ev, s));
-    h->stage_pending = true;
-  }
+  if (changed) SOAP_CUDA(h, soap::put_ptrs(h->d_ptrs, h->last_ptrs.data(), (int64_t)h->nptrs, s));
 
   h->t += 1;
   const int64_t t = h->t;
@@ -787,46 +987,58 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
   const bool refresh = (t % hp.eig_every) == 0;
   const float bc1 = hp.bias_correction ? 1.f - powf(hp.beta1, (float)t) : 1.f;
   const float bc2 = hp.bias_correction ? 1.f - powf(hp.beta2, (float)t) : 1.f;
-  auto params_of = [&](const ClassState& c) { return reinterpret_cast<float* const*>(h->d_ptrs + c.ptr_offset); };
-  auto grads_of = [&](const ClassState& c) {
-    return reinterpret_cast<const float* const*>(h->d_ptrs + c.ptr_offset + c.count);
+  auto params_of = [&](const Slice& sl) {
+    return reinterpret_cast<float* const*>(h->d_ptrs + h->classes[sl.cls].ptr_offset + sl.first);
   };
-  // Phase A class by class, each size group's refresh forked as soon as the last class feeding
-  // it is prepared (classes with the largest factors first, so the longest refresh starts
-  // earliest); phase C class by class, each waiting only for the groups its bases come from
-  // (classes with the smallest factors first, whose refreshes finish earliest).
-  // The stale variant refreshes from the factors as they stand and accumulates G_t into them
-  // at the end of the step.
-  for (int ci : h->prep_order) {
-    soap_status_t st = prepare_class(h, h->classes[ci], grads_of(h->classes[ci]), s);
-    if (st == SOAP_OK && !hp.stale) st = accumulate_factors(h, h->classes[ci], s);
-    if (st != SOAP_OK) return st;
-    if (refresh)
-      for (int gi : h->fork_after[ci]) {
-        st = refresh_group(h, h->groups[gi], s);
+  auto grads_of = [&](const Slice& sl) {
+    const ClassState& c = h->classes[sl.cls];
+    return reinterpret_cast<const float* const*>(h->d_ptrs + c.ptr_offset + c.count + sl.first);
+  };
+  // Wave by wave: phase A slice by slice, each size group's refresh forked as soon as the last
+  // slice feeding it is prepared (slices with the largest factors first, so the longest refresh
+  // starts earliest); phase C slice by slice, each waiting only for the groups its bases come
+  // from (slices with the smallest factors first, whose refreshes finish earliest). Every group
+  // is joined before the next wave reuses the workspace. The stale variant refreshes from the
+  // factors as they stand and accumulates G_t into them after the wave's updates.
+  for (const Wave& w : h->waves) {
+    for (int si : w.prep_order) {
+      const Slice& sl = w.slices[si];
+      const ClassState& c = h->classes[sl.cls];
+      const View v = view_of(h, sl);
+      soap_status_t st = prepare(h, c, v, grads_of(sl), s);
+      if (st == SOAP_OK && !hp.stale) st = accumulate_factors(h, c, v, s);
+      if (st != SOAP_OK) return st;
+      if (refresh)
+        for (int gi : w.fork_after[si]) {
+          st = refresh_group(h, w, w.groups[gi], s);
+          if (st != SOAP_OK) return st;
+        }
+    }
+    std::vector<bool> joined(w.groups.size(), !refresh);
+    for (int si : w.update_order) {
+      for (int gi : w.groups_of[si])
+        if (!joined[gi]) {
+          SOAP_CUDA(h, cudaStreamWaitEvent(s, h->slots[w.groups[gi].slot].done, 0));
+          joined[gi] = true;
+        }
+      const Slice& sl = w.slices[si];
+      soap_status_t st = rotate_update(h, h->classes[sl.cls], view_of(h, sl), params_of(sl), bc1, bc2, s);
+      if (st != SOAP_OK) return st;
+    }
+    for (size_t gi = 0; gi < w.groups.size(); ++gi)
+      if (!joined[gi]) SOAP_CUDA(h, cudaStreamWaitEvent(s, h->slots[w.groups[gi].slot].done, 0));
+    if (hp.stale)
+      for (int si : w.prep_order) {
+        const Slice& sl = w.slices[si];
+        soap_status_t st = accumulate_factors(h, h->classes[sl.cls], view_of(h, sl), s);
         if (st != SOAP_OK) return st;
       }
   }
-  std::vector<bool> joined(h->groups.size(), !refresh);
-  for (int ci : h->update_order) {
-    for (int gi : h->groups_of[ci])
-      if (!joined[gi]) {
-        SOAP_CUDA(h, cudaStreamWaitEvent(s, h->groups[gi].done, 0));
-        joined[gi] = true;
-      }
-    soap_status_t st = rotate_update_class(h, h->classes[ci], params_of(h->classes[ci]), bc1, bc2, s);
-    if (st != SOAP_OK) return st;
-  }
-  for (size_t gi = 0; gi < h->groups.size(); ++gi)
-    if (!joined[gi]) SOAP_CUDA(h, cudaStreamWaitEvent(s, h->groups[gi].done, 0));
-  if (hp.stale)
-    for (auto& c : h->classes) {
-      soap_status_t st = accumulate_factors(h, c, s);
-      if (st != SOAP_OK) return st;
-    }
   SOAP_CUDA(h, cudaMemcpyAsync(h->h_status, h->d_status, sizeof(int), cudaMemcpyDeviceToHost, s));
   SOAP_CUDA(h, cudaEventRecord(h->status_ev, s));
+  SOAP_CUDA(h, cudaEventRecord(h->step_done, s));
   h->status_pending = true;
+  h->step_recorded = true;
   return SOAP_OK;
 }
 
@@ -851,149 +1063,192 @@ size_t soap_state_bytes(soap_handle h, int32_t idx, int32_t which) {
   }
 }
 
+}  // extern "C"
+
 namespace {
-// Address of a stored state piece (not SOAP_STATE_M, which is derived).
-void* state_ptr(soap_handle h, int idx, int which) {
+// One matrix of the state as a slice of its own, with its workspace at the start of the arena
+// (state reads and writes are ordered with the steps, which use the same arena).
+View single_view(soap_handle h, int idx) {
   const auto [ci, slot] = h->loc[idx];
-  ClassState& c = h->classes[ci];
-  const size_t mn = (size_t)c.rows * c.cols, mm = (size_t)c.rows * c.rows, nn = (size_t)c.cols * c.cols;
+  View v;
+  make_view(h->classes[ci], ci, slot, 1, h->arena, &v);
+  return v;
+}
+
+// Address of a piece kept as it is handed out (not SOAP_STATE_M, which is derived, nor a
+// packed factor).
+void* state_ptr(const View& v, int which) {
   switch (which) {
-    case SOAP_STATE_V: return c.V + slot * mn;
-    case SOAP_STATE_MHAT: return c.Mhat + slot * mn;
-    case SOAP_STATE_L: return c.L ? c.L + slot * mm : nullptr;
-    case SOAP_STATE_QL: return c.QL ? c.QL + slot * mm : nullptr;
-    case SOAP_STATE_R: return c.R ? c.R + slot * nn : nullptr;
-    case SOAP_STATE_QR: return c.QR ? c.QR + slot * nn : nullptr;
-    case SOAP_STATE_SKIP_L: return c.skipL ? c.skipL + slot * c.rows : nullptr;
-    case SOAP_STATE_SKIP_R: return c.skipR ? c.skipR + slot * c.cols : nullptr;
-    case SOAP_STATE_LAMBDA_L: return c.lamL ? c.lamL + slot * c.rows : nullptr;
-    case SOAP_STATE_LAMBDA_R: return c.lamR ? c.lamR + slot * c.cols : nullptr;
+    case SOAP_STATE_V: return v.V;
+    case SOAP_STATE_MHAT: return v.Mhat;
+    case SOAP_STATE_QL: return v.QL;
+    case SOAP_STATE_QR: return v.QR;
+    case SOAP_STATE_SKIP_L: return v.skipL;
+    case SOAP_STATE_SKIP_R: return v.skipR;
+    case SOAP_STATE_LAMBDA_L: return v.lamL;
+    case SOAP_STATE_LAMBDA_R: return v.lamR;
     default: return nullptr;
   }
 }
-}  // namespace
 
-soap_status_t soap_state_get(soap_handle h, int32_t idx, int32_t which, void* dst, soap_stream_t stream_) {
-  if (!h) return SOAP_ERR_INVALID_ARG;
+soap_status_t state_get_impl(soap_handle h, int32_t idx, int32_t which, void* dst, soap_stream_t stream_) {
   const size_t bytes = soap_state_bytes(h, idx, which);
   if (bytes == 0 || !dst) return fail(h, SOAP_ERR_INVALID_ARG, "soap_state_get: no such state piece");
   DeviceGuard g(h->device);
   cudaStream_t s = (cudaStream_t)stream_;
-  const auto [ci, slot] = h->loc[idx];
-  ClassState& c = h->classes[ci];
+  const ClassState& c = h->classes[h->loc[idx].first];
+  const View v = single_view(h, idx);
   const int m = (int)c.rows, nc = (int)c.cols;
   const int64_t mn = (int64_t)m * nc;
   if (c.tr && (which == SOAP_STATE_V || which == SOAP_STATE_MHAT)) {
     // stored transposed (n x m): hand out the m x n matrix
-    SOAP_CUDA(h, soap::transpose((const float*)state_ptr(h, idx, which), h->X1, nc, m, 1, s));
+    SOAP_CUDA(h, soap::transpose((const float*)state_ptr(v, which), h->X1, nc, m, 1, s));
     SOAP_CUDA(h, cudaMemcpyAsync(dst, h->X1, bytes, cudaMemcpyDefault, s));
     return SOAP_OK;
   }
+  if (which == SOAP_STATE_L || which == SOAP_STATE_R) {
+    const bool left = which == SOAP_STATE_L;
+    const float* F = left ? v.L : v.R;
+    if (c.tc) {
+      SOAP_CUDA(h, soap::unpack_sym(F, left ? v.Lf : v.Rf, nullptr, left ? m : nc, 1, s));
+      F = left ? v.Lf : v.Rf;
+    }
+    SOAP_CUDA(h, cudaMemcpyAsync(dst, F, bytes, cudaMemcpyDefault, s));
+    return SOAP_OK;
+  }
   if (which != SOAP_STATE_M) {
-    SOAP_CUDA(h, cudaMemcpyAsync(dst, state_ptr(h, idx, which), bytes, cudaMemcpyDefault, s));
+    SOAP_CUDA(h, cudaMemcpyAsync(dst, state_ptr(v, which), bytes, cudaMemcpyDefault, s));
     return SOAP_OK;
   }
-  // m = Q_L^T M_hat Q_R, computed into the workspace
-  const float* x = c.Mhat + slot * mn;
-  if (c.tc && c.basis_dirty) {
-    if (c.left) SOAP_CUDA(h, soap::basis_split(c.QL, c.QL_lo, c.QLt, c.QLt_lo, m, c.count, s));
-    if (c.right) SOAP_CUDA(h, soap::basis_split(c.QR, c.QR_lo, c.QRt, c.QRt_lo, nc, c.count, s));
-    c.basis_dirty = false;
-  }
-  if (c.tc && !(c.left && c.right)) {
-    // the step's product [X | M_hat] Q for this matrix alone (bit-identical), written in the
-    // original orientation
-    const int rr = c.tr ? nc : m, cc = c.tr ? m : nc;
-    const int64_t qq = (int64_t)cc * cc;
-    const float* Qt = (c.tr ? c.QLt : c.QRt) + slot * qq;
-    const float* Qt_lo = (c.tr ? c.QLt_lo : c.QRt_lo) + slot * qq;
-    SOAP_CUDA(h, soap::gemm_tc_nt(rr, cc, cc, 1, opnd(x, c.Mhat_lo + slot * mn, cc, mn, 1), opnd(Qt, Qt_lo, cc, qq, 1),
-                                  epi(h, h->Gp, c.tr ? rr : cc, mn, nullptr, c.tr ? 1 : 0, 1.f, 0.f), s));
-    SOAP_CUDA(h, cudaMemcpyAsync(dst, h->Gp, bytes, cudaMemcpyDefault, s));
-    return SOAP_OK;
-  }
+  // m = Q_L^T M_hat Q_R, computed into the workspace with the operands and products of the step
+  const float* x = v.Mhat;
   if (c.tc) {
+    if (c.left) SOAP_CUDA(h, soap::basis_split(v.QL, v.QL_lo, v.QLt, v.QLt_lo, m, 1, s));
+    if (c.right) SOAP_CUDA(h, soap::basis_split(v.QR, v.QR_lo, v.QRt, v.QRt_lo, nc, 1, s));
+    float* x_lo = v.Mc_lo;
+    SOAP_CUDA(h, soap::split_tf32(x, nullptr, x_lo, mn, s));
+    if (!(c.left && c.right)) {
+      // the step's product [X | M_hat] Q for this matrix alone (bit-identical), written in the
+      // original orientation
+      const int rr = c.tr ? nc : m, cc = c.tr ? m : nc;
+      const int64_t qq = (int64_t)cc * cc;
+      SOAP_CUDA(h, soap::gemm_tc_nt(rr, cc, cc, 1, opnd(x, x_lo, cc, mn, 1),
+                                    opnd(c.tr ? v.QLt : v.QRt, c.tr ? v.QLt_lo : v.QRt_lo, cc, qq, 1),
+                                    epi(h, h->Gp, c.tr ? rr : cc, mn, nullptr, c.tr ? 1 : 0, 1.f, 0.f), s));
+      SOAP_CUDA(h, cudaMemcpyAsync(dst, h->Gp, bytes, cudaMemcpyDefault, s));
+      return SOAP_OK;
+    }
     // the same tensor-core products, on the same operands, as the step's rotation of M_hat:
     // bit-identical to the m the last step used
     const int64_t mm = (int64_t)m * m, nn = (int64_t)nc * nc;
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, nc, nc, 1, opnd(x, c.Mhat_lo + slot * mn, nc, mn, 1),
-                                  opnd(c.QRt + slot * nn, c.QRt_lo + slot * nn, nc, nn, 1),
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, nc, nc, 1, opnd(x, x_lo, nc, mn, 1), opnd(v.QRt, v.QRt_lo, nc, nn, 1),
                                   epi(h, h->X1, m, mn, h->X2, 1, 1.f, 0.f), s));
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, nc, m, 1, opnd(c.QLt + slot * mm, c.QLt_lo + slot * mm, m, mm, 1),
-                                  opnd(h->X1, h->X2, m, mn, 1), epi(h, h->Gp, nc, mn, nullptr, 0, 1.f, 0.f), s));
+    SOAP_CUDA(h, soap::gemm_tc_nt(m, nc, m, 1, opnd(v.QLt, v.QLt_lo, m, mm, 1), opnd(h->X1, h->X2, m, mn, 1),
+                                  epi(h, h->Gp, nc, mn, nullptr, 0, 1.f, 0.f), s));
     SOAP_CUDA(h, cudaMemcpyAsync(dst, h->Gp, bytes, cudaMemcpyDefault, s));
     return SOAP_OK;
   }
   using soap::strided;
   using soap::strided_mut;
   if (c.left) {
-    SOAP_CUDA(h, soap::gemm(true, false, m, nc, m, 1.f, strided(c.QL + (int64_t)slot * m * m, m, 0), strided(x, nc, 0),
-                            0.f, strided_mut(h->X1, nc, 0), 1, s));
+    SOAP_CUDA(h, soap::gemm(true, false, m, nc, m, 1.f, strided(v.QL, m, 0), strided(x, nc, 0), 0.f,
+                            strided_mut(h->X1, nc, 0), 1, s));
     x = h->X1;
   }
   if (c.right) {
-    SOAP_CUDA(h, soap::gemm(false, false, m, nc, nc, 1.f, strided(x, nc, 0), strided(c.QR + (int64_t)slot * nc * nc, nc, 0),
-                            0.f, strided_mut(h->Gp, nc, 0), 1, s));
+    SOAP_CUDA(h, soap::gemm(false, false, m, nc, nc, 1.f, strided(x, nc, 0), strided(v.QR, nc, 0), 0.f,
+                            strided_mut(h->Gp, nc, 0), 1, s));
     x = h->Gp;
   }
   SOAP_CUDA(h, cudaMemcpyAsync(dst, x, bytes, cudaMemcpyDefault, s));
   return SOAP_OK;
 }
 
-soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const void* src, soap_stream_t stream_) {
-  if (!h) return SOAP_ERR_INVALID_ARG;
+soap_status_t state_set_impl(soap_handle h, int32_t idx, int32_t which, const void* src, soap_stream_t stream_) {
   const size_t bytes = soap_state_bytes(h, idx, which);
   if (bytes == 0 || !src) return fail(h, SOAP_ERR_INVALID_ARG, "soap_state_set: no such state piece");
   if (which == SOAP_STATE_LAMBDA_L || which == SOAP_STATE_LAMBDA_R)
     return fail(h, SOAP_ERR_INVALID_ARG, "soap_state_set: the KL eigenvalue estimates are read-only");
   DeviceGuard g(h->device);
   cudaStream_t s = (cudaStream_t)stream_;
-  const auto [ci, slot] = h->loc[idx];
-  ClassState& c = h->classes[ci];
+  const ClassState& c = h->classes[h->loc[idx].first];
+  const View v = single_view(h, idx);
   const int m = (int)c.rows, nc = (int)c.cols;
-  const int64_t mn = (int64_t)m * nc;
-  float* dstm = c.Mhat + slot * mn;
+  if (which == SOAP_STATE_L || which == SOAP_STATE_R) {
+    const bool left = which == SOAP_STATE_L;
+    if (!c.tc) {
+      SOAP_CUDA(h, cudaMemcpyAsync(left ? v.L : v.R, src, bytes, cudaMemcpyDefault, s));
+      return SOAP_OK;
+    }
+    // the lower triangle is kept (the factor is symmetric)
+    float* F = left ? v.Lf : v.Rf;
+    SOAP_CUDA(h, cudaMemcpyAsync(F, src, bytes, cudaMemcpyDefault, s));
+    SOAP_CUDA(h, soap::pack_sym(F, left ? v.L : v.R, left ? m : nc, 1, s));
+    return SOAP_OK;
+  }
   if (which != SOAP_STATE_M) {
     if (c.tr && (which == SOAP_STATE_V || which == SOAP_STATE_MHAT)) {
       // stored transposed (n x m)
       SOAP_CUDA(h, cudaMemcpyAsync(h->X1, src, bytes, cudaMemcpyDefault, s));
-      SOAP_CUDA(h, soap::transpose(h->X1, (float*)state_ptr(h, idx, which), m, nc, 1, s));
+      SOAP_CUDA(h, soap::transpose(h->X1, (float*)state_ptr(v, which), m, nc, 1, s));
     } else {
-      SOAP_CUDA(h, cudaMemcpyAsync(state_ptr(h, idx, which), src, bytes, cudaMemcpyDefault, s));
+      SOAP_CUDA(h, cudaMemcpyAsync(state_ptr(v, which), src, bytes, cudaMemcpyDefault, s));
     }
-    if (which == SOAP_STATE_QL || which == SOAP_STATE_QR) c.basis_dirty = true;
-    if (which == SOAP_STATE_MHAT && c.tc)
-      SOAP_CUDA(h, soap::split_tf32(dstm, nullptr, c.Mhat_lo + slot * mn, mn, s));
-    // the factors' lo parts: the KL form reads them (lambda = diag(Q^T F Q)) before S1 rewrites them
-    if (which == SOAP_STATE_L && c.tc)
-      SOAP_CUDA(h, soap::split_tf32(c.L + slot * (int64_t)m * m, nullptr, c.L_lo + slot * (int64_t)m * m,
-                                    (int64_t)m * m, s));
-    if (which == SOAP_STATE_R && c.tc)
-      SOAP_CUDA(h, soap::split_tf32(c.R + slot * (int64_t)nc * nc, nullptr, c.R_lo + slot * (int64_t)nc * nc,
-                                    (int64_t)nc * nc, s));
     return SOAP_OK;
   }
   // M_hat = Q_L m Q_R^T
   using soap::strided;
   using soap::strided_mut;
+  float* dstm = v.Mhat;
   SOAP_CUDA(h, cudaMemcpyAsync(h->Gp, src, bytes, cudaMemcpyDefault, s));
   const float* x = h->Gp;
   if (c.left) {
     float* out = (c.right || c.tr) ? h->X1 : dstm;
-    SOAP_CUDA(h, soap::gemm(false, false, m, nc, m, 1.f, strided(c.QL + (int64_t)slot * m * m, m, 0), strided(x, nc, 0),
-                            0.f, strided_mut(out, nc, 0), 1, s));
+    SOAP_CUDA(h, soap::gemm(false, false, m, nc, m, 1.f, strided(v.QL, m, 0), strided(x, nc, 0), 0.f,
+                            strided_mut(out, nc, 0), 1, s));
     x = out;
   }
   if (c.right) {
-    SOAP_CUDA(h, soap::gemm(false, true, m, nc, nc, 1.f, strided(x, nc, 0), strided(c.QR + (int64_t)slot * nc * nc, nc, 0),
-                            0.f, strided_mut(dstm, nc, 0), 1, s));
+    SOAP_CUDA(h, soap::gemm(false, true, m, nc, nc, 1.f, strided(x, nc, 0), strided(v.QR, nc, 0), 0.f,
+                            strided_mut(dstm, nc, 0), 1, s));
   } else if (c.tr) {
     SOAP_CUDA(h, soap::transpose(x, dstm, m, nc, 1, s));
   } else if (!c.left) {
     SOAP_CUDA(h, cudaMemcpyAsync(dstm, x, bytes, cudaMemcpyDeviceToDevice, s));
   }
-  if (c.tc) SOAP_CUDA(h, soap::split_tf32(dstm, nullptr, c.Mhat_lo + slot * mn, mn, s));
   return SOAP_OK;
+}
+
+// State reads and writes use the step's workspace: each is ordered after the last enqueued
+// step (or state access), and the next step after it, whatever streams they come on.
+soap_status_t ordered_state_op(soap_handle h, cudaStream_t s, soap_status_t (*op)(soap_handle, int32_t, int32_t, void*,
+                                                                                 soap_stream_t),
+                               int32_t idx, int32_t which, void* buf) {
+  DeviceGuard g(h->device);
+  if (h->step_recorded) SOAP_CUDA(h, cudaStreamWaitEvent(s, h->step_done, 0));
+  soap_status_t st = op(h, idx, which, buf, (soap_stream_t)s);
+  cudaError_t e = cudaEventRecord(h->step_done, s);
+  if (e == cudaSuccess) h->step_recorded = true;
+  if (st == SOAP_OK && e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord(step_done)");
+  return st;
+}
+
+soap_status_t state_set_void(soap_handle h, int32_t idx, int32_t which, void* src, soap_stream_t s) {
+  return state_set_impl(h, idx, which, src, s);
+}
+
+}  // namespace
+
+extern "C" {
+
+soap_status_t soap_state_get(soap_handle h, int32_t idx, int32_t which, void* dst, soap_stream_t stream) {
+  if (!h) return SOAP_ERR_INVALID_ARG;
+  return ordered_state_op(h, (cudaStream_t)stream, state_get_impl, idx, which, dst);
+}
+
+soap_status_t soap_state_set(soap_handle h, int32_t idx, int32_t which, const void* src, soap_stream_t stream) {
+  if (!h) return SOAP_ERR_INVALID_ARG;
+  return ordered_state_op(h, (cudaStream_t)stream, state_set_void, idx, which, const_cast<void*>(src));
 }
 
 int64_t soap_get_step(soap_handle h) { return h ? h->t : -1; }
@@ -1130,19 +1385,21 @@ size_t soap_qr_workspace_bytes(int32_t n, int32_t batch) {
 }
 
 soap_status_t soap_qr(int32_t n, int32_t batch, const float* P, float* Q, uint8_t* skip, float tol, void* workspace,
-                      size_t workspace_bytes, soap_stream_t stream) {
+                      size_t workspace_bytes, int32_t* status, soap_stream_t stream) {
   if (n <= 0 || n > 8192 || (n & 3) || batch <= 0 || batch > 65535 || !P || !Q || !skip || !workspace ||
       !(tol >= 0.f))
     return SOAP_ERR_INVALID_ARG;
-  if (!aligned16(P) || !aligned16(Q) || (reinterpret_cast<uintptr_t>(workspace) & 255))
+  if (!aligned16(P) || !aligned16(Q) || (reinterpret_cast<uintptr_t>(workspace) & 255) ||
+      (reinterpret_cast<uintptr_t>(status) & 3))
     return SOAP_ERR_INVALID_ARG;
   if (workspace_bytes < soap_qr_workspace_bytes(n, batch)) return SOAP_ERR_INVALID_ARG;
   cudaStream_t s = (cudaStream_t)stream;
-  // the status word lives in the last 256 bytes of the caller's workspace
+  // the kernels OR their status bits into the caller's word, or else into the last 256 bytes of
+  // the workspace
   const size_t qb = soap::qr_workspace_bytes(n, batch);
-  int* status = reinterpret_cast<int*>(static_cast<char*>(workspace) + qb);
-  if (cudaMemsetAsync(status, 0, sizeof(int), s) != cudaSuccess) return SOAP_ERR_CUDA;
-  cudaError_t e = soap::qr_q(n, batch, P, Q, skip, tol, workspace, qb, status, s);
+  int* word = status ? reinterpret_cast<int*>(status) : reinterpret_cast<int*>(static_cast<char*>(workspace) + qb);
+  if (cudaMemsetAsync(word, 0, sizeof(int), s) != cudaSuccess) return SOAP_ERR_CUDA;
+  cudaError_t e = soap::qr_q(n, batch, P, Q, skip, tol, workspace, qb, word, s);
   return e == cudaSuccess ? SOAP_OK : SOAP_ERR_CUDA;
 }
 

@@ -149,11 +149,26 @@ cudaError_t adam_in_basis(float* Gp, const float* Mp, float* V, int rows, int co
                           const uint8_t* skipL, const uint8_t* skipR, float* N_lo, int* status,
                           cudaStream_t stream);
 // Tensor-core operand preparation: G and G^T with their lo parts, and the momentum EMA
-// M_hat <- b1 M_hat + (1-b1) G with its lo part, M_hat stored in G's orientation or (if
-// mhat_transposed) as M_hat^T.
+// M_hat <- b1 M_hat + (1-b1) G in place, with a copy of the new M_hat and its lo part
+// (Mcopy, Mcopy_lo); M_hat is stored in G's orientation or (if mhat_transposed) as M_hat^T,
+// and so is its copy.
 cudaError_t momentum_split(const float* const* grads, float* Gn, float* Gn_lo, float* Gt, float* Gt_lo,
-                           float* Mhat, float* Mhat_lo, int rows, int cols, int batch, float beta1,
+                           float* Mhat, float* Mcopy, float* Mcopy_lo, int rows, int cols, int batch, float beta1,
                            bool mhat_transposed, int* status, cudaStream_t stream);
+// Packed symmetric storage: the lower-triangular 32 x 32 tiles of an n x n matrix, tile (I, J)
+// (I >= J) at tile index I (I + 1) / 2 + J, each row-major; packed_floats(n) per matrix.
+int64_t packed_floats(int n);
+// F_b (full, n x n) and, if F_lo is given, its lo part from the packed tiles P_b.
+cudaError_t unpack_sym(const float* P, float* F, float* F_lo, int n, int batch, cudaStream_t stream);
+// P_b from the lower triangle of F_b.
+cudaError_t pack_sym(const float* F, float* P, int n, int batch, cudaStream_t stream);
+// Device pointer table written from a host array through kernel parameters (no host buffer
+// has to outlive the call, and nothing waits on the host).
+constexpr int kPtrChunk = 480;
+struct PtrChunk {
+  void* p[kPtrChunk];
+};
+cudaError_t put_ptrs(void** dst, void* const* src, int64_t n, cudaStream_t stream);
 // dst_b = src_b^T for `batch` contiguous rows x cols matrices.
 cudaError_t transpose(const float* src, float* dst, int rows, int cols, int batch, cudaStream_t stream);
 // From Q^T: a copy of it with its lo part, and Q with its lo part (any output may be null;

@@ -17,13 +17,14 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_lib", platform.machine(), "libsoap.so")
 
 SOAP_OK = 0
+STATUS_NONFINITE, STATUS_QR_BREAKDOWN, STATUS_TIMEOUT = 1, 2, 4  # device status bits (SOAP_STATUS_*)
 STATUS_NAMES = {0: "SOAP_OK", 1: "SOAP_ERR_INVALID_ARG", 2: "SOAP_ERR_CUDA", 3: "SOAP_ERR_OOM",
                 4: "SOAP_ERR_NONFINITE", 5: "SOAP_ERR_QR_BREAKDOWN", 6: "SOAP_ERR_TIMEOUT"}
 (STATE_M, STATE_V, STATE_L, STATE_QL, STATE_R, STATE_QR, STATE_MHAT, STATE_SKIP_L, STATE_SKIP_R,
  STATE_LAMBDA_L, STATE_LAMBDA_R) = range(11)
 
 # every symbol include/soap.h declares
-EXPORTS = ("soap_default_hparams", "soap_create", "soap_step", "soap_set_lr", "soap_state_bytes",
+EXPORTS = ("soap_default_hparams", "soap_create", "soap_create_ex", "soap_plan_info", "soap_step", "soap_set_lr", "soap_state_bytes",
            "soap_state_get", "soap_state_set", "soap_get_step", "soap_set_step", "soap_status",
            "soap_clear_status", "soap_last_error", "soap_destroy", "soap_qr_workspace_bytes",
            "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_profile_records",
@@ -85,6 +86,9 @@ def load_library(path: str = LIB_PATH):
     sig = {
         "soap_default_hparams": (None, [ctypes.POINTER(soap_hparams)]),
         "soap_create": (I32, [ctypes.POINTER(soap_shape), I32, ctypes.POINTER(soap_hparams), I32, ctypes.POINTER(P)]),
+        "soap_create_ex": (I32, [ctypes.POINTER(soap_shape), I32, ctypes.POINTER(soap_hparams), I32, SZ,
+                                 ctypes.POINTER(P)]),
+        "soap_plan_info": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(SZ), ctypes.POINTER(SZ)]),
         "soap_step": (I32, [P, P, P, P]),
         "soap_set_lr": (I32, [P, F, F]),
         "soap_state_bytes": (SZ, [P, I32, I32]),
@@ -97,7 +101,7 @@ def load_library(path: str = LIB_PATH):
         "soap_last_error": (ctypes.c_char_p, [P]),
         "soap_destroy": (None, [P]),
         "soap_qr_workspace_bytes": (SZ, [I32, I32]),
-        "soap_qr": (I32, [I32, I32, P, P, P, F, P, SZ, P]),
+        "soap_qr": (I32, [I32, I32, P, P, P, F, P, SZ, P, P]),
         "soap_profile_begin": (I32, [P, I64]),
         "soap_profile_end": (I32, [P, P, ctypes.POINTER(soap_kernel_stats), ctypes.POINTER(I32)]),
         "soap_profile_records": (I32, [P, ctypes.POINTER(soap_launch_record), I64, ctypes.POINTER(I64)]),
@@ -105,7 +109,7 @@ def load_library(path: str = LIB_PATH):
         "soap_gemm_tf32x4": (I32, [I32, I32, I32, I32, P, P, I64, I64, P, P, I64, I64, I32, F, F, P, I64, I64,
                                    I32, P, P, P]),
         "soap_split_tf32": (I32, [P, P, P, I64, P]),
-        "soap_qr_static": (I32, [I32, I32, P, P, P, F, P]),
+        "soap_qr_static": (I32, [I32, I32, P, P, P, F, P, P]),
         "soap_layerwise_assign": (I32, [ctypes.POINTER(soap_shape), I32, I32, I32, ctypes.POINTER(I32),
                                         ctypes.POINTER(ctypes.c_double)]),
         "muon_default_hparams": (None, [ctypes.POINTER(muon_hparams)]),
@@ -128,9 +132,15 @@ def load_library(path: str = LIB_PATH):
     return lib
 
 
-def _stream(stream=None):
+def _stream(stream=None, dev=None):
+    """The cudaStream_t of `stream`, or of the current stream of device `dev` (else of the current
+    device); a stream of another device than `dev` is refused before it reaches the library."""
+    if dev is not None:
+        dev = torch.device("cuda", dev) if isinstance(dev, int) else torch.device(dev)
     if stream is None:
-        stream = torch.cuda.current_stream()
+        stream = torch.cuda.current_stream(dev)
+    elif dev is not None and torch.device(stream.device).index != dev.index:
+        raise ValueError(f"stream of {stream.device} given for work on {dev}")
     return ctypes.c_void_p(stream.cuda_stream)
 
 
@@ -173,9 +183,13 @@ class Shape:
 
 
 class SoapOptimizer:
-    """One libsoap handle: soap_create / soap_step / soap_state_get / soap_state_set."""
+    """One libsoap handle: soap_create / soap_step / soap_state_get / soap_state_set.
 
-    def __init__(self, shapes, hparams: soap_hparams | None = None, device: int | None = None):
+    workspace_limit (bytes, 0 = automatic) bounds the step's workspace (soap_create_ex): a model
+    whose workspace does not fit is stepped in several waves of matrices."""
+
+    def __init__(self, shapes, hparams: soap_hparams | None = None, device: int | None = None,
+                 workspace_limit: int = 0):
         lib = load_library()
         self.shapes = [Shape(*s) if not isinstance(s, Shape) else s for s in shapes]
         arr = (soap_shape * len(self.shapes))(*[soap_shape(s.rows, s.cols, int(s.left), int(s.right))
@@ -183,7 +197,8 @@ class SoapOptimizer:
         self.hparams = hparams if hparams is not None else default_hparams()
         self.device = torch.cuda.current_device() if device is None else device
         h = ctypes.c_void_p()
-        _check(lib.soap_create(arr, len(self.shapes), ctypes.byref(self.hparams), self.device, ctypes.byref(h)))
+        _check(lib.soap_create_ex(arr, len(self.shapes), ctypes.byref(self.hparams), self.device,
+                                  int(workspace_limit), ctypes.byref(h)))
         self._h = h
         n = len(self.shapes)
         self._pp = (ctypes.c_void_p * n)()
@@ -210,7 +225,14 @@ class SoapOptimizer:
                 raise ValueError(f"matrix {i}: tensors must be contiguous")
             self._pp[i] = p.data_ptr()
             self._gp[i] = g.data_ptr()
-        _check(load_library().soap_step(self._handle(), self._pp, self._gp, _stream(stream)), self._h)
+        _check(load_library().soap_step(self._handle(), self._pp, self._gp, _stream(stream, self.device)), self._h)
+
+    def plan_info(self) -> dict:
+        """soap_plan_info: waves per step, workspace and state bytes."""
+        w, ws, st = ctypes.c_int32(0), ctypes.c_size_t(0), ctypes.c_size_t(0)
+        _check(load_library().soap_plan_info(self._handle(), ctypes.byref(w), ctypes.byref(ws), ctypes.byref(st)),
+               self._h)
+        return {"waves": w.value, "workspace_bytes": ws.value, "state_bytes": st.value}
 
     def set_lr(self, lr: float, weight_decay: float):
         _check(load_library().soap_set_lr(self._handle(), lr, weight_decay), self._h)
@@ -230,14 +252,14 @@ class SoapOptimizer:
         dtype = torch.uint8 if which in (STATE_SKIP_L, STATE_SKIP_R) else torch.float32
         out = torch.empty(shape, dtype=dtype, device=f"cuda:{self.device}")
         _check(load_library().soap_state_get(self._handle(), idx, which, ctypes.c_void_p(out.data_ptr()),
-                                             _stream(stream)), self._h)
+                                             _stream(stream, self.device)), self._h)
         return out
 
     def state_set(self, idx: int, which: int, src: torch.Tensor, stream=None):
         if src.numel() * src.element_size() != self.state_bytes(idx, which) or not src.is_contiguous():
             raise ValueError("state_set: wrong size or non-contiguous source")
         _check(load_library().soap_state_set(self._handle(), idx, which, ctypes.c_void_p(src.data_ptr()),
-                                             _stream(stream)), self._h)
+                                             _stream(stream, self.device)), self._h)
 
     @property
     def t(self) -> int:
@@ -249,10 +271,10 @@ class SoapOptimizer:
 
     def status(self, stream=None) -> int:
         """Synchronises the stream and returns the sticky device status code."""
-        return load_library().soap_status(self._handle(), _stream(stream))
+        return load_library().soap_status(self._handle(), _stream(stream, self.device))
 
     def clear_status(self, stream=None):
-        _check(load_library().soap_clear_status(self._handle(), _stream(stream)), self._h)
+        _check(load_library().soap_clear_status(self._handle(), _stream(stream, self.device)), self._h)
 
     def profile_begin(self, max_launches: int = 1 << 16):
         """Time every kernel launch of the following calls with CUDA events."""
@@ -262,7 +284,7 @@ class SoapOptimizer:
         """Synchronise and return {family: {launches, ms, flops, bytes}} plus an overflow flag."""
         out = (soap_kernel_stats * len(KERNEL_FAMILIES))()
         ov = ctypes.c_int32(0)
-        _check(load_library().soap_profile_end(self._handle(), _stream(stream), out, ctypes.byref(ov)), self._h)
+        _check(load_library().soap_profile_end(self._handle(), _stream(stream, self.device), out, ctypes.byref(ov)), self._h)
         res = {KERNEL_FAMILIES[o.family]: dict(launches=o.launches, ms=o.ms, flops=o.flops, bytes=o.bytes)
                for o in out}
         res["overflow"] = bool(ov.value)
@@ -309,8 +331,9 @@ def soap_state_set(opt: SoapOptimizer, idx, which, src, stream=None):
     opt.state_set(idx, which, src, stream)
 
 
-def soap_qr(P: torch.Tensor, tol: float = 0.0, stream=None):
-    """Batched QR refresh on device: P [batch, n, n] fp32 -> (Q, skip[batch, n] uint8)."""
+def soap_qr(P: torch.Tensor, tol: float = 0.0, stream=None, return_status=False):
+    """Batched QR refresh on device: P [batch, n, n] fp32 -> (Q, skip[batch, n] uint8), and with
+    return_status the call's device status word (an int32 tensor: 0, or SOAP_STATUS_* bits)."""
     lib = load_library()
     if P.dim() == 2:
         P = P.unsqueeze(0)
@@ -322,19 +345,21 @@ def soap_qr(P: torch.Tensor, tol: float = 0.0, stream=None):
     skip = torch.empty(batch, n, dtype=torch.uint8, device=P.device)
     ws_bytes = lib.soap_qr_workspace_bytes(n, batch)
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device=P.device)
+    status = torch.empty(1, dtype=torch.int32, device=P.device)
     with torch.cuda.device(P.device):
         _check(lib.soap_qr(n, batch, ctypes.c_void_p(P.data_ptr()), ctypes.c_void_p(Q.data_ptr()),
                            ctypes.c_void_p(skip.data_ptr()), float(tol), ctypes.c_void_p(ws.data_ptr()), ws_bytes,
-                           _stream(stream)))
-    return Q, skip
+                           ctypes.c_void_p(status.data_ptr()), _stream(stream, P.device)))
+    return (Q, skip, status) if return_status else (Q, skip)
 
 
-def soap_qr_static(P: torch.Tensor, tol: float = 0.0, stream=None):
+def soap_qr_static(P: torch.Tensor, tol: float = 0.0, stream=None, return_status=False):
     """soap_qr without a caller-supplied workspace, for code that cannot allocate device memory
     when it needs the QR: libsoap.so uses a fixed 32 MiB array of its own (enough for one
     1024 x 1024 matrix). The output tensors here are allocated by torch for convenience; a
     caller without an allocator passes its own buffers to the C entry point. Raises
-    SoapError(SOAP_ERR_INVALID_ARG) for work larger than the array."""
+    SoapError(SOAP_ERR_INVALID_ARG) for work larger than the array. With return_status, also
+    returns the call's device status word (an int32 tensor: 0, or SOAP_STATUS_* bits)."""
     lib = load_library()
     if P.dim() == 2:
         P = P.unsqueeze(0)
@@ -344,14 +369,16 @@ def soap_qr_static(P: torch.Tensor, tol: float = 0.0, stream=None):
     batch, n = P.shape[0], P.shape[1]
     Q = torch.empty_like(P)
     skip = torch.empty(batch, n, dtype=torch.uint8, device=P.device)
+    status = torch.empty(1, dtype=torch.int32, device=P.device)
     with torch.cuda.device(P.device):
         code = lib.soap_qr_static(n, batch, ctypes.c_void_p(P.data_ptr()), ctypes.c_void_p(Q.data_ptr()),
-                                  ctypes.c_void_p(skip.data_ptr()), float(tol), _stream(stream))
+                                  ctypes.c_void_p(skip.data_ptr()), float(tol), ctypes.c_void_p(status.data_ptr()),
+                                  _stream(stream, P.device))
     if code != SOAP_OK:
         raise SoapError(code, f"soap_qr_static(n={n}, batch={batch}): needs "
                               f"{lib.soap_qr_workspace_bytes(n, batch)} bytes of workspace; the fixed array "
                               "holds 32 MiB" if code == 1 else "soap_qr_static failed")
-    return Q, skip
+    return (Q, skip, status) if return_status else (Q, skip)
 
 
 def soap_gemm(A: torch.Tensor, B: torch.Tensor, trans_a=False, trans_b=False, alpha=1.0, beta=0.0,
@@ -376,7 +403,7 @@ def soap_gemm(A: torch.Tensor, B: torch.Tensor, trans_a=False, trans_b=False, al
         _check(lib.soap_gemm(int(trans_a), int(trans_b), M, N, K, float(alpha),
                              ctypes.c_void_p(A3.data_ptr()), A3.shape[2], A3.shape[1] * A3.shape[2],
                              ctypes.c_void_p(B3.data_ptr()), B3.shape[2], B3.shape[1] * B3.shape[2], float(beta),
-                             ctypes.c_void_p(C3.data_ptr()), N, M * N, batch, _stream(stream)))
+                             ctypes.c_void_p(C3.data_ptr()), N, M * N, batch, _stream(stream, dev)))
     return C3[0] if squeeze else C3
 
 
@@ -387,7 +414,7 @@ def soap_split_tf32(x: torch.Tensor, stream=None):
     hi, lo = torch.empty_like(x), torch.empty_like(x)
     with torch.cuda.device(dev):
         _check(load_library().soap_split_tf32(ctypes.c_void_p(x.data_ptr()), ctypes.c_void_p(hi.data_ptr()),
-                                              ctypes.c_void_p(lo.data_ptr()), x.numel(), _stream(stream)))
+                                              ctypes.c_void_p(lo.data_ptr()), x.numel(), _stream(stream, dev)))
     return hi, lo
 
 
@@ -425,7 +452,7 @@ def soap_gemm_tf32x4(A, B, alpha=1.0, beta=0.0, C=None, transpose_c=False, A_spl
                                     shape[1] * shape[2], int(transpose_c),
                                     ctypes.c_void_p(lo.data_ptr()) if with_lo else None,
                                     ctypes.c_void_p(status.data_ptr()) if status is not None else None,
-                                    _stream(stream)))
+                                    _stream(stream, dev)))
     out = C3[0] if A.dim() == 2 and (C is None or C.dim() == 2) else C3
     if with_lo:
         return out, (lo[0] if out.dim() == 2 else lo)
@@ -487,7 +514,7 @@ class MuonOptimizer:
                 raise ValueError(f"matrix {i}: expected a contiguous {s} tensor")
             self._pp[i] = p.data_ptr()
             self._gp[i] = g.data_ptr()
-        self._check(load_library().muon_step(self._handle(), self._pp, self._gp, _stream(stream)))
+        self._check(load_library().muon_step(self._handle(), self._pp, self._gp, _stream(stream, self.device)))
 
     def set_lr(self, lr: float, weight_decay: float):
         self._check(load_library().muon_set_lr(self._handle(), lr, weight_decay))
@@ -496,17 +523,17 @@ class MuonOptimizer:
         """The momentum M of matrix idx as a new device tensor."""
         out = torch.empty(self.shapes[idx], dtype=torch.float32, device=f"cuda:{self.device}")
         self._check(load_library().muon_state_get(self._handle(), idx, ctypes.c_void_p(out.data_ptr()),
-                                                  _stream(stream)))
+                                                  _stream(stream, self.device)))
         return out
 
     def state_set(self, idx: int, src: torch.Tensor, stream=None):
         if tuple(src.shape) != self.shapes[idx] or src.dtype != torch.float32 or not src.is_contiguous():
             raise ValueError("state_set: wrong shape, dtype or layout")
         self._check(load_library().muon_state_set(self._handle(), idx, ctypes.c_void_p(src.data_ptr()),
-                                                  _stream(stream)))
+                                                  _stream(stream, self.device)))
 
     def status(self, stream=None) -> int:
-        return load_library().muon_status(self._handle(), _stream(stream))
+        return load_library().muon_status(self._handle(), _stream(stream, self.device))
 
     def last_error(self) -> str:
         return load_library().muon_last_error(self._h).decode() if self._h else "handle destroyed"
@@ -519,7 +546,7 @@ class MuonOptimizer:
         """Synchronise and return {family: {launches, ms, flops, bytes}} plus an overflow flag."""
         out = (soap_kernel_stats * len(KERNEL_FAMILIES))()
         ov = ctypes.c_int32(0)
-        self._check(load_library().muon_profile_end(self._handle(), _stream(stream), out, ctypes.byref(ov)))
+        self._check(load_library().muon_profile_end(self._handle(), _stream(stream, self.device), out, ctypes.byref(ov)))
         res = {KERNEL_FAMILIES[o.family]: dict(launches=o.launches, ms=o.ms, flops=o.flops, bytes=o.bytes)
                for o in out}
         res["overflow"] = bool(ov.value)

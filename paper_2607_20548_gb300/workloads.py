@@ -10,15 +10,17 @@ rank-structured plus noise:
 
     G_t = c * (A + 0.3 * N_t),   A = U diag(s) V^T,  s_i = i^-1.5 / ||(i^-1.5)||_2,
 
-with U (rows x k), V (cols x k) random orthonormal (QR of a Gaussian), k = min(rows,
-cols, 1024) (the spectrum beyond i = 1024 lies far below the noise: s_1024 / s_1 = 3e-5, so
-the cap only keeps the host QR of the 28672-wide matrices cheap), N_t i.i.d. N(0, 1/cols) drawn afresh every step, W_0 ~ N(0, 0.02^2), and c = 1
-except for MoE experts, whose c is drawn once per expert, log-uniform in [1e-2, 1],
-to mimic uneven token routing.
+with U (rows x k), V (cols x k) random orthonormal (QR of a Gaussian), k = min(rows, cols),
+N_t i.i.d. N(0, 1/cols) drawn afresh every step, W_0 ~ N(0, 0.02^2), and c = 1 except for MoE
+experts, whose c is drawn once per expert, log-uniform in [1e-2, 1], to mimic uneven token
+routing.
 
-All tensors are float32. U, V (and so A) are drawn on the host; W_0 and the per-step
-noise are drawn with torch on the requested device; the oracle gets host copies of
-exactly the same values.
+All tensors are float32 and drawn on the stream's device (U and V by a QR of a Gaussian there);
+the oracle gets host copies of exactly the same values. A shape group of more than
+SHARED_BASES matrices (the 24-layer stack has thousands of experts of one shape) draws
+SHARED_BASES Haar-random bases per side and gives each matrix one of them with its columns
+permuted and their signs flipped at random (still exactly orthonormal, with the same
+power-law spectrum); such a group keeps no A and forms it chunk by chunk when drawing G.
 """
 from __future__ import annotations
 
@@ -95,6 +97,10 @@ def _seed(*parts: int) -> int:
     return h & 0x7FFFFFFFFFFFFFFF
 
 
+SHARED_BASES = 64
+_CHUNK_ELEMS = 1 << 27  # matrices per chunk: about this many elements (512 MB) at a time
+
+
 class GradientStream:
     """Draws W_0 and G_t for a list of matrices, grouped into same-shape batches.
 
@@ -110,40 +116,72 @@ class GradientStream:
         for j, s in enumerate(self.specs):
             order.setdefault((s.rows, s.cols), []).append(j)
         self.groups = [(self.specs[idx[0]], idx) for idx in order.values()]
-        self._A = []
+        self._A = []      # per group: A [B, rows, cols], or None if formed per chunk
+        self._bases = []  # per group (chunked only): U, V bases and each matrix's pick
         self._c = []
         for gi, (s, idx) in enumerate(self.groups):
-            # U, V and A are drawn on the host (the same values whatever the device), then moved
-            k = min(s.rows, s.cols, 1024)
-            g = torch.Generator().manual_seed(_seed(seed, gi, 1))
+            k = min(s.rows, s.cols)
             B = len(idx)
-            U = torch.linalg.qr(torch.randn(B, s.rows, k, generator=g))[0]
-            V = torch.linalg.qr(torch.randn(B, s.cols, k, generator=g))[0]
+            g = torch.Generator(device=self.device).manual_seed(_seed(seed, gi, 1))
+            nb = min(B, SHARED_BASES)
+            U = torch.linalg.qr(torch.randn(nb, s.rows, k, generator=g, device=self.device))[0]
+            V = torch.linalg.qr(torch.randn(nb, s.cols, k, generator=g, device=self.device))[0]
             i = torch.arange(1, k + 1, dtype=torch.float64)
             sv = i.pow(-1.5)
-            sv = (sv / sv.norm()).to(torch.float32)
-            A = torch.matmul(U * sv, V.transpose(1, 2))
-            self._A.append(A.contiguous().to(self.device))
+            sv = (sv / sv.norm()).to(torch.float32).to(self.device)
             self._c.append(torch.tensor([self.scales[j] for j in idx], dtype=torch.float32,
                                         device=self.device).view(B, 1, 1))
+            if nb == B:
+                self._A.append(torch.matmul(U * sv, V.transpose(1, 2)).contiguous())
+                self._bases.append(None)
+                continue
+            # each matrix: one of the nb bases per side, columns permuted, signs flipped
+            pick = torch.randint(0, nb, (B,), generator=g, device=self.device)
+            perm_u = torch.argsort(torch.rand(B, k, generator=g, device=self.device), dim=1)
+            perm_v = torch.argsort(torch.rand(B, k, generator=g, device=self.device), dim=1)
+            sgn_u = torch.randint(0, 2, (B, k), generator=g, device=self.device).float().mul_(2).sub_(1)
+            sgn_v = torch.randint(0, 2, (B, k), generator=g, device=self.device).float().mul_(2).sub_(1)
+            self._A.append(None)
+            self._bases.append((U, V, sv, pick, perm_u, perm_v, sgn_u, sgn_v))
+
+    def _A_chunk(self, gi, b0, b1):
+        A = self._A[gi]
+        if A is not None:
+            return A[b0:b1]
+        U, V, sv, pick, pu, pv, su, sv_sign = self._bases[gi]
+        Uc = torch.gather(U[pick[b0:b1]], 2, pu[b0:b1, None, :].expand(-1, U.shape[1], -1)) * su[b0:b1, None, :]
+        Vc = torch.gather(V[pick[b0:b1]], 2, pv[b0:b1, None, :].expand(-1, V.shape[1], -1)) * sv_sign[b0:b1, None, :]
+        return torch.matmul(Uc * sv, Vc.transpose(1, 2))
 
     def weights(self):
         """W_0 ~ N(0, 0.02^2), one [batch, rows, cols] tensor per group."""
         out = []
         for gi, (s, idx) in enumerate(self.groups):
             g = torch.Generator(device=self.device).manual_seed(_seed(self.seed, gi, 2))
-            out.append(0.02 * torch.randn(len(idx), s.rows, s.cols, generator=g, device=self.device))
+            out.append(torch.randn(len(idx), s.rows, s.cols, generator=g, device=self.device).mul_(0.02))
         return out
 
-    def grads(self, step: int):
-        """G_t for step ``step`` (1-based), one [batch, rows, cols] tensor per group."""
-        out = []
+    def grads(self, step: int, out=None):
+        """G_t for step ``step`` (1-based), one [batch, rows, cols] tensor per group (written into
+        ``out``, a list of such tensors, if given)."""
+        res = []
         for gi, (s, idx) in enumerate(self.groups):
-            g = torch.Generator(device=self.device).manual_seed(_seed(self.seed, gi, 3, step))
-            N = torch.randn(len(idx), s.rows, s.cols, generator=g, device=self.device)
-            N.mul_(0.3 / math.sqrt(s.cols)).add_(self._A[gi]).mul_(self._c[gi])
-            out.append(N)
-        return out
+            B = len(idx)
+            dst = out[gi] if out is not None else torch.empty(B, s.rows, s.cols, device=self.device)
+            if self._A[gi] is not None and B * s.rows * s.cols <= _CHUNK_ELEMS:
+                g = torch.Generator(device=self.device).manual_seed(_seed(self.seed, gi, 3, step))
+                torch.randn(B, s.rows, s.cols, generator=g, device=self.device, out=dst)
+                dst.mul_(0.3 / math.sqrt(s.cols)).add_(self._A[gi]).mul_(self._c[gi])
+            else:
+                per = max(1, _CHUNK_ELEMS // (s.rows * s.cols))
+                for ci, b0 in enumerate(range(0, B, per)):
+                    b1 = min(B, b0 + per)
+                    g = torch.Generator(device=self.device).manual_seed(_seed(self.seed, gi, 3, step, ci))
+                    d = dst[b0:b1]
+                    torch.randn(b1 - b0, s.rows, s.cols, generator=g, device=self.device, out=d)
+                    d.mul_(0.3 / math.sqrt(s.cols)).add_(self._A_chunk(gi, b0, b1)).mul_(self._c[gi][b0:b1])
+            res.append(dst)
+        return res
 
 
 def make_stream(name: str, seed: int = 0, device="cpu", specs=None):

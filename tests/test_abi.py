@@ -64,7 +64,7 @@ def test_host_side_validation_needs_no_gpu():
     assert lib.soap_create(ok_shape, 1, ctypes.byref(st_hp), 0, ctypes.byref(h)) == 1
     assert lib.soap_gemm(0, 0, -1, 1, 1, 1.0, None, 1, 0, None, 1, 0, 0.0, None, 1, 0, 1, None) == 1
     assert lib.soap_gemm(0, 0, 0, 1, 1, 1.0, None, 1, 0, None, 1, 0, 0.0, None, 1, 0, 1, None) == 0
-    assert lib.soap_qr(0, 1, None, None, None, 0.0, None, 0, None) == 1
+    assert lib.soap_qr(0, 1, None, None, None, 0.0, None, 0, None, None) == 1
     assert lib.soap_qr_workspace_bytes(64, 2) > 2 * 64 * 64 * 4
     assert lib.soap_state_bytes(None, 0, 0) == 0
     assert lib.soap_get_step(None) == -1
@@ -181,3 +181,21 @@ def test_plain_c_consumer_builds_and_runs():
         assert r.returncode == 0, r.stderr
         r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
         assert r.returncode == 0 and "c abi ok" in r.stdout, (r.returncode, r.stdout, r.stderr)
+
+
+def test_stream_of_another_device_is_refused():
+    """A caller's stream must belong to the device the work runs on: one of another device is
+    refused on the host with a clear error instead of reaching the library."""
+    import pytest
+    import torch
+
+    class _FakeStream:
+        def __init__(self, index):
+            self.device = torch.device("cuda", index)
+            self.cuda_stream = 0
+
+    assert S._stream(_FakeStream(1), 1).value in (0, None)
+    with pytest.raises(ValueError):
+        S._stream(_FakeStream(1), 0)
+    with pytest.raises(ValueError):
+        S._stream(_FakeStream(0), torch.device("cuda", 2))

@@ -113,3 +113,18 @@ def test_qr_full_size_8192_properties(cuda):
     assert torch.diagonal(R)[~skip].min().item() >= 0.0
     del P, Q, R, Qd, X, low
     torch.cuda.empty_cache()
+
+
+def test_qr_status_word_reports_breakdown(cuda):
+    """soap_qr's status word: 0 for a finite input, the QR-breakdown bit where a pivot norm is
+    not finite (no exception: the host reads the word once the stream has passed the call)."""
+    g = torch.Generator(device=cuda).manual_seed(9)
+    X = torch.randn(2, 128, 128, device=cuda, generator=g)
+    P = (X @ X.transpose(1, 2)).contiguous()
+    _, _, status = S.soap_qr(P, 1e-4, return_status=True)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    P[1, 0, 5] = float("inf")
+    _, _, status = S.soap_qr(P, 1e-4, return_status=True)
+    torch.cuda.synchronize()
+    assert status.item() & S.STATUS_QR_BREAKDOWN

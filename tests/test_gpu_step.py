@@ -280,4 +280,4 @@ def test_invalid_arguments(cuda):
         opt.state_get(0, 99)
     opt.destroy()
     lib = S.load_library()
-    assert lib.soap_qr(9000, 1, None, None, None, 0.0, None, 0, None) == 1
+    assert lib.soap_qr(9000, 1, None, None, None, 0.0, None, 0, None, None) == 1

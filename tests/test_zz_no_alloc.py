@@ -25,8 +25,9 @@ def test_static_workspace_qr_matches_soap_qr(cuda):
     for n, batch in ((1024, 1), (512, 3)):
         P = torch.from_numpy(_psd(rng, batch, n, n // 2)).to(cuda)
         Q_ref, skip_ref = S.soap_qr(P, 1e-4)
-        Q, skip = S.soap_qr_static(P, 1e-4)
+        Q, skip, status = S.soap_qr_static(P, 1e-4, return_status=True)
         torch.cuda.synchronize()
+        assert status.item() == 0
         assert torch.equal(skip, skip_ref)
         assert (Q - Q_ref).abs().max().item() <= 1e-5
         Qd = Q.double()
@@ -39,3 +40,18 @@ def test_static_workspace_refuses_more_than_it_holds(cuda):
     with pytest.raises(S.SoapError) as err:
         S.soap_qr_static(P, 1e-4)
     assert err.value.code == 1  # SOAP_ERR_INVALID_ARG
+
+
+def test_static_workspace_reports_a_breakdown(cuda):
+    """The call's device status reaches the caller: a non-finite input sets the QR-breakdown
+    bit in the caller's word, and the next clean call clears it again."""
+    rng = np.random.default_rng(5)
+    P = torch.from_numpy(_psd(rng, 1, 256, 64)).to(cuda)
+    bad = P.clone()
+    bad[0, 3, 7] = float("nan")
+    _, _, status = S.soap_qr_static(bad, 1e-4, return_status=True)
+    torch.cuda.synchronize()
+    assert status.item() & S.STATUS_QR_BREAKDOWN
+    _, _, status = S.soap_qr_static(P, 1e-4, return_status=True)
+    torch.cuda.synchronize()
+    assert status.item() == 0
