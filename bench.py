@@ -153,9 +153,12 @@ def measured_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
-# tensor-core fp32 products take 4 tf32 MMAs (hi/lo split of both operands); TF32 runs at
-# half the bf16 rate on this part
+# tensor-core fp32 products take 4 tf32 MMAs (hi/lo split of both operands)
 TC_PRODUCTS = 4
+# TF32 dense matmul throughput of the GB300s, measured with `python bench.py --peaks`
+# (torch.matmul 8192^3 with TF32 allowed: best of 10, and back to back for 4 s); the summary is
+# profiles/peaks_gb300.md. The driver's MEASURED_PEAKS.json has the bf16 and HBM figures only.
+TF32_TFLOPS = {"burst": 1047.2, "sustained": 951.8}
 
 # DRAM bytes (ncu dram__bytes_read.sum + dram__bytes_write.sum) per algorithmic byte of each
 # kernel family, measured with ncu over one step of the block's 2048x8192 matrix alone
@@ -179,18 +182,24 @@ def roofline(family, st, peaks, peak_src, products=None, dtype_ratio=2.0):
         return dict(base, bound="alu", achieved=ach, peak=FP32_SIMT_PEAK_TFLOPS, unit="TFLOP/s",
                     frac=ach / FP32_SIMT_PEAK_TFLOPS,
                     peak_source="fp32 FMA peak of the CUDA cores, 152 SMs x 128 lanes x 2 x 2.07 GHz")
-    # the kernels run inside a long step: the sustained tensor peak; fp32 products take
-    # TC_PRODUCTS tf32 MMAs at half the bf16 rate, bf16 products (Muon) one MMA at the bf16 rate
+    # the kernels run inside a long step: the sustained tensor peak. fp32 products take
+    # TC_PRODUCTS tf32 MMAs at the measured TF32 rate; bf16 products (Muon) one MMA at the
+    # measured bf16 rate
     products = TC_PRODUCTS if products is None else products
-    tc_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]) / dtype_ratio / products
+    if products > 1:
+        tc_peak = TF32_TFLOPS["sustained"] / products
+        tc_src = f"measured sustained tf32 dense ({TF32_TFLOPS['sustained']} TFLOP/s, bench.py --peaks) / {products}" \
+                 " (tf32 products per fp32 product)"
+    else:
+        tc_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
+        tc_src = f"{peak_src} sustained bf16 dense"
     ridge = tc_peak * 1e12 / (peaks["hbm_gbs"] * 1e9)  # FLOP per byte where the two bounds meet
     # a tensor-core family whose FLOPs per algorithmic byte reach the ridge is bound by the tensor
     # pipe (the QR's block products sit at the ridge: 2 x 128 fp32 FLOP per 4-8 bytes of C)
     if family in ("gemm_tc", "qr_update") and st["flops"] / max(1.0, st["bytes"]) >= ridge:
         ach = st["flops"] / secs / 1e12
         return dict(base, bound="tensor", achieved=ach, peak=tc_peak, unit="TFLOP/s", frac=ach / tc_peak,
-                    peak_source=f"{peak_src} sustained bf16 dense" + (
-                        f" / 2 (tf32) / {products} (tf32 products per fp32 product)" if products > 1 else ""))
+                    peak_source=tc_src)
     ach = st["bytes"] / secs / 1e9
     return dict(base, bound="hbm", achieved=ach, peak=peaks["hbm_gbs"], unit="GB/s", frac=ach / peaks["hbm_gbs"],
                 peak_source=peak_src)
@@ -606,7 +615,7 @@ def run_soap(args):
     if not (muon or args.kl or layerwise or subset):
         lib_v, lib_note = library_sample(specs, dev)
         lib_line = {"value": lib_v, "unit": "steps/s", "kind": "torch + cuSOLVER", "sample": lib_note}
-    tc_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]) / (1.0 if muon else 2.0 * TC_PRODUCTS)
+    tc_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]) if muon else TF32_TFLOPS["sustained"] / TC_PRODUCTS
     line = {
         "metric": MUON_METRIC if muon else METRIC, "value": value, "unit": "steps/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps,

@@ -86,7 +86,7 @@ typedef struct {
 
 /* Fills *hp with the defaults used for the paper's workloads: lr 3e-3,
  * beta1 = beta2 = factor_beta = 0.95, eps 1e-8, weight_decay 0.1, F = 1, no bias
- * correction, qr_tol 1e-4, guard on, standard factor EMAs (kl 0) with the current gradient
+ * correction, qr_tol 2e-5, guard on, standard factor EMAs (kl 0) with the current gradient
  * (stale 0). */
 void soap_default_hparams(soap_hparams* hp);
 
@@ -231,6 +231,16 @@ typedef struct {
  * before soap_profile_end, which discards them. The library's QR streams run concurrently
  * with each other and with the caller's stream, so records may overlap in time. */
 soap_status_t soap_profile_records(soap_handle h, soap_launch_record* out, int64_t max, int64_t* count);
+
+/* Failure detection (the paper has no counterpart). Every device-side wait of the tensor-core
+ * products is bounded: after `limit_ns` nanoseconds (0: the default, 2 s) it gives up, the
+ * kernel drains what it has in flight, frees its tensor memory and returns, and the status word
+ * gets SOAP_STATUS_TIMEOUT (soap_status then returns SOAP_ERR_TIMEOUT). `hold`, if not NULL, is
+ * a device int32 that every such product first waits for to become non-zero -- a flag that
+ * nothing sets makes the waits run out, which is how the timeout path is tested without a
+ * fault. Applies to launches enqueued after the call, from any thread; soap_wait_limit(0, NULL)
+ * restores the defaults. Results of a product whose wait gave up are not valid. */
+soap_status_t soap_wait_limit(uint64_t limit_ns, const int32_t* hold);
 
 /* ---- stand-alone sub-steps (the same kernels soap_step runs) ------------------- */
 

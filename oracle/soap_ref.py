@@ -137,7 +137,7 @@ class HParams:
     eig_every: int = 1            # F: refresh the basis when t mod F == 0
     bias_correction: bool = False
     guard: bool = True
-    qr_tol: float = 1e-4
+    qr_tol: float = 2e-5
     kl: bool = False              # KL-Shampoo factor form (Alg. 1's "Accumulate Kronecker Factors")
     stale: bool = False           # factors updated after the refresh (the stale variant of section 5)
     refresh: str = "qr"           # "qr" (Alg. 1) or "eigh" (the appendix's alternative)

@@ -29,9 +29,10 @@
 // (beta != 0), the epilogue warps copy their part of the C tile into shared memory with
 // cp.async while the MMAs run. For short K a CTA runs several consecutive tiles, so that
 // the next tile's loads and MMAs proceed while the epilogue stores the current one.
-// Stages are handed over with mbarriers; every wait gives up after ~2 s of %globaltimer
-// time, records kStatusTimeout and lets the CTA drain and free its tensor memory instead
-// of hanging.
+// Stages are handed over with mbarriers; every wait gives up after a bounded time (2 s of
+// %globaltimer time unless soap_wait_limit set another), records kStatusTimeout and lets the
+// CTA drain -- TMA copies already issued land, issued MMAs complete -- and free its tensor
+// memory instead of hanging. The drains themselves always keep the full 2 s bound.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -101,15 +102,25 @@ __device__ __forceinline__ bool mbar_try(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Bounded wait on an mbarrier phase: false after kWaitNs without completion.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+// Bounded wait on an mbarrier phase: false after `limit_ns` without completion.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
   if (mbar_try(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   for (;;) {
-    for (int i = 0; i < 256; ++i)
+    for (int i = 0; i < 16; ++i)
       if (mbar_try(bar, parity)) return true;
-    if (globaltimer() - t0 > kWaitNs) return false;
+    if (globaltimer() - t0 > limit_ns) return false;
   }
+}
+
+// Bounded wait until *flag != 0 (a flag set from outside the kernel): false after `limit_ns`.
+__device__ __forceinline__ bool flag_wait(const int* flag, uint64_t limit_ns) {
+  const volatile int* f = flag;
+  if (*f != 0) return true;
+  const uint64_t t0 = globaltimer();
+  while (*f == 0)
+    if (globaltimer() - t0 > limit_ns) return false;
+  return true;
 }
 
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, uint64_t* bar, int c0, int c1,
@@ -229,11 +240,13 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
   uint64_t* conv = empty + STAGES;          // [STAGES] CVTA: the stage's A lo part is in place
   uint64_t* acc_full = conv + STAGES;       // [NACC] accumulator a holds a finished K block
   uint64_t* acc_empty = acc_full + C::NACC;  // [NACC] accumulator a has been drained
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acc_empty + C::NACC);
+  uint64_t* mma_done = acc_empty + C::NACC;  // every MMA this CTA issued has completed
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(mma_done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
   volatile int* consumed = abort_flag + 1;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint64_t lim = ep.wait_ns ? ep.wait_ns : kWaitNs;  // bound of every wait but the drains
   const int kblocks = (K + BK - 1) / BK;
   const int kper = (kblocks + ksplit - 1) / ksplit;  // K blocks of one split
   const int ntn = (N + BN - 1) / BN, ntm = (M + BM - 1) / BM;
@@ -256,6 +269,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
       mbar_init(&acc_full[a], 1);
       mbar_init(&acc_empty[a], C::EPI);  // one arrival per epilogue warp
     }
+    mbar_init(mma_done, 1);
     *abort_flag = 0;
     *consumed = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -287,8 +301,9 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
         for (int kb = kb0; kb < kb1; ++kb, ++g) {
           const int s = g % STAGES;
           const uint32_t ph = (g / STAGES) & 1;
-          if (!mbar_wait(&empty[s], ph ^ 1) || *abort_flag) {
+          if (!mbar_wait(&empty[s], ph ^ 1, lim) || *abort_flag) {
             *abort_flag = 1;
+            if (ep.status) atomicOr(ep.status, kStatusTimeout);
             break;
           }
           mbar_expect_tx(&full[s], CVTA ? C::STAGE - C::TILE_A : C::STAGE);
@@ -303,7 +318,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
       }
       if (*abort_flag) {
         // let copies already in flight land before the CTA's shared memory goes away
-        for (int gg = *consumed; gg < issued; ++gg) mbar_wait(&full[gg % STAGES], (gg / STAGES) & 1);
+        for (int gg = *consumed; gg < issued; ++gg) mbar_wait(&full[gg % STAGES], (gg / STAGES) & 1, kWaitNs);
       }
     }
   } else if (warp == 1) {
@@ -318,10 +333,11 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
           const int s = g % STAGES;
           const uint32_t ph = (g / STAGES) & 1;
           const int a = g % C::NACC;
-          if (!mbar_wait(CVTA ? &conv[s] : &full[s], ph) ||
-              (g >= C::NACC && !mbar_wait(&acc_empty[a], ((g / C::NACC) & 1) ^ 1)) ||
+          if (!mbar_wait(CVTA ? &conv[s] : &full[s], ph, lim) ||
+              (g >= C::NACC && !mbar_wait(&acc_empty[a], ((g / C::NACC) & 1) ^ 1, lim)) ||
               *abort_flag) {
             *abort_flag = 1;
+            if (ep.status) atomicOr(ep.status, kStatusTimeout);
             break;
           }
           *consumed = g + 1;
@@ -343,6 +359,12 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
           umma_commit(&acc_full[a]);  // hands the K block's sum to the epilogue warps
         }
       }
+      // the tensor memory is freed below: every MMA issued must have completed first (this
+      // matters only when a wait gave up; otherwise the epilogue has drained them all)
+      if (g > 0) {
+        umma_commit(mma_done);
+        mbar_wait(mma_done, 0, kWaitNs);
+      }
     }
   } else {
     const int q = warp & 3;  // this warp may read accumulator lanes 32q .. 32q+31
@@ -353,7 +375,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     // written beside it for the tensor core (which reads it through the async proxy)
     auto convert = [&](int gc) -> bool {
       const int s = gc % STAGES;
-      if (!mbar_wait(&full[s], (gc / STAGES) & 1) || *abort_flag) return false;
+      if (!mbar_wait(&full[s], (gc / STAGES) & 1, lim) || *abort_flag) return false;
       const float4* src = reinterpret_cast<const float4*>(smem + s * C::STAGE);
       float4* dst = reinterpret_cast<float4*>(smem + s * C::STAGE + C::TILE_A);
       for (int u = (warp - 2) * 32 + lane; u < C::TILE_A / 16; u += C::EPI * 32) {
@@ -376,6 +398,12 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     int gconv = 0;  // next K block to convert, kept STAGES - 1 ahead of the drains
     int g = 0;
     bool valid = true;
+    if (ep.hold && !flag_wait(ep.hold, lim)) {
+      // the timeout path under test: no tile is drained, the other warps' waits run out too
+      valid = false;
+      *abort_flag = 1;
+      if (lane == 0 && ep.status) atomicOr(ep.status, kStatusTimeout);
+    }
     for (int t = t_begin; t < t_end && valid; ++t) {
       int m0, n0, b, kb0, kb1;  // b: output matrix (split * batch + operand matrix)
       tile_coords(t, ntm, ntn, BN, m0, n0, b);
@@ -420,7 +448,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
         if (CVTA)
           while (valid && gconv < gtotal && gconv <= g + STAGES - 1) valid = convert(gconv++);
         const int a = g % C::NACC;
-        if (!valid || !mbar_wait(&acc_full[a], (g / C::NACC) & 1) || *abort_flag) {
+        if (!valid || !mbar_wait(&acc_full[a], (g / C::NACC) & 1, lim) || *abort_flag) {
           valid = false;
           break;
         }
@@ -687,9 +715,23 @@ int choose_ksplit(int64_t tiles, int kblocks, int64_t cap) {
 
 }  // namespace tc
 
-cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const TcOperand& B, const TcEpilogue& ep,
-                       cudaStream_t s, int family, float* split_ws, size_t split_ws_floats) {
+namespace {
+// soap_wait_limit's settings, read by every launch
+std::atomic<uint64_t> g_wait_ns{0};
+std::atomic<const int*> g_hold{nullptr};
+}  // namespace
+
+void set_wait_limit(uint64_t ns, const int* hold) {
+  g_wait_ns.store(ns, std::memory_order_relaxed);
+  g_hold.store(hold, std::memory_order_relaxed);
+}
+
+cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const TcOperand& B,
+                       const TcEpilogue& ep_in, cudaStream_t s, int family, float* split_ws, size_t split_ws_floats) {
   if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
+  TcEpilogue ep = ep_in;
+  ep.wait_ns = g_wait_ns.load(std::memory_order_relaxed);
+  ep.hold = g_hold.load(std::memory_order_relaxed);
   if (batch > 65535) return cudaErrorInvalidValue;
   const double flops = 2.0 * M * N * (double)K * batch;  // algorithmic (4 tf32 products each on the pipe)
   const double bytes = 4.0 * ((A.lo ? 2.0 : 1.0) * (double)M * K * (A.batch > 0 ? A.batch : batch) +
@@ -718,7 +760,9 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
   if (cvt && (pre || ep.transpose)) return cudaErrorInvalidValue;
   if (B.lo == nullptr) return cudaErrorInvalidValue;
   if (ksplit > 1) {
-    const TcEpilogue pe{split_ws, nullptr, N, (int64_t)M * N, nullptr, N, (int64_t)M * N, 0, 1.f, 0.f, ep.status};
+    TcEpilogue pe{split_ws, nullptr, N, (int64_t)M * N, nullptr, N, (int64_t)M * N, 0, 1.f, 0.f, ep.status};
+    pe.wait_ns = ep.wait_ns;
+    pe.hold = ep.hold;
     cudaError_t e = N <= 32 ? (cvt ? tc::launch<32, 5, false, true>(A, B, M, N, K, batch, pe, s, ksplit)
                                    : tc::launch<32, 5, false>(A, B, M, N, K, batch, pe, s, ksplit))
                             : (cvt ? tc::launch<128, 3, false, true>(A, B, M, N, K, batch, pe, s, ksplit)

@@ -285,8 +285,8 @@ soap_status_t muon_step(muon_handle h, float* const* params, const float* const*
   if (h->status_pending && cudaEventQuery(h->status_ev) == cudaSuccess) {
     h->status_pending = false;
     const int bits = *h->h_status;
-    if (bits & soap::kStatusNonFinite) return fail(h, SOAP_ERR_NONFINITE, "muon_step: non-finite gradient earlier");
     if (bits & soap::kStatusTimeout) return fail(h, SOAP_ERR_TIMEOUT, "muon_step: a device wait timed out earlier");
+    if (bits & soap::kStatusNonFinite) return fail(h, SOAP_ERR_NONFINITE, "muon_step: non-finite gradient earlier");
   }
   bool changed = false;
   for (auto& c : h->classes)
@@ -348,8 +348,8 @@ soap_status_t muon_status(muon_handle h, soap_stream_t stream) {
   MUON_CUDA(h, cudaMemcpyAsync(h->h_status, h->d_status, sizeof(int), cudaMemcpyDeviceToHost, (cudaStream_t)stream));
   MUON_CUDA(h, cudaStreamSynchronize((cudaStream_t)stream));
   const int bits = *h->h_status;
-  if (bits & soap::kStatusNonFinite) return SOAP_ERR_NONFINITE;
   if (bits & soap::kStatusTimeout) return SOAP_ERR_TIMEOUT;
+  if (bits & soap::kStatusNonFinite) return SOAP_ERR_NONFINITE;
   return SOAP_OK;
 }
 

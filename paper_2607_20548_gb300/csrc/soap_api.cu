@@ -263,11 +263,12 @@ soap_status_t cuda_fail(soap_handle h, cudaError_t e, const char* what) {
     if (e_ != cudaSuccess) return cuda_fail(h, e_, #expr); \
   } while (0)
 
-// A non-finite gradient also makes the QR of that step break down; report the cause.
+// Report the cause: a product whose wait gave up leaves its output unwritten, which can make
+// later values non-finite, and a non-finite gradient also makes the QR of that step break down.
 soap_status_t status_code(int bits) {
+  if (bits & soap::kStatusTimeout) return SOAP_ERR_TIMEOUT;
   if (bits & soap::kStatusNonFinite) return SOAP_ERR_NONFINITE;
   if (bits & soap::kStatusQrBreakdown) return SOAP_ERR_QR_BREAKDOWN;
-  if (bits & soap::kStatusTimeout) return SOAP_ERR_TIMEOUT;
   return SOAP_OK;
 }
 
@@ -750,7 +751,7 @@ void soap_default_hparams(soap_hparams* hp) {
   hp->weight_decay = 0.1f;
   hp->eig_every = 1;
   hp->bias_correction = 0;
-  hp->qr_tol = 1e-4f;
+  hp->qr_tol = 2e-5f;
   hp->guard = 1;
   hp->kl = 0;
   hp->stale = 0;
@@ -1440,6 +1441,12 @@ soap_status_t soap_gemm_tf32x4(int32_t M, int32_t N, int32_t K, int32_t batch, c
                       reinterpret_cast<int*>(status)};
   cudaError_t e = soap::gemm_tc_nt(M, N, K, batch, A, B, ep, (cudaStream_t)stream);
   return e == cudaSuccess ? SOAP_OK : (e == cudaErrorInvalidValue ? SOAP_ERR_INVALID_ARG : SOAP_ERR_CUDA);
+}
+
+soap_status_t soap_wait_limit(uint64_t limit_ns, const int32_t* hold) {
+  if ((reinterpret_cast<uintptr_t>(hold) & 3) != 0) return SOAP_ERR_INVALID_ARG;
+  soap::set_wait_limit(limit_ns, reinterpret_cast<const int*>(hold));
+  return SOAP_OK;
 }
 
 soap_status_t soap_split_tf32(const float* x, float* hi, float* lo, int64_t n, soap_stream_t stream) {

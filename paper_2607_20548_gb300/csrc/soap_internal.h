@@ -71,6 +71,9 @@ struct TcEpilogue {
   int transpose;         // write C^T (C_b is then N x M with leading dimension ldc)
   float alpha, beta;     // beta != 0 reads C
   int* status;           // device status word for a timed-out wait (may be nullptr)
+  // set by gemm_tc_nt from the library's wait settings (soap_wait_limit), not by callers:
+  uint64_t wait_ns = 0;       // bounded waits give up after this long
+  const int* hold = nullptr;  // testing the timeout path: the epilogue first waits for *hold != 0
 };
 // `family` tags the launch for the library's profiler. With a split workspace (room for
 // ksplit * batch * M * N floats) a launch of few tiles and long K may split K over more CTAs
@@ -78,6 +81,9 @@ struct TcEpilogue {
 cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const TcOperand& B,
                        const TcEpilogue& ep, cudaStream_t stream, int family = kFamGemmTc,
                        float* split_ws = nullptr, size_t split_ws_floats = 0);
+// Bound of the tensor-core products' device waits (0: 2 s) and, for testing the timeout path, a
+// device flag their epilogues first wait for (nullptr: none); applies to later launches.
+void set_wait_limit(uint64_t ns, const int* hold);
 // hi = trunc_tf32(x), lo = x - hi (exact), elementwise over n values.
 cudaError_t split_tf32(const float* x, float* hi, float* lo, int64_t n, cudaStream_t stream);
 

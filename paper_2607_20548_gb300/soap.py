@@ -29,7 +29,7 @@ EXPORTS = ("soap_default_hparams", "soap_create", "soap_create_ex", "soap_plan_i
            "soap_clear_status", "soap_last_error", "soap_destroy", "soap_qr_workspace_bytes",
            "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_profile_records",
            "soap_gemm_tf32x4",
-           "soap_split_tf32", "soap_qr_static", "soap_layerwise_assign")
+           "soap_split_tf32", "soap_qr_static", "soap_layerwise_assign", "soap_wait_limit")
 # every symbol include/muon.h declares
 MUON_EXPORTS = ("muon_default_hparams", "muon_create", "muon_step", "muon_set_lr", "muon_state_get",
                 "muon_state_set", "muon_status", "muon_last_error", "muon_destroy", "muon_profile_begin",
@@ -109,6 +109,7 @@ def load_library(path: str = LIB_PATH):
         "soap_gemm_tf32x4": (I32, [I32, I32, I32, I32, P, P, I64, I64, P, P, I64, I64, I32, F, F, P, I64, I64,
                                    I32, P, P, P]),
         "soap_split_tf32": (I32, [P, P, P, I64, P]),
+        "soap_wait_limit": (I32, [ctypes.c_uint64, P]),
         "soap_qr_static": (I32, [I32, I32, P, P, P, F, P, P]),
         "soap_layerwise_assign": (I32, [ctypes.POINTER(soap_shape), I32, I32, I32, ctypes.POINTER(I32),
                                         ctypes.POINTER(ctypes.c_double)]),
@@ -379,6 +380,14 @@ def soap_qr_static(P: torch.Tensor, tol: float = 0.0, stream=None, return_status
                               f"{lib.soap_qr_workspace_bytes(n, batch)} bytes of workspace; the fixed array "
                               "holds 32 MiB" if code == 1 else "soap_qr_static failed")
     return (Q, skip, status) if return_status else (Q, skip)
+
+
+def soap_wait_limit(limit_ns: int = 0, hold: torch.Tensor | None = None):
+    """soap_wait_limit: bound of the tensor-core products' device waits (0 = default 2 s) and an
+    optional int32 CUDA flag their epilogues first wait for (testing the timeout path)."""
+    if hold is not None:
+        _one_device("soap_wait_limit hold", hold, dtype=torch.int32)
+    _check(load_library().soap_wait_limit(int(limit_ns), ctypes.c_void_p(hold.data_ptr()) if hold is not None else None))
 
 
 def soap_gemm(A: torch.Tensor, B: torch.Tensor, trans_a=False, trans_b=False, alpha=1.0, beta=0.0,

@@ -8,15 +8,20 @@ Tolerance (derived from the arithmetic): the bound is a relative Frobenius error
 <= 1e-3 of each step's update, or 4x the fp32 twin's error where the twin -- a faithful
 fp32 implementation -- cannot do better.
 
-Some steps are beyond fp32 resolution altogether: when the refreshed basis rotates
-momentum into directions whose second moment is still ~0 (v is not re-projected), Adam's
-m / (sqrt(v) + eps) turns a G' entry of ~1e-7 into |N| in the thousands, so the update
-depends on the rounding of that tiny entry (the twin and the GPU then differ from fp64,
-and from each other, by O(1e-2..1)). Such a step (twin error > 1e-3 / 4, or oracle
-max|N| > 100, far past the bound |N| <= 1 that Adam obeys without a basis change) is
-verified piece by piece instead: the GPU's m, v, L, R, Q after the step against the
-teacher-forced oracle, and the GPU's update against Q_L N Q_R^T recomputed in fp64 from
-the GPU's own m, v and bases -- every well-conditioned quantity of the step.
+Some steps are beyond fp32 resolution as a whole: when the refreshed basis rotates momentum
+into directions whose second moment is still ~0 (v is not re-projected), Adam's
+m / (sqrt(v) + eps) turns a G' entry of ~1e-7 into |N| in the thousands, so those entries of
+N depend on the rounding of that tiny entry, and the whole update of any fp32 implementation
+(the twin, the GPU) lands anywhere between 1e-4 and 1e-1 of fp64's, at random (measured on one
+such step: twin 7e-4, GPU 4e-2). Every step must meet the bound on the whole update; a step that
+misses it may instead be checked on Adam's normal range, but only if the oracle's N has entries
+outside it. With m and v accumulated in one basis and beta1 = beta2, |m| <= sqrt(v), so |N| <= 1
+(normal_bound gives the bound for any betas); an entry above it exists only through a basis
+change. The fallback compares the update with the oracle's entry by entry of N: Q_L (N o mask)
+Q_R^T with mask = |N_oracle| <= bound, from the GPU's m, v and bases against the same from the
+oracle's, at 1e-3 (or 4x the twin's masked error). The amplified entries (mask = 0) are counted
+and reported, with both full-update errors. The state after the step (m, v, L, R) is held to
+1e-4, or to 4x the twin's own error of that piece where the twin's floor is higher.
 """
 from __future__ import annotations
 
@@ -28,7 +33,43 @@ from paper_2607_20548_gb300 import soap as S
 
 TOL = 1e-3
 TWIN_FACTOR = 4.0
-N_CAP = 100.0
+N_NORMAL = 1.0  # Adam's normal range for beta1 = beta2: |m| <= sqrt(v) without a basis change
+
+
+def normal_bound(hp) -> float:
+    """Largest |N| = |m| / sqrt(v) Adam reaches without a basis change (Cauchy-Schwarz over the
+    EMA weights; bias correction leaves it unchanged): 1 for beta1 = beta2, in general
+    sqrt((1 - b1)^2 / ((1 - b2) (1 - b1^2 / b2))), unbounded for b1^2 >= b2."""
+    b1, b2 = float(hp.beta1), float(hp.beta2)
+    if b1 * b1 >= b2:
+        return float("inf")
+    return float(np.sqrt((1 - b1) ** 2 / ((1 - b2) * (1 - b1 * b1 / b2)))) * (1 + 1e-6)
+
+
+def adam_direction(m, v, hp, t, skipL=None, skipR=None):
+    """N = m / (sqrt(v) + eps) in fp64 (bias-corrected if set) with the guard's zero rows/cols."""
+    m = np.asarray(m, np.float64)
+    v = np.asarray(v, np.float64)
+    if hp.bias_correction:
+        N = (m / (1 - hp.beta1 ** t)) / (np.sqrt(v / (1 - hp.beta2 ** t)) + hp.eps)
+    else:
+        N = m / (np.sqrt(v) + hp.eps)
+    if hp.guard:
+        if skipL is not None:
+            N[np.asarray(skipL, bool), :] = 0
+        if skipR is not None:
+            N[:, np.asarray(skipR, bool)] = 0
+    return N
+
+
+def masked_update(QL, N, QR, mask):
+    """Q_L (N o mask) Q_R^T in fp64 (an identity side: Q = None)."""
+    X = np.where(mask, N, 0.0)
+    if QL is not None:
+        X = np.asarray(QL, np.float64) @ X
+    if QR is not None:
+        X = X @ np.asarray(QR, np.float64).T
+    return X
 
 
 def rel(a, b):
@@ -88,34 +129,47 @@ class TeacherForcedCheck:
         d_ref = W64 - W0
         e_gpu = rel(W1 - W0, d_ref)
         e_twin = rel(W32.astype(np.float64) - W0, d_ref)
-        N64 = st64.m / (np.sqrt(st64.v) + hp.eps)
-        Nmax = float(np.abs(N64).max())
         sp = self.opt.shapes[idx]
+        N64 = adam_direction(st64.m, st64.v, hp, t, st64.skipL if sp.left else None,
+                             st64.skipR if sp.right else None)
+        N32 = adam_direction(st32.m, st32.v, hp, t, st32.skipL if sp.left else None,
+                             st32.skipR if sp.right else None)
+        Nmax = float(np.abs(N64).max())
         g = lambda w: self.opt.state_get(idx, w).cpu().numpy()
         m_gpu, v_gpu = g(S.STATE_M).astype(np.float64), g(S.STATE_V).astype(np.float64)
         row = dict(idx=idx, t=t, e_gpu=e_gpu, e_twin=e_twin, max_abs_N=Nmax,
-                   e_m=rel(m_gpu, st64.m), e_v=rel(v_gpu, st64.v))
-        row["ill"] = bool(TWIN_FACTOR * e_twin > TOL or Nmax > N_CAP)
-        # the GPU's update against Q_L N Q_R^T from its own state, in fp64
-        N = m_gpu / (np.sqrt(v_gpu) + hp.eps) if not hp.bias_correction else \
-            (m_gpu / (1 - hp.beta1 ** t)) / (np.sqrt(v_gpu / (1 - hp.beta2 ** t)) + hp.eps)
+                   e_m=rel(m_gpu, st64.m), e_v=rel(v_gpu, st64.v),
+                   twin_m=rel(st32.m, st64.m), twin_v=rel(st32.v, st64.v))
+        bound_N = normal_bound(hp)
         QL = QR = None
+        skL = skR = None
         if sp.left:
             QL = g(S.STATE_QL).astype(np.float64)
             row["e_L"] = rel(g(S.STATE_L), st64.L)
+            row["twin_L"] = rel(st32.L, st64.L)
             skL = g(S.STATE_SKIP_L).astype(bool)
             row["skipL_same"] = bool(np.array_equal(skL, st64.skipL))
             row["orth_L"] = orth_err(self.opt.state_get(idx, S.STATE_QL))
-            if hp.guard:
-                N[skL, :] = 0
         if sp.right:
             QR = g(S.STATE_QR).astype(np.float64)
             row["e_R"] = rel(g(S.STATE_R), st64.R)
+            row["twin_R"] = rel(st32.R, st64.R)
             skR = g(S.STATE_SKIP_R).astype(bool)
             row["skipR_same"] = bool(np.array_equal(skR, st64.skipR))
             row["orth_R"] = orth_err(self.opt.state_get(idx, S.STATE_QR))
-            if hp.guard:
-                N[:, skR] = 0
+        # the GPU's own direction N from its m, v and zero-column flags
+        N = adam_direction(m_gpu, v_gpu, hp, t, skL, skR)
+        # the update on Adam's normal range against the oracle's, entry by entry of N
+        mask = np.abs(N64) <= bound_N
+        ref_QL = st64.QL if sp.left else None
+        ref_QR = st64.QR if sp.right else None
+        d_mask = masked_update(ref_QL, N64, ref_QR, mask)
+        row["e_mask"] = rel(masked_update(QL, N, QR, mask), d_mask)
+        row["e_mask_twin"] = rel(masked_update(st32.QL if sp.left else None, N32, st32.QR if sp.right else None,
+                                               mask), d_mask)
+        row["amplified"] = int((~mask).sum())
+        # the full update beyond fp32 resolution: it misses the bound and N has amplified entries
+        row["ill"] = bool(e_gpu > max(TOL, TWIN_FACTOR * e_twin) and row["amplified"] > 0)
         dW_self = (QL @ N if QL is not None else N)
         dW_self = dW_self @ QR.T if QR is not None else dW_self
         keep = 1 - hp.lr * hp.weight_decay
@@ -126,7 +180,8 @@ class TeacherForcedCheck:
     def report(self) -> str:
         out = []
         for r in self.rows:
-            tag = "  [beyond fp32 resolution: verified piece by piece]" if r["ill"] else ""
+            tag = (f"  [whole update beyond fp32 resolution; on Adam's normal range gpu {r['e_mask']:.1e} "
+                   f"twin {r['e_mask_twin']:.1e}, {r['amplified']} amplified entries]") if r["ill"] else ""
             out.append(f"matrix {r['idx']:4d} step {r['t']:3d}: gpu {r['e_gpu']:.2e} twin {r['e_twin']:.2e} "
                        f"max|N| {r['max_abs_N']:.0f} m {r['e_m']:.1e} v {r['e_v']:.1e} self {r['e_self']:.1e}{tag}")
         return "\n".join(out)
@@ -134,16 +189,19 @@ class TeacherForcedCheck:
     def assert_ok(self, state_tol=1e-4):
         bad = []
         for r in self.rows:
-            if not r["ill"] and not r["e_gpu"] <= max(TOL, TWIN_FACTOR * r["e_twin"]):
-                bad.append(f"update: {r}")
+            if not r["ill"]:
+                if not r["e_gpu"] <= max(TOL, TWIN_FACTOR * r["e_twin"]):
+                    bad.append(f"update: {r}")
+            elif not r["e_mask"] <= max(TOL, TWIN_FACTOR * r["e_mask_twin"]):
+                bad.append(f"update on Adam's normal range: {r}")
             # the update against Q_L N(m, v) Q_R^T from the GPU's own state: m is re-derived through
             # other fp32 products than the step used, so on ordinary steps it shares the update's
-            # bound; on steps beyond fp32 resolution it is the main check and is held tight
+            # bound; on steps beyond fp32 resolution it is held tight
             if not r["e_self"] <= (2e-4 if r["ill"] else max(TOL, TWIN_FACTOR * r["e_twin"])):
                 bad.append(f"self-consistency of the update: {r}")
-            for k in ("e_L", "e_R", "e_v", "e_m"):
-                if k in r and not r[k] <= max(state_tol, TWIN_FACTOR * r["e_twin"] if not r["ill"] else 0.0):
-                    bad.append(f"{k}: {r}")
+            for k in ("L", "R", "v", "m"):
+                if "e_" + k in r and not r["e_" + k] <= max(state_tol, TWIN_FACTOR * r["twin_" + k]):
+                    bad.append(f"e_{k}: {r}")
             for k in ("orth_L", "orth_R"):
                 if k in r and not r[k] <= 1e-5:
                     bad.append(f"{k}: {r}")

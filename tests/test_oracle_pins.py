@@ -495,3 +495,41 @@ def test_eigh_and_qr_refreshes_agree_at_the_fixed_point():
 def test_unknown_refresh_is_rejected():
     with pytest.raises(ValueError):
         soap_step(MatrixState(2, 2, True, True), np.zeros((2, 2)), np.ones((2, 2)), HParams(refresh="svd"))
+
+
+def _planted(n, lam, rng):
+    U, _ = np.linalg.qr(rng.standard_normal((n, n)))
+    return U, (U * lam) @ U.T
+
+
+def test_guard_zeroes_nothing_on_a_full_rank_factor():
+    """Reading R12's zero-column rule on a full-rank factor with kappa = 1e3 (eigenvalues
+    log-spaced in [1e-3, 1]): the refresh treats no column as zero, from Q = I and from a random
+    basis, over several refreshes, at the default qr_tol."""
+    rng = np.random.default_rng(31)
+    n = 64
+    _, L = _planted(n, np.logspace(-3, 0, n), rng)
+    for Q0 in (np.eye(n), np.linalg.qr(rng.standard_normal((n, n)))[0]):
+        Q = Q0
+        for _ in range(6):
+            Q, skip, _ = householder_q(L @ Q, HParams().qr_tol)
+            assert not skip.any()
+
+
+@pytest.mark.parametrize("lo, tol", [(1e-6, 1e-9), (1e-2, None)])
+def test_guard_zeroes_exactly_a_planted_null_space(lo, tol):
+    """A factor of rank 40 of 64 whose nonzero eigenvalues are log-spaced in [lo, 1]: the refresh
+    zeroes exactly 24 columns, and they span the planted null space (the kept ones its
+    complement). With nonzero eigenvalues down to 1e-6 this needs a qr_tol below their QR residuals
+    (1e-9 here, far above fp64 rounding); the default qr_tol, set just above the fp32 noise floor
+    of the step's refresh, does the same on a spectrum in [1e-2, 1]."""
+    rng = np.random.default_rng(32)
+    n, r = 64, 40
+    lam = np.concatenate([np.logspace(np.log10(lo), 0, r), np.zeros(n - r)])
+    U, L = _planted(n, lam, rng)
+    tol = HParams().qr_tol if tol is None else tol
+    for Q0 in (np.eye(n), np.linalg.qr(rng.standard_normal((n, n)))[0]):
+        Q, skip, _ = householder_q(L @ Q0, tol)
+        assert skip.sum() == n - r
+        assert np.abs(U[:, :r].T @ Q[:, skip]).max() <= 1e-8
+        assert np.abs(U[:, r:].T @ Q[:, ~skip]).max() <= 1e-8
