@@ -629,6 +629,7 @@ def run_soap(args):
                    "optimizer": "muon (16 quintic Newton-Schulz steps)" if muon else
                    ("soap, KL factor form" if args.kl else "soap, standard factor form"),
                    "waves_per_step": plan["waves"] if plan else None,
+                   "waves_pipelined": plan["pipelined"] if plan else None,
                    "workspace_gb": plan["workspace_bytes"] / 1e9 if plan else None,
                    "state_gb": plan["state_bytes"] / 1e9 if plan else None,
                    "gradients": (f"{npool} distinct step(s) of gradients resident"

@@ -114,9 +114,13 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
 soap_status_t soap_create_ex(const soap_shape* shapes, int32_t n, const soap_hparams* hp, int32_t device,
                              size_t workspace_limit, soap_handle* out);
 
-/* The plan soap_create chose: number of waves per step, workspace bytes and state bytes
- * (device memory held by the handle is their sum). Any pointer may be NULL. */
-soap_status_t soap_plan_info(soap_handle h, int32_t* waves, size_t* workspace_bytes, size_t* state_bytes);
+/* The plan soap_create chose: number of waves per step; whether they are pipelined (1: the
+ * workspace holds two waves, each in its half, so that one wave's preparation and factor
+ * update run while the previous wave's QR does; 0: waves run one after another); workspace
+ * bytes and state bytes (device memory held by the handle is their sum). Any pointer may be
+ * NULL. */
+soap_status_t soap_plan_info(soap_handle h, int32_t* waves, int32_t* pipelined, size_t* workspace_bytes,
+                             size_t* state_bytes);
 
 /* One SOAP step (Alg. 1) over all n matrices, enqueued on `stream`:
  * factor EMAs with the current gradient, power step P = L Q and QR refresh with

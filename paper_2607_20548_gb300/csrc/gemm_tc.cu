@@ -219,6 +219,19 @@ __device__ __forceinline__ void tile_coords(int t, int ntm, int ntn, int BN_, in
   n0 = (w / gsz) * BN_;
 }
 
+// Symmetric products (C = alpha A A^T + beta C, M = N): tile t -> (m0, n0, batch index) over the
+// tiles on or below the diagonal only, row by row (tile (i, j), j <= i, at i (i + 1) / 2 + j).
+__device__ __forceinline__ void tile_coords_sym(int t, int ntm, int& m0, int& n0, int& b) {
+  const int per = ntm * (ntm + 1) / 2;
+  b = t / per;
+  const int r = t - b * per;
+  int i = (int)((sqrtf(8.f * (float)r + 1.f) - 1.f) * 0.5f);
+  while ((i + 1) * (i + 2) / 2 <= r) ++i;
+  while (i * (i + 1) / 2 > r) --i;
+  m0 = i * BM;
+  n0 = (r - i * (i + 1) / 2) * BM;
+}
+
 // A CTA takes `tpc` consecutive tiles, so that the loads and MMAs of its next tile overlap
 // the epilogue of the current one. With ksplit > 1 the K blocks are split into ksplit
 // consecutive ranges; split s of matrix b is written as output matrix s * batch + b (partial
@@ -226,7 +239,10 @@ __device__ __forceinline__ void tile_coords(int t, int ntm, int ntn, int BN_, in
 // With CVTA the A operand comes as fp32 only: the epilogue warps form its lo part in shared
 // memory, beside the tile TMA brought in (for HBM-bound products whose A is read once; the
 // extra shared-memory traffic would slow a compute-bound product).
-template <int BN, int STAGES, bool PRE, bool CVTA, bool TR, bool LO, bool VEC>
+// With SYM (A = B, M = N, BN = BM) only the tiles on or below the diagonal are computed, and each
+// one below it is also stored transposed in the mirror position, so C stays exactly symmetric
+// with about half of the MMAs.
+template <int BN, int STAGES, bool PRE, bool CVTA, bool TR, bool LO, bool VEC, bool SYM>
 __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap ta_hi, const __grid_constant__ CUtensorMap ta_lo,
                    const __grid_constant__ CUtensorMap tb_hi, const __grid_constant__ CUtensorMap tb_lo, int M,
@@ -250,7 +266,7 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
   const int kblocks = (K + BK - 1) / BK;
   const int kper = (kblocks + ksplit - 1) / ksplit;  // K blocks of one split
   const int ntn = (N + BN - 1) / BN, ntm = (M + BM - 1) / BM;
-  const int ntiles = ntn * ntm * batch * ksplit;
+  const int ntiles = (SYM ? ntm * (ntm + 1) / 2 : ntn * ntm) * batch * ksplit;
   // the K blocks [kb0, kb1) of tile t, and its operand and output matrix indices
   auto krange = [&](int bo, int& kb0, int& kb1) {
     kb0 = (bo / batch) * kper;
@@ -295,7 +311,8 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
       int g = 0, issued = 0;  // k blocks over all of this CTA's tiles
       for (int t = t_begin; t < t_end && !*abort_flag; ++t) {
         int m0, n0, bo, kb0, kb1;
-        tile_coords(t, ntm, ntn, BN, m0, n0, bo);
+        if (SYM) tile_coords_sym(t, ntm, m0, n0, bo);
+        else tile_coords(t, ntm, ntn, BN, m0, n0, bo);
         krange(bo, kb0, kb1);
         const int b = bo % batch;
         for (int kb = kb0; kb < kb1; ++kb, ++g) {
@@ -325,19 +342,19 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_tf32(BM, BN);
       int g = 0;
-      for (int t = t_begin; t < t_end && !*abort_flag; ++t) {
+      bool ok = true;
+      for (int t = t_begin; t < t_end && ok && !*abort_flag; ++t) {
         int m0, n0, bo, kb0, kb1;
-        tile_coords(t, ntm, ntn, BN, m0, n0, bo);
+        if (SYM) tile_coords_sym(t, ntm, m0, n0, bo);
+        else tile_coords(t, ntm, ntn, BN, m0, n0, bo);
         krange(bo, kb0, kb1);
         for (int kb = kb0; kb < kb1; ++kb, ++g) {
           const int s = g % STAGES;
           const uint32_t ph = (g / STAGES) & 1;
           const int a = g % C::NACC;
           if (!mbar_wait(CVTA ? &conv[s] : &full[s], ph, lim) ||
-              (g >= C::NACC && !mbar_wait(&acc_empty[a], ((g / C::NACC) & 1) ^ 1, lim)) ||
-              *abort_flag) {
-            *abort_flag = 1;
-            if (ep.status) atomicOr(ep.status, kStatusTimeout);
+              (g >= C::NACC && !mbar_wait(&acc_empty[a], ((g / C::NACC) & 1) ^ 1, lim)) || *abort_flag) {
+            ok = false;
             break;
           }
           *consumed = g + 1;
@@ -358,6 +375,10 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
           umma_commit(&empty[s]);     // frees the stage once these MMAs have read it
           umma_commit(&acc_full[a]);  // hands the K block's sum to the epilogue warps
         }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        if (ep.status) atomicOr(ep.status, kStatusTimeout);
       }
       // the tensor memory is freed below: every MMA issued must have completed first (this
       // matters only when a wait gave up; otherwise the epilogue has drained them all)
@@ -391,7 +412,8 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     if (CVTA)
       for (int t = t_begin; t < t_end; ++t) {
         int m0, n0, bo, kb0, kb1;
-        tile_coords(t, ntm, ntn, BN, m0, n0, bo);
+        if (SYM) tile_coords_sym(t, ntm, m0, n0, bo);
+        else tile_coords(t, ntm, ntn, BN, m0, n0, bo);
         krange(bo, kb0, kb1);
         gtotal += kb1 - kb0;
       }
@@ -406,7 +428,8 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
     }
     for (int t = t_begin; t < t_end && valid; ++t) {
       int m0, n0, b, kb0, kb1;  // b: output matrix (split * batch + operand matrix)
-      tile_coords(t, ntm, ntn, BN, m0, n0, b);
+      if (SYM) tile_coords_sym(t, ntm, m0, n0, b);
+      else tile_coords(t, ntm, ntn, BN, m0, n0, b);
       krange(b, kb0, kb1);
       float* Cb = ep.C_ptrs ? ep.C_ptrs[b] : (ep.C ? ep.C + (int64_t)b * ep.c_stride : nullptr);
       float* Lb = LO && ep.C_lo ? ep.C_lo + (int64_t)b * ep.lo_stride : nullptr;
@@ -528,6 +551,21 @@ __global__ void __launch_bounds__(Cfg<BN, STAGES, PRE>::THREADS, 1)
               }
             }
           }
+          if (SYM && m0 != n0) {
+            // the mirror tile: element (r, j) of this block also goes to C[j][r]
+#pragma unroll 1
+            for (int it = 0; it < 8; ++it) {
+              const int jj = 4 * it + (lane >> 3), r4 = 4 * (lane & 7);
+              const int mrow = cc0 + jj, mcol = row0 + r4;  // row and column in C
+              if (mrow >= N || mcol + 3 >= M) continue;    // M = N, a multiple of 4
+              const float4 o = make_float4(cb[swz(r4, jj)], cb[swz(r4 + 1, jj)], cb[swz(r4 + 2, jj)],
+                                           cb[swz(r4 + 3, jj)]);
+              *reinterpret_cast<float4*>(Cb + (int64_t)mrow * ep.ldc + mcol) = o;
+              if (Lb)
+                *reinterpret_cast<float4*>(Lb + (int64_t)mrow * ep.ld_lo + mcol) =
+                    make_float4(tf32_lo(o.x), tf32_lo(o.y), tf32_lo(o.z), tf32_lo(o.w));
+            }
+          }
           __syncwarp();
         } else {
           // C^T: element (row r = this lane, column j) is stored at column-major block position (j, r)
@@ -612,7 +650,8 @@ bool make_map(CUtensorMap* map, const float* base, int rows, int K, int64_t ld, 
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES, bool PRE, bool CVTA = false, bool TR = false, bool LO = false, bool VEC = false>
+template <int BN, int STAGES, bool PRE, bool CVTA = false, bool TR = false, bool LO = false, bool VEC = false,
+          bool SYM = false>
 cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, int batch, const TcEpilogue& ep,
                    cudaStream_t s, int ksplit = 1) {
   using C = Cfg<BN, STAGES, PRE>;
@@ -630,19 +669,21 @@ cudaError_t launch(const TcOperand& A, const TcOperand& B, int M, int N, int K, 
   const uint64_t bit = (dev >= 0 && dev < 64) ? uint64_t(1) << dev : 0;
   if (bit == 0 || !(attr_set.load(std::memory_order_relaxed) & bit)) {
     cudaError_t e =
-        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO, VEC, SYM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set.fetch_or(bit, std::memory_order_relaxed);
   }
-  const int64_t ntiles = (int64_t)((N + BN - 1) / BN) * ((M + BM - 1) / BM) * batch * ksplit;
+  const int64_t ntm = (M + BM - 1) / BM;
+  const int64_t ntiles = (SYM ? ntm * (ntm + 1) / 2 : (int64_t)((N + BN - 1) / BN) * ntm) * batch * ksplit;
   if (ntiles > (int64_t)1 << 30) return cudaErrorInvalidValue;
-  // short K: a CTA runs several tiles so that the next tile's loads and MMAs overlap the
-  // current epilogue, keeping about four waves of CTAs over the 152 SMs
+  // K up to 2048: a CTA runs several tiles so that the next tile's loads and MMAs overlap the
+  // current epilogue, keeping about four waves of CTAs over the 152 SMs (for longer K the
+  // epilogue is a small part of a tile's time)
   const int kblocks = (K + BK - 1) / BK;
-  const int tpc = kblocks > 16 ? 1 : (int)std::max<int64_t>(1, std::min<int64_t>(8, ntiles / (4 * 152)));
+  const int tpc = kblocks > 64 ? 1 : (int)std::max<int64_t>(1, std::min<int64_t>(8, ntiles / (4 * 152)));
   const int grid = (int)((ntiles + tpc - 1) / tpc);
-  gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO, VEC><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
+  gemm_tc_kernel<BN, STAGES, PRE, CVTA, TR, LO, VEC, SYM><<<grid, C::THREADS, C::SMEM, s>>>(m[0], m[1], m[2], m[3], M, N, K, batch, amod,
                                                                      bmod, tpc, ksplit, ep);
   return cudaGetLastError();
 }
@@ -786,6 +827,29 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
                : tc::launch_tl<32, 5, false, false>(tr, lo, vec, A, B, M, N, K, batch, ep, s);
   return pre ? tc::launch_tl<128, 2, true, false>(tr, lo, vec, A, B, M, N, K, batch, ep, s)
              : tc::launch_tl<128, 3, false, false>(tr, lo, vec, A, B, M, N, K, batch, ep, s);
+}
+
+cudaError_t gemm_tc_syrk(int M, int K, int batch, const TcOperand& A, const TcEpilogue& ep_in, cudaStream_t s,
+                         int family) {
+  if (M <= 0 || batch <= 0) return cudaSuccess;
+  if (batch > 65535) return cudaErrorInvalidValue;
+  auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+  // the symmetric kernel stores row-major C and its lo part with 16-byte stores, both halves
+  const bool ok = ep_in.C && !ep_in.C_ptrs && !ep_in.transpose && ep_in.C_lo && A.lo && al16(ep_in.C) &&
+                  al16(ep_in.C_lo) && (M & 3) == 0 && (ep_in.ldc & 3) == 0 && (ep_in.c_stride & 3) == 0 &&
+                  (ep_in.ld_lo & 3) == 0 && (ep_in.lo_stride & 3) == 0;
+  if (!ok) return gemm_tc_nt(M, M, K, batch, A, A, ep_in, s, family);
+  TcEpilogue ep = ep_in;
+  ep.wait_ns = g_wait_ns.load(std::memory_order_relaxed);
+  ep.hold = g_hold.load(std::memory_order_relaxed);
+  const double ntm = (double)((M + tc::BM - 1) / tc::BM);
+  const double tiles = ntm * (ntm + 1) / 2 * batch;
+  const double flops = 2.0 * tc::BM * tc::BM * (double)K * tiles;  // the lower tiles' products
+  const double bytes = 4.0 * (2.0 * (double)M * K * (A.batch > 0 ? A.batch : batch) +
+                              (double)M * M * batch * ((ep.beta != 0.f ? 1.5 : 1.0) + 1.0));
+  ProfScope prof(family, flops, bytes, s);
+  return ep.beta != 0.f ? tc::launch<128, 2, true, false, false, true, true, true>(A, A, M, M, K, batch, ep, s)
+                        : tc::launch<128, 3, false, false, false, true, true, true>(A, A, M, M, K, batch, ep, s);
 }
 
 }  // namespace soap

@@ -688,27 +688,35 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
 
 // ||P_b||_F: per-chunk partial sums in double (chunks of whole 16-byte units: nn is a
 // multiple of 16), then tol * sqrt(sum)
-constexpr int NORM_CHUNKS = 512;
+constexpr int NORM_CHUNKS = 64;
 
+// Partial sums of squares of P_b over NORM_CHUNKS chunks. The threshold needs ||P||_F to a few
+// digits only, so each thread sums in fp32 (at most a few hundred terms) and the warps' sums are
+// added in fp32 too; the chunks' partial sums are added in double by thresh_kernel.
 __global__ void frob_partial_kernel(const float* P, int64_t nn, double* part) {
   const int b = blockIdx.y;
   const float4* x = reinterpret_cast<const float4*>(P + (int64_t)b * nn);
   const int64_t n4 = nn / 4;
   const int64_t per = (n4 + NORM_CHUNKS - 1) / NORM_CHUNKS;
   const int64_t beg = blockIdx.x * per, end = min(n4, beg + per);
-  double s = 0.0;
+  float s = 0.f;
   for (int64_t i = beg + threadIdx.x; i < end; i += blockDim.x) {
     const float4 v = x[i];
-    s += (double)v.x * v.x + (double)v.y * v.y + (double)v.z * v.z + (double)v.w * v.w;
+    s = fmaf(v.x, v.x, s);
+    s = fmaf(v.y, v.y, s);
+    s = fmaf(v.z, v.z, s);
+    s = fmaf(v.w, v.w, s);
   }
-  __shared__ double red[256];
-  red[threadIdx.x] = s;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  __shared__ float red[8];
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
   __syncthreads();
-  for (int o = 128; o > 0; o >>= 1) {
-    if ((int)threadIdx.x < o) red[threadIdx.x] += red[threadIdx.x + o];
-    __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+    part[(int64_t)b * NORM_CHUNKS + blockIdx.x] = t;
   }
-  if (threadIdx.x == 0) part[(int64_t)b * NORM_CHUNKS + blockIdx.x] = red[0];
 }
 
 __global__ void thresh_kernel(const double* part, float tol, int batch, float* thresh) {

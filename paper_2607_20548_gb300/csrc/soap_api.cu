@@ -177,7 +177,9 @@ struct Wave {
   std::vector<std::vector<int>> fork_after;  // per slice: groups whose last feeding slice it is
   std::vector<std::vector<int>> groups_of;   // per slice: the groups its bases come from
   std::vector<QrGroup> groups;
-  size_t bytes = 0;  // arena bytes the wave uses
+  size_t bytes = 0;    // arena bytes the wave uses
+  size_t base = 0;     // where its half of the arena starts (waves alternate between two halves)
+  int slot_base = 0;   // its groups' stream pairs are slots slot_base + g.slot
 };
 
 // Streams and events of one QR group slot (reused by every wave).
@@ -212,6 +214,7 @@ struct soap_s {
   std::vector<std::pair<int, int>> loc;  // matrix index -> (class, slot)
   std::vector<ClassState> classes;
   std::vector<Wave> waves;
+  bool pipelined = false;  // waves alternate between two halves of the arena
   std::vector<GroupStreams> slots;
   char* arena = nullptr;  // workspace of one wave at a time
   size_t arena_bytes = 0;
@@ -311,9 +314,9 @@ soap::TcEpilogue epi(soap_handle h, float* C, int64_t ldc, int64_t c_stride, flo
   return soap::TcEpilogue{C, nullptr, ldc, c_stride, C_lo, ldc, c_stride, transpose, alpha, beta, h->d_status};
 }
 
-View view_of(soap_handle h, const Slice& sl) {
+View view_of(soap_handle h, const Wave& w, const Slice& sl) {
   View v;
-  make_view(h->classes[sl.cls], sl.cls, sl.first, sl.count, h->arena + sl.off, &v);
+  make_view(h->classes[sl.cls], sl.cls, sl.first, sl.count, h->arena + w.base + sl.off, &v);
   return v;
 }
 
@@ -406,17 +409,16 @@ soap_status_t accumulate_factors(soap_handle h, const ClassState& c, const View&
     SOAP_CUDA(h, soap::gemm_tc_nt(n, m, m, B, opnd(v.Gt, v.Gt_lo, m, mn, B), opnd(v.QLt, v.QLt_lo, m, mm, B),
                                   epi(h, X, m, mn, nullptr, 0, 1.f, 0.f), s));
     SOAP_CUDA(h, soap::scale_cols_split(X, X_lo, v.lamL, n, m, B, (float)((1.0 - fb) / m), hp.eps, s));
-    SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(Y, Y_lo, n, mn, B), opnd(Y, Y_lo, n, mn, B),
-                                  epi(h, v.Lf, m, mm, v.Lf_lo, 0, 1.f, fb), s));
-    SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(X, X_lo, m, mn, B), opnd(X, X_lo, m, mn, B),
-                                  epi(h, v.Rf, n, nn, v.Rf_lo, 0, 1.f, fb), s));
+    SOAP_CUDA(h, soap::gemm_tc_syrk(m, n, B, opnd(Y, Y_lo, n, mn, B), epi(h, v.Lf, m, mm, v.Lf_lo, 0, 1.f, fb), s));
+    SOAP_CUDA(h, soap::gemm_tc_syrk(n, m, B, opnd(X, X_lo, m, mn, B), epi(h, v.Rf, n, nn, v.Rf_lo, 0, 1.f, fb), s));
   } else {
+    // S1 as symmetric products: the lower tiles of G G^T (G^T G), mirrored
     if (c.left)
-      SOAP_CUDA(h, soap::gemm_tc_nt(m, m, n, B, opnd(v.Gc, v.Gc_lo, n, mn, B), opnd(v.Gc, v.Gc_lo, n, mn, B),
-                                    epi(h, v.Lf, m, mm, v.Lf_lo, 0, aL, fb), s));
+      SOAP_CUDA(h, soap::gemm_tc_syrk(m, n, B, opnd(v.Gc, v.Gc_lo, n, mn, B), epi(h, v.Lf, m, mm, v.Lf_lo, 0, aL, fb),
+                                      s));
     if (c.right)
-      SOAP_CUDA(h, soap::gemm_tc_nt(n, n, m, B, opnd(v.Gt, v.Gt_lo, m, mn, B), opnd(v.Gt, v.Gt_lo, m, mn, B),
-                                    epi(h, v.Rf, n, nn, v.Rf_lo, 0, aR, fb), s));
+      SOAP_CUDA(h, soap::gemm_tc_syrk(n, m, B, opnd(v.Gt, v.Gt_lo, m, mn, B), epi(h, v.Rf, n, nn, v.Rf_lo, 0, aR, fb),
+                                      s));
   }
   if (c.left) SOAP_CUDA(h, soap::pack_sym(v.Lf, v.L, m, B, s));
   if (c.right) SOAP_CUDA(h, soap::pack_sym(v.Rf, v.R, n, B, s));
@@ -432,19 +434,19 @@ soap_status_t refresh_group(soap_handle h, const Wave& w, const QrGroup& g, cuda
   const soap_hparams& hp = h->hp;
   using soap::strided;
   using soap::strided_mut;
-  GroupStreams& gs = h->slots[g.slot];
+  GroupStreams& gs = h->slots[w.slot_base + g.slot];
   SOAP_CUDA(h, cudaEventRecord(gs.fork, s));
   SOAP_CUDA(h, cudaStreamWaitEvent(gs.stream, gs.fork, 0));
   const int n = g.n;
   const int64_t nn = (int64_t)n * n;
-  void* ws = h->arena + g.ws_off;
-  uint8_t* skip = reinterpret_cast<uint8_t*>(h->arena + g.skip_off);
+  void* ws = h->arena + w.base + g.ws_off;
+  uint8_t* skip = reinterpret_cast<uint8_t*>(h->arena + w.base + g.skip_off);
   float* At;
   soap::qr_input_buffers(ws, n, g.batch, &At);
   for (const QrJob& j : g.jobs) {
     const Slice& sl = w.slices[j.slice];
     const ClassState& c = h->classes[sl.cls];
-    const View v = view_of(h, sl);
+    const View v = view_of(h, w, sl);
     float* at = At + (int64_t)j.offset * nn;
     if (c.tc) {
       SOAP_CUDA(h, soap::gemm_tc_nt(n, n, n, v.count, opnd(j.left ? v.QLt : v.QRt, j.left ? v.QLt_lo : v.QRt_lo, n, nn,
@@ -463,7 +465,7 @@ soap_status_t refresh_group(soap_handle h, const Wave& w, const QrGroup& g, cuda
   for (const QrJob& j : g.jobs) {
     const Slice& sl = w.slices[j.slice];
     const ClassState& c = h->classes[sl.cls];
-    const View v = view_of(h, sl);
+    const View v = view_of(h, w, sl);
     const float* qt = At + (int64_t)j.offset * nn;
     float* Q = j.left ? v.QL : v.QR;
     if (c.tc)
@@ -669,7 +671,9 @@ constexpr int kMaxSlice = 32767;
 
 // Cuts the classes into waves whose workspace (arena + rotation intermediates) fits `budget`
 // bytes. Returns false if some class cannot fit even one matrix.
-bool plan_waves(soap_handle h, size_t budget, bool single_ok, std::vector<Wave>* out, RotSizes* rot) {
+bool plan_waves(soap_handle h, size_t budget, bool single_ok, std::vector<Wave>* out, RotSizes* rot,
+                bool* pipelined) {
+  *pipelined = false;
   const int nc = (int)h->classes.size();
   std::vector<int> order(nc);
   for (int ci = 0; ci < nc; ++ci) order[ci] = ci;
@@ -704,34 +708,51 @@ bool plan_waves(soap_handle h, size_t budget, bool single_ok, std::vector<Wave>*
     if (c.right) b += soap::qr_workspace_bytes((int)c.cols, 1, true) + (size_t)c.cols + 64 * 256;
     return b + 8 * 256;
   };
-  std::vector<Wave> waves;
-  Wave cur;
-  size_t used = 0;
-  for (int ci : order) {
-    const ClassState& c = h->classes[ci];
-    const size_t pm = per_matrix(c);
-    if (pm > budget) return false;
-    int first = 0;
-    while (first < c.count) {
-      int k = (int)std::min<size_t>((size_t)(c.count - first), (budget - used) / pm);
-      k = std::min(k, kMaxSlice);
-      if (k <= 0) {
-        waves.push_back(cur);
-        cur = Wave();
-        used = 0;
-        continue;
+  auto cut = [&](size_t wave_budget, std::vector<Wave>* waves) -> bool {
+    waves->clear();
+    Wave cur;
+    size_t used = 0;
+    for (int ci : order) {
+      const ClassState& c = h->classes[ci];
+      const size_t pm = per_matrix(c);
+      if (pm > wave_budget) return false;
+      int first = 0;
+      while (first < c.count) {
+        int k = (int)std::min<size_t>((size_t)(c.count - first), (wave_budget - used) / pm);
+        k = std::min(k, kMaxSlice);
+        if (k <= 0) {
+          waves->push_back(cur);
+          cur = Wave();
+          used = 0;
+          continue;
+        }
+        cur.slices.push_back(Slice{ci, first, k, 0});
+        used += (size_t)k * pm;
+        first += k;
       }
-      cur.slices.push_back(Slice{ci, first, k, 0});
-      used += (size_t)k * pm;
-      first += k;
     }
-  }
-  if (!cur.slices.empty()) waves.push_back(cur);
+    if (!cur.slices.empty()) waves->push_back(cur);
+    return true;
+  };
+  // Waves are pipelined where the budget allows (a wave's preparation and factor update run while
+  // the previous wave's QR does): two waves hold the arena at a time, each in its half; else they
+  // run one after another in the whole budget.
+  std::vector<Wave> waves;
+  *pipelined = cut(budget / 2, &waves) && waves.size() > 1;
+  if (!*pipelined && !cut(budget, &waves)) return false;
   RotSizes r;
+  size_t half = 0, groups = 0;
   for (Wave& w : waves) {
     layout_wave(h, w);
+    half = std::max(half, align256(w.bytes));
+    groups = std::max(groups, w.groups.size());
     for (const Slice& sl : w.slices) r.grow(rot_sizes(h->classes[sl.cls], sl.count, kl));
   }
+  if (*pipelined)
+    for (size_t wi = 0; wi < waves.size(); ++wi) {
+      waves[wi].base = (wi & 1) ? half : 0;
+      waves[wi].slot_base = (wi & 1) ? (int)groups : 0;
+    }
   *out = waves;
   *rot = r;
   return true;
@@ -855,14 +876,15 @@ soap_status_t soap_create_ex(const soap_shape* shapes, int32_t n, const soap_hpa
     const size_t reserve = (size_t(1) << 30) + total_b / 100;
     const size_t avail = free_b > reserve ? free_b - reserve : 0;
     const size_t budget = workspace_limit ? std::min(workspace_limit, avail) : avail;
-    if (e == cudaSuccess && !plan_waves(h, budget, true, &h->waves, &rot)) e = cudaErrorMemoryAllocation;
+    if (e == cudaSuccess && !plan_waves(h, budget, true, &h->waves, &rot, &h->pipelined))
+      e = cudaErrorMemoryAllocation;
   }
   if (e == cudaSuccess) {
-    for (const Wave& w : h->waves) h->arena_bytes = std::max(h->arena_bytes, w.bytes);
+    for (const Wave& w : h->waves) h->arena_bytes = std::max(h->arena_bytes, w.base + w.bytes);
     e = dalloc(h, (void**)&h->arena, h->arena_bytes);
   }
   size_t nslots = 0;
-  for (const Wave& w : h->waves) nslots = std::max(nslots, w.groups.size());
+  for (const Wave& w : h->waves) nslots = std::max(nslots, (size_t)w.slot_base + w.groups.size());
   h->slots.resize(nslots);
   for (GroupStreams& gs : h->slots) {
     // the panel chain is latency-bound: its stream goes first when SMs free up
@@ -932,9 +954,11 @@ soap_status_t soap_create(const soap_shape* shapes, int32_t n, const soap_hparam
   return soap_create_ex(shapes, n, hp, device, 0, out);
 }
 
-soap_status_t soap_plan_info(soap_handle h, int32_t* waves, size_t* workspace_bytes, size_t* state_bytes) {
+soap_status_t soap_plan_info(soap_handle h, int32_t* waves, int32_t* pipelined, size_t* workspace_bytes,
+                             size_t* state_bytes) {
   if (!h) return SOAP_ERR_INVALID_ARG;
   if (waves) *waves = (int32_t)h->waves.size();
+  if (pipelined) *pipelined = h->pipelined ? 1 : 0;
   if (workspace_bytes) *workspace_bytes = h->arena_bytes + h->rot_bytes;
   if (state_bytes) *state_bytes = h->state_bytes;
   return SOAP_OK;
@@ -995,17 +1019,20 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
     const ClassState& c = h->classes[sl.cls];
     return reinterpret_cast<const float* const*>(h->d_ptrs + c.ptr_offset + c.count + sl.first);
   };
-  // Wave by wave: phase A slice by slice, each size group's refresh forked as soon as the last
+  // Per wave: phase A slice by slice, each size group's refresh forked as soon as the last
   // slice feeding it is prepared (slices with the largest factors first, so the longest refresh
   // starts earliest); phase C slice by slice, each waiting only for the groups its bases come
-  // from (slices with the smallest factors first, whose refreshes finish earliest). Every group
-  // is joined before the next wave reuses the workspace. The stale variant refreshes from the
-  // factors as they stand and accumulates G_t into them after the wave's updates.
-  for (const Wave& w : h->waves) {
+  // from (slices with the smallest factors first, whose refreshes finish earliest). Pipelined
+  // waves run on the caller's stream as A0, A1, C0, A2, C1, ...: the next wave's preparation
+  // and factor update run while this wave's QR does, in the other half of the arena; a wave
+  // reuses a half only after the wave before it in that half has finished (its phase C, which
+  // joined its groups, precedes on the stream). The stale variant refreshes from the factors
+  // as they stand and accumulates G_t into them after the wave's updates.
+  auto phase_a = [&](const Wave& w) -> soap_status_t {
     for (int si : w.prep_order) {
       const Slice& sl = w.slices[si];
       const ClassState& c = h->classes[sl.cls];
-      const View v = view_of(h, sl);
+      const View v = view_of(h, w, sl);
       soap_status_t st = prepare(h, c, v, grads_of(sl), s);
       if (st == SOAP_OK && !hp.stale) st = accumulate_factors(h, c, v, s);
       if (st != SOAP_OK) return st;
@@ -1015,25 +1042,45 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
           if (st != SOAP_OK) return st;
         }
     }
+    return SOAP_OK;
+  };
+  auto phase_c = [&](const Wave& w) -> soap_status_t {
     std::vector<bool> joined(w.groups.size(), !refresh);
     for (int si : w.update_order) {
       for (int gi : w.groups_of[si])
         if (!joined[gi]) {
-          SOAP_CUDA(h, cudaStreamWaitEvent(s, h->slots[w.groups[gi].slot].done, 0));
+          SOAP_CUDA(h, cudaStreamWaitEvent(s, h->slots[w.slot_base + w.groups[gi].slot].done, 0));
           joined[gi] = true;
         }
       const Slice& sl = w.slices[si];
-      soap_status_t st = rotate_update(h, h->classes[sl.cls], view_of(h, sl), params_of(sl), bc1, bc2, s);
+      soap_status_t st = rotate_update(h, h->classes[sl.cls], view_of(h, w, sl), params_of(sl), bc1, bc2, s);
       if (st != SOAP_OK) return st;
     }
     for (size_t gi = 0; gi < w.groups.size(); ++gi)
-      if (!joined[gi]) SOAP_CUDA(h, cudaStreamWaitEvent(s, h->slots[w.groups[gi].slot].done, 0));
+      if (!joined[gi]) SOAP_CUDA(h, cudaStreamWaitEvent(s, h->slots[w.slot_base + w.groups[gi].slot].done, 0));
     if (hp.stale)
       for (int si : w.prep_order) {
         const Slice& sl = w.slices[si];
-        soap_status_t st = accumulate_factors(h, h->classes[sl.cls], view_of(h, sl), s);
+        soap_status_t st = accumulate_factors(h, h->classes[sl.cls], view_of(h, w, sl), s);
         if (st != SOAP_OK) return st;
       }
+    return SOAP_OK;
+  };
+  const size_t nw = h->waves.size();
+  if (h->pipelined) {
+    soap_status_t st = phase_a(h->waves[0]);
+    if (st != SOAP_OK) return st;
+    for (size_t wi = 0; wi < nw; ++wi) {
+      st = wi + 1 < nw ? phase_a(h->waves[wi + 1]) : SOAP_OK;
+      if (st == SOAP_OK) st = phase_c(h->waves[wi]);
+      if (st != SOAP_OK) return st;
+    }
+  } else {
+    for (size_t wi = 0; wi < nw; ++wi) {
+      soap_status_t st = phase_a(h->waves[wi]);
+      if (st == SOAP_OK) st = phase_c(h->waves[wi]);
+      if (st != SOAP_OK) return st;
+    }
   }
   SOAP_CUDA(h, cudaMemcpyAsync(h->h_status, h->d_status, sizeof(int), cudaMemcpyDeviceToHost, s));
   SOAP_CUDA(h, cudaEventRecord(h->status_ev, s));

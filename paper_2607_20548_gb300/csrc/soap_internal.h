@@ -84,6 +84,11 @@ cudaError_t gemm_tc_nt(int M, int N, int K, int batch, const TcOperand& A, const
 // Bound of the tensor-core products' device waits (0: 2 s) and, for testing the timeout path, a
 // device flag their epilogues first wait for (nullptr: none); applies to later launches.
 void set_wait_limit(uint64_t ns, const int* hold);
+// Symmetric product C_b = alpha A_b A_b^T + beta C_b (M x M, A_b M x K): only the 128 x 128 tiles on
+// or below the diagonal are computed, each below it also stored (with its lo part) in the mirror
+// position. Needs a row-major, 16-byte aligned C with its lo part; other forms go to gemm_tc_nt.
+cudaError_t gemm_tc_syrk(int M, int K, int batch, const TcOperand& A, const TcEpilogue& ep, cudaStream_t stream,
+                         int family = kFamGemmTc);
 // hi = trunc_tf32(x), lo = x - hi (exact), elementwise over n values.
 cudaError_t split_tf32(const float* x, float* hi, float* lo, int64_t n, cudaStream_t stream);
 

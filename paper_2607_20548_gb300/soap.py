@@ -88,7 +88,8 @@ def load_library(path: str = LIB_PATH):
         "soap_create": (I32, [ctypes.POINTER(soap_shape), I32, ctypes.POINTER(soap_hparams), I32, ctypes.POINTER(P)]),
         "soap_create_ex": (I32, [ctypes.POINTER(soap_shape), I32, ctypes.POINTER(soap_hparams), I32, SZ,
                                  ctypes.POINTER(P)]),
-        "soap_plan_info": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(SZ), ctypes.POINTER(SZ)]),
+        "soap_plan_info": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(I32), ctypes.POINTER(SZ),
+                                 ctypes.POINTER(SZ)]),
         "soap_step": (I32, [P, P, P, P]),
         "soap_set_lr": (I32, [P, F, F]),
         "soap_state_bytes": (SZ, [P, I32, I32]),
@@ -229,11 +230,11 @@ class SoapOptimizer:
         _check(load_library().soap_step(self._handle(), self._pp, self._gp, _stream(stream, self.device)), self._h)
 
     def plan_info(self) -> dict:
-        """soap_plan_info: waves per step, workspace and state bytes."""
-        w, ws, st = ctypes.c_int32(0), ctypes.c_size_t(0), ctypes.c_size_t(0)
-        _check(load_library().soap_plan_info(self._handle(), ctypes.byref(w), ctypes.byref(ws), ctypes.byref(st)),
-               self._h)
-        return {"waves": w.value, "workspace_bytes": ws.value, "state_bytes": st.value}
+        """soap_plan_info: waves per step, whether they are pipelined, workspace and state bytes."""
+        w, pl, ws, st = ctypes.c_int32(0), ctypes.c_int32(0), ctypes.c_size_t(0), ctypes.c_size_t(0)
+        _check(load_library().soap_plan_info(self._handle(), ctypes.byref(w), ctypes.byref(pl), ctypes.byref(ws),
+                                             ctypes.byref(st)), self._h)
+        return {"waves": w.value, "pipelined": bool(pl.value), "workspace_bytes": ws.value, "state_bytes": st.value}
 
     def set_lr(self, lr: float, weight_decay: float):
         _check(load_library().soap_set_lr(self._handle(), lr, weight_decay), self._h)

@@ -62,6 +62,13 @@ def adam_direction(m, v, hp, t, skipL=None, skipR=None):
     return N
 
 
+def numerical_rank(F, rel_tol=1e-12):
+    """Rank of a symmetric PSD factor in fp64: eigenvalues above rel_tol * the largest (fp64
+    rounding of an exactly rank-deficient factor leaves ~1e-16 of it)."""
+    lam = np.linalg.eigvalsh(np.asarray(F, np.float64))
+    return int((lam > rel_tol * max(lam.max(), 0.0)).sum()) if lam.size else 0
+
+
 def masked_update(QL, N, QR, mask):
     """Q_L (N o mask) Q_R^T in fp64 (an identity side: Q = None)."""
     X = np.where(mask, N, 0.0)
@@ -149,6 +156,7 @@ class TeacherForcedCheck:
             row["twin_L"] = rel(st32.L, st64.L)
             skL = g(S.STATE_SKIP_L).astype(bool)
             row["skipL_same"] = bool(np.array_equal(skL, st64.skipL))
+            row["zeroed_L"], row["rank_L"] = int(skL.sum()), numerical_rank(st64.L)
             row["orth_L"] = orth_err(self.opt.state_get(idx, S.STATE_QL))
         if sp.right:
             QR = g(S.STATE_QR).astype(np.float64)
@@ -156,6 +164,7 @@ class TeacherForcedCheck:
             row["twin_R"] = rel(st32.R, st64.R)
             skR = g(S.STATE_SKIP_R).astype(bool)
             row["skipR_same"] = bool(np.array_equal(skR, st64.skipR))
+            row["zeroed_R"], row["rank_R"] = int(skR.sum()), numerical_rank(st64.R)
             row["orth_R"] = orth_err(self.opt.state_get(idx, S.STATE_QR))
         # the GPU's own direction N from its m, v and zero-column flags
         N = adam_direction(m_gpu, v_gpu, hp, t, skL, skR)
@@ -182,8 +191,11 @@ class TeacherForcedCheck:
         for r in self.rows:
             tag = (f"  [whole update beyond fp32 resolution; on Adam's normal range gpu {r['e_mask']:.1e} "
                    f"twin {r['e_mask_twin']:.1e}, {r['amplified']} amplified entries]") if r["ill"] else ""
+            zero = "".join(f" zeroed {side} {r['zeroed_' + side]} (fp64 rank {r['rank_' + side]})"
+                           for side in ("L", "R") if "zeroed_" + side in r)
             out.append(f"matrix {r['idx']:4d} step {r['t']:3d}: gpu {r['e_gpu']:.2e} twin {r['e_twin']:.2e} "
-                       f"max|N| {r['max_abs_N']:.0f} m {r['e_m']:.1e} v {r['e_v']:.1e} self {r['e_self']:.1e}{tag}")
+                       f"max|N| {r['max_abs_N']:.0f} m {r['e_m']:.1e} v {r['e_v']:.1e} self {r['e_self']:.1e}"
+                       f"{zero}{tag}")
         return "\n".join(out)
 
     def assert_ok(self, state_tol=1e-4):

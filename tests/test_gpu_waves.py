@@ -27,25 +27,37 @@ def _inputs(cuda, steps, seed=17):
     return W, Gs
 
 
-def _limit_for_waves(cuda, hp):
-    """A workspace bound that fits a few matrices at a time (measured from a one-wave plan)."""
+def _limit_for_waves(cuda, hp, pipelined):
+    """A workspace bound under which the model takes at least 3 waves, pipelined (two waves in
+    halves of the workspace) or one after another: found by shrinking the one-wave plan's size."""
     probe = S.SoapOptimizer(SHAPES, hp)
     info = probe.plan_info()
     probe.destroy()
     assert info["waves"] == 1
-    return info["workspace_bytes"] // 5
+    for divisor in (2.5, 3, 4, 5, 6, 8, 10, 12, 16, 20, 24, 32):
+        limit = int(info["workspace_bytes"] / divisor)
+        try:
+            opt = S.SoapOptimizer(SHAPES, hp, workspace_limit=limit)
+        except S.SoapError:
+            break
+        plan = opt.plan_info()
+        opt.destroy()
+        if plan["waves"] >= 3 and plan["pipelined"] == pipelined:
+            return limit
+    pytest.fail(f"no workspace limit gives >= 3 {'pipelined' if pipelined else 'serial'} waves")
 
 
+@pytest.mark.parametrize("pipelined", [True, False])
 @pytest.mark.parametrize("variant", [dict(), dict(kl=1), dict(stale=1, guard=0), dict(eig_every=2)])
-def test_waves_match_one_wave(cuda, variant):
+def test_waves_match_one_wave(cuda, variant, pipelined):
     hp = S.default_hparams(**variant)
     steps = 5
     W0, Gs = _inputs(cuda, steps)
     one = S.SoapOptimizer(SHAPES, hp)
-    many = S.SoapOptimizer(SHAPES, hp, workspace_limit=_limit_for_waves(cuda, hp))
+    many = S.SoapOptimizer(SHAPES, hp, workspace_limit=_limit_for_waves(cuda, hp, pipelined))
     info = many.plan_info()
     print(f"\nplan: {info}")
-    assert info["waves"] >= 3
+    assert info["waves"] >= 3 and info["pipelined"] == pipelined
     Wa = [w.clone() for w in W0]
     Wb = [w.clone() for w in W0]
     for t in range(steps):
@@ -73,8 +85,8 @@ def test_waves_against_oracle(cuda):
     hp = S.default_hparams()
     steps = 6
     W, Gs = _inputs(cuda, steps, seed=23)
-    opt = S.SoapOptimizer(SHAPES, hp, workspace_limit=_limit_for_waves(cuda, hp))
-    assert opt.plan_info()["waves"] >= 3
+    opt = S.SoapOptimizer(SHAPES, hp, workspace_limit=_limit_for_waves(cuda, hp, True))
+    assert opt.plan_info()["waves"] >= 3 and opt.plan_info()["pipelined"]
     chk = TeacherForcedCheck(opt, oracle_hparams(hp))
     sample = [0, 4, 5, 8, 10, 12, 15]
     for t in range(steps):
