@@ -160,12 +160,12 @@ TC_PRODUCTS = 4
 # profiles/peaks_gb300.md. The driver's MEASURED_PEAKS.json has the bf16 and HBM figures only.
 TF32_TFLOPS = {"burst": 1047.2, "sustained": 951.8}
 
-# DRAM bytes (ncu dram__bytes_read.sum + dram__bytes_write.sum) per algorithmic byte of each
-# kernel family, measured with ncu over one step of the block's 2048x8192 matrix alone
-# (both of its QR sizes) for the current kernels. The QR products read their small operands
-# from L2 across tiles and write split-K partial sums (ratio about 1); the large contractions
-# re-read operand panels (ratio > 1); the panel kernel keeps its panel on chip.
-TRAFFIC_PER_ALGORITHMIC_BYTE = {"qr_update": 1.059, "qr_panel": 0.383, "gemm_tc": 1.617}
+# DRAM bytes (ncu dram__bytes_read.sum + dram__bytes_write.sum) per algorithmic byte, from one
+# full capture of each family's representative launch (profiles/): the QR's K = 128 trailing
+# update of an 8192 factor (0.89) and the power step of an 8192 factor, whose operand panels are
+# re-read across tiles (5.1). Applied to a family's average algorithmic bytes per launch, the
+# mixed launches of a family make it an estimate; the other families have no current capture.
+TRAFFIC_PER_ALGORITHMIC_BYTE = {"qr_update": 0.89, "gemm_tc": 5.12}
 
 
 def roofline(family, st, peaks, peak_src, products=None, dtype_ratio=2.0):

@@ -483,7 +483,7 @@ cudaError_t transpose(const float* src, float* dst, int rows, int cols, int batc
 cudaError_t basis_split(const float* Q, float* Q_lo, float* Qt, float* Qt_lo, int n, int batch, cudaStream_t s) {
   if (n <= 0 || batch <= 0) return cudaSuccess;
   const double e = (double)n * n * batch;
-  ProfScope prof(kFamElementwise, 2.0 * e, 16.0 * e, s);
+  ProfScope prof(kFamElementwise, 2.0 * e, (Q_lo ? 16.0 : 12.0) * e, s);
   dim3 grid((n + 31) / 32, (n + 31) / 32, batch);
   basis_split_kernel<<<grid, dim3(32, 8), 0, s>>>(Q, Q_lo, Qt, Qt_lo, n);
   return cudaGetLastError();

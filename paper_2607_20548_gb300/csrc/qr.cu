@@ -783,7 +783,9 @@ cudaError_t prepare_panel(PanelKernel* pk, bool wide) {
 // 16 x 512 positions where the device can place them, 2 = clusters of 8 x 1024.
 std::atomic<int> g_panel_choice[64];
 
-cudaError_t panel_kernel(PanelKernel* pk) {
+cudaError_t panel_kernel(PanelKernel* pk, int n) {
+  // a factor of at most 1024 rows fits one CTA's 1024 positions: no cluster barrier per column
+  if (n <= 1024) return prepare_panel<1024>(pk, false);
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) dev = 0;
   std::atomic<int>* slot = dev < 64 ? &g_panel_choice[dev] : nullptr;
@@ -936,7 +938,7 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     thresh_kernel<<<(batch + 127) / 128, 128, 0, s>>>(w.part, tol, batch, w.thresh);
   }
   PanelKernel pk;
-  e = panel_kernel(&pk);
+  e = panel_kernel(&pk, n);
   if (e != cudaSuccess) return e;
 
   if (la) {

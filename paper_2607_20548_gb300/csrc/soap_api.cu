@@ -337,7 +337,8 @@ View view_of(soap_handle h, const Wave& w, const Slice& sl) {
 // One-sided slices take the same route with one rotation on each side of Adam (a left-only
 // class as the right-only problem of G^T). Classes whose rows or columns are not a multiple
 // of 4 (rows of an operand must be 16-byte multiples for TMA) run on CUDA cores.
-soap_status_t prepare(soap_handle h, const ClassState& c, const View& v, const float* const* d_grads, cudaStream_t s) {
+soap_status_t prepare(soap_handle h, const ClassState& c, const View& v, const float* const* d_grads, bool refresh,
+                      cudaStream_t s) {
   const soap_hparams& hp = h->hp;
   const int B = v.count, m = (int)c.rows, n = (int)c.cols;
   const int64_t mn = (int64_t)m * n;
@@ -350,12 +351,14 @@ soap_status_t prepare(soap_handle h, const ClassState& c, const View& v, const f
   // the factors' lo parts are read before S1 rewrites them by the KL form's eigenvalue product
   // and by the stale variant's refresh
   const bool lo = hp.kl || hp.stale;
+  // Q^T and its lo part feed S2 (and the KL eigenvalues); Q's own lo part only the rotations,
+  // for which a refresh writes it anew
   if (c.left) {
-    SOAP_CUDA(h, soap::basis_split(v.QL, v.QL_lo, v.QLt, v.QLt_lo, m, B, s));
+    SOAP_CUDA(h, soap::basis_split(v.QL, refresh ? nullptr : v.QL_lo, v.QLt, v.QLt_lo, m, B, s));
     SOAP_CUDA(h, soap::unpack_sym(v.L, v.Lf, lo ? v.Lf_lo : nullptr, m, B, s));
   }
   if (c.right) {
-    SOAP_CUDA(h, soap::basis_split(v.QR, v.QR_lo, v.QRt, v.QRt_lo, n, B, s));
+    SOAP_CUDA(h, soap::basis_split(v.QR, refresh ? nullptr : v.QR_lo, v.QRt, v.QRt_lo, n, B, s));
     SOAP_CUDA(h, soap::unpack_sym(v.R, v.Rf, lo ? v.Rf_lo : nullptr, n, B, s));
   }
   return SOAP_OK;
@@ -1033,7 +1036,7 @@ soap_status_t soap_step(soap_handle h, float* const* params, const float* const*
       const Slice& sl = w.slices[si];
       const ClassState& c = h->classes[sl.cls];
       const View v = view_of(h, w, sl);
-      soap_status_t st = prepare(h, c, v, grads_of(sl), s);
+      soap_status_t st = prepare(h, c, v, grads_of(sl), refresh, s);
       if (st == SOAP_OK && !hp.stale) st = accumulate_factors(h, c, v, s);
       if (st != SOAP_OK) return st;
       if (refresh)
