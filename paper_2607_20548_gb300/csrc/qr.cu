@@ -719,11 +719,14 @@ __global__ void frob_partial_kernel(const float* P, int64_t nn, double* part) {
   }
 }
 
-__global__ void thresh_kernel(const double* part, float tol, int batch, float* thresh) {
+// The zero-column threshold tol * ||P_b||_F; a non-finite norm (a NaN or Inf anywhere in P_b,
+// wherever the Householder steps would meet it) is a breakdown of that QR.
+__global__ void thresh_kernel(const double* part, float tol, int batch, float* thresh, int* status) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= batch) return;
   double s = 0.0;
   for (int i = 0; i < NORM_CHUNKS; ++i) s += part[(int64_t)b * NORM_CHUNKS + i];
+  if (!isfinite(s) && status) atomicOr(status, kStatusQrBreakdown);
   thresh[b] = (float)((double)tol * sqrt(s));
 }
 
@@ -935,7 +938,7 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
   }
   {
     ProfScope prof(kFamOther, 0, 8.0 * NORM_CHUNKS * batch, s);
-    thresh_kernel<<<(batch + 127) / 128, 128, 0, s>>>(w.part, tol, batch, w.thresh);
+    thresh_kernel<<<(batch + 127) / 128, 128, 0, s>>>(w.part, tol, batch, w.thresh, status);
   }
   PanelKernel pk;
   e = panel_kernel(&pk, n);
