@@ -585,6 +585,16 @@ def run_soap(args):
     if opt.status() != 0:
         raise RuntimeError("device status after timed steps: " + opt.last_error())
     del host_pool, host_w
+    # one more step (outside the timed regions) with every launch timed alone: each starts on an
+    # idle device, so the per-family rates are the kernels' own, without the contention of the
+    # library's concurrent QR streams that the live figures include
+    iso = None
+    if not (muon or layerwise):
+        opt.profile_begin(max(1024, per_step + 1024), serial=True)
+        opt.step(W, grads_for(base + args.steps))
+        iso = {k: v for k, v in opt.profile_end().items() if k != "overflow"}
+        if opt.status() != 0:
+            raise RuntimeError("device status after the isolated step: " + opt.last_error())
 
     if rank != 0:
         opt.destroy()
@@ -602,6 +612,12 @@ def run_soap(args):
     if muon:
         # the DRAM/algorithmic ratios above were measured for the fp32 (tf32 x4) kernels
         roof["traffic"], roof["traffic_note"] = None, "not measured for the bf16 kernel"
+    if iso and iso.get(top, {}).get("launches"):
+        r = roofline(top, iso[top], peaks, peak_src)
+        roof["isolated"] = {k: r[k] for k in ("bound", "achieved", "peak", "unit", "frac", "avg_launch_us")}
+        roof["isolated"]["note"] = ("one further step with each launch timed alone (the device idle when it starts): "
+                                    "the kernel's own rate; the figures above are live, beside the concurrent "
+                                    "QR streams")
     opt.destroy()
     del Wg, pool, W, grads_seq
     torch.cuda.empty_cache()
@@ -647,6 +663,10 @@ def run_soap(args):
                                 "tflops": v["flops"] / max(1e-12, v["ms"] / 1e3) / 1e12,
                                 "gbs": v["bytes"] / max(1e-12, v["ms"] / 1e3) / 1e9}
                             for k, v in fams.items() if v["launches"]},
+        "kernel_families_isolated": {k: {"ms_per_step": v["ms"], "launches_per_step": v["launches"],
+                                         "tflops": v["flops"] / max(1e-12, v["ms"] / 1e3) / 1e12,
+                                         "gbs": v["bytes"] / max(1e-12, v["ms"] / 1e3) / 1e9}
+                                     for k, v in iso.items() if v["launches"]} if iso else None,
         "cpu_baseline": {"value": sps, "unit": "steps/s", "cores": threads, "kind": "oracle", "sample": cpu_desc},
         "e2e": {"value": units * args.steps / e2e_s, "unit": "steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},

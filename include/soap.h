@@ -217,17 +217,27 @@ typedef struct {
  * launch is bracketed by two CUDA events on its own stream. */
 soap_status_t soap_profile_begin(soap_handle h, int64_t max_launches);
 
+/* soap_profile_begin with flags. SOAP_PROFILE_SERIAL makes every timed launch wait for the
+ * device to be idle before it starts (a host-side device synchronisation), so that each
+ * launch runs alone and its time measures the kernel in isolation rather than beside the
+ * library's concurrent streams; a step timed this way runs slower as a whole. */
+#define SOAP_PROFILE_SERIAL 1
+soap_status_t soap_profile_begin_ex(soap_handle h, int64_t max_launches, int32_t flags);
+
 /* Synchronises `stream`, stops timing and writes one soap_kernel_stats per family
  * (6 entries) to out[]. *overflow is set to 1 if max_launches was exceeded. */
 soap_status_t soap_profile_end(soap_handle h, soap_stream_t stream, soap_kernel_stats* out,
                                int32_t* overflow);
 
-/* One timed launch: its family and its start and end, in ms after the first timed launch
- * started (CUDA events on the launch's stream). */
+/* One timed launch: its family, its start and end, in ms after the first timed launch
+ * started (CUDA events on the launch's stream), and the algorithmic FLOPs and bytes it was
+ * tagged with (the same figures soap_profile_end sums per family). */
 typedef struct {
   int32_t family;   /* soap_kernel_family */
   double start_ms;
   double end_ms;
+  double flops;
+  double bytes;
 } soap_launch_record;
 
 /* Synchronises the device and copies the launches timed since soap_profile_begin, in launch

@@ -11,6 +11,7 @@ ProfScope::ProfScope(int family, double flops, double bytes, cudaStream_t s) : s
     p->overflow = true;
     return;
   }
+  if (p->serial) cudaDeviceSynchronize();
   idx_ = (int)p->recs.size();
   p->recs.push_back({family, flops, bytes});
   cudaEventRecord(p->events[2 * idx_], s_);

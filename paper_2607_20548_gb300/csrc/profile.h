@@ -32,6 +32,7 @@ struct Profiler {
   std::vector<Rec> recs;
   size_t capacity = 0;  // records
   bool overflow = false;
+  bool serial = false;  // each timed launch starts on an idle device
 };
 
 extern thread_local Profiler* t_profiler;

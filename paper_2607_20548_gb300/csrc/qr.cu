@@ -50,6 +50,7 @@
 
 #include "profile.h"
 #include "soap_internal.h"
+#include "tc_ptx.h"
 
 namespace cg = cooperative_groups;
 
@@ -64,6 +65,7 @@ constexpr int MAXC = 16;          // largest cluster (16 needs the non-portable 
 constexpr int NWARP = PT / 32;
 constexpr int NREST = NBO - NB;   // most block rows after a panel
 constexpr int KSPLIT = 8;         // split-K workspace: 8 partial n x NBO products (shorter ones split up to 16 ways)
+constexpr uint64_t kWaitNs = 2000000000ull;  // bound of every mbarrier wait in the panel kernel
 
 // lo part of x for the tensor-core products: x - trunc_tf32(x) rounded to the nearest tf32
 __device__ __forceinline__ float tf32_lo(float x) {
@@ -105,12 +107,6 @@ __device__ __forceinline__ void mma_tf32_16x8x8(float (&d)[4], const uint32_t (&
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
 // One 32-column panel, spread over a cluster: CTA c holds positions k + c*COLS .. of the
 // panel rows in shared memory (row stride LDS, 16-byte aligned rows).
 template <int COLS>
@@ -136,9 +132,18 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   __shared__ float s_T[NB][NB + 1];
   __shared__ float s_Y[NBO][NB + 1];     // rank 0: S V_panel summed over the cluster
   __shared__ __align__(16) float s_Z[NREST][NB];  // (S_rest V_panel) T_panel, the in-block update
-  // staging of S (STG chunks of 128 x 36) while Y is formed
-  constexpr int STG = COLS <= 512 ? 4 : 2;
-  __shared__ __align__(16) float s_scratch[STG * NBO * 36];
+  // S V_panel: with 512 positions per CTA on the tensor cores (tcgen05): SV_STG chunks of S
+  // (128 rows x 32 positions, 128-byte-swizzled) in flight, and two sets of S's lo part and
+  // V's hi and lo parts; with 1024 positions as warp-level MMAs over STG staged chunks of
+  // 128 x 36
+  constexpr int STG = 2;
+  constexpr int SV_STG = 4;
+  constexpr int A_BYTES = NBO * 32 * 4;
+  constexpr int B_BYTES = NB * 32 * 4;
+  constexpr int SV_BYTES = COLS == PT ? SV_STG * A_BYTES + 2 * (A_BYTES + 2 * B_BYTES) + 1024 : STG * NBO * 36 * 4;
+  __shared__ __align__(1024) uint8_t s_sv[SV_BYTES];
+  __shared__ __align__(8) uint64_t s_mma_bar[2];
+  __shared__ uint32_t s_tmem;
 
   const int n = p.n, k = p.k, kb = p.kb, k0 = p.k0, kbo = p.kbo;
   const int jb = k - k0;                // panel offset inside its block
@@ -457,13 +462,164 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   __syncthreads();  // this CTA's Vt rows are read back below
 
   // Y = S V_panel over this CTA's positions, S = the block's rows k0 .. k0+kbo-1: the block's
-  // Householder vectors so far (rows before the panel's end, from Vt) and the block rows
-  // still to be factored (from At). S is streamed through shared memory in 32-position
-  // chunks (cp.async, STG buffers, rows padded to 36 floats), and the product runs on the
-  // tensor cores as warp-level m16n8k8 TF32 MMAs with both operands split into tf32 hi and lo
-  // parts (four products: fp32 accuracy). Warp w owns rows 16 (w mod 8) .. +15 and columns
-  // 16 (w / 8) .. +15; each chunk is accumulated afresh and added to fp32 registers, so the
-  // tensor core's own accumulation never runs longer than 32 positions.
+  // Householder vectors so far (rows before the panel's end, from Vt) and the block rows still
+  // to be factored (from At), with both operands split into tf32 hi and lo parts (four
+  // products: fp32 accuracy), each 32-position chunk summed afresh and added to fp32 registers,
+  // so that the tensor core's own accumulation never runs longer than 32 positions.
+  if constexpr (COLS == PT) {
+    // On the tcgen05 tensor cores: D[128 x 32] (tensor memory) = S chunk (A: 128 rows x 32
+    // positions) x V chunk^T (B: 32 rows x 32 positions), both K-major in the 128-byte-swizzled
+    // layout. S's rows other than the panel's are copied with cp.async straight into that
+    // layout, SV_STG - 1 chunks ahead, and each thread forms the lo part of the units it copied;
+    // the panel's rows of S and the V chunk (hi and lo) come from sA. Two accumulators and two
+    // lo sets alternate: while the MMAs of chunk ch run, warps 0-3 drain chunk ch-1 (warp w
+    // reads lanes 32w..) and its S stage is refilled.
+    uint8_t* sv = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(s_sv) + 1023) & ~uintptr_t(1023));
+    uint8_t* st_a = sv;                          // [SV_STG] S chunks (fp32, read by the MMA as its hi part)
+    uint8_t* st_lo = sv + SV_STG * A_BYTES;      // [2] S lo | V hi | V lo
+    constexpr int LO_SET = A_BYTES + 2 * B_BYTES;
+    const int nchunk = (npos + 31) / 32;
+    if (tid == 0) {
+      tc::mbar_init(&s_mma_bar[0], 1);
+      tc::mbar_init(&s_mma_bar[1], 1);
+      asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(tc::smem_u32(&s_tmem)),
+                   "r"(64));
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = s_tmem;
+    // byte offset of 16-byte unit q of row r in a tile of 128-byte rows, swizzled within
+    // 1024-byte groups of 8 rows
+    auto swz16 = [](int r, int q) { return (r >> 3) * 1024 + (r & 7) * 128 + ((q ^ (r & 7)) << 4); };
+    auto issue = [&](int ch) {
+      uint8_t* dst = st_a + (ch % SV_STG) * A_BYTES;
+      for (int u = tid; u < NBO * 8; u += PT) {
+        const int r = u >> 3, q = u & 7;
+        if (r >= jb && r < jb + NB) continue;  // the panel's own rows: V, from sA
+        const int row = k0 + r, i = ch * 32 + 4 * q;
+        const bool ok = r < kbo && i < npos;  // zero-filled outside the block and past the positions
+        const float* src = ok ? (r < jb ? Vt : At) + (int64_t)row * n + pos0 + i : At;
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(tc::smem_u32(dst + swz16(r, q))),
+                     "l"(src), "r"(ok ? 16 : 0)
+                     : "memory");
+      }
+    };
+    auto lo4 = [](float4 x) { return make_float4(tf32_lo(x.x), tf32_lo(x.y), tf32_lo(x.z), tf32_lo(x.w)); };
+    float y[NB];
+#pragma unroll
+    for (int l = 0; l < NB; ++l) y[l] = 0.f;
+    for (int st0 = 0; st0 < SV_STG - 1; ++st0) {
+      if (st0 < nchunk) issue(st0);
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    }
+    int issued = 0;  // chunks whose MMAs were issued
+    bool aborted = false, bad = false;
+    for (int ch = 0; ch < nchunk; ++ch) {
+      const int set = ch & 1;
+      // this thread's copies of chunk ch have landed: their lo parts; the panel's rows of S and
+      // the V chunk (hi and lo) from sA
+      asm volatile("cp.async.wait_group %0;" ::"n"(SV_STG - 2) : "memory");
+      {
+        uint8_t* a = st_a + (ch % SV_STG) * A_BYTES;
+        uint8_t* lo = st_lo + set * LO_SET;
+        for (int u = tid; u < NBO * 8; u += PT) {
+          const int r = u >> 3;
+          if (r >= jb && r < jb + NB) continue;
+          const int off = swz16(r, u & 7);
+          *reinterpret_cast<float4*>(lo + off) = lo4(*reinterpret_cast<const float4*>(a + off));
+        }
+        uint8_t* bh = lo + A_BYTES;
+        uint8_t* bl = bh + B_BYTES;
+        for (int u = tid; u < NB * 8; u += PT) {
+          const int jj = u >> 3, q = u & 7;
+          const float4 x = *reinterpret_cast<const float4*>(&sA[jj * LDS + ch * 32 + 4 * q]);
+          const float4 xl = lo4(x);
+          const int off = swz16(jj, q), offa = swz16(jb + jj, q);
+          *reinterpret_cast<float4*>(bh + off) = x;
+          *reinterpret_cast<float4*>(bl + off) = xl;
+          *reinterpret_cast<float4*>(a + offa) = x;
+          *reinterpret_cast<float4*>(lo + offa) = xl;
+        }
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      if (__syncthreads_or(bad)) {
+        aborted = true;
+        break;
+      }
+      // the MMAs of chunk ch (its lo set and accumulator were released in the previous pass)
+      if (tid == 0) {
+        tc::tc_fence_after();
+        constexpr uint32_t idesc = tc::idesc_tf32(NBO, NB);
+        const uint32_t d = tmem + (uint32_t)(set * 32);
+        const uint32_t a_hi = tc::smem_u32(st_a + (ch % SV_STG) * A_BYTES);
+        const uint32_t a_lo = tc::smem_u32(st_lo + set * LO_SET);
+        const uint32_t b_hi = a_lo + A_BYTES;
+        const uint32_t b_lo = b_hi + B_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint32_t off = kk * 32;  // 8 tf32 = 32 bytes along the positions
+          tc::umma_tf32(d, tc::desc_sw128(a_lo + off), tc::desc_sw128(b_lo + off), idesc, kk != 0);
+          tc::umma_tf32(d, tc::desc_sw128(a_lo + off), tc::desc_sw128(b_hi + off), idesc, 1u);
+          tc::umma_tf32(d, tc::desc_sw128(a_hi + off), tc::desc_sw128(b_lo + off), idesc, 1u);
+          tc::umma_tf32(d, tc::desc_sw128(a_hi + off), tc::desc_sw128(b_hi + off), idesc, 1u);
+        }
+        tc::umma_commit(&s_mma_bar[set]);
+      }
+      issued = ch + 1;
+      // while they run: chunk ch-1's MMAs have completed, so its accumulator is drained and its
+      // S stage refilled with chunk ch + SV_STG - 1
+      if (ch >= 1) {
+        bool ok = tc::mbar_wait(&s_mma_bar[(ch - 1) & 1], ((ch - 1) >> 1) & 1, kWaitNs);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) {
+          bad = true;
+        } else if (warp < 4) {
+          float v[32];
+          tc::tmem_ld32(tmem + (uint32_t)(((ch - 1) & 1) * 32) + ((uint32_t)(32 * warp) << 16), v);
+#pragma unroll
+          for (int l = 0; l < NB; ++l) y[l] += v[l];
+        }
+      }
+      if (!bad && ch + SV_STG - 1 < nchunk) issue(ch + SV_STG - 1);
+      asm volatile("cp.async.commit_group;" ::: "memory");
+      tc::tc_fence_before();
+    }
+    // the last chunk's sum; after a wait that gave up, only the wait for every issued MMA (with
+    // the full bound), so that the tensor memory is not freed under one
+    bool ok_last = true;
+    if (issued > 0)
+      ok_last = __all_sync(0xffffffffu, tc::mbar_wait(&s_mma_bar[(issued - 1) & 1], ((issued - 1) >> 1) & 1, kWaitNs));
+    if (!aborted && !bad && ok_last && issued > 0 && warp < 4) {
+      float v[32];
+      tc::tmem_ld32(tmem + (uint32_t)(((issued - 1) & 1) * 32) + ((uint32_t)(32 * warp) << 16), v);
+#pragma unroll
+      for (int l = 0; l < NB; ++l) y[l] += v[l];
+    }
+    if (aborted || bad || !ok_last) atomicOr(p.status, kStatusTimeout);
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+      tc::tc_fence_after();
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(64));
+    }
+    // this CTA's partial product, kept in shared memory (the S stages are free) for the cluster
+    if (warp < 4) {
+      float* yp = reinterpret_cast<float*>(sv) + (32 * warp + lane) * NB;
+#pragma unroll
+      for (int l4 = 0; l4 < NB / 4; ++l4)
+        *reinterpret_cast<float4*>(yp + 4 * l4) = make_float4(y[4 * l4], y[4 * l4 + 1], y[4 * l4 + 2], y[4 * l4 + 3]);
+    }
+  } else
+  // With 1024 positions per CTA (factors of at most 1024 rows): S is streamed through shared
+  // memory in 32-position chunks (cp.async, STG buffers, rows padded to 36 floats), and the
+  // product runs as warp-level m16n8k8 TF32 MMAs. Warp w owns rows 16 (w mod 8) .. +15 and
+  // columns 16 (w / 8) .. +15.
   {
     static_assert(NBO == 128 && NB == 32 && NWARP == 16, "8 x 2 warp tiles of 16 x 16");
     constexpr int CH = 32;       // positions per chunk
@@ -475,7 +631,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     for (int e = 0; e < 4; ++e) y[0][e] = y[1][e] = 0.f;
     const int nchunk = (npos + CH - 1) / CH;
     auto issue = [&](int ch, int buf) {
-      float* dst = s_scratch + buf * NBO * CHP;
+      float* dst = reinterpret_cast<float*>(s_sv) + buf * NBO * CHP;
       for (int e = tid; e < NBO * (CH / 4); e += PT) {
         const int r = e / (CH / 4), q4 = e % (CH / 4);
         const int row = k0 + r, i = ch * CH + 4 * q4;
@@ -495,7 +651,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       else asm volatile("cp.async.commit_group;" ::: "memory");  // keeps the group count uniform
       asm volatile("cp.async.wait_group %0;" ::"n"(STG - 1) : "memory");
       __syncthreads();
-      const float* st = s_scratch + (ch % STG) * NBO * CHP;
+      const float* st = reinterpret_cast<const float*>(s_sv) + (ch % STG) * NBO * CHP;
       const int i0 = ch * CH;
       float d[2][4];
 #pragma unroll
@@ -535,39 +691,25 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       *reinterpret_cast<float2*>(yp + (m0 + gq + 8) * NB + col) = make_float2(y[nt][2], y[nt][3]);
     }
   }
-  cluster.sync();  // orders the partials in global memory before rank 0 reads them
-
-  // rank 0 sums the partials, forms T_panel, U = X T_panel and Z, and hands Z, U and T_panel
-  // to the cluster through global memory (rank 0's slots of Ypart, free once it has summed
-  // them): Z at 0, U at 3072 (jb <= 96 rows), T_panel at 6144 floats
-  float* xg = p.Ypart + (int64_t)b * MAXC * NBO * NB;
-  float* Ug = xg + NREST * NB;
-  float* Tpg = xg + 2 * NREST * NB;
-  if (c == 0) {
-    // sum the partials in a fixed order
-    const float* yp = p.Ypart + (int64_t)b * MAXC * NBO * NB;
-    for (int e = tid; e < kbo * NB; e += PT) {
-      float part[MAXC];
-#pragma unroll
-      for (int q = 0; q < MAXC; ++q) part[q] = q < C ? yp[(int64_t)q * NBO * NB + e] : 0.f;
-      float sum = 0.f;
-#pragma unroll
-      for (int q = 0; q < MAXC; ++q) sum += part[q];
-      s_Y[e / NB][e % NB] = sum;
-    }
-    __syncthreads();
+  // T_panel from the Gram rows of Y, then U = X T_panel (in place) and Z (rows after the panel);
+  // every thread of the CTA takes part (the barriers inside)
+  auto form_tuz = [&]() {
     // T of the panel from its Gram matrix g (rows jb.. of Y): T^-1 = diag(1/tau) + striu(g)
     // (H_1 ... H_kb = I - V T V^T); a reflector with tau = 0 (v = 0) gets a zero row and column.
-    // Warp w solves columns w and w + 16 by back substitution, lane l holding x_l:
+    // Warp w solves columns w and w + 16 by back substitution, lane i holding x_i:
     //   x_i = tau_i (delta_{i,cc} - sum_{i < l <= cc} g_il x_l)   (tau_i read as 1 where it is 0)
+    // Each solved x_l is broadcast once and every lane i < l adds g_il x_l to its running sum,
+    // so a step costs one shuffle instead of a warp-wide reduction.
     for (int cc = warp; cc < NB; cc += NWARP) {
-      float x = 0.f;
-      for (int i = cc; i >= 0; --i) {
-        const float part = warp_sum((lane > i && lane <= cc) ? s_Y[jb + i][lane] * x : 0.f);
-        if (lane == i) {
-          const float ti = i < kb ? s_tau[i] : 0.f;
-          x = ((i == cc ? 1.f : 0.f) - part) * (ti != 0.f ? ti : 1.f);
+      float x = 0.f, acc = 0.f;
+      for (int l = cc; l >= 0; --l) {
+        const float g = s_Y[jb + lane][l];
+        if (lane == l) {
+          const float tl = l < kb ? s_tau[l] : 0.f;
+          x = ((l == cc ? 1.f : 0.f) - acc) * (tl != 0.f ? tl : 1.f);
         }
+        const float xl = __shfl_sync(0xffffffffu, x, l);
+        if (lane < l) acc = fmaf(g, xl, acc);
       }
       const bool live = cc < kb && s_tau[cc] != 0.f;
       s_T[lane][cc] = (live && lane <= cc && lane < kb && s_tau[lane] != 0.f) ? x : 0.f;
@@ -597,21 +739,75 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       }
     }
     __syncthreads();
-    for (int e = tid; e < nrest * NB; e += PT) xg[e] = s_Z[e / NB][e % NB];
-    for (int e = tid; e < jb * NB; e += PT) Ug[e] = s_Y[e / NB][e % NB];
-    for (int e = tid; e < NB * NB; e += PT) Tpg[e] = s_T[e / NB][e % NB];
-    if (tid < kb) {
+  };
+  if constexpr (COLS == PT) {
+    // The partial products reduced through distributed shared memory: CTA c sums rows
+    // r = c mod C of every CTA's partial, in a fixed order, and every CTA then gathers the summed
+    // rows and forms T_panel, U and Z itself (the same values on every CTA).
+    uint8_t* sv = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(s_sv) + 1023) & ~uintptr_t(1023));
+    float* P_own = reinterpret_cast<float*>(sv);
+    float* Ysum = P_own + NBO * NB;
+    cluster.sync();  // every CTA's partial is in place
+    for (int r = c + C * warp; r < kbo; r += C * NWARP) {
+      float part[MAXC];
+#pragma unroll
+      for (int q = 0; q < MAXC; ++q) part[q] = q < C ? cluster.map_shared_rank(P_own, q)[r * NB + lane] : 0.f;
+      float sum = 0.f;
+#pragma unroll
+      for (int q = 0; q < MAXC; ++q) sum += part[q];
+      Ysum[r * NB + lane] = sum;
+    }
+    cluster.sync();  // every summed row is in place
+    for (int e = tid; e < kbo * NB; e += PT) s_Y[e / NB][e % NB] = cluster.map_shared_rank(Ysum, (e / NB) % C)[e];
+    // the peers may read this CTA's summed rows until they have gathered theirs: arrive now and
+    // wait at the end of the kernel
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+    __syncthreads();
+    form_tuz();
+    __syncthreads();
+    if (c == 0 && tid < kb) {
       p.skip[(int64_t)b * n + k + tid] = (uint8_t)s_skip[tid];
       p.dsign[(int64_t)b * n + k + tid] = s_dsign[tid];
     }
+  } else {
+    cluster.sync();  // orders the partials in global memory before rank 0 reads them
+    // rank 0 sums the partials, forms T_panel, U = X T_panel and Z, and hands Z, U and T_panel
+    // to the cluster through global memory (rank 0's slots of Ypart, free once it has summed
+    // them): Z at 0, U at 3072 (jb <= 96 rows), T_panel at 6144 floats
+    float* xg = p.Ypart + (int64_t)b * MAXC * NBO * NB;
+    float* Ug = xg + NREST * NB;
+    float* Tpg = xg + 2 * NREST * NB;
+    if (c == 0) {
+      // sum the partials in a fixed order
+      const float* yp = p.Ypart + (int64_t)b * MAXC * NBO * NB;
+      for (int e = tid; e < kbo * NB; e += PT) {
+        float part[MAXC];
+#pragma unroll
+        for (int q = 0; q < MAXC; ++q) part[q] = q < C ? yp[(int64_t)q * NBO * NB + e] : 0.f;
+        float sum = 0.f;
+#pragma unroll
+        for (int q = 0; q < MAXC; ++q) sum += part[q];
+        s_Y[e / NB][e % NB] = sum;
+      }
+      __syncthreads();
+      form_tuz();
+      __syncthreads();
+      for (int e = tid; e < nrest * NB; e += PT) xg[e] = s_Z[e / NB][e % NB];
+      for (int e = tid; e < jb * NB; e += PT) Ug[e] = s_Y[e / NB][e % NB];
+      for (int e = tid; e < NB * NB; e += PT) Tpg[e] = s_T[e / NB][e % NB];
+      if (tid < kb) {
+        p.skip[(int64_t)b * n + k + tid] = (uint8_t)s_skip[tid];
+        p.dsign[(int64_t)b * n + k + tid] = s_dsign[tid];
+      }
+    }
+    cluster.sync();  // Z, U and T_panel in global memory are visible to the cluster
+    if (c != 0) {
+      for (int e = tid; e < nrest * NB; e += PT) s_Z[e / NB][e % NB] = xg[e];
+      for (int e = tid; e < jb * NB; e += PT) s_Y[e / NB][e % NB] = Ug[e];
+      for (int e = tid; e < NB * NB; e += PT) s_T[e / NB][e % NB] = Tpg[e];
+    }
+    __syncthreads();
   }
-  cluster.sync();  // Z, U and T_panel in global memory are visible to the cluster
-  if (c != 0) {
-    for (int e = tid; e < nrest * NB; e += PT) s_Z[e / NB][e % NB] = xg[e];
-    for (int e = tid; e < jb * NB; e += PT) s_Y[e / NB][e % NB] = Ug[e];
-    for (int e = tid; e < NB * NB; e += PT) s_T[e / NB][e % NB] = Tpg[e];
-  }
-  __syncthreads();
   // the block's T, rows spread over the cluster (row r by CTA r mod C): column block jb =
   // [-T_before U ; T_panel ; 0] and the row block jb left of it = 0; thread (rl, g) writes
   // columns jb + 8g .. jb + 8g+7 of row r = c + C rl
@@ -620,14 +816,30 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     float* T_lo = p.T_lo + (int64_t)b * NBO * NBO;
     float* Tt = p.Tt + (int64_t)b * NBO * NBO;
     float* Tt_lo = p.Tt_lo + (int64_t)b * NBO * NBO;
+    // the rows of T_before (written by the block's earlier panels) that this CTA's rows need,
+    // staged in shared memory with independent loads: the S V area is free (on the cluster path
+    // past its first 32 KB, the summed rows that peers may still read)
+    constexpr int TBS = NBO - NB;  // jb <= 96
+    float* Tb = reinterpret_cast<float*>(
+        COLS == PT ? ((reinterpret_cast<uintptr_t>(s_sv) + 1023) & ~uintptr_t(1023)) + 2 * NBO * NB * sizeof(float)
+                   : reinterpret_cast<uintptr_t>(s_sv));
+    static_assert(TBS * TBS * sizeof(float) <= (COLS == PT ? SV_BYTES - 1024 - 2 * NBO * NB * sizeof(float) : SV_BYTES),
+                  "T_before staging");
+    const int nrl = jb > c ? (jb - c + C - 1) / C : 0;  // this CTA's rows r = c + C rl below jb
+    for (int e = tid; e < nrl * jb; e += PT) {
+      const int rl = e / jb, l = e - rl * jb, rr = c + C * rl;
+      Tb[rl * TBS + l] = l >= rr ? T[rr * NBO + l] : 0.f;
+    }
+    __syncthreads();
     const int r = c + C * (tid >> 2), g8 = (tid & 3) * 8;
     if (r < NBO) {
       float t[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) t[u] = 0.f;
       if (r < jb) {
+        const float* tb_row = Tb + (tid >> 2) * TBS;
         for (int l = r; l < jb; ++l) {
-          const float tb = T[r * NBO + l];  // T_before, written by the block's earlier panels
+          const float tb = tb_row[l];
 #pragma unroll
           for (int u = 0; u < 8; ++u) t[u] = fmaf(-tb, s_Y[l][g8 + u], t[u]);
         }
@@ -655,13 +867,28 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   }
 
   // the panel's reflectors on the block rows after it: a_r -= Z_r V^T at this CTA's
-  // positions, four rows at a time
+  // positions, eight rows at a time (eight independent loads in flight), then four, then one
   for (int i = tid; i < npos; i += PT) {
     float v[NB];
 #pragma unroll
     for (int jj = 0; jj < NB; ++jj) v[jj] = sA[jj * LDS + i];
     float* a = At + (int64_t)(k + kb) * n + pos0 + i;
     int r = 0;
+    for (; r + 8 <= nrest; r += 8) {
+      float x[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) x[u] = a[(int64_t)(r + u) * n];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        float acc = 0.f;
+#pragma unroll
+        for (int j4 = 0; j4 < NB / 4; ++j4) {
+          const float4 z = *reinterpret_cast<const float4*>(&s_Z[r + u][4 * j4]);
+          acc = fmaf(z.x, v[4 * j4], fmaf(z.y, v[4 * j4 + 1], fmaf(z.z, v[4 * j4 + 2], fmaf(z.w, v[4 * j4 + 3], acc))));
+        }
+        a[(int64_t)(r + u) * n] = x[u] - acc;
+      }
+    }
     for (; r + 4 <= nrest; r += 4) {
       float x[4];
 #pragma unroll
@@ -684,6 +911,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       a[(int64_t)r * n] -= acc;
     }
   }
+  if constexpr (COLS == PT) asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 // ||P_b||_F: per-chunk partial sums in double (chunks of whole 16-byte units: nn is a

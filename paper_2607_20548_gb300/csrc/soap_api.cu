@@ -1341,7 +1341,12 @@ void soap_destroy(soap_handle h) {
 }
 
 soap_status_t soap_profile_begin(soap_handle h, int64_t max_launches) {
-  if (!h || max_launches < 1 || max_launches > (int64_t(1) << 22)) return SOAP_ERR_INVALID_ARG;
+  return soap_profile_begin_ex(h, max_launches, 0);
+}
+
+soap_status_t soap_profile_begin_ex(soap_handle h, int64_t max_launches, int32_t flags) {
+  if (!h || max_launches < 1 || max_launches > (int64_t(1) << 22) || (flags & ~SOAP_PROFILE_SERIAL))
+    return SOAP_ERR_INVALID_ARG;
   DeviceGuard g(h->device);
   soap::Profiler& p = h->prof;
   while ((int64_t)p.events.size() < 2 * max_launches) {
@@ -1352,6 +1357,7 @@ soap_status_t soap_profile_begin(soap_handle h, int64_t max_launches) {
   p.capacity = (size_t)max_launches;
   p.recs.clear();
   p.overflow = false;
+  p.serial = (flags & SOAP_PROFILE_SERIAL) != 0;
   soap::t_profiler = &p;
   return SOAP_OK;
 }
@@ -1388,7 +1394,7 @@ soap_status_t soap_profile_records(soap_handle h, soap_launch_record* out, int64
     float t0 = 0.f, t1 = 0.f;
     SOAP_CUDA(h, cudaEventElapsedTime(&t0, p.events[0], p.events[2 * i]));
     SOAP_CUDA(h, cudaEventElapsedTime(&t1, p.events[0], p.events[2 * i + 1]));
-    out[i] = soap_launch_record{p.recs[i].family, (double)t0, (double)t1};
+    out[i] = soap_launch_record{p.recs[i].family, (double)t0, (double)t1, p.recs[i].flops, p.recs[i].bytes};
   }
   *count = n;
   return SOAP_OK;

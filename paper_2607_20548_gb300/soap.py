@@ -27,7 +27,8 @@ STATUS_NAMES = {0: "SOAP_OK", 1: "SOAP_ERR_INVALID_ARG", 2: "SOAP_ERR_CUDA", 3: 
 EXPORTS = ("soap_default_hparams", "soap_create", "soap_create_ex", "soap_plan_info", "soap_step", "soap_set_lr", "soap_state_bytes",
            "soap_state_get", "soap_state_set", "soap_get_step", "soap_set_step", "soap_status",
            "soap_clear_status", "soap_last_error", "soap_destroy", "soap_qr_workspace_bytes",
-           "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_end", "soap_profile_records",
+           "soap_qr", "soap_gemm", "soap_profile_begin", "soap_profile_begin_ex", "soap_profile_end",
+           "soap_profile_records",
            "soap_gemm_tf32x4",
            "soap_split_tf32", "soap_qr_static", "soap_layerwise_assign", "soap_wait_limit")
 # every symbol include/muon.h declares
@@ -35,6 +36,7 @@ MUON_EXPORTS = ("muon_default_hparams", "muon_create", "muon_step", "muon_set_lr
                 "muon_state_set", "muon_status", "muon_last_error", "muon_destroy", "muon_profile_begin",
                 "muon_profile_end")
 KERNEL_FAMILIES = ("gemm_simt", "gemm_tc", "qr_panel", "elementwise", "other", "qr_update")
+PROFILE_SERIAL = 1  # SOAP_PROFILE_SERIAL
 
 
 class muon_hparams(ctypes.Structure):
@@ -62,7 +64,8 @@ class soap_kernel_stats(ctypes.Structure):
 
 
 class soap_launch_record(ctypes.Structure):
-    _fields_ = [("family", ctypes.c_int32), ("start_ms", ctypes.c_double), ("end_ms", ctypes.c_double)]
+    _fields_ = [("family", ctypes.c_int32), ("start_ms", ctypes.c_double), ("end_ms", ctypes.c_double),
+                ("flops", ctypes.c_double), ("bytes", ctypes.c_double)]
 
 
 class SoapError(RuntimeError):
@@ -104,6 +107,7 @@ def load_library(path: str = LIB_PATH):
         "soap_qr_workspace_bytes": (SZ, [I32, I32]),
         "soap_qr": (I32, [I32, I32, P, P, P, F, P, SZ, P, P]),
         "soap_profile_begin": (I32, [P, I64]),
+        "soap_profile_begin_ex": (I32, [P, I64, I32]),
         "soap_profile_end": (I32, [P, P, ctypes.POINTER(soap_kernel_stats), ctypes.POINTER(I32)]),
         "soap_profile_records": (I32, [P, ctypes.POINTER(soap_launch_record), I64, ctypes.POINTER(I64)]),
         "soap_gemm": (I32, [I32, I32, I32, I32, I32, F, P, I64, I64, P, I64, I64, F, P, I64, I64, I32, P]),
@@ -278,9 +282,12 @@ class SoapOptimizer:
     def clear_status(self, stream=None):
         _check(load_library().soap_clear_status(self._handle(), _stream(stream, self.device)), self._h)
 
-    def profile_begin(self, max_launches: int = 1 << 16):
-        """Time every kernel launch of the following calls with CUDA events."""
-        _check(load_library().soap_profile_begin(self._handle(), max_launches), self._h)
+    def profile_begin(self, max_launches: int = 1 << 16, serial: bool = False):
+        """Time every kernel launch of the following calls with CUDA events; with serial, each
+        launch starts on an idle device (soap_profile_begin_ex, SOAP_PROFILE_SERIAL), so its time
+        is the kernel's alone."""
+        _check(load_library().soap_profile_begin_ex(self._handle(), max_launches, PROFILE_SERIAL if serial else 0),
+               self._h)
 
     def profile_end(self, stream=None) -> dict:
         """Synchronise and return {family: {launches, ms, flops, bytes}} plus an overflow flag."""
@@ -292,12 +299,15 @@ class SoapOptimizer:
         res["overflow"] = bool(ov.value)
         return res
 
-    def profile_records(self, max_records=1 << 20) -> list:
+    def profile_records(self, max_records=1 << 20, detail=False) -> list:
         """The launches timed since profile_begin as (family, start_ms, end_ms), in launch order
-        (call before profile_end)."""
+        (call before profile_end); with detail, (family, start_ms, end_ms, flops, bytes)."""
         out = (soap_launch_record * max_records)()
         cnt = ctypes.c_int64(0)
         _check(load_library().soap_profile_records(self._handle(), out, max_records, ctypes.byref(cnt)), self._h)
+        if detail:
+            return [(KERNEL_FAMILIES[out[i].family], out[i].start_ms, out[i].end_ms, out[i].flops, out[i].bytes)
+                    for i in range(cnt.value)]
         return [(KERNEL_FAMILIES[out[i].family], out[i].start_ms, out[i].end_ms) for i in range(cnt.value)]
 
     def last_error(self) -> str:
