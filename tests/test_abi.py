@@ -70,6 +70,10 @@ def test_host_side_validation_needs_no_gpu():
     assert lib.soap_get_step(None) == -1
     assert lib.soap_last_error(None) == b"null handle"
     lib.soap_destroy(None)
+    # profiling: a null handle, and (checked before any device work) unknown flags, are refused
+    assert lib.soap_profile_begin_ex(None, 16, S.PROFILE_SERIAL) == 1
+    assert lib.soap_profile_records(None, None, 0, None) == 1
+    assert ctypes.sizeof(S.soap_launch_record) == 40  # int32 family (padded), start, end, flops, bytes
     # Muon: sides must be multiples of 8, ns_steps in 1..64
     mh = S.muon_hparams()
     lib.muon_default_hparams(ctypes.byref(mh))
