@@ -186,8 +186,6 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       // strictly after the pivot (pivot = local position j of rank 0)
       const float x = (have && (c != 0 || i > j)) ? a[0] : 0.f;
       float v[NB];
-#pragma unroll
-      for (int l = 0; l < NB; ++l) v[l] = x * a[l];
       // transposing butterfly over the warp: lane l ends with the warp's sum for row j + l
 #define SOAP_BFLY(o, nh)                                                   \
   {                                                                        \
@@ -198,11 +196,25 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       v[q] = keep + __shfl_xor_sync(0xffffffffu, send, (o));               \
     }                                                                      \
   }
-      SOAP_BFLY(16, 16)
-      SOAP_BFLY(8, 8)
-      SOAP_BFLY(4, 4)
-      SOAP_BFLY(2, 2)
-      SOAP_BFLY(1, 1)
+      if (kb - j > NB / 2) {
+#pragma unroll
+        for (int l = 0; l < NB; ++l) v[l] = x * a[l];
+        SOAP_BFLY(16, 16)
+        SOAP_BFLY(8, 8)
+        SOAP_BFLY(4, 4)
+        SOAP_BFLY(2, 2)
+        SOAP_BFLY(1, 1)
+      } else {
+        // at most 16 rows left (the rest of a[] is zero): the butterfly over the 16 live values
+        // within each half-warp (lane l ends with row j + (l mod 16)), then across the halves
+#pragma unroll
+        for (int l = 0; l < NB / 2; ++l) v[l] = x * a[l];
+        SOAP_BFLY(8, 8)
+        SOAP_BFLY(4, 4)
+        SOAP_BFLY(2, 2)
+        SOAP_BFLY(1, 1)
+        v[0] += __shfl_xor_sync(0xffffffffu, v[0], 16);
+      }
 #undef SOAP_BFLY
       s_red[warp][lane] = v[0];
       // rank 0's pivot position: alpha and the later rows' values there
