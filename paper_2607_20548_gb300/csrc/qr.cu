@@ -821,8 +821,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     __syncthreads();
   }
   // the block's T, rows spread over the cluster (row r by CTA r mod C): column block jb =
-  // [-T_before U ; T_panel ; 0] and the row block jb left of it = 0; thread (rl, g) writes
-  // columns jb + 8g .. jb + 8g+7 of row r = c + C rl
+  // [-T_before U ; T_panel ; 0] and the row block jb left of it = 0
   {
     float* T = p.T + (int64_t)b * NBO * NBO;
     float* T_lo = p.T_lo + (int64_t)b * NBO * NBO;
@@ -843,36 +842,53 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
       Tb[rl * TBS + l] = l >= rr ? T[rr * NBO + l] : 0.f;
     }
     __syncthreads();
-    const int r = c + C * (tid >> 2), g8 = (tid & 3) * 8;
-    if (r < NBO) {
-      float t[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) t[u] = 0.f;
+    // one entry (row r = c + C rl, column jb + cc) per work unit, the 32 units of a row on
+    // consecutive threads: the triangular product's long rows are spread over all threads in
+    // turn. On the cluster path the column block is also staged transposed, so that Tt's rows
+    // are written with consecutive stores.
+    const int nr = (NBO - c + C - 1) / C;  // this CTA's rows
+    float* stt = COLS == PT ? Tb + TBS * TBS : nullptr;  // [NB][NBO]: entry (cc, rl)
+    static_assert(COLS != PT || (TBS * TBS + NB * NBO) * sizeof(float) <= SV_BYTES - 1024 - 2 * NBO * NB * sizeof(float),
+                  "T column block staging");
+    for (int u = tid; u < nr * NB; u += PT) {
+      const int rl = u >> 5, cc = u & 31, r = c + C * rl;
+      float t = 0.f;
       if (r < jb) {
-        const float* tb_row = Tb + (tid >> 2) * TBS;
-        for (int l = r; l < jb; ++l) {
-          const float tb = tb_row[l];
-#pragma unroll
-          for (int u = 0; u < 8; ++u) t[u] = fmaf(-tb, s_Y[l][g8 + u], t[u]);
-        }
+        const float* tb_row = Tb + rl * TBS;
+#pragma unroll 4
+        for (int l = r; l < jb; ++l) t = fmaf(-tb_row[l], s_Y[l][cc], t);
       } else if (r < jb + NB) {
-#pragma unroll
-        for (int u = 0; u < 8; ++u) t[u] = s_T[r - jb][g8 + u];
+        t = s_T[r - jb][cc];
       }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int col = jb + g8 + u;
-        T[r * NBO + col] = t[u];
-        T_lo[r * NBO + col] = tf32_lo(t[u]);
-        Tt[col * NBO + r] = t[u];
-        Tt_lo[col * NBO + r] = tf32_lo(t[u]);
+      const int col = jb + cc;
+      T[r * NBO + col] = t;
+      T_lo[r * NBO + col] = tf32_lo(t);
+      if (COLS == PT) {
+        stt[cc * NBO + rl] = t;
+      } else {
+        Tt[col * NBO + r] = t;
+        Tt_lo[col * NBO + r] = tf32_lo(t);
       }
     }
+    if (COLS == PT) {
+      __syncthreads();
+      for (int e = tid; e < NB * nr; e += PT) {
+        const int cc = e / nr, rl = e - cc * nr;
+        const float t = stt[cc * NBO + rl];
+        Tt[(jb + cc) * NBO + c + C * rl] = t;
+        Tt_lo[(jb + cc) * NBO + c + C * rl] = tf32_lo(t);
+      }
+    }
+    // the row block jb left of the panel is zero: T's rows jb.. and Tt's columns jb.. there
     for (int e = tid; e < NB * jb; e += PT) {
       const int rr = jb + e / jb, col = e % jb;
       if (rr % C != c) continue;
       T[rr * NBO + col] = 0.f;
       T_lo[rr * NBO + col] = 0.f;
+    }
+    for (int e = tid; e < NB * jb; e += PT) {
+      const int col = e / NB, rr = jb + e % NB;
+      if (rr % C != c) continue;
       Tt[col * NBO + rr] = 0.f;
       Tt_lo[col * NBO + rr] = 0.f;
     }
