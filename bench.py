@@ -565,15 +565,31 @@ def run_soap(args):
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
     torch.cuda.synchronize()
+    # the copies run on two side streams, so that a step's weights going out overlap the next
+    # step's gradients coming in (the two directions of the link); each step waits for its
+    # gradients and for the previous step's weights to be out before it rewrites them
+    s_in, s_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    ev_in, ev_out, ev_done = torch.cuda.Event(), torch.cuda.Event(), torch.cuda.Event()
     e0.record(stream)
     base = step0 + args.steps
     for t in range(args.steps):
         k = (base + t) % npool
-        for d, hsrc in zip(pool[k], host_pool[k]):
-            d.copy_(hsrc, non_blocking=True)
+        s_in.wait_stream(stream)  # the previous step has read the gradient buffers
+        with torch.cuda.stream(s_in):
+            for d, hsrc in zip(pool[k], host_pool[k]):
+                d.copy_(hsrc, non_blocking=True)
+            ev_in.record(s_in)
+        stream.wait_event(ev_in)
+        if t > 0:
+            stream.wait_event(ev_out)
         opt.step(W, grads_for(base + t))
-        for hdst, w in zip(host_w, Wg):
-            hdst.copy_(w, non_blocking=True)
+        ev_done.record(stream)
+        s_out.wait_event(ev_done)
+        with torch.cuda.stream(s_out):
+            for hdst, w in zip(host_w, Wg):
+                hdst.copy_(w, non_blocking=True)
+            ev_out.record(s_out)
+    stream.wait_event(ev_out)
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_s = e0.elapsed_time(e1) / 1e3
