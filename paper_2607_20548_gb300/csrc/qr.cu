@@ -87,6 +87,7 @@ struct PanelArgs {
   float* Ypart;        // [batch][MAXC][NBO][NB] per-CTA partial products S V_panel
   uint8_t* skip;       // [batch][n]
   float* dsign;        // [batch][n] sign of R_pp (+1 for zero columns)
+  float* tau;          // [batch][n] the reflectors' tau (handed from the column kernel)
   const float* thresh; // [batch]
   int* status;
   int n, k0, kbo, k, kb;  // block start and width, panel start and width
@@ -109,8 +110,9 @@ __device__ __forceinline__ void mma_tf32_16x8x8(float (&d)[4], const uint32_t (&
 
 // One 32-column panel, spread over a cluster: CTA c holds positions k + c*COLS .. of the
 // panel rows in shared memory (row stride LDS, 16-byte aligned rows).
-template <int COLS>
+template <int COLS, bool SPLIT = false>
 __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
+  static_assert(!SPLIT || COLS == PT, "the column loop runs on its own only for 512 positions per CTA");
   constexpr int LDS = COLS + 4;
   cg::cluster_group cluster = cg::this_cluster();
   const int c = (int)cluster.block_rank();
@@ -159,18 +161,25 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     for (int e = tid; e < NB * q4n; e += PT) {
       const int jj = e / q4n, i = 4 * (e % q4n);
       const bool ok = jj < kb && i < npos;
-      const float* src = ok ? At + (int64_t)(k + jj) * n + pos0 + i : At;
+      // after the column kernel: the panel's Householder vectors, as rows of Vt
+      const float* rows = SPLIT ? p.Vt + (int64_t)b * nn : At;
+      const float* src = ok ? rows + (int64_t)(k + jj) * n + pos0 + i : rows;
       const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(&sA[jj * LDS + i]));
       asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(ok ? 16 : 0) : "memory");
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
     asm volatile("cp.async.wait_group 0;" ::: "memory");
   }
+  if constexpr (SPLIT) {
+    if (tid < NB) s_tau[tid] = tid < kb ? p.tau[(int64_t)b * n + k + tid] : 0.f;
+  }
   __syncthreads();
   const float thresh = p.thresh[b];
   int nonfinite = 0;
 
-  if constexpr (COLS == PT) {
+  if constexpr (SPLIT) {
+    // the column loop ran in qr_cols_kernel
+  } else if constexpr (COLS == PT) {
     // One position per thread: thread tid holds the panel rows' values at position tid in
     // registers, the current row first (a[l] = row j + l; rows past the panel are zero), so
     // that the per-column dot products and the reflector's update never touch shared memory;
@@ -425,8 +434,9 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   }
   if (nonfinite) atomicOr(p.status, kStatusQrBreakdown);
 
-  // V with its unit diagonal and zeros before it (rank 0 holds the first kb positions)
-  if (c == 0) {
+  // V with its unit diagonal and zeros before it (rank 0 holds the first kb positions; the
+  // column kernel wrote them so)
+  if (!SPLIT && c == 0) {
     for (int e = tid; e < kb * kb; e += PT) {
       const int jj = e / kb, i = e % kb;
       if (i < jj) sA[jj * LDS + i] = 0.f;
@@ -441,7 +451,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   float* Vt_lo = p.Vt_lo + (int64_t)b * nn;
   float* Vpos = p.Vpos + (int64_t)b * n * NBO;
   float* Vpos_lo = p.Vpos_lo + (int64_t)b * n * NBO;
-  {
+  if constexpr (!SPLIT) {  // (the column kernel wrote Vt)
     const int q4n = npos / 4;
     for (int e = tid; e < kb * q4n; e += PT) {
       const int jj = e / q4n, q = e - jj * q4n;
@@ -459,12 +469,13 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     *reinterpret_cast<float4*>(Vpos_lo + o) = make_float4(tf32_lo(v.x), tf32_lo(v.y), tf32_lo(v.z), tf32_lo(v.w));
   }
   if (c == 0) {
-    for (int jj = 0; jj < kb; ++jj)
-      for (int i = tid; i < jb; i += PT) {
-        const int64_t o = (int64_t)(k + jj) * n + k0 + i;
-        Vt[o] = 0.f;
-        Vt_lo[o] = 0.f;
-      }
+    if (!SPLIT)
+      for (int jj = 0; jj < kb; ++jj)
+        for (int i = tid; i < jb; i += PT) {
+          const int64_t o = (int64_t)(k + jj) * n + k0 + i;
+          Vt[o] = 0.f;
+          Vt_lo[o] = 0.f;
+        }
     for (int e = tid; e < jb * NB; e += PT) {
       const int64_t o = (int64_t)(k0 + e / NB) * NBO + jb + e % NB;
       Vpos[o] = 0.f;
@@ -777,7 +788,7 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
     __syncthreads();
     form_tuz();
     __syncthreads();
-    if (c == 0 && tid < kb) {
+    if (!SPLIT && c == 0 && tid < kb) {
       p.skip[(int64_t)b * n + k + tid] = (uint8_t)s_skip[tid];
       p.dsign[(int64_t)b * n + k + tid] = s_dsign[tid];
     }
@@ -942,6 +953,222 @@ __global__ void __launch_bounds__(PT, 1) qr_panel_kernel(PanelArgs p) {
   if constexpr (COLS == PT) asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
+// The column loop of a 32-column panel on its own, for factors of more than 1024 rows (the
+// Householder steps of qr_panel_kernel's register path): CTA c of the cluster holds positions
+// k + 512 c .. of the panel rows, two per thread, in registers. It writes V as rows of Vt with
+// their lo parts (zeros before each pivot and at the block's positions before the panel, one at
+// the pivot), and tau, skip and dsign; qr_panel_kernel<512, true> then forms the block product,
+// T and the in-block update from them. With 256 threads of at most 128 registers and a few KB of
+// shared memory, two of these CTAs fit on one SM, so the latency-bound loop holds half an SM
+// instead of a whole one.
+constexpr int PTA = 256;
+constexpr int NWA = PTA / 32;
+
+__global__ void __launch_bounds__(PTA, 2) qr_cols_kernel(PanelArgs p) {
+  constexpr int COLS = 2 * PTA;
+  cg::cluster_group cluster = cg::this_cluster();
+  const int c = (int)cluster.block_rank();
+  const int C = (int)cluster.num_blocks();
+  const int b = blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  __shared__ float s_part[2][NB];
+  __shared__ float s_pv[2][NB];
+  __shared__ float s_scal[2];
+  __shared__ __align__(16) float s_wl[NB];
+  __shared__ float s_red[NWA][NB];
+
+  const int n = p.n, k = p.k, kb = p.kb, k0 = p.k0;
+  const int jb = k - k0;
+  const int64_t nn = (int64_t)n * n;
+  const float* At = p.At + (int64_t)b * nn;
+  float* Vt = p.Vt + (int64_t)b * nn;
+  float* Vt_lo = p.Vt_lo + (int64_t)b * nn;
+  const int pos0 = k + c * COLS;
+  const int npos = max(0, min(COLS, n - pos0));
+  const int i0 = tid, i1 = tid + PTA;  // this thread's positions; i1 is past every pivot
+  const bool have0 = i0 < npos, have1 = i1 < npos;
+  float a0[NB], a1[NB];
+#pragma unroll
+  for (int l = 0; l < NB; ++l) {
+    a0[l] = (have0 && l < kb) ? At[(int64_t)(k + l) * n + pos0 + i0] : 0.f;
+    a1[l] = (have1 && l < kb) ? At[(int64_t)(k + l) * n + pos0 + i1] : 0.f;
+  }
+  const float thresh = p.thresh[b];
+  int nonfinite = 0;
+  for (int j = 0; j < kb; ++j) {
+    const int par = j & 1;
+    // this thread's shares of sigma and of x . a_(j+l), positions strictly after the pivot
+    const float x0 = (have0 && (c != 0 || i0 > j)) ? a0[0] : 0.f;
+    const float x1 = have1 ? a1[0] : 0.f;
+    float v[NB];
+#define SOAP_BFLY(o, nh)                                                   \
+  {                                                                        \
+    const bool up = (lane & (o)) != 0;                                     \
+    _Pragma("unroll") for (int q = 0; q < (nh); ++q) {                     \
+      const float keep = up ? v[q + (nh)] : v[q];                          \
+      const float send = up ? v[q] : v[q + (nh)];                          \
+      v[q] = keep + __shfl_xor_sync(0xffffffffu, send, (o));               \
+    }                                                                      \
+  }
+    if (kb - j > NB / 2) {
+#pragma unroll
+      for (int l = 0; l < NB; ++l) v[l] = fmaf(x1, a1[l], x0 * a0[l]);
+      SOAP_BFLY(16, 16)
+      SOAP_BFLY(8, 8)
+      SOAP_BFLY(4, 4)
+      SOAP_BFLY(2, 2)
+      SOAP_BFLY(1, 1)
+    } else {
+#pragma unroll
+      for (int l = 0; l < NB / 2; ++l) v[l] = fmaf(x1, a1[l], x0 * a0[l]);
+      SOAP_BFLY(8, 8)
+      SOAP_BFLY(4, 4)
+      SOAP_BFLY(2, 2)
+      SOAP_BFLY(1, 1)
+      v[0] += __shfl_xor_sync(0xffffffffu, v[0], 16);
+    }
+#undef SOAP_BFLY
+    s_red[warp][lane] = v[0];
+    if (c == 0 && i0 == j) {
+#pragma unroll
+      for (int l = 0; l < NB; ++l)
+        if (j + l < kb) s_pv[par][j + l] = a0[l];
+    }
+    __syncthreads();
+    if (warp == 0) {
+      float sum = 0.f;
+#pragma unroll
+      for (int w = 0; w < NWA; ++w) sum += s_red[w][lane];
+      if (j + lane < kb) s_part[par][j + lane] = sum;
+    }
+    cluster.sync();
+    if (warp == 0) {
+      s_wl[lane] = 0.f;
+      __syncwarp();
+    }
+    if (tid >= j && tid < kb) {
+      // the cluster's partial sums in rank order (the same order on every CTA), four peers'
+      // loads in flight at a time
+      const float* pv0 = cluster.map_shared_rank(&s_pv[par][0], 0);
+      const float alpha = pv0[j], apiv = pv0[tid];
+      float d = 0.f, sigma = 0.f;
+#pragma unroll
+      for (int q0 = 0; q0 < MAXC; q0 += 4) {
+        if (q0 < C) {
+          float ps[4], pd[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const float* rp = cluster.map_shared_rank(&s_part[par][0], q0 + u < C ? q0 + u : 0);
+            ps[u] = rp[j];
+            pd[u] = rp[tid];
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            if (q0 + u < C) {
+              sigma += ps[u];
+              d += pd[u];
+            }
+          }
+        }
+      }
+      const float xnorm = sqrtf(fmaf(alpha, alpha, sigma));
+      const bool skip = !(xnorm > thresh);
+      float tau = 0.f, v0 = 1.f, rsign = 1.f;
+      if (!skip) {
+        if (sigma == 0.f) {
+          rsign = alpha < 0.f ? -1.f : 1.f;  // H = I, R_pp = alpha
+        } else {
+          const float beta = alpha >= 0.f ? -xnorm : xnorm;
+          v0 = alpha - beta;  // same sign as alpha: no cancellation
+          tau = (beta - alpha) / beta;
+          rsign = beta < 0.f ? -1.f : 1.f;
+        }
+      }
+      if (tid == j) {
+        if (!isfinite(xnorm)) nonfinite = 1;
+        s_scal[0] = tau;
+        s_scal[1] = tau != 0.f ? 1.f / v0 : 0.f;
+        if (c == 0) {
+          p.tau[(int64_t)b * n + k + j] = tau;
+          p.skip[(int64_t)b * n + k + j] = skip ? 1 : 0;
+          p.dsign[(int64_t)b * n + k + j] = rsign;
+        }
+      } else {
+        s_wl[tid - j] = tau != 0.f ? apiv + d / v0 : 0.f;  // v^T a_tid, with v = x / v0 after the pivot
+      }
+    }
+    __syncthreads();
+    const float tau = s_scal[0], rv0 = s_scal[1];
+    // v at this thread's positions (x / v0 after the pivot, 1 at it, 0 before it on rank 0) into
+    // row j of Vt, and H_j = I - tau v v^T on the later rows, shifting them down one register
+    {
+      const int64_t o = (int64_t)(k + j) * n + pos0 + i0;
+      if (have0 && (c != 0 || i0 >= j)) {
+        const bool at_pivot = (c == 0 && i0 == j);
+        const float vi = at_pivot ? 1.f : a0[0] * rv0;
+        Vt[o] = vi;
+        Vt_lo[o] = tf32_lo(vi);
+        if (tau != 0.f) {
+          const float tv = tau * vi;
+#pragma unroll
+          for (int l4 = 0; l4 < NB / 4; ++l4) {
+            const float4 w4 = reinterpret_cast<const float4*>(s_wl)[l4];
+            if (l4 > 0) a0[4 * l4 - 1] = fmaf(-tv, w4.x, a0[4 * l4]);
+            a0[4 * l4] = fmaf(-tv, w4.y, a0[4 * l4 + 1]);
+            a0[4 * l4 + 1] = fmaf(-tv, w4.z, a0[4 * l4 + 2]);
+            a0[4 * l4 + 2] = fmaf(-tv, w4.w, a0[4 * l4 + 3]);
+          }
+          a0[NB - 1] = 0.f;
+        } else {
+#pragma unroll
+          for (int l = 0; l < NB - 1; ++l) a0[l] = a0[l + 1];
+          a0[NB - 1] = 0.f;
+        }
+      } else {
+        if (have0) {  // rank 0, before the pivot
+          Vt[o] = 0.f;
+          Vt_lo[o] = 0.f;
+        }
+#pragma unroll
+        for (int l = 0; l < NB - 1; ++l) a0[l] = a0[l + 1];
+        a0[NB - 1] = 0.f;
+      }
+    }
+    if (have1) {
+      const int64_t o = (int64_t)(k + j) * n + pos0 + i1;
+      const float vi = a1[0] * rv0;
+      Vt[o] = vi;
+      Vt_lo[o] = tf32_lo(vi);
+      if (tau != 0.f) {
+        const float tv = tau * vi;
+#pragma unroll
+        for (int l4 = 0; l4 < NB / 4; ++l4) {
+          const float4 w4 = reinterpret_cast<const float4*>(s_wl)[l4];
+          if (l4 > 0) a1[4 * l4 - 1] = fmaf(-tv, w4.x, a1[4 * l4]);
+          a1[4 * l4] = fmaf(-tv, w4.y, a1[4 * l4 + 1]);
+          a1[4 * l4 + 1] = fmaf(-tv, w4.z, a1[4 * l4 + 2]);
+          a1[4 * l4 + 2] = fmaf(-tv, w4.w, a1[4 * l4 + 3]);
+        }
+        a1[NB - 1] = 0.f;
+      } else {
+#pragma unroll
+        for (int l = 0; l < NB - 1; ++l) a1[l] = a1[l + 1];
+        a1[NB - 1] = 0.f;
+      }
+    }
+    __syncthreads();  // s_wl, s_red and s_scal are rewritten by the next column
+  }
+  if (nonfinite) atomicOr(p.status, kStatusQrBreakdown);
+  // the block's positions before the panel are zero in the panel's rows of Vt
+  if (c == 0)
+    for (int e = tid; e < kb * jb; e += PTA) {
+      const int64_t o = (int64_t)(k + e / jb) * n + k0 + e % jb;
+      Vt[o] = 0.f;
+      Vt_lo[o] = 0.f;
+    }
+  cluster.sync();  // the peers have read this CTA's partial sums
+}
+
 // ||P_b||_F: per-chunk partial sums in double (chunks of whole 16-byte units: nn is a
 // multiple of 16), then tol * sqrt(sum)
 constexpr int NORM_CHUNKS = 64;
@@ -1024,17 +1251,21 @@ __global__ void transpose_out_kernel(const float* Qt, float* Q, float* Q_lo, int
 // where the device runs 16-CTA clusters of it, else 1024 positions in clusters of up to 8.
 struct PanelKernel {
   void (*fn)(PanelArgs);
+  void (*cols_fn)(PanelArgs);  // the column loop on its own (then fn forms the rest), or null
   int cols;
   size_t smem;
 };
 
-template <int COLS>
+template <int COLS, bool SPLIT = false>
 cudaError_t prepare_panel(PanelKernel* pk, bool wide) {
-  pk->fn = qr_panel_kernel<COLS>;
+  pk->fn = qr_panel_kernel<COLS, SPLIT>;
+  pk->cols_fn = SPLIT ? qr_cols_kernel : nullptr;
   pk->cols = COLS;
   pk->smem = (size_t)NB * (COLS + 4) * sizeof(float);
   cudaError_t e = cudaFuncSetAttribute(pk->fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pk->smem);
   if (e == cudaSuccess && wide) e = cudaFuncSetAttribute(pk->fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e == cudaSuccess && wide && pk->cols_fn)
+    e = cudaFuncSetAttribute(pk->cols_fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   return e;
 }
 
@@ -1042,7 +1273,13 @@ cudaError_t prepare_panel(PanelKernel* pk, bool wide) {
 // 16 x 512 positions where the device can place them, 2 = clusters of 8 x 1024.
 std::atomic<int> g_panel_choice[64];
 
-cudaError_t panel_kernel(PanelKernel* pk, int n) {
+// Batches of at least this many factors take the column loop as its own kernel: on a GPU
+// shared with the other QR groups and the next wave's products, two column-loop CTAs fit on one
+// SM and the rest of the panel's work holds the SM for half as long. A smaller batch leaves SMs
+// idle anyway, and there the second launch per panel only lengthens the chain.
+constexpr int kSplitBatch = 16;
+
+cudaError_t panel_kernel(PanelKernel* pk, int n, int batch) {
   // a factor of at most 1024 rows fits one CTA's 1024 positions: no cluster barrier per column
   if (n <= 1024) return prepare_panel<1024>(pk, false);
   int dev = 0;
@@ -1051,7 +1288,7 @@ cudaError_t panel_kernel(PanelKernel* pk, int n) {
   int choice = slot ? slot->load(std::memory_order_relaxed) : 0;
   if (choice == 0) {
     int ok = 0;
-    if (prepare_panel<512>(pk, true) == cudaSuccess) {
+    if (prepare_panel<512, true>(pk, true) == cudaSuccess) {
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(16, 1, 1);
       cfg.blockDim = dim3(PT, 1, 1);
@@ -1070,7 +1307,8 @@ cudaError_t panel_kernel(PanelKernel* pk, int n) {
     choice = ok ? 1 : 2;
     if (slot) slot->store(choice, std::memory_order_relaxed);
   }
-  return choice == 1 ? prepare_panel<512>(pk, true) : prepare_panel<1024>(pk, false);
+  if (choice != 1) return prepare_panel<1024>(pk, false);
+  return batch >= kSplitBatch ? prepare_panel<512, true>(pk, true) : prepare_panel<512, false>(pk, true);
 }
 
 struct Workspace {
@@ -1108,6 +1346,7 @@ struct Workspace {
   float* Tt2_lo;
   float* thresh;
   float* dsign;
+  float* tau;     // [batch][n] the reflectors' tau, from the column kernel to the panel kernel
   double* part;
 };
 
@@ -1139,6 +1378,7 @@ Workspace carve(void* base, int n, int batch, size_t* total, bool lookahead) {
   const size_t oTt2 = lookahead ? take(tsq) : 0, oTt2l = lookahead ? take(tsq) : 0;
   const size_t oth = take((size_t)batch * sizeof(float));
   const size_t osg = take((size_t)batch * n * sizeof(float));
+  const size_t otau = take((size_t)batch * n * sizeof(float));
   const size_t opart = take((size_t)batch * NORM_CHUNKS * sizeof(double));
   if (total) *total = off;
   char* c = (char*)base;
@@ -1147,7 +1387,7 @@ Workspace carve(void* base, int n, int batch, size_t* total, bool lookahead) {
   return Workspace{f(oAt), nullptr, f(oVt), f(oVtl), f(oVq), f(oVql), f(oVr), f(oVrl), f(oVp),  f(oVpl),
                    f(oW),  f(oWl),  f(oT),  f(oTl),  f(oTt), f(oTtl), f(oY),  f(oWs), g(oW2),  g(oW2l),
                    g(oWs2), g(oVr2), g(oVr2l), g(oVp2), g(oVp2l), g(oT2),  g(oT2l),  g(oTt2), g(oTt2l),
-                   f(oth), f(osg), (double*)(c + opart)};
+                   f(oth), f(osg), f(otau), (double*)(c + opart)};
 }
 
 TcOperand op(const float* hi, const float* lo, int64_t ld, int64_t stride, int batch) {
@@ -1197,7 +1437,7 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     thresh_kernel<<<(batch + 127) / 128, 128, 0, s>>>(w.part, tol, batch, w.thresh, status);
   }
   PanelKernel pk;
-  e = panel_kernel(&pk, n);
+  e = panel_kernel(&pk, n, batch);
   if (e != cudaSuccess) return e;
 
   if (la) {
@@ -1226,7 +1466,7 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
     for (int k = k0; k < k0 + kbo; k += NB) {
       const int kb = std::min(NB, n - k);
       const int C = (n - k + pk.cols - 1) / pk.cols;
-      PanelArgs a{w.At, w.Vt, w.Vt_lo, vp, vp_lo, Tb, Tb_lo, Ttb, Ttb_lo, w.Ypart, skip, w.dsign,
+      PanelArgs a{w.At, w.Vt, w.Vt_lo, vp, vp_lo, Tb, Tb_lo, Ttb, Ttb_lo, w.Ypart, skip, w.dsign, w.tau,
                   w.thresh, status, n, k0, kbo, k, kb};
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(C, batch, 1);
@@ -1240,11 +1480,22 @@ cudaError_t qr_q_t(int n, int batch, float* Qt, float* Qt_lo, float* Q, float* Q
       attr[0].val.clusterDim.z = 1;
       cfg.attrs = attr;
       cfg.numAttrs = 1;
+      // Householder steps on the kb x (n-k) panel (~4 kb^2 (n-k)), S V over kbo rows
+      // (2 kbo kb (n-k)) and the in-block update (2 kb (kbo-kb) (n-k))
+      const double mk = (double)(n - k) * batch;
+      if (pk.cols_fn) {
+        // the column loop first, on its own (the panel read, V written with its lo part)
+        cudaLaunchConfig_t cc = cfg;
+        cc.blockDim = dim3(PTA, 1, 1);
+        cc.dynamicSmemBytes = 0;
+        ProfScope prof(kFamQrPanel, 4.0 * kb * kb * mk, 4.0 * 3.0 * kb * mk, s);
+        e = cudaLaunchKernelEx(&cc, pk.cols_fn, a);
+        if (e != cudaSuccess) return e;
+      }
       {
-        // Householder steps on the kb x (n-k) panel (~4 kb^2 (n-k)), S V over kbo rows
-        // (2 kbo kb (n-k)) and the in-block update (2 kb (kbo-kb) (n-k))
-        const double mk = (double)(n - k) * batch;
-        ProfScope prof(kFamQrPanel, (4.0 * kb * kb + 4.0 * kbo * kb) * mk, 4.0 * (3.0 * kb + 2.0 * kbo) * mk, s);
+        const double f = pk.cols_fn ? 4.0 * kbo * kb * mk : (4.0 * kb * kb + 4.0 * kbo * kb) * mk;
+        const double by = pk.cols_fn ? 4.0 * 2.0 * kbo * mk : 4.0 * (3.0 * kb + 2.0 * kbo) * mk;
+        ProfScope prof(kFamQrPanel, f, by, s);
         e = cudaLaunchKernelEx(&cfg, pk.fn, a);
       }
       if (e != cudaSuccess) return e;
