@@ -10,7 +10,8 @@
 //
 //   for each block of 128 rows of At at k0 (columns k0..k0+127 of P):
 //     for each 32-row panel at k in the block:
-//       qr_panel_kernel factors the panel rows, writes the Householder vectors as rows of
+//       qr_panel_kernel (or qr_cols_kernel, then qr_panel_kernel) factors the panel rows,
+//       writes the Householder vectors as rows of
 //       Vt (row k+a = v_a over positions k0..n-1, zeros before its pivot) and as columns
 //       of Vpos (position-major), extends the block's T (H_k0 ... H_k+31 = I - V T V^T)
 //       by this panel's columns, and applies the panel's reflectors to the block's rows
@@ -26,13 +27,17 @@
 //
 // The panel of an n x n matrix spans up to n positions; it is spread over a thread-block
 // cluster of ceil((n-k)/512) CTAs (<= 16 for n <= 8192), 512 positions each, or, on a
-// device that cannot run 16-CTA clusters of it, 1024 positions in clusters of <= 8. Each
-// Householder step needs one cluster-wide reduction: the squared norm of the column
-// below the pivot and its dot products with the later panel columns are reduced
-// together (the dot products with v follow from them once the reflector is known), and
-// the partial sums are combined through distributed shared memory at one cluster
-// barrier. No CTA waits on a flag: the only waits are hardware cluster barriers that
-// every CTA of the cluster reaches unconditionally.
+// device that cannot run 16-CTA clusters of it, 1024 positions in clusters of <= 8 (a
+// factor of at most 1024 rows takes one CTA of 1024 positions). Each Householder step needs
+// one cluster-wide reduction: the squared norm of the column below the pivot and its dot
+// products with the later panel columns are reduced together (the dot products with v
+// follow from them once the reflector is known), and the partial sums are combined through
+// distributed shared memory at one cluster barrier. No CTA waits on a flag: the only waits
+// are hardware cluster barriers that every CTA of the cluster reaches unconditionally, and
+// the tensor-core block product's mbarrier waits, which give up after a bounded time.
+// For a batch of at least kSplitBatch factors the panel's 32 Householder steps run as a
+// kernel of their own (qr_cols_kernel: two positions per thread, small enough for two CTAs
+// per SM), and qr_panel_kernel<512, true> does the rest from the vectors it wrote.
 //
 // Reflector convention (LAPACK larfg): for x = A[p:n, p] with alpha = x_1 and
 // sigma = ||x_2:||^2, beta = -sign(alpha) ||x||, v = x / (alpha - beta) with v_1 = 1,
